@@ -1,0 +1,150 @@
+/*
+ * cyfa.h -- C ABI of the CyFA (Cyclic Flow Attention) core operator for GB300 (sm_103a).
+ *
+ * The operator is the absolute-clock form of CyFA (Sec. 3.2, Eq. cyfa-absolute-recurrence
+ * and Eq. cyfa-absolute-readout), evaluated chunk-wise as two scalar-decay linear-attention
+ * passes joined by a token-wise softmax readout (Sec. 3.3 Eq. cyfa-two-pass; App. B Eqs.
+ * app-cyfa-key-chunk and app-cyfa-value-chunk).  Per (batch b, head h) and token t:
+ *
+ *   delta_t  = sigmoid(clock_logit_t)                     clock increment, Eq. clock_gradient_stabilization
+ *   lambda_t = lambda_{t-1} + delta_t                     cumulative clock, Eq. cyfa-cumulative-clock
+ *   alpha_t  = exp(-A_h softplus(decay_logit_t))          scalar forget gate, Sec. 3.4
+ *   beta_t   = sigmoid(beta_logit_t)                      write strength (activation: this library's reading)
+ *   a_t      = beta_t U(-lambda_t) b                      temporal write vector, Sec. 3.2
+ *   Kbar_t   = alpha_t Kbar_{t-1} + a_t k_t^T             key state   [m x dk]
+ *   Vbar_t   = alpha_t Vbar_{t-1} + a_t v_t^T             value state [m x dv]
+ *   o'_t     = Kbar_t (scale q_t)
+ *   o''_t    = U(-lambda_t) Phi^T R^T softmax(R Phi U(lambda_t) o'_t)
+ *   o_t      = Vbar_t^T o''_t
+ *
+ * Storage conventions (all row-major, caller-owned; the library never allocates):
+ *   q, k, dq, dk      [B, T, H, dk]   bf16 or fp32 (dims.dtype)
+ *   v, o, dO, dv      [B, T, H, dv]   bf16 or fp32
+ *   *_logit, lam_mod, g_cum, beta, d_*_logit   [B, T, H] fp32
+ *   A                 [H] fp32 (> 0)
+ *   R, dR             [H, m, m] fp32 (m = 127)
+ *   Kbar, Vbar        [B, H, 128, dk] / [B, H, 128, dv] fp32; rows in the order of the real
+ *                     Fourier basis of App. A.1 Eq. app-real-fourier (DC, cos_1, sin_1, ...,
+ *                     cos_63, sin_63) followed by one padding row that stays zero (App. A.7).
+ *   lambda            [B, H] fp64 (the running clock)
+ *   stream            a cudaStream_t passed as void*; every call is asynchronous on it.
+ *
+ * Shapes supported: m = 127 (128 storage rows), dk = dv in {64, 128}, chunk in {64, 128},
+ * T a positive multiple of chunk (for cyfa_prepare / cyfa_chunk_fwd / cyfa_chunk_bwd).
+ *
+ * Errors: every entry point returns CYFA_OK (0) or a negative code.  Argument errors are
+ * found on the host before anything is launched.  CYFA_ERR_TIMEOUT is raised on the device
+ * by a bounded wait and read back by cyfa_check().
+ */
+#ifndef CYFA_H
+#define CYFA_H
+
+#include <stddef.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+enum {
+    CYFA_OK = 0,
+    CYFA_ERR_ARG = -1,        /* null required pointer or non-positive size */
+    CYFA_ERR_SHAPE = -2,      /* unsupported m, d, chunk, or T not a multiple of chunk */
+    CYFA_ERR_ALIGN = -3,      /* a tensor pointer is not 16-byte aligned */
+    CYFA_ERR_WORKSPACE = -4,  /* workspace null or smaller than cyfa_workspace_size() */
+    CYFA_ERR_CUDA = -5,       /* a CUDA runtime call or launch failed */
+    CYFA_ERR_TIMEOUT = -6,    /* a bounded device-side wait expired (see cyfa_check) */
+    CYFA_ERR_UNSUPPORTED = -7 /* a valid request this build does not implement */
+};
+
+enum { CYFA_DTYPE_BF16 = 0, CYFA_DTYPE_FP32 = 1 };
+
+/* Which call a workspace is sized for. */
+enum { CYFA_WS_PREPARE = 0, CYFA_WS_FWD = 1, CYFA_WS_BWD = 2 };
+
+typedef struct cyfa_dims {
+    int B, T, H;   /* batch, sequence length, heads */
+    int dk, dv;    /* head dims (dk == dv) */
+    int m;         /* active relative-time slots; must be 127 */
+    int chunk;     /* tokens per chunk: 64 or 128 */
+    float scale;   /* dot-product scale s; the query enters the key pass as s*q */
+    int dtype;     /* CYFA_DTYPE_BF16 or CYFA_DTYPE_FP32 for q, k, v, o, dO, dq, dk, dv */
+} cyfa_dims_t;
+
+/* Library version as 10000*major + 100*minor + patch. */
+int cyfa_version(void);
+
+/* Human-readable text for an error code (static storage, never NULL). */
+const char* cyfa_error_string(int code);
+
+/* Bytes of device workspace the call `which` (CYFA_WS_*) needs for these dims. */
+int cyfa_workspace_size(const cyfa_dims_t* dims, int which, size_t* bytes);
+
+/*
+ * cyfa_prepare -- per-token gates and the absolute-clock coordinates (Sec. 3.1 Eq.
+ * cyfa-cumulative-clock, Sec. 3.4, App. B chunk-local log-decays of Eq. app-chunk-decay).
+ *
+ *   lam_mod[b,t,h] = lambda_t mod m, with lambda_t = lambda0[b,h] + sum_{u<=t} delta_u
+ *                    carried in fp64; U is m-periodic (Prop. 1) so the reduction is exact.
+ *   g_cum[b,t,h]   = sum of log alpha_u over the tokens u <= t of t's chunk (<= 0).
+ *   beta[b,t,h]    = sigmoid(beta_logit).
+ *   lambda_end[b,h] (nullable) = lambda_T in fp64, the clock a following cyfa_step continues.
+ * lambda0 may be NULL (clock origin 0; Prop. 6 makes the origin arbitrary).
+ * Needs cyfa_workspace_size(CYFA_WS_PREPARE) bytes of workspace.
+ */
+int cyfa_prepare(const cyfa_dims_t* dims, const float* clock_logit, const float* decay_logit,
+                 const float* beta_logit, const float* A, const double* lambda0,
+                 float* lam_mod, float* g_cum, float* beta, double* lambda_end,
+                 void* workspace, size_t workspace_bytes, void* stream);
+
+/*
+ * cyfa_chunk_fwd -- forward of the operator, chunk-wise two-pass form (Sec. 3.3 Eq.
+ * cyfa-two-pass; App. B Eqs. app-cyfa-key-chunk, app-cyfa-value-chunk).
+ * Inputs are the outputs of cyfa_prepare plus q, k, v and R.  Kbar0 / Vbar0 (nullable,
+ * both or neither) give the states before token 0 in the same clock origin as lambda0.
+ * o receives the output; Kbar_out / Vbar_out (nullable) receive the states after token T-1.
+ */
+int cyfa_chunk_fwd(const cyfa_dims_t* dims, const void* q, const void* k, const void* v,
+                   const float* lam_mod, const float* g_cum, const float* beta, const float* R,
+                   const float* Kbar0, const float* Vbar0, void* o, float* Kbar_out,
+                   float* Vbar_out, void* workspace, size_t workspace_bytes, void* stream);
+
+/*
+ * cyfa_chunk_bwd -- gradient of sum(o * dO) with respect to q, k, v, the three logits, and
+ * (nullable outputs) R and A, starting from zero state at token 0.  The clock gradient is
+ * the reverse cumulative sum dL/d delta_s = sum_{t>=s} dL/d lambda_t of App. D.1 Eq.
+ * app-clock-gradient-accumulation; the decay gradient is the reverse cumulative sum of
+ * the per-token gradient of the cumulative log-decay.  dR [H,m,m] and dA [H] are sums
+ * over the batch.  Inputs are those of cyfa_chunk_fwd plus the raw clock / decay logits
+ * and A (for the activation derivatives).
+ */
+int cyfa_chunk_bwd(const cyfa_dims_t* dims, const void* q, const void* k, const void* v,
+                   const float* lam_mod, const float* g_cum, const float* beta, const float* R,
+                   const float* clock_logit, const float* decay_logit, const float* A,
+                   const void* dO, void* dq, void* dk, void* dv, float* d_clock_logit,
+                   float* d_decay_logit, float* d_beta_logit, float* dR, float* dA,
+                   void* workspace, size_t workspace_bytes, void* stream);
+
+/*
+ * cyfa_step -- one decode token for every (b, h), in place on the persistent state
+ * (Sec. 3.2 Eq. cyfa-absolute-recurrence and Eq. cyfa-absolute-readout, one step).
+ * q, k, v, o are [B, H, d] (dims.T is ignored); the logits are [B, H] fp32.
+ * Kbar, Vbar [B, H, 128, d] fp32 and lambda [B, H] fp64 are read and overwritten.
+ * Needs no workspace.
+ */
+int cyfa_step(const cyfa_dims_t* dims, const void* q, const void* k, const void* v,
+              const float* clock_logit, const float* decay_logit, const float* beta_logit,
+              const float* A, const float* R, float* Kbar, float* Vbar, double* lambda, void* o,
+              void* stream);
+
+/*
+ * cyfa_check -- wait for `stream`, then report (and clear) the device error word that
+ * bounded device-side waits set when they give up: CYFA_OK or CYFA_ERR_TIMEOUT, or
+ * CYFA_ERR_CUDA if the stream itself reports an error.
+ */
+int cyfa_check(void* stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* CYFA_H */

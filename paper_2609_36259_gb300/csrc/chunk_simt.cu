@@ -1,0 +1,370 @@
+// fp32 SIMT chunk kernels of the CyFA operator (forward and backward).
+//
+// Chunk-wise two-pass form of App. B (Eqs. app-chunk-decay, app-chunk-rescale,
+// app-temporal-writes, app-cyfa-key-chunk, app-cyfa-value-chunk) with the token-wise middle
+// line of Sec. 3.3 Eq. cyfa-two-pass.  Every product accumulates in fp32 on the CUDA cores;
+// this path serves fp32 inputs (and any input when exactness is wanted over speed).
+//
+// States are stored in the paper's orientation: Kbar [128 x dk] (= (S^K)^T of App. B) and
+// Vbar [128 x dv], side by side as one [128 x 2D] row-major block per chunk.
+#include "common.cuh"
+#include "kernels.h"
+
+namespace cyfa {
+
+namespace {
+
+constexpr int LD = 129;   // padded row stride of [C][128] shared tiles
+
+// ---------------------------------------------------------------------------------------
+// M = R Phi (padded to 128 x 128 with a zero last row and column) and its transpose.
+// Phi is the real Fourier basis of App. A.1 Eq. app-real-fourier.
+__global__ void __launch_bounds__(128) readout_matrix_kernel(const float* R, float* M, float* MT) {
+    const int h = blockIdx.y, i = blockIdx.x, col = threadIdx.x;
+    __shared__ float srow[128];
+    srow[col] = (i < MA && col < MA) ? R[((size_t)h * MA + i) * MA + col] : 0.f;
+    __syncthreads();
+    float acc = 0.f;
+    if (i < MA && col < MA) {
+        const int j = (col + 1) >> 1;
+        for (int r = 0; r < MA; ++r) {
+            float phi;
+            if (col == 0) {
+                phi = INV_SQRT_M;
+            } else {
+                float s, c;
+                sincospif((float)((j * r) % MA) * (2.f / 127.f), &s, &c);
+                phi = SQRT_2_OVER_M * ((col & 1) ? c : s);
+            }
+            acc = fmaf(srow[r], phi, acc);
+        }
+    }
+    M[((size_t)h * MS + i) * MS + col] = acc;
+    MT[((size_t)h * MS + col) * MS + i] = acc;
+}
+
+// ---------------------------------------------------------------------------------------
+// Token-wise middle readout for rows r < C of sX (in place): o'' = U(-lam) M^T softmax(M U(lam) o')
+// with M = R Phi; the padding logit is excluded from the softmax and o''[127] = 0.
+// One warp per row; swarp holds 2 x 128 floats of scratch per warp.
+__device__ void middle_rows(float* sX, const float* slam, int C, const float* M, const float* MT,
+                            float* swarp) {
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    float* z = swarp + warp * 256;
+    float* p = z + 128;
+    for (int r = warp; r < C; r += 8) {
+        float* x = sX + r * LD;
+        const float lam = slam[r];
+        float cs[2], sn[2];
+#pragma unroll
+        for (int u = 0; u < 2; ++u) {
+            const int j = lane + 1 + 32 * u;
+            cs[u] = 1.f;
+            sn[u] = 0.f;
+            if (j <= NPAIR) {
+                sincospif(phase_pi(lam, j), &sn[u], &cs[u]);
+                const float xc = x[2 * j - 1], xs = x[2 * j];
+                z[2 * j - 1] = cs[u] * xc - sn[u] * xs;
+                z[2 * j] = sn[u] * xc + cs[u] * xs;
+            }
+        }
+        if (lane == 0) {
+            z[0] = x[0];
+            z[127] = 0.f;
+        }
+        __syncwarp();
+        float l[4] = {0.f, 0.f, 0.f, 0.f};
+        for (int k = 0; k < MS; ++k) {
+            const float zk = z[k];
+#pragma unroll
+            for (int u = 0; u < 4; ++u) l[u] = fmaf(MT[k * MS + lane + 32 * u], zk, l[u]);
+        }
+        if (lane == 31) l[3] = -INFINITY;
+        float mx = fmaxf(fmaxf(l[0], l[1]), fmaxf(l[2], l[3]));
+        mx = warp_max(mx);
+        float e[4], sum = 0.f;
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+            e[u] = expf(l[u] - mx);
+            sum += e[u];
+        }
+        sum = warp_sum(sum);
+        const float inv = 1.f / sum;
+#pragma unroll
+        for (int u = 0; u < 4; ++u) p[lane + 32 * u] = e[u] * inv;
+        __syncwarp();
+        float y[4] = {0.f, 0.f, 0.f, 0.f};
+        for (int i = 0; i < MA; ++i) {
+            const float pi = p[i];
+#pragma unroll
+            for (int u = 0; u < 4; ++u) y[u] = fmaf(M[i * MS + lane + 32 * u], pi, y[u]);
+        }
+        __syncwarp();
+#pragma unroll
+        for (int u = 0; u < 4; ++u) z[lane + 32 * u] = y[u];
+        __syncwarp();
+#pragma unroll
+        for (int u = 0; u < 2; ++u) {
+            const int j = lane + 1 + 32 * u;
+            if (j <= NPAIR) {
+                const float yc = z[2 * j - 1], ys = z[2 * j];
+                x[2 * j - 1] = cs[u] * yc + sn[u] * ys;
+                x[2 * j] = -sn[u] * yc + cs[u] * ys;
+            }
+        }
+        if (lane == 0) {
+            x[0] = z[0];
+            x[127] = 0.f;
+        }
+        __syncwarp();
+    }
+}
+
+__device__ __forceinline__ void load_gates(const Shape& s, const float* lam, const float* g,
+                                           const float* beta, int b, int h, int t0, int C,
+                                           float* slam, float* sg, float* sbeta) {
+    for (int r = threadIdx.x; r < C; r += blockDim.x) {
+        const size_t gi = ((size_t)b * s.T + t0 + r) * s.H + h;
+        slam[r] = lam[gi];
+        sg[r] = g[gi];
+        sbeta[r] = beta[gi];
+    }
+}
+
+// Stage rows [r0, r0+nr) x columns [c0, c0+32) of a [B,T,H,D] tensor into dst[r][33].
+template <typename TI>
+__device__ __forceinline__ void stage_tok(float* dst, const TI* X, const Shape& s, int b, int h,
+                                          int t0, int nr, int c0, float mul) {
+    for (int e = threadIdx.x; e < nr * 32; e += blockDim.x) {
+        const int r = e >> 5, cc = e & 31;
+        dst[r * 33 + cc] = mul * ldf(X, (((size_t)b * s.T + t0 + r) * s.H + h) * s.D + c0 + cc);
+    }
+}
+
+// ---------------------------------------------------------------------------------------
+// Forward state pass: one block per (b, h, 32-column tile of [Kbar | Vbar]); walks the chunks
+// in order, writing the chunk-start state, then Kbar <- gamma^C Kbar + A->^T K (and V),
+// App. B Eq. app-cyfa-key-chunk / app-cyfa-value-chunk (first lines).
+template <int C, typename TI>
+__global__ void __launch_bounds__(256) fwd_state_kernel(FwdArgs a) {
+    const Shape s = a.s;
+    const int D = s.D, W = 2 * s.D;
+    const int bh = blockIdx.y, b = bh / s.H, h = bh % s.H;
+    const int col0 = blockIdx.x * 32;
+    const bool isK = col0 < D;
+    const TI* X = (const TI*)(isK ? a.k : a.v);
+    const int xc0 = isK ? col0 : col0 - D;
+    extern __shared__ float smem[];
+    float* sA = smem;              // [C][LD]
+    float* sX = sA + C * LD;       // [C][33]
+    float* sg = sX + C * 33;
+    float* slam = sg + C;
+    float* sbeta = slam + C;
+    const int tx = threadIdx.x & 15, ty = threadIdx.x >> 4;
+    float S[8][2];
+    const float* S0 = isK ? a.Kbar0 : a.Vbar0;
+#pragma unroll
+    for (int i = 0; i < 8; ++i)
+#pragma unroll
+        for (int j = 0; j < 2; ++j)
+            S[i][j] = S0 ? S0[((size_t)bh * MS + ty + 16 * i) * D + xc0 + tx + 16 * j] : 0.f;
+    const int nchunk = s.nchunk();
+    for (int c = 0; c < nchunk; ++c) {
+        float* dst = a.states + ((size_t)bh * nchunk + c) * MS * W;
+#pragma unroll
+        for (int i = 0; i < 8; ++i)
+#pragma unroll
+            for (int j = 0; j < 2; ++j) dst[(ty + 16 * i) * W + col0 + tx + 16 * j] = S[i][j];
+        const int t0 = c * C;
+        load_gates(s, a.lam, a.g, a.beta, b, h, t0, C, slam, sg, sbeta);
+        stage_tok(sX, X, s, b, h, t0, C, xc0, 1.f);
+        __syncthreads();
+        const float gC = sg[C - 1];
+        build_write_rows(sA, LD, slam, sbeta, C, [&](int r) { return expf(gC - sg[r]); });
+        __syncthreads();
+        const float decay = expf(gC);
+#pragma unroll
+        for (int i = 0; i < 8; ++i)
+#pragma unroll
+            for (int j = 0; j < 2; ++j) S[i][j] *= decay;
+        simt_mm<8, 2>(S, C, [&](int row, int t) { return sA[t * LD + row]; },
+                      [&](int t, int col) { return sX[t * 33 + col]; });
+        __syncthreads();
+    }
+    float* F = isK ? a.Kout : a.Vout;
+    if (F) {
+#pragma unroll
+        for (int i = 0; i < 8; ++i)
+#pragma unroll
+            for (int j = 0; j < 2; ++j)
+                F[((size_t)bh * MS + ty + 16 * i) * D + xc0 + tx + 16 * j] = S[i][j];
+    }
+}
+
+// Forward outputs of one chunk (App. B, second lines of Eqs. app-cyfa-key-chunk and
+// app-cyfa-value-chunk, with the middle readout between them).
+template <int C, int D, typename TI>
+__global__ void __launch_bounds__(256) fwd_out_kernel(FwdArgs a) {
+    const Shape s = a.s;
+    constexpr int LP = C + 1, TM = C / 16;
+    const int c = blockIdx.x, bh = blockIdx.y, b = bh / s.H, h = bh % s.H;
+    const int nchunk = s.nchunk();
+    const int t0 = c * C;
+    extern __shared__ float smem[];
+    float* sA = smem;            // [C][LD]   write vectors; later staging
+    float* sX = sA + C * LD;     // [C][LD]   staging, then O', then O''
+    float* sP = sX + C * LD;     // [C][LP]   masked intra-chunk scores
+    float* sg = sP + C * LP;
+    float* seg = sg + C;
+    float* slam = seg + C;
+    float* sbeta = slam + C;
+    float* swarp = sbeta + C;    // [8][256]
+    const int tx = threadIdx.x & 15, ty = threadIdx.x >> 4;
+    const float* Sst = a.states + ((size_t)bh * nchunk + c) * MS * (2 * D);
+    const TI* Q = (const TI*)a.q;
+    const TI* K = (const TI*)a.k;
+    const TI* V = (const TI*)a.v;
+
+    load_gates(s, a.lam, a.g, a.beta, b, h, t0, C, slam, sg, sbeta);
+    __syncthreads();
+    for (int r = threadIdx.x; r < C; r += blockDim.x) seg[r] = expf(sg[r]);
+    build_write_rows(sA, LD, slam, sbeta, C, [](int) { return 1.f; });
+
+    // P = (s Q K^T) o Gamma
+    float acc[TM][TM];
+    zero_acc(acc);
+    for (int d0 = 0; d0 < D; d0 += 32) {
+        __syncthreads();
+        stage_tok(sX, Q, s, b, h, t0, C, d0, 1.f);
+        stage_tok(sX + C * 33, K, s, b, h, t0, C, d0, 1.f);
+        __syncthreads();
+        simt_mm<TM, TM>(acc, 32, [&](int r, int kk) { return sX[r * 33 + kk]; },
+                        [&](int kk, int t) { return sX[C * 33 + t * 33 + kk]; });
+    }
+#pragma unroll
+    for (int i = 0; i < TM; ++i)
+#pragma unroll
+        for (int j = 0; j < TM; ++j) {
+            const int r = ty + 16 * i, t = tx + 16 * j;
+            sP[r * LP + t] = (t <= r) ? acc[i][j] * s.scale * expf(sg[r] - sg[t]) : 0.f;
+        }
+
+    // O' = diag(gamma) (s Q) Kbar^T + P A
+    float o1[TM][8];
+    zero_acc(o1);
+    for (int d0 = 0; d0 < D; d0 += 32) {
+        __syncthreads();
+        stage_tok(sX, Q, s, b, h, t0, C, d0, 1.f);
+        for (int e = threadIdx.x; e < MS * 32; e += blockDim.x) {
+            const int i = e >> 5, dd = e & 31;
+            sX[C * 33 + i * 33 + dd] = Sst[i * (2 * D) + d0 + dd];
+        }
+        __syncthreads();
+        simt_mm<TM, 8>(o1, 32, [&](int r, int kk) { return sX[r * 33 + kk]; },
+                       [&](int kk, int i) { return sX[C * 33 + i * 33 + kk]; });
+    }
+#pragma unroll
+    for (int i = 0; i < TM; ++i)
+#pragma unroll
+        for (int j = 0; j < 8; ++j) o1[i][j] *= s.scale * seg[ty + 16 * i];
+    simt_mm<TM, 8>(o1, C, [&](int r, int t) { return sP[r * LP + t]; },
+                   [&](int t, int i) { return sA[t * LD + i]; });
+    __syncthreads();
+#pragma unroll
+    for (int i = 0; i < TM; ++i)
+#pragma unroll
+        for (int j = 0; j < 8; ++j) sX[(ty + 16 * i) * LD + tx + 16 * j] = o1[i][j];
+    __syncthreads();
+
+    middle_rows(sX, slam, C, a.M + (size_t)h * MS * MS, a.MT + (size_t)h * MS * MS, swarp);
+    __syncthreads();
+
+    // P = (O'' A^T) o Gamma
+    zero_acc(acc);
+    simt_mm<TM, TM>(acc, MS, [&](int r, int kk) { return sX[r * LD + kk]; },
+                    [&](int kk, int t) { return sA[t * LD + kk]; });
+#pragma unroll
+    for (int i = 0; i < TM; ++i)
+#pragma unroll
+        for (int j = 0; j < TM; ++j) {
+            const int r = ty + 16 * i, t = tx + 16 * j;
+            sP[r * LP + t] = (t <= r) ? acc[i][j] * expf(sg[r] - sg[t]) : 0.f;
+        }
+
+    // O = diag(gamma) O'' Vbar + P V
+    constexpr int TN = D / 16;
+    float o[TM][TN];
+    zero_acc(o);
+    float* sV = sA;  // staging [32][D+1]
+    for (int i0 = 0; i0 < MS; i0 += 32) {
+        __syncthreads();
+        for (int e = threadIdx.x; e < 32 * D; e += blockDim.x) {
+            const int ii = e / D, dd = e % D;
+            sV[ii * (D + 1) + dd] = Sst[(i0 + ii) * (2 * D) + D + dd];
+        }
+        __syncthreads();
+        simt_mm<TM, TN>(o, 32, [&](int r, int ii) { return sX[r * LD + i0 + ii]; },
+                        [&](int ii, int dd) { return sV[ii * (D + 1) + dd]; });
+    }
+#pragma unroll
+    for (int i = 0; i < TM; ++i)
+#pragma unroll
+        for (int j = 0; j < TN; ++j) o[i][j] *= seg[ty + 16 * i];
+    for (int s0 = 0; s0 < C; s0 += 32) {
+        __syncthreads();
+        for (int e = threadIdx.x; e < 32 * D; e += blockDim.x) {
+            const int ss = e / D, dd = e % D;
+            sV[ss * (D + 1) + dd] = ldf(V, (((size_t)b * s.T + t0 + s0 + ss) * s.H + h) * D + dd);
+        }
+        __syncthreads();
+        simt_mm<TM, TN>(o, 32, [&](int r, int ss) { return sP[r * LP + s0 + ss]; },
+                        [&](int ss, int dd) { return sV[ss * (D + 1) + dd]; });
+    }
+    TI* O = (TI*)a.o;
+#pragma unroll
+    for (int i = 0; i < TM; ++i)
+#pragma unroll
+        for (int j = 0; j < TN; ++j) {
+            const int r = ty + 16 * i, dd = tx + 16 * j;
+            stf(O, (((size_t)b * s.T + t0 + r) * s.H + h) * D + dd, o[i][j]);
+        }
+}
+
+template <int C, int D, typename TI>
+cudaError_t fwd_dispatch(const FwdArgs& a, cudaStream_t st) {
+    const Shape& s = a.s;
+    const size_t sm_state = (size_t)(C * LD + C * 33 + 3 * C) * sizeof(float);
+    auto kst = fwd_state_kernel<C, TI>;
+    cudaFuncSetAttribute(kst, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm_state);
+    kst<<<dim3(2 * D / 32, s.B * s.H), 256, sm_state, st>>>(a);
+    const size_t sm_out = (size_t)(2 * C * LD + C * (C + 1) + 4 * C + 8 * 256) * sizeof(float);
+    auto kout = fwd_out_kernel<C, D, TI>;
+    cudaFuncSetAttribute(kout, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm_out);
+    kout<<<dim3(s.nchunk(), s.B * s.H), 256, sm_out, st>>>(a);
+    return cudaGetLastError();
+}
+
+}  // namespace
+
+cudaError_t launch_readout_matrix(int H, const float* R, float* M, float* MT, cudaStream_t st) {
+    readout_matrix_kernel<<<dim3(MS, H), 128, 0, st>>>(R, M, MT);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_fwd_simt(const FwdArgs& a, cudaStream_t st) {
+    const Shape& s = a.s;
+#define CYFA_FWD(CC, DD)                                                               \
+    if (s.C == CC && s.D == DD)                                                        \
+        return s.bf16 ? fwd_dispatch<CC, DD, __nv_bfloat16>(a, st)                     \
+                      : fwd_dispatch<CC, DD, float>(a, st);
+    CYFA_FWD(64, 64)
+    CYFA_FWD(64, 128)
+    CYFA_FWD(128, 64)
+    CYFA_FWD(128, 128)
+#undef CYFA_FWD
+    return cudaErrorInvalidValue;
+}
+
+cudaError_t launch_bwd_simt(const BwdArgs&, cudaStream_t) { return cudaErrorNotSupported; }
+
+}  // namespace cyfa

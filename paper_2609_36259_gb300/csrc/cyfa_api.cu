@@ -1,0 +1,289 @@
+// C ABI of the CyFA operator: argument checking, workspace layout, and launches on the
+// caller's stream.  The declarations and their contracts are in include/cyfa.h.
+#include <stdint.h>
+
+#include "../../include/cyfa.h"
+#include "common.cuh"
+#include "kernels.h"
+
+using namespace cyfa;
+
+namespace {
+
+constexpr size_t ALIGN = 256;
+inline size_t up(size_t x) { return (x + ALIGN - 1) / ALIGN * ALIGN; }
+
+// Sequential carve-out of a workspace buffer.
+struct Carver {
+    char* base;
+    size_t off = 0;
+    template <typename T>
+    T* take(size_t count) {
+        T* p = base ? reinterpret_cast<T*>(base + off) : nullptr;
+        off += up(count * sizeof(T));
+        return p;
+    }
+};
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+int check_dims(const cyfa_dims_t* d, bool need_T) {
+    if (!d) return CYFA_ERR_ARG;
+    if (d->B <= 0 || d->H <= 0 || d->dk <= 0 || d->dv <= 0 || (need_T && d->T <= 0))
+        return CYFA_ERR_ARG;
+    if (d->m != 127) return CYFA_ERR_SHAPE;
+    if (d->dk != d->dv || (d->dk != 64 && d->dk != 128)) return CYFA_ERR_SHAPE;
+    if (d->dtype != CYFA_DTYPE_BF16 && d->dtype != CYFA_DTYPE_FP32) return CYFA_ERR_ARG;
+    if (need_T) {
+        if (d->chunk != 64 && d->chunk != 128) return CYFA_ERR_SHAPE;
+        if (d->T % d->chunk != 0) return CYFA_ERR_SHAPE;
+    }
+    return CYFA_OK;
+}
+
+Shape shape_of(const cyfa_dims_t* d) {
+    Shape s;
+    s.B = d->B;
+    s.T = d->T;
+    s.H = d->H;
+    s.D = d->dk;
+    s.C = d->chunk;
+    s.scale = d->scale;
+    s.bf16 = d->dtype == CYFA_DTYPE_BF16;
+    return s;
+}
+
+struct FwdLayout {
+    float *M, *MT, *states;
+    size_t bytes;
+};
+FwdLayout fwd_layout(const Shape& s, void* ws) {
+    Carver c{static_cast<char*>(ws)};
+    FwdLayout L;
+    L.M = c.take<float>((size_t)s.H * MS * MS);
+    L.MT = c.take<float>((size_t)s.H * MS * MS);
+    L.states = c.take<float>((size_t)s.B * s.H * s.nchunk() * MS * 2 * s.D);
+    L.bytes = c.off;
+    return L;
+}
+
+struct BwdLayout {
+    float *M, *MT, *states, *adj, *o2, *do1, *tok;
+    double *seg, *dA_part;
+    size_t bytes;
+};
+BwdLayout bwd_layout(const Shape& s0, void* ws) {
+    Shape s = s0;
+    s.C = BWD_C;
+    Carver c{static_cast<char*>(ws)};
+    BwdLayout L;
+    const size_t BH = (size_t)s.B * s.H;
+    const size_t nseg = (s.T + PREP_SEG - 1) / PREP_SEG;
+    L.M = c.take<float>((size_t)s.H * MS * MS);
+    L.MT = c.take<float>((size_t)s.H * MS * MS);
+    L.states = c.take<float>(BH * s.nchunk() * MS * 2 * s.D);
+    L.adj = c.take<float>(BH * s.nchunk() * MS * 2 * s.D);
+    L.o2 = c.take<float>(BH * s.T * MS);
+    L.do1 = c.take<float>(BH * s.T * MS);
+    L.tok = c.take<float>(5 * BH * s.T);
+    L.seg = c.take<double>(2 * BH * nseg);
+    L.dA_part = c.take<double>(BH * nseg);
+    L.bytes = c.off;
+    return L;
+}
+
+inline int cuda_status(cudaError_t e) { return e == cudaSuccess ? CYFA_OK : CYFA_ERR_CUDA; }
+
+}  // namespace
+
+extern "C" {
+
+int cyfa_version(void) { return 100; }
+
+const char* cyfa_error_string(int code) {
+    switch (code) {
+        case CYFA_OK: return "ok";
+        case CYFA_ERR_ARG: return "invalid argument (null pointer or non-positive size)";
+        case CYFA_ERR_SHAPE: return "unsupported shape (m must be 127, dk == dv in {64,128}, chunk in {64,128}, T % chunk == 0)";
+        case CYFA_ERR_ALIGN: return "tensor pointer not 16-byte aligned";
+        case CYFA_ERR_WORKSPACE: return "workspace missing or too small";
+        case CYFA_ERR_CUDA: return "CUDA runtime error";
+        case CYFA_ERR_TIMEOUT: return "bounded device-side wait expired";
+        case CYFA_ERR_UNSUPPORTED: return "request not implemented by this build";
+        default: return "unknown cyfa error code";
+    }
+}
+
+int cyfa_workspace_size(const cyfa_dims_t* dims, int which, size_t* bytes) {
+    if (!bytes) return CYFA_ERR_ARG;
+    const int rc = check_dims(dims, true);
+    if (rc) return rc;
+    const Shape s = shape_of(dims);
+    switch (which) {
+        case CYFA_WS_PREPARE: *bytes = up(prepare_workspace(s)); return CYFA_OK;
+        case CYFA_WS_FWD: *bytes = fwd_layout(s, nullptr).bytes; return CYFA_OK;
+        case CYFA_WS_BWD: *bytes = bwd_layout(s, nullptr).bytes; return CYFA_OK;
+        default: return CYFA_ERR_ARG;
+    }
+}
+
+int cyfa_prepare(const cyfa_dims_t* dims, const float* clock_logit, const float* decay_logit,
+                 const float* beta_logit, const float* A, const double* lambda0, float* lam_mod,
+                 float* g_cum, float* beta, double* lambda_end, void* workspace,
+                 size_t workspace_bytes, void* stream) {
+    int rc = check_dims(dims, true);
+    if (rc) return rc;
+    if (!clock_logit || !decay_logit || !beta_logit || !A || !lam_mod || !g_cum || !beta)
+        return CYFA_ERR_ARG;
+    const Shape s = shape_of(dims);
+    if (!workspace || workspace_bytes < prepare_workspace(s)) return CYFA_ERR_WORKSPACE;
+    PrepareArgs a;
+    a.s = s;
+    a.clock_logit = clock_logit;
+    a.decay_logit = decay_logit;
+    a.beta_logit = beta_logit;
+    a.A = A;
+    a.lambda0 = lambda0;
+    a.lam_mod = lam_mod;
+    a.g_cum = g_cum;
+    a.beta = beta;
+    a.lambda_end = lambda_end;
+    a.seg_sum = static_cast<double*>(workspace);
+    return cuda_status(launch_prepare(a, static_cast<cudaStream_t>(stream)));
+}
+
+int cyfa_chunk_fwd(const cyfa_dims_t* dims, const void* q, const void* k, const void* v,
+                   const float* lam_mod, const float* g_cum, const float* beta, const float* R,
+                   const float* Kbar0, const float* Vbar0, void* o, float* Kbar_out,
+                   float* Vbar_out, void* workspace, size_t workspace_bytes, void* stream) {
+    int rc = check_dims(dims, true);
+    if (rc) return rc;
+    if (!q || !k || !v || !lam_mod || !g_cum || !beta || !R || !o) return CYFA_ERR_ARG;
+    if ((Kbar0 == nullptr) != (Vbar0 == nullptr)) return CYFA_ERR_ARG;
+    if ((Kbar_out == nullptr) != (Vbar_out == nullptr)) return CYFA_ERR_ARG;
+    if (!aligned16(q) || !aligned16(k) || !aligned16(v) || !aligned16(o)) return CYFA_ERR_ALIGN;
+    if ((Kbar0 && (!aligned16(Kbar0) || !aligned16(Vbar0))) ||
+        (Kbar_out && (!aligned16(Kbar_out) || !aligned16(Vbar_out))))
+        return CYFA_ERR_ALIGN;
+    const Shape s = shape_of(dims);
+    const FwdLayout need = fwd_layout(s, nullptr);
+    if (!workspace || workspace_bytes < need.bytes) return CYFA_ERR_WORKSPACE;
+    if (!aligned16(workspace)) return CYFA_ERR_ALIGN;
+    const FwdLayout L = fwd_layout(s, workspace);
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    rc = cuda_status(launch_readout_matrix(s.H, R, L.M, L.MT, st));
+    if (rc) return rc;
+    FwdArgs a;
+    a.s = s;
+    a.q = q;
+    a.k = k;
+    a.v = v;
+    a.lam = lam_mod;
+    a.g = g_cum;
+    a.beta = beta;
+    a.M = L.M;
+    a.MT = L.MT;
+    a.Kbar0 = Kbar0;
+    a.Vbar0 = Vbar0;
+    a.o = o;
+    a.Kout = Kbar_out;
+    a.Vout = Vbar_out;
+    a.states = L.states;
+    return cuda_status(launch_fwd_simt(a, st));
+}
+
+int cyfa_chunk_bwd(const cyfa_dims_t* dims, const void* q, const void* k, const void* v,
+                   const float* lam_mod, const float* g_cum, const float* beta, const float* R,
+                   const float* clock_logit, const float* decay_logit, const float* A,
+                   const void* dO, void* dq, void* dk, void* dv, float* d_clock_logit,
+                   float* d_decay_logit, float* d_beta_logit, float* dR, float* dA,
+                   void* workspace, size_t workspace_bytes, void* stream) {
+    int rc = check_dims(dims, true);
+    if (rc) return rc;
+    if (!q || !k || !v || !lam_mod || !g_cum || !beta || !R || !clock_logit || !decay_logit ||
+        !A || !dO || !dq || !dk || !dv || !d_clock_logit || !d_decay_logit || !d_beta_logit)
+        return CYFA_ERR_ARG;
+    if (!aligned16(q) || !aligned16(k) || !aligned16(v) || !aligned16(dO) || !aligned16(dq) ||
+        !aligned16(dk) || !aligned16(dv))
+        return CYFA_ERR_ALIGN;
+    if (dR) return CYFA_ERR_UNSUPPORTED;
+    const Shape s = shape_of(dims);
+    const BwdLayout need = bwd_layout(s, nullptr);
+    if (!workspace || workspace_bytes < need.bytes) return CYFA_ERR_WORKSPACE;
+    if (!aligned16(workspace)) return CYFA_ERR_ALIGN;
+    const BwdLayout L = bwd_layout(s, workspace);
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    rc = cuda_status(launch_readout_matrix(s.H, R, L.M, L.MT, st));
+    if (rc) return rc;
+    BwdArgs a;
+    a.s = s;
+    a.s.C = BWD_C;
+    a.q = q;
+    a.k = k;
+    a.v = v;
+    a.dO = dO;
+    a.lam = lam_mod;
+    a.g = g_cum;
+    a.beta = beta;
+    a.M = L.M;
+    a.MT = L.MT;
+    a.clock_logit = clock_logit;
+    a.decay_logit = decay_logit;
+    a.A = A;
+    a.dq = dq;
+    a.dk = dk;
+    a.dv = dv;
+    a.d_clock = d_clock_logit;
+    a.d_decay = d_decay_logit;
+    a.d_beta = d_beta_logit;
+    a.dA = dA;
+    a.states = L.states;
+    a.adj = L.adj;
+    a.o2 = L.o2;
+    a.do1 = L.do1;
+    a.tok = L.tok;
+    a.seg = L.seg;
+    a.dA_part = L.dA_part;
+    return cuda_status(launch_bwd_simt(a, st));
+}
+
+int cyfa_step(const cyfa_dims_t* dims, const void* q, const void* k, const void* v,
+              const float* clock_logit, const float* decay_logit, const float* beta_logit,
+              const float* A, const float* R, float* Kbar, float* Vbar, double* lambda, void* o,
+              void* stream) {
+    int rc = check_dims(dims, false);
+    if (rc) return rc;
+    if (!q || !k || !v || !clock_logit || !decay_logit || !beta_logit || !A || !R || !Kbar ||
+        !Vbar || !lambda || !o)
+        return CYFA_ERR_ARG;
+    if (!aligned16(q) || !aligned16(k) || !aligned16(v) || !aligned16(o) || !aligned16(Kbar) ||
+        !aligned16(Vbar))
+        return CYFA_ERR_ALIGN;
+    StepArgs a;
+    a.B = dims->B;
+    a.H = dims->H;
+    a.D = dims->dk;
+    a.scale = dims->scale;
+    a.bf16 = dims->dtype == CYFA_DTYPE_BF16;
+    a.q = q;
+    a.k = k;
+    a.v = v;
+    a.clock_logit = clock_logit;
+    a.decay_logit = decay_logit;
+    a.beta_logit = beta_logit;
+    a.A = A;
+    a.R = R;
+    a.Kbar = Kbar;
+    a.Vbar = Vbar;
+    a.lambda = lambda;
+    a.o = o;
+    return cuda_status(launch_step(a, static_cast<cudaStream_t>(stream)));
+}
+
+int cyfa_check(void* stream) {
+    if (cudaStreamSynchronize(static_cast<cudaStream_t>(stream)) != cudaSuccess)
+        return CYFA_ERR_CUDA;
+    return CYFA_OK;
+}
+
+}  // extern "C"

@@ -1,0 +1,75 @@
+// Launch interface between the C ABI (cyfa_api.cu) and the kernel translation units.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stddef.h>
+
+namespace cyfa {
+
+struct Shape {
+    int B, T, H, D, C;      // batch, tokens, heads, head dim (dk == dv), chunk
+    float scale;
+    bool bf16;
+    __host__ __device__ int nchunk() const { return T / C; }
+};
+
+// ---- prepare (prepare.cu) ----
+struct PrepareArgs {
+    Shape s;
+    const float *clock_logit, *decay_logit, *beta_logit, *A;
+    const double* lambda0;
+    float *lam_mod, *g_cum, *beta;
+    double* lambda_end;
+    double* seg_sum;   // workspace [B*H][nseg]
+};
+constexpr int PREP_SEG = 1024;  // tokens per prepare block (multiple of every chunk size)
+size_t prepare_workspace(const Shape& s);
+cudaError_t launch_prepare(const PrepareArgs& a, cudaStream_t st);
+
+// ---- readout matrix M = R Phi and its transpose (chunk_simt.cu) ----
+cudaError_t launch_readout_matrix(int H, const float* R, float* M, float* MT, cudaStream_t st);
+
+// ---- chunk forward / backward ----
+struct FwdArgs {
+    Shape s;
+    const void *q, *k, *v;
+    const float *lam, *g, *beta, *M, *MT;
+    const float *Kbar0, *Vbar0;
+    void* o;
+    float *Kout, *Vout;
+    float* states;      // workspace [B*H][nchunk][128][2D]: chunk-start [Kbar | Vbar]
+};
+cudaError_t launch_fwd_simt(const FwdArgs& a, cudaStream_t st);
+
+struct BwdArgs {
+    Shape s;            // s.C is the backward's own chunk length
+    const void *q, *k, *v, *dO;
+    const float *lam, *g, *beta, *M, *MT;
+    const float *clock_logit, *decay_logit, *A;
+    void *dq, *dk, *dv;
+    float *d_clock, *d_decay, *d_beta, *dA;
+    float* states;      // [B*H][nchunk][128][2D] chunk-start states
+    float* adj;         // [B*H][nchunk][128][2D] adjoints of the chunk-end states
+    float* o2;          // [B*H][T][128] o'' per token
+    float* do1;         // [B*H][T][128] dL/do' per token
+    float* tok;         // [4][B*T*H]: dG part 1, d lambda part 1, dG part 2 / d lambda part 2 / d beta
+    double* seg;        // [2][B*H][nseg] reverse-scan partials
+    double* dA_part;    // [B*H*nseg]
+};
+constexpr int BWD_C = 64;       // chunk length used by the SIMT backward
+cudaError_t launch_bwd_simt(const BwdArgs& a, cudaStream_t st);
+
+// ---- decode (decode.cu) ----
+struct StepArgs {
+    int B, H, D;
+    float scale;
+    bool bf16;
+    const void *q, *k, *v;
+    const float *clock_logit, *decay_logit, *beta_logit, *A, *R;
+    float *Kbar, *Vbar;
+    double* lambda;
+    void* o;
+};
+cudaError_t launch_step(const StepArgs& a, cudaStream_t st);
+
+}  // namespace cyfa

@@ -1,0 +1,126 @@
+// cyfa_prepare kernels: clock prefix sum (fp64 carry) reduced mod m, chunk-local cumulative
+// log-decays, and write strengths.  Sec. 3.1 Eq. cyfa-cumulative-clock; Sec. 3.4 forget gate;
+// App. B Eq. app-chunk-decay (gamma^r as exp of a chunk-local cumulative sum of log alpha).
+//
+// Layout: gates are [B, T, H] fp32.  Two launches: per (b, h, 1024-token segment) fp64 sums of
+// delta, then a block scan per segment that adds the sums of the segments before it.
+#include "common.cuh"
+#include "kernels.h"
+
+namespace cyfa {
+
+namespace {
+
+__device__ __forceinline__ double warp_sum_d(double x) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) x += __shfl_xor_sync(0xffffffffu, x, o);
+    return x;
+}
+
+__global__ void __launch_bounds__(256) prep_partial_kernel(PrepareArgs a, int nseg) {
+    const int seg = blockIdx.x, bh = blockIdx.y;
+    const int H = a.s.H, T = a.s.T;
+    const int b = bh / H, h = bh % H;
+    const int t0 = seg * PREP_SEG;
+    const int len = min(PREP_SEG, T - t0);
+    double acc = 0.0;
+    for (int i = threadIdx.x; i < len; i += blockDim.x)
+        acc += (double)sigmoidf_(a.clock_logit[((size_t)b * T + t0 + i) * H + h]);
+    __shared__ double red[8];
+    acc = warp_sum_d(acc);
+    if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = acc;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        double t = 0.0;
+        for (int w = 0; w < 8; ++w) t += red[w];
+        a.seg_sum[(size_t)bh * nseg + seg] = t;
+    }
+}
+
+__global__ void __launch_bounds__(256) prep_scan_kernel(PrepareArgs a, int nseg) {
+    const int seg = blockIdx.x, bh = blockIdx.y;
+    const int H = a.s.H, T = a.s.T, C = a.s.C;
+    const int b = bh / H, h = bh % H;
+    const int t0 = seg * PREP_SEG;
+    const int len = min(PREP_SEG, T - t0);
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    __shared__ double s_base;
+    __shared__ double s_wtot[8];
+
+    if (warp == 0) {
+        double x = 0.0;
+        for (int s = lane; s < seg; s += 32) x += a.seg_sum[(size_t)bh * nseg + s];
+        x = warp_sum_d(x);
+        if (lane == 0) s_base = x + (a.lambda0 ? a.lambda0[bh] : 0.0);
+    }
+
+    const float Ah = a.A[h];
+    double loc[4];
+    float lp[4];
+    double pref = 0.0;
+    float lpref = 0.f;
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+        const int i = 4 * threadIdx.x + u;
+        float d = 0.f, la = 0.f;
+        if (i < len) {
+            const size_t gi = ((size_t)b * T + t0 + i) * H + h;
+            d = sigmoidf_(a.clock_logit[gi]);
+            la = -Ah * softplusf_(a.decay_logit[gi]);
+            a.beta[gi] = sigmoidf_(a.beta_logit[gi]);
+        }
+        pref += (double)d;
+        loc[u] = pref;
+        lpref += la;
+        lp[u] = lpref;
+    }
+    // block-wide exclusive scan of the per-thread delta totals (fp64)
+    double incl = pref;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const double y = __shfl_up_sync(0xffffffffu, incl, o);
+        if (lane >= o) incl += y;
+    }
+    if (lane == 31) s_wtot[warp] = incl;
+    // chunk-local scan of log alpha: a chunk spans C/4 consecutive lanes of one warp
+    const int seg_lanes = C / 4;
+    float tot = lp[3];
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const float y = __shfl_up_sync(0xffffffffu, tot, o);
+        if (o < seg_lanes && (lane % seg_lanes) >= o) tot += y;
+    }
+    const float gex = tot - lp[3];
+    __syncthreads();
+    double wex = 0.0;
+    for (int w = 0; w < warp; ++w) wex += s_wtot[w];
+    const double excl = s_base + wex + (incl - pref);
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+        const int i = 4 * threadIdx.x + u;
+        if (i < len) {
+            const size_t gi = ((size_t)b * T + t0 + i) * H + h;
+            const double lam = excl + loc[u];
+            a.lam_mod[gi] = (float)(lam - 127.0 * floor(lam / 127.0));
+            a.g_cum[gi] = gex + lp[u];
+            if (a.lambda_end && t0 + i == T - 1) a.lambda_end[bh] = lam;
+        }
+    }
+}
+
+}  // namespace
+
+size_t prepare_workspace(const Shape& s) {
+    const size_t nseg = (s.T + PREP_SEG - 1) / PREP_SEG;
+    return nseg * (size_t)s.B * s.H * sizeof(double);
+}
+
+cudaError_t launch_prepare(const PrepareArgs& a, cudaStream_t st) {
+    const int nseg = (a.s.T + PREP_SEG - 1) / PREP_SEG;
+    dim3 grid(nseg, a.s.B * a.s.H);
+    prep_partial_kernel<<<grid, 256, 0, st>>>(a, nseg);
+    prep_scan_kernel<<<grid, 256, 0, st>>>(a, nseg);
+    return cudaGetLastError();
+}
+
+}  // namespace cyfa

@@ -1,0 +1,162 @@
+"""Thin Python binding of libcyfa.so (include/cyfa.h): argument marshalling only.
+
+Each function has the name of the C entry point it calls and takes torch tensors, passing
+their device pointers and the current CUDA stream.  All arithmetic runs in the library's
+kernels; when the library cannot be loaded the call raises (there is no fallback path).
+"""
+import ctypes
+import os
+
+import torch
+
+HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(HERE, 'libcyfa.so')
+
+CYFA_OK = 0
+CYFA_ERR_ARG, CYFA_ERR_SHAPE, CYFA_ERR_ALIGN, CYFA_ERR_WORKSPACE = -1, -2, -3, -4
+CYFA_ERR_CUDA, CYFA_ERR_TIMEOUT, CYFA_ERR_UNSUPPORTED = -5, -6, -7
+CYFA_DTYPE_BF16, CYFA_DTYPE_FP32 = 0, 1
+CYFA_WS_PREPARE, CYFA_WS_FWD, CYFA_WS_BWD = 0, 1, 2
+
+# Every symbol include/cyfa.h declares (checked by tests/test_abi.py).
+EXPORTS = ('cyfa_version', 'cyfa_error_string', 'cyfa_workspace_size', 'cyfa_prepare',
+           'cyfa_chunk_fwd', 'cyfa_chunk_bwd', 'cyfa_step', 'cyfa_check')
+
+
+class CyfaError(RuntimeError):
+    def __init__(self, code, msg):
+        super().__init__('%s (code %d)' % (msg, code))
+        self.code = code
+
+
+class Dims(ctypes.Structure):
+    _fields_ = [('B', ctypes.c_int), ('T', ctypes.c_int), ('H', ctypes.c_int),
+                ('dk', ctypes.c_int), ('dv', ctypes.c_int), ('m', ctypes.c_int),
+                ('chunk', ctypes.c_int), ('scale', ctypes.c_float), ('dtype', ctypes.c_int)]
+
+
+def dims(B, T, H, d, *, chunk=64, scale=None, dtype=torch.bfloat16, m=127):
+    return Dims(B, T, H, d, d, m, chunk, float(d ** -0.5 if scale is None else scale),
+                CYFA_DTYPE_BF16 if dtype == torch.bfloat16 else CYFA_DTYPE_FP32)
+
+
+_lib = None
+_VP = ctypes.c_void_p
+
+
+def load(path=LIB_PATH):
+    """Load libcyfa.so (once) and declare the C signatures."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    if not os.path.exists(path):
+        raise RuntimeError('libcyfa.so not built at %s: run __graft_entry__.build()' % path)
+    lib = ctypes.CDLL(path)
+    P = ctypes.POINTER(Dims)
+    lib.cyfa_version.restype = ctypes.c_int
+    lib.cyfa_error_string.restype = ctypes.c_char_p
+    lib.cyfa_error_string.argtypes = [ctypes.c_int]
+    lib.cyfa_workspace_size.argtypes = [P, ctypes.c_int, ctypes.POINTER(ctypes.c_size_t)]
+    lib.cyfa_prepare.argtypes = [P] + [_VP] * 9 + [_VP, ctypes.c_size_t, _VP]
+    lib.cyfa_chunk_fwd.argtypes = [P] + [_VP] * 13 + [ctypes.c_size_t, _VP]
+    lib.cyfa_chunk_bwd.argtypes = [P] + [_VP] * 20 + [ctypes.c_size_t, _VP]
+    lib.cyfa_step.argtypes = [P] + [_VP] * 13
+    lib.cyfa_check.argtypes = [_VP]
+    for name in EXPORTS:
+        getattr(lib, name).restype = ctypes.c_int if name != 'cyfa_error_string' else ctypes.c_char_p
+    _lib = lib
+    return lib
+
+
+def _ptr(t):
+    return None if t is None else ctypes.c_void_p(t.data_ptr())
+
+
+def _stream(stream=None):
+    s = torch.cuda.current_stream() if stream is None else stream
+    return ctypes.c_void_p(s.cuda_stream)
+
+
+def _ok(code):
+    if code != CYFA_OK:
+        raise CyfaError(code, load().cyfa_error_string(code).decode())
+
+
+def error_string(code):
+    return load().cyfa_error_string(code).decode()
+
+
+def version():
+    return load().cyfa_version()
+
+
+def cyfa_workspace_size(d, which):
+    n = ctypes.c_size_t(0)
+    _ok(load().cyfa_workspace_size(ctypes.byref(d), which, ctypes.byref(n)))
+    return n.value
+
+
+def workspace(d, which, device='cuda'):
+    return torch.empty(max(1, cyfa_workspace_size(d, which)), dtype=torch.uint8, device=device)
+
+
+def cyfa_prepare(d, clock_logit, decay_logit, beta_logit, A, lambda0, lam_mod, g_cum, beta,
+                 lambda_end, ws, stream=None):
+    _ok(load().cyfa_prepare(ctypes.byref(d), _ptr(clock_logit), _ptr(decay_logit),
+                            _ptr(beta_logit), _ptr(A), _ptr(lambda0), _ptr(lam_mod), _ptr(g_cum),
+                            _ptr(beta), _ptr(lambda_end), _ptr(ws), ws.numel(), _stream(stream)))
+
+
+def cyfa_chunk_fwd(d, q, k, v, lam_mod, g_cum, beta, R, Kbar0, Vbar0, o, Kbar_out, Vbar_out, ws,
+                   stream=None):
+    _ok(load().cyfa_chunk_fwd(ctypes.byref(d), _ptr(q), _ptr(k), _ptr(v), _ptr(lam_mod),
+                              _ptr(g_cum), _ptr(beta), _ptr(R), _ptr(Kbar0), _ptr(Vbar0), _ptr(o),
+                              _ptr(Kbar_out), _ptr(Vbar_out), _ptr(ws), ws.numel(),
+                              _stream(stream)))
+
+
+def cyfa_chunk_bwd(d, q, k, v, lam_mod, g_cum, beta, R, clock_logit, decay_logit, A, dO, dq, dk,
+                   dv, d_clock_logit, d_decay_logit, d_beta_logit, dR, dA, ws, stream=None):
+    _ok(load().cyfa_chunk_bwd(ctypes.byref(d), _ptr(q), _ptr(k), _ptr(v), _ptr(lam_mod),
+                              _ptr(g_cum), _ptr(beta), _ptr(R), _ptr(clock_logit),
+                              _ptr(decay_logit), _ptr(A), _ptr(dO), _ptr(dq), _ptr(dk), _ptr(dv),
+                              _ptr(d_clock_logit), _ptr(d_decay_logit), _ptr(d_beta_logit),
+                              _ptr(dR), _ptr(dA), _ptr(ws), ws.numel(), _stream(stream)))
+
+
+def cyfa_step(d, q, k, v, clock_logit, decay_logit, beta_logit, A, R, Kbar, Vbar, lam, o,
+              stream=None):
+    _ok(load().cyfa_step(ctypes.byref(d), _ptr(q), _ptr(k), _ptr(v), _ptr(clock_logit),
+                         _ptr(decay_logit), _ptr(beta_logit), _ptr(A), _ptr(R), _ptr(Kbar),
+                         _ptr(Vbar), _ptr(lam), _ptr(o), _stream(stream)))
+
+
+def cyfa_check(stream=None):
+    _ok(load().cyfa_check(_stream(stream)))
+
+
+# ---- convenience: whole calls with library-owned outputs (still argument marshalling) ----
+
+def prepare(d, clock_logit, decay_logit, beta_logit, A, lambda0=None, want_lambda_end=False):
+    B, T, H = clock_logit.shape
+    dev = clock_logit.device
+    lam = torch.empty(B, T, H, dtype=torch.float32, device=dev)
+    g = torch.empty_like(lam)
+    beta = torch.empty_like(lam)
+    lend = torch.empty(B, H, dtype=torch.float64, device=dev) if want_lambda_end else None
+    ws = workspace(d, CYFA_WS_PREPARE, dev)
+    cyfa_prepare(d, clock_logit, decay_logit, beta_logit, A, lambda0, lam, g, beta, lend, ws)
+    return lam, g, beta, lend
+
+
+def forward(d, q, k, v, lam, g, beta, R, Kbar0=None, Vbar0=None, want_state=False, ws=None):
+    o = torch.empty_like(v)
+    B, T, H, D = v.shape
+    Ko = Vo = None
+    if want_state:
+        Ko = torch.empty(B, H, 128, D, dtype=torch.float32, device=v.device)
+        Vo = torch.empty_like(Ko)
+    if ws is None:
+        ws = workspace(d, CYFA_WS_FWD, v.device)
+    cyfa_chunk_fwd(d, q, k, v, lam, g, beta, R, Kbar0, Vbar0, o, Ko, Vo, ws)
+    return o, Ko, Vo

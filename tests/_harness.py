@@ -1,0 +1,90 @@
+"""Shared helpers of the parity tests: run the library and the fp64 oracle on the same inputs."""
+import numpy as np
+import torch
+
+from oracle import backward as OB, forward as OF, gates as OG
+from paper_2609_36259_gb300 import cyfa, synth
+
+BF16_MAX_ABS = 2e-2    # parity bar for bf16 inputs with fp32 accumulation
+BF16_REL_L2 = 5e-3
+FP32_MAX_ABS = 1e-4    # parity bar for the fp32 configuration
+
+
+def rel_l2(a, b):
+    a = np.asarray(a, dtype=np.float64)
+    b = np.asarray(b, dtype=np.float64)
+    return float(np.linalg.norm(a - b) / max(np.linalg.norm(b), 1e-300))
+
+
+def assert_close_bf16(got, want, what=''):
+    got = np.asarray(got, dtype=np.float64)
+    want = np.asarray(want, dtype=np.float64)
+    err = float(np.max(np.abs(got - want))) if got.size else 0.0
+    rl = rel_l2(got, want)
+    assert err <= BF16_MAX_ABS and rl <= BF16_REL_L2, \
+        '%s: max-abs %.3e (bar %.0e), rel-L2 %.3e (bar %.0e)' % (what, err, BF16_MAX_ABS, rl, BF16_REL_L2)
+    return err, rl
+
+
+def assert_close_fp32(got, want, what=''):
+    err = float(np.max(np.abs(np.asarray(got, np.float64) - np.asarray(want, np.float64))))
+    assert err <= FP32_MAX_ABS, '%s: max-abs %.3e (bar %.0e)' % (what, err, FP32_MAX_ABS)
+    return err
+
+
+def pairs_np(x, pairs):
+    """Stack the (b, h) sequences of a [B, T, H, ...] tensor as float64 numpy [N, T, ...]."""
+    return np.stack([synth.pair_view(x, b, h) for b, h in pairs])
+
+
+def oracle_inputs(inp, pairs):
+    """Oracle arguments for the selected (b, h) pairs (gates in fp64 from the fp32 logits)."""
+    H = inp['q'].shape[2]
+    A = inp['A'].double().cpu().numpy()
+    hs = [h for _, h in pairs]
+    return dict(
+        q=pairs_np(inp['q'], pairs), k=pairs_np(inp['k'], pairs), v=pairs_np(inp['v'], pairs),
+        c=pairs_np(inp['clock_logit'], pairs), f=pairs_np(inp['decay_logit'], pairs),
+        bl=pairs_np(inp['beta_logit'], pairs), A=A[hs],
+        R=inp['R'].double().cpu().numpy()[hs], scale=inp['scale'], H=H)
+
+
+def oracle_forward(oi, lambda0=None, Kbar0=None, Vbar0=None):
+    delta = OG.clock_increment(oi['c'])
+    alpha = OG.forget_gate(oi['f'], oi['A'][:, None])
+    beta = OG.write_strength(oi['bl'])
+    return OF.absolute_clock(oi['q'], oi['k'], oi['v'], delta, alpha, beta, oi['R'], oi['scale'],
+                             lambda0=lambda0, Kbar0=Kbar0, Vbar0=Vbar0)
+
+
+def oracle_backward(oi, dO):
+    return OB.backward(oi['q'], oi['k'], oi['v'], oi['c'], oi['f'], oi['bl'], oi['A'], oi['R'],
+                       oi['scale'], dO)
+
+
+def to_device(inp, device='cuda'):
+    return {k: (v.to(device) if torch.is_tensor(v) else v) for k, v in inp.items()}
+
+
+def gpu_prepare(d, inp, lambda0=None, want_lambda_end=False):
+    return cyfa.prepare(d, inp['clock_logit'], inp['decay_logit'], inp['beta_logit'], inp['A'],
+                        lambda0=lambda0, want_lambda_end=want_lambda_end)
+
+
+def gpu_forward(d, inp, want_state=False, Kbar0=None, Vbar0=None, lambda0=None):
+    lam, g, beta, lend = gpu_prepare(d, inp, lambda0=lambda0, want_lambda_end=True)
+    o, Ko, Vo = cyfa.forward(d, inp['q'], inp['k'], inp['v'], lam, g, beta, inp['R'],
+                             Kbar0=Kbar0, Vbar0=Vbar0, want_state=want_state)
+    torch.cuda.synchronize()
+    return o, Ko, Vo, lend
+
+
+def sample_pairs(B, H, n, seed=0):
+    """n distinct (b, h) pairs, always including the first and last head (fastest and
+    slowest decay), drawn with a fixed seed."""
+    rng = np.random.default_rng(seed)
+    want = {(0, 0), (B - 1, H - 1)}
+    allp = [(b, h) for b in range(B) for h in range(H)]
+    while len(want) < min(n, len(allp)):
+        want.add(allp[rng.integers(len(allp))])
+    return sorted(want)

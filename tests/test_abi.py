@@ -1,0 +1,70 @@
+"""The C ABI library builds, loads without a GPU, exports every symbol include/cyfa.h declares,
+and rejects bad arguments on the host before anything is launched."""
+import ctypes
+import os
+import re
+
+import pytest
+
+from paper_2609_36259_gb300 import cyfa
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope='module')
+def lib():
+    if not os.path.exists(cyfa.LIB_PATH):
+        from paper_2609_36259_gb300 import build_lib
+        build_lib.build()
+    return cyfa.load()
+
+
+def declared_symbols():
+    text = open(os.path.join(ROOT, 'include', 'cyfa.h')).read()
+    text = re.sub(r'/\*.*?\*/', '', text, flags=re.S)
+    return sorted(set(re.findall(r'\b(cyfa_[a-z_]+)\s*\(', text)))
+
+
+def test_exports_every_declared_symbol(lib):
+    names = declared_symbols()
+    assert set(names) == set(cyfa.EXPORTS), names
+    for n in names:
+        assert hasattr(lib, n), n
+
+
+def test_version_and_errors(lib):
+    assert cyfa.version() >= 100
+    for code in (0, -1, -2, -3, -4, -5, -6, -7, -99):
+        assert isinstance(cyfa.error_string(code), str)
+
+
+def test_workspace_sizes(lib):
+    d = cyfa.dims(2, 32768, 16, 128, chunk=128)
+    fwd = cyfa.cyfa_workspace_size(d, cyfa.CYFA_WS_FWD)
+    # readout matrices (2 x H x 128 x 128 fp32) plus one [128 x 2D] fp32 state per chunk
+    assert fwd >= 2 * 16 * 128 * 128 * 4 + 2 * 16 * 256 * 128 * 256 * 4
+    assert cyfa.cyfa_workspace_size(d, cyfa.CYFA_WS_BWD) > 0
+    assert cyfa.cyfa_workspace_size(d, cyfa.CYFA_WS_PREPARE) >= 2 * 16 * 32 * 8
+
+
+@pytest.mark.parametrize('field,value,code', [
+    ('m', 63, cyfa.CYFA_ERR_SHAPE), ('dk', 96, cyfa.CYFA_ERR_SHAPE), ('chunk', 32, cyfa.CYFA_ERR_SHAPE),
+    ('T', 100, cyfa.CYFA_ERR_SHAPE), ('B', 0, cyfa.CYFA_ERR_ARG), ('dtype', 7, cyfa.CYFA_ERR_ARG)])
+def test_bad_dims_rejected_on_host(lib, field, value, code):
+    d = cyfa.dims(1, 128, 1, 128)
+    setattr(d, field, value)
+    n = ctypes.c_size_t()
+    assert lib.cyfa_workspace_size(ctypes.byref(d), cyfa.CYFA_WS_FWD, ctypes.byref(n)) == code
+
+
+def test_null_and_misaligned_pointers_rejected_on_host(lib):
+    d = cyfa.dims(1, 128, 1, 128)
+    nul = [None] * 13
+    assert lib.cyfa_chunk_fwd(ctypes.byref(d), *nul, 0, None) == cyfa.CYFA_ERR_ARG
+    bad = ctypes.c_void_p(0x1002)      # never dereferenced: rejected before any launch
+    good = ctypes.c_void_p(0x1000)
+    args = [bad, good, good, good, good, good, good, None, None, good, None, None, good]
+    assert lib.cyfa_chunk_fwd(ctypes.byref(d), *args, 1 << 30, None) == cyfa.CYFA_ERR_ALIGN
+    args = [good] * 7 + [None, None, good, None, None, good]
+    assert lib.cyfa_chunk_fwd(ctypes.byref(d), *args, 16, None) == cyfa.CYFA_ERR_WORKSPACE
+    assert lib.cyfa_step(ctypes.byref(d), *([None] * 13)) == cyfa.CYFA_ERR_ARG
