@@ -7,14 +7,11 @@
 //
 // States are stored in the paper's orientation: Kbar [128 x dk] (= (S^K)^T of App. B) and
 // Vbar [128 x dv], side by side as one [128 x 2D] row-major block per chunk.
-#include "common.cuh"
-#include "kernels.h"
+#include "simt_tiles.cuh"
 
 namespace cyfa {
 
 namespace {
-
-constexpr int LD = 129;   // padded row stride of [C][128] shared tiles
 
 // ---------------------------------------------------------------------------------------
 // M = R Phi (padded to 128 x 128 with a zero last row and column) and its transpose.
@@ -41,104 +38,6 @@ __global__ void __launch_bounds__(128) readout_matrix_kernel(const float* R, flo
     }
     M[((size_t)h * MS + i) * MS + col] = acc;
     MT[((size_t)h * MS + col) * MS + i] = acc;
-}
-
-// ---------------------------------------------------------------------------------------
-// Token-wise middle readout for rows r < C of sX (in place): o'' = U(-lam) M^T softmax(M U(lam) o')
-// with M = R Phi; the padding logit is excluded from the softmax and o''[127] = 0.
-// One warp per row; swarp holds 2 x 128 floats of scratch per warp.
-__device__ void middle_rows(float* sX, const float* slam, int C, const float* M, const float* MT,
-                            float* swarp) {
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    float* z = swarp + warp * 256;
-    float* p = z + 128;
-    for (int r = warp; r < C; r += 8) {
-        float* x = sX + r * LD;
-        const float lam = slam[r];
-        float cs[2], sn[2];
-#pragma unroll
-        for (int u = 0; u < 2; ++u) {
-            const int j = lane + 1 + 32 * u;
-            cs[u] = 1.f;
-            sn[u] = 0.f;
-            if (j <= NPAIR) {
-                sincospif(phase_pi(lam, j), &sn[u], &cs[u]);
-                const float xc = x[2 * j - 1], xs = x[2 * j];
-                z[2 * j - 1] = cs[u] * xc - sn[u] * xs;
-                z[2 * j] = sn[u] * xc + cs[u] * xs;
-            }
-        }
-        if (lane == 0) {
-            z[0] = x[0];
-            z[127] = 0.f;
-        }
-        __syncwarp();
-        float l[4] = {0.f, 0.f, 0.f, 0.f};
-        for (int k = 0; k < MS; ++k) {
-            const float zk = z[k];
-#pragma unroll
-            for (int u = 0; u < 4; ++u) l[u] = fmaf(MT[k * MS + lane + 32 * u], zk, l[u]);
-        }
-        if (lane == 31) l[3] = -INFINITY;
-        float mx = fmaxf(fmaxf(l[0], l[1]), fmaxf(l[2], l[3]));
-        mx = warp_max(mx);
-        float e[4], sum = 0.f;
-#pragma unroll
-        for (int u = 0; u < 4; ++u) {
-            e[u] = expf(l[u] - mx);
-            sum += e[u];
-        }
-        sum = warp_sum(sum);
-        const float inv = 1.f / sum;
-#pragma unroll
-        for (int u = 0; u < 4; ++u) p[lane + 32 * u] = e[u] * inv;
-        __syncwarp();
-        float y[4] = {0.f, 0.f, 0.f, 0.f};
-        for (int i = 0; i < MA; ++i) {
-            const float pi = p[i];
-#pragma unroll
-            for (int u = 0; u < 4; ++u) y[u] = fmaf(M[i * MS + lane + 32 * u], pi, y[u]);
-        }
-        __syncwarp();
-#pragma unroll
-        for (int u = 0; u < 4; ++u) z[lane + 32 * u] = y[u];
-        __syncwarp();
-#pragma unroll
-        for (int u = 0; u < 2; ++u) {
-            const int j = lane + 1 + 32 * u;
-            if (j <= NPAIR) {
-                const float yc = z[2 * j - 1], ys = z[2 * j];
-                x[2 * j - 1] = cs[u] * yc + sn[u] * ys;
-                x[2 * j] = -sn[u] * yc + cs[u] * ys;
-            }
-        }
-        if (lane == 0) {
-            x[0] = z[0];
-            x[127] = 0.f;
-        }
-        __syncwarp();
-    }
-}
-
-__device__ __forceinline__ void load_gates(const Shape& s, const float* lam, const float* g,
-                                           const float* beta, int b, int h, int t0, int C,
-                                           float* slam, float* sg, float* sbeta) {
-    for (int r = threadIdx.x; r < C; r += blockDim.x) {
-        const size_t gi = ((size_t)b * s.T + t0 + r) * s.H + h;
-        slam[r] = lam[gi];
-        sg[r] = g[gi];
-        sbeta[r] = beta[gi];
-    }
-}
-
-// Stage rows [r0, r0+nr) x columns [c0, c0+32) of a [B,T,H,D] tensor into dst[r][33].
-template <typename TI>
-__device__ __forceinline__ void stage_tok(float* dst, const TI* X, const Shape& s, int b, int h,
-                                          int t0, int nr, int c0, float mul) {
-    for (int e = threadIdx.x; e < nr * 32; e += blockDim.x) {
-        const int r = e >> 5, cc = e & 31;
-        dst[r * 33 + cc] = mul * ldf(X, (((size_t)b * s.T + t0 + r) * s.H + h) * s.D + c0 + cc);
-    }
 }
 
 // ---------------------------------------------------------------------------------------
@@ -351,6 +250,22 @@ cudaError_t launch_readout_matrix(int H, const float* R, float* M, float* MT, cu
     return cudaGetLastError();
 }
 
+cudaError_t launch_state_simt(const FwdArgs& a, cudaStream_t st) {
+    const Shape& s = a.s;
+#define CYFA_ST(CC)                                                                      \
+    if (s.C == CC) {                                                                     \
+        const size_t sm = (size_t)(CC * LD + CC * 33 + 3 * CC) * sizeof(float);         \
+        auto k = s.bf16 ? fwd_state_kernel<CC, __nv_bfloat16> : fwd_state_kernel<CC, float>; \
+        cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);   \
+        k<<<dim3(2 * s.D / 32, s.B * s.H), 256, sm, st>>>(a);                            \
+        return cudaGetLastError();                                                       \
+    }
+    CYFA_ST(64)
+    CYFA_ST(128)
+#undef CYFA_ST
+    return cudaErrorInvalidValue;
+}
+
 cudaError_t launch_fwd_simt(const FwdArgs& a, cudaStream_t st) {
     const Shape& s = a.s;
 #define CYFA_FWD(CC, DD)                                                               \
@@ -364,7 +279,5 @@ cudaError_t launch_fwd_simt(const FwdArgs& a, cudaStream_t st) {
 #undef CYFA_FWD
     return cudaErrorInvalidValue;
 }
-
-cudaError_t launch_bwd_simt(const BwdArgs&, cudaStream_t) { return cudaErrorNotSupported; }
 
 }  // namespace cyfa

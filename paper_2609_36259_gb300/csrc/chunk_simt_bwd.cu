@@ -1,0 +1,750 @@
+// fp32 SIMT backward of the CyFA operator (chunk length 64).
+//
+// The forward (App. B Eqs. app-cyfa-key-chunk / app-cyfa-value-chunk with the middle line of
+// Sec. 3.3 Eq. cyfa-two-pass) is differentiated chunk by chunk:
+//   1. chunk-start states are recomputed (forward state pass);
+//   2. bwd_intra1: per chunk, recompute O' and O''; dO'' = gamma o (dO Vbar^T) + (dO V^T o Gamma) A;
+//      the middle readout's gradient gives dO'; dQ = s [gamma o (dO' Kbar) + (dO' A^T o Gamma) K];
+//   3. a reverse chunk scan of the state adjoints, D_c = gamma^C D_{c+1} + sum_r gamma^r [dO'_r q~_r^T | o''_r dO_r^T];
+//   4. bwd_intra2: per chunk, dK, dV and dA (the write-vector gradient of both passes) from the
+//      intra-chunk scores and the adjoint D_{c+1} of the chunk-end state;
+//   5. reverse cumulative sums over tokens: d log alpha_s = sum_{t>=s} dG_t and
+//      d delta_s = sum_{t>=s} d lambda_t (App. D.1 Eq. app-clock-gradient-accumulation), then the
+//      activation derivatives to the logits.
+// Per token, with the scalar-gated identity dG_t = <q_t, dq_t> - <k_t, dk_t> applied to each pass
+// (key pass: q = s q, k = k, v = a; value pass: q = o'', k = a, v = v), and, from the three places
+// lambda_t enters (a_t = beta U(-lambda) b, z_t = U(lambda) o', o'' = U(-lambda) y):
+//   d lambda_t = -<da_t, Omega a_t> + <dz_t, Omega z_t> - <do''_t, Omega o''_t>,
+// Omega the generator of U (blocks (2 pi j / m) [[0, -1], [1, 0]]).
+#include "simt_tiles.cuh"
+
+namespace cyfa {
+
+namespace {
+
+constexpr int CB = BWD_C;          // 64
+constexpr int LPB = CB + 1;
+constexpr int TMB = CB / 16;       // 4 rows per thread
+
+__device__ __forceinline__ float freq(int j) { return 6.283185307179586f * (float)j / 127.f; }
+
+// <x, Omega y> for 128-vectors in shared memory, summed over the warp (pairs j = lane+1, lane+33).
+__device__ __forceinline__ float warp_omega_dot(const float* x, const float* y, int lane) {
+    float acc = 0.f;
+#pragma unroll
+    for (int u = 0; u < 2; ++u) {
+        const int j = lane + 1 + 32 * u;
+        if (j <= NPAIR)
+            acc += freq(j) * (x[2 * j] * y[2 * j - 1] - x[2 * j - 1] * y[2 * j]);
+    }
+    return warp_sum(acc);
+}
+
+// Gradient of the middle readout, one warp per row:
+// given o' (sO1), o'' (sO2) and dL/do'' (sD), writes dL/do' into sD and the row scalars
+// sdG[r] = <o'', do''> and sdL[r] = <dz, Omega z> - <do'', Omega o''>.
+__device__ __noinline__ void middle_rows_bwd(const float* sO1, const float* sO2, float* sD,
+                                             const float* slam, int C, const float* M,
+                                             const float* MT, float* swarp, float* sdG,
+                                             float* sdL) {
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    float* z = swarp + warp * 640;
+    float* p = z + 128;
+    float* dy = p + 128;
+    float* dl = dy + 128;
+    float* dz = dl + 128;
+    for (int r = warp; r < C; r += 8) {
+        const float* x1 = sO1 + r * LD;
+        const float* x2 = sO2 + r * LD;
+        float* xd = sD + r * LD;
+        const float lam = slam[r];
+        float cs[2], sn[2];
+#pragma unroll
+        for (int u = 0; u < 2; ++u) {
+            const int j = lane + 1 + 32 * u;
+            cs[u] = 1.f;
+            sn[u] = 0.f;
+            if (j <= NPAIR) {
+                sincospif(phase_pi(lam, j), &sn[u], &cs[u]);
+                const float xc = x1[2 * j - 1], xs = x1[2 * j];
+                z[2 * j - 1] = cs[u] * xc - sn[u] * xs;
+                z[2 * j] = sn[u] * xc + cs[u] * xs;
+                const float gc = xd[2 * j - 1], gs = xd[2 * j];
+                dy[2 * j - 1] = cs[u] * gc - sn[u] * gs;     // dy = U(lam) do''
+                dy[2 * j] = sn[u] * gc + cs[u] * gs;
+            }
+        }
+        if (lane == 0) {
+            z[0] = x1[0];
+            z[127] = 0.f;
+            dy[0] = xd[0];
+            dy[127] = 0.f;
+        }
+        __syncwarp();
+        float g1 = 0.f;
+#pragma unroll
+        for (int u = 0; u < 4; ++u) g1 += x2[lane + 32 * u] * xd[lane + 32 * u];
+        g1 = warp_sum(g1);
+        const float om2 = warp_omega_dot(xd, x2, lane);      // <do'', Omega o''>
+        // logits and softmax
+        float l[4] = {0.f, 0.f, 0.f, 0.f}, dp[4] = {0.f, 0.f, 0.f, 0.f};
+        for (int k = 0; k < MS; ++k) {
+            const float zk = z[k], dyk = dy[k];
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+                const float mt = MT[k * MS + lane + 32 * u];
+                l[u] = fmaf(mt, zk, l[u]);
+                dp[u] = fmaf(mt, dyk, dp[u]);           // dp = M dy
+            }
+        }
+        if (lane == 31) l[3] = -INFINITY;
+        float mx = warp_max(fmaxf(fmaxf(l[0], l[1]), fmaxf(l[2], l[3])));
+        float e[4], sum = 0.f;
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+            e[u] = expf(l[u] - mx);
+            sum += e[u];
+        }
+        sum = warp_sum(sum);
+        const float inv = 1.f / sum;
+        float pdp = 0.f;
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+            e[u] *= inv;
+            pdp += e[u] * dp[u];
+        }
+        pdp = warp_sum(pdp);
+#pragma unroll
+        for (int u = 0; u < 4; ++u) dl[lane + 32 * u] = e[u] * (dp[u] - pdp);
+        __syncwarp();
+        float g[4] = {0.f, 0.f, 0.f, 0.f};                   // dz = M^T dl
+        for (int i = 0; i < MA; ++i) {
+            const float di = dl[i];
+#pragma unroll
+            for (int u = 0; u < 4; ++u) g[u] = fmaf(M[i * MS + lane + 32 * u], di, g[u]);
+        }
+#pragma unroll
+        for (int u = 0; u < 4; ++u) dz[lane + 32 * u] = g[u];
+        __syncwarp();
+        const float om1 = warp_omega_dot(dz, z, lane);       // <dz, Omega z>
+        // do' = U(-lam) dz
+#pragma unroll
+        for (int u = 0; u < 2; ++u) {
+            const int j = lane + 1 + 32 * u;
+            if (j <= NPAIR) {
+                const float gc = dz[2 * j - 1], gs = dz[2 * j];
+                xd[2 * j - 1] = cs[u] * gc + sn[u] * gs;
+                xd[2 * j] = -sn[u] * gc + cs[u] * gs;
+            }
+        }
+        if (lane == 0) {
+            xd[0] = dz[0];
+            xd[127] = 0.f;
+            sdG[r] = g1;
+            sdL[r] = om1 - om2;
+        }
+        __syncwarp();
+    }
+}
+
+// sP[r][t] = mul * (sum_k X(r,k) Y(t,k)) * exp(g_r - g_t) for t <= r, else 0
+template <class FX, class FY>
+__device__ __forceinline__ void masked_scores(float* sP, const float* sg, int K, float mul,
+                                              const FX& fx, const FY& fy) {
+    const int tx = threadIdx.x & 15, ty = threadIdx.x >> 4;
+    float acc[TMB][TMB];
+    zero_acc(acc);
+    simt_mm<TMB, TMB>(acc, K, fx, fy);
+#pragma unroll
+    for (int i = 0; i < TMB; ++i)
+#pragma unroll
+        for (int j = 0; j < TMB; ++j) {
+            const int r = ty + 16 * i, t = tx + 16 * j;
+            sP[r * LPB + t] = (t <= r) ? acc[i][j] * mul * expf(sg[r] - sg[t]) : 0.f;
+        }
+}
+
+// masked scores from two token tensors staged 32 columns at a time through sS
+template <typename TI>
+__device__ __forceinline__ void masked_scores_tok(float* sP, float* sS, const float* sg,
+                                                  const TI* X, const TI* Y, const Shape& s, int b,
+                                                  int h, int t0, float mul) {
+    const int tx = threadIdx.x & 15, ty = threadIdx.x >> 4;
+    float acc[TMB][TMB];
+    zero_acc(acc);
+    for (int d0 = 0; d0 < s.D; d0 += 32) {
+        __syncthreads();
+        stage_tok(sS, X, s, b, h, t0, CB, d0, 1.f);
+        stage_tok(sS + CB * 33, Y, s, b, h, t0, CB, d0, 1.f);
+        __syncthreads();
+        simt_mm<TMB, TMB>(acc, 32, [&](int r, int kk) { return sS[r * 33 + kk]; },
+                          [&](int kk, int t) { return sS[CB * 33 + t * 33 + kk]; });
+    }
+#pragma unroll
+    for (int i = 0; i < TMB; ++i)
+#pragma unroll
+        for (int j = 0; j < TMB; ++j) {
+            const int r = ty + 16 * i, t = tx + 16 * j;
+            sP[r * LPB + t] = (t <= r) ? acc[i][j] * mul * expf(sg[r] - sg[t]) : 0.f;
+        }
+}
+
+// acc[r][i] += sum_d X[r][d] * Sst[i][coff + d]  (X a token tensor, Sst a [128][2D] state block)
+template <typename TI>
+__device__ __forceinline__ void tok_times_stateT(float (&acc)[TMB][8], float* sS, const TI* X,
+                                                 const float* Sst, int coff, const Shape& s,
+                                                 int b, int h, int t0) {
+    for (int d0 = 0; d0 < s.D; d0 += 32) {
+        __syncthreads();
+        stage_tok(sS, X, s, b, h, t0, CB, d0, 1.f);
+        for (int e = threadIdx.x; e < MS * 32; e += blockDim.x) {
+            const int i = e >> 5, dd = e & 31;
+            sS[CB * 33 + i * 33 + dd] = Sst[i * (2 * s.D) + coff + d0 + dd];
+        }
+        __syncthreads();
+        simt_mm<TMB, 8>(acc, 32, [&](int r, int kk) { return sS[r * 33 + kk]; },
+                        [&](int kk, int i) { return sS[CB * 33 + i * 33 + kk]; });
+    }
+}
+
+// acc[r][dd] += sum_i Y(r, i) * Sst[i][coff + dd]  (Y rows in shared memory with stride LD)
+template <int TN>
+__device__ __forceinline__ void rows_times_state(float (&acc)[TMB][TN], float* sS, const float* Y,
+                                                 const float* Sst, int coff, int D) {
+    for (int i0 = 0; i0 < MS; i0 += 32) {
+        __syncthreads();
+        for (int e = threadIdx.x; e < 32 * D; e += blockDim.x) {
+            const int ii = e / D, dd = e % D;
+            sS[ii * (D + 1) + dd] = Sst[(i0 + ii) * (2 * D) + coff + dd];
+        }
+        __syncthreads();
+        simt_mm<TMB, TN>(acc, 32, [&](int r, int ii) { return Y[r * LD + i0 + ii]; },
+                         [&](int ii, int dd) { return sS[ii * (D + 1) + dd]; });
+    }
+}
+
+// acc[r][dd] += sum_t P(r, t) * X[t][dd]  with P given by an accessor (K = CB tokens)
+template <int TN, typename TI, class FP>
+__device__ __forceinline__ void scores_times_tok(float (&acc)[TMB][TN], float* sS, const FP& fp,
+                                                 const TI* X, const Shape& s, int b, int h,
+                                                 int t0, float mul) {
+    const int D = s.D;
+    for (int s0 = 0; s0 < CB; s0 += 32) {
+        __syncthreads();
+        for (int e = threadIdx.x; e < 32 * D; e += blockDim.x) {
+            const int ss = e / D, dd = e % D;
+            sS[ss * (D + 1) + dd] = mul * ldf(X, (((size_t)b * s.T + t0 + s0 + ss) * s.H + h) * D + dd);
+        }
+        __syncthreads();
+        simt_mm<TMB, TN>(acc, 32, [&](int r, int ss) { return fp(r, s0 + ss); },
+                         [&](int ss, int dd) { return sS[ss * (D + 1) + dd]; });
+    }
+}
+
+// ---------------------------------------------------------------------------------------
+template <int D, typename TI>
+__global__ void __launch_bounds__(256) bwd_intra1_kernel(BwdArgs a) {
+    const Shape s = a.s;
+    constexpr int TN = D / 16;
+    const int c = blockIdx.x, bh = blockIdx.y, b = bh / s.H, h = bh % s.H;
+    const int nchunk = s.nchunk(), t0 = c * CB;
+    extern __shared__ float smem[];
+    float* sA = smem;
+    float* sO1 = sA + CB * LD;
+    float* sO2 = sO1 + CB * LD;
+    float* sD = sO2 + CB * LD;
+    float* sS = sD + CB * LD;
+    float* sP = sS + CB * LD;
+    float* sg = sP + CB * LPB;
+    float* seg = sg + CB;
+    float* slam = seg + CB;
+    float* sbeta = slam + CB;
+    float* sdG = sbeta + CB;
+    float* sdL = sdG + CB;
+    float* swarp = sdL + CB;     // [8][640]
+    const int tx = threadIdx.x & 15, ty = threadIdx.x >> 4;
+    const float* Sst = a.states + ((size_t)bh * nchunk + c) * MS * (2 * D);
+    const float* Mh = a.M + (size_t)h * MS * MS;
+    const float* MTh = a.MT + (size_t)h * MS * MS;
+    const TI* Q = (const TI*)a.q;
+    const TI* K = (const TI*)a.k;
+    const TI* V = (const TI*)a.v;
+    const TI* dO = (const TI*)a.dO;
+
+    load_gates(s, a.lam, a.g, a.beta, b, h, t0, CB, slam, sg, sbeta);
+    __syncthreads();
+    for (int r = threadIdx.x; r < CB; r += blockDim.x) seg[r] = expf(sg[r]);
+    build_write_rows(sA, LD, slam, sbeta, CB, [](int) { return 1.f; });
+
+    // O' = s gamma o (Q Kbar^T) + (s Q K^T o Gamma) A
+    masked_scores_tok(sP, sS, sg, Q, K, s, b, h, t0, s.scale);
+    {
+        float o1[TMB][8];
+        zero_acc(o1);
+        tok_times_stateT(o1, sS, Q, Sst, 0, s, b, h, t0);
+#pragma unroll
+        for (int i = 0; i < TMB; ++i)
+#pragma unroll
+            for (int j = 0; j < 8; ++j) o1[i][j] *= s.scale * seg[ty + 16 * i];
+        simt_mm<TMB, 8>(o1, CB, [&](int r, int t) { return sP[r * LPB + t]; },
+                        [&](int t, int i) { return sA[t * LD + i]; });
+#pragma unroll
+        for (int i = 0; i < TMB; ++i)
+#pragma unroll
+            for (int j = 0; j < 8; ++j) {
+                sO1[(ty + 16 * i) * LD + tx + 16 * j] = o1[i][j];
+                sO2[(ty + 16 * i) * LD + tx + 16 * j] = o1[i][j];
+            }
+    }
+    __syncthreads();
+    middle_rows(sO2, slam, CB, Mh, MTh, swarp);
+
+    // dO'' = gamma o (dO Vbar^T) + (dO V^T o Gamma) A
+    masked_scores_tok(sP, sS, sg, dO, V, s, b, h, t0, 1.f);
+    {
+        float g2[TMB][8];
+        zero_acc(g2);
+        tok_times_stateT(g2, sS, dO, Sst, D, s, b, h, t0);
+#pragma unroll
+        for (int i = 0; i < TMB; ++i)
+#pragma unroll
+            for (int j = 0; j < 8; ++j) g2[i][j] *= seg[ty + 16 * i];
+        simt_mm<TMB, 8>(g2, CB, [&](int r, int t) { return sP[r * LPB + t]; },
+                        [&](int t, int i) { return sA[t * LD + i]; });
+#pragma unroll
+        for (int i = 0; i < TMB; ++i)
+#pragma unroll
+            for (int j = 0; j < 8; ++j) sD[(ty + 16 * i) * LD + tx + 16 * j] = g2[i][j];
+    }
+    __syncthreads();
+    middle_rows_bwd(sO1, sO2, sD, slam, CB, Mh, MTh, swarp, sdG, sdL);
+    __syncthreads();
+
+    // dQ~ = gamma o (dO' Kbar) + (dO' A^T o Gamma) K ;  dq = s dQ~
+    masked_scores(sP, sg, MS, 1.f, [&](int r, int kk) { return sD[r * LD + kk]; },
+                  [&](int kk, int t) { return sA[t * LD + kk]; });
+    {
+        float dqa[TMB][TN];
+        zero_acc(dqa);
+        rows_times_state<TN>(dqa, sS, sD, Sst, 0, D);
+#pragma unroll
+        for (int i = 0; i < TMB; ++i)
+#pragma unroll
+            for (int j = 0; j < TN; ++j) dqa[i][j] *= seg[ty + 16 * i];
+        scores_times_tok<TN>(dqa, sS, [&](int r, int t) { return sP[r * LPB + t]; }, K, s, b, h,
+                             t0, 1.f);
+        TI* dQ = (TI*)a.dq;
+#pragma unroll
+        for (int i = 0; i < TMB; ++i) {
+            const int r = ty + 16 * i;
+            float part = 0.f;
+#pragma unroll
+            for (int j = 0; j < TN; ++j) {
+                const size_t idx = (((size_t)b * s.T + t0 + r) * s.H + h) * D + tx + 16 * j;
+                part += ldf(Q, idx) * dqa[i][j];             // <q, dq~ / s> * s = <q~, dq~>
+                stf(dQ, idx, s.scale * dqa[i][j]);
+            }
+            part = half_warp_sum(part) * s.scale;
+            if (tx == 0) sdG[r] += part;
+        }
+    }
+    __syncthreads();
+    // stash o'' and dL/do' for the adjoint scan and the second intra-chunk pass
+    float* o2 = a.o2 + ((size_t)bh * s.T + t0) * MS;
+    float* do1 = a.do1 + ((size_t)bh * s.T + t0) * MS;
+    for (int e = threadIdx.x; e < CB * MS; e += blockDim.x) {
+        const int r = e >> 7, i = e & 127;
+        o2[e] = sO2[r * LD + i];
+        do1[e] = sD[r * LD + i];
+    }
+    const size_t BTH = (size_t)s.B * s.T * s.H;
+    for (int r = threadIdx.x; r < CB; r += blockDim.x) {
+        const size_t gi = ((size_t)b * s.T + t0 + r) * s.H + h;
+        a.tok[gi] = sdG[r];
+        a.tok[BTH + gi] = sdL[r];
+    }
+}
+
+// Reverse scan of the state adjoints, one block per (b, h, 32-column tile of [D^K | D^V]).
+// Stores, for every chunk c, the adjoint of the state at the end of chunk c.
+template <typename TI>
+__global__ void __launch_bounds__(256) adj_state_kernel(BwdArgs a) {
+    const Shape s = a.s;
+    const int D = s.D, W = 2 * s.D;
+    const int bh = blockIdx.y, b = bh / s.H, h = bh % s.H;
+    const int col0 = blockIdx.x * 32;
+    const bool isK = col0 < D;
+    const int xc0 = isK ? col0 : col0 - D;
+    const TI* X = (const TI*)(isK ? a.q : a.dO);
+    const float* Y = isK ? a.do1 : a.o2;
+    const float xmul = isK ? s.scale : 1.f;
+    extern __shared__ float smem[];
+    float* sY = smem;            // [CB][LD]
+    float* sX = sY + CB * LD;    // [CB][33]
+    float* sg = sX + CB * 33;
+    const int tx = threadIdx.x & 15, ty = threadIdx.x >> 4;
+    float S[8][2];
+    zero_acc(S);
+    const int nchunk = s.nchunk();
+    for (int c = nchunk - 1; c >= 0; --c) {
+        float* dst = a.adj + ((size_t)bh * nchunk + c) * MS * W;
+#pragma unroll
+        for (int i = 0; i < 8; ++i)
+#pragma unroll
+            for (int j = 0; j < 2; ++j) dst[(ty + 16 * i) * W + col0 + tx + 16 * j] = S[i][j];
+        const int t0 = c * CB;
+        __syncthreads();
+        for (int r = threadIdx.x; r < CB; r += blockDim.x)
+            sg[r] = a.g[((size_t)b * s.T + t0 + r) * s.H + h];
+        stage_tok(sX, X, s, b, h, t0, CB, xc0, xmul);
+        __syncthreads();
+        const float* Yc = Y + ((size_t)bh * s.T + t0) * MS;
+        for (int e = threadIdx.x; e < CB * MS; e += blockDim.x) {
+            const int r = e >> 7, i = e & 127;
+            sY[r * LD + i] = Yc[e] * expf(sg[r]);
+        }
+        __syncthreads();
+        const float decay = expf(sg[CB - 1]);
+#pragma unroll
+        for (int i = 0; i < 8; ++i)
+#pragma unroll
+            for (int j = 0; j < 2; ++j) S[i][j] *= decay;
+        simt_mm<8, 2>(S, CB, [&](int row, int t) { return sY[t * LD + row]; },
+                      [&](int t, int col) { return sX[t * 33 + col]; });
+    }
+}
+
+template <int D, typename TI>
+__global__ void __launch_bounds__(256) bwd_intra2_kernel(BwdArgs a) {
+    const Shape s = a.s;
+    constexpr int TN = D / 16;
+    const int c = blockIdx.x, bh = blockIdx.y, b = bh / s.H, h = bh % s.H;
+    const int nchunk = s.nchunk(), t0 = c * CB;
+    extern __shared__ float smem[];
+    float* sA = smem;
+    float* sY1 = sA + CB * LD;     // dL/do'
+    float* sY2 = sY1 + CB * LD;    // o''
+    float* sDA = sY2 + CB * LD;    // dL/da
+    float* sS = sDA + CB * LD;
+    float* sP = sS + CB * LD;
+    float* sg = sP + CB * LPB;
+    float* sfw = sg + CB;
+    float* slam = sfw + CB;
+    float* sbeta = slam + CB;
+    float* sdG = sbeta + CB;
+    const int tx = threadIdx.x & 15, ty = threadIdx.x >> 4;
+    const float* Dst = a.adj + ((size_t)bh * nchunk + c) * MS * (2 * D);
+    const TI* Q = (const TI*)a.q;
+    const TI* K = (const TI*)a.k;
+    const TI* V = (const TI*)a.v;
+    const TI* dO = (const TI*)a.dO;
+    const size_t tokbase = ((size_t)b * s.T + t0) * s.H + h;
+
+    load_gates(s, a.lam, a.g, a.beta, b, h, t0, CB, slam, sg, sbeta);
+    {
+        const float* y1 = a.do1 + ((size_t)bh * s.T + t0) * MS;
+        const float* y2 = a.o2 + ((size_t)bh * s.T + t0) * MS;
+        for (int e = threadIdx.x; e < CB * MS; e += blockDim.x) {
+            const int r = e >> 7, i = e & 127;
+            sY1[r * LD + i] = y1[e];
+            sY2[r * LD + i] = y2[e];
+        }
+    }
+    __syncthreads();
+    for (int r = threadIdx.x; r < CB; r += blockDim.x) {
+        sfw[r] = expf(sg[CB - 1] - sg[r]);
+        sdG[r] = 0.f;
+    }
+    build_write_rows(sA, LD, slam, sbeta, CB, [](int) { return 1.f; });
+    __syncthreads();
+
+    // dK = P3^T (s Q) + diag(fw) A D^K,  P3 = (dO' A^T) o Gamma
+    masked_scores(sP, sg, MS, 1.f, [&](int r, int kk) { return sY1[r * LD + kk]; },
+                  [&](int kk, int t) { return sA[t * LD + kk]; });
+    {
+        float acc[TMB][TN];
+        zero_acc(acc);
+        rows_times_state<TN>(acc, sS, sA, Dst, 0, D);
+#pragma unroll
+        for (int i = 0; i < TMB; ++i)
+#pragma unroll
+            for (int j = 0; j < TN; ++j) acc[i][j] *= sfw[ty + 16 * i];
+        scores_times_tok<TN>(acc, sS, [&](int t, int r) { return sP[r * LPB + t]; }, Q, s, b, h,
+                             t0, s.scale);
+        TI* dK = (TI*)a.dk;
+#pragma unroll
+        for (int i = 0; i < TMB; ++i) {
+            const int t = ty + 16 * i;
+            float part = 0.f;
+#pragma unroll
+            for (int j = 0; j < TN; ++j) {
+                const size_t idx = ((tokbase + (size_t)t * s.H)) * D + tx + 16 * j;
+                part += ldf(K, idx) * acc[i][j];
+                stf(dK, idx, acc[i][j]);
+            }
+            part = half_warp_sum(part);
+            if (tx == 0) sdG[t] -= part;
+        }
+    }
+    // dV = P2^T dO + diag(fw) A D^V,  P2 = (O'' A^T) o Gamma
+    __syncthreads();
+    masked_scores(sP, sg, MS, 1.f, [&](int r, int kk) { return sY2[r * LD + kk]; },
+                  [&](int kk, int t) { return sA[t * LD + kk]; });
+    {
+        float acc[TMB][TN];
+        zero_acc(acc);
+        rows_times_state<TN>(acc, sS, sA, Dst, D, D);
+#pragma unroll
+        for (int i = 0; i < TMB; ++i)
+#pragma unroll
+            for (int j = 0; j < TN; ++j) acc[i][j] *= sfw[ty + 16 * i];
+        scores_times_tok<TN>(acc, sS, [&](int t, int r) { return sP[r * LPB + t]; }, dO, s, b, h,
+                             t0, 1.f);
+        TI* dV = (TI*)a.dv;
+#pragma unroll
+        for (int i = 0; i < TMB; ++i)
+#pragma unroll
+            for (int j = 0; j < TN; ++j)
+                stf(dV, (tokbase + (size_t)(ty + 16 * i) * s.H) * D + tx + 16 * j, acc[i][j]);
+    }
+    // dA^V = P4^T O'' + diag(fw) V (D^V)^T,  P4 = (dO V^T) o Gamma
+    masked_scores_tok(sP, sS, sg, dO, V, s, b, h, t0, 1.f);
+    {
+        float acc[TMB][8];
+        zero_acc(acc);
+        tok_times_stateT(acc, sS, V, Dst, D, s, b, h, t0);
+#pragma unroll
+        for (int i = 0; i < TMB; ++i)
+#pragma unroll
+            for (int j = 0; j < 8; ++j) acc[i][j] *= sfw[ty + 16 * i];
+        simt_mm<TMB, 8>(acc, CB, [&](int t, int r) { return sP[r * LPB + t]; },
+                        [&](int r, int i) { return sY2[r * LD + i]; });
+#pragma unroll
+        for (int i = 0; i < TMB; ++i) {
+            const int t = ty + 16 * i;
+            float part = 0.f;
+#pragma unroll
+            for (int j = 0; j < 8; ++j) {
+                sDA[t * LD + tx + 16 * j] = acc[i][j];
+                part += sA[t * LD + tx + 16 * j] * acc[i][j];
+            }
+            part = half_warp_sum(part);
+            if (tx == 0) sdG[t] -= part;
+        }
+    }
+    // dA^K = P1^T dO' + diag(fw) K (D^K)^T,  P1 = (s Q K^T) o Gamma
+    masked_scores_tok(sP, sS, sg, Q, K, s, b, h, t0, s.scale);
+    {
+        float acc[TMB][8];
+        zero_acc(acc);
+        tok_times_stateT(acc, sS, K, Dst, 0, s, b, h, t0);
+#pragma unroll
+        for (int i = 0; i < TMB; ++i)
+#pragma unroll
+            for (int j = 0; j < 8; ++j) acc[i][j] *= sfw[ty + 16 * i];
+        simt_mm<TMB, 8>(acc, CB, [&](int t, int r) { return sP[r * LPB + t]; },
+                        [&](int r, int i) { return sY1[r * LD + i]; });
+#pragma unroll
+        for (int i = 0; i < TMB; ++i)
+#pragma unroll
+            for (int j = 0; j < 8; ++j) sDA[(ty + 16 * i) * LD + tx + 16 * j] += acc[i][j];
+    }
+    __syncthreads();
+    // per token: d beta, d lambda from the write vector, dG
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const size_t BTH = (size_t)s.B * s.T * s.H;
+    for (int t = warp; t < CB; t += 8) {
+        const float* da = sDA + t * LD;
+        const float* av = sA + t * LD;
+        float db = 0.f;
+#pragma unroll
+        for (int u = 0; u < 4; ++u) db += da[lane + 32 * u] * av[lane + 32 * u];
+        db = warp_sum(db);
+        const float om = warp_omega_dot(da, av, lane);       // <da, Omega a>
+        if (lane == 0) {
+            const size_t gi = tokbase + (size_t)t * s.H;
+            a.tok[2 * BTH + gi] = sdG[t];
+            a.tok[3 * BTH + gi] = -om;
+            a.tok[4 * BTH + gi] = db / sbeta[t];
+        }
+    }
+}
+
+// ---------------------------------------------------------------------------------------
+// Reverse cumulative sums over tokens (fp64) and the activation derivatives.
+__device__ __forceinline__ double warp_sum_d(double x) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) x += __shfl_xor_sync(0xffffffffu, x, o);
+    return x;
+}
+
+__global__ void __launch_bounds__(256) gate_partial_kernel(BwdArgs a, int nseg) {
+    const Shape s = a.s;
+    const int seg = blockIdx.x, bh = blockIdx.y, b = bh / s.H, h = bh % s.H;
+    const int t0 = seg * PREP_SEG, len = min(PREP_SEG, s.T - t0);
+    const size_t BTH = (size_t)s.B * s.T * s.H;
+    double sg = 0.0, sl = 0.0;
+    for (int i = threadIdx.x; i < len; i += blockDim.x) {
+        const size_t gi = ((size_t)b * s.T + t0 + i) * s.H + h;
+        sg += (double)a.tok[gi] + (double)a.tok[2 * BTH + gi];
+        sl += (double)a.tok[BTH + gi] + (double)a.tok[3 * BTH + gi];
+    }
+    __shared__ double red[2][8];
+    sg = warp_sum_d(sg);
+    sl = warp_sum_d(sl);
+    if ((threadIdx.x & 31) == 0) {
+        red[0][threadIdx.x >> 5] = sg;
+        red[1][threadIdx.x >> 5] = sl;
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        double x = 0.0, y = 0.0;
+        for (int w = 0; w < 8; ++w) {
+            x += red[0][w];
+            y += red[1][w];
+        }
+        const size_t BHn = (size_t)s.B * s.H * nseg;
+        a.seg[(size_t)bh * nseg + seg] = x;
+        a.seg[BHn + (size_t)bh * nseg + seg] = y;
+    }
+}
+
+__global__ void __launch_bounds__(256) gate_scan_kernel(BwdArgs a, int nseg) {
+    const Shape s = a.s;
+    const int seg = blockIdx.x, bh = blockIdx.y, b = bh / s.H, h = bh % s.H;
+    const int t0 = seg * PREP_SEG, len = min(PREP_SEG, s.T - t0);
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const size_t BTH = (size_t)s.B * s.T * s.H;
+    const size_t BHn = (size_t)s.B * s.H * nseg;
+    __shared__ double s_base[2], s_wt[2][8], s_red[8];
+    if (warp == 0) {
+        double x = 0.0, y = 0.0;
+        for (int k = seg + 1 + lane; k < nseg; k += 32) {
+            x += a.seg[(size_t)bh * nseg + k];
+            y += a.seg[BHn + (size_t)bh * nseg + k];
+        }
+        x = warp_sum_d(x);
+        y = warp_sum_d(y);
+        if (lane == 0) {
+            s_base[0] = x;
+            s_base[1] = y;
+        }
+    }
+    double xg[4], xl[4], tg = 0.0, tl = 0.0;
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+        const int i = 4 * threadIdx.x + u;
+        xg[u] = xl[u] = 0.0;
+        if (i < len) {
+            const size_t gi = ((size_t)b * s.T + t0 + i) * s.H + h;
+            xg[u] = (double)a.tok[gi] + (double)a.tok[2 * BTH + gi];
+            xl[u] = (double)a.tok[BTH + gi] + (double)a.tok[3 * BTH + gi];
+        }
+        tg += xg[u];
+        tl += xl[u];
+    }
+    double ig = tg, il = tl;     // inclusive prefix over lanes
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const double yg = __shfl_up_sync(0xffffffffu, ig, o);
+        const double yl = __shfl_up_sync(0xffffffffu, il, o);
+        if (lane >= o) {
+            ig += yg;
+            il += yl;
+        }
+    }
+    const double wg = __shfl_sync(0xffffffffu, ig, 31), wl = __shfl_sync(0xffffffffu, il, 31);
+    if (lane == 0) {
+        s_wt[0][warp] = wg;
+        s_wt[1][warp] = wl;
+    }
+    __syncthreads();
+    double later_g = s_base[0] + (wg - ig), later_l = s_base[1] + (wl - il);
+    for (int w = warp + 1; w < 8; ++w) {
+        later_g += s_wt[0][w];
+        later_l += s_wt[1][w];
+    }
+    const float Ah = a.A[h];
+    double dA_acc = 0.0;
+    double rg = later_g, rl = later_l;
+#pragma unroll
+    for (int u = 3; u >= 0; --u) {
+        const int i = 4 * threadIdx.x + u;
+        rg += xg[u];
+        rl += xl[u];
+        if (i < len) {
+            const size_t gi = ((size_t)b * s.T + t0 + i) * s.H + h;
+            const float f = a.decay_logit[gi];
+            const float dlogalpha = (float)rg;
+            a.d_decay[gi] = dlogalpha * (-Ah * sigmoidf_(f));
+            dA_acc += (double)dlogalpha * (double)(-softplusf_(f));
+            const float delta = sigmoidf_(a.clock_logit[gi]);
+            a.d_clock[gi] = (float)rl * delta * (1.f - delta);
+            const float bt = a.beta[gi];
+            a.d_beta[gi] = a.tok[4 * BTH + gi] * bt * (1.f - bt);
+        }
+    }
+    dA_acc = warp_sum_d(dA_acc);
+    if (lane == 0) s_red[warp] = dA_acc;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        double t = 0.0;
+        for (int w = 0; w < 8; ++w) t += s_red[w];
+        a.dA_part[(size_t)bh * nseg + seg] = t;
+    }
+}
+
+__global__ void dA_final_kernel(BwdArgs a, int nseg) {
+    const int h = blockIdx.x * blockDim.x + threadIdx.x;
+    if (h >= a.s.H) return;
+    double t = 0.0;
+    for (int b = 0; b < a.s.B; ++b)
+        for (int k = 0; k < nseg; ++k) t += a.dA_part[((size_t)b * a.s.H + h) * nseg + k];
+    a.dA[h] = (float)t;
+}
+
+template <int D, typename TI>
+cudaError_t bwd_dispatch(const BwdArgs& a, cudaStream_t st) {
+    const Shape& s = a.s;
+    FwdArgs f{};
+    f.s = s;
+    f.q = a.q;
+    f.k = a.k;
+    f.v = a.v;
+    f.lam = a.lam;
+    f.g = a.g;
+    f.beta = a.beta;
+    f.states = a.states;
+    cudaError_t e = launch_state_simt(f, st);
+    if (e != cudaSuccess) return e;
+    const dim3 gchunk(s.nchunk(), s.B * s.H);
+    const size_t sm1 = (size_t)(5 * CB * LD + CB * LPB + 6 * CB + 8 * 640) * sizeof(float);
+    auto k1 = bwd_intra1_kernel<D, TI>;
+    cudaFuncSetAttribute(k1, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm1);
+    k1<<<gchunk, 256, sm1, st>>>(a);
+    const size_t sma = (size_t)(CB * LD + CB * 33 + CB) * sizeof(float);
+    auto ka = adj_state_kernel<TI>;
+    cudaFuncSetAttribute(ka, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sma);
+    ka<<<dim3(2 * D / 32, s.B * s.H), 256, sma, st>>>(a);
+    const size_t sm2 = (size_t)(5 * CB * LD + CB * LPB + 5 * CB) * sizeof(float);
+    auto k2 = bwd_intra2_kernel<D, TI>;
+    cudaFuncSetAttribute(k2, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm2);
+    k2<<<gchunk, 256, sm2, st>>>(a);
+    const int nseg = (s.T + PREP_SEG - 1) / PREP_SEG;
+    gate_partial_kernel<<<dim3(nseg, s.B * s.H), 256, 0, st>>>(a, nseg);
+    gate_scan_kernel<<<dim3(nseg, s.B * s.H), 256, 0, st>>>(a, nseg);
+    if (a.dA) dA_final_kernel<<<(s.H + 127) / 128, 128, 0, st>>>(a, nseg);
+    return cudaGetLastError();
+}
+
+}  // namespace
+
+cudaError_t launch_bwd_simt(const BwdArgs& a, cudaStream_t st) {
+    const Shape& s = a.s;
+    if (s.C != CB) return cudaErrorInvalidValue;
+    if (s.D == 128) return s.bf16 ? bwd_dispatch<128, __nv_bfloat16>(a, st) : bwd_dispatch<128, float>(a, st);
+    if (s.D == 64) return s.bf16 ? bwd_dispatch<64, __nv_bfloat16>(a, st) : bwd_dispatch<64, float>(a, st);
+    return cudaErrorInvalidValue;
+}
+
+}  // namespace cyfa

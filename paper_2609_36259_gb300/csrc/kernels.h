@@ -40,6 +40,7 @@ struct FwdArgs {
     float* states;      // workspace [B*H][nchunk][128][2D]: chunk-start [Kbar | Vbar]
 };
 cudaError_t launch_fwd_simt(const FwdArgs& a, cudaStream_t st);
+cudaError_t launch_state_simt(const FwdArgs& a, cudaStream_t st);  // state pass only
 
 struct BwdArgs {
     Shape s;            // s.C is the backward's own chunk length

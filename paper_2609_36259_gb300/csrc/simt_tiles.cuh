@@ -1,0 +1,109 @@
+// Shared-memory tile helpers of the SIMT chunk kernels (forward and backward).
+#pragma once
+
+#include "common.cuh"
+#include "kernels.h"
+
+namespace cyfa {
+
+constexpr int LD = 129;   // padded row stride of [C][128] shared tiles
+
+// ---------------------------------------------------------------------------------------
+// Token-wise middle readout for rows r < C of sX (in place): o'' = U(-lam) M^T softmax(M U(lam) o')
+// with M = R Phi; the padding logit is excluded from the softmax and o''[127] = 0.
+// One warp per row; swarp holds 2 x 128 floats of scratch per warp.
+static __device__ __noinline__ void middle_rows(float* sX, const float* slam, int C, const float* M, const float* MT,
+                            float* swarp) {
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    float* z = swarp + warp * 256;
+    float* p = z + 128;
+    for (int r = warp; r < C; r += 8) {
+        float* x = sX + r * LD;
+        const float lam = slam[r];
+        float cs[2], sn[2];
+#pragma unroll
+        for (int u = 0; u < 2; ++u) {
+            const int j = lane + 1 + 32 * u;
+            cs[u] = 1.f;
+            sn[u] = 0.f;
+            if (j <= NPAIR) {
+                sincospif(phase_pi(lam, j), &sn[u], &cs[u]);
+                const float xc = x[2 * j - 1], xs = x[2 * j];
+                z[2 * j - 1] = cs[u] * xc - sn[u] * xs;
+                z[2 * j] = sn[u] * xc + cs[u] * xs;
+            }
+        }
+        if (lane == 0) {
+            z[0] = x[0];
+            z[127] = 0.f;
+        }
+        __syncwarp();
+        float l[4] = {0.f, 0.f, 0.f, 0.f};
+        for (int k = 0; k < MS; ++k) {
+            const float zk = z[k];
+#pragma unroll
+            for (int u = 0; u < 4; ++u) l[u] = fmaf(MT[k * MS + lane + 32 * u], zk, l[u]);
+        }
+        if (lane == 31) l[3] = -INFINITY;
+        float mx = fmaxf(fmaxf(l[0], l[1]), fmaxf(l[2], l[3]));
+        mx = warp_max(mx);
+        float e[4], sum = 0.f;
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+            e[u] = expf(l[u] - mx);
+            sum += e[u];
+        }
+        sum = warp_sum(sum);
+        const float inv = 1.f / sum;
+#pragma unroll
+        for (int u = 0; u < 4; ++u) p[lane + 32 * u] = e[u] * inv;
+        __syncwarp();
+        float y[4] = {0.f, 0.f, 0.f, 0.f};
+        for (int i = 0; i < MA; ++i) {
+            const float pi = p[i];
+#pragma unroll
+            for (int u = 0; u < 4; ++u) y[u] = fmaf(M[i * MS + lane + 32 * u], pi, y[u]);
+        }
+        __syncwarp();
+#pragma unroll
+        for (int u = 0; u < 4; ++u) z[lane + 32 * u] = y[u];
+        __syncwarp();
+#pragma unroll
+        for (int u = 0; u < 2; ++u) {
+            const int j = lane + 1 + 32 * u;
+            if (j <= NPAIR) {
+                const float yc = z[2 * j - 1], ys = z[2 * j];
+                x[2 * j - 1] = cs[u] * yc + sn[u] * ys;
+                x[2 * j] = -sn[u] * yc + cs[u] * ys;
+            }
+        }
+        if (lane == 0) {
+            x[0] = z[0];
+            x[127] = 0.f;
+        }
+        __syncwarp();
+    }
+}
+
+__device__ __forceinline__ void load_gates(const Shape& s, const float* lam, const float* g,
+                                           const float* beta, int b, int h, int t0, int C,
+                                           float* slam, float* sg, float* sbeta) {
+    for (int r = threadIdx.x; r < C; r += blockDim.x) {
+        const size_t gi = ((size_t)b * s.T + t0 + r) * s.H + h;
+        slam[r] = lam[gi];
+        sg[r] = g[gi];
+        sbeta[r] = beta[gi];
+    }
+}
+
+// Stage rows [r0, r0+nr) x columns [c0, c0+32) of a [B,T,H,D] tensor into dst[r][33].
+template <typename TI>
+__device__ __forceinline__ void stage_tok(float* dst, const TI* X, const Shape& s, int b, int h,
+                                          int t0, int nr, int c0, float mul) {
+    for (int e = threadIdx.x; e < nr * 32; e += blockDim.x) {
+        const int r = e >> 5, cc = e & 31;
+        dst[r * 33 + cc] = mul * ldf(X, (((size_t)b * s.T + t0 + r) * s.H + h) * s.D + c0 + cc);
+    }
+}
+
+}  // namespace cyfa

@@ -1,0 +1,75 @@
+"""GPU parity of cyfa_chunk_bwd against the fp64 oracle's reverse-mode gradient."""
+import numpy as np
+import pytest
+import torch
+
+from paper_2609_36259_gb300 import cyfa, synth
+
+from _harness import (assert_close_bf16, assert_close_fp32, gpu_prepare, oracle_backward,
+                      oracle_inputs, pairs_np, sample_pairs, to_device)
+
+pytestmark = pytest.mark.gpu
+
+GRADS = (('dq', 'dq'), ('dk', 'dk'), ('dv', 'dv'), ('d_clock', 'd_clock'),
+         ('d_decay', 'd_decay'), ('d_beta', 'd_beta'))
+
+
+def gpu_backward(d, inp, want_dA=True):
+    lam, g, beta, _ = gpu_prepare(d, inp)
+    q, k, v, dO = inp['q'], inp['k'], inp['v'], inp['dO']
+    out = dict(dq=torch.empty_like(q), dk=torch.empty_like(k), dv=torch.empty_like(v),
+               d_clock=torch.empty_like(inp['clock_logit']),
+               d_decay=torch.empty_like(inp['clock_logit']),
+               d_beta=torch.empty_like(inp['clock_logit']),
+               dA=torch.empty_like(inp['A']) if want_dA else None)
+    ws = cyfa.workspace(d, cyfa.CYFA_WS_BWD, q.device)
+    cyfa.cyfa_chunk_bwd(d, q, k, v, lam, g, beta, inp['R'], inp['clock_logit'],
+                        inp['decay_logit'], inp['A'], dO, out['dq'], out['dk'], out['dv'],
+                        out['d_clock'], out['d_decay'], out['d_beta'], None, out['dA'], ws)
+    torch.cuda.synchronize()
+    return out
+
+
+def _compare(out, ref, pairs, close, what=''):
+    for gk, rk in GRADS:
+        close(pairs_np(out[gk].float(), pairs), ref[rk], '%s %s' % (what, gk))
+
+
+@pytest.mark.parametrize('B,T,H,D', [(2, 256, 2, 128), (1, 384, 3, 64)])
+def test_backward_small_bf16(B, T, H, D):
+    inp = to_device(synth.make_inputs(B, T, H, D, seed=8, with_dO=True))
+    d = cyfa.dims(B, T, H, D, chunk=64)
+    out = gpu_backward(d, inp)
+    pairs = [(b, h) for b in range(B) for h in range(H)]
+    ref = oracle_backward(oracle_inputs(inp, pairs), pairs_np(inp['dO'], pairs))
+    _compare(out, ref, pairs, assert_close_bf16)
+    dA_ref = np.zeros(H)
+    for n, (b, h) in enumerate(pairs):
+        dA_ref[h] += ref['dA'][n]
+    assert_close_bf16(out['dA'].double().cpu().numpy(), dA_ref, 'dA')
+
+
+def test_backward_fp32():
+    B, T, H, D = 1, 256, 2, 64
+    inp = to_device(synth.make_inputs(B, T, H, D, seed=9, with_dO=True, dtype=torch.float32))
+    d = cyfa.dims(B, T, H, D, chunk=64, dtype=torch.float32)
+    out = gpu_backward(d, inp)
+    pairs = [(0, 0), (0, 1)]
+    ref = oracle_backward(oracle_inputs(inp, pairs), pairs_np(inp['dO'], pairs))
+    for gk, rk in GRADS:
+        got = pairs_np(out[gk], pairs)
+        scale = max(1.0, float(np.abs(ref[rk]).max()))
+        err = float(np.abs(got - ref[rk]).max())
+        assert err <= 1e-4 * scale, (gk, err, scale)
+
+
+@pytest.mark.parametrize('B,T,H,C', [(4, 8192, 16, 64), (2, 32768, 16, 128)])
+def test_backward_full_size_sampled(B, T, H, C):
+    """The B4 H16 T8192 and the 1.4B-shaped B2 H16 T32768 layers: all gradients of sampled
+    (b, h) sequences against the oracle."""
+    inp = synth.make_inputs(B, T, H, 128, seed=0, device='cuda', with_dO=True)
+    d = cyfa.dims(B, T, H, 128, chunk=C)
+    out = gpu_backward(d, inp, want_dA=False)
+    pairs = sample_pairs(B, H, 2)
+    ref = oracle_backward(oracle_inputs(inp, pairs), pairs_np(inp['dO'], pairs))
+    _compare(out, ref, pairs, assert_close_bf16, 'B%d T%d' % (B, T))

@@ -37,12 +37,15 @@ def test_prepare_matches_oracle(B, T, H, C):
     got_lam = pairs_np(lam, pairs)
     dist = np.abs(got_lam - np.mod(lam_ref, 127.0))
     dist = np.minimum(dist, 127.0 - dist)            # compare on the circle of period m
-    assert dist.max() < 2e-5 + 1e-9 * T, dist.max()
+    # delta = sigmoid(logit) is formed in fp32 (rounding <= 2^-25 per token, with a small mean
+    # bias) and summed in fp64, so the clock may drift by up to ~T * 2^-28 from the fp64 oracle.
+    lam_tol = 1e-6 + 4e-9 * T
+    assert dist.max() < lam_tol, dist.max()
     np.testing.assert_allclose(pairs_np(g, pairs), _chunk_local_logdecay(f, A, C), rtol=1e-5,
                                atol=2e-5)
     np.testing.assert_allclose(pairs_np(beta, pairs), OG.write_strength(bl), rtol=1e-6, atol=1e-7)
     lend_got = np.array([lend[b, h].item() for b, h in pairs])
-    np.testing.assert_allclose(lend_got, lam_ref[:, -1], rtol=0, atol=1e-6)
+    np.testing.assert_allclose(lend_got, lam_ref[:, -1], rtol=0, atol=lam_tol)
 
 
 def test_fp32_config_parity():
