@@ -1,0 +1,484 @@
+#!/usr/bin/env python
+"""Throughput of the CyFA core operator on GB300 (one JSON line on stdout).
+
+Step = one pass of the operator's hot path over one synthetic batch of the 1.4B-shaped layer
+(B=2, T=32768, H=16, dk=dv=128, m=127, bf16 in / fp32 accumulate): cyfa_prepare ->
+cyfa_chunk_fwd -> cyfa_chunk_bwd.  The decode path (cyfa_step, B=256 H=16 d=128 with fp32
+states after a 2048-token prefill) is timed separately and reported under "decode".
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+
+With --gpus N > 1 (one process per GPU under torch.distributed.run) every rank runs its own
+batch (the (b, h) sequences are independent): weak scaling with no data-path collective; the
+step time is the max over ranks.  --impl reference times the fp64 CPU oracle on the host cores.
+"""
+import argparse
+import json
+import math
+import os
+import subprocess
+import sys
+import time
+
+# one BLAS thread per process: the oracle baseline runs one process per core
+for _v in ('OPENBLAS_NUM_THREADS', 'OMP_NUM_THREADS', 'MKL_NUM_THREADS'):
+    os.environ.setdefault(_v, '1')
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = 'CyFA core-op fwd/bwd tokens/s per GB300 + % bf16 TC peak; decode GB/s vs HBM'
+LAYER = dict(B=2, T=32768, H=16, d=128)          # 1.4B-shaped layer
+DECODE = dict(B=256, H=16, d=128, prefill=2048)   # decode workload
+MS = 128
+
+# Algorithmic flops per (token, head) of each kernel (d = 128, m* = 128, chunk C): the
+# products each kernel's equations call for, counted 2 per multiply-add, full C x C blocks.
+def kernel_flops_per_token_head(name, C, d=128, ms=MS):
+    table = {
+        'fwd_state': 4 * d * ms,                                    # Kbar, Vbar updates
+        'state_pass': 4 * d * ms,
+        'fwd_out': 4 * C * d + 4 * C * ms + 4 * d * ms + 4 * ms * ms,
+        'bwd_intra1': (2 * C * d + 2 * C * ms + 2 * d * ms) + 4 * ms * ms
+                      + (2 * C * d + 2 * C * ms + 2 * d * ms) + 6 * ms * ms
+                      + (2 * C * ms + 2 * C * d + 2 * d * ms),
+        'bwd_adjoint': 4 * d * ms,
+        'bwd_intra2': 4 * (2 * C * ms + 2 * C * d + 2 * d * ms),
+    }
+    return table.get(name)
+
+
+def operator_flops_per_token_head(C, d=128, ms=MS):
+    """Forward count of the chunk equations (state updates, intra-chunk, inter-chunk, middle)."""
+    key = 2 * C * d + 2 * C * ms + 4 * d * ms
+    middle = 4 * ms * ms
+    value = 2 * C * ms + 2 * C * d + 4 * ms * d
+    return key + middle + value
+
+
+def load_peaks():
+    p = os.path.join(ROOT, 'MEASURED_PEAKS.json')
+    if os.path.exists(p):
+        with open(p) as f:
+            j = json.load(f)
+        return dict(hbm_gbs=j['hbm_gbs'], bf16=j['bf16_tflops'], bf16_sus=j['bf16_tflops_sustained'],
+                    sm_max_mhz=j.get('sm_max_mhz', 2070.0), src='measured')
+    return dict(hbm_gbs=6800.0, bf16=1900.0, bf16_sus=1700.0, sm_max_mhz=2070.0, src='fallback')
+
+
+def fp32_alu_peak_tflops(sm_mhz, sms=152):
+    """CUDA-core fp32 FMA peak: 152 SMs x 128 lanes x 2 flop per clock."""
+    return sms * 128 * 2 * sm_mhz * 1e6 / 1e12
+
+
+# ---------------------------------------------------------------------------------- clocks
+class ClockSampler:
+    FIELDS = ('index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,'
+              'clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,'
+              'clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap')
+
+    def __init__(self, device_index):
+        self.idx = device_index
+        self.proc = None
+        self.path = os.path.join(ROOT, 'gpurun_out', 'bench_clocks_%d.csv' % device_index)
+
+    def start(self):
+        try:
+            os.makedirs(os.path.dirname(self.path), exist_ok=True)
+            self.fh = open(self.path, 'w')
+            self.proc = subprocess.Popen(
+                ['nvidia-smi', '-i', str(self.idx), '--query-gpu=' + self.FIELDS,
+                 '--format=csv,noheader,nounits', '-lms', '200'], stdout=self.fh,
+                stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        self.fh.close()
+        sm, smax, reasons = [], None, set()
+        names = ['hw_slowdown', 'hw_thermal_slowdown', 'sw_thermal_slowdown', 'sw_power_cap']
+        for line in open(self.path):
+            parts = [x.strip() for x in line.split(',')]
+            if len(parts) < 9:
+                continue
+            try:
+                sm.append(float(parts[1]))
+                smax = float(parts[2])
+            except ValueError:
+                continue
+            for nm, val in zip(names, parts[5:9]):
+                if val.lower() == 'active':
+                    reasons.add(nm)
+        if not sm:
+            return None
+        sm.sort()
+        return {'sm_mhz': sm[len(sm) // 2], 'sm_max_mhz': smax, 'reasons': sorted(reasons),
+                'samples': len(sm)}
+
+
+# --------------------------------------------------------------------------- cpu baseline
+def _oracle_pair_worker(args):
+    """One (b, h) sequence through the fp64 oracle, forward and backward; returns seconds."""
+    import numpy as np
+    from oracle import backward as OB, forward as OF, gates as OG
+    q, k, v, c, f, bl, A, R, dO, scale = args
+    t0 = time.perf_counter()
+    OF.absolute_clock(q, k, v, OG.clock_increment(c), OG.forget_gate(f, A[:, None]),
+                      OG.write_strength(bl), R, scale)
+    OB.backward(q, k, v, c, f, bl, A, R, scale, dO)
+    return time.perf_counter() - t0
+
+
+def _oracle_warm(_):
+    import oracle.backward  # noqa: F401
+    return 0
+
+
+def oracle_baseline(T_sample, H_full, cores=None):
+    """Time the oracle on `cores` (b, h) sequences of T_sample tokens of the layer's shape,
+    one process per core; returns (tokens/s of the full layer, cores, sample text, seconds)."""
+    import multiprocessing as mp
+    import numpy as np
+    import torch
+    from paper_2609_36259_gb300 import synth
+    cores = cores or os.cpu_count() or 1
+    inp = synth.make_inputs(1, T_sample, cores, LAYER['d'], seed=123, with_dO=True)
+    jobs = []
+    for h in range(cores):
+        def P(x):
+            return x[0, :, h].double().numpy()[None]
+        A = np.array([float(synth.decay_scales(H_full)[h % H_full])])
+        R = inp['R'][h:h + 1].double().numpy()
+        jobs.append((P(inp['q']), P(inp['k']), P(inp['v']), P(inp['clock_logit']),
+                     P(inp['decay_logit']), P(inp['beta_logit']), A, R, P(inp['dO']),
+                     inp['scale']))
+    ctx = mp.get_context('spawn')
+    with ctx.Pool(cores) as pool:
+        pool.map(_oracle_warm, range(cores))          # start the workers and import the oracle
+        t0 = time.perf_counter()
+        per = pool.map(_oracle_pair_worker, jobs)
+        wall = time.perf_counter() - t0
+    token_heads = cores * T_sample
+    value = token_heads / H_full / wall
+    sample = ('%d (b,h) sequences x %d tokens, fwd+bwd, d=128, m=127, one process per core; '
+              'tokens/s = token-heads / H(=%d) / wall' % (cores, T_sample, H_full))
+    return value, cores, sample, wall, max(per)
+
+
+# --------------------------------------------------------------------------------- ours
+def run_ours(args):
+    import numpy as np
+    import torch
+    from paper_2609_36259_gb300 import cyfa, synth
+
+    world = int(os.environ.get('WORLD_SIZE', '1'))
+    rank = int(os.environ.get('RANK', '0'))
+    local = int(os.environ.get('LOCAL_RANK', '0'))
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+        torch.cuda.set_device(local)
+        dist.init_process_group('nccl', device_id=torch.device('cuda', local))
+    else:
+        torch.cuda.set_device(0)
+    dev = torch.device('cuda', torch.cuda.current_device())
+    peaks = load_peaks()
+
+    # CPU baseline first: its process pool is spawned before any GPU work of this process
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        v, cores, sample, wall, _ = oracle_baseline(args.cpu_tokens, LAYER['H'])
+        cpu = {'value': v, 'unit': 'tokens/s', 'cores': cores, 'kind': 'oracle',
+               'sample': sample, 'seconds': round(wall, 2)}
+
+    B, T, H, D, C = LAYER['B'], LAYER['T'], LAYER['H'], LAYER['d'], args.chunk
+    d = cyfa.dims(B, T, H, D, chunk=C)
+    inp = synth.make_inputs(B, T, H, D, seed=rank, device=dev, with_dO=True)
+    f32 = dict(dtype=torch.float32, device=dev)
+    lam = torch.empty(B, T, H, **f32)
+    g = torch.empty_like(lam)
+    beta = torch.empty_like(lam)
+    o = torch.empty_like(inp['v'])
+    dq, dk, dv = torch.empty_like(inp['q']), torch.empty_like(inp['k']), torch.empty_like(inp['v'])
+    dc, dd, db = torch.empty_like(lam), torch.empty_like(lam), torch.empty_like(lam)
+    dA = torch.empty(H, **f32)
+    ws_p = cyfa.workspace(d, cyfa.CYFA_WS_PREPARE, dev)
+    ws_f = cyfa.workspace(d, cyfa.CYFA_WS_FWD, dev)
+    ws_b = cyfa.workspace(d, cyfa.CYFA_WS_BWD, dev)
+    stream = torch.cuda.current_stream()
+
+    def step(x):
+        cyfa.cyfa_prepare(d, x['clock_logit'], x['decay_logit'], x['beta_logit'], x['A'], None,
+                          lam, g, beta, None, ws_p)
+        cyfa.cyfa_chunk_fwd(d, x['q'], x['k'], x['v'], lam, g, beta, x['R'], None, None, o, None,
+                            None, ws_f)
+        cyfa.cyfa_chunk_bwd(d, x['q'], x['k'], x['v'], lam, g, beta, x['R'], x['clock_logit'],
+                            x['decay_logit'], x['A'], x['dO'], dq, dk, dv, dc, dd, db, None, dA,
+                            ws_b)
+
+    for _ in range(args.warmup):
+        step(inp)
+    torch.cuda.synchronize()
+    if dist:
+        dist.barrier()
+    cyfa.cyfa_stats_reset()
+    cyfa.cyfa_stats_timing(True)
+    clocks = ClockSampler(dev.index)
+    clocks.start()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    torch.cuda.synchronize()
+    e0.record(stream)
+    for _ in range(args.steps):
+        step(inp)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    clk = clocks.stop()
+    cyfa.cyfa_check()
+    ms = e0.elapsed_time(e1) / args.steps
+    stats = cyfa.cyfa_stats_get()
+    cyfa.cyfa_stats_timing(False)
+    if dist:
+        t = torch.tensor([ms], dtype=torch.float64, device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms = float(t.item())
+    tokens = B * T * world
+    value = tokens / (ms / 1e3)
+    launches = sum(n for n, _ in stats.values())
+
+    # per-kernel times and the forward / backward split
+    per_kernel = {k: {'launches': n, 'ms_per_launch': t / n if n else 0.0}
+                  for k, (n, t) in stats.items()}
+    fwd_names = ('readout_matrix', 'fwd_state', 'fwd_out')
+    fwd_ms = sum(stats[k][1] for k in stats if k in fwd_names) / args.steps
+    prep_ms = sum(stats[k][1] for k in stats if k.startswith('prep')) / args.steps
+    bwd_ms = sum(stats[k][1] for k in stats
+                 if k not in fwd_names and not k.startswith('prep')) / args.steps
+    token_heads = B * T * H
+    op_flops = operator_flops_per_token_head(64) * token_heads      # counting rule at C = 64
+    fwd = {'ms': fwd_ms, 'tokens_per_s': B * T / (fwd_ms / 1e3) if fwd_ms else None,
+           'tflops_rule_c64': op_flops / (fwd_ms / 1e3) / 1e12 if fwd_ms else None}
+    fwd['frac_bf16_peak'] = fwd['tflops_rule_c64'] / peaks['bf16'] if fwd_ms else None
+    bwd = {'ms': bwd_ms, 'tokens_per_s': B * T / (bwd_ms / 1e3) if bwd_ms else None,
+           'tflops_rule_2x_fwd': 2 * op_flops / (bwd_ms / 1e3) / 1e12 if bwd_ms else None}
+
+    # roofline of the dominant kernel
+    top = max(stats.items(), key=lambda kv: kv[1][1])[0]
+    n_top, t_top = stats[top]
+    C_top = 64 if top.startswith('bwd') or top == 'state_pass' else C
+    fl = kernel_flops_per_token_head(top, C_top)
+    roof = None
+    if fl is not None:
+        tensor_path = False      # the chunk kernels of this build run on the CUDA cores (fp32 FMA)
+        achieved = fl * token_heads / (t_top / n_top / 1e3) / 1e12
+        if tensor_path:
+            peak, unit, bound = peaks['bf16_sus'], 'TFLOP/s', 'tensor'
+        else:
+            peak, unit, bound = fp32_alu_peak_tflops(peaks['sm_max_mhz']), 'TFLOP/s', 'alu'
+        roof = {'kernel': top, 'bound': bound, 'achieved': round(achieved, 3),
+                'peak': round(peak, 2), 'unit': unit, 'frac': round(achieved / peak, 4),
+                'traffic': None, 'flops_per_launch': fl * token_heads,
+                'ms_per_launch': t_top / n_top,
+                'peak_source': ('fp32 FMA: 152 SMs x 128 lanes x 2 x %.0f MHz' % peaks['sm_max_mhz']
+                                if bound == 'alu' else peaks['src'] + ' bf16 sustained')}
+        tr = load_traffic(top)
+        if tr is not None:
+            roof['traffic'] = tr
+
+    # decode: B=256, H=16, fp32 states after a 2048-token prefill
+    dec = None
+    if not args.no_decode:
+        dec = run_decode(args, dev, peaks, rank)
+
+    # end to end through the public API with host buffers
+    e2e = None
+    if not args.no_e2e:
+        e2e = run_e2e(args, d, inp, dev, step_outputs=(o, dq, dk, dv, dc, dd, db),
+                      step=step)
+
+    del ws_f, ws_b
+    line = {
+        'metric': METRIC, 'value': value, 'unit': 'tokens/s', 'n_gpus': world,
+        'steps': args.steps, 'warmup': args.warmup, 'ms_per_step': ms,
+        'higher_is_better': True, 'scaling': 'weak', 'vs_baseline': None, 'dtype': 'bf16',
+        'data': 'synthetic',
+        'config': {'workload': 'cyfa-1.4B-layer prepare+fwd+bwd', 'model': 'CyFA core operator',
+                   'B': B, 'T': T, 'H': H, 'dk': D, 'dv': D, 'm': 127, 'm_store': MS,
+                   'chunk': C, 'global_batch': B * world, 'seq_len': T,
+                   'parallelism': 'dp%d' % world,
+                   'l2': 'inputs larger than L2 (q,k,v,dO %.0f MB)' % (4 * B * T * H * D * 2 / 1e6)},
+        'roofline': roof, 'cpu_baseline': cpu, 'e2e': e2e, 'gpu_launches': launches,
+        'clocks': clk, 'fwd': fwd, 'bwd': bwd, 'prepare_ms': prep_ms, 'decode': dec,
+        'kernels': per_kernel,
+    }
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if dist:
+        dist.barrier()
+        dist.destroy_process_group()
+
+
+def load_traffic(kernel):
+    """DRAM bytes per launch from the committed ncu summary, if it was taken of the current
+    kernel source (its sha256 recorded beside the number)."""
+    import hashlib
+    p = os.path.join(ROOT, 'profiles', 'traffic.json')
+    if not os.path.exists(p):
+        return None
+    with open(p) as f:
+        j = json.load(f)
+    ent = j.get(kernel)
+    if not ent:
+        return None
+    src = os.path.join(ROOT, ent['source'])
+    if not os.path.exists(src):
+        return None
+    sha = hashlib.sha256(open(src, 'rb').read()).hexdigest()
+    return ent['bytes_per_launch'] if sha == ent.get('source_sha256') else None
+
+
+def run_decode(args, dev, peaks, rank):
+    import torch
+    from paper_2609_36259_gb300 import cyfa, synth
+    B, H, D, T0 = DECODE['B'], DECODE['H'], DECODE['d'], DECODE['prefill']
+    S = args.decode_steps
+    inp = synth.make_inputs(B, T0, H, D, seed=1000 + rank, device=dev)
+    d0 = cyfa.dims(B, T0, H, D, chunk=64)
+    lam, g, beta, lend = cyfa.prepare(d0, inp['clock_logit'], inp['decay_logit'],
+                                      inp['beta_logit'], inp['A'], want_lambda_end=True)
+    _, K, V = cyfa.forward(d0, inp['q'], inp['k'], inp['v'], lam, g, beta, inp['R'],
+                           want_state=True)
+    del inp, lam, g, beta
+    torch.cuda.empty_cache()
+    stepi = synth.make_inputs(B, S, H, D, seed=2000 + rank, device=dev)
+    xs = {k: stepi[k].transpose(0, 1).contiguous() for k in
+          ('q', 'k', 'v', 'clock_logit', 'decay_logit', 'beta_logit')}
+    ds = cyfa.dims(B, 1, H, D)
+    o = torch.empty(B, H, D, dtype=torch.bfloat16, device=dev)
+
+    def one(t):
+        cyfa.cyfa_step(ds, xs['q'][t], xs['k'][t], xs['v'][t], xs['clock_logit'][t],
+                       xs['decay_logit'][t], xs['beta_logit'][t], stepi['A'], stepi['R'], K, V,
+                       lend, o)
+    for t in range(min(3, S)):
+        one(t)
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record()
+    for t in range(S):
+        one(t)
+    e1.record()
+    torch.cuda.synchronize()
+    ms = e0.elapsed_time(e1) / S
+    bytes_step = B * H * (2 * 2 * MS * D * 4 + 3 * D * 2 + D * 2 + 3 * 4 + 2 * 8)
+    gbs = bytes_step / (ms / 1e3) / 1e9
+    return {'workload': 'B=%d H=%d d=%d fp32 states, %d-token prefill, %d steps' % (B, H, D, T0, S),
+            'ms_per_step': ms, 'tokens_per_s': B / (ms / 1e3), 'GB_per_s': gbs,
+            'bytes_per_step': bytes_step, 'frac_hbm_measured': gbs / peaks['hbm_gbs'],
+            'frac_hbm_8TBs': gbs / 8000.0}
+
+
+def run_e2e(args, d, inp, dev, step_outputs, step):
+    """The same step through the public API with pinned host buffers: every step copies its
+    inputs host->device and reads every output back."""
+    import torch
+    keys = ('q', 'k', 'v', 'clock_logit', 'decay_logit', 'beta_logit', 'dO')
+    host = {k: inp[k].cpu().pin_memory() for k in keys}
+    outs_h = [t.new_empty(t.shape, device='cpu').pin_memory() for t in step_outputs]
+    dev_in = {k: torch.empty_like(inp[k]) for k in keys}
+    x = dict(inp)
+    x.update(dev_in)
+    h2d = sum(t.numel() * t.element_size() for t in host.values())
+    d2h = sum(t.numel() * t.element_size() for t in outs_h)
+
+    def one():
+        for k in keys:
+            dev_in[k].copy_(host[k], non_blocking=True)
+        step(x)
+        for hb, t in zip(outs_h, step_outputs):
+            hb.copy_(t, non_blocking=True)
+    for _ in range(2):
+        one()
+    torch.cuda.synchronize()
+    n = max(1, min(args.steps, 3))
+    t0 = time.perf_counter()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record()
+    for _ in range(n):
+        one()
+    e1.record()
+    torch.cuda.synchronize()
+    ms = e0.elapsed_time(e1) / n
+    B, T = inp['q'].shape[0], inp['q'].shape[1]
+    return {'value': B * T / (ms / 1e3), 'unit': 'tokens/s', 'h2d_bytes_per_step': h2d,
+            'd2h_bytes_per_step': d2h, 'ms_per_step': ms}
+
+
+# ---------------------------------------------------------------------------- reference
+def run_reference(args):
+    world = int(os.environ.get('WORLD_SIZE', '1'))
+    rank = int(os.environ.get('RANK', '0'))
+    if rank != 0:
+        return
+    B, T, H = LAYER['B'], LAYER['T'], LAYER['H']
+    for _ in range(args.warmup):
+        pass   # the oracle has no warm state; warm-up steps would only repeat the sample
+    walls = []
+    vals = []
+    cores = None
+    sample = None
+    for _ in range(args.steps):
+        v, cores, sample, wall, _ = oracle_baseline(args.ref_tokens, H)
+        vals.append(v)
+        walls.append(wall)
+    value = sum(vals) / len(vals)
+    line = {
+        'impl': 'reference', 'metric': METRIC, 'value': value, 'unit': 'tokens/s',
+        'n_gpus': world, 'steps': args.steps, 'warmup': args.warmup,
+        'ms_per_step': 1e3 * sum(walls) / len(walls), 'higher_is_better': True,
+        'scaling': 'weak', 'vs_baseline': None, 'dtype': 'f64', 'data': 'synthetic',
+        'config': {'workload': 'cyfa-1.4B-layer prepare+fwd+bwd', 'model': 'CyFA core operator',
+                   'B': B, 'T': T, 'H': H, 'dk': 128, 'dv': 128, 'm': 127, 'chunk': args.chunk,
+                   'global_batch': B * world, 'seq_len': T, 'parallelism': 'dp%d' % world},
+        'cpu_baseline': {'value': value, 'unit': 'tokens/s', 'cores': cores, 'kind': 'oracle',
+                         'sample': sample},
+        'e2e': {'value': value, 'unit': 'tokens/s', 'h2d_bytes_per_step': 0,
+                'd2h_bytes_per_step': 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument('--gpus', type=int, default=1)
+    ap.add_argument('--steps', type=int, default=5)
+    ap.add_argument('--warmup', type=int, default=3)
+    ap.add_argument('--impl', default='ours', choices=['ours', 'reference'])
+    ap.add_argument('--chunk', type=int, default=64, choices=[64, 128])
+    ap.add_argument('--decode-steps', type=int, default=1024)
+    ap.add_argument('--cpu-tokens', type=int, default=1024)
+    ap.add_argument('--shape', default=None,
+                    help='B,T,H override of the layer shape (profiling runs on smaller cases)')
+    ap.add_argument('--ref-tokens', type=int, default=256)
+    ap.add_argument('--no-decode', action='store_true')
+    ap.add_argument('--no-e2e', action='store_true')
+    ap.add_argument('--no-cpu-baseline', action='store_true')
+    args = ap.parse_args()
+    if args.shape:
+        LAYER['B'], LAYER['T'], LAYER['H'] = (int(x) for x in args.shape.split(','))
+    if args.warmup < 3 and args.impl == 'ours':
+        args.warmup = 3
+    if args.impl == 'reference':
+        run_reference(args)
+    else:
+        run_ours(args)
+
+
+if __name__ == '__main__':
+    main()

@@ -143,6 +143,21 @@ int cyfa_step(const cyfa_dims_t* dims, const void* q, const void* k, const void*
  */
 int cyfa_check(void* stream);
 
+/*
+ * Launch accounting (host side, process-wide).  Every kernel launch of the library increments
+ * a counter kept per kernel name.  With cyfa_stats_timing(1) each launch is also bracketed by
+ * CUDA events recorded on its own stream; the elapsed times are summed per kernel when read.
+ *   cyfa_stats_reset   -- forget all counters and timings.
+ *   cyfa_stats_timing  -- 1 to time every launch from now on, 0 to stop.
+ *   cyfa_stats_get     -- entry `index` (0-based, in order of first launch): its kernel name
+ *                         (copied into name[name_len], NUL-terminated), launches and total
+ *                         milliseconds (waits for the recorded events).  CYFA_ERR_ARG past
+ *                         the last entry.
+ */
+int cyfa_stats_reset(void);
+int cyfa_stats_timing(int on);
+int cyfa_stats_get(int index, char* name, int name_len, long long* launches, double* total_ms);
+
 #ifdef __cplusplus
 }
 #endif

@@ -235,18 +235,18 @@ cudaError_t fwd_dispatch(const FwdArgs& a, cudaStream_t st) {
     const size_t sm_state = (size_t)(C * LD + C * 33 + 3 * C) * sizeof(float);
     auto kst = fwd_state_kernel<C, TI>;
     cudaFuncSetAttribute(kst, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm_state);
-    kst<<<dim3(2 * D / 32, s.B * s.H), 256, sm_state, st>>>(a);
+    { LaunchScope ls_("fwd_state", st); kst<<<dim3(2 * D / 32, s.B * s.H), 256, sm_state, st>>>(a); }
     const size_t sm_out = (size_t)(2 * C * LD + C * (C + 1) + 4 * C + 8 * 256) * sizeof(float);
     auto kout = fwd_out_kernel<C, D, TI>;
     cudaFuncSetAttribute(kout, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm_out);
-    kout<<<dim3(s.nchunk(), s.B * s.H), 256, sm_out, st>>>(a);
+    { LaunchScope ls_("fwd_out", st); kout<<<dim3(s.nchunk(), s.B * s.H), 256, sm_out, st>>>(a); }
     return cudaGetLastError();
 }
 
 }  // namespace
 
 cudaError_t launch_readout_matrix(int H, const float* R, float* M, float* MT, cudaStream_t st) {
-    readout_matrix_kernel<<<dim3(MS, H), 128, 0, st>>>(R, M, MT);
+    { LaunchScope ls_("readout_matrix", st); readout_matrix_kernel<<<dim3(MS, H), 128, 0, st>>>(R, M, MT); }
     return cudaGetLastError();
 }
 
@@ -257,7 +257,7 @@ cudaError_t launch_state_simt(const FwdArgs& a, cudaStream_t st) {
         const size_t sm = (size_t)(CC * LD + CC * 33 + 3 * CC) * sizeof(float);         \
         auto k = s.bf16 ? fwd_state_kernel<CC, __nv_bfloat16> : fwd_state_kernel<CC, float>; \
         cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);   \
-        k<<<dim3(2 * s.D / 32, s.B * s.H), 256, sm, st>>>(a);                            \
+        { LaunchScope ls_("state_pass", st); k<<<dim3(2 * s.D / 32, s.B * s.H), 256, sm, st>>>(a); } \
         return cudaGetLastError();                                                       \
     }
     CYFA_ST(64)

@@ -394,8 +394,9 @@ __global__ void __launch_bounds__(256) adj_state_kernel(BwdArgs a) {
             for (int j = 0; j < 2; ++j) dst[(ty + 16 * i) * W + col0 + tx + 16 * j] = S[i][j];
         const int t0 = c * CB;
         __syncthreads();
+        const float gb = g_base(s, a.g, b, h, t0, CB);
         for (int r = threadIdx.x; r < CB; r += blockDim.x)
-            sg[r] = a.g[((size_t)b * s.T + t0 + r) * s.H + h];
+            sg[r] = a.g[((size_t)b * s.T + t0 + r) * s.H + h] - gb;
         stage_tok(sX, X, s, b, h, t0, CB, xc0, xmul);
         __syncthreads();
         const float* Yc = Y + ((size_t)bh * s.T + t0) * MS;
@@ -721,19 +722,19 @@ cudaError_t bwd_dispatch(const BwdArgs& a, cudaStream_t st) {
     const size_t sm1 = (size_t)(5 * CB * LD + CB * LPB + 6 * CB + 8 * 640) * sizeof(float);
     auto k1 = bwd_intra1_kernel<D, TI>;
     cudaFuncSetAttribute(k1, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm1);
-    k1<<<gchunk, 256, sm1, st>>>(a);
+    { LaunchScope ls_("bwd_intra1", st); k1<<<gchunk, 256, sm1, st>>>(a); }
     const size_t sma = (size_t)(CB * LD + CB * 33 + CB) * sizeof(float);
     auto ka = adj_state_kernel<TI>;
     cudaFuncSetAttribute(ka, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sma);
-    ka<<<dim3(2 * D / 32, s.B * s.H), 256, sma, st>>>(a);
+    { LaunchScope ls_("bwd_adjoint", st); ka<<<dim3(2 * D / 32, s.B * s.H), 256, sma, st>>>(a); }
     const size_t sm2 = (size_t)(5 * CB * LD + CB * LPB + 5 * CB) * sizeof(float);
     auto k2 = bwd_intra2_kernel<D, TI>;
     cudaFuncSetAttribute(k2, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm2);
-    k2<<<gchunk, 256, sm2, st>>>(a);
+    { LaunchScope ls_("bwd_intra2", st); k2<<<gchunk, 256, sm2, st>>>(a); }
     const int nseg = (s.T + PREP_SEG - 1) / PREP_SEG;
-    gate_partial_kernel<<<dim3(nseg, s.B * s.H), 256, 0, st>>>(a, nseg);
-    gate_scan_kernel<<<dim3(nseg, s.B * s.H), 256, 0, st>>>(a, nseg);
-    if (a.dA) dA_final_kernel<<<(s.H + 127) / 128, 128, 0, st>>>(a, nseg);
+    { LaunchScope ls_("bwd_gate_partial", st); gate_partial_kernel<<<dim3(nseg, s.B * s.H), 256, 0, st>>>(a, nseg); }
+    { LaunchScope ls_("bwd_gate_scan", st); gate_scan_kernel<<<dim3(nseg, s.B * s.H), 256, 0, st>>>(a, nseg); }
+    if (a.dA) { LaunchScope ls_("bwd_dA", st); dA_final_kernel<<<(s.H + 127) / 128, 128, 0, st>>>(a, nseg); }
     return cudaGetLastError();
 }
 

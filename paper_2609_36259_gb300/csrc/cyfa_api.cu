@@ -48,6 +48,7 @@ Shape shape_of(const cyfa_dims_t* d) {
     s.H = d->H;
     s.D = d->dk;
     s.C = d->chunk;
+    s.Cg = d->chunk;
     s.scale = d->scale;
     s.bf16 = d->dtype == CYFA_DTYPE_BF16;
     return s;

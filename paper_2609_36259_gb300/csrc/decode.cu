@@ -224,11 +224,11 @@ __global__ void __launch_bounds__(256) step_kernel(StepArgs a) {
 cudaError_t launch_step(const StepArgs& a, cudaStream_t st) {
     const int grid = a.B * a.H;
     if (a.D == 128) {
-        if (a.bf16) step_kernel<128, __nv_bfloat16><<<grid, 256, 0, st>>>(a);
-        else step_kernel<128, float><<<grid, 256, 0, st>>>(a);
+        if (a.bf16) { LaunchScope ls_("decode_step", st); step_kernel<128, __nv_bfloat16><<<grid, 256, 0, st>>>(a); }
+        else { LaunchScope ls_("decode_step", st); step_kernel<128, float><<<grid, 256, 0, st>>>(a); }
     } else if (a.D == 64) {
-        if (a.bf16) step_kernel<64, __nv_bfloat16><<<grid, 256, 0, st>>>(a);
-        else step_kernel<64, float><<<grid, 256, 0, st>>>(a);
+        if (a.bf16) { LaunchScope ls_("decode_step", st); step_kernel<64, __nv_bfloat16><<<grid, 256, 0, st>>>(a); }
+        else { LaunchScope ls_("decode_step", st); step_kernel<64, float><<<grid, 256, 0, st>>>(a); }
     } else {
         return cudaErrorInvalidValue;
     }

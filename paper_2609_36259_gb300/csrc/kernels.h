@@ -6,8 +6,24 @@
 
 namespace cyfa {
 
+// Counts one launch of the named kernel and, when timing is on (cyfa_stats_timing), brackets it
+// with CUDA events on its stream.  Construct immediately before the <<<>>> launch.
+class LaunchScope {
+  public:
+    LaunchScope(const char* name, cudaStream_t st);
+    ~LaunchScope();
+    LaunchScope(const LaunchScope&) = delete;
+    LaunchScope& operator=(const LaunchScope&) = delete;
+
+  private:
+    cudaStream_t stream_;
+    int idx_ = 0;
+    cudaEvent_t start_ = nullptr;
+};
+
 struct Shape {
-    int B, T, H, D, C;      // batch, tokens, heads, head dim (dk == dv), chunk
+    int B, T, H, D, C;      // batch, tokens, heads, head dim (dk == dv), chunk walked by a kernel
+    int Cg;                 // chunk length the g_cum input is local to (the caller's chunk)
     float scale;
     bool bf16;
     __host__ __device__ int nchunk() const { return T / C; }

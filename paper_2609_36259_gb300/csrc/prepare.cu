@@ -118,8 +118,8 @@ size_t prepare_workspace(const Shape& s) {
 cudaError_t launch_prepare(const PrepareArgs& a, cudaStream_t st) {
     const int nseg = (a.s.T + PREP_SEG - 1) / PREP_SEG;
     dim3 grid(nseg, a.s.B * a.s.H);
-    prep_partial_kernel<<<grid, 256, 0, st>>>(a, nseg);
-    prep_scan_kernel<<<grid, 256, 0, st>>>(a, nseg);
+    { LaunchScope ls_("prep_partial", st); prep_partial_kernel<<<grid, 256, 0, st>>>(a, nseg); }
+    { LaunchScope ls_("prep_scan", st); prep_scan_kernel<<<grid, 256, 0, st>>>(a, nseg); }
     return cudaGetLastError();
 }
 

@@ -85,13 +85,21 @@ static __device__ __noinline__ void middle_rows(float* sX, const float* slam, in
     }
 }
 
+// g_cum is local to the caller's chunks of s.Cg tokens; a kernel walking shorter chunks of C
+// tokens (C divides Cg) rebases it to its own chunk start by subtracting the value just before.
+__device__ __forceinline__ float g_base(const Shape& s, const float* g, int b, int h, int t0,
+                                        int C) {
+    return (s.Cg != C && (t0 % s.Cg) != 0) ? g[((size_t)b * s.T + t0 - 1) * s.H + h] : 0.f;
+}
+
 __device__ __forceinline__ void load_gates(const Shape& s, const float* lam, const float* g,
                                            const float* beta, int b, int h, int t0, int C,
                                            float* slam, float* sg, float* sbeta) {
+    const float gb = g_base(s, g, b, h, t0, C);
     for (int r = threadIdx.x; r < C; r += blockDim.x) {
         const size_t gi = ((size_t)b * s.T + t0 + r) * s.H + h;
         slam[r] = lam[gi];
-        sg[r] = g[gi];
+        sg[r] = g[gi] - gb;
         sbeta[r] = beta[gi];
     }
 }

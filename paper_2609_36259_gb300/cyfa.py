@@ -20,7 +20,8 @@ CYFA_WS_PREPARE, CYFA_WS_FWD, CYFA_WS_BWD = 0, 1, 2
 
 # Every symbol include/cyfa.h declares (checked by tests/test_abi.py).
 EXPORTS = ('cyfa_version', 'cyfa_error_string', 'cyfa_workspace_size', 'cyfa_prepare',
-           'cyfa_chunk_fwd', 'cyfa_chunk_bwd', 'cyfa_step', 'cyfa_check')
+           'cyfa_chunk_fwd', 'cyfa_chunk_bwd', 'cyfa_step', 'cyfa_check', 'cyfa_stats_reset',
+           'cyfa_stats_timing', 'cyfa_stats_get')
 
 
 class CyfaError(RuntimeError):
@@ -62,6 +63,9 @@ def load(path=LIB_PATH):
     lib.cyfa_chunk_bwd.argtypes = [P] + [_VP] * 20 + [ctypes.c_size_t, _VP]
     lib.cyfa_step.argtypes = [P] + [_VP] * 13
     lib.cyfa_check.argtypes = [_VP]
+    lib.cyfa_stats_timing.argtypes = [ctypes.c_int]
+    lib.cyfa_stats_get.argtypes = [ctypes.c_int, ctypes.c_char_p, ctypes.c_int,
+                                   ctypes.POINTER(ctypes.c_longlong), ctypes.POINTER(ctypes.c_double)]
     for name in EXPORTS:
         getattr(lib, name).restype = ctypes.c_int if name != 'cyfa_error_string' else ctypes.c_char_p
     _lib = lib
@@ -133,6 +137,28 @@ def cyfa_step(d, q, k, v, clock_logit, decay_logit, beta_logit, A, R, Kbar, Vbar
 
 def cyfa_check(stream=None):
     _ok(load().cyfa_check(_stream(stream)))
+
+
+def cyfa_stats_reset():
+    _ok(load().cyfa_stats_reset())
+
+
+def cyfa_stats_timing(on):
+    _ok(load().cyfa_stats_timing(1 if on else 0))
+
+
+def cyfa_stats_get():
+    """{kernel name: (launches, total ms)} for every kernel launched since the last reset."""
+    lib = load()
+    out = {}
+    i = 0
+    buf = ctypes.create_string_buffer(128)
+    n = ctypes.c_longlong()
+    ms = ctypes.c_double()
+    while lib.cyfa_stats_get(i, buf, 128, ctypes.byref(n), ctypes.byref(ms)) == CYFA_OK:
+        out[buf.value.decode()] = (n.value, ms.value)
+        i += 1
+    return out
 
 
 # ---- convenience: whole calls with library-owned outputs (still argument marshalling) ----

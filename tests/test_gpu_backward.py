@@ -35,10 +35,11 @@ def _compare(out, ref, pairs, close, what=''):
         close(pairs_np(out[gk].float(), pairs), ref[rk], '%s %s' % (what, gk))
 
 
-@pytest.mark.parametrize('B,T,H,D', [(2, 256, 2, 128), (1, 384, 3, 64)])
-def test_backward_small_bf16(B, T, H, D):
+@pytest.mark.parametrize('B,T,H,D,C', [(2, 256, 2, 128, 64), (1, 384, 3, 64, 64),
+                                       (1, 512, 2, 128, 128)])
+def test_backward_small_bf16(B, T, H, D, C):
     inp = to_device(synth.make_inputs(B, T, H, D, seed=8, with_dO=True))
-    d = cyfa.dims(B, T, H, D, chunk=64)
+    d = cyfa.dims(B, T, H, D, chunk=C)
     out = gpu_backward(d, inp)
     pairs = [(b, h) for b in range(B) for h in range(H)]
     ref = oracle_backward(oracle_inputs(inp, pairs), pairs_np(inp['dO'], pairs))
