@@ -97,6 +97,26 @@ int cyfa_prepare(const cyfa_dims_t* dims, const float* clock_logit, const float*
                  void* workspace, size_t workspace_bytes, void* stream);
 
 /*
+ * cyfa_prepare_noalloc -- cyfa_prepare for callers that cannot provide any device memory of
+ * their own beyond the tensors (the paper has no counterpart: this is a deployment variant).
+ * Typical such callers are a serving process or plugin host that reserves all device memory
+ * up front through its own allocator and forbids later cudaMalloc calls, or a latency-critical
+ * loop that must not allocate.  Arguments and results are those of cyfa_prepare, without the
+ * workspace.  It calls no allocator: the per-segment partial sums live in one fixed array
+ * compiled into the library (256 KiB of fp64, held on every GPU that loads the library until
+ * the process exits), which limits B * H * ceil(T / 1024) to 32768; larger shapes return
+ * CYFA_ERR_WORKSPACE before anything is launched.  The first call made on a device looks up
+ * the array's device address (cudaGetSymbolAddress) with that device current; make that first
+ * call before any stream capture.  All calls share the array and each call overwrites it
+ * entirely before reading it, so nothing needs clearing, but calls that may run concurrently
+ * on the GPU (on different streams, or different host threads) race on it and must not overlap.
+ */
+int cyfa_prepare_noalloc(const cyfa_dims_t* dims, const float* clock_logit,
+                         const float* decay_logit, const float* beta_logit, const float* A,
+                         const double* lambda0, float* lam_mod, float* g_cum, float* beta,
+                         double* lambda_end, void* stream);
+
+/*
  * cyfa_chunk_fwd -- forward of the operator, chunk-wise two-pass form (Sec. 3.3 Eq.
  * cyfa-two-pass; App. B Eqs. app-cyfa-key-chunk, app-cyfa-value-chunk).
  * Inputs are the outputs of cyfa_prepare plus q, k, v and R.  Kbar0 / Vbar0 (nullable,

@@ -4,6 +4,9 @@
 //
 // Layout: gates are [B, T, H] fp32.  Two launches: per (b, h, 1024-token segment) fp64 sums of
 // delta, then a block scan per segment that adds the sums of the segments before it.
+#include <mutex>
+
+#include "../../include/cyfa.h"
 #include "common.cuh"
 #include "kernels.h"
 
@@ -124,3 +127,84 @@ cudaError_t launch_prepare(const PrepareArgs& a, cudaStream_t st) {
 }
 
 }  // namespace cyfa
+
+// ---------------------------------------------------------------------------------------
+// cyfa_prepare_noalloc: cyfa_prepare without a caller workspace.
+//
+// Some callers cannot give the library any device memory beyond the tensors themselves: an
+// inference server or plugin host that reserves all device memory up front through its own
+// allocator and forbids later cudaMalloc calls, or a latency-critical loop that must never
+// allocate.  This entry point runs the same two prepare kernels, but the per-segment partial
+// sums live in a fixed array compiled into the library instead of a workspace.
+//
+// The array is a file-scope __device__ variable: every GPU that loads the library holds it
+// (256 KiB) until the process exits.  Its host-side name is only a stand-in, never a device
+// address, so the address is looked up with cudaGetSymbolAddress once per device, with that
+// device current, on the first call made on the device.
+namespace cyfa {
+namespace {
+
+constexpr int kNoAllocMaxSegSums = 32768;   // B * H * ceil(T / 1024) fp64 partial sums
+static __device__ __align__(256) double g_noalloc_seg_sum[kNoAllocMaxSegSums];
+
+constexpr int kMaxDevices = 64;
+std::mutex g_noalloc_mu;
+double* g_noalloc_ptr[kMaxDevices] = {};
+
+// Device address of g_noalloc_seg_sum on the current device (looked up once per device).
+cudaError_t noalloc_scratch(double** out) {
+    int dev = -1;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    if (dev < 0 || dev >= kMaxDevices) return cudaErrorInvalidDevice;
+    std::lock_guard<std::mutex> lk(g_noalloc_mu);
+    if (!g_noalloc_ptr[dev]) {
+        void* p = nullptr;
+        e = cudaGetSymbolAddress(&p, g_noalloc_seg_sum);
+        if (e != cudaSuccess) return e;
+        g_noalloc_ptr[dev] = static_cast<double*>(p);
+    }
+    *out = g_noalloc_ptr[dev];
+    return cudaSuccess;
+}
+
+}  // namespace
+}  // namespace cyfa
+
+extern "C" int cyfa_prepare_noalloc(const cyfa_dims_t* dims, const float* clock_logit,
+                                    const float* decay_logit, const float* beta_logit,
+                                    const float* A, const double* lambda0, float* lam_mod,
+                                    float* g_cum, float* beta, double* lambda_end, void* stream) {
+    using namespace cyfa;
+    if (!dims || dims->B <= 0 || dims->T <= 0 || dims->H <= 0) return CYFA_ERR_ARG;
+    if (dims->m != 127 || dims->dk != dims->dv || (dims->dk != 64 && dims->dk != 128) ||
+        (dims->chunk != 64 && dims->chunk != 128) || dims->T % dims->chunk != 0)
+        return CYFA_ERR_SHAPE;
+    if (!clock_logit || !decay_logit || !beta_logit || !A || !lam_mod || !g_cum || !beta)
+        return CYFA_ERR_ARG;
+    const long long nseg = (dims->T + PREP_SEG - 1) / PREP_SEG;
+    if ((long long)dims->B * dims->H * nseg > kNoAllocMaxSegSums) return CYFA_ERR_WORKSPACE;
+    double* scratch = nullptr;
+    if (noalloc_scratch(&scratch) != cudaSuccess) return CYFA_ERR_CUDA;
+    PrepareArgs a;
+    a.s.B = dims->B;
+    a.s.T = dims->T;
+    a.s.H = dims->H;
+    a.s.D = dims->dk;
+    a.s.C = dims->chunk;
+    a.s.Cg = dims->chunk;
+    a.s.scale = dims->scale;
+    a.s.bf16 = dims->dtype == CYFA_DTYPE_BF16;
+    a.clock_logit = clock_logit;
+    a.decay_logit = decay_logit;
+    a.beta_logit = beta_logit;
+    a.A = A;
+    a.lambda0 = lambda0;
+    a.lam_mod = lam_mod;
+    a.g_cum = g_cum;
+    a.beta = beta;
+    a.lambda_end = lambda_end;
+    a.seg_sum = scratch;   // every entry is written by the first kernel before the second reads it
+    return launch_prepare(a, static_cast<cudaStream_t>(stream)) == cudaSuccess ? CYFA_OK
+                                                                                 : CYFA_ERR_CUDA;
+}

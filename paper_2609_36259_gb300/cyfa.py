@@ -21,7 +21,7 @@ CYFA_WS_PREPARE, CYFA_WS_FWD, CYFA_WS_BWD = 0, 1, 2
 # Every symbol include/cyfa.h declares (checked by tests/test_abi.py).
 EXPORTS = ('cyfa_version', 'cyfa_error_string', 'cyfa_workspace_size', 'cyfa_prepare',
            'cyfa_chunk_fwd', 'cyfa_chunk_bwd', 'cyfa_step', 'cyfa_check', 'cyfa_stats_reset',
-           'cyfa_stats_timing', 'cyfa_stats_get')
+           'cyfa_stats_timing', 'cyfa_stats_get', 'cyfa_prepare_noalloc')
 
 
 class CyfaError(RuntimeError):
@@ -63,6 +63,7 @@ def load(path=LIB_PATH):
     lib.cyfa_chunk_bwd.argtypes = [P] + [_VP] * 20 + [ctypes.c_size_t, _VP]
     lib.cyfa_step.argtypes = [P] + [_VP] * 13
     lib.cyfa_check.argtypes = [_VP]
+    lib.cyfa_prepare_noalloc.argtypes = [P] + [_VP] * 9 + [_VP]
     lib.cyfa_stats_timing.argtypes = [ctypes.c_int]
     lib.cyfa_stats_get.argtypes = [ctypes.c_int, ctypes.c_char_p, ctypes.c_int,
                                    ctypes.POINTER(ctypes.c_longlong), ctypes.POINTER(ctypes.c_double)]
@@ -109,6 +110,15 @@ def cyfa_prepare(d, clock_logit, decay_logit, beta_logit, A, lambda0, lam_mod, g
     _ok(load().cyfa_prepare(ctypes.byref(d), _ptr(clock_logit), _ptr(decay_logit),
                             _ptr(beta_logit), _ptr(A), _ptr(lambda0), _ptr(lam_mod), _ptr(g_cum),
                             _ptr(beta), _ptr(lambda_end), _ptr(ws), ws.numel(), _stream(stream)))
+
+
+def cyfa_prepare_noalloc(d, clock_logit, decay_logit, beta_logit, A, lambda0, lam_mod, g_cum,
+                         beta, lambda_end, stream=None):
+    """cyfa_prepare without a workspace, for callers that must not allocate device memory
+    (its partial sums use a fixed array inside the library; see include/cyfa.h)."""
+    _ok(load().cyfa_prepare_noalloc(ctypes.byref(d), _ptr(clock_logit), _ptr(decay_logit),
+                                    _ptr(beta_logit), _ptr(A), _ptr(lambda0), _ptr(lam_mod),
+                                    _ptr(g_cum), _ptr(beta), _ptr(lambda_end), _stream(stream)))
 
 
 def cyfa_chunk_fwd(d, q, k, v, lam_mod, g_cum, beta, R, Kbar0, Vbar0, o, Kbar_out, Vbar_out, ws,
