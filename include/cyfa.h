@@ -164,6 +164,16 @@ int cyfa_step(const cyfa_dims_t* dims, const void* q, const void* k, const void*
 int cyfa_check(void* stream);
 
 /*
+ * cyfa_selftest_mma -- self-check of the tensor-core (tcgen05 / TMEM / TMA) operand layouts the
+ * chunk kernels rely on; the paper has no counterpart.  Computes D = op(X) op(Y) for row-major
+ * bf16 X, Y [128 x 128] (device pointers, 16-byte aligned) into fp32 D [128 x 128]:
+ * variant bit 0 selects op(X) = X^T (A operand MN-major) instead of X (K-major); bit 1 selects
+ * op(Y) = Y (B operand MN-major) instead of Y^T (K-major); bit 2 writes the operand tiles with
+ * threads instead of TMA.  Synchronises `stream`; CYFA_ERR_TIMEOUT if a bounded wait expired.
+ */
+int cyfa_selftest_mma(int variant, const void* X, const void* Y, float* D, void* stream);
+
+/*
  * Launch accounting (host side, process-wide).  Every kernel launch of the library increments
  * a counter kept per kernel name.  With cyfa_stats_timing(1) each launch is also bracketed by
  * CUDA events recorded on its own stream; the elapsed times are summed per kernel when read.

@@ -1,6 +1,7 @@
 // Launch interface between the C ABI (cyfa_api.cu) and the kernel translation units.
 #pragma once
 
+#include <cuda.h>
 #include <cuda_runtime.h>
 #include <stddef.h>
 
@@ -75,6 +76,14 @@ struct BwdArgs {
 };
 constexpr int BWD_C = 64;       // chunk length used by the SIMT backward
 cudaError_t launch_bwd_simt(const BwdArgs& a, cudaStream_t st);
+
+// ---- tensor-core path (tc_*.cu) ----
+// Encode a bf16 TMA tensor map with 128-byte swizzle (dims / strides innermost first; strides
+// in bytes for dims 1..rank-1).  False if the driver entry point is missing or encoding fails.
+bool make_tmap_bf16(CUtensorMap* map, const void* base, int rank, const unsigned long long* dims,
+                    const unsigned long long* strides_bytes, const unsigned* box);
+cudaError_t launch_selftest_mma(int variant, const void* X, const void* Y, float* D,
+                                cudaStream_t st, int* host_err);
 
 // ---- decode (decode.cu) ----
 struct StepArgs {

@@ -21,7 +21,8 @@ CYFA_WS_PREPARE, CYFA_WS_FWD, CYFA_WS_BWD = 0, 1, 2
 # Every symbol include/cyfa.h declares (checked by tests/test_abi.py).
 EXPORTS = ('cyfa_version', 'cyfa_error_string', 'cyfa_workspace_size', 'cyfa_prepare',
            'cyfa_chunk_fwd', 'cyfa_chunk_bwd', 'cyfa_step', 'cyfa_check', 'cyfa_stats_reset',
-           'cyfa_stats_timing', 'cyfa_stats_get', 'cyfa_prepare_noalloc')
+           'cyfa_stats_timing', 'cyfa_stats_get', 'cyfa_prepare_noalloc',
+           'cyfa_selftest_mma')
 
 
 class CyfaError(RuntimeError):
@@ -63,6 +64,7 @@ def load(path=LIB_PATH):
     lib.cyfa_chunk_bwd.argtypes = [P] + [_VP] * 20 + [ctypes.c_size_t, _VP]
     lib.cyfa_step.argtypes = [P] + [_VP] * 13
     lib.cyfa_check.argtypes = [_VP]
+    lib.cyfa_selftest_mma.argtypes = [ctypes.c_int, _VP, _VP, _VP, _VP]
     lib.cyfa_prepare_noalloc.argtypes = [P] + [_VP] * 9 + [_VP]
     lib.cyfa_stats_timing.argtypes = [ctypes.c_int]
     lib.cyfa_stats_get.argtypes = [ctypes.c_int, ctypes.c_char_p, ctypes.c_int,
@@ -147,6 +149,10 @@ def cyfa_step(d, q, k, v, clock_logit, decay_logit, beta_logit, A, R, Kbar, Vbar
 
 def cyfa_check(stream=None):
     _ok(load().cyfa_check(_stream(stream)))
+
+
+def cyfa_selftest_mma(variant, X, Y, D, stream=None):
+    _ok(load().cyfa_selftest_mma(variant, _ptr(X), _ptr(Y), _ptr(D), _stream(stream)))
 
 
 def cyfa_stats_reset():
