@@ -68,7 +68,12 @@ typedef struct cyfa_dims {
     int chunk;     /* tokens per chunk: 64 or 128 */
     float scale;   /* dot-product scale s; the query enters the key pass as s*q */
     int dtype;     /* CYFA_DTYPE_BF16 or CYFA_DTYPE_FP32 for q, k, v, o, dO, dq, dk, dv */
+    int flags;     /* CYFA_FLAG_* bits; 0 for the default kernels */
 } cyfa_dims_t;
+
+/* dims.flags: run the chunk calls on the fp32 CUDA-core kernels even where the tensor-core
+ * kernels apply (bf16, d = 128, T a multiple of 128).  Slower; exact fp32 intermediates. */
+enum { CYFA_FLAG_CUDA_CORES = 1 };
 
 /* Library version as 10000*major + 100*minor + patch. */
 int cyfa_version(void);

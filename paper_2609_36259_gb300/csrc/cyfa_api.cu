@@ -54,16 +54,30 @@ Shape shape_of(const cyfa_dims_t* d) {
     return s;
 }
 
+bool use_tc(const cyfa_dims_t* d, const Shape& s) {
+    return !(d->flags & CYFA_FLAG_CUDA_CORES) && tc_fwd_supported(s);
+}
+
 struct FwdLayout {
-    float *M, *MT, *states;
+    float *M, *MT, *states;          // CUDA-core path
+    float *segS, *segG;              // tensor-core path
+    __nv_bfloat16* Mb;
+    int nseg;
     size_t bytes;
 };
-FwdLayout fwd_layout(const Shape& s, void* ws) {
+FwdLayout fwd_layout(const Shape& s, bool tc_path, void* ws) {
     Carver c{static_cast<char*>(ws)};
-    FwdLayout L;
+    FwdLayout L{};
     L.M = c.take<float>((size_t)s.H * MS * MS);
     L.MT = c.take<float>((size_t)s.H * MS * MS);
-    L.states = c.take<float>((size_t)s.B * s.H * s.nchunk() * MS * 2 * s.D);
+    if (tc_path) {
+        L.nseg = tc_fwd_segments(s);
+        L.Mb = c.take<__nv_bfloat16>((size_t)s.H * MS * MS);
+        L.segS = c.take<float>((size_t)s.B * s.H * L.nseg * MS * 256);
+        L.segG = c.take<float>((size_t)s.B * s.H * L.nseg);
+    } else {
+        L.states = c.take<float>((size_t)s.B * s.H * s.nchunk() * MS * 2 * s.D);
+    }
     L.bytes = c.off;
     return L;
 }
@@ -122,7 +136,7 @@ int cyfa_workspace_size(const cyfa_dims_t* dims, int which, size_t* bytes) {
     const Shape s = shape_of(dims);
     switch (which) {
         case CYFA_WS_PREPARE: *bytes = up(prepare_workspace(s)); return CYFA_OK;
-        case CYFA_WS_FWD: *bytes = fwd_layout(s, nullptr).bytes; return CYFA_OK;
+        case CYFA_WS_FWD: *bytes = fwd_layout(s, use_tc(dims, s), nullptr).bytes; return CYFA_OK;
         case CYFA_WS_BWD: *bytes = bwd_layout(s, nullptr).bytes; return CYFA_OK;
         default: return CYFA_ERR_ARG;
     }
@@ -167,13 +181,31 @@ int cyfa_chunk_fwd(const cyfa_dims_t* dims, const void* q, const void* k, const 
         (Kbar_out && (!aligned16(Kbar_out) || !aligned16(Vbar_out))))
         return CYFA_ERR_ALIGN;
     const Shape s = shape_of(dims);
-    const FwdLayout need = fwd_layout(s, nullptr);
+    const bool tc_path = use_tc(dims, s);
+    const FwdLayout need = fwd_layout(s, tc_path, nullptr);
     if (!workspace || workspace_bytes < need.bytes) return CYFA_ERR_WORKSPACE;
     if (!aligned16(workspace)) return CYFA_ERR_ALIGN;
-    const FwdLayout L = fwd_layout(s, workspace);
+    const FwdLayout L = fwd_layout(s, tc_path, workspace);
     cudaStream_t st = static_cast<cudaStream_t>(stream);
     rc = cuda_status(launch_readout_matrix(s.H, R, L.M, L.MT, st));
     if (rc) return rc;
+    if (tc_path) {
+        TcFwdArgs t;
+        t.s = s;
+        t.lam = lam_mod;
+        t.g = g_cum;
+        t.beta = beta;
+        t.Kbar0 = Kbar0;
+        t.Vbar0 = Vbar0;
+        t.Kout = Kbar_out;
+        t.Vout = Vbar_out;
+        t.o = o;
+        t.segS = L.segS;
+        t.segG = L.segG;
+        t.Mb = L.Mb;
+        t.nseg = L.nseg;
+        return cuda_status(launch_fwd_tc(t, q, k, v, L.M, st));
+    }
     FwdArgs a;
     a.s = s;
     a.q = q;
@@ -282,9 +314,11 @@ int cyfa_step(const cyfa_dims_t* dims, const void* q, const void* k, const void*
 }
 
 int cyfa_check(void* stream) {
-    if (cudaStreamSynchronize(static_cast<cudaStream_t>(stream)) != cudaSuccess)
-        return CYFA_ERR_CUDA;
-    return CYFA_OK;
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    if (cudaStreamSynchronize(st) != cudaSuccess) return CYFA_ERR_CUDA;
+    int err = 0;
+    if (tc_read_error(st, &err) != cudaSuccess) return CYFA_ERR_CUDA;
+    return err ? CYFA_ERR_TIMEOUT : CYFA_OK;
 }
 
 }  // extern "C"

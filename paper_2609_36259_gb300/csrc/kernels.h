@@ -2,6 +2,7 @@
 #pragma once
 
 #include <cuda.h>
+#include <cuda_bf16.h>
 #include <cuda_runtime.h>
 #include <stddef.h>
 
@@ -84,6 +85,24 @@ bool make_tmap_bf16(CUtensorMap* map, const void* base, int rank, const unsigned
                     const unsigned long long* strides_bytes, const unsigned* box);
 cudaError_t launch_selftest_mma(int variant, const void* X, const void* Y, float* D,
                                 cudaStream_t st, int* host_err);
+
+struct TcFwdArgs {
+    Shape s;
+    const float *lam, *g, *beta;
+    const float *Kbar0, *Vbar0;   // nullable initial states [B,H,128,128]
+    float *Kout, *Vout;           // nullable final states
+    void* o;                      // bf16 [B,T,H,128]
+    float* segS;                  // [B*H][nseg][128][256]: segment deltas, then segment-start states
+    float* segG;                  // [B*H][nseg] total log-decay of each segment
+    const __nv_bfloat16* Mb;      // [H][128][128] bf16 M = R Phi
+    int nseg;
+};
+bool tc_fwd_supported(const Shape& s);
+int tc_fwd_segments(const Shape& s);
+cudaError_t launch_fwd_tc(const TcFwdArgs& a, const void* q, const void* k, const void* v,
+                          const float* Mf, cudaStream_t st);
+// Reads (and clears) the error word of the tensor-core kernels; synchronises the stream.
+cudaError_t tc_read_error(cudaStream_t st, int* err);
 
 // ---- decode (decode.cu) ----
 struct StepArgs {

@@ -34,12 +34,17 @@ class CyfaError(RuntimeError):
 class Dims(ctypes.Structure):
     _fields_ = [('B', ctypes.c_int), ('T', ctypes.c_int), ('H', ctypes.c_int),
                 ('dk', ctypes.c_int), ('dv', ctypes.c_int), ('m', ctypes.c_int),
-                ('chunk', ctypes.c_int), ('scale', ctypes.c_float), ('dtype', ctypes.c_int)]
+                ('chunk', ctypes.c_int), ('scale', ctypes.c_float), ('dtype', ctypes.c_int),
+                ('flags', ctypes.c_int)]
 
 
-def dims(B, T, H, d, *, chunk=64, scale=None, dtype=torch.bfloat16, m=127):
+CYFA_FLAG_CUDA_CORES = 1
+
+
+def dims(B, T, H, d, *, chunk=64, scale=None, dtype=torch.bfloat16, m=127, cuda_cores=False):
     return Dims(B, T, H, d, d, m, chunk, float(d ** -0.5 if scale is None else scale),
-                CYFA_DTYPE_BF16 if dtype == torch.bfloat16 else CYFA_DTYPE_FP32)
+                CYFA_DTYPE_BF16 if dtype == torch.bfloat16 else CYFA_DTYPE_FP32,
+                CYFA_FLAG_CUDA_CORES if cuda_cores else 0)
 
 
 _lib = None

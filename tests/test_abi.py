@@ -39,10 +39,15 @@ def test_version_and_errors(lib):
 
 
 def test_workspace_sizes(lib):
-    d = cyfa.dims(2, 32768, 16, 128, chunk=128)
+    d = cyfa.dims(2, 32768, 16, 128, chunk=128, cuda_cores=True)
     fwd = cyfa.cyfa_workspace_size(d, cyfa.CYFA_WS_FWD)
-    # readout matrices (2 x H x 128 x 128 fp32) plus one [128 x 2D] fp32 state per chunk
+    # CUDA-core path: readout matrices (2 x H x 128 x 128 fp32) plus one [128 x 2D] fp32 state
+    # per chunk
     assert fwd >= 2 * 16 * 128 * 128 * 4 + 2 * 16 * 256 * 128 * 256 * 4
+    # tensor-core path: one fp32 [128 x 256] state per (b, h, 1024-token segment)
+    d = cyfa.dims(2, 32768, 16, 128, chunk=128)
+    fwd_tc = cyfa.cyfa_workspace_size(d, cyfa.CYFA_WS_FWD)
+    assert 2 * 16 * 32 * 128 * 256 * 4 <= fwd_tc < fwd
     assert cyfa.cyfa_workspace_size(d, cyfa.CYFA_WS_BWD) > 0
     assert cyfa.cyfa_workspace_size(d, cyfa.CYFA_WS_PREPARE) >= 2 * 16 * 32 * 8
 

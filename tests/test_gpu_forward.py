@@ -64,11 +64,15 @@ def test_fp32_config_parity():
     assert np.all(Kg[:, 127] == 0) and np.all(Vg[:, 127] == 0)
 
 
+@pytest.mark.parametrize('cuda_cores', [False, True])
 @pytest.mark.parametrize('B,T,H,D,C', [(2, 384, 3, 128, 64), (1, 512, 2, 128, 128),
-                                       (3, 256, 1, 64, 128), (1, 64, 1, 128, 64)])
-def test_bf16_forward_small(B, T, H, D, C):
+                                       (3, 256, 1, 64, 128), (1, 64, 1, 128, 64),
+                                       (1, 2304, 2, 128, 64)])
+def test_bf16_forward_small(B, T, H, D, C, cuda_cores):
+    """Tensor-core kernels (bf16, d = 128, T a multiple of 128) and the CUDA-core kernels;
+    T = 2304 spans several 1024-token segments plus a partial one."""
     inp = to_device(synth.make_inputs(B, T, H, D, seed=2))
-    d = cyfa.dims(B, T, H, D, chunk=C)
+    d = cyfa.dims(B, T, H, D, chunk=C, cuda_cores=cuda_cores)
     o, Ko, Vo, _ = gpu_forward(d, inp, want_state=True)
     pairs = [(b, h) for b in range(B) for h in range(H)]
     oi = oracle_inputs(inp, pairs)
@@ -104,9 +108,10 @@ def test_extreme_gates():
     assert_close_bf16(pairs_np(o.float(), pairs), o_ref, 'o (saturated gates)')
 
 
-def test_state_continuation():
+@pytest.mark.parametrize('T,T1', [(512, 192), (2560, 1280)])
+def test_state_continuation(T, T1):
     """Forward over [0, T1) exporting (Kbar, Vbar, lambda), then [T1, T) from them, equals one call."""
-    B, T, H, D, T1 = 1, 512, 2, 128, 192
+    B, H, D = 1, 2, 128
     inp = to_device(synth.make_inputs(B, T, H, D, seed=5))
     d = cyfa.dims(B, T, H, D, chunk=64)
     o_full, K_full, _, _ = gpu_forward(d, inp, want_state=True)
@@ -121,12 +126,14 @@ def test_state_continuation():
     np.testing.assert_allclose(K2.cpu().numpy(), K_full.cpu().numpy(), atol=2e-3, rtol=2e-3)
 
 
-@pytest.mark.parametrize('B,T,H,C', [(8, 4096, 8, 64), (2, 32768, 16, 128)])
-def test_full_size_forward_sampled(B, T, H, C):
+@pytest.mark.parametrize('B,T,H,C,cuda_cores', [(8, 4096, 8, 64, False), (8, 4096, 8, 64, True),
+                                                 (2, 32768, 16, 64, False),
+                                                 (2, 32768, 16, 128, True)])
+def test_full_size_forward_sampled(B, T, H, C, cuda_cores):
     """The 400M-shaped (B8 H8 T4096) and 1.4B-shaped (B2 H16 T32768) layers: every output of
     sampled (b, h) sequences against the oracle."""
     inp = synth.make_inputs(B, T, H, 128, seed=0, device='cuda')
-    d = cyfa.dims(B, T, H, 128, chunk=C)
+    d = cyfa.dims(B, T, H, 128, chunk=C, cuda_cores=cuda_cores)
     o, _, _, _ = gpu_forward(d, inp)
     pairs = sample_pairs(B, H, 3)
     o_ref = oracle_forward(oracle_inputs(inp, pairs))[0]
