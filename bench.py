@@ -44,8 +44,14 @@ def kernel_flops_per_token_head(name, C, d=128, ms=MS):
                       + (2 * C * ms + 2 * C * d + 2 * d * ms),
         'bwd_adjoint': 4 * d * ms,
         'bwd_intra2': 4 * (2 * C * ms + 2 * C * d + 2 * d * ms),
+        # tensor-core kernels (128-token chunks)
+        'tc_seg_state': 4 * d * ms,
+        'tc_seg_out': 4 * 128 * d + 4 * 128 * ms + 8 * d * ms + 4 * ms * ms,
     }
     return table.get(name)
+
+
+TENSOR_KERNELS = ('tc_seg_state', 'tc_seg_out')
 
 
 def operator_flops_per_token_head(C, d=128, ms=MS):
@@ -199,7 +205,7 @@ def run_ours(args):
                'sample': sample, 'seconds': round(wall, 2)}
 
     B, T, H, D, C = LAYER['B'], LAYER['T'], LAYER['H'], LAYER['d'], args.chunk
-    d = cyfa.dims(B, T, H, D, chunk=C)
+    d = cyfa.dims(B, T, H, D, chunk=C, cuda_cores=args.cuda_cores)
     inp = synth.make_inputs(B, T, H, D, seed=rank, device=dev, with_dO=True)
     f32 = dict(dtype=torch.float32, device=dev)
     lam = torch.empty(B, T, H, **f32)
@@ -219,6 +225,8 @@ def run_ours(args):
                           lam, g, beta, None, ws_p)
         cyfa.cyfa_chunk_fwd(d, x['q'], x['k'], x['v'], lam, g, beta, x['R'], None, None, o, None,
                             None, ws_f)
+        if args.no_bwd:
+            return
         cyfa.cyfa_chunk_bwd(d, x['q'], x['k'], x['v'], lam, g, beta, x['R'], x['clock_logit'],
                             x['decay_logit'], x['A'], x['dO'], dq, dk, dv, dc, dd, db, None, dA,
                             ws_b)
@@ -255,7 +263,8 @@ def run_ours(args):
     # per-kernel times and the forward / backward split
     per_kernel = {k: {'launches': n, 'ms_per_launch': t / n if n else 0.0}
                   for k, (n, t) in stats.items()}
-    fwd_names = ('readout_matrix', 'fwd_state', 'fwd_out')
+    fwd_names = ('readout_matrix', 'fwd_state', 'fwd_out', 'm_to_bf16', 'tc_seg_state',
+                 'tc_seg_scan', 'tc_seg_out')
     fwd_ms = sum(stats[k][1] for k in stats if k in fwd_names) / args.steps
     prep_ms = sum(stats[k][1] for k in stats if k.startswith('prep')) / args.steps
     bwd_ms = sum(stats[k][1] for k in stats
@@ -268,28 +277,29 @@ def run_ours(args):
     bwd = {'ms': bwd_ms, 'tokens_per_s': B * T / (bwd_ms / 1e3) if bwd_ms else None,
            'tflops_rule_2x_fwd': 2 * op_flops / (bwd_ms / 1e3) / 1e12 if bwd_ms else None}
 
-    # roofline of the dominant kernel
-    top = max(stats.items(), key=lambda kv: kv[1][1])[0]
-    n_top, t_top = stats[top]
-    C_top = 64 if top.startswith('bwd') or top == 'state_pass' else C
-    fl = kernel_flops_per_token_head(top, C_top)
-    roof = None
-    if fl is not None:
-        tensor_path = False      # the chunk kernels of this build run on the CUDA cores (fp32 FMA)
-        achieved = fl * token_heads / (t_top / n_top / 1e3) / 1e12
-        if tensor_path:
-            peak, unit, bound = peaks['bf16_sus'], 'TFLOP/s', 'tensor'
+    # roofline of every chunk kernel, and of the dominant one
+    def roofline_of(name):
+        n_k, t_k = stats[name]
+        C_k = 64 if name.startswith('bwd') or name == 'state_pass' else C
+        fl = kernel_flops_per_token_head(name, C_k)
+        if fl is None or n_k == 0 or t_k <= 0:
+            return None
+        achieved = fl * token_heads / (t_k / n_k / 1e3) / 1e12
+        if name in TENSOR_KERNELS:
+            peak, bound = peaks['bf16_sus'], 'tensor'
+            src = '%s bf16 sustained (kernel timed inside the step)' % peaks['src']
         else:
-            peak, unit, bound = fp32_alu_peak_tflops(peaks['sm_max_mhz']), 'TFLOP/s', 'alu'
-        roof = {'kernel': top, 'bound': bound, 'achieved': round(achieved, 3),
-                'peak': round(peak, 2), 'unit': unit, 'frac': round(achieved / peak, 4),
-                'traffic': None, 'flops_per_launch': fl * token_heads,
-                'ms_per_launch': t_top / n_top,
-                'peak_source': ('fp32 FMA: 152 SMs x 128 lanes x 2 x %.0f MHz' % peaks['sm_max_mhz']
-                                if bound == 'alu' else peaks['src'] + ' bf16 sustained')}
-        tr = load_traffic(top)
-        if tr is not None:
-            roof['traffic'] = tr
+            peak, bound = fp32_alu_peak_tflops(peaks['sm_max_mhz']), 'alu'
+            src = 'fp32 FMA: 152 SMs x 128 lanes x 2 x %.0f MHz' % peaks['sm_max_mhz']
+        r = {'kernel': name, 'bound': bound, 'achieved': round(achieved, 3),
+             'peak': round(peak, 2), 'unit': 'TFLOP/s', 'frac': round(achieved / peak, 4),
+             'traffic': load_traffic(name), 'flops_per_launch': fl * token_heads,
+             'ms_per_launch': t_k / n_k, 'peak_source': src}
+        return r
+    rooflines = {k: roofline_of(k) for k in stats}
+    rooflines = {k: v for k, v in rooflines.items() if v is not None}
+    top = max(stats.items(), key=lambda kv: kv[1][1])[0]
+    roof = rooflines.get(top)
 
     # decode: B=256, H=16, fp32 states after a 2048-token prefill
     dec = None
@@ -313,7 +323,7 @@ def run_ours(args):
                    'chunk': C, 'global_batch': B * world, 'seq_len': T,
                    'parallelism': 'dp%d' % world,
                    'l2': 'inputs larger than L2 (q,k,v,dO %.0f MB)' % (4 * B * T * H * D * 2 / 1e6)},
-        'roofline': roof, 'cpu_baseline': cpu, 'e2e': e2e, 'gpu_launches': launches,
+        'roofline': roof, 'kernel_rooflines': rooflines, 'cpu_baseline': cpu, 'e2e': e2e, 'gpu_launches': launches,
         'clocks': clk, 'fwd': fwd, 'bwd': bwd, 'prepare_ms': prep_ms, 'decode': dec,
         'kernels': per_kernel,
     }
@@ -462,13 +472,17 @@ def main():
     ap.add_argument('--impl', default='ours', choices=['ours', 'reference'])
     ap.add_argument('--chunk', type=int, default=64, choices=[64, 128])
     ap.add_argument('--decode-steps', type=int, default=1024)
-    ap.add_argument('--cpu-tokens', type=int, default=1024)
+    ap.add_argument('--cpu-tokens', type=int, default=2048)
     ap.add_argument('--shape', default=None,
                     help='B,T,H override of the layer shape (profiling runs on smaller cases)')
     ap.add_argument('--ref-tokens', type=int, default=256)
     ap.add_argument('--no-decode', action='store_true')
     ap.add_argument('--no-e2e', action='store_true')
     ap.add_argument('--no-cpu-baseline', action='store_true')
+    ap.add_argument('--no-bwd', action='store_true',
+                    help='time prepare + forward only (profiling runs; not the headline step)')
+    ap.add_argument('--cuda-cores', action='store_true',
+                    help='run the chunk calls on the fp32 CUDA-core kernels')
     args = ap.parse_args()
     if args.shape:
         LAYER['B'], LAYER['T'], LAYER['H'] = (int(x) for x in args.shape.split(','))

@@ -44,21 +44,44 @@ __device__ __forceinline__ float cum128(const Shape& s, const float* g, int b, i
     return v;
 }
 
-// The 63 rotation angles theta_j = 2 pi j lam / m, produced in order by angle addition from
-// theta_1 (cos(x + y) = cos x cos y - sin x sin y, sin(x + y) = sin x cos y + cos x sin y),
-// re-seeded from sincospif every 16 steps to bound the rounding drift.
-struct Angles {
-    float c1, s1, c, s;
-    float lam;
-    __device__ __forceinline__ explicit Angles(float lam_) : lam(lam_) {
+// Order of the 128 Fourier-axis rows inside the tensor-core kernels.  Column half hf (0 or 1)
+// holds the pairs j = 32 hf + jj + 1 (jj < 32): cosine entry at 64 hf + jj, sine entry at
+// 64 hf + jj + 32, so every rotation block of U lies inside one half.  The DC entry sits at 95
+// and the padding entry at 127.  Exported / imported states use the paper's order
+// [DC, cos_1, sin_1, ..., cos_63, sin_63, pad]; these map between the two.
+__host__ __device__ __forceinline__ int tc_slot(int p) {
+    if (p == 0) return 95;
+    if (p == 127) return 127;
+    const int j = (p + 1) >> 1, hf = (j - 1) >> 5, jj = (j - 1) & 31;
+    return 64 * hf + jj + ((p & 1) ? 0 : 32);
+}
+__host__ __device__ __forceinline__ int paper_slot(int t) {
+    if (t == 95) return 0;
+    if (t == 127) return 127;
+    const int hf = t >> 6, l = t & 63, jj = l & 31;
+    const int j = 32 * hf + jj + 1;
+    return (l >= 32) ? 2 * j : 2 * j - 1;
+}
+
+// Rotation angles theta_j = 2 pi j lam / m for the 32 pairs of one column half, produced in
+// order by angle addition from theta_1 (cos(x + y) = cos x cos y - sin x sin y,
+// sin(x + y) = sin x cos y + cos x sin y), re-seeded from sincospif every 16 steps.
+struct HalfAngles {
+    float c1, s1, c, s, lam;
+    int j0;
+    __device__ __forceinline__ HalfAngles(float lam_, int hf) : lam(lam_), j0(32 * hf + 1) {
         sincospif(phase_pi(lam, 1), &s1, &c1);
-        c = c1;
-        s = s1;
+        if (j0 == 1) {
+            c = c1;
+            s = s1;
+        } else {
+            sincospif(phase_pi(lam, j0), &s, &c);
+        }
     }
-    // advance from pair j-1 to pair j (j >= 2)
-    __device__ __forceinline__ void step(int j) {
-        if (((j - 1) & 15) == 0) {
-            sincospif(phase_pi(lam, j), &s, &c);
+    // advance to local pair jj (1..31)
+    __device__ __forceinline__ void step(int jj) {
+        if (jj == 16) {
+            sincospif(phase_pi(lam, j0 + 16), &s, &c);
         } else {
             const float cn = c * c1 - s * s1;
             const float sn = s * c1 + c * s1;
@@ -68,87 +91,116 @@ struct Angles {
     }
 };
 
-// Store a 128-value fp32 row as bf16 into row r of a swizzled K-major tile.
-__device__ __forceinline__ void store_row_bf16(uint8_t* tile, int r, const float (&x)[128]) {
+// Store 64 fp32 values as bf16 into columns [64 hf, 64 hf + 64) of row r of a swizzled tile.
+__device__ __forceinline__ void store_half_bf16(uint8_t* tile, int r, int hf, const float (&x)[64]) {
 #pragma unroll
-    for (int q = 0; q < 16; ++q) {
+    for (int q = 0; q < 8; ++q) {
         uint4 u;
         u.x = pack_bf16(x[8 * q + 0], x[8 * q + 1]);
         u.y = pack_bf16(x[8 * q + 2], x[8 * q + 3]);
         u.z = pack_bf16(x[8 * q + 4], x[8 * q + 5]);
         u.w = pack_bf16(x[8 * q + 6], x[8 * q + 7]);
-        *reinterpret_cast<uint4*>(tile + swz_off(r, 8 * q, 128)) = u;
+        *reinterpret_cast<uint4*>(tile + swz_off(r, 64 * hf + 8 * q, 128)) = u;
     }
 }
 
-// Temporal write vector w * U(-lam) b of one token (Sec. 3.2; b of Eq. app-b-explicit) as row r.
-__device__ __forceinline__ void write_vector_row(uint8_t* tile, int r, float lam, float w) {
-    float x[128];
-    Angles ang(lam);
+// One column half of the temporal write vector w U(-lam) b of a token (Sec. 3.2, b of
+// Eq. app-b-explicit), in the tensor-core row order.
+__device__ __forceinline__ void write_vector_half(uint8_t* tile, int r, int hf, float lam, float w) {
+    float x[64];
+    HalfAngles ang(lam, hf);
     const float wa = w * SQRT_2_OVER_M;
-    x[0] = w * INV_SQRT_M;
 #pragma unroll
-    for (int j = 1; j <= NPAIR; ++j) {
-        if (j > 1) ang.step(j);
-        x[2 * j - 1] = wa * ang.c;
-        x[2 * j] = -wa * ang.s;
+    for (int jj = 0; jj < 32; ++jj) {
+        if (jj > 0) ang.step(jj);
+        x[jj] = wa * ang.c;
+        x[jj + 32] = -wa * ang.s;
     }
-    x[127] = 0.f;
-    store_row_bf16(tile, r, x);
+    if (hf == 1) {
+        x[31] = w * INV_SQRT_M;
+        x[63] = 0.f;
+    }
+    store_half_bf16(tile, r, hf, x);
 }
 
-// In-place x <- U(sign * lam) x on the pairs (2j-1, 2j); the DC entry is untouched and the
-// padding entry set to 0.
+// x <- U(sign lam) x on one column half (tensor-core row order); DC kept, padding zeroed.
 template <int SIGN>
-__device__ __forceinline__ void rotate_row(float (&x)[128], float lam) {
-    Angles ang(lam);
+__device__ __forceinline__ void rotate_half(float (&x)[64], int hf, float lam) {
+    HalfAngles ang(lam, hf);
+    const float dc = x[31];
 #pragma unroll
-    for (int j = 1; j <= NPAIR; ++j) {
-        if (j > 1) ang.step(j);
+    for (int jj = 0; jj < 32; ++jj) {
+        if (jj > 0) ang.step(jj);
         const float c = ang.c, s = SIGN * ang.s;
-        const float xc = x[2 * j - 1], xs = x[2 * j];
-        x[2 * j - 1] = c * xc - s * xs;
-        x[2 * j] = s * xc + c * xs;
+        const float xc = x[jj], xs = x[jj + 32];
+        x[jj] = c * xc - s * xs;
+        x[jj + 32] = s * xc + c * xs;
     }
-    x[127] = 0.f;
+    if (hf == 1) {
+        x[31] = dc;
+        x[63] = 0.f;
+    }
 }
 
-__device__ __forceinline__ void tmem_ld_row(uint32_t taddr, float (&x)[128]) {
+__device__ __forceinline__ void tmem_ld64(uint32_t taddr, float (&x)[64]) {
+    float v[32];
+    tmem_ld32(taddr, v);
+#pragma unroll
+    for (int i = 0; i < 32; ++i) x[i] = v[i];
+    tmem_ld32(taddr + 32, v);
+#pragma unroll
+    for (int i = 0; i < 32; ++i) x[32 + i] = v[i];
+}
+__device__ __forceinline__ void tmem_st64(uint32_t taddr, const float (&x)[64]) {
     float v[32];
 #pragma unroll
-    for (int q = 0; q < 4; ++q) {
-        tmem_ld32(taddr + 32 * q, v);
+    for (int i = 0; i < 32; ++i) v[i] = x[i];
+    tmem_st32(taddr, v);
 #pragma unroll
-        for (int i = 0; i < 32; ++i) x[32 * q + i] = v[i];
-    }
+    for (int i = 0; i < 32; ++i) v[i] = x[32 + i];
+    tmem_st32(taddr + 32, v);
 }
+
+// Lane quarter / column half owned by this thread in the 256-thread tensor-core kernels:
+// warps w and w + 4 share TMEM lanes 32 (w % 4) .. + 31 (one row each per thread) and split the
+// 128 columns of a tile into halves hf = w / 4.
+struct Role {
+    int warp, lane, q, hf, row;
+    __device__ __forceinline__ Role() {
+        warp = threadIdx.x >> 5;
+        lane = threadIdx.x & 31;
+        q = warp & 3;
+        hf = warp >> 2;
+        row = 32 * q + lane;
+    }
+};
 
 // ---------------------------------------------------------------------------------------
 template <int SEGC>
-__global__ void __launch_bounds__(128) seg_state_tc(const __grid_constant__ CUtensorMap tk,
-                                                     const __grid_constant__ CUtensorMap tv,
-                                                     TcFwdArgs a) {
+__global__ void __launch_bounds__(256, 1) seg_state_tc(const __grid_constant__ CUtensorMap tk,
+                                                        const __grid_constant__ CUtensorMap tv,
+                                                        TcFwdArgs a) {
     const Shape s = a.s;
     const int seg = blockIdx.x, bh = blockIdx.y, b = bh / s.H, h = bh % s.H;
     const int nct = s.T / CT;
     const int c_begin = seg * SEGC;
     const int nc = min(SEGC, nct - c_begin);
-    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const int tid = threadIdx.x;
+    const Role ro;
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                                ~uintptr_t(1023));
-    // [buf][A | K | V] tiles
-    uint8_t* tiles = smem;
-    uint64_t* bars = reinterpret_cast<uint64_t*>(smem + 6 * TILE);   // tma[2], mma[2]
-    uint32_t* s_taddr = reinterpret_cast<uint32_t*>(bars + 4);
-    float* s_tot = reinterpret_cast<float*>(s_taddr + 4);            // [SEGC]
+    uint64_t* bars = reinterpret_cast<uint64_t*>(smem);              // tma[2], mma[2]
+    uint32_t* s_taddr = reinterpret_cast<uint32_t*>(smem + 64);
+    float* s_tot = reinterpret_cast<float*>(smem + 128);             // [SEGC]
     float* s_sfx = s_tot + SEGC;                                     // [SEGC]
+    uint8_t* tiles = smem + 1024;                                    // [buf][A | K | V]
 
     if (tid == 0) {
         for (int i = 0; i < 4; ++i) mbar_init(&bars[i], 1);
         fence_mbar_init();
     }
-    if (warp == 0) tmem_alloc(s_taddr, 256);
+    if (ro.warp == 0) tmem_alloc(s_taddr, 256);
     if (tid < nc) {
         const int t0 = (c_begin + tid) * CT;
         s_tot[tid] = cum128(s, a.g, b, h, t0, t0 + CT - 1);
@@ -185,11 +237,11 @@ __global__ void __launch_bounds__(128) seg_state_tc(const __grid_constant__ CUte
         if (tid == 0 && ok && c + 1 < nc) issue_kv(c + 1, (c + 1) & 1);
         // A-> rows of this chunk, scaled by the decay from the token to the segment end
         {
-            const int t0 = (c_begin + c) * CT, t = t0 + tid;
+            const int t0 = (c_begin + c) * CT, t = t0 + ro.row;
             const size_t gi = ((size_t)b * s.T + t) * s.H + h;
             const float w = a.beta[gi] *
                             ex2((s_tot[c] - cum128(s, a.g, b, h, t0, t) + s_sfx[c]) * LOG2E);
-            write_vector_row(tiles + 3 * buf * TILE, tid, a.lam[gi], w);
+            write_vector_half(tiles + 3 * buf * TILE, ro.row, ro.hf, a.lam[gi], w);
         }
         fence_async_smem();
         ok = __syncthreads_and(ok);
@@ -215,11 +267,11 @@ __global__ void __launch_bounds__(128) seg_state_tc(const __grid_constant__ CUte
     tc_fence_after();
     ok = __syncthreads_and(ok);
     if (ok) {
-        const int row = warp * 32 + lane;
-        float* dst = a.segS + (((size_t)bh * a.nseg + seg) * 128 + row) * 256;
-        for (int c0 = 0; c0 < 256; c0 += 32) {
+        float* dst = a.segS + (((size_t)bh * a.nseg + seg) * 128 + ro.row) * 256 + 128 * ro.hf;
+        const uint32_t tl = taddr + ((uint32_t)(32 * ro.q) << 16) + 128 * ro.hf;
+        for (int c0 = 0; c0 < 128; c0 += 32) {
             float v[32];
-            tmem_ld32(taddr + ((uint32_t)(warp * 32) << 16) + c0, v);
+            tmem_ld32(tl + c0, v);
 #pragma unroll
             for (int i = 0; i < 32; i += 4)
                 *reinterpret_cast<float4*>(dst + c0 + i) = make_float4(v[i], v[i + 1], v[i + 2], v[i + 3]);
@@ -231,78 +283,97 @@ __global__ void __launch_bounds__(128) seg_state_tc(const __grid_constant__ CUte
     }
     tc_fence_before();
     __syncthreads();
-    if (warp == 0) tmem_dealloc(taddr, 256);
+    if (ro.warp == 0) tmem_dealloc(taddr, 256);
 }
 
 // Segment-start states: S_start(0) = initial state, S_start(j+1) = exp(G_j) S_start(j) + dS(j),
-// in place over the dS buffer; the final state goes to Kout / Vout (paper row order).
+// in place over the dS buffer (tensor-core row order); the final state goes to Kout / Vout in
+// the paper's row order.  Eight segments are loaded before they are folded in.
 __global__ void __launch_bounds__(256) seg_scan_kernel(TcFwdArgs a) {
     const int bh = blockIdx.y;
     const int e = blockIdx.x * 256 + threadIdx.x;   // element of the [128 x 256] state block
     const int row = e >> 8, col = e & 255;
     const bool isK = col < 128;
     const int dcol = col & 127;
+    const int prow = paper_slot(row);
     float S = 0.f;
     const float* init = isK ? a.Kbar0 : a.Vbar0;
-    if (init) S = init[((size_t)bh * 128 + row) * 128 + dcol];
-    for (int j = 0; j < a.nseg; ++j) {
-        float* p = a.segS + ((size_t)bh * a.nseg + j) * 128 * 256 + e;
-        const float dS = *p;
-        *p = S;
-        S = expf(a.segG[(size_t)bh * a.nseg + j]) * S + dS;
+    if (init) S = init[((size_t)bh * 128 + prow) * 128 + dcol];
+    float* base = a.segS + (size_t)bh * a.nseg * 128 * 256 + e;
+    const float* G = a.segG + (size_t)bh * a.nseg;
+    for (int j0 = 0; j0 < a.nseg; j0 += 8) {
+        float d[8], gj[8];
+#pragma unroll
+        for (int u = 0; u < 8; ++u) {
+            const bool in = j0 + u < a.nseg;
+            d[u] = in ? base[(size_t)(j0 + u) * 128 * 256] : 0.f;
+            gj[u] = in ? G[j0 + u] : 0.f;
+        }
+#pragma unroll
+        for (int u = 0; u < 8; ++u) {
+            if (j0 + u < a.nseg) {
+                base[(size_t)(j0 + u) * 128 * 256] = S;
+                S = expf(gj[u]) * S + d[u];
+            }
+        }
     }
     float* out = isK ? a.Kout : a.Vout;
-    if (out) out[((size_t)bh * 128 + row) * 128 + dcol] = S;
+    if (out) out[((size_t)bh * 128 + prow) * 128 + dcol] = S;
 }
 
 // ---------------------------------------------------------------------------------------
+// Chunk walk of one (b, h, segment).  256 threads: thread (row, hf) owns TMEM lane `row` and
+// columns [64 hf, 64 hf + 64) of each 128-column accumulator; thread 0 issues TMA and MMA.
 template <int SEGC>
-__global__ void __launch_bounds__(128) seg_out_tc(const __grid_constant__ CUtensorMap tq,
-                                                   const __grid_constant__ CUtensorMap tk,
-                                                   const __grid_constant__ CUtensorMap tv,
-                                                   const __grid_constant__ CUtensorMap tm,
-                                                   TcFwdArgs a) {
+__global__ void __launch_bounds__(256, 1) seg_out_tc(const __grid_constant__ CUtensorMap tq,
+                                                      const __grid_constant__ CUtensorMap tk,
+                                                      const __grid_constant__ CUtensorMap tv,
+                                                      const __grid_constant__ CUtensorMap tm,
+                                                      TcFwdArgs a) {
     const Shape s = a.s;
     const int seg = blockIdx.x, bh = blockIdx.y, b = bh / s.H, h = bh % s.H;
     const int nct = s.T / CT;
     const int c_begin = seg * SEGC;
     const int nc = min(SEGC, nct - c_begin);
-    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const int tid = threadIdx.x;
+    const Role ro;
+    const int row = ro.row, hf = ro.hf;
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                                ~uintptr_t(1023));
-    uint8_t* T_Q = smem;               // Q, later A-> (state-update operand)
-    uint8_t* T_K = smem + 1 * TILE;
-    uint8_t* T_V = smem + 2 * TILE;
-    uint8_t* T_A = smem + 3 * TILE;    // write vectors a_s (rows = tokens)
-    uint8_t* T_S = smem + 4 * TILE;    // staging: P1, z, p, O'', P2 (rows = tokens)
-    uint8_t* T_N = smem + 5 * TILE;    // state snapshot: Kbar, then Vbar (rows = slots)
-    uint8_t* T_M = smem + 6 * TILE;    // M = R Phi (rows = slots r, cols = Fourier index)
-    uint64_t* bars = reinterpret_cast<uint64_t*>(smem + 7 * TILE);   // tma, mma, m
-    uint32_t* s_taddr = reinterpret_cast<uint32_t*>(bars + 4);
-    float* s_g2 = reinterpret_cast<float*>(s_taddr + 4);             // [128] log2-domain decays
+    uint64_t* bars = reinterpret_cast<uint64_t*>(smem);          // tma, mma, m
+    uint32_t* s_taddr = reinterpret_cast<uint32_t*>(smem + 32);
+    float* s_g2 = reinterpret_cast<float*>(smem + 64);            // [128] log2-domain decays
+    float* s_red = s_g2 + 128;                                    // [2][128] row reductions
+    uint8_t* T_Q = smem + 2048;        // Q, later A-> (state-update operand)
+    uint8_t* T_K = T_Q + 1 * TILE;
+    uint8_t* T_V = T_Q + 2 * TILE;
+    uint8_t* T_A = T_Q + 3 * TILE;     // write vectors a_s (rows = tokens)
+    uint8_t* T_S = T_Q + 4 * TILE;     // staging: P1, z, p, O'', P2 (rows = tokens)
+    uint8_t* T_N = T_Q + 5 * TILE;     // state snapshot: Kbar, then Vbar (rows = slots)
+    uint8_t* T_M = T_Q + 6 * TILE;     // M = R Phi (rows = slots r, cols = Fourier index)
 
     if (tid == 0) {
         for (int i = 0; i < 3; ++i) mbar_init(&bars[i], 1);
         fence_mbar_init();
     }
-    if (warp == 0) tmem_alloc(s_taddr, 512);
+    if (ro.warp == 0) tmem_alloc(s_taddr, 512);
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
     const uint32_t taddr = *s_taddr;
-    const uint32_t tl = taddr + ((uint32_t)(warp * 32) << 16);   // this warp's lane quarter
-    const uint32_t S_COL = 0, X1 = 256, X2 = 384;
+    const uint32_t tl = taddr + ((uint32_t)(32 * ro.q) << 16);   // this thread's TMEM lane
+    const uint32_t S_COL = 0, X1 = 256 + 64 * hf, X2 = 384 + 64 * hf;
 
     auto issue_qkv = [&](int c) {
-        const int row = b * s.T + (c_begin + c) * CT;
+        const int r0 = b * s.T + (c_begin + c) * CT;
         mbar_expect_tx(&bars[0], 3 * TILE);
-        tma_load_3d(T_Q, &tq, 0, h, row, &bars[0]);
-        tma_load_3d(T_Q + TILE / 2, &tq, 64, h, row, &bars[0]);
-        tma_load_3d(T_K, &tk, 0, h, row, &bars[0]);
-        tma_load_3d(T_K + TILE / 2, &tk, 64, h, row, &bars[0]);
-        tma_load_3d(T_V, &tv, 0, h, row, &bars[0]);
-        tma_load_3d(T_V + TILE / 2, &tv, 64, h, row, &bars[0]);
+        tma_load_3d(T_Q, &tq, 0, h, r0, &bars[0]);
+        tma_load_3d(T_Q + TILE / 2, &tq, 64, h, r0, &bars[0]);
+        tma_load_3d(T_K, &tk, 0, h, r0, &bars[0]);
+        tma_load_3d(T_K + TILE / 2, &tk, 64, h, r0, &bars[0]);
+        tma_load_3d(T_V, &tv, 0, h, r0, &bars[0]);
+        tma_load_3d(T_V + TILE / 2, &tv, 64, h, r0, &bars[0]);
     };
     if (tid == 0) {
         mbar_expect_tx(&bars[2], TILE);
@@ -310,25 +381,20 @@ __global__ void __launch_bounds__(128) seg_out_tc(const __grid_constant__ CUtens
         tma_load_2d(T_M + TILE / 2, &tm, 64, h * 128, &bars[2]);
         issue_qkv(0);
     }
-    // segment-start state into TMEM, Kbar snapshot into T_N (row = slot = tid)
+    // segment-start state into TMEM; Kbar snapshot into T_N (row = slot)
     {
-        const float* src = a.segS + (((size_t)bh * a.nseg + seg) * 128 + tid) * 256;
-        float kr[128];
+        const float* src = a.segS + (((size_t)bh * a.nseg + seg) * 128 + row) * 256 + 128 * hf;
 #pragma unroll
-        for (int q = 0; q < 8; ++q) {
-            float v[32];
+        for (int q2 = 0; q2 < 2; ++q2) {
+            float x[64];
 #pragma unroll
-            for (int i = 0; i < 32; i += 4) {
-                const float4 f = *reinterpret_cast<const float4*>(src + 32 * q + i);
-                v[i] = f.x; v[i + 1] = f.y; v[i + 2] = f.z; v[i + 3] = f.w;
+            for (int i = 0; i < 64; i += 4) {
+                const float4 f = *reinterpret_cast<const float4*>(src + 64 * q2 + i);
+                x[i] = f.x; x[i + 1] = f.y; x[i + 2] = f.z; x[i + 3] = f.w;
             }
-            tmem_st32(tl + S_COL + 32 * q, v);
-            if (q < 4) {
-#pragma unroll
-                for (int i = 0; i < 32; ++i) kr[32 * q + i] = v[i];
-            }
+            tmem_st64(tl + S_COL + 128 * hf + 64 * q2, x);
+            if (hf == 0) store_half_bf16(T_N, row, q2, x);
         }
-        store_row_bf16(T_N, tid, kr);
     }
     fence_async_smem();
     tc_fence_before();
@@ -345,91 +411,113 @@ __global__ void __launch_bounds__(128) seg_out_tc(const __grid_constant__ CUtens
                    uA = smem_u32(T_A), uS = smem_u32(T_S), uN = smem_u32(T_N),
                    uM = smem_u32(T_M);
 
-    // all threads: wait for the MMAs committed so far, then order TMEM reads after them
     auto wait_mma = [&]() {
         if (ok) ok = mbar_wait(&bars[1], mma_ph);
         mma_ph ^= 1;
         tc_fence_after();
     };
-    auto mma_ok = [&]() { return tid == 0 && ok; };
-    // all threads: publish shared-memory operand writes (and TMEM stores) to the MMA thread
-    // (the block agrees on `ok`, so every later branch on it is uniform)
+    // publish shared-memory operand writes / TMEM stores to the MMA issuer; the block agrees
+    // on `ok`, so every later branch on it is uniform
     auto publish = [&]() {
         fence_async_smem();
         tc_fence_before();
         ok = __syncthreads_and(ok);
         tc_fence_after();
     };
+    auto issuer = [&]() { return tid == 0 && ok; };
+    // masked decay of the intra-chunk scores for this thread's 64 columns (t <= row only);
+    // whole 32-column groups above the diagonal of this warp's rows are skipped
+    auto mask_scores = [&](float (&x)[64], float g2, float mul) {
+#pragma unroll
+        for (int grp = 0; grp < 2; ++grp) {
+            const int sg = 2 * hf + grp;
+            if (sg > ro.q) {
+#pragma unroll
+                for (int i = 0; i < 32; ++i) x[32 * grp + i] = 0.f;
+            } else {
+#pragma unroll
+                for (int i = 0; i < 32; ++i) {
+                    const int t = 32 * sg + i;
+                    x[32 * grp + i] = (t <= row) ? mul * x[32 * grp + i] * ex2(g2 - s_g2[t]) : 0.f;
+                }
+            }
+        }
+    };
 
+    // gates of the first chunk; later chunks are prefetched one chunk ahead
+    float n_lam, n_beta, n_g;
+    {
+        const int t0 = c_begin * CT;
+        const size_t gi = ((size_t)b * s.T + t0 + row) * s.H + h;
+        n_lam = a.lam[gi];
+        n_beta = a.beta[gi];
+        n_g = cum128(s, a.g, b, h, t0, t0 + row);
+    }
     for (int c = 0; c < nc && ok; ++c) {
         const int t0 = (c_begin + c) * CT;
-        const int tok = t0 + tid;
-        const size_t gi = ((size_t)b * s.T + tok) * s.H + h;
-        const float lam = a.lam[gi];
-        const float beta = a.beta[gi];
-        const float g2 = cum128(s, a.g, b, h, t0, tok) * LOG2E;
-        s_g2[tid] = g2;
-        write_vector_row(T_A, tid, lam, beta);
+        const size_t gi = ((size_t)b * s.T + t0 + row) * s.H + h;
+        const float lam = n_lam, beta = n_beta, g2 = n_g * LOG2E;
+        if (c + 1 < nc) {
+            const int t1 = t0 + CT;
+            const size_t g1 = ((size_t)b * s.T + t1 + row) * s.H + h;
+            n_lam = a.lam[g1];
+            n_beta = a.beta[g1];
+            n_g = cum128(s, a.g, b, h, t1, t1 + row);
+        }
+        if (hf == 0) s_g2[row] = g2;
+        write_vector_half(T_A, row, hf, lam, beta);
         publish();
         if (!ok) break;
         const float g2C = s_g2[CT - 1];
         const float gam = ex2(g2);
 
         // X1 = Q K^T, X2 = Q Kbar^T
-        if (mma_ok()) {
+        if (issuer()) {
             ok = mbar_wait(&bars[0], tma_ph);
             if (ok) {
                 tc_fence_after();
 #pragma unroll
                 for (int k = 0; k < 8; ++k) {
-                    mma_bf16(taddr + X1, kmajor_desc(uQ, 128, k), kmajor_desc(uK, 128, k), id_kk, k > 0);
-                    mma_bf16(taddr + X2, kmajor_desc(uQ, 128, k), kmajor_desc(uN, 128, k), id_kk, k > 0);
+                    mma_bf16(taddr + 256, kmajor_desc(uQ, 128, k), kmajor_desc(uK, 128, k), id_kk, k > 0);
+                    mma_bf16(taddr + 384, kmajor_desc(uQ, 128, k), kmajor_desc(uN, 128, k), id_kk, k > 0);
                 }
                 mma_commit(&bars[1]);
             }
         }
         tma_ph ^= 1;
         wait_mma();
-        // P1 = s (Q K^T) o Gamma
-        {
-            float x[128];
-            tmem_ld_row(tl + X1, x);
-#pragma unroll
-            for (int j = 0; j < 128; ++j)
-                x[j] = (j <= tid) ? scale * x[j] * ex2(g2 - s_g2[j]) : 0.f;
-            store_row_bf16(T_S, tid, x);
+        {   // P1 = s (Q K^T) o Gamma
+            float x[64];
+            tmem_ld64(tl + X1, x);
+            mask_scores(x, g2, scale);
+            store_half_bf16(T_S, row, hf, x);
         }
         publish();
         if (!ok) break;
-        if (mma_ok()) {
+        if (issuer()) {
 #pragma unroll
             for (int k = 0; k < 8; ++k)
-                mma_bf16(taddr + X1, kmajor_desc(uS, 128, k), mnmajor_desc(uA, 128, k), id_kn, k > 0);
+                mma_bf16(taddr + 256, kmajor_desc(uS, 128, k), mnmajor_desc(uA, 128, k), id_kn, k > 0);
             mma_commit(&bars[1]);
         }
         // A-> rows into T_Q (Q is consumed), Vbar snapshot into T_N, state scaled by gamma^C
-        write_vector_row(T_Q, tid, lam, beta * ex2(g2C - g2));
+        write_vector_half(T_Q, row, hf, lam, beta * ex2(g2C - g2));
         {
             const float gC = ex2(g2C);
-            float vr[128];
+            float x[64];
+            tmem_ld64(tl + S_COL + 64 * hf, x);            // Kbar columns of this half
 #pragma unroll
-            for (int q = 0; q < 8; ++q) {
-                float v[32];
-                tmem_ld32(tl + S_COL + 32 * q, v);
-                if (q >= 4) {
+            for (int i = 0; i < 64; ++i) x[i] *= gC;
+            tmem_st64(tl + S_COL + 64 * hf, x);
+            tmem_ld64(tl + S_COL + 128 + 64 * hf, x);      // Vbar columns of this half
+            store_half_bf16(T_N, row, hf, x);
 #pragma unroll
-                    for (int i = 0; i < 32; ++i) vr[32 * (q - 4) + i] = v[i];
-                }
-#pragma unroll
-                for (int i = 0; i < 32; ++i) v[i] *= gC;
-                tmem_st32(tl + S_COL + 32 * q, v);
-            }
-            store_row_bf16(T_N, tid, vr);
+            for (int i = 0; i < 64; ++i) x[i] *= gC;
+            tmem_st64(tl + S_COL + 128 + 64 * hf, x);
         }
         publish();
         if (!ok) break;
-        if (mma_ok()) {
-            // state update: [Kbar | Vbar] += A->^T [K | V]
+        if (issuer()) {   // state update: [Kbar | Vbar] += A->^T [K | V]
 #pragma unroll
             for (int k = 0; k < 8; ++k) {
                 mma_bf16(taddr + S_COL, mnmajor_desc(uQ, 128, k), mnmajor_desc(uK, 128, k), id_nn, 1u);
@@ -437,135 +525,132 @@ __global__ void __launch_bounds__(128) seg_out_tc(const __grid_constant__ CUtens
             }
         }
         wait_mma();   // P1 A
-        // z = U(lam) o',  o' = s gamma_r (Q Kbar^T) + P1 A
-        {
-            float x[128], y[32];
-            tmem_ld_row(tl + X2, x);
+        {   // z = U(lam) o',  o' = s gamma_r (Q Kbar^T) + P1 A
+            float x[64], y[64];
+            tmem_ld64(tl + X2, x);
+            tmem_ld64(tl + X1, y);
             const float f = scale * gam;
 #pragma unroll
-            for (int q = 0; q < 4; ++q) {
-                tmem_ld32(tl + X1 + 32 * q, y);
-#pragma unroll
-                for (int i = 0; i < 32; ++i) x[32 * q + i] = fmaf(f, x[32 * q + i], y[i]);
-            }
-            rotate_row<1>(x, lam);
-            store_row_bf16(T_S, tid, x);
+            for (int i = 0; i < 64; ++i) x[i] = fmaf(f, x[i], y[i]);
+            rotate_half<1>(x, hf, lam);
+            store_half_bf16(T_S, row, hf, x);
         }
         publish();
         if (!ok) break;
-        if (mma_ok()) {
+        if (issuer()) {
 #pragma unroll
             for (int k = 0; k < 8; ++k)
-                mma_bf16(taddr + X1, kmajor_desc(uS, 128, k), kmajor_desc(uM, 128, k), id_kk, k > 0);
+                mma_bf16(taddr + 256, kmajor_desc(uS, 128, k), kmajor_desc(uM, 128, k), id_kk, k > 0);
             mma_commit(&bars[1]);
         }
         wait_mma();   // also covers the state update issued before this commit
-        // p = softmax over the 127 active slots of l = z M^T
-        {
-            float x[128];
-            tmem_ld_row(tl + X1, x);
+        {   // p = softmax over the 127 active slots of l = z M^T
+            float x[64];
+            tmem_ld64(tl + X1, x);
+            const int nvalid = hf ? 63 : 64;           // slot 127 is the padding row
             float mx = -INFINITY;
 #pragma unroll
-            for (int j = 0; j < MA; ++j) mx = fmaxf(mx, x[j]);
+            for (int i = 0; i < 64; ++i)
+                if (i < nvalid) mx = fmaxf(mx, x[i]);
+            s_red[128 * hf + row] = mx;
+            __syncthreads();
+            mx = fmaxf(s_red[row], s_red[128 + row]);
             float sum = 0.f;
 #pragma unroll
-            for (int j = 0; j < MA; ++j) {
-                x[j] = ex2((x[j] - mx) * LOG2E);
-                sum += x[j];
+            for (int i = 0; i < 64; ++i) {
+                x[i] = (i < nvalid) ? ex2((x[i] - mx) * LOG2E) : 0.f;
+                sum += x[i];
             }
-            const float inv = 1.f / sum;
+            __syncthreads();
+            s_red[128 * hf + row] = sum;
+            __syncthreads();
+            const float inv = 1.f / (s_red[row] + s_red[128 + row]);
 #pragma unroll
-            for (int j = 0; j < MA; ++j) x[j] *= inv;
-            x[127] = 0.f;
-            store_row_bf16(T_S, tid, x);
+            for (int i = 0; i < 64; ++i) x[i] *= inv;
+            store_half_bf16(T_S, row, hf, x);
         }
         publish();
         if (!ok) break;
-        if (mma_ok()) {
+        if (issuer()) {
 #pragma unroll
             for (int k = 0; k < 8; ++k)
-                mma_bf16(taddr + X2, kmajor_desc(uS, 128, k), mnmajor_desc(uM, 128, k), id_kn, k > 0);
+                mma_bf16(taddr + 384, kmajor_desc(uS, 128, k), mnmajor_desc(uM, 128, k), id_kn, k > 0);
             mma_commit(&bars[1]);
         }
         wait_mma();
-        // o'' = U(-lam) (p M)
-        {
-            float x[128];
-            tmem_ld_row(tl + X2, x);
-            rotate_row<-1>(x, lam);
-            store_row_bf16(T_S, tid, x);
+        {   // o'' = U(-lam) (p M)
+            float x[64];
+            tmem_ld64(tl + X2, x);
+            rotate_half<-1>(x, hf, lam);
+            store_half_bf16(T_S, row, hf, x);
         }
         publish();
         if (!ok) break;
-        if (mma_ok()) {
+        if (issuer()) {
 #pragma unroll
             for (int k = 0; k < 8; ++k) {
-                mma_bf16(taddr + X1, kmajor_desc(uS, 128, k), kmajor_desc(uA, 128, k), id_kk, k > 0);
-                mma_bf16(taddr + X2, kmajor_desc(uS, 128, k), mnmajor_desc(uN, 128, k), id_kn, k > 0);
+                mma_bf16(taddr + 256, kmajor_desc(uS, 128, k), kmajor_desc(uA, 128, k), id_kk, k > 0);
+                mma_bf16(taddr + 384, kmajor_desc(uS, 128, k), mnmajor_desc(uN, 128, k), id_kn, k > 0);
             }
             mma_commit(&bars[1]);
         }
         wait_mma();
-        // P2 = (O'' A^T) o Gamma
-        {
-            float x[128];
-            tmem_ld_row(tl + X1, x);
-#pragma unroll
-            for (int j = 0; j < 128; ++j) x[j] = (j <= tid) ? x[j] * ex2(g2 - s_g2[j]) : 0.f;
-            store_row_bf16(T_S, tid, x);
+        {   // P2 = (O'' A^T) o Gamma
+            float x[64];
+            tmem_ld64(tl + X1, x);
+            mask_scores(x, g2, 1.f);
+            store_half_bf16(T_S, row, hf, x);
         }
         publish();
         if (!ok) break;
-        if (mma_ok()) {
+        if (issuer()) {
 #pragma unroll
             for (int k = 0; k < 8; ++k)
-                mma_bf16(taddr + X1, kmajor_desc(uS, 128, k), mnmajor_desc(uV, 128, k), id_kn, k > 0);
+                mma_bf16(taddr + 256, kmajor_desc(uS, 128, k), mnmajor_desc(uV, 128, k), id_kn, k > 0);
             mma_commit(&bars[1]);
         }
         wait_mma();
         // next chunk's tiles (Q, K, V are consumed), then o = gamma_r (O'' Vbar) + P2 V
-        if (mma_ok() && c + 1 < nc) issue_qkv(c + 1);
+        if (issuer() && c + 1 < nc) issue_qkv(c + 1);
         {
-            float x[128], y[32];
-            tmem_ld_row(tl + X2, x);
+            float x[64], y[64];
+            tmem_ld64(tl + X2, x);
+            tmem_ld64(tl + X1, y);
 #pragma unroll
-            for (int q = 0; q < 4; ++q) {
-                tmem_ld32(tl + X1 + 32 * q, y);
+            for (int i = 0; i < 64; ++i) x[i] = fmaf(gam, x[i], y[i]);
+            __nv_bfloat16* O = static_cast<__nv_bfloat16*>(a.o) + gi * 128 + 64 * hf;
 #pragma unroll
-                for (int i = 0; i < 32; ++i) x[32 * q + i] = fmaf(gam, x[32 * q + i], y[i]);
-            }
-            __nv_bfloat16* O = static_cast<__nv_bfloat16*>(a.o) + gi * 128;
-#pragma unroll
-            for (int q = 0; q < 16; ++q) {
+            for (int q2 = 0; q2 < 8; ++q2) {
                 uint4 u;
-                u.x = pack_bf16(x[8 * q + 0], x[8 * q + 1]);
-                u.y = pack_bf16(x[8 * q + 2], x[8 * q + 3]);
-                u.z = pack_bf16(x[8 * q + 4], x[8 * q + 5]);
-                u.w = pack_bf16(x[8 * q + 6], x[8 * q + 7]);
-                *reinterpret_cast<uint4*>(O + 8 * q) = u;
+                u.x = pack_bf16(x[8 * q2 + 0], x[8 * q2 + 1]);
+                u.y = pack_bf16(x[8 * q2 + 2], x[8 * q2 + 3]);
+                u.z = pack_bf16(x[8 * q2 + 4], x[8 * q2 + 5]);
+                u.w = pack_bf16(x[8 * q2 + 6], x[8 * q2 + 7]);
+                *reinterpret_cast<uint4*>(O + 8 * q2) = u;
             }
         }
-        // Kbar snapshot of the next chunk's start state
-        {
-            float kr[128];
-            tmem_ld_row(tl + S_COL, kr);
-            store_row_bf16(T_N, tid, kr);
+        {   // Kbar snapshot of the next chunk's start state
+            float x[64];
+            tmem_ld64(tl + S_COL + 64 * hf, x);
+            store_half_bf16(T_N, row, hf, x);
         }
         publish();
     }
-    if (!ok && lane == 0) flag_error(CYFA_ERR_TIMEOUT);
-    // let copies still in flight land before the shared memory is released
     if (!ok && tid == 0) {
-        mbar_wait(&bars[0], tma_ph);
+        flag_error(CYFA_ERR_TIMEOUT);
+        mbar_wait(&bars[0], tma_ph);   // let copies still in flight land
     }
     tc_fence_before();
     __syncthreads();
-    if (warp == 0) tmem_dealloc(taddr, 512);
+    if (ro.warp == 0) tmem_dealloc(taddr, 512);
 }
 
-__global__ void m_to_bf16_kernel(const float* M, __nv_bfloat16* Mb, int n) {
+// M (fp32, paper order) -> bf16 with its Fourier (column) index in the tensor-core order.
+__global__ void m_to_bf16_kernel(const float* M, __nv_bfloat16* Mb, int H) {
     const int i = blockIdx.x * blockDim.x + threadIdx.x;
-    if (i < n) Mb[i] = __float2bfloat16_rn(M[i]);
+    if (i >= H * 128 * 128) return;
+    const int p = i & 127, rest = i >> 7;
+    Mb[rest * 128 + tc_slot(p)] = __float2bfloat16_rn(M[i]);
 }
 
 constexpr int SEGC_DEFAULT = 8;    // 1024-token segments
@@ -597,18 +682,18 @@ cudaError_t launch_fwd_tc(const TcFwdArgs& a, const void* q, const void* k, cons
     const int n = s.H * 128 * 128;
     {
         LaunchScope ls_("m_to_bf16", st);
-        m_to_bf16_kernel<<<(n + 255) / 256, 256, 0, st>>>(Mf, const_cast<__nv_bfloat16*>(a.Mb), n);
+        m_to_bf16_kernel<<<(n + 255) / 256, 256, 0, st>>>(Mf, const_cast<__nv_bfloat16*>(a.Mb), s.H);
     }
     const dim3 grid(a.nseg, s.B * s.H);
-    const int smA = 6 * TILE + 1024 + 256;
+    const int smA = 1024 + 6 * TILE + 1024;
     auto kA = seg_state_tc<SEGC_DEFAULT>;
     cudaFuncSetAttribute(kA, cudaFuncAttributeMaxDynamicSharedMemorySize, smA);
-    { LaunchScope ls_("tc_seg_state", st); kA<<<grid, 128, smA, st>>>(mk, mv, a); }
+    { LaunchScope ls_("tc_seg_state", st); kA<<<grid, 256, smA, st>>>(mk, mv, a); }
     { LaunchScope ls_("tc_seg_scan", st); seg_scan_kernel<<<dim3(128, s.B * s.H), 256, 0, st>>>(a); }
-    const int smC = 7 * TILE + 1024 + 1024;
+    const int smC = 2048 + 7 * TILE + 1024;
     auto kC = seg_out_tc<SEGC_DEFAULT>;
     cudaFuncSetAttribute(kC, cudaFuncAttributeMaxDynamicSharedMemorySize, smC);
-    { LaunchScope ls_("tc_seg_out", st); kC<<<grid, 128, smC, st>>>(mq, mk, mv, mm, a); }
+    { LaunchScope ls_("tc_seg_out", st); kC<<<grid, 256, smC, st>>>(mq, mk, mv, mm, a); }
     return cudaGetLastError();
 }
 

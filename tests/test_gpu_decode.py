@@ -44,7 +44,10 @@ def test_decode_small(dtype, D):
     else:
         assert_close_bf16(got, o_ref[:, T0:], 'decode o')
     Kg = np.stack([K[b, h].double().cpu().numpy() for b, h in pairs])
-    assert np.max(np.abs(Kg[:, :127] - Kb)) < 1e-4
+    if dtype == torch.float32:
+        assert np.max(np.abs(Kg[:, :127] - Kb)) < 1e-4
+    else:   # bf16 prefill: the tensor-core kernels round the write vectors to bf16
+        assert_close_bf16(Kg[:, :127], Kb, 'Kbar after decode')
     assert np.all(Kg[:, 127] == 0)
     np.testing.assert_allclose([lam[b, h].item() for b, h in pairs], lam_ref, atol=1e-6)
 
