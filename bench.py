@@ -44,14 +44,20 @@ def kernel_flops_per_token_head(name, C, d=128, ms=MS):
                       + (2 * C * ms + 2 * C * d + 2 * d * ms),
         'bwd_adjoint': 4 * d * ms,
         'bwd_intra2': 4 * (2 * C * ms + 2 * C * d + 2 * d * ms),
-        # tensor-core kernels (128-token chunks)
+        # tensor-core kernels (128-token chunks; every product a 128 x 128 x 128 tcgen05 GEMM)
         'tc_seg_state': 4 * d * ms,
         'tc_seg_out': 4 * 128 * d + 4 * 128 * ms + 8 * d * ms + 4 * ms * ms,
+        'tc_snap_fwd': 4 * d * ms,
+        'tc_bwd_chunk1': 13 * 2 * 128 * 128,
+        'tc_adj_segment': 4 * d * ms,
+        'tc_snap_adj': 4 * d * ms,
+        'tc_bwd_chunk2': 12 * 2 * 128 * 128,
     }
     return table.get(name)
 
 
-TENSOR_KERNELS = ('tc_seg_state', 'tc_seg_out')
+TENSOR_KERNELS = ('tc_seg_state', 'tc_seg_out', 'tc_snap_fwd', 'tc_bwd_chunk1', 'tc_adj_segment',
+                  'tc_snap_adj', 'tc_bwd_chunk2')
 
 
 def operator_flops_per_token_head(C, d=128, ms=MS):
@@ -263,12 +269,16 @@ def run_ours(args):
     # per-kernel times and the forward / backward split
     per_kernel = {k: {'launches': n, 'ms_per_launch': t / n if n else 0.0}
                   for k, (n, t) in stats.items()}
-    fwd_names = ('readout_matrix', 'fwd_state', 'fwd_out', 'm_to_bf16', 'tc_seg_state',
+    fwd_names = ('readout_matrix', 'fwd_state', 'fwd_out', 'm_to_k16', 'tc_seg_state',
                  'tc_seg_scan', 'tc_seg_out')
-    fwd_ms = sum(stats[k][1] for k in stats if k in fwd_names) / args.steps
+    # the forward's kernels are launched again inside the backward (recomputation): split by
+    # launch count, one forward's worth per step belongs to cyfa_chunk_fwd
+    def fwd_share(k):
+        n, t = stats[k]
+        return t * min(1.0, args.steps / n) if n else 0.0
+    fwd_ms = sum(fwd_share(k) for k in stats if k in fwd_names) / args.steps
     prep_ms = sum(stats[k][1] for k in stats if k.startswith('prep')) / args.steps
-    bwd_ms = sum(stats[k][1] for k in stats
-                 if k not in fwd_names and not k.startswith('prep')) / args.steps
+    bwd_ms = (sum(stats[k][1] for k in stats if not k.startswith('prep')) / args.steps) - fwd_ms
     token_heads = B * T * H
     op_flops = operator_flops_per_token_head(64) * token_heads      # counting rule at C = 64
     fwd = {'ms': fwd_ms, 'tokens_per_s': B * T / (fwd_ms / 1e3) if fwd_ms else None,

@@ -731,14 +731,19 @@ cudaError_t bwd_dispatch(const BwdArgs& a, cudaStream_t st) {
     auto k2 = bwd_intra2_kernel<D, TI>;
     cudaFuncSetAttribute(k2, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm2);
     { LaunchScope ls_("bwd_intra2", st); k2<<<gchunk, 256, sm2, st>>>(a); }
+    return launch_bwd_gates(a, st);
+}
+
+}  // namespace
+
+cudaError_t launch_bwd_gates(const BwdArgs& a, cudaStream_t st) {
+    const Shape& s = a.s;
     const int nseg = (s.T + PREP_SEG - 1) / PREP_SEG;
     { LaunchScope ls_("bwd_gate_partial", st); gate_partial_kernel<<<dim3(nseg, s.B * s.H), 256, 0, st>>>(a, nseg); }
     { LaunchScope ls_("bwd_gate_scan", st); gate_scan_kernel<<<dim3(nseg, s.B * s.H), 256, 0, st>>>(a, nseg); }
     if (a.dA) { LaunchScope ls_("bwd_dA", st); dA_final_kernel<<<(s.H + 127) / 128, 128, 0, st>>>(a, nseg); }
     return cudaGetLastError();
 }
-
-}  // namespace
 
 cudaError_t launch_bwd_simt(const BwdArgs& a, cudaStream_t st) {
     const Shape& s = a.s;

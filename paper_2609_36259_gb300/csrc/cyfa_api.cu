@@ -83,26 +83,45 @@ FwdLayout fwd_layout(const Shape& s, bool tc_path, void* ws) {
 }
 
 struct BwdLayout {
-    float *M, *MT, *states, *adj, *o2, *do1, *tok;
+    float *M, *MT, *states, *adj, *o2, *do1, *tok;     // CUDA-core path (+ shared M, tok)
     double *seg, *dA_part;
+    __half *Mb, *snapF, *snapA, *O2b, *DO1b;   // tensor-core path (fp16 operands)
+    float *segS, *segG, *segD, *bnd;
+    double* dA_chunk;
+    int nseg;
     size_t bytes;
 };
-BwdLayout bwd_layout(const Shape& s0, void* ws) {
+BwdLayout bwd_layout(const Shape& s0, bool tc_path, void* ws) {
     Shape s = s0;
     s.C = BWD_C;
     Carver c{static_cast<char*>(ws)};
-    BwdLayout L;
+    BwdLayout L{};
     const size_t BH = (size_t)s.B * s.H;
     const size_t nseg = (s.T + PREP_SEG - 1) / PREP_SEG;
     L.M = c.take<float>((size_t)s.H * MS * MS);
     L.MT = c.take<float>((size_t)s.H * MS * MS);
-    L.states = c.take<float>(BH * s.nchunk() * MS * 2 * s.D);
-    L.adj = c.take<float>(BH * s.nchunk() * MS * 2 * s.D);
-    L.o2 = c.take<float>(BH * s.T * MS);
-    L.do1 = c.take<float>(BH * s.T * MS);
-    L.tok = c.take<float>(5 * BH * s.T);
+    L.tok = c.take<float>((tc_path ? 7 : 5) * BH * s.T);
     L.seg = c.take<double>(2 * BH * nseg);
     L.dA_part = c.take<double>(BH * nseg);
+    if (tc_path) {
+        const size_t nct = s.T / 128;
+        L.nseg = tc_fwd_segments(s0);
+        L.Mb = c.take<__half>((size_t)s.H * MS * MS);
+        L.segS = c.take<float>(BH * L.nseg * MS * 256);
+        L.segD = c.take<float>(BH * L.nseg * MS * 256);
+        L.segG = c.take<float>(BH * L.nseg);
+        L.snapF = c.take<__half>(BH * nct * 2 * MS * 128);
+        L.snapA = c.take<__half>(BH * nct * 2 * MS * 128);
+        L.O2b = c.take<__half>(BH * s.T * MS);
+        L.DO1b = c.take<__half>(BH * s.T * MS);
+        L.bnd = c.take<float>(BH * nct * 2);
+        L.dA_chunk = c.take<double>(BH * nct);
+    } else {
+        L.states = c.take<float>(BH * s.nchunk() * MS * 2 * s.D);
+        L.adj = c.take<float>(BH * s.nchunk() * MS * 2 * s.D);
+        L.o2 = c.take<float>(BH * s.T * MS);
+        L.do1 = c.take<float>(BH * s.T * MS);
+    }
     L.bytes = c.off;
     return L;
 }
@@ -137,7 +156,7 @@ int cyfa_workspace_size(const cyfa_dims_t* dims, int which, size_t* bytes) {
     switch (which) {
         case CYFA_WS_PREPARE: *bytes = up(prepare_workspace(s)); return CYFA_OK;
         case CYFA_WS_FWD: *bytes = fwd_layout(s, use_tc(dims, s), nullptr).bytes; return CYFA_OK;
-        case CYFA_WS_BWD: *bytes = bwd_layout(s, nullptr).bytes; return CYFA_OK;
+        case CYFA_WS_BWD: *bytes = bwd_layout(s, use_tc(dims, s), nullptr).bytes; return CYFA_OK;
         default: return CYFA_ERR_ARG;
     }
 }
@@ -241,10 +260,11 @@ int cyfa_chunk_bwd(const cyfa_dims_t* dims, const void* q, const void* k, const 
         return CYFA_ERR_ALIGN;
     if (dR) return CYFA_ERR_UNSUPPORTED;
     const Shape s = shape_of(dims);
-    const BwdLayout need = bwd_layout(s, nullptr);
+    const bool tc_path = use_tc(dims, s);
+    const BwdLayout need = bwd_layout(s, tc_path, nullptr);
     if (!workspace || workspace_bytes < need.bytes) return CYFA_ERR_WORKSPACE;
     if (!aligned16(workspace)) return CYFA_ERR_ALIGN;
-    const BwdLayout L = bwd_layout(s, workspace);
+    const BwdLayout L = bwd_layout(s, tc_path, workspace);
     cudaStream_t st = static_cast<cudaStream_t>(stream);
     rc = cuda_status(launch_readout_matrix(s.H, R, L.M, L.MT, st));
     if (rc) return rc;
@@ -277,6 +297,47 @@ int cyfa_chunk_bwd(const cyfa_dims_t* dims, const void* q, const void* k, const 
     a.tok = L.tok;
     a.seg = L.seg;
     a.dA_part = L.dA_part;
+    if (tc_path) {
+        TcFwdArgs f{};
+        f.s = s;
+        f.lam = lam_mod;
+        f.g = g_cum;
+        f.beta = beta;
+        f.segS = L.segS;
+        f.segG = L.segG;
+        f.Mb = reinterpret_cast<const __nv_bfloat16*>(L.Mb);   // filled as fp16 (f16 launch)
+        f.nseg = L.nseg;
+        TcBwdArgs t{};
+        t.s = s;
+        t.lam = lam_mod;
+        t.g = g_cum;
+        t.beta = beta;
+        t.segS = L.segS;
+        t.segG = L.segG;
+        t.segD = L.segD;
+        t.nseg = L.nseg;
+        t.snapF = L.snapF;
+        t.snapA = L.snapA;
+        t.O2 = L.O2b;
+        t.DO1 = L.DO1b;
+        t.Mb = L.Mb;
+        t.q = q;
+        t.k = k;
+        t.dq = dq;
+        t.dk = dk;
+        t.dv = dv;
+        t.tok = L.tok;
+        t.bnd = L.bnd;
+        t.clock_logit = clock_logit;
+        t.decay_logit = decay_logit;
+        t.A = A;
+        t.d_clock = d_clock_logit;
+        t.d_decay = d_decay_logit;
+        t.d_beta = d_beta_logit;
+        t.dA = dA;
+        t.dA_part = L.dA_chunk;
+        return cuda_status(launch_bwd_tc(t, f, q, k, v, dO, L.M, st));
+    }
     return cuda_status(launch_bwd_simt(a, st));
 }
 
@@ -316,9 +377,10 @@ int cyfa_step(const cyfa_dims_t* dims, const void* q, const void* k, const void*
 int cyfa_check(void* stream) {
     cudaStream_t st = static_cast<cudaStream_t>(stream);
     if (cudaStreamSynchronize(st) != cudaSuccess) return CYFA_ERR_CUDA;
-    int err = 0;
+    int err = 0, err2 = 0;
     if (tc_read_error(st, &err) != cudaSuccess) return CYFA_ERR_CUDA;
-    return err ? CYFA_ERR_TIMEOUT : CYFA_OK;
+    if (tc_bwd_read_error(st, &err2) != cudaSuccess) return CYFA_ERR_CUDA;
+    return (err || err2) ? CYFA_ERR_TIMEOUT : CYFA_OK;
 }
 
 }  // extern "C"

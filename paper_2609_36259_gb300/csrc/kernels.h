@@ -3,6 +3,7 @@
 
 #include <cuda.h>
 #include <cuda_bf16.h>
+#include <cuda_fp16.h>
 #include <cuda_runtime.h>
 #include <stddef.h>
 
@@ -77,12 +78,15 @@ struct BwdArgs {
 };
 constexpr int BWD_C = 64;       // chunk length used by the SIMT backward
 cudaError_t launch_bwd_simt(const BwdArgs& a, cudaStream_t st);
+// reverse cumulative sums of the per-token scalars in a.tok and the logit gradients
+cudaError_t launch_bwd_gates(const BwdArgs& a, cudaStream_t st);
 
 // ---- tensor-core path (tc_*.cu) ----
-// Encode a bf16 TMA tensor map with 128-byte swizzle (dims / strides innermost first; strides
-// in bytes for dims 1..rank-1).  False if the driver entry point is missing or encoding fails.
+// Encode a 16-bit (bf16, or fp16 with f16 = true) TMA tensor map with 128-byte swizzle (dims /
+// strides innermost first; strides in bytes for dims 1..rank-1).  False if the driver entry
+// point is missing or encoding fails.
 bool make_tmap_bf16(CUtensorMap* map, const void* base, int rank, const unsigned long long* dims,
-                    const unsigned long long* strides_bytes, const unsigned* box);
+                    const unsigned long long* strides_bytes, const unsigned* box, bool f16 = false);
 cudaError_t launch_selftest_mma(int variant, const void* X, const void* Y, float* D,
                                 cudaStream_t st, int* host_err);
 
@@ -103,6 +107,41 @@ cudaError_t launch_fwd_tc(const TcFwdArgs& a, const void* q, const void* k, cons
                           const float* Mf, cudaStream_t st);
 // Reads (and clears) the error word of the tensor-core kernels; synchronises the stream.
 cudaError_t tc_read_error(cudaStream_t st, int* err);
+cudaError_t tc_bwd_read_error(cudaStream_t st, int* err);
+// TMA maps of [B, T, H, 128] bf16 tensors (128-token boxes of one head) and of row-major
+// [rows x 128] bf16 arrays (128-row boxes); null outputs are skipped.
+bool tc_qkv_maps(const Shape& s, const void* q, const void* k, const void* v, CUtensorMap* mq,
+                 CUtensorMap* mk, CUtensorMap* mv);
+bool tc_rows_map(CUtensorMap* map, const void* base, unsigned long long rows, bool f16 = false);
+// M -> 16-bit (tensor-core order), segment state contributions, segment scan (forward); with
+// f16 the operands of the tensor-core products are fp16 (a.Mb then points to fp16 storage).
+cudaError_t launch_fwd_segment_states(const TcFwdArgs& a, const void* k, const void* v,
+                                      const float* Mf, cudaStream_t st, bool f16 = false);
+
+struct TcBwdArgs {
+    Shape s;
+    const float *lam, *g, *beta;
+    float* segS;                 // forward segment-start states (tensor-core row order)
+    float* segG;                 // total log-decay per segment
+    float* segD;                 // adjoint: per-segment contributions, then end-of-segment adjoints
+    int nseg;
+    __half* snapF;               // [B*H][T/128][2][128][128] fp16: Kbar, Vbar at each chunk start
+    __half* snapA;               // [B*H][T/128][2][128][128] fp16: D^K, D^V at each chunk end
+    __half* O2;                  // [B*H][T][128] fp16: o'' (tensor-core order)
+    __half* DO1;                 // [B*H][T][128] fp16: dL/do' (tensor-core order)
+    const __half* Mb;            // [H][128][128] fp16 M = R Phi
+    const void *q, *k;           // [B,T,H,128] bf16 (row reads of the epilogues)
+    void *dq, *dk, *dv;
+    float* tok;                  // [7][B*T*H] per-token scalars: row side of dG, d lambda;
+                                 // intra-chunk column side of dG, d lambda; d beta;
+                                 // inter-chunk column side of dG, d lambda
+    float* bnd;                  // [B*H][T/128][2]: gamma^C <D, S>, gamma^C <D, Omega S>
+    const float *clock_logit, *decay_logit, *A;
+    float *d_clock, *d_decay, *d_beta, *dA;
+    double* dA_part;             // [B*H][T/128]
+};
+cudaError_t launch_bwd_tc(const TcBwdArgs& a, const TcFwdArgs& f, const void* q, const void* k,
+                          const void* v, const void* dO, const float* Mf, cudaStream_t st);
 
 // ---- decode (decode.cu) ----
 struct StepArgs {

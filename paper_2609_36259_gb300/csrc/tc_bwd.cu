@@ -1,0 +1,1203 @@
+// Tensor-core (tcgen05 / TMEM / TMA) backward of the CyFA operator for bf16 inputs, d = 128.
+// Every tensor-core operand of the backward is fp16: the bf16 inputs are converted exactly in
+// shared memory after their TMA loads, and the stored intermediates (states, adjoints, o'', dO',
+// score matrices) carry fp16's 11-bit significand.  The clock gradient is a difference of
+// nearly cancelling paths (<dz, Omega z> against <do'', Omega o''>), so the 8-bit significand of
+// bf16 intermediates would show in it at long sequence lengths.
+//
+// Gradient of sum(o * dO) through the chunk form of App. B and the middle line of Sec. 3.3
+// Eq. cyfa-two-pass, on 128-token chunks (segments of TC_SEGC chunks):
+//   forward segment states (tc_fwd.cu)  S_start per segment;
+//   snap_fwd_tc   walks each segment and stores the fp16 chunk-start states [Kbar | Vbar];
+//   bwd_chunk1_tc per chunk: recompute O', O''; dO'' = gamma (dO Vbar^T) + (dO V^T o Gamma) A;
+//                 the middle readout's gradient (softmax backward through R Phi) gives dO';
+//                 dq = s [gamma (dO' Kbar) + (dO' A^T o Gamma) K]; stores o'', dO' and the
+//                 per-token scalars <o'', do''> + <q~, dq~> and <dz, Omega z> - <do'', Omega o''>;
+//   adj_walk_tc   the adjoint states of the reversed recurrence
+//                 D_c = gamma^C D_{c+1} + sum_r gamma^r [dO'_r q~_r^T | o''_r dO_r^T]:
+//                 per-segment contributions, a reverse segment scan, then per-chunk snapshots;
+//   bwd_chunk2_tc per chunk: dK = P3^T Q~ + A-> D^K, dV = P2^T dO + A-> D^V,
+//                 dA = P4^T O'' + V-> D^V^T + P1^T dO' + K-> D^K^T (rows -> scaled by
+//                 gamma^C / gamma^s), and the per-token scalars of the gate gradients;
+//   tc_gate       the reverse cumulative sums of App. D.1 (d delta_s = sum_{t>=s} d lambda_t,
+//                 d log alpha_s = sum_{t>=s} dG_t), split at the end of s's chunk: the tokens of
+//                 the chunk are summed directly, everything after the chunk enters as one
+//                 state-level term.  Moving the clock of every later token by e is, by the
+//                 clock-origin invariance of Prop. 6, the same as rotating the chunk-end states
+//                 S by U(e); raising the log-decay of every later token by e is the same as
+//                 scaling S by exp(e).  So the later tokens contribute <D, Omega S> to the clock
+//                 gradient and <D, S> to the decay gradient, with D the adjoint of S.  This keeps
+//                 the per-token terms, which are small differences of large products, from being
+//                 summed over the whole sequence.
+#include "tc_chunk.cuh"
+
+namespace cyfa {
+
+namespace {
+
+using namespace tc;
+
+__device__ __forceinline__ void load_gates_row(const Shape& s, const TcBwdArgs& a, int b, int h,
+                                               int t0, int row, float& lam, float& beta,
+                                               float& g) {
+    const size_t gi = ((size_t)b * s.T + t0 + row) * s.H + h;
+    lam = a.lam[gi];
+    beta = a.beta[gi];
+    g = cum128(s, a.g, b, h, t0, t0 + row);
+}
+
+// 64 fp32 values -> 16-bit OT at dst (plain row-major, 128 bytes)
+template <typename OT>
+__device__ __forceinline__ void store_global_half(OT* dst, const float (&x)[64]) {
+#pragma unroll
+    for (int q = 0; q < 8; ++q) {
+        uint4 u;
+        u.x = pack2<OT>(x[8 * q + 0], x[8 * q + 1]);
+        u.y = pack2<OT>(x[8 * q + 2], x[8 * q + 3]);
+        u.z = pack2<OT>(x[8 * q + 4], x[8 * q + 5]);
+        u.w = pack2<OT>(x[8 * q + 6], x[8 * q + 7]);
+        *reinterpret_cast<uint4*>(dst + 8 * q) = u;
+    }
+}
+
+// eight fp16 values -> fp32
+__device__ __forceinline__ void unpack8(const uint4& u, float* f) {
+    const __half2* p = reinterpret_cast<const __half2*>(&u);
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        const float2 t = __half22float2(p[i]);
+        f[2 * i] = t.x;
+        f[2 * i + 1] = t.y;
+    }
+}
+
+// Columns [64 hf, 64 hf + 64) of row r of a swizzled fp16 tile, as fp32.
+__device__ __forceinline__ void load_half_smem(const uint8_t* tile, int r, int hf, float (&x)[64]) {
+#pragma unroll
+    for (int q = 0; q < 8; ++q) {
+        const uint4 u = *reinterpret_cast<const uint4*>(tile + swz_off(r, 64 * hf + 8 * q, 128));
+        unpack8(u, x + 8 * q);
+    }
+}
+
+// Multiply columns [64 hf, +64) of row r of a swizzled fp16 tile by w, in place.
+__device__ __forceinline__ void scale_half_smem(uint8_t* tile, int r, int hf, float w) {
+    float x[64];
+    load_half_smem(tile, r, hf, x);
+#pragma unroll
+    for (int i = 0; i < 64; ++i) x[i] *= w;
+    store_half_bf16<__half>(tile, r, hf, x);
+}
+
+// Fourier-axis write vector of a token on this thread's column half, in fp32 (tensor-core order).
+__device__ __forceinline__ void write_vector_vals(float (&x)[64], int hf, float lam, float w) {
+    HalfAngles ang(lam, hf);
+    const float wa = w * SQRT_2_OVER_M;
+#pragma unroll
+    for (int jj = 0; jj < 32; ++jj) {
+        if (jj > 0) ang.step(jj);
+        x[jj] = wa * ang.c;
+        x[jj + 32] = -wa * ang.s;
+    }
+    if (hf == 1) {
+        x[31] = w * INV_SQRT_M;
+        x[63] = 0.f;
+    }
+}
+
+// <x, Omega y> restricted to the pairs of this column half (tensor-core order):
+// sum_j (2 pi j / m) (x_sin,j y_cos,j - x_cos,j y_sin,j).
+__device__ __forceinline__ float omega_dot_half(const float (&x)[64], const float (&y)[64], int hf) {
+    float acc = 0.f;
+#pragma unroll
+    for (int jj = 0; jj < 32; ++jj) {
+        const int j = 32 * hf + jj + 1;
+        if (j <= NPAIR) acc += (6.283185307179586f * (float)j / 127.f) * (x[jj + 32] * y[jj] - x[jj] * y[jj + 32]);
+    }
+    return acc;
+}
+
+__device__ __forceinline__ float dot64(const float (&x)[64], const float (&y)[64]) {
+    float acc = 0.f;
+#pragma unroll
+    for (int i = 0; i < 64; ++i) acc = fmaf(x[i], y[i], acc);
+    return acc;
+}
+
+// ---------------------------------------------------------------------------------------
+// Chunk-start states of every chunk, walking each segment from its start state.
+__global__ void __launch_bounds__(256, 1) snap_fwd_tc(const __grid_constant__ CUtensorMap tk,
+                                                       const __grid_constant__ CUtensorMap tv,
+                                                       TcBwdArgs a) {
+    const Shape s = a.s;
+    const int seg = blockIdx.x, bh = blockIdx.y, b = bh / s.H, h = bh % s.H;
+    const int nct = s.T / CT;
+    const int c_begin = seg * TC_SEGC;
+    const int nc = min(TC_SEGC, nct - c_begin);
+    const int tid = threadIdx.x;
+    const Role ro;
+    const int row = ro.row, hf = ro.hf;
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                               ~uintptr_t(1023));
+    uint64_t* bars = reinterpret_cast<uint64_t*>(smem);   // tma[2], mma[2]
+    uint32_t* s_taddr = reinterpret_cast<uint32_t*>(smem + 64);
+    uint8_t* tiles = smem + 1024;                         // [buf][A-> | K | V]
+    if (tid == 0) {
+        for (int i = 0; i < 4; ++i) mbar_init(&bars[i], 1);
+        fence_mbar_init();
+    }
+    if (ro.warp == 0) tmem_alloc(s_taddr, 256);
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t taddr = *s_taddr;
+    const uint32_t tl = taddr + ((uint32_t)(32 * ro.q) << 16);
+    auto issue_kv = [&](int c, int buf) {
+        uint8_t* tK = tiles + (3 * buf + 1) * TILE;
+        uint8_t* tV = tiles + (3 * buf + 2) * TILE;
+        const int r0 = b * s.T + (c_begin + c) * CT;
+        mbar_expect_tx(&bars[buf], 2 * TILE);
+        tma_load_3d(tK, &tk, 0, h, r0, &bars[buf]);
+        tma_load_3d(tK + TILE / 2, &tk, 64, h, r0, &bars[buf]);
+        tma_load_3d(tV, &tv, 0, h, r0, &bars[buf]);
+        tma_load_3d(tV + TILE / 2, &tv, 64, h, r0, &bars[buf]);
+    };
+    if (tid == 0) issue_kv(0, 0);
+    {   // segment-start state into TMEM: thread half hf takes columns [128 hf, 128 hf + 128)
+        const float* src = a.segS + (((size_t)bh * a.nseg + seg) * 128 + row) * 256 + 128 * hf;
+#pragma unroll
+        for (int q2 = 0; q2 < 2; ++q2) {
+            float x[64];
+#pragma unroll
+            for (int i = 0; i < 64; i += 4) {
+                const float4 f = *reinterpret_cast<const float4*>(src + 64 * q2 + i);
+                x[i] = f.x; x[i + 1] = f.y; x[i + 2] = f.z; x[i + 3] = f.w;
+            }
+            tmem_st64(tl + 128 * hf + 64 * q2, x);
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    bool ok = true;
+    const uint32_t id_nn = idesc_f16(128, 128, 1, 1);
+    for (int c = 0; c < nc; ++c) {
+        const int buf = c & 1, cg = c_begin + c, t0 = cg * CT;
+        if (c >= 1 && ok) ok = mbar_wait(&bars[2 + ((c - 1) & 1)], ((c - 1) >> 1) & 1);
+        tc_fence_after();
+        if (tid == 0 && ok && c + 1 < nc) issue_kv(c + 1, (c + 1) & 1);
+        float lam, beta, g;
+        load_gates_row(s, a, b, h, t0, row, lam, beta, g);
+        const float gC = cum128(s, a.g, b, h, t0, t0 + CT - 1);
+        {   // snapshot of this chunk's start state, then S <- gamma^C S
+            __half* dst = a.snapF + (((size_t)bh * nct + cg) * 2 + hf) * 128 * 128 + row * 128;
+            const float dC = ex2(gC * LOG2E);
+#pragma unroll
+            for (int q2 = 0; q2 < 2; ++q2) {
+                float x[64];
+                tmem_ld64(tl + 128 * hf + 64 * q2, x);
+                store_global_half(dst + 64 * q2, x);
+#pragma unroll
+                for (int i = 0; i < 64; ++i) x[i] *= dC;
+                tmem_st64(tl + 128 * hf + 64 * q2, x);
+            }
+        }
+        write_vector_half<__half>(tiles + 3 * buf * TILE, row, hf, lam, beta * ex2((gC - g) * LOG2E));
+        if (ok) ok = mbar_wait(&bars[buf], (c >> 1) & 1);
+        if (ok) {
+            bf16_to_f16_half(tiles + (3 * buf + 1) * TILE, row, hf);
+            bf16_to_f16_half(tiles + (3 * buf + 2) * TILE, row, hf);
+        }
+        fence_async_smem();
+        tc_fence_before();
+        ok = __syncthreads_and(ok);
+        tc_fence_after();
+        if (!ok) break;
+        if (tid == 0) {
+            {
+                const uint32_t tA = smem_u32(tiles + 3 * buf * TILE);
+                const uint32_t tK = smem_u32(tiles + (3 * buf + 1) * TILE);
+                const uint32_t tV = smem_u32(tiles + (3 * buf + 2) * TILE);
+#pragma unroll
+                for (int k = 0; k < 8; ++k) {
+                    mma_bf16(taddr, mnmajor_desc(tA, 128, k), mnmajor_desc(tK, 128, k), id_nn, 1u);
+                    mma_bf16(taddr + 128, mnmajor_desc(tA, 128, k), mnmajor_desc(tV, 128, k), id_nn, 1u);
+                }
+                mma_commit(&bars[2 + buf]);
+            }
+        }
+    }
+    if (ok) ok = mbar_wait(&bars[2 + ((nc - 1) & 1)], ((nc - 1) >> 1) & 1);
+    ok = __syncthreads_and(ok);
+    if (!ok && tid == 0) {
+        flag_error(CYFA_ERR_TIMEOUT);
+        for (int i = 0; i < 2; ++i) mbar_wait(&bars[i], 0);
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (ro.warp == 0) tmem_dealloc(taddr, 256);
+}
+
+// ---------------------------------------------------------------------------------------
+// Per chunk: recompute O', O''; dO''; middle-readout gradient; dO'; dq; per-token scalars.
+__global__ void __launch_bounds__(256, 1) bwd_chunk1_tc(const __grid_constant__ CUtensorMap tq,
+                                                         const __grid_constant__ CUtensorMap tk,
+                                                         const __grid_constant__ CUtensorMap tv,
+                                                         const __grid_constant__ CUtensorMap tdo,
+                                                         const __grid_constant__ CUtensorMap tm,
+                                                         const __grid_constant__ CUtensorMap tsf,
+                                                         TcBwdArgs a) {
+    const Shape s = a.s;
+    const int cg = blockIdx.x, bh = blockIdx.y, b = bh / s.H, h = bh % s.H;
+    const int nct = s.T / CT, t0 = cg * CT;
+    const int tid = threadIdx.x;
+    const Role ro;
+    const int row = ro.row, hf = ro.hf;
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                               ~uintptr_t(1023));
+    uint64_t* bars = reinterpret_cast<uint64_t*>(smem);            // tma0, tma1, mma
+    uint32_t* s_taddr = reinterpret_cast<uint32_t*>(smem + 32);
+    float* s_g2 = reinterpret_cast<float*>(smem + 64);
+    float* s_red = s_g2 + 128;                                      // [2][128]
+    uint8_t* T_K = smem + 2048;       // V (first), then K
+    uint8_t* T_KB = T_K + 1 * TILE;   // Kbar snapshot (rows = slots)
+    uint8_t* T_A = T_K + 2 * TILE;    // write vectors (rows = tokens)
+    uint8_t* T_M = T_K + 3 * TILE;    // M = R Phi
+    uint8_t* T_S = T_K + 4 * TILE;    // staging
+    uint8_t* T_L1 = T_K + 5 * TILE;   // dO, then Q
+    uint8_t* T_L2 = T_K + 6 * TILE;   // Vbar snapshot
+    if (tid == 0) {
+        for (int i = 0; i < 3; ++i) mbar_init(&bars[i], 1);
+        fence_mbar_init();
+    }
+    if (ro.warp == 0) tmem_alloc(s_taddr, 512);
+    float lam, beta, g;
+    load_gates_row(s, a, b, h, t0, row, lam, beta, g);
+    const float g2 = g * LOG2E;
+    if (hf == 0) s_g2[row] = g2;
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t taddr = *s_taddr;
+    const uint32_t tl = taddr + ((uint32_t)(32 * ro.q) << 16);
+    const uint32_t X1 = 64 * hf, X2 = 128 + 64 * hf, X3 = 256 + 64 * hf, X4 = 384 + 64 * hf;
+    const int rowtok = b * s.T + t0;
+    const int snap_row = (bh * nct + cg) * 2 * 128;
+    if (tid == 0) {
+        mbar_expect_tx(&bars[0], 5 * TILE);
+        tma_load_3d(T_L1, &tdo, 0, h, rowtok, &bars[0]);
+        tma_load_3d(T_L1 + TILE / 2, &tdo, 64, h, rowtok, &bars[0]);
+        tma_load_3d(T_K, &tv, 0, h, rowtok, &bars[0]);
+        tma_load_3d(T_K + TILE / 2, &tv, 64, h, rowtok, &bars[0]);
+        tma_load_2d(T_L2, &tsf, 0, snap_row + 128, &bars[0]);
+        tma_load_2d(T_L2 + TILE / 2, &tsf, 64, snap_row + 128, &bars[0]);
+        tma_load_2d(T_KB, &tsf, 0, snap_row, &bars[0]);
+        tma_load_2d(T_KB + TILE / 2, &tsf, 64, snap_row, &bars[0]);
+        tma_load_2d(T_M, &tm, 0, h * 128, &bars[0]);
+        tma_load_2d(T_M + TILE / 2, &tm, 64, h * 128, &bars[0]);
+    }
+    write_vector_half<__half>(T_A, row, hf, lam, beta);
+    bool ok = mbar_wait(&bars[0], 0);
+    if (ok) {   // dO and V: bf16 -> fp16
+        bf16_to_f16_half(T_L1, row, hf);
+        bf16_to_f16_half(T_K, row, hf);
+    }
+    uint32_t mma_ph = 0;
+    auto publish = [&]() {
+        fence_async_smem();
+        tc_fence_before();
+        ok = __syncthreads_and(ok);
+        tc_fence_after();
+    };
+    auto wait_mma = [&]() {
+        if (ok) ok = mbar_wait(&bars[2], mma_ph);
+        mma_ph ^= 1;
+        tc_fence_after();
+    };
+    auto issuer = [&]() { return tid == 0 && ok; };
+    auto mask_scores = [&](float (&x)[64], float mul) {
+#pragma unroll
+        for (int grp = 0; grp < 2; ++grp) {
+            const int sg = 2 * hf + grp;
+            if (sg > ro.q) {
+#pragma unroll
+                for (int i = 0; i < 32; ++i) x[32 * grp + i] = 0.f;
+            } else {
+#pragma unroll
+                for (int i = 0; i < 32; ++i) {
+                    const int t = 32 * sg + i;
+                    x[32 * grp + i] = (t <= row) ? mul * x[32 * grp + i] * ex2(g2 - s_g2[t]) : 0.f;
+                }
+            }
+        }
+    };
+    // sum of a per-thread partial over the two column halves of this row
+    auto row_sum = [&](float v) {
+        s_red[128 * hf + row] = v;
+        __syncthreads();
+        const float t = s_red[row] + s_red[128 + row];
+        __syncthreads();
+        return t;
+    };
+    const uint32_t id_kk = idesc_f16(128, 128, 0, 0), id_kn = idesc_f16(128, 128, 0, 1);
+    const uint32_t uK = smem_u32(T_K), uKB = smem_u32(T_KB), uA = smem_u32(T_A), uM = smem_u32(T_M),
+                   uS = smem_u32(T_S), uL1 = smem_u32(T_L1), uL2 = smem_u32(T_L2);
+    const float scale = s.scale;
+    const float gam = ex2(g2);
+    float s1 = 0.f, s2 = 0.f, s3 = 0.f, s4 = 0.f;
+    publish();
+    // G1: X1 = dO V^T, X2 = dO Vbar^T
+    if (issuer()) {
+        {
+#pragma unroll
+            for (int k = 0; k < 8; ++k) {
+                mma_bf16(taddr + 0, kmajor_desc(uL1, 128, k), kmajor_desc(uK, 128, k), id_kk, k > 0);
+                mma_bf16(taddr + 128, kmajor_desc(uL1, 128, k), kmajor_desc(uL2, 128, k), id_kk, k > 0);
+            }
+            mma_commit(&bars[2]);
+        }
+    }
+    wait_mma();
+    if (issuer()) {   // dO and V are consumed: Q and K
+        mbar_expect_tx(&bars[1], 2 * TILE);
+        tma_load_3d(T_L1, &tq, 0, h, rowtok, &bars[1]);
+        tma_load_3d(T_L1 + TILE / 2, &tq, 64, h, rowtok, &bars[1]);
+        tma_load_3d(T_K, &tk, 0, h, rowtok, &bars[1]);
+        tma_load_3d(T_K + TILE / 2, &tk, 64, h, rowtok, &bars[1]);
+    }
+    {   // P4 = (dO V^T) o Gamma
+        float x[64];
+        tmem_ld64(tl + X1, x);
+        mask_scores(x, 1.f);
+        store_half_bf16<__half>(T_S, row, hf, x);
+    }
+    publish();
+    if (issuer()) {   // G2: X3 = P4 A
+#pragma unroll
+        for (int k = 0; k < 8; ++k)
+            mma_bf16(taddr + 256, kmajor_desc(uS, 128, k), mnmajor_desc(uA, 128, k), id_kn, k > 0);
+        mma_commit(&bars[2]);
+    }
+    wait_mma();
+    {   // do'' = gamma (dO Vbar^T) + P4 A, kept in X2
+        float x[64], y[64];
+        tmem_ld64(tl + X2, x);
+        tmem_ld64(tl + X3, y);
+#pragma unroll
+        for (int i = 0; i < 64; ++i) x[i] = fmaf(gam, x[i], y[i]);
+        tmem_st64(tl + X2, x);
+        if (ok) ok = mbar_wait(&bars[1], 0);
+        if (ok) {   // Q and K: bf16 -> fp16
+            bf16_to_f16_half(T_L1, row, hf);
+            bf16_to_f16_half(T_K, row, hf);
+        }
+    }
+    publish();
+    if (issuer()) {   // G3: X1 = Q K^T, X3 = Q Kbar^T
+        {
+#pragma unroll
+            for (int k = 0; k < 8; ++k) {
+                mma_bf16(taddr + 0, kmajor_desc(uL1, 128, k), kmajor_desc(uK, 128, k), id_kk, k > 0);
+                mma_bf16(taddr + 256, kmajor_desc(uL1, 128, k), kmajor_desc(uKB, 128, k), id_kk, k > 0);
+            }
+            mma_commit(&bars[2]);
+        }
+    }
+    wait_mma();
+    {   // P1 = s (Q K^T) o Gamma
+        float x[64];
+        tmem_ld64(tl + X1, x);
+        mask_scores(x, scale);
+        store_half_bf16<__half>(T_S, row, hf, x);
+    }
+    publish();
+    if (issuer()) {   // G4: X4 = P1 A
+#pragma unroll
+        for (int k = 0; k < 8; ++k)
+            mma_bf16(taddr + 384, kmajor_desc(uS, 128, k), mnmajor_desc(uA, 128, k), id_kn, k > 0);
+        mma_commit(&bars[2]);
+    }
+    wait_mma();
+    {   // z = U(lam) o', kept in X3
+        float x[64], y[64];
+        tmem_ld64(tl + X3, x);
+        tmem_ld64(tl + X4, y);
+        const float f = scale * gam;
+#pragma unroll
+        for (int i = 0; i < 64; ++i) x[i] = fmaf(f, x[i], y[i]);
+        rotate_half<1>(x, hf, lam);
+        store_half_bf16<__half>(T_S, row, hf, x);
+        tmem_st64(tl + X3, x);
+    }
+    publish();
+    if (issuer()) {   // G5: X1 = z M^T
+#pragma unroll
+        for (int k = 0; k < 8; ++k)
+            mma_bf16(taddr + 0, kmajor_desc(uS, 128, k), kmajor_desc(uM, 128, k), id_kk, k > 0);
+        mma_commit(&bars[2]);
+    }
+    wait_mma();
+    {   // p = softmax(l), kept in X1
+        float x[64];
+        tmem_ld64(tl + X1, x);
+        const int nvalid = hf ? 63 : 64;
+        float mx = -INFINITY;
+#pragma unroll
+        for (int i = 0; i < 64; ++i)
+            if (i < nvalid) mx = fmaxf(mx, x[i]);
+        s_red[128 * hf + row] = mx;
+        __syncthreads();
+        mx = fmaxf(s_red[row], s_red[128 + row]);
+        __syncthreads();
+        float sum = 0.f;
+#pragma unroll
+        for (int i = 0; i < 64; ++i) {
+            x[i] = (i < nvalid) ? ex2((x[i] - mx) * LOG2E) : 0.f;
+            sum += x[i];
+        }
+        const float inv = 1.f / row_sum(sum);
+#pragma unroll
+        for (int i = 0; i < 64; ++i) x[i] *= inv;
+        store_half_bf16<__half>(T_S, row, hf, x);
+        tmem_st64(tl + X1, x);
+    }
+    publish();
+    if (issuer()) {   // G6: X4 = p M
+#pragma unroll
+        for (int k = 0; k < 8; ++k)
+            mma_bf16(taddr + 384, kmajor_desc(uS, 128, k), mnmajor_desc(uM, 128, k), id_kn, k > 0);
+        mma_commit(&bars[2]);
+    }
+    wait_mma();
+    {   // o'' = U(-lam) (p M); scalars with do'' (o'' as stored in bf16); dy = U(lam) do''
+        float o2[64], g2v[64];
+        tmem_ld64(tl + X4, o2);
+        rotate_half<-1>(o2, hf, lam);
+        store_global_half(a.O2 + ((size_t)bh * s.T + t0 + row) * 128 + 64 * hf, o2);
+#pragma unroll
+        for (int i = 0; i < 64; ++i) o2[i] = round16<__half>((o2[i]));
+        tmem_ld64(tl + X2, g2v);
+        s1 = dot64(o2, g2v);
+        s2 = omega_dot_half(o2, g2v, hf);   // <o'', Omega do''> = -<do'', Omega o''>
+        rotate_half<1>(g2v, hf, lam);
+        store_half_bf16<__half>(T_S, row, hf, g2v);
+    }
+    publish();
+    if (issuer()) {   // G7: X4 = dy M^T = M dy
+#pragma unroll
+        for (int k = 0; k < 8; ++k)
+            mma_bf16(taddr + 384, kmajor_desc(uS, 128, k), kmajor_desc(uM, 128, k), id_kk, k > 0);
+        mma_commit(&bars[2]);
+    }
+    wait_mma();
+    {   // dl = p o (dp - <p, dp>)
+        float p[64], dp[64];
+        tmem_ld64(tl + X1, p);
+        tmem_ld64(tl + X4, dp);
+        const float pdp = row_sum(dot64(p, dp));
+#pragma unroll
+        for (int i = 0; i < 64; ++i) p[i] = p[i] * (dp[i] - pdp);
+        store_half_bf16<__half>(T_S, row, hf, p);
+    }
+    publish();
+    if (issuer()) {   // G8: X2 = dl M = M^T dl
+#pragma unroll
+        for (int k = 0; k < 8; ++k)
+            mma_bf16(taddr + 128, kmajor_desc(uS, 128, k), mnmajor_desc(uM, 128, k), id_kn, k > 0);
+        mma_commit(&bars[2]);
+    }
+    wait_mma();
+    {   // do' = U(-lam) dz; <do', Omega o'> with do' as stored in bf16 (= <dz, Omega z> exactly)
+        float dz[64], z[64];
+        tmem_ld64(tl + X2, dz);
+        tmem_ld64(tl + X3, z);
+        rotate_half<-1>(dz, hf, lam);
+        store_half_bf16<__half>(T_S, row, hf, dz);
+        store_global_half(a.DO1 + ((size_t)bh * s.T + t0 + row) * 128 + 64 * hf, dz);
+        rotate_half<-1>(z, hf, lam);   // o'
+#pragma unroll
+        for (int i = 0; i < 64; ++i) dz[i] = round16<__half>((dz[i]));
+        s3 = omega_dot_half(dz, z, hf);
+    }
+    publish();
+    if (issuer()) {   // G9: X1 = dO' A^T, X3 = dO' Kbar
+#pragma unroll
+        for (int k = 0; k < 8; ++k) {
+            mma_bf16(taddr + 0, kmajor_desc(uS, 128, k), kmajor_desc(uA, 128, k), id_kk, k > 0);
+            mma_bf16(taddr + 256, kmajor_desc(uS, 128, k), mnmajor_desc(uKB, 128, k), id_kn, k > 0);
+        }
+        mma_commit(&bars[2]);
+    }
+    wait_mma();
+    {   // P3 = s (dO' A^T) o Gamma
+        float x[64];
+        tmem_ld64(tl + X1, x);
+        mask_scores(x, scale);
+        store_half_bf16<__half>(T_S, row, hf, x);
+    }
+    publish();
+    if (issuer()) {   // G10: X4 = P3 K
+#pragma unroll
+        for (int k = 0; k < 8; ++k)
+            mma_bf16(taddr + 384, kmajor_desc(uS, 128, k), mnmajor_desc(uK, 128, k), id_kn, k > 0);
+        mma_commit(&bars[2]);
+    }
+    wait_mma();
+    if (ok) {   // dq = s gamma (dO' Kbar) + P3 K  (P3 carries s) ; <q, dq> = <q~, dq~>
+        float x[64], y[64], qv[64];
+        tmem_ld64(tl + X3, x);
+        tmem_ld64(tl + X4, y);
+        const float f = scale * gam;
+#pragma unroll
+        for (int i = 0; i < 64; ++i) x[i] = fmaf(f, x[i], y[i]);
+        load_half_smem(T_L1, row, hf, qv);
+        s4 = dot64(qv, x);
+        const size_t gi = ((size_t)b * s.T + t0 + row) * s.H + h;
+        store_global_half(static_cast<__nv_bfloat16*>(a.dq) + gi * 128 + 64 * hf, x);
+    }
+    {
+        const float dG = row_sum(s1 + s4);
+        const float dL = row_sum(s3 + s2);
+        if (hf == 0 && ok) {
+            const size_t gi = ((size_t)b * s.T + t0 + row) * s.H + h;
+            const size_t BTH = (size_t)s.B * s.T * s.H;
+            a.tok[gi] = dG;
+            a.tok[BTH + gi] = dL;
+        }
+    }
+    ok = __syncthreads_and(ok);
+    if (!ok && tid == 0) {
+        flag_error(CYFA_ERR_TIMEOUT);
+        mbar_wait(&bars[0], 0);
+        mbar_wait(&bars[1], 0);
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (ro.warp == 0) tmem_dealloc(taddr, 512);
+}
+
+// ---------------------------------------------------------------------------------------
+// Adjoint states of the reversed recurrence, per segment.  SNAP = false: the segment's own
+// contribution  dD = sum_r exp(G_r - G_start) [dO'_r q~_r^T | o''_r dO_r^T]  (into segD);
+// SNAP = true: walk the segment backwards from its end adjoint (segD after the reverse scan),
+// storing before each chunk the adjoint of that chunk's end state, then
+// D <- gamma^C D + sum_r gamma^r [...].  The K part (dO', q~) and the V part (o'', dO) run one
+// after the other with double-buffered tiles.
+template <bool SNAP>
+__global__ void __launch_bounds__(256, 1) adj_walk_tc(const __grid_constant__ CUtensorMap tdo1,
+                                                       const __grid_constant__ CUtensorMap to2,
+                                                       const __grid_constant__ CUtensorMap tq,
+                                                       const __grid_constant__ CUtensorMap tdo,
+                                                       TcBwdArgs a) {
+    const Shape s = a.s;
+    const int seg = blockIdx.x, bh = blockIdx.y, b = bh / s.H, h = bh % s.H;
+    const int nct = s.T / CT;
+    const int c_begin = seg * TC_SEGC;
+    const int nc = min(TC_SEGC, nct - c_begin);
+    const int tid = threadIdx.x;
+    const Role ro;
+    const int row = ro.row, hf = ro.hf;
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                               ~uintptr_t(1023));
+    uint64_t* bars = reinterpret_cast<uint64_t*>(smem);   // tma[2], mma[2]
+    uint32_t* s_taddr = reinterpret_cast<uint32_t*>(smem + 64);
+    float* s_tot = reinterpret_cast<float*>(smem + 128);   // [TC_SEGC]
+    float* s_pre = s_tot + TC_SEGC;                         // [TC_SEGC]
+    float* s_bnd = s_pre + TC_SEGC;                         // [TC_SEGC][2]
+    uint8_t* tiles = smem + 1024;                          // [buf][X | Y]
+    if (tid == 0) {
+        for (int i = 0; i < 4; ++i) mbar_init(&bars[i], 1);
+        fence_mbar_init();
+    }
+    if (ro.warp == 0) tmem_alloc(s_taddr, 256);
+    if (tid < nc) {
+        const int t0 = (c_begin + tid) * CT;
+        s_tot[tid] = cum128(s, a.g, b, h, t0, t0 + CT - 1);
+        s_bnd[2 * tid] = 0.f;
+        s_bnd[2 * tid + 1] = 0.f;
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t taddr = *s_taddr;
+    const uint32_t tl = taddr + ((uint32_t)(32 * ro.q) << 16);
+    if (tid == 0) {
+        float acc = 0.f;
+        for (int c = 0; c < nc; ++c) {
+            s_pre[c] = acc;
+            acc += s_tot[c];
+        }
+    }
+    if (SNAP) {   // end-of-segment adjoint into TMEM
+        const float* src = a.segD + (((size_t)bh * a.nseg + seg) * 128 + row) * 256 + 128 * hf;
+#pragma unroll
+        for (int q2 = 0; q2 < 2; ++q2) {
+            float x[64];
+#pragma unroll
+            for (int i = 0; i < 64; i += 4) {
+                const float4 f = *reinterpret_cast<const float4*>(src + 64 * q2 + i);
+                x[i] = f.x; x[i + 1] = f.y; x[i + 2] = f.z; x[i + 3] = f.w;
+            }
+            tmem_st64(tl + 128 * hf + 64 * q2, x);
+        }
+    }
+    const int total = 2 * nc;   // iterations: part 0 (K) chunks, then part 1 (V) chunks
+    auto chunk_of = [&](int it) {
+        const int i = it % nc;
+        return SNAP ? nc - 1 - i : i;
+    };
+    auto issue = [&](int it) {
+        const int part = it / nc, c = chunk_of(it), buf = it & 1;
+        uint8_t* tX = tiles + (2 * buf) * TILE;
+        uint8_t* tY = tiles + (2 * buf + 1) * TILE;
+        const int t0 = (c_begin + c) * CT;
+        const int xrow = bh * s.T + t0, yrow = b * s.T + t0;
+        const CUtensorMap* mx = part == 0 ? &tdo1 : &to2;
+        const CUtensorMap* my = part == 0 ? &tq : &tdo;
+        mbar_expect_tx(&bars[buf], 2 * TILE);
+        tma_load_2d(tX, mx, 0, xrow, &bars[buf]);
+        tma_load_2d(tX + TILE / 2, mx, 64, xrow, &bars[buf]);
+        tma_load_3d(tY, my, 0, h, yrow, &bars[buf]);
+        tma_load_3d(tY + TILE / 2, my, 64, h, yrow, &bars[buf]);
+    };
+    if (tid == 0) issue(0);
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    bool ok = true;
+    const uint32_t id_nn = idesc_f16(128, 128, 1, 1);
+    for (int it = 0; it < total; ++it) {
+        const int part = it / nc, c = chunk_of(it), buf = it & 1;
+        const int cg = c_begin + c, t0 = cg * CT;
+        if (it >= 1 && ok) ok = mbar_wait(&bars[2 + ((it - 1) & 1)], ((it - 1) >> 1) & 1);
+        tc_fence_after();
+        if (tid == 0 && ok && it + 1 < total) issue(it + 1);
+        if (ok) ok = mbar_wait(&bars[buf], (it >> 1) & 1);
+        const float g = cum128(s, a.g, b, h, t0, t0 + row);
+        float w;
+        if (SNAP) {
+            // adjoint of this chunk's end state, then D <- gamma^C D (this part's 128 columns)
+            __half* dst = a.snapA + (((size_t)bh * nct + cg) * 2 + part) * 128 * 128 + row * 128 + 64 * hf;
+            const float dC = ex2(s_tot[c] * LOG2E);
+            float x[64];
+            tmem_ld64(tl + 128 * part + 64 * hf, x);
+            store_global_half(dst, x);
+            {
+                // gamma^C <D, S> and gamma^C <D, Omega S> with S this chunk's start state (the
+                // chunk's own writes enter through the inter-chunk column terms of
+                // bwd_chunk2_tc); this thread's row and 64 columns
+                const __half* Sp = a.snapF + (((size_t)bh * nct + cg) * 2 + part) * 128 * 128;
+                const int l = row & 63, jj = l & 31, j = 32 * (row >> 6) + jj + 1;
+                const bool paired = j <= NPAIR;
+                const int partner = (l >= 32) ? row - 32 : row + 32;
+                const float f = paired ? ((l >= 32) ? 1.f : -1.f) * 6.283185307179586f * (float)j / 127.f : 0.f;
+                float sr[64], sp[64];
+#pragma unroll
+                for (int q2 = 0; q2 < 8; ++q2) {
+                    unpack8(*reinterpret_cast<const uint4*>(Sp + row * 128 + 64 * hf + 8 * q2), sr + 8 * q2);
+                    unpack8(*reinterpret_cast<const uint4*>(Sp + (paired ? partner : row) * 128 + 64 * hf + 8 * q2), sp + 8 * q2);
+                }
+                float bG = dC * dot64(x, sr), bL = dC * f * dot64(x, sp);
+                bG = warp_sum(bG);
+                bL = warp_sum(bL);
+                if (ro.lane == 0) {
+                    atomicAdd(&s_bnd[2 * c], bG);
+                    atomicAdd(&s_bnd[2 * c + 1], bL);
+                }
+            }
+#pragma unroll
+            for (int i = 0; i < 64; ++i) x[i] *= dC;
+            tmem_st64(tl + 128 * part + 64 * hf, x);
+            w = ex2(g * LOG2E);
+        } else {
+            w = ex2((s_pre[c] + g) * LOG2E);
+        }
+        if (part == 0) w *= s.scale;   // q~ = s q
+        if (ok) {
+            scale_half_smem(tiles + (2 * buf) * TILE, row, hf, w);
+            bf16_to_f16_half(tiles + (2 * buf + 1) * TILE, row, hf);   // q or dO
+        }
+        fence_async_smem();
+        tc_fence_before();
+        ok = __syncthreads_and(ok);
+        tc_fence_after();
+        if (!ok) break;
+        if (tid == 0) {
+            const uint32_t tX = smem_u32(tiles + (2 * buf) * TILE);
+            const uint32_t tY = smem_u32(tiles + (2 * buf + 1) * TILE);
+            const bool first = !SNAP && (it % nc) == 0;
+#pragma unroll
+            for (int k = 0; k < 8; ++k)
+                mma_bf16(taddr + 128 * part, mnmajor_desc(tX, 128, k), mnmajor_desc(tY, 128, k),
+                         id_nn, (first && k == 0) ? 0u : 1u);
+            mma_commit(&bars[2 + buf]);
+        }
+    }
+    if (ok) ok = mbar_wait(&bars[2 + ((total - 1) & 1)], ((total - 1) >> 1) & 1);
+    tc_fence_after();
+    ok = __syncthreads_and(ok);
+    if (SNAP && ok && tid < nc) {
+        float* dst = a.bnd + ((size_t)bh * nct + c_begin + tid) * 2;
+        dst[0] = s_bnd[2 * tid];
+        dst[1] = s_bnd[2 * tid + 1];
+    }
+    if (ok && !SNAP) {
+        float* dst = a.segD + (((size_t)bh * a.nseg + seg) * 128 + row) * 256 + 128 * hf;
+#pragma unroll
+        for (int q2 = 0; q2 < 2; ++q2) {
+            float x[64];
+            tmem_ld64(tl + 128 * hf + 64 * q2, x);
+#pragma unroll
+            for (int i = 0; i < 64; i += 4)
+                *reinterpret_cast<float4*>(dst + 64 * q2 + i) = make_float4(x[i], x[i + 1], x[i + 2], x[i + 3]);
+        }
+    }
+    if (!ok && tid == 0) {
+        flag_error(CYFA_ERR_TIMEOUT);
+        for (int i = 0; i < 2; ++i) mbar_wait(&bars[i], 0);
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (ro.warp == 0) tmem_dealloc(taddr, 256);
+}
+
+// End-of-segment adjoints: D_end(last) = 0, D_end(j-1) = exp(G_j) D_end(j) + dD(j), in place.
+__global__ void __launch_bounds__(256) seg_scan_rev_kernel(TcBwdArgs a) {
+    const int bh = blockIdx.y;
+    const int e = blockIdx.x * 256 + threadIdx.x;
+    float* base = a.segD + (size_t)bh * a.nseg * 128 * 256 + e;
+    const float* G = a.segG + (size_t)bh * a.nseg;
+    float cur = 0.f;
+    for (int j1 = a.nseg - 1; j1 >= 0; j1 -= 8) {
+        float d[8], gj[8];
+#pragma unroll
+        for (int u = 0; u < 8; ++u) {
+            const int j = j1 - u;
+            d[u] = j >= 0 ? base[(size_t)j * 128 * 256] : 0.f;
+            gj[u] = j >= 0 ? G[j] : 0.f;
+        }
+#pragma unroll
+        for (int u = 0; u < 8; ++u) {
+            const int j = j1 - u;
+            if (j >= 0) {
+                base[(size_t)j * 128 * 256] = cur;
+                cur = expf(gj[u]) * cur + d[u];
+            }
+        }
+    }
+}
+
+// ---------------------------------------------------------------------------------------
+// Per chunk: dK, dV, dA (both passes) and the column-side gate scalars, from the adjoint
+// snapshot.  The intra-chunk and the inter-chunk parts of dA are kept apart (X3 / X4) so that
+// the gate kernel can pair every intra-chunk term with its row-side twin from bwd_chunk1_tc,
+// which uses bit-identical score matrices and roundings.
+__global__ void __launch_bounds__(256, 1) bwd_chunk2_tc(const __grid_constant__ CUtensorMap tq,
+                                                         const __grid_constant__ CUtensorMap tk,
+                                                         const __grid_constant__ CUtensorMap tv,
+                                                         const __grid_constant__ CUtensorMap tdo,
+                                                         const __grid_constant__ CUtensorMap to2,
+                                                         const __grid_constant__ CUtensorMap tdo1,
+                                                         const __grid_constant__ CUtensorMap tsa,
+                                                         TcBwdArgs a) {
+    const Shape s = a.s;
+    const int cg = blockIdx.x, bh = blockIdx.y, b = bh / s.H, h = bh % s.H;
+    const int nct = s.T / CT, t0 = cg * CT;
+    const int tid = threadIdx.x;
+    const Role ro;
+    const int row = ro.row, hf = ro.hf;
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                               ~uintptr_t(1023));
+    uint64_t* bars = reinterpret_cast<uint64_t*>(smem);   // tma0..tma3, mma
+    uint32_t* s_taddr = reinterpret_cast<uint32_t*>(smem + 64);
+    float* s_g2 = reinterpret_cast<float*>(smem + 128);
+    float* s_red = s_g2 + 128;
+    uint8_t* T_A = smem + 2048;       // write vectors a (fp16)
+    uint8_t* T_AS = T_A + 1 * TILE;   // write vectors scaled by gamma^C / gamma^s
+    uint8_t* T_S = T_A + 2 * TILE;    // staging
+    uint8_t* L1 = T_A + 3 * TILE;     // dO, then Q
+    uint8_t* L2 = T_A + 4 * TILE;     // V (-> V->), then K (-> K->)
+    uint8_t* L3 = T_A + 5 * TILE;     // O'', then dO'
+    uint8_t* L4 = T_A + 6 * TILE;     // D^V, then D^K
+    if (tid == 0) {
+        for (int i = 0; i < 5; ++i) mbar_init(&bars[i], 1);
+        fence_mbar_init();
+    }
+    if (ro.warp == 0) tmem_alloc(s_taddr, 512);
+    float lam, beta, g;
+    load_gates_row(s, a, b, h, t0, row, lam, beta, g);
+    const float g2 = g * LOG2E;
+    if (hf == 0) s_g2[row] = g2;
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t taddr = *s_taddr;
+    const uint32_t tl = taddr + ((uint32_t)(32 * ro.q) << 16);
+    const uint32_t X1 = 64 * hf, X2 = 128 + 64 * hf, X3 = 256 + 64 * hf, X4 = 384 + 64 * hf;
+    const int rowtok = b * s.T + t0, rowbh = bh * s.T + t0;
+    const int snap_row = (bh * nct + cg) * 2 * 128;
+    if (tid == 0) {
+        mbar_expect_tx(&bars[0], 4 * TILE);
+        tma_load_3d(L1, &tdo, 0, h, rowtok, &bars[0]);
+        tma_load_3d(L1 + TILE / 2, &tdo, 64, h, rowtok, &bars[0]);
+        tma_load_3d(L2, &tv, 0, h, rowtok, &bars[0]);
+        tma_load_3d(L2 + TILE / 2, &tv, 64, h, rowtok, &bars[0]);
+        tma_load_2d(L3, &to2, 0, rowbh, &bars[0]);
+        tma_load_2d(L3 + TILE / 2, &to2, 64, rowbh, &bars[0]);
+        tma_load_2d(L4, &tsa, 0, snap_row + 128, &bars[0]);
+        tma_load_2d(L4 + TILE / 2, &tsa, 64, snap_row + 128, &bars[0]);
+    }
+    const float g2C = cum128(s, a.g, b, h, t0, t0 + CT - 1) * LOG2E;
+    const float fw = ex2(g2C - g2);
+    write_vector_half<__half>(T_A, row, hf, lam, beta);
+    write_vector_half<__half>(T_AS, row, hf, lam, beta * fw);
+    bool ok = true;
+    uint32_t mma_ph = 0;
+    auto publish = [&]() {
+        fence_async_smem();
+        tc_fence_before();
+        ok = __syncthreads_and(ok);
+        tc_fence_after();
+    };
+    auto wait_mma = [&]() {
+        if (ok) ok = mbar_wait(&bars[4], mma_ph);
+        mma_ph ^= 1;
+        tc_fence_after();
+    };
+    auto issuer = [&]() { return tid == 0 && ok; };
+    auto mask_scores = [&](float (&x)[64], float mul) {
+#pragma unroll
+        for (int grp = 0; grp < 2; ++grp) {
+            const int sg = 2 * hf + grp;
+            if (sg > ro.q) {
+#pragma unroll
+                for (int i = 0; i < 32; ++i) x[32 * grp + i] = 0.f;
+            } else {
+#pragma unroll
+                for (int i = 0; i < 32; ++i) {
+                    const int t = 32 * sg + i;
+                    x[32 * grp + i] = (t <= row) ? mul * x[32 * grp + i] * ex2(g2 - s_g2[t]) : 0.f;
+                }
+            }
+        }
+    };
+    auto row_sum = [&](float v) {
+        s_red[128 * hf + row] = v;
+        __syncthreads();
+        const float t = s_red[row] + s_red[128 + row];
+        __syncthreads();
+        return t;
+    };
+    const uint32_t id_kk = idesc_f16(128, 128, 0, 0), id_kn = idesc_f16(128, 128, 0, 1),
+                   id_nn = idesc_f16(128, 128, 1, 1);
+    const uint32_t uA = smem_u32(T_A), uAS = smem_u32(T_AS), uS = smem_u32(T_S),
+                   u1 = smem_u32(L1), u2 = smem_u32(L2), u3 = smem_u32(L3), u4 = smem_u32(L4);
+    const float scale = s.scale;
+    const size_t gi = ((size_t)b * s.T + t0 + row) * s.H + h;
+    float av[64];   // the fp16 write vector entries of this token (as the MMAs see them)
+    write_vector_vals(av, hf, lam, beta);
+#pragma unroll
+    for (int i = 0; i < 64; ++i) av[i] = round16<__half>((av[i]));
+    float cG = 0.f;
+    ok = mbar_wait(&bars[0], 0);
+    if (ok) {   // dO and V: bf16 -> fp16
+        bf16_to_f16_half(L1, row, hf);
+        bf16_to_f16_half(L2, row, hf);
+    }
+    publish();
+    if (issuer()) {   // X1 = dO V^T
+        {
+#pragma unroll
+            for (int k = 0; k < 8; ++k)
+                mma_bf16(taddr + 0, kmajor_desc(u1, 128, k), kmajor_desc(u2, 128, k), id_kk, k > 0);
+            mma_commit(&bars[4]);
+        }
+    }
+    wait_mma();
+    {   // P4 = (dO V^T) o Gamma ; V -> V-> (rows scaled by gamma^C / gamma^s)
+        float x[64];
+        tmem_ld64(tl + X1, x);
+        mask_scores(x, 1.f);
+        store_half_bf16<__half>(T_S, row, hf, x);
+        if (ok) scale_half_smem(L2, row, hf, fw);
+    }
+    publish();
+    if (issuer()) {   // X3 = P4^T O'' ; X4 = V-> D^V^T ; X1 = O'' A^T
+#pragma unroll
+        for (int k = 0; k < 8; ++k) {
+            mma_bf16(taddr + 256, mnmajor_desc(uS, 128, k), mnmajor_desc(u3, 128, k), id_nn, k > 0);
+            mma_bf16(taddr + 384, kmajor_desc(u2, 128, k), kmajor_desc(u4, 128, k), id_kk, k > 0);
+            mma_bf16(taddr + 0, kmajor_desc(u3, 128, k), kmajor_desc(uA, 128, k), id_kk, k > 0);
+        }
+        mma_commit(&bars[4]);
+    }
+    wait_mma();
+    if (issuer()) {   // V and O'' are consumed: K, dO'
+        mbar_expect_tx(&bars[1], TILE);
+        tma_load_3d(L2, &tk, 0, h, rowtok, &bars[1]);
+        tma_load_3d(L2 + TILE / 2, &tk, 64, h, rowtok, &bars[1]);
+        mbar_expect_tx(&bars[2], TILE);
+        tma_load_2d(L3, &tdo1, 0, rowbh, &bars[2]);
+        tma_load_2d(L3 + TILE / 2, &tdo1, 64, rowbh, &bars[2]);
+    }
+    {   // <a, (P4^T O'')_t> ; P2 = (O'' A^T) o Gamma
+        float x[64];
+        tmem_ld64(tl + X3, x);
+        cG = dot64(av, x);
+        tmem_ld64(tl + X1, x);
+        mask_scores(x, 1.f);
+        store_half_bf16<__half>(T_S, row, hf, x);
+    }
+    publish();
+    if (issuer()) {   // X2 = P2^T dO + A-> D^V  (dv)
+#pragma unroll
+        for (int k = 0; k < 8; ++k)
+            mma_bf16(taddr + 128, mnmajor_desc(uS, 128, k), mnmajor_desc(u1, 128, k), id_nn, k > 0);
+#pragma unroll
+        for (int k = 0; k < 8; ++k)
+            mma_bf16(taddr + 128, kmajor_desc(uAS, 128, k), mnmajor_desc(u4, 128, k), id_kn, 1u);
+        mma_commit(&bars[4]);
+    }
+    wait_mma();
+    if (issuer()) {   // dO and D^V are consumed: Q, D^K
+        mbar_expect_tx(&bars[3], 2 * TILE);
+        tma_load_3d(L1, &tq, 0, h, rowtok, &bars[3]);
+        tma_load_3d(L1 + TILE / 2, &tq, 64, h, rowtok, &bars[3]);
+        tma_load_2d(L4, &tsa, 0, snap_row, &bars[3]);
+        tma_load_2d(L4 + TILE / 2, &tsa, 64, snap_row, &bars[3]);
+    }
+    if (ok) {   // dv
+        float x[64];
+        tmem_ld64(tl + X2, x);
+        store_global_half(static_cast<__nv_bfloat16*>(a.dv) + gi * 128 + 64 * hf, x);
+    }
+    publish();
+    if (issuer()) {   // X1 = dO' A^T
+        ok = mbar_wait(&bars[2], 0);
+        if (ok) {
+            tc_fence_after();
+#pragma unroll
+            for (int k = 0; k < 8; ++k)
+                mma_bf16(taddr + 0, kmajor_desc(u3, 128, k), kmajor_desc(uA, 128, k), id_kk, k > 0);
+            mma_commit(&bars[4]);
+        }
+    }
+    wait_mma();
+    {   // P3 = s (dO' A^T) o Gamma (the s of q~ = s q folded in, exactly as bwd_chunk1_tc does)
+        float x[64];
+        tmem_ld64(tl + X1, x);
+        mask_scores(x, scale);
+        store_half_bf16<__half>(T_S, row, hf, x);
+        if (ok) ok = mbar_wait(&bars[3], 0) && mbar_wait(&bars[1], 0);
+        if (ok) {   // Q and K: bf16 -> fp16
+            bf16_to_f16_half(L1, row, hf);
+            bf16_to_f16_half(L2, row, hf);
+        }
+    }
+    publish();
+    if (issuer()) {   // X2 = P3^T Q (intra part of dk) ;  X1 = Q K^T
+        {
+#pragma unroll
+            for (int k = 0; k < 8; ++k) {
+                mma_bf16(taddr + 128, mnmajor_desc(uS, 128, k), mnmajor_desc(u1, 128, k), id_nn, k > 0);
+                mma_bf16(taddr + 0, kmajor_desc(u1, 128, k), kmajor_desc(u2, 128, k), id_kk, k > 0);
+            }
+            mma_commit(&bars[4]);
+        }
+    }
+    wait_mma();
+    {   // <k, (P3^T Q)_t> ; P1 = s (Q K^T) o Gamma ; K -> K->
+        float x[64], kv[64];
+        tmem_ld64(tl + X2, x);
+        load_half_smem(L2, row, hf, kv);
+        cG += dot64(kv, x);
+        tmem_ld64(tl + X1, x);
+        mask_scores(x, scale);
+        store_half_bf16<__half>(T_S, row, hf, x);
+        __syncthreads();   // the Q K^T product has read K; rows are rescaled in place below
+        if (ok) scale_half_smem(L2, row, hf, fw);
+    }
+    publish();
+    if (issuer()) {   // X1 = A-> D^K (inter part of dk) ; X3 += P1^T dO' ; X4 += K-> D^K^T
+#pragma unroll
+        for (int k = 0; k < 8; ++k) {
+            mma_bf16(taddr + 0, kmajor_desc(uAS, 128, k), mnmajor_desc(u4, 128, k), id_kn, k > 0);
+            mma_bf16(taddr + 256, mnmajor_desc(uS, 128, k), mnmajor_desc(u3, 128, k), id_nn, 1u);
+            mma_bf16(taddr + 384, kmajor_desc(u2, 128, k), kmajor_desc(u4, 128, k), id_kk, 1u);
+        }
+        mma_commit(&bars[4]);
+    }
+    wait_mma();
+    float cIG = 0.f, cL = 0.f, cIL = 0.f, db = 0.f;
+    if (ok) {
+        float x[64], y[64];
+        tmem_ld64(tl + X2, x);          // dk = P3^T Q + A-> D^K
+        tmem_ld64(tl + X1, y);
+#pragma unroll
+        for (int i = 0; i < 64; ++i) x[i] += y[i];
+        store_global_half(static_cast<__nv_bfloat16*>(a.dk) + gi * 128 + 64 * hf, x);
+        tmem_ld64(tl + X3, x);          // intra-chunk da (both passes)
+        tmem_ld64(tl + X4, y);          // inter-chunk da (both passes)
+        cL = -omega_dot_half(x, av, hf);
+        cIG = dot64(av, y);
+        cIL = -omega_dot_half(y, av, hf);
+        float af[64];
+        write_vector_vals(af, hf, lam, beta);
+#pragma unroll
+        for (int i = 0; i < 64; ++i) x[i] += y[i];
+        db = dot64(x, af);
+    }
+    {
+        const float vG = row_sum(cG), vL = row_sum(cL), vIG = row_sum(cIG), vIL = row_sum(cIL);
+        const float vB = row_sum(db);
+        if (hf == 0 && ok) {
+            const size_t BTH = (size_t)s.B * s.T * s.H;
+            a.tok[2 * BTH + gi] = vG;
+            a.tok[3 * BTH + gi] = vL;
+            a.tok[4 * BTH + gi] = vB / beta;
+            a.tok[5 * BTH + gi] = vIG;
+            a.tok[6 * BTH + gi] = vIL;
+        }
+    }
+    ok = __syncthreads_and(ok);
+    if (!ok && tid == 0) {
+        flag_error(CYFA_ERR_TIMEOUT);
+        for (int i = 0; i < 4; ++i) mbar_wait(&bars[i], 0);
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (ro.warp == 0) tmem_dealloc(taddr, 512);
+}
+
+// Gate gradients of one chunk: chunk-local suffix sums of the per-token scalars plus the
+// state-level term of everything after the chunk, then the activation derivatives.
+__global__ void __launch_bounds__(128) tc_gate_kernel(TcBwdArgs a) {
+    const Shape s = a.s;
+    const int cg = blockIdx.x, bh = blockIdx.y, b = bh / s.H, h = bh % s.H;
+    const int nct = s.T / CT, tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const size_t BTH = (size_t)s.B * s.T * s.H;
+    const size_t gi = ((size_t)b * s.T + cg * CT + tid) * s.H + h;
+    // row side (bwd_chunk1_tc) minus intra-chunk column side (bwd_chunk2_tc): suffix sums;
+    // inter-chunk column side: prefix sums over the earlier tokens of the chunk
+    const float xg = a.tok[gi] - a.tok[2 * BTH + gi];
+    const float xl = a.tok[BTH + gi] + a.tok[3 * BTH + gi];
+    const float pg = a.tok[5 * BTH + gi];
+    const float pl = a.tok[6 * BTH + gi];
+    float sg = xg, sl = xl;   // inclusive suffix
+    float qg = pg, ql = pl;   // inclusive prefix
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const float yg = __shfl_down_sync(0xffffffffu, sg, o);
+        const float yl = __shfl_down_sync(0xffffffffu, sl, o);
+        const float ug = __shfl_up_sync(0xffffffffu, qg, o);
+        const float ul = __shfl_up_sync(0xffffffffu, ql, o);
+        if (lane + o < 32) {
+            sg += yg;
+            sl += yl;
+        }
+        if (lane >= o) {
+            qg += ug;
+            ql += ul;
+        }
+    }
+    __shared__ float s_w[4][4];
+    __shared__ double s_dA[4];
+    if (lane == 0) {
+        s_w[0][warp] = sg;
+        s_w[1][warp] = sl;
+    }
+    if (lane == 31) {
+        s_w[2][warp] = qg;
+        s_w[3][warp] = ql;
+    }
+    __syncthreads();
+    for (int w = warp + 1; w < 4; ++w) {
+        sg += s_w[0][w];
+        sl += s_w[1][w];
+    }
+    for (int w = 0; w < warp; ++w) {
+        qg += s_w[2][w];
+        ql += s_w[3][w];
+    }
+    qg -= pg;   // exclusive prefix: tokens before this one
+    ql -= pl;
+    const float* bd = a.bnd + ((size_t)bh * nct + cg) * 2;
+    const float dlogalpha = sg + qg + bd[0];
+    const float ddelta = sl - ql + bd[1];
+    const float f = a.decay_logit[gi];
+    a.d_decay[gi] = dlogalpha * (-a.A[h] * sigmoidf_(f));
+    const float delta = sigmoidf_(a.clock_logit[gi]);
+    a.d_clock[gi] = ddelta * delta * (1.f - delta);
+    const float bt = a.beta[gi];
+    a.d_beta[gi] = a.tok[4 * BTH + gi] * bt * (1.f - bt);
+    double da = (double)dlogalpha * (double)(-softplusf_(f));
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) da += __shfl_xor_sync(0xffffffffu, da, o);
+    if (lane == 0) s_dA[warp] = da;
+    __syncthreads();
+    if (tid == 0) a.dA_part[(size_t)bh * nct + cg] = s_dA[0] + s_dA[1] + s_dA[2] + s_dA[3];
+}
+
+__global__ void tc_dA_kernel(TcBwdArgs a) {
+    const int h = blockIdx.x * blockDim.x + threadIdx.x;
+    if (h >= a.s.H) return;
+    const int nct = a.s.T / CT;
+    double t = 0.0;
+    for (int b = 0; b < a.s.B; ++b)
+        for (int c = 0; c < nct; ++c) t += a.dA_part[((size_t)b * a.s.H + h) * nct + c];
+    a.dA[h] = (float)t;
+}
+
+}  // namespace
+
+cudaError_t launch_bwd_tc(const TcBwdArgs& a, const TcFwdArgs& f, const void* q, const void* k,
+                          const void* v, const void* dO, const float* Mf, cudaStream_t st) {
+    const Shape& s = a.s;
+    const int nct = s.T / CT;
+    const unsigned long long BH = (unsigned long long)s.B * s.H;
+    CUtensorMap mq, mk, mv, mdo, mm, msf, msa, mo2, mdo1;
+    if (!tc_qkv_maps(s, q, k, v, &mq, &mk, &mv) || !tc_qkv_maps(s, dO, nullptr, nullptr, &mdo, nullptr, nullptr) ||
+        !tc_rows_map(&mm, a.Mb, (unsigned long long)s.H * 128, true) ||
+        !tc_rows_map(&msf, a.snapF, BH * nct * 2 * 128, true) ||
+        !tc_rows_map(&msa, a.snapA, BH * nct * 2 * 128, true) ||
+        !tc_rows_map(&mo2, a.O2, BH * s.T, true) || !tc_rows_map(&mdo1, a.DO1, BH * s.T, true))
+        return cudaErrorInvalidValue;
+    cudaError_t e = launch_fwd_segment_states(f, k, v, Mf, st, true);
+    if (e != cudaSuccess) return e;
+    const dim3 gseg(a.nseg, s.B * s.H), gchunk(nct, s.B * s.H);
+    const int sm_walk6 = 1024 + 6 * TILE + 1024, sm_walk4 = 1024 + 4 * TILE + 1024;
+    const int sm_chunk = 2048 + 7 * TILE + 1024;
+    cudaFuncSetAttribute(snap_fwd_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, sm_walk6);
+    { LaunchScope ls_("tc_snap_fwd", st); snap_fwd_tc<<<gseg, 256, sm_walk6, st>>>(mk, mv, a); }
+    cudaFuncSetAttribute(bwd_chunk1_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, sm_chunk);
+    { LaunchScope ls_("tc_bwd_chunk1", st); bwd_chunk1_tc<<<gchunk, 256, sm_chunk, st>>>(mq, mk, mv, mdo, mm, msf, a); }
+    cudaFuncSetAttribute(adj_walk_tc<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, sm_walk4);
+    { LaunchScope ls_("tc_adj_segment", st); adj_walk_tc<false><<<gseg, 256, sm_walk4, st>>>(mdo1, mo2, mq, mdo, a); }
+    { LaunchScope ls_("tc_adj_scan", st); seg_scan_rev_kernel<<<dim3(128, s.B * s.H), 256, 0, st>>>(a); }
+    cudaFuncSetAttribute(adj_walk_tc<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, sm_walk4);
+    { LaunchScope ls_("tc_snap_adj", st); adj_walk_tc<true><<<gseg, 256, sm_walk4, st>>>(mdo1, mo2, mq, mdo, a); }
+    cudaFuncSetAttribute(bwd_chunk2_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, sm_chunk);
+    { LaunchScope ls_("tc_bwd_chunk2", st); bwd_chunk2_tc<<<gchunk, 256, sm_chunk, st>>>(mq, mk, mv, mdo, mo2, mdo1, msa, a); }
+    { LaunchScope ls_("tc_gate", st); tc_gate_kernel<<<gchunk, 128, 0, st>>>(a); }
+    if (a.dA) { LaunchScope ls_("tc_dA", st); tc_dA_kernel<<<(s.H + 127) / 128, 128, 0, st>>>(a); }
+    return cudaGetLastError();
+}
+
+cudaError_t tc_bwd_read_error(cudaStream_t st, int* err) {
+    cudaError_t e = cudaMemcpyFromSymbolAsync(err, g_tc_err, sizeof(int), 0,
+                                              cudaMemcpyDeviceToHost, st);
+    if (e != cudaSuccess) return e;
+    e = cudaStreamSynchronize(st);
+    if (e != cudaSuccess) return e;
+    if (*err) {
+        int zero = 0;
+        e = cudaMemcpyToSymbol(g_tc_err, &zero, sizeof(int));
+    }
+    return e;
+}
+
+}  // namespace cyfa

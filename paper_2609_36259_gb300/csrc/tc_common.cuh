@@ -14,8 +14,11 @@
 
 #include <cuda.h>
 #include <cuda_bf16.h>
+#include <cuda_fp16.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
+
+#include <type_traits>
 
 namespace cyfa {
 namespace tc {
@@ -172,6 +175,15 @@ __host__ __device__ constexpr uint32_t idesc_bf16(int M, int N, int a_mn, int b_
     return (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)a_mn << 15) | ((uint32_t)b_mn << 16) |
            ((uint32_t)(N >> 3) << 17) | ((uint32_t)(M >> 4) << 24);
 }
+// Same with fp16 A and B (operand format 0).
+__host__ __device__ constexpr uint32_t idesc_f16(int M, int N, int a_mn, int b_mn) {
+    return (1u << 4) | ((uint32_t)a_mn << 15) | ((uint32_t)b_mn << 16) |
+           ((uint32_t)(N >> 3) << 17) | ((uint32_t)(M >> 4) << 24);
+}
+template <typename OT>
+__host__ __device__ constexpr uint32_t idesc_k16(int M, int N, int a_mn, int b_mn) {
+    return std::is_same<OT, __half>::value ? idesc_f16(M, N, a_mn, b_mn) : idesc_bf16(M, N, a_mn, b_mn);
+}
 
 // Descriptor of K-step k (16 bf16) of a K-major tile of `rows` rows at smem address base.
 __device__ __forceinline__ uint64_t kmajor_desc(uint32_t base, int rows, int k) {
@@ -191,6 +203,21 @@ __device__ __forceinline__ uint32_t swz_off(int row, int col, int rows) {
 __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
     __nv_bfloat162 p = __floats2bfloat162_rn(lo, hi);
     return *reinterpret_cast<uint32_t*>(&p);
+}
+__device__ __forceinline__ uint32_t pack_f16(float lo, float hi) {
+    __half2 p = __floats2half2_rn(lo, hi);
+    return *reinterpret_cast<uint32_t*>(&p);
+}
+// Two 16-bit operands of type OT (__nv_bfloat16 or __half) packed into 32 bits.
+template <typename OT>
+__device__ __forceinline__ uint32_t pack2(float lo, float hi) {
+    if constexpr (std::is_same<OT, __half>::value) return pack_f16(lo, hi);
+    else return pack_bf16(lo, hi);
+}
+template <typename OT>
+__device__ __forceinline__ float round16(float x) {
+    if constexpr (std::is_same<OT, __half>::value) return __half2float(__float2half_rn(x));
+    else return __bfloat162float(__float2bfloat16_rn(x));
 }
 
 }  // namespace tc

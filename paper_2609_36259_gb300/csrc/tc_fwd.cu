@@ -11,10 +11,7 @@
 //                  (Sec. 3.3 Eq. cyfa-two-pass) on the tensor cores, then advances the state.
 // States never round-trip through HBM at chunk granularity.  All operand tiles are 128 x 128 bf16
 // in 128-byte-swizzled shared memory; accumulators are fp32 in TMEM.
-#include "../../include/cyfa.h"
-#include "common.cuh"
-#include "kernels.h"
-#include "tc_common.cuh"
+#include "tc_chunk.cuh"
 
 namespace cyfa {
 
@@ -22,161 +19,8 @@ namespace {
 
 using namespace tc;
 
-constexpr int CT = 128;              // tokens per chunk on this path
-constexpr int TILE = CT * 128 * 2;   // one 128 x 128 bf16 tile (32 KiB)
-constexpr float LOG2E = 1.4426950408889634f;
-
-static __device__ int g_tc_err;
-
-__device__ __forceinline__ void flag_error(int code) { atomicExch(&g_tc_err, code); }
-
-__device__ __forceinline__ float ex2(float x) {
-    float y;
-    asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
-    return y;
-}
-
-// g_cum of token t rebased to the start of its 128-token chunk t0 (g_cum is local to s.Cg).
-__device__ __forceinline__ float cum128(const Shape& s, const float* g, int b, int h, int t0,
-                                       int t) {
-    float v = g[((size_t)b * s.T + t) * s.H + h];
-    if (s.Cg == 64 && t - t0 >= 64) v += g[((size_t)b * s.T + t0 + 63) * s.H + h];
-    return v;
-}
-
-// Order of the 128 Fourier-axis rows inside the tensor-core kernels.  Column half hf (0 or 1)
-// holds the pairs j = 32 hf + jj + 1 (jj < 32): cosine entry at 64 hf + jj, sine entry at
-// 64 hf + jj + 32, so every rotation block of U lies inside one half.  The DC entry sits at 95
-// and the padding entry at 127.  Exported / imported states use the paper's order
-// [DC, cos_1, sin_1, ..., cos_63, sin_63, pad]; these map between the two.
-__host__ __device__ __forceinline__ int tc_slot(int p) {
-    if (p == 0) return 95;
-    if (p == 127) return 127;
-    const int j = (p + 1) >> 1, hf = (j - 1) >> 5, jj = (j - 1) & 31;
-    return 64 * hf + jj + ((p & 1) ? 0 : 32);
-}
-__host__ __device__ __forceinline__ int paper_slot(int t) {
-    if (t == 95) return 0;
-    if (t == 127) return 127;
-    const int hf = t >> 6, l = t & 63, jj = l & 31;
-    const int j = 32 * hf + jj + 1;
-    return (l >= 32) ? 2 * j : 2 * j - 1;
-}
-
-// Rotation angles theta_j = 2 pi j lam / m for the 32 pairs of one column half, produced in
-// order by angle addition from theta_1 (cos(x + y) = cos x cos y - sin x sin y,
-// sin(x + y) = sin x cos y + cos x sin y), re-seeded from sincospif every 16 steps.
-struct HalfAngles {
-    float c1, s1, c, s, lam;
-    int j0;
-    __device__ __forceinline__ HalfAngles(float lam_, int hf) : lam(lam_), j0(32 * hf + 1) {
-        sincospif(phase_pi(lam, 1), &s1, &c1);
-        if (j0 == 1) {
-            c = c1;
-            s = s1;
-        } else {
-            sincospif(phase_pi(lam, j0), &s, &c);
-        }
-    }
-    // advance to local pair jj (1..31)
-    __device__ __forceinline__ void step(int jj) {
-        if (jj == 16) {
-            sincospif(phase_pi(lam, j0 + 16), &s, &c);
-        } else {
-            const float cn = c * c1 - s * s1;
-            const float sn = s * c1 + c * s1;
-            c = cn;
-            s = sn;
-        }
-    }
-};
-
-// Store 64 fp32 values as bf16 into columns [64 hf, 64 hf + 64) of row r of a swizzled tile.
-__device__ __forceinline__ void store_half_bf16(uint8_t* tile, int r, int hf, const float (&x)[64]) {
-#pragma unroll
-    for (int q = 0; q < 8; ++q) {
-        uint4 u;
-        u.x = pack_bf16(x[8 * q + 0], x[8 * q + 1]);
-        u.y = pack_bf16(x[8 * q + 2], x[8 * q + 3]);
-        u.z = pack_bf16(x[8 * q + 4], x[8 * q + 5]);
-        u.w = pack_bf16(x[8 * q + 6], x[8 * q + 7]);
-        *reinterpret_cast<uint4*>(tile + swz_off(r, 64 * hf + 8 * q, 128)) = u;
-    }
-}
-
-// One column half of the temporal write vector w U(-lam) b of a token (Sec. 3.2, b of
-// Eq. app-b-explicit), in the tensor-core row order.
-__device__ __forceinline__ void write_vector_half(uint8_t* tile, int r, int hf, float lam, float w) {
-    float x[64];
-    HalfAngles ang(lam, hf);
-    const float wa = w * SQRT_2_OVER_M;
-#pragma unroll
-    for (int jj = 0; jj < 32; ++jj) {
-        if (jj > 0) ang.step(jj);
-        x[jj] = wa * ang.c;
-        x[jj + 32] = -wa * ang.s;
-    }
-    if (hf == 1) {
-        x[31] = w * INV_SQRT_M;
-        x[63] = 0.f;
-    }
-    store_half_bf16(tile, r, hf, x);
-}
-
-// x <- U(sign lam) x on one column half (tensor-core row order); DC kept, padding zeroed.
-template <int SIGN>
-__device__ __forceinline__ void rotate_half(float (&x)[64], int hf, float lam) {
-    HalfAngles ang(lam, hf);
-    const float dc = x[31];
-#pragma unroll
-    for (int jj = 0; jj < 32; ++jj) {
-        if (jj > 0) ang.step(jj);
-        const float c = ang.c, s = SIGN * ang.s;
-        const float xc = x[jj], xs = x[jj + 32];
-        x[jj] = c * xc - s * xs;
-        x[jj + 32] = s * xc + c * xs;
-    }
-    if (hf == 1) {
-        x[31] = dc;
-        x[63] = 0.f;
-    }
-}
-
-__device__ __forceinline__ void tmem_ld64(uint32_t taddr, float (&x)[64]) {
-    float v[32];
-    tmem_ld32(taddr, v);
-#pragma unroll
-    for (int i = 0; i < 32; ++i) x[i] = v[i];
-    tmem_ld32(taddr + 32, v);
-#pragma unroll
-    for (int i = 0; i < 32; ++i) x[32 + i] = v[i];
-}
-__device__ __forceinline__ void tmem_st64(uint32_t taddr, const float (&x)[64]) {
-    float v[32];
-#pragma unroll
-    for (int i = 0; i < 32; ++i) v[i] = x[i];
-    tmem_st32(taddr, v);
-#pragma unroll
-    for (int i = 0; i < 32; ++i) v[i] = x[32 + i];
-    tmem_st32(taddr + 32, v);
-}
-
-// Lane quarter / column half owned by this thread in the 256-thread tensor-core kernels:
-// warps w and w + 4 share TMEM lanes 32 (w % 4) .. + 31 (one row each per thread) and split the
-// 128 columns of a tile into halves hf = w / 4.
-struct Role {
-    int warp, lane, q, hf, row;
-    __device__ __forceinline__ Role() {
-        warp = threadIdx.x >> 5;
-        lane = threadIdx.x & 31;
-        q = warp & 3;
-        hf = warp >> 2;
-        row = 32 * q + lane;
-    }
-};
-
 // ---------------------------------------------------------------------------------------
-template <int SEGC>
+template <int SEGC, typename OT>
 __global__ void __launch_bounds__(256, 1) seg_state_tc(const __grid_constant__ CUtensorMap tk,
                                                         const __grid_constant__ CUtensorMap tv,
                                                         TcFwdArgs a) {
@@ -230,7 +74,8 @@ __global__ void __launch_bounds__(256, 1) seg_state_tc(const __grid_constant__ C
     if (tid == 0) issue_kv(0, 0);
     __syncthreads();
     bool ok = true;
-    const uint32_t idesc = idesc_bf16(128, 128, 1, 1);
+    constexpr bool F16 = std::is_same<OT, __half>::value;
+    const uint32_t idesc = idesc_k16<OT>(128, 128, 1, 1);
     for (int c = 0; c < nc; ++c) {
         const int buf = c & 1;
         if (c >= 1 && ok) ok = mbar_wait(&bars[2 + ((c - 1) & 1)], ((c - 1) >> 1) & 1);
@@ -241,13 +86,20 @@ __global__ void __launch_bounds__(256, 1) seg_state_tc(const __grid_constant__ C
             const size_t gi = ((size_t)b * s.T + t) * s.H + h;
             const float w = a.beta[gi] *
                             ex2((s_tot[c] - cum128(s, a.g, b, h, t0, t) + s_sfx[c]) * LOG2E);
-            write_vector_half(tiles + 3 * buf * TILE, ro.row, ro.hf, a.lam[gi], w);
+            write_vector_half<OT>(tiles + 3 * buf * TILE, ro.row, ro.hf, a.lam[gi], w);
+        }
+        if (F16) {   // the bf16 K and V tiles become fp16 operands
+            if (ok) ok = mbar_wait(&bars[buf], (c >> 1) & 1);
+            if (ok) {
+                bf16_to_f16_half(tiles + (3 * buf + 1) * TILE, ro.row, ro.hf);
+                bf16_to_f16_half(tiles + (3 * buf + 2) * TILE, ro.row, ro.hf);
+            }
         }
         fence_async_smem();
         ok = __syncthreads_and(ok);
         if (!ok) break;
         if (tid == 0) {
-            if (mbar_wait(&bars[buf], (c >> 1) & 1)) {
+            if (F16 || mbar_wait(&bars[buf], (c >> 1) & 1)) {
                 tc_fence_after();
                 const uint32_t tA = smem_u32(tiles + 3 * buf * TILE);
                 const uint32_t tK = smem_u32(tiles + (3 * buf + 1) * TILE);
@@ -645,15 +497,17 @@ __global__ void __launch_bounds__(256, 1) seg_out_tc(const __grid_constant__ CUt
     if (ro.warp == 0) tmem_dealloc(taddr, 512);
 }
 
-// M (fp32, paper order) -> bf16 with its Fourier (column) index in the tensor-core order.
-__global__ void m_to_bf16_kernel(const float* M, __nv_bfloat16* Mb, int H) {
+// M (fp32, paper order) -> 16-bit OT with its Fourier (column) index in the tensor-core order.
+template <typename OT>
+__global__ void m_to_k16_kernel(const float* M, OT* Mb, int H) {
     const int i = blockIdx.x * blockDim.x + threadIdx.x;
     if (i >= H * 128 * 128) return;
     const int p = i & 127, rest = i >> 7;
-    Mb[rest * 128 + tc_slot(p)] = __float2bfloat16_rn(M[i]);
+    if constexpr (std::is_same<OT, __half>::value) Mb[rest * 128 + tc_slot(p)] = __float2half_rn(M[i]);
+    else Mb[rest * 128 + tc_slot(p)] = __float2bfloat16_rn(M[i]);
 }
 
-constexpr int SEGC_DEFAULT = 8;    // 1024-token segments
+constexpr int SEGC_DEFAULT = TC_SEGC;
 
 }  // namespace
 
@@ -664,32 +518,56 @@ int tc_fwd_segments(const Shape& s) {
 
 bool tc_fwd_supported(const Shape& s) { return s.bf16 && s.D == 128 && s.T % CT == 0; }
 
-cudaError_t launch_fwd_tc(const TcFwdArgs& a, const void* q, const void* k, const void* v,
-                          const float* Mf, cudaStream_t st) {
-    const Shape& s = a.s;
-    CUtensorMap mq, mk, mv, mm;
+bool tc_qkv_maps(const Shape& s, const void* q, const void* k, const void* v, CUtensorMap* mq,
+                 CUtensorMap* mk, CUtensorMap* mv) {
     const unsigned long long dims[3] = {128ull, (unsigned long long)s.H,
                                         (unsigned long long)s.B * s.T};
     const unsigned long long strides[2] = {128ull * 2, (unsigned long long)s.H * 128 * 2};
     const unsigned box[3] = {64, 1, CT};
-    const unsigned long long mdims[2] = {128ull, (unsigned long long)s.H * 128};
-    const unsigned long long mstr[1] = {256ull};
-    const unsigned mbox[2] = {64, 128};
-    if (!make_tmap_bf16(&mq, q, 3, dims, strides, box) || !make_tmap_bf16(&mk, k, 3, dims, strides, box) ||
-        !make_tmap_bf16(&mv, v, 3, dims, strides, box) ||
-        !make_tmap_bf16(&mm, a.Mb, 2, mdims, mstr, mbox))
-        return cudaErrorInvalidValue;
+    return (!mq || make_tmap_bf16(mq, q, 3, dims, strides, box)) &&
+           (!mk || make_tmap_bf16(mk, k, 3, dims, strides, box)) &&
+           (!mv || make_tmap_bf16(mv, v, 3, dims, strides, box));
+}
+
+bool tc_rows_map(CUtensorMap* map, const void* base, unsigned long long rows, bool f16) {
+    const unsigned long long dims[2] = {128ull, rows};
+    const unsigned long long str[1] = {256ull};
+    const unsigned box[2] = {64, 128};
+    return make_tmap_bf16(map, base, 2, dims, str, box, f16);
+}
+
+cudaError_t launch_fwd_segment_states(const TcFwdArgs& a, const void* k, const void* v,
+                                      const float* Mf, cudaStream_t st, bool f16) {
+    const Shape& s = a.s;
+    CUtensorMap mk, mv;
+    if (!tc_qkv_maps(s, nullptr, k, v, nullptr, &mk, &mv)) return cudaErrorInvalidValue;
     const int n = s.H * 128 * 128;
     {
-        LaunchScope ls_("m_to_bf16", st);
-        m_to_bf16_kernel<<<(n + 255) / 256, 256, 0, st>>>(Mf, const_cast<__nv_bfloat16*>(a.Mb), s.H);
+        LaunchScope ls_("m_to_k16", st);
+        if (f16)
+            m_to_k16_kernel<__half><<<(n + 255) / 256, 256, 0, st>>>(Mf, (__half*)(a.Mb), s.H);
+        else
+            m_to_k16_kernel<__nv_bfloat16><<<(n + 255) / 256, 256, 0, st>>>(Mf, const_cast<__nv_bfloat16*>(a.Mb), s.H);
     }
     const dim3 grid(a.nseg, s.B * s.H);
     const int smA = 1024 + 6 * TILE + 1024;
-    auto kA = seg_state_tc<SEGC_DEFAULT>;
+    auto kA = f16 ? seg_state_tc<SEGC_DEFAULT, __half> : seg_state_tc<SEGC_DEFAULT, __nv_bfloat16>;
     cudaFuncSetAttribute(kA, cudaFuncAttributeMaxDynamicSharedMemorySize, smA);
     { LaunchScope ls_("tc_seg_state", st); kA<<<grid, 256, smA, st>>>(mk, mv, a); }
     { LaunchScope ls_("tc_seg_scan", st); seg_scan_kernel<<<dim3(128, s.B * s.H), 256, 0, st>>>(a); }
+    return cudaGetLastError();
+}
+
+cudaError_t launch_fwd_tc(const TcFwdArgs& a, const void* q, const void* k, const void* v,
+                          const float* Mf, cudaStream_t st) {
+    const Shape& s = a.s;
+    CUtensorMap mq, mk, mv, mm;
+    if (!tc_qkv_maps(s, q, k, v, &mq, &mk, &mv) ||
+        !tc_rows_map(&mm, a.Mb, (unsigned long long)s.H * 128))
+        return cudaErrorInvalidValue;
+    cudaError_t e = launch_fwd_segment_states(a, k, v, Mf, st);
+    if (e != cudaSuccess) return e;
+    const dim3 grid(a.nseg, s.B * s.H);
     const int smC = 2048 + 7 * TILE + 1024;
     auto kC = seg_out_tc<SEGC_DEFAULT>;
     cudaFuncSetAttribute(kC, cudaFuncAttributeMaxDynamicSharedMemorySize, smC);

@@ -14,7 +14,7 @@ std::once_flag g_once;
 }  // namespace
 
 bool make_tmap_bf16(CUtensorMap* map, const void* base, int rank, const unsigned long long* dims,
-                    const unsigned long long* strides_bytes, const unsigned* box) {
+                    const unsigned long long* strides_bytes, const unsigned* box, bool f16) {
     std::call_once(g_once, [] {
         void* fn = nullptr;
         cudaDriverEntryPointQueryResult q;
@@ -32,7 +32,7 @@ bool make_tmap_bf16(CUtensorMap* map, const void* base, int rank, const unsigned
         estr[i] = 1;
         if (i + 1 < rank) gstr[i] = strides_bytes[i];
     }
-    const CUresult r = g_encode(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, (cuuint32_t)rank,
+    const CUresult r = g_encode(map, f16 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT16 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, (cuuint32_t)rank,
                                 const_cast<void*>(base), gdim, gstr, bdim, estr,
                                 CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
                                 CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);

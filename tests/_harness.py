@@ -26,6 +26,18 @@ def assert_close_bf16(got, want, what=''):
     return err, rl
 
 
+def assert_close_sum(got, want, l1, what=''):
+    """A sum over many tokens (dA = sum_t d log alpha_t * (-softplus f_t)): each of its terms
+    carries the per-token bf16 tolerance, so the sum's error is bounded by that tolerance times
+    the L1 mass of the terms (l1), not by the sum's own size, which cancellation can make small."""
+    got = np.asarray(got, dtype=np.float64)
+    want = np.asarray(want, dtype=np.float64)
+    bar = BF16_REL_L2 * np.asarray(l1, dtype=np.float64) + BF16_MAX_ABS
+    err = np.abs(got - want)
+    assert np.all(err <= bar), '%s: errors %s above bars %s' % (what, err, bar)
+    return err
+
+
 def assert_close_fp32(got, want, what=''):
     err = float(np.max(np.abs(np.asarray(got, np.float64) - np.asarray(want, np.float64))))
     assert err <= FP32_MAX_ABS, '%s: max-abs %.3e (bar %.0e)' % (what, err, FP32_MAX_ABS)

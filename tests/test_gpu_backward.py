@@ -5,7 +5,8 @@ import torch
 
 from paper_2609_36259_gb300 import cyfa, synth
 
-from _harness import (assert_close_bf16, assert_close_fp32, gpu_prepare, oracle_backward,
+from _harness import (assert_close_bf16, assert_close_fp32, assert_close_sum, gpu_prepare,
+                      oracle_backward,
                       oracle_inputs, pairs_np, sample_pairs, to_device)
 
 pytestmark = pytest.mark.gpu
@@ -35,19 +36,25 @@ def _compare(out, ref, pairs, close, what=''):
         close(pairs_np(out[gk].float(), pairs), ref[rk], '%s %s' % (what, gk))
 
 
+@pytest.mark.parametrize('cuda_cores', [False, True])
 @pytest.mark.parametrize('B,T,H,D,C', [(2, 256, 2, 128, 64), (1, 384, 3, 64, 64),
-                                       (1, 512, 2, 128, 128)])
-def test_backward_small_bf16(B, T, H, D, C):
+                                       (1, 512, 2, 128, 128), (1, 2304, 2, 128, 64)])
+def test_backward_small_bf16(B, T, H, D, C, cuda_cores):
+    """Tensor-core kernels (bf16, d = 128, T a multiple of 128) and the CUDA-core kernels;
+    T = 2304 spans several 1024-token segments plus a partial one."""
     inp = to_device(synth.make_inputs(B, T, H, D, seed=8, with_dO=True))
-    d = cyfa.dims(B, T, H, D, chunk=C)
+    d = cyfa.dims(B, T, H, D, chunk=C, cuda_cores=cuda_cores)
     out = gpu_backward(d, inp)
     pairs = [(b, h) for b in range(B) for h in range(H)]
     ref = oracle_backward(oracle_inputs(inp, pairs), pairs_np(inp['dO'], pairs))
     _compare(out, ref, pairs, assert_close_bf16)
-    dA_ref = np.zeros(H)
+    dA_ref, l1 = np.zeros(H), np.zeros(H)
+    f = pairs_np(inp['decay_logit'], pairs)
+    softplus = np.logaddexp(0.0, f)
     for n, (b, h) in enumerate(pairs):
         dA_ref[h] += ref['dA'][n]
-    assert_close_bf16(out['dA'].double().cpu().numpy(), dA_ref, 'dA')
+        l1[h] += np.abs(ref['d_logalpha'][n] * softplus[n]).sum()
+    assert_close_sum(out['dA'].double().cpu().numpy(), dA_ref, l1, 'dA')
 
 
 def test_backward_fp32():
@@ -64,12 +71,14 @@ def test_backward_fp32():
         assert err <= 1e-4 * scale, (gk, err, scale)
 
 
-@pytest.mark.parametrize('B,T,H,C', [(4, 8192, 16, 64), (2, 32768, 16, 128)])
-def test_backward_full_size_sampled(B, T, H, C):
+@pytest.mark.parametrize('B,T,H,C,cuda_cores', [(4, 8192, 16, 64, False), (4, 8192, 16, 64, True),
+                                                 (2, 32768, 16, 64, False),
+                                                 (2, 32768, 16, 128, True)])
+def test_backward_full_size_sampled(B, T, H, C, cuda_cores):
     """The B4 H16 T8192 and the 1.4B-shaped B2 H16 T32768 layers: all gradients of sampled
     (b, h) sequences against the oracle."""
     inp = synth.make_inputs(B, T, H, 128, seed=0, device='cuda', with_dO=True)
-    d = cyfa.dims(B, T, H, 128, chunk=C)
+    d = cyfa.dims(B, T, H, 128, chunk=C, cuda_cores=cuda_cores)
     out = gpu_backward(d, inp, want_dA=False)
     pairs = sample_pairs(B, H, 2)
     ref = oracle_backward(oracle_inputs(inp, pairs), pairs_np(inp['dO'], pairs))
