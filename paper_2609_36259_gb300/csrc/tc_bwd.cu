@@ -584,12 +584,16 @@ __global__ void __launch_bounds__(256, 1) bwd_chunk1_tc(const __grid_constant__ 
 // SNAP = true: walk the segment backwards from its end adjoint (segD after the reverse scan),
 // storing before each chunk the adjoint of that chunk's end state, then
 // D <- gamma^C D + sum_r gamma^r [...].  The K part (dO', q~) and the V part (o'', dO) run one
-// after the other with double-buffered tiles.
+// after the other with double-buffered tiles.  In the SNAP walk the chunk-start state S of
+// the forward (for the boundary terms of the gate gradients) arrives by TMA with the operand
+// tiles, and the adjoint snapshot leaves through the same shared tile by a TMA store.
 template <bool SNAP>
 __global__ void __launch_bounds__(256, 1) adj_walk_tc(const __grid_constant__ CUtensorMap tdo1,
                                                        const __grid_constant__ CUtensorMap to2,
                                                        const __grid_constant__ CUtensorMap tq,
                                                        const __grid_constant__ CUtensorMap tdo,
+                                                       const __grid_constant__ CUtensorMap tsf,
+                                                       const __grid_constant__ CUtensorMap tsa,
                                                        TcBwdArgs a) {
     const Shape s = a.s;
     const int seg = blockIdx.x, bh = blockIdx.y, b = bh / s.H, h = bh % s.H;
@@ -607,7 +611,8 @@ __global__ void __launch_bounds__(256, 1) adj_walk_tc(const __grid_constant__ CU
     float* s_tot = reinterpret_cast<float*>(smem + 128);   // [TC_SEGC]
     float* s_pre = s_tot + TC_SEGC;                         // [TC_SEGC]
     float* s_bnd = s_pre + TC_SEGC;                         // [TC_SEGC][2]
-    uint8_t* tiles = smem + 1024;                          // [buf][X | Y]
+    constexpr int NT = SNAP ? 3 : 2;                       // tiles per buffer
+    uint8_t* tiles = smem + 1024;                          // [buf][X | Y (| S)]
     if (tid == 0) {
         for (int i = 0; i < 4; ++i) mbar_init(&bars[i], 1);
         fence_mbar_init();
@@ -651,17 +656,23 @@ __global__ void __launch_bounds__(256, 1) adj_walk_tc(const __grid_constant__ CU
     };
     auto issue = [&](int it) {
         const int part = it / nc, c = chunk_of(it), buf = it & 1;
-        uint8_t* tX = tiles + (2 * buf) * TILE;
-        uint8_t* tY = tiles + (2 * buf + 1) * TILE;
+        uint8_t* tX = tiles + (NT * buf) * TILE;
+        uint8_t* tY = tX + TILE;
         const int t0 = (c_begin + c) * CT;
         const int xrow = bh * s.T + t0, yrow = b * s.T + t0;
         const CUtensorMap* mx = part == 0 ? &tdo1 : &to2;
         const CUtensorMap* my = part == 0 ? &tq : &tdo;
-        mbar_expect_tx(&bars[buf], 2 * TILE);
+        mbar_expect_tx(&bars[buf], NT * TILE);
         tma_load_2d(tX, mx, 0, xrow, &bars[buf]);
         tma_load_2d(tX + TILE / 2, mx, 64, xrow, &bars[buf]);
         tma_load_3d(tY, my, 0, h, yrow, &bars[buf]);
         tma_load_3d(tY + TILE / 2, my, 64, h, yrow, &bars[buf]);
+        if (SNAP) {
+            uint8_t* tS = tX + 2 * TILE;
+            const int srow = ((bh * nct + c_begin + c) * 2 + part) * 128;
+            tma_load_2d(tS, &tsf, 0, srow, &bars[buf]);
+            tma_load_2d(tS + TILE / 2, &tsf, 64, srow, &bars[buf]);
+        }
     };
     if (tid == 0) issue(0);
     tc_fence_before();
@@ -674,32 +685,31 @@ __global__ void __launch_bounds__(256, 1) adj_walk_tc(const __grid_constant__ CU
         const int cg = c_begin + c, t0 = cg * CT;
         if (it >= 1 && ok) ok = mbar_wait(&bars[2 + ((it - 1) & 1)], ((it - 1) >> 1) & 1);
         tc_fence_after();
-        if (tid == 0 && ok && it + 1 < total) issue(it + 1);
+        if (tid == 0 && ok && it + 1 < total) {
+            if (SNAP) bulk_wait_read_all();   // the other buffer's S tile may be a store's source
+            issue(it + 1);
+        }
         if (ok) ok = mbar_wait(&bars[buf], (it >> 1) & 1);
         const float g = cum128(s, a.g, b, h, t0, t0 + row);
+        uint8_t* tX = tiles + (NT * buf) * TILE;
         float w;
         if (SNAP) {
             // adjoint of this chunk's end state, then D <- gamma^C D (this part's 128 columns)
-            __half* dst = a.snapA + (((size_t)bh * nct + cg) * 2 + part) * 128 * 128 + row * 128 + 64 * hf;
+            uint8_t* tS = tX + 2 * TILE;
             const float dC = ex2(s_tot[c] * LOG2E);
             float x[64];
             tmem_ld64(tl + 128 * part + 64 * hf, x);
-            store_global_half(dst, x);
             {
                 // gamma^C <D, S> and gamma^C <D, Omega S> with S this chunk's start state (the
                 // chunk's own writes enter through the inter-chunk column terms of
                 // bwd_chunk2_tc); this thread's row and 64 columns
-                const __half* Sp = a.snapF + (((size_t)bh * nct + cg) * 2 + part) * 128 * 128;
                 const int l = row & 63, jj = l & 31, j = 32 * (row >> 6) + jj + 1;
                 const bool paired = j <= NPAIR;
                 const int partner = (l >= 32) ? row - 32 : row + 32;
                 const float f = paired ? ((l >= 32) ? 1.f : -1.f) * 6.283185307179586f * (float)j / 127.f : 0.f;
                 float sr[64], sp[64];
-#pragma unroll
-                for (int q2 = 0; q2 < 8; ++q2) {
-                    unpack8(*reinterpret_cast<const uint4*>(Sp + row * 128 + 64 * hf + 8 * q2), sr + 8 * q2);
-                    unpack8(*reinterpret_cast<const uint4*>(Sp + (paired ? partner : row) * 128 + 64 * hf + 8 * q2), sp + 8 * q2);
-                }
+                load_half_smem(tS, row, hf, sr);
+                load_half_smem(tS, paired ? partner : row, hf, sp);
                 float bG = dC * dot64(x, sr), bL = dC * f * dot64(x, sp);
                 bG = warp_sum(bG);
                 bL = warp_sum(bL);
@@ -708,6 +718,8 @@ __global__ void __launch_bounds__(256, 1) adj_walk_tc(const __grid_constant__ CU
                     atomicAdd(&s_bnd[2 * c + 1], bL);
                 }
             }
+            __syncthreads();   // the S tile is read: it now stages the snapshot for its TMA store
+            store_half_bf16<__half>(tS, row, hf, x);
 #pragma unroll
             for (int i = 0; i < 64; ++i) x[i] *= dC;
             tmem_st64(tl + 128 * part + 64 * hf, x);
@@ -717,8 +729,8 @@ __global__ void __launch_bounds__(256, 1) adj_walk_tc(const __grid_constant__ CU
         }
         if (part == 0) w *= s.scale;   // q~ = s q
         if (ok) {
-            scale_half_smem(tiles + (2 * buf) * TILE, row, hf, w);
-            bf16_to_f16_half(tiles + (2 * buf + 1) * TILE, row, hf);   // q or dO
+            scale_half_smem(tX, row, hf, w);
+            bf16_to_f16_half(tX + TILE, row, hf);   // q or dO
         }
         fence_async_smem();
         tc_fence_before();
@@ -726,12 +738,18 @@ __global__ void __launch_bounds__(256, 1) adj_walk_tc(const __grid_constant__ CU
         tc_fence_after();
         if (!ok) break;
         if (tid == 0) {
-            const uint32_t tX = smem_u32(tiles + (2 * buf) * TILE);
-            const uint32_t tY = smem_u32(tiles + (2 * buf + 1) * TILE);
+            if (SNAP) {
+                const int arow = ((bh * nct + cg) * 2 + part) * 128;
+                tma_store_2d(&tsa, tX + 2 * TILE, 0, arow);
+                tma_store_2d(&tsa, tX + 2 * TILE + TILE / 2, 64, arow);
+                bulk_commit();
+            }
+            const uint32_t uX = smem_u32(tX);
+            const uint32_t uY = smem_u32(tX + TILE);
             const bool first = !SNAP && (it % nc) == 0;
 #pragma unroll
             for (int k = 0; k < 8; ++k)
-                mma_bf16(taddr + 128 * part, mnmajor_desc(tX, 128, k), mnmajor_desc(tY, 128, k),
+                mma_bf16(taddr + 128 * part, mnmajor_desc(uX, 128, k), mnmajor_desc(uY, 128, k),
                          id_nn, (first && k == 0) ? 0u : 1u);
             mma_commit(&bars[2 + buf]);
         }
@@ -759,6 +777,7 @@ __global__ void __launch_bounds__(256, 1) adj_walk_tc(const __grid_constant__ CU
         flag_error(CYFA_ERR_TIMEOUT);
         for (int i = 0; i < 2; ++i) mbar_wait(&bars[i], 0);
     }
+    if (SNAP && tid == 0) bulk_wait_all();
     tc_fence_before();
     __syncthreads();
     if (ro.warp == 0) tmem_dealloc(taddr, 256);
@@ -1142,14 +1161,25 @@ __global__ void __launch_bounds__(128) tc_gate_kernel(TcBwdArgs a) {
     if (tid == 0) a.dA_part[(size_t)bh * nct + cg] = s_dA[0] + s_dA[1] + s_dA[2] + s_dA[3];
 }
 
-__global__ void tc_dA_kernel(TcBwdArgs a) {
-    const int h = blockIdx.x * blockDim.x + threadIdx.x;
-    if (h >= a.s.H) return;
-    const int nct = a.s.T / CT;
+// dA[h] = sum over batch rows and chunks of the per-chunk partials; one block per head.
+__global__ void __launch_bounds__(256) tc_dA_kernel(TcBwdArgs a) {
+    const int h = blockIdx.x, tid = threadIdx.x;
+    const int nct = a.s.T / CT, n = a.s.B * nct;
     double t = 0.0;
-    for (int b = 0; b < a.s.B; ++b)
-        for (int c = 0; c < nct; ++c) t += a.dA_part[((size_t)b * a.s.H + h) * nct + c];
-    a.dA[h] = (float)t;
+    for (int i = tid; i < n; i += 256) {
+        const int b = i / nct, c = i - b * nct;
+        t += a.dA_part[((size_t)b * a.s.H + h) * nct + c];
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) t += __shfl_xor_sync(0xffffffffu, t, o);
+    __shared__ double s_t[8];
+    if ((tid & 31) == 0) s_t[tid >> 5] = t;
+    __syncthreads();
+    if (tid == 0) {
+        double r = 0.0;
+        for (int w = 0; w < 8; ++w) r += s_t[w];
+        a.dA[h] = (float)r;
+    }
 }
 
 }  // namespace
@@ -1176,14 +1206,14 @@ cudaError_t launch_bwd_tc(const TcBwdArgs& a, const TcFwdArgs& f, const void* q,
     cudaFuncSetAttribute(bwd_chunk1_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, sm_chunk);
     { LaunchScope ls_("tc_bwd_chunk1", st); bwd_chunk1_tc<<<gchunk, 256, sm_chunk, st>>>(mq, mk, mv, mdo, mm, msf, a); }
     cudaFuncSetAttribute(adj_walk_tc<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, sm_walk4);
-    { LaunchScope ls_("tc_adj_segment", st); adj_walk_tc<false><<<gseg, 256, sm_walk4, st>>>(mdo1, mo2, mq, mdo, a); }
+    { LaunchScope ls_("tc_adj_segment", st); adj_walk_tc<false><<<gseg, 256, sm_walk4, st>>>(mdo1, mo2, mq, mdo, msf, msa, a); }
     { LaunchScope ls_("tc_adj_scan", st); seg_scan_rev_kernel<<<dim3(128, s.B * s.H), 256, 0, st>>>(a); }
-    cudaFuncSetAttribute(adj_walk_tc<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, sm_walk4);
-    { LaunchScope ls_("tc_snap_adj", st); adj_walk_tc<true><<<gseg, 256, sm_walk4, st>>>(mdo1, mo2, mq, mdo, a); }
+    cudaFuncSetAttribute(adj_walk_tc<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, sm_walk6);
+    { LaunchScope ls_("tc_snap_adj", st); adj_walk_tc<true><<<gseg, 256, sm_walk6, st>>>(mdo1, mo2, mq, mdo, msf, msa, a); }
     cudaFuncSetAttribute(bwd_chunk2_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, sm_chunk);
     { LaunchScope ls_("tc_bwd_chunk2", st); bwd_chunk2_tc<<<gchunk, 256, sm_chunk, st>>>(mq, mk, mv, mdo, mo2, mdo1, msa, a); }
     { LaunchScope ls_("tc_gate", st); tc_gate_kernel<<<gchunk, 128, 0, st>>>(a); }
-    if (a.dA) { LaunchScope ls_("tc_dA", st); tc_dA_kernel<<<(s.H + 127) / 128, 128, 0, st>>>(a); }
+    if (a.dA) { LaunchScope ls_("tc_dA", st); tc_dA_kernel<<<s.H, 256, 0, st>>>(a); }
     return cudaGetLastError();
 }
 
