@@ -241,7 +241,8 @@ __global__ void __launch_bounds__(256, 1) snap_fwd_tc(const __grid_constant__ CU
 
 // ---------------------------------------------------------------------------------------
 // Per chunk: recompute O', O''; dO''; middle-readout gradient; dO'; dq; per-token scalars.
-__global__ void __launch_bounds__(256, 1) bwd_chunk1_tc(const __grid_constant__ CUtensorMap tq,
+// 512 threads: one row and one column quarter each (QRole).
+__global__ void __launch_bounds__(512, 1) bwd_chunk1_tc(const __grid_constant__ CUtensorMap tq,
                                                          const __grid_constant__ CUtensorMap tk,
                                                          const __grid_constant__ CUtensorMap tv,
                                                          const __grid_constant__ CUtensorMap tdo,
@@ -252,37 +253,36 @@ __global__ void __launch_bounds__(256, 1) bwd_chunk1_tc(const __grid_constant__ 
     const int cg = blockIdx.x, bh = blockIdx.y, b = bh / s.H, h = bh % s.H;
     const int nct = s.T / CT, t0 = cg * CT;
     const int tid = threadIdx.x;
-    const Role ro;
-    const int row = ro.row, hf = ro.hf;
+    const QRole ro;
+    const int row = ro.row, hf = ro.hf, u = ro.u, c0 = ro.c0, cq = ro.cq;
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                                ~uintptr_t(1023));
     uint64_t* bars = reinterpret_cast<uint64_t*>(smem);            // tma0, tma1, mma
     uint32_t* s_taddr = reinterpret_cast<uint32_t*>(smem + 32);
-    float* s_g2 = reinterpret_cast<float*>(smem + 64);
-    float* s_red = s_g2 + 128;                                      // [2][128]
-    uint8_t* T_K = smem + 2048;       // V (first), then K
+    float* s_g2 = reinterpret_cast<float*>(smem + 64);              // [128]
+    float* s_red = s_g2 + 128;                                      // [2][4][128]
+    uint8_t* T_K = smem + 5120;       // V (first), then K
     uint8_t* T_KB = T_K + 1 * TILE;   // Kbar snapshot (rows = slots)
     uint8_t* T_A = T_K + 2 * TILE;    // write vectors (rows = tokens)
     uint8_t* T_M = T_K + 3 * TILE;    // M = R Phi
-    uint8_t* T_S = T_K + 4 * TILE;    // staging
+    uint8_t* T_S = T_K + 4 * TILE;    // Vbar snapshot (first), then staging
     uint8_t* T_L1 = T_K + 5 * TILE;   // dO, then Q
-    uint8_t* T_L2 = T_K + 6 * TILE;   // Vbar snapshot
     if (tid == 0) {
         for (int i = 0; i < 3; ++i) mbar_init(&bars[i], 1);
         fence_mbar_init();
     }
     if (ro.warp == 0) tmem_alloc(s_taddr, 512);
-    float lam, beta, g;
-    load_gates_row(s, a, b, h, t0, row, lam, beta, g);
-    const float g2 = g * LOG2E;
-    if (hf == 0) s_g2[row] = g2;
+    const size_t gi = ((size_t)b * s.T + t0 + row) * s.H + h;
+    const float lam = a.lam[gi], beta = a.beta[gi];
+    const float g2 = cum128(s, a.g, b, h, t0, t0 + row) * LOG2E;
+    if (cq == 0) s_g2[row] = g2;
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
     const uint32_t taddr = *s_taddr;
-    const uint32_t tl = taddr + ((uint32_t)(32 * ro.q) << 16);
-    const uint32_t X1 = 64 * hf, X2 = 128 + 64 * hf, X3 = 256 + 64 * hf, X4 = 384 + 64 * hf;
+    const uint32_t tl = taddr + ((uint32_t)(32 * ro.q) << 16) + c0;
+    const uint32_t X1 = 0, X2 = 128, X3 = 256, X4 = 384;
     const int rowtok = b * s.T + t0;
     const int snap_row = (bh * nct + cg) * 2 * 128;
     if (tid == 0) {
@@ -291,18 +291,18 @@ __global__ void __launch_bounds__(256, 1) bwd_chunk1_tc(const __grid_constant__ 
         tma_load_3d(T_L1 + TILE / 2, &tdo, 64, h, rowtok, &bars[0]);
         tma_load_3d(T_K, &tv, 0, h, rowtok, &bars[0]);
         tma_load_3d(T_K + TILE / 2, &tv, 64, h, rowtok, &bars[0]);
-        tma_load_2d(T_L2, &tsf, 0, snap_row + 128, &bars[0]);
-        tma_load_2d(T_L2 + TILE / 2, &tsf, 64, snap_row + 128, &bars[0]);
+        tma_load_2d(T_S, &tsf, 0, snap_row + 128, &bars[0]);
+        tma_load_2d(T_S + TILE / 2, &tsf, 64, snap_row + 128, &bars[0]);
         tma_load_2d(T_KB, &tsf, 0, snap_row, &bars[0]);
         tma_load_2d(T_KB + TILE / 2, &tsf, 64, snap_row, &bars[0]);
         tma_load_2d(T_M, &tm, 0, h * 128, &bars[0]);
         tma_load_2d(T_M + TILE / 2, &tm, 64, h * 128, &bars[0]);
     }
-    write_vector_half<__half>(T_A, row, hf, lam, beta);
+    write_vector_q<__half>(T_A, row, hf, u, lam, beta);
     bool ok = mbar_wait(&bars[0], 0);
     if (ok) {   // dO and V: bf16 -> fp16
-        bf16_to_f16_half(T_L1, row, hf);
-        bf16_to_f16_half(T_K, row, hf);
+        bf16_to_f16_q(T_L1, row, c0);
+        bf16_to_f16_q(T_K, row, c0);
     }
     uint32_t mma_ph = 0;
     auto publish = [&]() {
@@ -317,47 +317,48 @@ __global__ void __launch_bounds__(256, 1) bwd_chunk1_tc(const __grid_constant__ 
         tc_fence_after();
     };
     auto issuer = [&]() { return tid == 0 && ok; };
-    auto mask_scores = [&](float (&x)[64], float mul) {
+    // x o Gamma (times mul) with the causal mask; columns are tokens of this chunk
+    auto mask_scores = [&](float (&x)[32], float mul) {
 #pragma unroll
-        for (int grp = 0; grp < 2; ++grp) {
-            const int sg = 2 * hf + grp;
-            if (sg > ro.q) {
+        for (int blk = 0; blk < 2; ++blk) {
+            const int tb = c0 + 32 * blk;
+            if (tb >= 32 * (ro.q + 1)) {   // every token of the block is after every row of the warp
 #pragma unroll
-                for (int i = 0; i < 32; ++i) x[32 * grp + i] = 0.f;
+                for (int i = 0; i < 16; ++i) x[16 * blk + i] = 0.f;
             } else {
 #pragma unroll
-                for (int i = 0; i < 32; ++i) {
-                    const int t = 32 * sg + i;
-                    x[32 * grp + i] = (t <= row) ? mul * x[32 * grp + i] * ex2(g2 - s_g2[t]) : 0.f;
+                for (int i = 0; i < 16; ++i) {
+                    const int t = tb + i;
+                    x[16 * blk + i] = (t <= row) ? mul * x[16 * blk + i] * ex2(g2 - s_g2[t]) : 0.f;
                 }
             }
         }
     };
-    // sum of a per-thread partial over the two column halves of this row
-    auto row_sum = [&](float v) {
-        s_red[128 * hf + row] = v;
+    // sum / max of a per-thread partial over the four column quarters of this row (the same
+    // order on every quarter, so all four get bit-identical results)
+    int red_buf = 0;
+    auto row_reduce = [&](float v, bool is_max) {
+        float* r = s_red + 512 * red_buf;
+        red_buf ^= 1;
+        r[128 * cq + row] = v;
         __syncthreads();
-        const float t = s_red[row] + s_red[128 + row];
-        __syncthreads();
-        return t;
+        return is_max ? fmaxf(fmaxf(r[row], r[128 + row]), fmaxf(r[256 + row], r[384 + row]))
+                      : (r[row] + r[128 + row]) + (r[256 + row] + r[384 + row]);
     };
     const uint32_t id_kk = idesc_f16(128, 128, 0, 0), id_kn = idesc_f16(128, 128, 0, 1);
     const uint32_t uK = smem_u32(T_K), uKB = smem_u32(T_KB), uA = smem_u32(T_A), uM = smem_u32(T_M),
-                   uS = smem_u32(T_S), uL1 = smem_u32(T_L1), uL2 = smem_u32(T_L2);
+                   uS = smem_u32(T_S), uL1 = smem_u32(T_L1);
     const float scale = s.scale;
     const float gam = ex2(g2);
     float s1 = 0.f, s2 = 0.f, s3 = 0.f, s4 = 0.f;
     publish();
-    // G1: X1 = dO V^T, X2 = dO Vbar^T
-    if (issuer()) {
-        {
+    if (issuer()) {   // G1: X1 = dO V^T, X2 = dO Vbar^T
 #pragma unroll
-            for (int k = 0; k < 8; ++k) {
-                mma_bf16(taddr + 0, kmajor_desc(uL1, 128, k), kmajor_desc(uK, 128, k), id_kk, k > 0);
-                mma_bf16(taddr + 128, kmajor_desc(uL1, 128, k), kmajor_desc(uL2, 128, k), id_kk, k > 0);
-            }
-            mma_commit(&bars[2]);
+        for (int k = 0; k < 8; ++k) {
+            mma_bf16(taddr + X1, kmajor_desc(uL1, 128, k), kmajor_desc(uK, 128, k), id_kk, k > 0);
+            mma_bf16(taddr + X2, kmajor_desc(uL1, 128, k), kmajor_desc(uS, 128, k), id_kk, k > 0);
         }
+        mma_commit(&bars[2]);
     }
     wait_mma();
     if (issuer()) {   // dO and V are consumed: Q and K
@@ -368,200 +369,193 @@ __global__ void __launch_bounds__(256, 1) bwd_chunk1_tc(const __grid_constant__ 
         tma_load_3d(T_K + TILE / 2, &tk, 64, h, rowtok, &bars[1]);
     }
     {   // P4 = (dO V^T) o Gamma
-        float x[64];
-        tmem_ld64(tl + X1, x);
+        float x[32];
+        tmem_ld16x2(tl + X1, x);
         mask_scores(x, 1.f);
-        store_half_bf16<__half>(T_S, row, hf, x);
+        store_q<__half>(T_S, row, c0, x);
     }
     publish();
     if (issuer()) {   // G2: X3 = P4 A
 #pragma unroll
         for (int k = 0; k < 8; ++k)
-            mma_bf16(taddr + 256, kmajor_desc(uS, 128, k), mnmajor_desc(uA, 128, k), id_kn, k > 0);
+            mma_bf16(taddr + X3, kmajor_desc(uS, 128, k), mnmajor_desc(uA, 128, k), id_kn, k > 0);
         mma_commit(&bars[2]);
     }
     wait_mma();
     {   // do'' = gamma (dO Vbar^T) + P4 A, kept in X2
-        float x[64], y[64];
-        tmem_ld64(tl + X2, x);
-        tmem_ld64(tl + X3, y);
+        float x[32], y[32];
+        tmem_ld16x2(tl + X2, x);
+        tmem_ld16x2(tl + X3, y);
 #pragma unroll
-        for (int i = 0; i < 64; ++i) x[i] = fmaf(gam, x[i], y[i]);
-        tmem_st64(tl + X2, x);
+        for (int i = 0; i < 32; ++i) x[i] = fmaf(gam, x[i], y[i]);
+        tmem_st16x2(tl + X2, x);
         if (ok) ok = mbar_wait(&bars[1], 0);
         if (ok) {   // Q and K: bf16 -> fp16
-            bf16_to_f16_half(T_L1, row, hf);
-            bf16_to_f16_half(T_K, row, hf);
+            bf16_to_f16_q(T_L1, row, c0);
+            bf16_to_f16_q(T_K, row, c0);
         }
     }
     publish();
     if (issuer()) {   // G3: X1 = Q K^T, X3 = Q Kbar^T
-        {
 #pragma unroll
-            for (int k = 0; k < 8; ++k) {
-                mma_bf16(taddr + 0, kmajor_desc(uL1, 128, k), kmajor_desc(uK, 128, k), id_kk, k > 0);
-                mma_bf16(taddr + 256, kmajor_desc(uL1, 128, k), kmajor_desc(uKB, 128, k), id_kk, k > 0);
-            }
-            mma_commit(&bars[2]);
+        for (int k = 0; k < 8; ++k) {
+            mma_bf16(taddr + X1, kmajor_desc(uL1, 128, k), kmajor_desc(uK, 128, k), id_kk, k > 0);
+            mma_bf16(taddr + X3, kmajor_desc(uL1, 128, k), kmajor_desc(uKB, 128, k), id_kk, k > 0);
         }
+        mma_commit(&bars[2]);
     }
     wait_mma();
     {   // P1 = s (Q K^T) o Gamma
-        float x[64];
-        tmem_ld64(tl + X1, x);
+        float x[32];
+        tmem_ld16x2(tl + X1, x);
         mask_scores(x, scale);
-        store_half_bf16<__half>(T_S, row, hf, x);
+        store_q<__half>(T_S, row, c0, x);
     }
     publish();
     if (issuer()) {   // G4: X4 = P1 A
 #pragma unroll
         for (int k = 0; k < 8; ++k)
-            mma_bf16(taddr + 384, kmajor_desc(uS, 128, k), mnmajor_desc(uA, 128, k), id_kn, k > 0);
+            mma_bf16(taddr + X4, kmajor_desc(uS, 128, k), mnmajor_desc(uA, 128, k), id_kn, k > 0);
         mma_commit(&bars[2]);
     }
     wait_mma();
     {   // z = U(lam) o', kept in X3
-        float x[64], y[64];
-        tmem_ld64(tl + X3, x);
-        tmem_ld64(tl + X4, y);
+        float x[32], y[32];
+        tmem_ld16x2(tl + X3, x);
+        tmem_ld16x2(tl + X4, y);
         const float f = scale * gam;
 #pragma unroll
-        for (int i = 0; i < 64; ++i) x[i] = fmaf(f, x[i], y[i]);
-        rotate_half<1>(x, hf, lam);
-        store_half_bf16<__half>(T_S, row, hf, x);
-        tmem_st64(tl + X3, x);
+        for (int i = 0; i < 32; ++i) x[i] = fmaf(f, x[i], y[i]);
+        rotate_q<1>(x, hf, u, lam);
+        store_q<__half>(T_S, row, c0, x);
+        tmem_st16x2(tl + X3, x);
     }
     publish();
     if (issuer()) {   // G5: X1 = z M^T
 #pragma unroll
         for (int k = 0; k < 8; ++k)
-            mma_bf16(taddr + 0, kmajor_desc(uS, 128, k), kmajor_desc(uM, 128, k), id_kk, k > 0);
+            mma_bf16(taddr + X1, kmajor_desc(uS, 128, k), kmajor_desc(uM, 128, k), id_kk, k > 0);
         mma_commit(&bars[2]);
     }
     wait_mma();
-    {   // p = softmax(l), kept in X1
-        float x[64];
-        tmem_ld64(tl + X1, x);
-        const int nvalid = hf ? 63 : 64;
+    {   // p = softmax(l) over the m valid entries (the padding column is out), kept in X1
+        float x[32];
+        tmem_ld16x2(tl + X1, x);
+        const bool pad = (hf == 1 && u == 1);
         float mx = -INFINITY;
 #pragma unroll
-        for (int i = 0; i < 64; ++i)
-            if (i < nvalid) mx = fmaxf(mx, x[i]);
-        s_red[128 * hf + row] = mx;
-        __syncthreads();
-        mx = fmaxf(s_red[row], s_red[128 + row]);
-        __syncthreads();
+        for (int i = 0; i < 32; ++i)
+            if (!(pad && i == 31)) mx = fmaxf(mx, x[i]);
+        mx = row_reduce(mx, true);
         float sum = 0.f;
 #pragma unroll
-        for (int i = 0; i < 64; ++i) {
-            x[i] = (i < nvalid) ? ex2((x[i] - mx) * LOG2E) : 0.f;
+        for (int i = 0; i < 32; ++i) {
+            x[i] = (pad && i == 31) ? 0.f : ex2((x[i] - mx) * LOG2E);
             sum += x[i];
         }
-        const float inv = 1.f / row_sum(sum);
+        const float inv = 1.f / row_reduce(sum, false);
 #pragma unroll
-        for (int i = 0; i < 64; ++i) x[i] *= inv;
-        store_half_bf16<__half>(T_S, row, hf, x);
-        tmem_st64(tl + X1, x);
+        for (int i = 0; i < 32; ++i) x[i] *= inv;
+        store_q<__half>(T_S, row, c0, x);
+        tmem_st16x2(tl + X1, x);
     }
     publish();
     if (issuer()) {   // G6: X4 = p M
 #pragma unroll
         for (int k = 0; k < 8; ++k)
-            mma_bf16(taddr + 384, kmajor_desc(uS, 128, k), mnmajor_desc(uM, 128, k), id_kn, k > 0);
+            mma_bf16(taddr + X4, kmajor_desc(uS, 128, k), mnmajor_desc(uM, 128, k), id_kn, k > 0);
         mma_commit(&bars[2]);
     }
     wait_mma();
-    {   // o'' = U(-lam) (p M); scalars with do'' (o'' as stored in bf16); dy = U(lam) do''
-        float o2[64], g2v[64];
-        tmem_ld64(tl + X4, o2);
-        rotate_half<-1>(o2, hf, lam);
-        store_global_half(a.O2 + ((size_t)bh * s.T + t0 + row) * 128 + 64 * hf, o2);
+    {   // o'' = U(-lam) (p M); scalars with do'' (o'' as stored in fp16); dy = U(lam) do''
+        float o2[32], g2v[32];
+        tmem_ld16x2(tl + X4, o2);
+        rotate_q<-1>(o2, hf, u, lam);
+        store_global_q(a.O2 + ((size_t)bh * s.T + t0 + row) * 128, c0, o2);
 #pragma unroll
-        for (int i = 0; i < 64; ++i) o2[i] = round16<__half>((o2[i]));
-        tmem_ld64(tl + X2, g2v);
-        s1 = dot64(o2, g2v);
-        s2 = omega_dot_half(o2, g2v, hf);   // <o'', Omega do''> = -<do'', Omega o''>
-        rotate_half<1>(g2v, hf, lam);
-        store_half_bf16<__half>(T_S, row, hf, g2v);
+        for (int i = 0; i < 32; ++i) o2[i] = round16<__half>(o2[i]);
+        tmem_ld16x2(tl + X2, g2v);
+        s1 = dot32(o2, g2v);
+        s2 = omega_dot_q(o2, g2v, hf, u);   // <o'', Omega do''> = -<do'', Omega o''>
+        rotate_q<1>(g2v, hf, u, lam);
+        store_q<__half>(T_S, row, c0, g2v);
     }
     publish();
     if (issuer()) {   // G7: X4 = dy M^T = M dy
 #pragma unroll
         for (int k = 0; k < 8; ++k)
-            mma_bf16(taddr + 384, kmajor_desc(uS, 128, k), kmajor_desc(uM, 128, k), id_kk, k > 0);
+            mma_bf16(taddr + X4, kmajor_desc(uS, 128, k), kmajor_desc(uM, 128, k), id_kk, k > 0);
         mma_commit(&bars[2]);
     }
     wait_mma();
     {   // dl = p o (dp - <p, dp>)
-        float p[64], dp[64];
-        tmem_ld64(tl + X1, p);
-        tmem_ld64(tl + X4, dp);
-        const float pdp = row_sum(dot64(p, dp));
+        float p[32], dp[32];
+        tmem_ld16x2(tl + X1, p);
+        tmem_ld16x2(tl + X4, dp);
+        const float pdp = row_reduce(dot32(p, dp), false);
 #pragma unroll
-        for (int i = 0; i < 64; ++i) p[i] = p[i] * (dp[i] - pdp);
-        store_half_bf16<__half>(T_S, row, hf, p);
+        for (int i = 0; i < 32; ++i) p[i] = p[i] * (dp[i] - pdp);
+        store_q<__half>(T_S, row, c0, p);
     }
     publish();
     if (issuer()) {   // G8: X2 = dl M = M^T dl
 #pragma unroll
         for (int k = 0; k < 8; ++k)
-            mma_bf16(taddr + 128, kmajor_desc(uS, 128, k), mnmajor_desc(uM, 128, k), id_kn, k > 0);
+            mma_bf16(taddr + X2, kmajor_desc(uS, 128, k), mnmajor_desc(uM, 128, k), id_kn, k > 0);
         mma_commit(&bars[2]);
     }
     wait_mma();
-    {   // do' = U(-lam) dz; <do', Omega o'> with do' as stored in bf16 (= <dz, Omega z> exactly)
-        float dz[64], z[64];
-        tmem_ld64(tl + X2, dz);
-        tmem_ld64(tl + X3, z);
-        rotate_half<-1>(dz, hf, lam);
-        store_half_bf16<__half>(T_S, row, hf, dz);
-        store_global_half(a.DO1 + ((size_t)bh * s.T + t0 + row) * 128 + 64 * hf, dz);
-        rotate_half<-1>(z, hf, lam);   // o'
+    {   // do' = U(-lam) dz; <do', Omega o'> with do' as stored in fp16 (= <dz, Omega z> exactly)
+        float dz[32], z[32];
+        tmem_ld16x2(tl + X2, dz);
+        tmem_ld16x2(tl + X3, z);
+        rotate_q<-1>(dz, hf, u, lam);
+        store_q<__half>(T_S, row, c0, dz);
+        store_global_q(a.DO1 + ((size_t)bh * s.T + t0 + row) * 128, c0, dz);
+        rotate_q<-1>(z, hf, u, lam);   // o'
 #pragma unroll
-        for (int i = 0; i < 64; ++i) dz[i] = round16<__half>((dz[i]));
-        s3 = omega_dot_half(dz, z, hf);
+        for (int i = 0; i < 32; ++i) dz[i] = round16<__half>(dz[i]);
+        s3 = omega_dot_q(dz, z, hf, u);
     }
     publish();
     if (issuer()) {   // G9: X1 = dO' A^T, X3 = dO' Kbar
 #pragma unroll
         for (int k = 0; k < 8; ++k) {
-            mma_bf16(taddr + 0, kmajor_desc(uS, 128, k), kmajor_desc(uA, 128, k), id_kk, k > 0);
-            mma_bf16(taddr + 256, kmajor_desc(uS, 128, k), mnmajor_desc(uKB, 128, k), id_kn, k > 0);
+            mma_bf16(taddr + X1, kmajor_desc(uS, 128, k), kmajor_desc(uA, 128, k), id_kk, k > 0);
+            mma_bf16(taddr + X3, kmajor_desc(uS, 128, k), mnmajor_desc(uKB, 128, k), id_kn, k > 0);
         }
         mma_commit(&bars[2]);
     }
     wait_mma();
     {   // P3 = s (dO' A^T) o Gamma
-        float x[64];
-        tmem_ld64(tl + X1, x);
+        float x[32];
+        tmem_ld16x2(tl + X1, x);
         mask_scores(x, scale);
-        store_half_bf16<__half>(T_S, row, hf, x);
+        store_q<__half>(T_S, row, c0, x);
     }
     publish();
     if (issuer()) {   // G10: X4 = P3 K
 #pragma unroll
         for (int k = 0; k < 8; ++k)
-            mma_bf16(taddr + 384, kmajor_desc(uS, 128, k), mnmajor_desc(uK, 128, k), id_kn, k > 0);
+            mma_bf16(taddr + X4, kmajor_desc(uS, 128, k), mnmajor_desc(uK, 128, k), id_kn, k > 0);
         mma_commit(&bars[2]);
     }
     wait_mma();
     if (ok) {   // dq = s gamma (dO' Kbar) + P3 K  (P3 carries s) ; <q, dq> = <q~, dq~>
-        float x[64], y[64], qv[64];
-        tmem_ld64(tl + X3, x);
-        tmem_ld64(tl + X4, y);
+        float x[32], y[32];
+        tmem_ld16x2(tl + X3, x);
+        tmem_ld16x2(tl + X4, y);
         const float f = scale * gam;
 #pragma unroll
-        for (int i = 0; i < 64; ++i) x[i] = fmaf(f, x[i], y[i]);
-        load_half_smem(T_L1, row, hf, qv);
-        s4 = dot64(qv, x);
-        const size_t gi = ((size_t)b * s.T + t0 + row) * s.H + h;
-        store_global_half(static_cast<__nv_bfloat16*>(a.dq) + gi * 128 + 64 * hf, x);
+        for (int i = 0; i < 32; ++i) x[i] = fmaf(f, x[i], y[i]);
+        load_q(T_L1, row, c0, y);
+        s4 = dot32(y, x);
+        store_global_q(static_cast<__nv_bfloat16*>(a.dq) + gi * 128, c0, x);
     }
     {
-        const float dG = row_sum(s1 + s4);
-        const float dL = row_sum(s3 + s2);
-        if (hf == 0 && ok) {
-            const size_t gi = ((size_t)b * s.T + t0 + row) * s.H + h;
+        const float dG = row_reduce(s1 + s4, false);
+        const float dL = row_reduce(s3 + s2, false);
+        if (cq == 0 && ok) {
             const size_t BTH = (size_t)s.B * s.T * s.H;
             a.tok[gi] = dG;
             a.tok[BTH + gi] = dL;
@@ -813,8 +807,8 @@ __global__ void __launch_bounds__(256) seg_scan_rev_kernel(TcBwdArgs a) {
 // Per chunk: dK, dV, dA (both passes) and the column-side gate scalars, from the adjoint
 // snapshot.  The intra-chunk and the inter-chunk parts of dA are kept apart (X3 / X4) so that
 // the gate kernel can pair every intra-chunk term with its row-side twin from bwd_chunk1_tc,
-// which uses bit-identical score matrices and roundings.
-__global__ void __launch_bounds__(256, 1) bwd_chunk2_tc(const __grid_constant__ CUtensorMap tq,
+// which uses bit-identical score matrices and roundings.  512 threads (QRole).
+__global__ void __launch_bounds__(512, 1) bwd_chunk2_tc(const __grid_constant__ CUtensorMap tq,
                                                          const __grid_constant__ CUtensorMap tk,
                                                          const __grid_constant__ CUtensorMap tv,
                                                          const __grid_constant__ CUtensorMap tdo,
@@ -826,15 +820,14 @@ __global__ void __launch_bounds__(256, 1) bwd_chunk2_tc(const __grid_constant__ 
     const int cg = blockIdx.x, bh = blockIdx.y, b = bh / s.H, h = bh % s.H;
     const int nct = s.T / CT, t0 = cg * CT;
     const int tid = threadIdx.x;
-    const Role ro;
-    const int row = ro.row, hf = ro.hf;
+    const QRole ro;
+    const int row = ro.row, hf = ro.hf, u = ro.u, c0 = ro.c0, cq = ro.cq;
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                                ~uintptr_t(1023));
     uint64_t* bars = reinterpret_cast<uint64_t*>(smem);   // tma0..tma3, mma
     uint32_t* s_taddr = reinterpret_cast<uint32_t*>(smem + 64);
     float* s_g2 = reinterpret_cast<float*>(smem + 128);
-    float* s_red = s_g2 + 128;
     uint8_t* T_A = smem + 2048;       // write vectors a (fp16)
     uint8_t* T_AS = T_A + 1 * TILE;   // write vectors scaled by gamma^C / gamma^s
     uint8_t* T_S = T_A + 2 * TILE;    // staging
@@ -847,16 +840,16 @@ __global__ void __launch_bounds__(256, 1) bwd_chunk2_tc(const __grid_constant__ 
         fence_mbar_init();
     }
     if (ro.warp == 0) tmem_alloc(s_taddr, 512);
-    float lam, beta, g;
-    load_gates_row(s, a, b, h, t0, row, lam, beta, g);
-    const float g2 = g * LOG2E;
-    if (hf == 0) s_g2[row] = g2;
+    const size_t gi = ((size_t)b * s.T + t0 + row) * s.H + h;
+    const float lam = a.lam[gi], beta = a.beta[gi];
+    const float g2 = cum128(s, a.g, b, h, t0, t0 + row) * LOG2E;
+    if (cq == 0) s_g2[row] = g2;
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
     const uint32_t taddr = *s_taddr;
-    const uint32_t tl = taddr + ((uint32_t)(32 * ro.q) << 16);
-    const uint32_t X1 = 64 * hf, X2 = 128 + 64 * hf, X3 = 256 + 64 * hf, X4 = 384 + 64 * hf;
+    const uint32_t tl = taddr + ((uint32_t)(32 * ro.q) << 16) + c0;
+    const uint32_t X1 = 0, X2 = 128, X3 = 256, X4 = 384;
     const int rowtok = b * s.T + t0, rowbh = bh * s.T + t0;
     const int snap_row = (bh * nct + cg) * 2 * 128;
     if (tid == 0) {
@@ -872,10 +865,14 @@ __global__ void __launch_bounds__(256, 1) bwd_chunk2_tc(const __grid_constant__ 
     }
     const float g2C = cum128(s, a.g, b, h, t0, t0 + CT - 1) * LOG2E;
     const float fw = ex2(g2C - g2);
-    write_vector_half<__half>(T_A, row, hf, lam, beta);
-    write_vector_half<__half>(T_AS, row, hf, lam, beta * fw);
-    bool ok = true;
+    write_vector_q<__half>(T_A, row, hf, u, lam, beta);
+    write_vector_q<__half>(T_AS, row, hf, u, lam, beta * fw);
     uint32_t mma_ph = 0;
+    bool ok = mbar_wait(&bars[0], 0);
+    if (ok) {   // dO and V: bf16 -> fp16
+        bf16_to_f16_q(L1, row, c0);
+        bf16_to_f16_q(L2, row, c0);
+    }
     auto publish = [&]() {
         fence_async_smem();
         tc_fence_before();
@@ -888,69 +885,50 @@ __global__ void __launch_bounds__(256, 1) bwd_chunk2_tc(const __grid_constant__ 
         tc_fence_after();
     };
     auto issuer = [&]() { return tid == 0 && ok; };
-    auto mask_scores = [&](float (&x)[64], float mul) {
+    auto mask_scores = [&](float (&x)[32], float mul) {
 #pragma unroll
-        for (int grp = 0; grp < 2; ++grp) {
-            const int sg = 2 * hf + grp;
-            if (sg > ro.q) {
+        for (int blk = 0; blk < 2; ++blk) {
+            const int tb = c0 + 32 * blk;
+            if (tb >= 32 * (ro.q + 1)) {
 #pragma unroll
-                for (int i = 0; i < 32; ++i) x[32 * grp + i] = 0.f;
+                for (int i = 0; i < 16; ++i) x[16 * blk + i] = 0.f;
             } else {
 #pragma unroll
-                for (int i = 0; i < 32; ++i) {
-                    const int t = 32 * sg + i;
-                    x[32 * grp + i] = (t <= row) ? mul * x[32 * grp + i] * ex2(g2 - s_g2[t]) : 0.f;
+                for (int i = 0; i < 16; ++i) {
+                    const int t = tb + i;
+                    x[16 * blk + i] = (t <= row) ? mul * x[16 * blk + i] * ex2(g2 - s_g2[t]) : 0.f;
                 }
             }
         }
-    };
-    auto row_sum = [&](float v) {
-        s_red[128 * hf + row] = v;
-        __syncthreads();
-        const float t = s_red[row] + s_red[128 + row];
-        __syncthreads();
-        return t;
     };
     const uint32_t id_kk = idesc_f16(128, 128, 0, 0), id_kn = idesc_f16(128, 128, 0, 1),
                    id_nn = idesc_f16(128, 128, 1, 1);
     const uint32_t uA = smem_u32(T_A), uAS = smem_u32(T_AS), uS = smem_u32(T_S),
                    u1 = smem_u32(L1), u2 = smem_u32(L2), u3 = smem_u32(L3), u4 = smem_u32(L4);
     const float scale = s.scale;
-    const size_t gi = ((size_t)b * s.T + t0 + row) * s.H + h;
-    float av[64];   // the fp16 write vector entries of this token (as the MMAs see them)
-    write_vector_vals(av, hf, lam, beta);
-#pragma unroll
-    for (int i = 0; i < 64; ++i) av[i] = round16<__half>((av[i]));
     float cG = 0.f;
-    ok = mbar_wait(&bars[0], 0);
-    if (ok) {   // dO and V: bf16 -> fp16
-        bf16_to_f16_half(L1, row, hf);
-        bf16_to_f16_half(L2, row, hf);
-    }
     publish();
     if (issuer()) {   // X1 = dO V^T
-        {
 #pragma unroll
-            for (int k = 0; k < 8; ++k)
-                mma_bf16(taddr + 0, kmajor_desc(u1, 128, k), kmajor_desc(u2, 128, k), id_kk, k > 0);
-            mma_commit(&bars[4]);
-        }
+        for (int k = 0; k < 8; ++k)
+            mma_bf16(taddr + X1, kmajor_desc(u1, 128, k), kmajor_desc(u2, 128, k), id_kk, k > 0);
+        mma_commit(&bars[4]);
     }
     wait_mma();
     {   // P4 = (dO V^T) o Gamma ; V -> V-> (rows scaled by gamma^C / gamma^s)
-        float x[64];
-        tmem_ld64(tl + X1, x);
+        float x[32];
+        tmem_ld16x2(tl + X1, x);
         mask_scores(x, 1.f);
-        store_half_bf16<__half>(T_S, row, hf, x);
-        if (ok) scale_half_smem(L2, row, hf, fw);
+        store_q<__half>(T_S, row, c0, x);
+        if (ok) scale_q(L2, row, c0, fw);
     }
     publish();
     if (issuer()) {   // X3 = P4^T O'' ; X4 = V-> D^V^T ; X1 = O'' A^T
 #pragma unroll
         for (int k = 0; k < 8; ++k) {
-            mma_bf16(taddr + 256, mnmajor_desc(uS, 128, k), mnmajor_desc(u3, 128, k), id_nn, k > 0);
-            mma_bf16(taddr + 384, kmajor_desc(u2, 128, k), kmajor_desc(u4, 128, k), id_kk, k > 0);
-            mma_bf16(taddr + 0, kmajor_desc(u3, 128, k), kmajor_desc(uA, 128, k), id_kk, k > 0);
+            mma_bf16(taddr + X3, mnmajor_desc(uS, 128, k), mnmajor_desc(u3, 128, k), id_nn, k > 0);
+            mma_bf16(taddr + X4, kmajor_desc(u2, 128, k), kmajor_desc(u4, 128, k), id_kk, k > 0);
+            mma_bf16(taddr + X1, kmajor_desc(u3, 128, k), kmajor_desc(uA, 128, k), id_kk, k > 0);
         }
         mma_commit(&bars[4]);
     }
@@ -964,21 +942,22 @@ __global__ void __launch_bounds__(256, 1) bwd_chunk2_tc(const __grid_constant__ 
         tma_load_2d(L3 + TILE / 2, &tdo1, 64, rowbh, &bars[2]);
     }
     {   // <a, (P4^T O'')_t> ; P2 = (O'' A^T) o Gamma
-        float x[64];
-        tmem_ld64(tl + X3, x);
-        cG = dot64(av, x);
-        tmem_ld64(tl + X1, x);
+        float x[32], av[32];
+        tmem_ld16x2(tl + X3, x);
+        load_q(T_A, row, c0, av);   // the fp16 write vector entries, as the MMAs see them
+        cG = dot32(av, x);
+        tmem_ld16x2(tl + X1, x);
         mask_scores(x, 1.f);
-        store_half_bf16<__half>(T_S, row, hf, x);
+        store_q<__half>(T_S, row, c0, x);
     }
     publish();
     if (issuer()) {   // X2 = P2^T dO + A-> D^V  (dv)
 #pragma unroll
         for (int k = 0; k < 8; ++k)
-            mma_bf16(taddr + 128, mnmajor_desc(uS, 128, k), mnmajor_desc(u1, 128, k), id_nn, k > 0);
+            mma_bf16(taddr + X2, mnmajor_desc(uS, 128, k), mnmajor_desc(u1, 128, k), id_nn, k > 0);
 #pragma unroll
         for (int k = 0; k < 8; ++k)
-            mma_bf16(taddr + 128, kmajor_desc(uAS, 128, k), mnmajor_desc(u4, 128, k), id_kn, 1u);
+            mma_bf16(taddr + X2, kmajor_desc(uAS, 128, k), mnmajor_desc(u4, 128, k), id_kn, 1u);
         mma_commit(&bars[4]);
     }
     wait_mma();
@@ -990,9 +969,9 @@ __global__ void __launch_bounds__(256, 1) bwd_chunk2_tc(const __grid_constant__ 
         tma_load_2d(L4 + TILE / 2, &tsa, 64, snap_row, &bars[3]);
     }
     if (ok) {   // dv
-        float x[64];
-        tmem_ld64(tl + X2, x);
-        store_global_half(static_cast<__nv_bfloat16*>(a.dv) + gi * 128 + 64 * hf, x);
+        float x[32];
+        tmem_ld16x2(tl + X2, x);
+        store_global_q(static_cast<__nv_bfloat16*>(a.dv) + gi * 128, c0, x);
     }
     publish();
     if (issuer()) {   // X1 = dO' A^T
@@ -1001,88 +980,96 @@ __global__ void __launch_bounds__(256, 1) bwd_chunk2_tc(const __grid_constant__ 
             tc_fence_after();
 #pragma unroll
             for (int k = 0; k < 8; ++k)
-                mma_bf16(taddr + 0, kmajor_desc(u3, 128, k), kmajor_desc(uA, 128, k), id_kk, k > 0);
+                mma_bf16(taddr + X1, kmajor_desc(u3, 128, k), kmajor_desc(uA, 128, k), id_kk, k > 0);
             mma_commit(&bars[4]);
         }
     }
     wait_mma();
     {   // P3 = s (dO' A^T) o Gamma (the s of q~ = s q folded in, exactly as bwd_chunk1_tc does)
-        float x[64];
-        tmem_ld64(tl + X1, x);
+        float x[32];
+        tmem_ld16x2(tl + X1, x);
         mask_scores(x, scale);
-        store_half_bf16<__half>(T_S, row, hf, x);
+        store_q<__half>(T_S, row, c0, x);
         if (ok) ok = mbar_wait(&bars[3], 0) && mbar_wait(&bars[1], 0);
         if (ok) {   // Q and K: bf16 -> fp16
-            bf16_to_f16_half(L1, row, hf);
-            bf16_to_f16_half(L2, row, hf);
+            bf16_to_f16_q(L1, row, c0);
+            bf16_to_f16_q(L2, row, c0);
         }
     }
     publish();
     if (issuer()) {   // X2 = P3^T Q (intra part of dk) ;  X1 = Q K^T
-        {
 #pragma unroll
-            for (int k = 0; k < 8; ++k) {
-                mma_bf16(taddr + 128, mnmajor_desc(uS, 128, k), mnmajor_desc(u1, 128, k), id_nn, k > 0);
-                mma_bf16(taddr + 0, kmajor_desc(u1, 128, k), kmajor_desc(u2, 128, k), id_kk, k > 0);
-            }
-            mma_commit(&bars[4]);
+        for (int k = 0; k < 8; ++k) {
+            mma_bf16(taddr + X2, mnmajor_desc(uS, 128, k), mnmajor_desc(u1, 128, k), id_nn, k > 0);
+            mma_bf16(taddr + X1, kmajor_desc(u1, 128, k), kmajor_desc(u2, 128, k), id_kk, k > 0);
         }
+        mma_commit(&bars[4]);
     }
     wait_mma();
     {   // <k, (P3^T Q)_t> ; P1 = s (Q K^T) o Gamma ; K -> K->
-        float x[64], kv[64];
-        tmem_ld64(tl + X2, x);
-        load_half_smem(L2, row, hf, kv);
-        cG += dot64(kv, x);
-        tmem_ld64(tl + X1, x);
+        float x[32], kv[32];
+        tmem_ld16x2(tl + X2, x);
+        load_q(L2, row, c0, kv);
+        cG += dot32(kv, x);
+        tmem_ld16x2(tl + X1, x);
         mask_scores(x, scale);
-        store_half_bf16<__half>(T_S, row, hf, x);
+        store_q<__half>(T_S, row, c0, x);
         __syncthreads();   // the Q K^T product has read K; rows are rescaled in place below
-        if (ok) scale_half_smem(L2, row, hf, fw);
+        if (ok) scale_q(L2, row, c0, fw);
     }
     publish();
     if (issuer()) {   // X1 = A-> D^K (inter part of dk) ; X3 += P1^T dO' ; X4 += K-> D^K^T
 #pragma unroll
         for (int k = 0; k < 8; ++k) {
-            mma_bf16(taddr + 0, kmajor_desc(uAS, 128, k), mnmajor_desc(u4, 128, k), id_kn, k > 0);
-            mma_bf16(taddr + 256, mnmajor_desc(uS, 128, k), mnmajor_desc(u3, 128, k), id_nn, 1u);
-            mma_bf16(taddr + 384, kmajor_desc(u2, 128, k), kmajor_desc(u4, 128, k), id_kk, 1u);
+            mma_bf16(taddr + X1, kmajor_desc(uAS, 128, k), mnmajor_desc(u4, 128, k), id_kn, k > 0);
+            mma_bf16(taddr + X3, mnmajor_desc(uS, 128, k), mnmajor_desc(u3, 128, k), id_nn, 1u);
+            mma_bf16(taddr + X4, kmajor_desc(u2, 128, k), kmajor_desc(u4, 128, k), id_kk, 1u);
         }
         mma_commit(&bars[4]);
     }
     wait_mma();
     float cIG = 0.f, cL = 0.f, cIL = 0.f, db = 0.f;
     if (ok) {
-        float x[64], y[64];
-        tmem_ld64(tl + X2, x);          // dk = P3^T Q + A-> D^K
-        tmem_ld64(tl + X1, y);
+        float x[32], y[32];
+        tmem_ld16x2(tl + X2, x);          // dk = P3^T Q + A-> D^K
+        tmem_ld16x2(tl + X1, y);
 #pragma unroll
-        for (int i = 0; i < 64; ++i) x[i] += y[i];
-        store_global_half(static_cast<__nv_bfloat16*>(a.dk) + gi * 128 + 64 * hf, x);
-        tmem_ld64(tl + X3, x);          // intra-chunk da (both passes)
-        tmem_ld64(tl + X4, y);          // inter-chunk da (both passes)
-        cL = -omega_dot_half(x, av, hf);
-        cIG = dot64(av, y);
-        cIL = -omega_dot_half(y, av, hf);
-        float af[64];
-        write_vector_vals(af, hf, lam, beta);
+        for (int i = 0; i < 32; ++i) x[i] += y[i];
+        store_global_q(static_cast<__nv_bfloat16*>(a.dk) + gi * 128, c0, x);
+        float av[32];
+        load_q(T_A, row, c0, av);
+        tmem_ld16x2(tl + X3, x);          // intra-chunk da (both passes)
+        tmem_ld16x2(tl + X4, y);          // inter-chunk da (both passes)
+        cL = -omega_dot_q(x, av, hf, u);
+        cIG = dot32(av, y);
+        cIL = -omega_dot_q(y, av, hf, u);
 #pragma unroll
-        for (int i = 0; i < 64; ++i) x[i] += y[i];
-        db = dot64(x, af);
+        for (int i = 0; i < 32; ++i) x[i] += y[i];
+        write_vector_q_vals(av, hf, u, lam, beta);   // unrounded a
+        db = dot32(x, av);
     }
-    {
-        const float vG = row_sum(cG), vL = row_sum(cL), vIG = row_sum(cIG), vIL = row_sum(cIL);
-        const float vB = row_sum(db);
-        if (hf == 0 && ok) {
-            const size_t BTH = (size_t)s.B * s.T * s.H;
-            a.tok[2 * BTH + gi] = vG;
-            a.tok[3 * BTH + gi] = vL;
-            a.tok[4 * BTH + gi] = vB / beta;
-            a.tok[5 * BTH + gi] = vIG;
-            a.tok[6 * BTH + gi] = vIL;
-        }
-    }
+    // row sums over the four column quarters, staged in the (now idle) staging tile
+    float* s_fin = reinterpret_cast<float*>(T_S);   // [5][4][128]
+    s_fin[(0 * 4 + cq) * 128 + row] = cG;
+    s_fin[(1 * 4 + cq) * 128 + row] = cL;
+    s_fin[(2 * 4 + cq) * 128 + row] = db;
+    s_fin[(3 * 4 + cq) * 128 + row] = cIG;
+    s_fin[(4 * 4 + cq) * 128 + row] = cIL;
     ok = __syncthreads_and(ok);
+    if (cq == 0 && ok) {
+        float v[5];
+#pragma unroll
+        for (int k = 0; k < 5; ++k) {
+            const float* r = s_fin + 4 * 128 * k + row;
+            v[k] = (r[0] + r[128]) + (r[256] + r[384]);
+        }
+        const size_t BTH = (size_t)s.B * s.T * s.H;
+        a.tok[2 * BTH + gi] = v[0];
+        a.tok[3 * BTH + gi] = v[1];
+        a.tok[4 * BTH + gi] = v[2] / beta;
+        a.tok[5 * BTH + gi] = v[3];
+        a.tok[6 * BTH + gi] = v[4];
+    }
     if (!ok && tid == 0) {
         flag_error(CYFA_ERR_TIMEOUT);
         for (int i = 0; i < 4; ++i) mbar_wait(&bars[i], 0);
@@ -1200,18 +1187,18 @@ cudaError_t launch_bwd_tc(const TcBwdArgs& a, const TcFwdArgs& f, const void* q,
     if (e != cudaSuccess) return e;
     const dim3 gseg(a.nseg, s.B * s.H), gchunk(nct, s.B * s.H);
     const int sm_walk6 = 1024 + 6 * TILE + 1024, sm_walk4 = 1024 + 4 * TILE + 1024;
-    const int sm_chunk = 2048 + 7 * TILE + 1024;
+    const int sm_chunk1 = 5120 + 6 * TILE + 1024, sm_chunk2 = 2048 + 7 * TILE + 1024;
     cudaFuncSetAttribute(snap_fwd_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, sm_walk6);
     { LaunchScope ls_("tc_snap_fwd", st); snap_fwd_tc<<<gseg, 256, sm_walk6, st>>>(mk, mv, a); }
-    cudaFuncSetAttribute(bwd_chunk1_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, sm_chunk);
-    { LaunchScope ls_("tc_bwd_chunk1", st); bwd_chunk1_tc<<<gchunk, 256, sm_chunk, st>>>(mq, mk, mv, mdo, mm, msf, a); }
+    cudaFuncSetAttribute(bwd_chunk1_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, sm_chunk1);
+    { LaunchScope ls_("tc_bwd_chunk1", st); bwd_chunk1_tc<<<gchunk, 512, sm_chunk1, st>>>(mq, mk, mv, mdo, mm, msf, a); }
     cudaFuncSetAttribute(adj_walk_tc<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, sm_walk4);
     { LaunchScope ls_("tc_adj_segment", st); adj_walk_tc<false><<<gseg, 256, sm_walk4, st>>>(mdo1, mo2, mq, mdo, msf, msa, a); }
     { LaunchScope ls_("tc_adj_scan", st); seg_scan_rev_kernel<<<dim3(128, s.B * s.H), 256, 0, st>>>(a); }
     cudaFuncSetAttribute(adj_walk_tc<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, sm_walk6);
     { LaunchScope ls_("tc_snap_adj", st); adj_walk_tc<true><<<gseg, 256, sm_walk6, st>>>(mdo1, mo2, mq, mdo, msf, msa, a); }
-    cudaFuncSetAttribute(bwd_chunk2_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, sm_chunk);
-    { LaunchScope ls_("tc_bwd_chunk2", st); bwd_chunk2_tc<<<gchunk, 256, sm_chunk, st>>>(mq, mk, mv, mdo, mo2, mdo1, msa, a); }
+    cudaFuncSetAttribute(bwd_chunk2_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, sm_chunk2);
+    { LaunchScope ls_("tc_bwd_chunk2", st); bwd_chunk2_tc<<<gchunk, 512, sm_chunk2, st>>>(mq, mk, mv, mdo, mo2, mdo1, msa, a); }
     { LaunchScope ls_("tc_gate", st); tc_gate_kernel<<<gchunk, 128, 0, st>>>(a); }
     if (a.dA) { LaunchScope ls_("tc_dA", st); tc_dA_kernel<<<s.H, 256, 0, st>>>(a); }
     return cudaGetLastError();

@@ -187,5 +187,173 @@ struct Role {
     }
 };
 
+// ------------------------------------------------------------------ 512-thread column quarters
+// In the 512-thread kernels warps w, w + 4, w + 8, w + 12 share TMEM lanes 32 (w % 4) .. + 31 and
+// split a row's 128 columns into quarters cq = w / 4.  Quarter (hf, u) = (cq / 2, cq % 2) owns
+// the 16 rotation pairs j = 32 hf + 16 u + i + 1 (i < 16) of the tensor-core order: element i
+// of the thread's 32 values is column c0 + i (cosine entries) and element 16 + i is column
+// c0 + 32 + i (sine entries), c0 = 64 hf + 16 u.  In quarter (1, 1) element 15 is the DC entry
+// and element 31 the padding entry.
+struct QRole {
+    int warp, lane, q, cq, hf, u, row, c0;
+    __device__ __forceinline__ QRole() {
+        warp = threadIdx.x >> 5;
+        lane = threadIdx.x & 31;
+        q = warp & 3;
+        cq = warp >> 2;
+        hf = cq >> 1;
+        u = cq & 1;
+        row = 32 * q + lane;
+        c0 = 64 * hf + 16 * u;
+    }
+};
+
+// Angles of the 16 pairs of a quarter by angle addition from theta_1, seeded with sincospif at
+// the quarter's first pair (the same seeds as HalfAngles).
+struct QuarterAngles {
+    float c1, s1, c, s;
+    __device__ __forceinline__ QuarterAngles(float lam, int hf, int u) {
+        const int j0 = 32 * hf + 16 * u + 1;
+        sincospif(phase_pi(lam, 1), &s1, &c1);
+        if (j0 == 1) {
+            c = c1;
+            s = s1;
+        } else {
+            sincospif(phase_pi(lam, j0), &s, &c);
+        }
+    }
+    __device__ __forceinline__ void step() {
+        const float cn = c * c1 - s * s1;
+        const float sn = s * c1 + c * s1;
+        c = cn;
+        s = sn;
+    }
+};
+
+// The thread's 32 values <-> row r of a swizzled 16-bit tile (columns c0.. and c0 + 32..).
+template <typename OT>
+__device__ __forceinline__ void store_q(uint8_t* tile, int r, int c0, const float (&x)[32]) {
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+        const float* v = x + 8 * k;
+        uint4 w;
+        w.x = pack2<OT>(v[0], v[1]);
+        w.y = pack2<OT>(v[2], v[3]);
+        w.z = pack2<OT>(v[4], v[5]);
+        w.w = pack2<OT>(v[6], v[7]);
+        *reinterpret_cast<uint4*>(tile + swz_off(r, c0 + 32 * (k >> 1) + 8 * (k & 1), 128)) = w;
+    }
+}
+// fp16 tile -> fp32
+__device__ __forceinline__ void load_q(const uint8_t* tile, int r, int c0, float (&x)[32]) {
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+        const uint4 w = *reinterpret_cast<const uint4*>(tile + swz_off(r, c0 + 32 * (k >> 1) + 8 * (k & 1), 128));
+        const __half2* p = reinterpret_cast<const __half2*>(&w);
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            const float2 f = __half22float2(p[i]);
+            x[8 * k + 2 * i] = f.x;
+            x[8 * k + 2 * i + 1] = f.y;
+        }
+    }
+}
+// bf16 -> fp16 in place on the thread's 32 columns of row r
+__device__ __forceinline__ void bf16_to_f16_q(uint8_t* tile, int r, int c0) {
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+        uint4* p = reinterpret_cast<uint4*>(tile + swz_off(r, c0 + 32 * (k >> 1) + 8 * (k & 1), 128));
+        uint4 w = *p;
+        uint32_t* e = reinterpret_cast<uint32_t*>(&w);
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            const float2 f = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&e[i]));
+            e[i] = pack_f16(f.x, f.y);
+        }
+        *p = w;
+    }
+}
+// multiply the thread's 32 columns of row r of an fp16 tile by w, in place
+__device__ __forceinline__ void scale_q(uint8_t* tile, int r, int c0, float w) {
+    float x[32];
+    load_q(tile, r, c0, x);
+#pragma unroll
+    for (int i = 0; i < 32; ++i) x[i] *= w;
+    store_q<__half>(tile, r, c0, x);
+}
+// The thread's 32 values -> a plain row-major 16-bit row at dst (columns c0.. and c0 + 32..).
+template <typename OT>
+__device__ __forceinline__ void store_global_q(OT* dst, int c0, const float (&x)[32]) {
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+        const float* v = x + 8 * k;
+        uint4 w;
+        w.x = pack2<OT>(v[0], v[1]);
+        w.y = pack2<OT>(v[2], v[3]);
+        w.z = pack2<OT>(v[4], v[5]);
+        w.w = pack2<OT>(v[6], v[7]);
+        *reinterpret_cast<uint4*>(dst + c0 + 32 * (k >> 1) + 8 * (k & 1)) = w;
+    }
+}
+
+// The quarter's entries of the write vector w U(-lam) b (Sec. 3.2), fp32.
+__device__ __forceinline__ void write_vector_q_vals(float (&x)[32], int hf, int u, float lam, float w) {
+    QuarterAngles ang(lam, hf, u);
+    const float wa = w * SQRT_2_OVER_M;
+#pragma unroll
+    for (int i = 0; i < 16; ++i) {
+        if (i > 0) ang.step();
+        x[i] = wa * ang.c;
+        x[16 + i] = -wa * ang.s;
+    }
+    if (hf == 1 && u == 1) {
+        x[15] = w * INV_SQRT_M;
+        x[31] = 0.f;
+    }
+}
+template <typename OT>
+__device__ __forceinline__ void write_vector_q(uint8_t* tile, int r, int hf, int u, float lam, float w) {
+    float x[32];
+    write_vector_q_vals(x, hf, u, lam, w);
+    store_q<OT>(tile, r, 64 * hf + 16 * u, x);
+}
+
+// x <- U(sign lam) x on the quarter's pairs; DC kept, padding zeroed.
+template <int SIGN>
+__device__ __forceinline__ void rotate_q(float (&x)[32], int hf, int u, float lam) {
+    QuarterAngles ang(lam, hf, u);
+    const float dc = x[15];
+#pragma unroll
+    for (int i = 0; i < 16; ++i) {
+        if (i > 0) ang.step();
+        const float c = ang.c, sn = SIGN * ang.s;
+        const float xc = x[i], xs = x[16 + i];
+        x[i] = c * xc - sn * xs;
+        x[16 + i] = sn * xc + c * xs;
+    }
+    if (hf == 1 && u == 1) {
+        x[15] = dc;
+        x[31] = 0.f;
+    }
+}
+
+// <x, Omega y> over the quarter's pairs: sum_j (2 pi j / m) (x_sin,j y_cos,j - x_cos,j y_sin,j).
+__device__ __forceinline__ float omega_dot_q(const float (&x)[32], const float (&y)[32], int hf, int u) {
+    float acc = 0.f;
+#pragma unroll
+    for (int i = 0; i < 16; ++i) {
+        const int j = 32 * hf + 16 * u + i + 1;
+        if (j <= NPAIR) acc += (6.283185307179586f * (float)j / 127.f) * (x[16 + i] * y[i] - x[i] * y[16 + i]);
+    }
+    return acc;
+}
+
+__device__ __forceinline__ float dot32(const float (&x)[32], const float (&y)[32]) {
+    float acc = 0.f;
+#pragma unroll
+    for (int i = 0; i < 32; ++i) acc = fmaf(x[i], y[i], acc);
+    return acc;
+}
+
 }  // namespace
 }  // namespace cyfa
