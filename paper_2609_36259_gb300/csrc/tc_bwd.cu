@@ -467,18 +467,37 @@ __global__ void __launch_bounds__(512, 1) bwd_chunk1_tc(const __grid_constant__ 
         mma_commit(&bars[2]);
     }
     wait_mma();
-    {   // o'' = U(-lam) (p M); scalars with do'' (o'' as stored in fp16); dy = U(lam) do''
-        float o2[32], g2v[32];
-        tmem_ld16x2(tl + X4, o2);
-        rotate_q<-1>(o2, hf, u, lam);
-        store_global_q(a.O2 + ((size_t)bh * s.T + t0 + row) * 128, c0, o2);
+    {   // o'' = U(-lam) (p M); scalars with do'' (o'' as stored in fp16); dy = U(lam) do''.
+        // Eight rotation pairs at a time: cosine entries, then sine entries.
+        QuarterAngles ang(lam, hf, u);
+        const bool dcq = (hf == 1 && u == 1);   // pair 15 of this quarter is the DC / padding
+        __half* o2row = a.O2 + ((size_t)bh * s.T + t0 + row) * 128;
 #pragma unroll
-        for (int i = 0; i < 32; ++i) o2[i] = round16<__half>(o2[i]);
-        tmem_ld16x2(tl + X2, g2v);
-        s1 = dot32(o2, g2v);
-        s2 = omega_dot_q(o2, g2v, hf, u);   // <o'', Omega do''> = -<do'', Omega o''>
-        rotate_q<1>(g2v, hf, u, lam);
-        store_q<__half>(T_S, row, c0, g2v);
+        for (int p8 = 0; p8 < 2; ++p8) {
+            float o[16], gv[16];
+            tmem_ld8x2(tl + X4 + 8 * p8, o);
+            tmem_ld8x2(tl + X2 + 8 * p8, gv);
+#pragma unroll
+            for (int i = 0; i < 8; ++i) {
+                if (p8 + i > 0) ang.step();
+                const float c = ang.c, sn = ang.s;
+                const bool dc = dcq && p8 == 1 && i == 7;
+                const float xc = o[i], xs = o[8 + i];
+                o[i] = dc ? xc : c * xc + sn * xs;          // U(-lam)
+                o[8 + i] = dc ? 0.f : c * xs - sn * xc;
+                const float orc = round16<__half>(o[i]), ors = round16<__half>(o[8 + i]);
+                const float gc = gv[i], gs = gv[8 + i];
+                s1 = fmaf(orc, gc, fmaf(ors, gs, s1));
+                if (!dc) {   // <o'', Omega do''>
+                    const int j = 32 * hf + 16 * u + 8 * p8 + i + 1;
+                    s2 += (6.283185307179586f * (float)j / 127.f) * (ors * gc - orc * gs);
+                }
+                gv[i] = dc ? gc : c * gc - sn * gs;          // U(lam)
+                gv[8 + i] = dc ? 0.f : sn * gc + c * gs;
+            }
+            store8x2_global(o2row, c0 + 8 * p8, o);
+            store8x2<__half>(T_S, row, c0 + 8 * p8, gv);
+        }
     }
     publish();
     if (issuer()) {   // G7: X4 = dy M^T = M dy
@@ -506,16 +525,32 @@ __global__ void __launch_bounds__(512, 1) bwd_chunk1_tc(const __grid_constant__ 
     }
     wait_mma();
     {   // do' = U(-lam) dz; <do', Omega o'> with do' as stored in fp16 (= <dz, Omega z> exactly)
-        float dz[32], z[32];
-        tmem_ld16x2(tl + X2, dz);
-        tmem_ld16x2(tl + X3, z);
-        rotate_q<-1>(dz, hf, u, lam);
-        store_q<__half>(T_S, row, c0, dz);
-        store_global_q(a.DO1 + ((size_t)bh * s.T + t0 + row) * 128, c0, dz);
-        rotate_q<-1>(z, hf, u, lam);   // o'
+        QuarterAngles ang(lam, hf, u);
+        const bool dcq = (hf == 1 && u == 1);
+        __half* d1row = a.DO1 + ((size_t)bh * s.T + t0 + row) * 128;
 #pragma unroll
-        for (int i = 0; i < 32; ++i) dz[i] = round16<__half>(dz[i]);
-        s3 = omega_dot_q(dz, z, hf, u);
+        for (int p8 = 0; p8 < 2; ++p8) {
+            float dz[16], z[16];
+            tmem_ld8x2(tl + X2 + 8 * p8, dz);
+            tmem_ld8x2(tl + X3 + 8 * p8, z);
+#pragma unroll
+            for (int i = 0; i < 8; ++i) {
+                if (p8 + i > 0) ang.step();
+                const float c = ang.c, sn = ang.s;
+                const bool dc = dcq && p8 == 1 && i == 7;
+                const float xc = dz[i], xs = dz[8 + i];
+                dz[i] = dc ? xc : c * xc + sn * xs;         // U(-lam)
+                dz[8 + i] = dc ? 0.f : c * xs - sn * xc;
+                if (!dc) {   // o' = U(-lam) z
+                    const float zc = c * z[i] + sn * z[8 + i], zs = c * z[8 + i] - sn * z[i];
+                    const int j = 32 * hf + 16 * u + 8 * p8 + i + 1;
+                    s3 += (6.283185307179586f * (float)j / 127.f) *
+                          (round16<__half>(dz[8 + i]) * zc - round16<__half>(dz[i]) * zs);
+                }
+            }
+            store8x2<__half>(T_S, row, c0 + 8 * p8, dz);
+            store8x2_global(d1row, c0 + 8 * p8, dz);
+        }
     }
     publish();
     if (issuer()) {   // G9: X1 = dO' A^T, X3 = dO' Kbar

@@ -296,6 +296,34 @@ __device__ __forceinline__ void store_global_q(OT* dst, int c0, const float (&x)
     }
 }
 
+// 16 values (8 at column col, 8 at col + 32) -> row r of a swizzled 16-bit tile / a plain row.
+template <typename OT>
+__device__ __forceinline__ void store8x2(uint8_t* tile, int r, int col, const float (&x)[16]) {
+#pragma unroll
+    for (int k = 0; k < 2; ++k) {
+        const float* v = x + 8 * k;
+        uint4 w;
+        w.x = pack2<OT>(v[0], v[1]);
+        w.y = pack2<OT>(v[2], v[3]);
+        w.z = pack2<OT>(v[4], v[5]);
+        w.w = pack2<OT>(v[6], v[7]);
+        *reinterpret_cast<uint4*>(tile + swz_off(r, col + 32 * k, 128)) = w;
+    }
+}
+template <typename OT>
+__device__ __forceinline__ void store8x2_global(OT* rowp, int col, const float (&x)[16]) {
+#pragma unroll
+    for (int k = 0; k < 2; ++k) {
+        const float* v = x + 8 * k;
+        uint4 w;
+        w.x = pack2<OT>(v[0], v[1]);
+        w.y = pack2<OT>(v[2], v[3]);
+        w.z = pack2<OT>(v[4], v[5]);
+        w.w = pack2<OT>(v[6], v[7]);
+        *reinterpret_cast<uint4*>(rowp + col + 32 * k) = w;
+    }
+}
+
 // The quarter's entries of the write vector w U(-lam) b (Sec. 3.2), fp32.
 __device__ __forceinline__ void write_vector_q_vals(float (&x)[32], int hf, int u, float lam, float w) {
     QuarterAngles ang(lam, hf, u);

@@ -174,10 +174,10 @@ __global__ void __launch_bounds__(256) seg_scan_kernel(TcFwdArgs a) {
 }
 
 // ---------------------------------------------------------------------------------------
-// Chunk walk of one (b, h, segment).  256 threads: thread (row, hf) owns TMEM lane `row` and
-// columns [64 hf, 64 hf + 64) of each 128-column accumulator; thread 0 issues TMA and MMA.
+// Chunk walk of one (b, h, segment).  512 threads: thread (row, quarter) owns TMEM lane `row`
+// and the column quarter of QRole in each 128-column accumulator; thread 0 issues TMA and MMA.
 template <int SEGC>
-__global__ void __launch_bounds__(256, 1) seg_out_tc(const __grid_constant__ CUtensorMap tq,
+__global__ void __launch_bounds__(512, 1) seg_out_tc(const __grid_constant__ CUtensorMap tq,
                                                       const __grid_constant__ CUtensorMap tk,
                                                       const __grid_constant__ CUtensorMap tv,
                                                       const __grid_constant__ CUtensorMap tm,
@@ -188,15 +188,14 @@ __global__ void __launch_bounds__(256, 1) seg_out_tc(const __grid_constant__ CUt
     const int c_begin = seg * SEGC;
     const int nc = min(SEGC, nct - c_begin);
     const int tid = threadIdx.x;
-    const Role ro;
-    const int row = ro.row, hf = ro.hf;
+    const QRole ro;
+    const int row = ro.row, hf = ro.hf, u = ro.u, c0 = ro.c0, cq = ro.cq;
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                                ~uintptr_t(1023));
     uint64_t* bars = reinterpret_cast<uint64_t*>(smem);          // tma, mma, m
     uint32_t* s_taddr = reinterpret_cast<uint32_t*>(smem + 32);
     float* s_g2 = reinterpret_cast<float*>(smem + 64);            // [128] log2-domain decays
-    float* s_red = s_g2 + 128;                                    // [2][128] row reductions
     uint8_t* T_Q = smem + 2048;        // Q, later A-> (state-update operand)
     uint8_t* T_K = T_Q + 1 * TILE;
     uint8_t* T_V = T_Q + 2 * TILE;
@@ -214,8 +213,8 @@ __global__ void __launch_bounds__(256, 1) seg_out_tc(const __grid_constant__ CUt
     __syncthreads();
     tc_fence_after();
     const uint32_t taddr = *s_taddr;
-    const uint32_t tl = taddr + ((uint32_t)(32 * ro.q) << 16);   // this thread's TMEM lane
-    const uint32_t S_COL = 0, X1 = 256 + 64 * hf, X2 = 384 + 64 * hf;
+    const uint32_t tl = taddr + ((uint32_t)(32 * ro.q) << 16) + c0;   // lane, column quarter
+    const uint32_t SK = 0, SV = 128, X1 = 256, X2 = 384;
 
     auto issue_qkv = [&](int c) {
         const int r0 = b * s.T + (c_begin + c) * CT;
@@ -235,17 +234,17 @@ __global__ void __launch_bounds__(256, 1) seg_out_tc(const __grid_constant__ CUt
     }
     // segment-start state into TMEM; Kbar snapshot into T_N (row = slot)
     {
-        const float* src = a.segS + (((size_t)bh * a.nseg + seg) * 128 + row) * 256 + 128 * hf;
+        const float* src = a.segS + (((size_t)bh * a.nseg + seg) * 128 + row) * 256 + c0;
 #pragma unroll
-        for (int q2 = 0; q2 < 2; ++q2) {
-            float x[64];
+        for (int part = 0; part < 2; ++part) {
+            float x[32];
 #pragma unroll
-            for (int i = 0; i < 64; i += 4) {
-                const float4 f = *reinterpret_cast<const float4*>(src + 64 * q2 + i);
+            for (int i = 0; i < 32; i += 4) {
+                const float4 f = *reinterpret_cast<const float4*>(src + 128 * part + (i & 15) + 32 * (i >> 4));
                 x[i] = f.x; x[i + 1] = f.y; x[i + 2] = f.z; x[i + 3] = f.w;
             }
-            tmem_st64(tl + S_COL + 128 * hf + 64 * q2, x);
-            if (hf == 0) store_half_bf16(T_N, row, q2, x);
+            tmem_st16x2(tl + 128 * part, x);
+            if (part == 0) store_q<__nv_bfloat16>(T_N, row, c0, x);
         }
     }
     fence_async_smem();
@@ -277,20 +276,20 @@ __global__ void __launch_bounds__(256, 1) seg_out_tc(const __grid_constant__ CUt
         tc_fence_after();
     };
     auto issuer = [&]() { return tid == 0 && ok; };
-    // masked decay of the intra-chunk scores for this thread's 64 columns (t <= row only);
-    // whole 32-column groups above the diagonal of this warp's rows are skipped
-    auto mask_scores = [&](float (&x)[64], float g2, float mul) {
+    // masked decay of the intra-chunk scores for this thread's 32 columns (t <= row only);
+    // 16-column blocks wholly above the diagonal of this warp's rows are skipped
+    auto mask_scores = [&](float (&x)[32], float g2, float mul) {
 #pragma unroll
-        for (int grp = 0; grp < 2; ++grp) {
-            const int sg = 2 * hf + grp;
-            if (sg > ro.q) {
+        for (int blk = 0; blk < 2; ++blk) {
+            const int tb = c0 + 32 * blk;
+            if (tb >= 32 * (ro.q + 1)) {
 #pragma unroll
-                for (int i = 0; i < 32; ++i) x[32 * grp + i] = 0.f;
+                for (int i = 0; i < 16; ++i) x[16 * blk + i] = 0.f;
             } else {
 #pragma unroll
-                for (int i = 0; i < 32; ++i) {
-                    const int t = 32 * sg + i;
-                    x[32 * grp + i] = (t <= row) ? mul * x[32 * grp + i] * ex2(g2 - s_g2[t]) : 0.f;
+                for (int i = 0; i < 16; ++i) {
+                    const int t = tb + i;
+                    x[16 * blk + i] = (t <= row) ? mul * x[16 * blk + i] * ex2(g2 - s_g2[t]) : 0.f;
                 }
             }
         }
@@ -316,8 +315,8 @@ __global__ void __launch_bounds__(256, 1) seg_out_tc(const __grid_constant__ CUt
             n_beta = a.beta[g1];
             n_g = cum128(s, a.g, b, h, t1, t1 + row);
         }
-        if (hf == 0) s_g2[row] = g2;
-        write_vector_half(T_A, row, hf, lam, beta);
+        if (cq == 0) s_g2[row] = g2;
+        write_vector_q<__nv_bfloat16>(T_A, row, hf, u, lam, beta);
         publish();
         if (!ok) break;
         const float g2C = s_g2[CT - 1];
@@ -330,8 +329,8 @@ __global__ void __launch_bounds__(256, 1) seg_out_tc(const __grid_constant__ CUt
                 tc_fence_after();
 #pragma unroll
                 for (int k = 0; k < 8; ++k) {
-                    mma_bf16(taddr + 256, kmajor_desc(uQ, 128, k), kmajor_desc(uK, 128, k), id_kk, k > 0);
-                    mma_bf16(taddr + 384, kmajor_desc(uQ, 128, k), kmajor_desc(uN, 128, k), id_kk, k > 0);
+                    mma_bf16(taddr + X1, kmajor_desc(uQ, 128, k), kmajor_desc(uK, 128, k), id_kk, k > 0);
+                    mma_bf16(taddr + X2, kmajor_desc(uQ, 128, k), kmajor_desc(uN, 128, k), id_kk, k > 0);
                 }
                 mma_commit(&bars[1]);
             }
@@ -339,152 +338,145 @@ __global__ void __launch_bounds__(256, 1) seg_out_tc(const __grid_constant__ CUt
         tma_ph ^= 1;
         wait_mma();
         {   // P1 = s (Q K^T) o Gamma
-            float x[64];
-            tmem_ld64(tl + X1, x);
+            float x[32];
+            tmem_ld16x2(tl + X1, x);
             mask_scores(x, g2, scale);
-            store_half_bf16(T_S, row, hf, x);
+            store_q<__nv_bfloat16>(T_S, row, c0, x);
         }
         publish();
         if (!ok) break;
         if (issuer()) {
 #pragma unroll
             for (int k = 0; k < 8; ++k)
-                mma_bf16(taddr + 256, kmajor_desc(uS, 128, k), mnmajor_desc(uA, 128, k), id_kn, k > 0);
+                mma_bf16(taddr + X1, kmajor_desc(uS, 128, k), mnmajor_desc(uA, 128, k), id_kn, k > 0);
             mma_commit(&bars[1]);
         }
         // A-> rows into T_Q (Q is consumed), Vbar snapshot into T_N, state scaled by gamma^C
-        write_vector_half(T_Q, row, hf, lam, beta * ex2(g2C - g2));
+        write_vector_q<__nv_bfloat16>(T_Q, row, hf, u, lam, beta * ex2(g2C - g2));
         {
             const float gC = ex2(g2C);
-            float x[64];
-            tmem_ld64(tl + S_COL + 64 * hf, x);            // Kbar columns of this half
+            float x[32];
+            tmem_ld16x2(tl + SK, x);
 #pragma unroll
-            for (int i = 0; i < 64; ++i) x[i] *= gC;
-            tmem_st64(tl + S_COL + 64 * hf, x);
-            tmem_ld64(tl + S_COL + 128 + 64 * hf, x);      // Vbar columns of this half
-            store_half_bf16(T_N, row, hf, x);
+            for (int i = 0; i < 32; ++i) x[i] *= gC;
+            tmem_st16x2(tl + SK, x);
+            tmem_ld16x2(tl + SV, x);
+            store_q<__nv_bfloat16>(T_N, row, c0, x);
 #pragma unroll
-            for (int i = 0; i < 64; ++i) x[i] *= gC;
-            tmem_st64(tl + S_COL + 128 + 64 * hf, x);
+            for (int i = 0; i < 32; ++i) x[i] *= gC;
+            tmem_st16x2(tl + SV, x);
         }
         publish();
         if (!ok) break;
         if (issuer()) {   // state update: [Kbar | Vbar] += A->^T [K | V]
 #pragma unroll
             for (int k = 0; k < 8; ++k) {
-                mma_bf16(taddr + S_COL, mnmajor_desc(uQ, 128, k), mnmajor_desc(uK, 128, k), id_nn, 1u);
-                mma_bf16(taddr + S_COL + 128, mnmajor_desc(uQ, 128, k), mnmajor_desc(uV, 128, k), id_nn, 1u);
+                mma_bf16(taddr + SK, mnmajor_desc(uQ, 128, k), mnmajor_desc(uK, 128, k), id_nn, 1u);
+                mma_bf16(taddr + SV, mnmajor_desc(uQ, 128, k), mnmajor_desc(uV, 128, k), id_nn, 1u);
             }
         }
         wait_mma();   // P1 A
         {   // z = U(lam) o',  o' = s gamma_r (Q Kbar^T) + P1 A
-            float x[64], y[64];
-            tmem_ld64(tl + X2, x);
-            tmem_ld64(tl + X1, y);
+            float x[32], y[32];
+            tmem_ld16x2(tl + X2, x);
+            tmem_ld16x2(tl + X1, y);
             const float f = scale * gam;
 #pragma unroll
-            for (int i = 0; i < 64; ++i) x[i] = fmaf(f, x[i], y[i]);
-            rotate_half<1>(x, hf, lam);
-            store_half_bf16(T_S, row, hf, x);
+            for (int i = 0; i < 32; ++i) x[i] = fmaf(f, x[i], y[i]);
+            rotate_q<1>(x, hf, u, lam);
+            store_q<__nv_bfloat16>(T_S, row, c0, x);
         }
         publish();
         if (!ok) break;
         if (issuer()) {
 #pragma unroll
             for (int k = 0; k < 8; ++k)
-                mma_bf16(taddr + 256, kmajor_desc(uS, 128, k), kmajor_desc(uM, 128, k), id_kk, k > 0);
+                mma_bf16(taddr + X1, kmajor_desc(uS, 128, k), kmajor_desc(uM, 128, k), id_kk, k > 0);
             mma_commit(&bars[1]);
         }
         wait_mma();   // also covers the state update issued before this commit
-        {   // p = softmax over the 127 active slots of l = z M^T
-            float x[64];
-            tmem_ld64(tl + X1, x);
-            const int nvalid = hf ? 63 : 64;           // slot 127 is the padding row
+        {   // p = softmax over the 127 active slots of l = z M^T; the staging tile (z is
+            // consumed) holds the row reductions over the four column quarters
+            float* red = reinterpret_cast<float*>(T_S);
+            float x[32];
+            tmem_ld16x2(tl + X1, x);
+            const bool pad = (hf == 1 && u == 1);       // its element 31 is the padding slot
             float mx = -INFINITY;
 #pragma unroll
-            for (int i = 0; i < 64; ++i)
-                if (i < nvalid) mx = fmaxf(mx, x[i]);
-            s_red[128 * hf + row] = mx;
+            for (int i = 0; i < 32; ++i)
+                if (!(pad && i == 31)) mx = fmaxf(mx, x[i]);
+            red[128 * cq + row] = mx;
             __syncthreads();
-            mx = fmaxf(s_red[row], s_red[128 + row]);
+            mx = fmaxf(fmaxf(red[row], red[128 + row]), fmaxf(red[256 + row], red[384 + row]));
             float sum = 0.f;
 #pragma unroll
-            for (int i = 0; i < 64; ++i) {
-                x[i] = (i < nvalid) ? ex2((x[i] - mx) * LOG2E) : 0.f;
+            for (int i = 0; i < 32; ++i) {
+                x[i] = (pad && i == 31) ? 0.f : ex2((x[i] - mx) * LOG2E);
                 sum += x[i];
             }
+            red[512 + 128 * cq + row] = sum;
             __syncthreads();
-            s_red[128 * hf + row] = sum;
-            __syncthreads();
-            const float inv = 1.f / (s_red[row] + s_red[128 + row]);
+            const float inv = 1.f / ((red[512 + row] + red[640 + row]) + (red[768 + row] + red[896 + row]));
 #pragma unroll
-            for (int i = 0; i < 64; ++i) x[i] *= inv;
-            store_half_bf16(T_S, row, hf, x);
+            for (int i = 0; i < 32; ++i) x[i] *= inv;
+            __syncthreads();   // every quarter has read its sums before p overwrites them
+            store_q<__nv_bfloat16>(T_S, row, c0, x);
         }
         publish();
         if (!ok) break;
         if (issuer()) {
 #pragma unroll
             for (int k = 0; k < 8; ++k)
-                mma_bf16(taddr + 384, kmajor_desc(uS, 128, k), mnmajor_desc(uM, 128, k), id_kn, k > 0);
+                mma_bf16(taddr + X2, kmajor_desc(uS, 128, k), mnmajor_desc(uM, 128, k), id_kn, k > 0);
             mma_commit(&bars[1]);
         }
         wait_mma();
         {   // o'' = U(-lam) (p M)
-            float x[64];
-            tmem_ld64(tl + X2, x);
-            rotate_half<-1>(x, hf, lam);
-            store_half_bf16(T_S, row, hf, x);
+            float x[32];
+            tmem_ld16x2(tl + X2, x);
+            rotate_q<-1>(x, hf, u, lam);
+            store_q<__nv_bfloat16>(T_S, row, c0, x);
         }
         publish();
         if (!ok) break;
         if (issuer()) {
 #pragma unroll
             for (int k = 0; k < 8; ++k) {
-                mma_bf16(taddr + 256, kmajor_desc(uS, 128, k), kmajor_desc(uA, 128, k), id_kk, k > 0);
-                mma_bf16(taddr + 384, kmajor_desc(uS, 128, k), mnmajor_desc(uN, 128, k), id_kn, k > 0);
+                mma_bf16(taddr + X1, kmajor_desc(uS, 128, k), kmajor_desc(uA, 128, k), id_kk, k > 0);
+                mma_bf16(taddr + X2, kmajor_desc(uS, 128, k), mnmajor_desc(uN, 128, k), id_kn, k > 0);
             }
             mma_commit(&bars[1]);
         }
         wait_mma();
         {   // P2 = (O'' A^T) o Gamma
-            float x[64];
-            tmem_ld64(tl + X1, x);
+            float x[32];
+            tmem_ld16x2(tl + X1, x);
             mask_scores(x, g2, 1.f);
-            store_half_bf16(T_S, row, hf, x);
+            store_q<__nv_bfloat16>(T_S, row, c0, x);
         }
         publish();
         if (!ok) break;
         if (issuer()) {
 #pragma unroll
             for (int k = 0; k < 8; ++k)
-                mma_bf16(taddr + 256, kmajor_desc(uS, 128, k), mnmajor_desc(uV, 128, k), id_kn, k > 0);
+                mma_bf16(taddr + X1, kmajor_desc(uS, 128, k), mnmajor_desc(uV, 128, k), id_kn, k > 0);
             mma_commit(&bars[1]);
         }
         wait_mma();
         // next chunk's tiles (Q, K, V are consumed), then o = gamma_r (O'' Vbar) + P2 V
         if (issuer() && c + 1 < nc) issue_qkv(c + 1);
         {
-            float x[64], y[64];
-            tmem_ld64(tl + X2, x);
-            tmem_ld64(tl + X1, y);
+            float x[32], y[32];
+            tmem_ld16x2(tl + X2, x);
+            tmem_ld16x2(tl + X1, y);
 #pragma unroll
-            for (int i = 0; i < 64; ++i) x[i] = fmaf(gam, x[i], y[i]);
-            __nv_bfloat16* O = static_cast<__nv_bfloat16*>(a.o) + gi * 128 + 64 * hf;
-#pragma unroll
-            for (int q2 = 0; q2 < 8; ++q2) {
-                uint4 u;
-                u.x = pack_bf16(x[8 * q2 + 0], x[8 * q2 + 1]);
-                u.y = pack_bf16(x[8 * q2 + 2], x[8 * q2 + 3]);
-                u.z = pack_bf16(x[8 * q2 + 4], x[8 * q2 + 5]);
-                u.w = pack_bf16(x[8 * q2 + 6], x[8 * q2 + 7]);
-                *reinterpret_cast<uint4*>(O + 8 * q2) = u;
-            }
+            for (int i = 0; i < 32; ++i) x[i] = fmaf(gam, x[i], y[i]);
+            store_global_q(static_cast<__nv_bfloat16*>(a.o) + gi * 128, c0, x);
         }
         {   // Kbar snapshot of the next chunk's start state
-            float x[64];
-            tmem_ld64(tl + S_COL + 64 * hf, x);
-            store_half_bf16(T_N, row, hf, x);
+            float x[32];
+            tmem_ld16x2(tl + SK, x);
+            store_q<__nv_bfloat16>(T_N, row, c0, x);
         }
         publish();
     }
@@ -571,7 +563,7 @@ cudaError_t launch_fwd_tc(const TcFwdArgs& a, const void* q, const void* k, cons
     const int smC = 2048 + 7 * TILE + 1024;
     auto kC = seg_out_tc<SEGC_DEFAULT>;
     cudaFuncSetAttribute(kC, cudaFuncAttributeMaxDynamicSharedMemorySize, smC);
-    { LaunchScope ls_("tc_seg_out", st); kC<<<grid, 256, smC, st>>>(mq, mk, mv, mm, a); }
+    { LaunchScope ls_("tc_seg_out", st); kC<<<grid, 512, smC, st>>>(mq, mk, mv, mm, a); }
     return cudaGetLastError();
 }
 
