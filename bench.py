@@ -224,18 +224,21 @@ def run_ours(args):
     ws_p = cyfa.workspace(d, cyfa.CYFA_WS_PREPARE, dev)
     ws_f = cyfa.workspace(d, cyfa.CYFA_WS_FWD, dev)
     ws_b = cyfa.workspace(d, cyfa.CYFA_WS_BWD, dev)
+    # the forward saves its chunk-start states for the backward (a training step keeps them)
+    saved = None if args.no_saved else cyfa.saved_buffer(d, dev)
+    tc_path = cyfa.cyfa_saved_size(d) > 0
     stream = torch.cuda.current_stream()
 
     def step(x):
         cyfa.cyfa_prepare(d, x['clock_logit'], x['decay_logit'], x['beta_logit'], x['A'], None,
                           lam, g, beta, None, ws_p)
         cyfa.cyfa_chunk_fwd(d, x['q'], x['k'], x['v'], lam, g, beta, x['R'], None, None, o, None,
-                            None, ws_f)
+                            None, ws_f, saved=saved)
         if args.no_bwd:
             return
         cyfa.cyfa_chunk_bwd(d, x['q'], x['k'], x['v'], lam, g, beta, x['R'], x['clock_logit'],
                             x['decay_logit'], x['A'], x['dO'], dq, dk, dv, dc, dd, db, None, dA,
-                            ws_b)
+                            ws_b, saved=saved)
 
     for _ in range(args.warmup):
         step(inp)
@@ -269,7 +272,7 @@ def run_ours(args):
     # per-kernel times and the forward / backward split
     per_kernel = {k: {'launches': n, 'ms_per_launch': t / n if n else 0.0}
                   for k, (n, t) in stats.items()}
-    fwd_names = ('readout_matrix', 'fwd_state', 'fwd_out', 'm_to_k16', 'tc_seg_state',
+    fwd_names = ('readout_matrix', 'fwd_state', 'fwd_out', 'm_to_f16', 'tc_seg_state',
                  'tc_seg_scan', 'tc_seg_out')
     # the forward's kernels are launched again inside the backward (recomputation): split by
     # launch count, one forward's worth per step belongs to cyfa_chunk_fwd
@@ -326,11 +329,16 @@ def run_ours(args):
     line = {
         'metric': METRIC, 'value': value, 'unit': 'tokens/s', 'n_gpus': world,
         'steps': args.steps, 'warmup': args.warmup, 'ms_per_step': ms,
-        'higher_is_better': True, 'scaling': 'weak', 'vs_baseline': None, 'dtype': 'bf16',
+        'higher_is_better': True, 'scaling': 'weak', 'vs_baseline': None,
+        'dtype': 'fp16' if tc_path else 'fp32',
         'data': 'synthetic',
         'config': {'workload': 'cyfa-1.4B-layer prepare+fwd+bwd', 'model': 'CyFA core operator',
                    'B': B, 'T': T, 'H': H, 'dk': D, 'dv': D, 'm': 127, 'm_store': MS,
-                   'chunk': C, 'global_batch': B * world, 'seq_len': T,
+                   'chunk': 128 if tc_path else C, 'io_dtype': 'bf16',
+                   'arithmetic': ('tcgen05 fp16 operands, fp32 accumulate' if tc_path
+                                  else 'fp32 CUDA cores'),
+                   'saved_states': saved is not None,
+                   'global_batch': B * world, 'seq_len': T,
                    'parallelism': 'dp%d' % world,
                    'l2': 'inputs larger than L2 (q,k,v,dO %.0f MB)' % (4 * B * T * H * D * 2 / 1e6)},
         'roofline': roof, 'kernel_rooflines': rooflines, 'cpu_baseline': cpu, 'e2e': e2e, 'gpu_launches': launches,
@@ -488,6 +496,9 @@ def main():
     ap.add_argument('--ref-tokens', type=int, default=256)
     ap.add_argument('--no-decode', action='store_true')
     ap.add_argument('--no-e2e', action='store_true')
+    ap.add_argument('--no-saved', action='store_true',
+                    help='backward recomputes the chunk-start states instead of reading the '
+                         'ones the forward saved')
     ap.add_argument('--no-cpu-baseline', action='store_true')
     ap.add_argument('--no-bwd', action='store_true',
                     help='time prepare + forward only (profiling runs; not the headline step)')

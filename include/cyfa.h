@@ -122,16 +122,31 @@ int cyfa_prepare_noalloc(const cyfa_dims_t* dims, const float* clock_logit,
                          double* lambda_end, void* stream);
 
 /*
+ * cyfa_saved_size -- bytes of the forward intermediates that cyfa_chunk_fwd can save for
+ * cyfa_chunk_bwd: the states [Kbar | Vbar] at the start of every 128-token chunk (App. B's
+ * chunk-boundary states), fp16, [B*H][T/128][2][128][128] with the Fourier rows in the
+ * kernels' internal order.  0 where the call runs the CUDA-core kernels (nothing is saved).
+ * No paper counterpart beyond those states: this is the usual activation-saving trade of a
+ * training step (HBM traffic for recomputation).
+ */
+int cyfa_saved_size(const cyfa_dims_t* dims, size_t* bytes);
+
+/*
  * cyfa_chunk_fwd -- forward of the operator, chunk-wise two-pass form (Sec. 3.3 Eq.
  * cyfa-two-pass; App. B Eqs. app-cyfa-key-chunk, app-cyfa-value-chunk).
  * Inputs are the outputs of cyfa_prepare plus q, k, v and R.  Kbar0 / Vbar0 (nullable,
  * both or neither) give the states before token 0 in the same clock origin as lambda0.
  * o receives the output; Kbar_out / Vbar_out (nullable) receive the states after token T-1.
+ * saved (nullable, device, 16-byte aligned, cyfa_saved_size bytes) receives the chunk-start
+ * states for cyfa_chunk_bwd; ignored where cyfa_saved_size is 0.
+ * The tensor-core kernels (bf16, d = 128) compute with fp16 operands: q, k, v must lie within
+ * fp16's range (|x| < 65504).
  */
 int cyfa_chunk_fwd(const cyfa_dims_t* dims, const void* q, const void* k, const void* v,
                    const float* lam_mod, const float* g_cum, const float* beta, const float* R,
                    const float* Kbar0, const float* Vbar0, void* o, float* Kbar_out,
-                   float* Vbar_out, void* workspace, size_t workspace_bytes, void* stream);
+                   float* Vbar_out, void* saved, void* workspace, size_t workspace_bytes,
+                   void* stream);
 
 /*
  * cyfa_chunk_bwd -- gradient of sum(o * dO) with respect to q, k, v, the three logits, and
@@ -140,14 +155,16 @@ int cyfa_chunk_fwd(const cyfa_dims_t* dims, const void* q, const void* k, const 
  * app-clock-gradient-accumulation; the decay gradient is the reverse cumulative sum of
  * the per-token gradient of the cumulative log-decay.  dR [H,m,m] and dA [H] are sums
  * over the batch.  Inputs are those of cyfa_chunk_fwd plus the raw clock / decay logits
- * and A (for the activation derivatives).
+ * and A (for the activation derivatives).  saved (nullable): the buffer a cyfa_chunk_fwd call
+ * with the same dims, inputs and no initial state filled; the chunk-start states are then
+ * read from it instead of being recomputed.  Ignored where cyfa_saved_size is 0.
  */
 int cyfa_chunk_bwd(const cyfa_dims_t* dims, const void* q, const void* k, const void* v,
                    const float* lam_mod, const float* g_cum, const float* beta, const float* R,
                    const float* clock_logit, const float* decay_logit, const float* A,
                    const void* dO, void* dq, void* dk, void* dv, float* d_clock_logit,
                    float* d_decay_logit, float* d_beta_logit, float* dR, float* dA,
-                   void* workspace, size_t workspace_bytes, void* stream);
+                   const void* saved, void* workspace, size_t workspace_bytes, void* stream);
 
 /*
  * cyfa_step -- one decode token for every (b, h), in place on the persistent state

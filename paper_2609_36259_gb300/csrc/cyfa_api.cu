@@ -61,7 +61,7 @@ bool use_tc(const cyfa_dims_t* d, const Shape& s) {
 struct FwdLayout {
     float *M, *MT, *states;          // CUDA-core path
     float *segS, *segG;              // tensor-core path
-    __nv_bfloat16* Mb;
+    __half* Mb;
     int nseg;
     size_t bytes;
 };
@@ -72,7 +72,7 @@ FwdLayout fwd_layout(const Shape& s, bool tc_path, void* ws) {
     L.MT = c.take<float>((size_t)s.H * MS * MS);
     if (tc_path) {
         L.nseg = tc_fwd_segments(s);
-        L.Mb = c.take<__nv_bfloat16>((size_t)s.H * MS * MS);
+        L.Mb = c.take<__half>((size_t)s.H * MS * MS);
         L.segS = c.take<float>((size_t)s.B * s.H * L.nseg * MS * 256);
         L.segG = c.take<float>((size_t)s.B * s.H * L.nseg);
     } else {
@@ -161,6 +161,18 @@ int cyfa_workspace_size(const cyfa_dims_t* dims, int which, size_t* bytes) {
     }
 }
 
+// fp16 chunk-start states [B*H][T/128][2][128][128] of the tensor-core path
+size_t saved_bytes(const Shape& s) { return (size_t)s.B * s.H * (s.T / 128) * 2 * 128 * 128 * 2; }
+
+int cyfa_saved_size(const cyfa_dims_t* dims, size_t* bytes) {
+    if (!bytes) return CYFA_ERR_ARG;
+    const int rc = check_dims(dims, true);
+    if (rc) return rc;
+    const Shape s = shape_of(dims);
+    *bytes = use_tc(dims, s) ? saved_bytes(s) : 0;
+    return CYFA_OK;
+}
+
 int cyfa_prepare(const cyfa_dims_t* dims, const float* clock_logit, const float* decay_logit,
                  const float* beta_logit, const float* A, const double* lambda0, float* lam_mod,
                  float* g_cum, float* beta, double* lambda_end, void* workspace,
@@ -189,7 +201,8 @@ int cyfa_prepare(const cyfa_dims_t* dims, const float* clock_logit, const float*
 int cyfa_chunk_fwd(const cyfa_dims_t* dims, const void* q, const void* k, const void* v,
                    const float* lam_mod, const float* g_cum, const float* beta, const float* R,
                    const float* Kbar0, const float* Vbar0, void* o, float* Kbar_out,
-                   float* Vbar_out, void* workspace, size_t workspace_bytes, void* stream) {
+                   float* Vbar_out, void* saved, void* workspace, size_t workspace_bytes,
+                   void* stream) {
     int rc = check_dims(dims, true);
     if (rc) return rc;
     if (!q || !k || !v || !lam_mod || !g_cum || !beta || !R || !o) return CYFA_ERR_ARG;
@@ -201,6 +214,7 @@ int cyfa_chunk_fwd(const cyfa_dims_t* dims, const void* q, const void* k, const 
         return CYFA_ERR_ALIGN;
     const Shape s = shape_of(dims);
     const bool tc_path = use_tc(dims, s);
+    if (saved && !aligned16(saved)) return CYFA_ERR_ALIGN;
     const FwdLayout need = fwd_layout(s, tc_path, nullptr);
     if (!workspace || workspace_bytes < need.bytes) return CYFA_ERR_WORKSPACE;
     if (!aligned16(workspace)) return CYFA_ERR_ALIGN;
@@ -222,6 +236,7 @@ int cyfa_chunk_fwd(const cyfa_dims_t* dims, const void* q, const void* k, const 
         t.segS = L.segS;
         t.segG = L.segG;
         t.Mb = L.Mb;
+        t.snap = static_cast<__half*>(saved);
         t.nseg = L.nseg;
         return cuda_status(launch_fwd_tc(t, q, k, v, L.M, st));
     }
@@ -249,7 +264,7 @@ int cyfa_chunk_bwd(const cyfa_dims_t* dims, const void* q, const void* k, const 
                    const float* clock_logit, const float* decay_logit, const float* A,
                    const void* dO, void* dq, void* dk, void* dv, float* d_clock_logit,
                    float* d_decay_logit, float* d_beta_logit, float* dR, float* dA,
-                   void* workspace, size_t workspace_bytes, void* stream) {
+                   const void* saved, void* workspace, size_t workspace_bytes, void* stream) {
     int rc = check_dims(dims, true);
     if (rc) return rc;
     if (!q || !k || !v || !lam_mod || !g_cum || !beta || !R || !clock_logit || !decay_logit ||
@@ -259,6 +274,7 @@ int cyfa_chunk_bwd(const cyfa_dims_t* dims, const void* q, const void* k, const 
         !aligned16(dk) || !aligned16(dv))
         return CYFA_ERR_ALIGN;
     if (dR) return CYFA_ERR_UNSUPPORTED;
+    if (saved && !aligned16(saved)) return CYFA_ERR_ALIGN;
     const Shape s = shape_of(dims);
     const bool tc_path = use_tc(dims, s);
     const BwdLayout need = bwd_layout(s, tc_path, nullptr);
@@ -305,7 +321,8 @@ int cyfa_chunk_bwd(const cyfa_dims_t* dims, const void* q, const void* k, const 
         f.beta = beta;
         f.segS = L.segS;
         f.segG = L.segG;
-        f.Mb = reinterpret_cast<const __nv_bfloat16*>(L.Mb);   // filled as fp16 (f16 launch)
+        f.Mb = L.Mb;
+        f.snap = nullptr;
         f.nseg = L.nseg;
         TcBwdArgs t{};
         t.s = s;
@@ -316,7 +333,8 @@ int cyfa_chunk_bwd(const cyfa_dims_t* dims, const void* q, const void* k, const 
         t.segG = L.segG;
         t.segD = L.segD;
         t.nseg = L.nseg;
-        t.snapF = L.snapF;
+        t.snapF = saved ? static_cast<__half*>(const_cast<void*>(saved)) : L.snapF;
+        t.saved = saved != nullptr;
         t.snapA = L.snapA;
         t.O2 = L.O2b;
         t.DO1 = L.DO1b;

@@ -98,7 +98,9 @@ struct TcFwdArgs {
     void* o;                      // bf16 [B,T,H,128]
     float* segS;                  // [B*H][nseg][128][256]: segment deltas, then segment-start states
     float* segG;                  // [B*H][nseg] total log-decay of each segment
-    const __nv_bfloat16* Mb;      // [H][128][128] bf16 M = R Phi
+    const __half* Mb;             // [H][128][128] fp16 M = R Phi
+    __half* snap;                 // nullable [B*H][T/128][2][128][128] fp16: Kbar, Vbar at
+                                  // each chunk start, written for the backward
     int nseg;
 };
 bool tc_fwd_supported(const Shape& s);
@@ -113,10 +115,11 @@ cudaError_t tc_bwd_read_error(cudaStream_t st, int* err);
 bool tc_qkv_maps(const Shape& s, const void* q, const void* k, const void* v, CUtensorMap* mq,
                  CUtensorMap* mk, CUtensorMap* mv);
 bool tc_rows_map(CUtensorMap* map, const void* base, unsigned long long rows, bool f16 = false);
-// M -> 16-bit (tensor-core order), segment state contributions, segment scan (forward); with
-// f16 the operands of the tensor-core products are fp16 (a.Mb then points to fp16 storage).
+// M -> fp16 (tensor-core order), segment state contributions, segment scan.
 cudaError_t launch_fwd_segment_states(const TcFwdArgs& a, const void* k, const void* v,
-                                      const float* Mf, cudaStream_t st, bool f16 = false);
+                                      const float* Mf, cudaStream_t st);
+// M -> fp16 (tensor-core order) and the total log-decay of every segment, without the states.
+cudaError_t launch_m_and_segment_decay(const TcFwdArgs& a, const float* Mf, cudaStream_t st);
 
 struct TcBwdArgs {
     Shape s;
@@ -126,6 +129,7 @@ struct TcBwdArgs {
     float* segD;                 // adjoint: per-segment contributions, then end-of-segment adjoints
     int nseg;
     __half* snapF;               // [B*H][T/128][2][128][128] fp16: Kbar, Vbar at each chunk start
+    bool saved;                  // snapF holds the forward's saved states: no recomputation
     __half* snapA;               // [B*H][T/128][2][128][128] fp16: D^K, D^V at each chunk end
     __half* O2;                  // [B*H][T][128] fp16: o'' (tensor-core order)
     __half* DO1;                 // [B*H][T][128] fp16: dL/do' (tensor-core order)

@@ -1218,13 +1218,18 @@ cudaError_t launch_bwd_tc(const TcBwdArgs& a, const TcFwdArgs& f, const void* q,
         !tc_rows_map(&msa, a.snapA, BH * nct * 2 * 128, true) ||
         !tc_rows_map(&mo2, a.O2, BH * s.T, true) || !tc_rows_map(&mdo1, a.DO1, BH * s.T, true))
         return cudaErrorInvalidValue;
-    cudaError_t e = launch_fwd_segment_states(f, k, v, Mf, st, true);
+    // chunk-start states: the forward's saved snapshots, or recomputed (segment states, then a
+    // walk of every segment)
+    cudaError_t e = a.saved ? launch_m_and_segment_decay(f, Mf, st)
+                            : launch_fwd_segment_states(f, k, v, Mf, st);
     if (e != cudaSuccess) return e;
     const dim3 gseg(a.nseg, s.B * s.H), gchunk(nct, s.B * s.H);
     const int sm_walk6 = 1024 + 6 * TILE + 1024, sm_walk4 = 1024 + 4 * TILE + 1024;
     const int sm_chunk1 = 5120 + 6 * TILE + 1024, sm_chunk2 = 2048 + 7 * TILE + 1024;
-    cudaFuncSetAttribute(snap_fwd_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, sm_walk6);
-    { LaunchScope ls_("tc_snap_fwd", st); snap_fwd_tc<<<gseg, 256, sm_walk6, st>>>(mk, mv, a); }
+    if (!a.saved) {
+        cudaFuncSetAttribute(snap_fwd_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, sm_walk6);
+        { LaunchScope ls_("tc_snap_fwd", st); snap_fwd_tc<<<gseg, 256, sm_walk6, st>>>(mk, mv, a); }
+    }
     cudaFuncSetAttribute(bwd_chunk1_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, sm_chunk1);
     { LaunchScope ls_("tc_bwd_chunk1", st); bwd_chunk1_tc<<<gchunk, 512, sm_chunk1, st>>>(mq, mk, mv, mdo, mm, msf, a); }
     cudaFuncSetAttribute(adj_walk_tc<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, sm_walk4);

@@ -181,6 +181,7 @@ __global__ void __launch_bounds__(512, 1) seg_out_tc(const __grid_constant__ CUt
                                                       const __grid_constant__ CUtensorMap tk,
                                                       const __grid_constant__ CUtensorMap tv,
                                                       const __grid_constant__ CUtensorMap tm,
+                                                      const __grid_constant__ CUtensorMap tsnap,
                                                       TcFwdArgs a) {
     const Shape s = a.s;
     const int seg = blockIdx.x, bh = blockIdx.y, b = bh / s.H, h = bh % s.H;
@@ -244,7 +245,7 @@ __global__ void __launch_bounds__(512, 1) seg_out_tc(const __grid_constant__ CUt
                 x[i] = f.x; x[i + 1] = f.y; x[i + 2] = f.z; x[i + 3] = f.w;
             }
             tmem_st16x2(tl + 128 * part, x);
-            if (part == 0) store_q<__nv_bfloat16>(T_N, row, c0, x);
+            if (part == 0) store_q<__half>(T_N, row, c0, x);
         }
     }
     fence_async_smem();
@@ -255,9 +256,17 @@ __global__ void __launch_bounds__(512, 1) seg_out_tc(const __grid_constant__ CUt
     ok = __syncthreads_and(ok);
     uint32_t tma_ph = 0, mma_ph = 0;
     const float scale = s.scale;
-    const uint32_t id_kk = idesc_bf16(128, 128, 0, 0);
-    const uint32_t id_kn = idesc_bf16(128, 128, 0, 1);
-    const uint32_t id_nn = idesc_bf16(128, 128, 1, 1);
+    const uint32_t id_kk = idesc_f16(128, 128, 0, 0);
+    const uint32_t id_kn = idesc_f16(128, 128, 0, 1);
+    const uint32_t id_nn = idesc_f16(128, 128, 1, 1);
+    const bool save = a.snap != nullptr;
+    // the snapshot in T_N (part 0: Kbar, 1: Vbar) of chunk cg leaves by a TMA store
+    auto store_snap = [&](int cg, int part) {
+        const int r = ((bh * nct + cg) * 2 + part) * 128;
+        tma_store_2d(&tsnap, T_N, 0, r);
+        tma_store_2d(&tsnap, T_N + TILE / 2, 64, r);
+        bulk_commit();
+    };
     const uint32_t uQ = smem_u32(T_Q), uK = smem_u32(T_K), uV = smem_u32(T_V),
                    uA = smem_u32(T_A), uS = smem_u32(T_S), uN = smem_u32(T_N),
                    uM = smem_u32(T_M);
@@ -316,17 +325,22 @@ __global__ void __launch_bounds__(512, 1) seg_out_tc(const __grid_constant__ CUt
             n_g = cum128(s, a.g, b, h, t1, t1 + row);
         }
         if (cq == 0) s_g2[row] = g2;
-        write_vector_q<__nv_bfloat16>(T_A, row, hf, u, lam, beta);
+        write_vector_q<__half>(T_A, row, hf, u, lam, beta);
+        if (ok) ok = mbar_wait(&bars[0], tma_ph);
+        if (ok) {   // Q, K, V: bf16 -> fp16
+            bf16_to_f16_q(T_Q, row, c0);
+            bf16_to_f16_q(T_K, row, c0);
+            bf16_to_f16_q(T_V, row, c0);
+        }
         publish();
         if (!ok) break;
         const float g2C = s_g2[CT - 1];
         const float gam = ex2(g2);
+        if (save && tid == 0) store_snap(c_begin + c, 0);
 
         // X1 = Q K^T, X2 = Q Kbar^T
         if (issuer()) {
-            ok = mbar_wait(&bars[0], tma_ph);
-            if (ok) {
-                tc_fence_after();
+            {
 #pragma unroll
                 for (int k = 0; k < 8; ++k) {
                     mma_bf16(taddr + X1, kmajor_desc(uQ, 128, k), kmajor_desc(uK, 128, k), id_kk, k > 0);
@@ -341,8 +355,9 @@ __global__ void __launch_bounds__(512, 1) seg_out_tc(const __grid_constant__ CUt
             float x[32];
             tmem_ld16x2(tl + X1, x);
             mask_scores(x, g2, scale);
-            store_q<__nv_bfloat16>(T_S, row, c0, x);
+            store_q<__half>(T_S, row, c0, x);
         }
+        if (save && tid == 0) bulk_wait_read_all();   // T_N is rewritten after this barrier
         publish();
         if (!ok) break;
         if (issuer()) {
@@ -352,7 +367,7 @@ __global__ void __launch_bounds__(512, 1) seg_out_tc(const __grid_constant__ CUt
             mma_commit(&bars[1]);
         }
         // A-> rows into T_Q (Q is consumed), Vbar snapshot into T_N, state scaled by gamma^C
-        write_vector_q<__nv_bfloat16>(T_Q, row, hf, u, lam, beta * ex2(g2C - g2));
+        write_vector_q<__half>(T_Q, row, hf, u, lam, beta * ex2(g2C - g2));
         {
             const float gC = ex2(g2C);
             float x[32];
@@ -361,13 +376,14 @@ __global__ void __launch_bounds__(512, 1) seg_out_tc(const __grid_constant__ CUt
             for (int i = 0; i < 32; ++i) x[i] *= gC;
             tmem_st16x2(tl + SK, x);
             tmem_ld16x2(tl + SV, x);
-            store_q<__nv_bfloat16>(T_N, row, c0, x);
+            store_q<__half>(T_N, row, c0, x);
 #pragma unroll
             for (int i = 0; i < 32; ++i) x[i] *= gC;
             tmem_st16x2(tl + SV, x);
         }
         publish();
         if (!ok) break;
+        if (save && tid == 0) store_snap(c_begin + c, 1);
         if (issuer()) {   // state update: [Kbar | Vbar] += A->^T [K | V]
 #pragma unroll
             for (int k = 0; k < 8; ++k) {
@@ -384,7 +400,7 @@ __global__ void __launch_bounds__(512, 1) seg_out_tc(const __grid_constant__ CUt
 #pragma unroll
             for (int i = 0; i < 32; ++i) x[i] = fmaf(f, x[i], y[i]);
             rotate_q<1>(x, hf, u, lam);
-            store_q<__nv_bfloat16>(T_S, row, c0, x);
+            store_q<__half>(T_S, row, c0, x);
         }
         publish();
         if (!ok) break;
@@ -420,7 +436,7 @@ __global__ void __launch_bounds__(512, 1) seg_out_tc(const __grid_constant__ CUt
 #pragma unroll
             for (int i = 0; i < 32; ++i) x[i] *= inv;
             __syncthreads();   // every quarter has read its sums before p overwrites them
-            store_q<__nv_bfloat16>(T_S, row, c0, x);
+            store_q<__half>(T_S, row, c0, x);
         }
         publish();
         if (!ok) break;
@@ -435,7 +451,7 @@ __global__ void __launch_bounds__(512, 1) seg_out_tc(const __grid_constant__ CUt
             float x[32];
             tmem_ld16x2(tl + X2, x);
             rotate_q<-1>(x, hf, u, lam);
-            store_q<__nv_bfloat16>(T_S, row, c0, x);
+            store_q<__half>(T_S, row, c0, x);
         }
         publish();
         if (!ok) break;
@@ -452,8 +468,9 @@ __global__ void __launch_bounds__(512, 1) seg_out_tc(const __grid_constant__ CUt
             float x[32];
             tmem_ld16x2(tl + X1, x);
             mask_scores(x, g2, 1.f);
-            store_q<__nv_bfloat16>(T_S, row, c0, x);
+            store_q<__half>(T_S, row, c0, x);
         }
+        if (save && tid == 0) bulk_wait_read_all();   // T_N is rewritten after this barrier
         publish();
         if (!ok) break;
         if (issuer()) {
@@ -476,7 +493,7 @@ __global__ void __launch_bounds__(512, 1) seg_out_tc(const __grid_constant__ CUt
         {   // Kbar snapshot of the next chunk's start state
             float x[32];
             tmem_ld16x2(tl + SK, x);
-            store_q<__nv_bfloat16>(T_N, row, c0, x);
+            store_q<__half>(T_N, row, c0, x);
         }
         publish();
     }
@@ -484,19 +501,36 @@ __global__ void __launch_bounds__(512, 1) seg_out_tc(const __grid_constant__ CUt
         flag_error(CYFA_ERR_TIMEOUT);
         mbar_wait(&bars[0], tma_ph);   // let copies still in flight land
     }
+    if (save && tid == 0) bulk_wait_all();
     tc_fence_before();
     __syncthreads();
     if (ro.warp == 0) tmem_dealloc(taddr, 512);
 }
 
-// M (fp32, paper order) -> 16-bit OT with its Fourier (column) index in the tensor-core order.
-template <typename OT>
-__global__ void m_to_k16_kernel(const float* M, OT* Mb, int H) {
+// M (fp32, paper order) -> fp16 with its Fourier (column) index in the tensor-core order.
+__global__ void m_to_f16_kernel(const float* M, __half* Mb, int H) {
     const int i = blockIdx.x * blockDim.x + threadIdx.x;
     if (i >= H * 128 * 128) return;
     const int p = i & 127, rest = i >> 7;
-    if constexpr (std::is_same<OT, __half>::value) Mb[rest * 128 + tc_slot(p)] = __float2half_rn(M[i]);
-    else Mb[rest * 128 + tc_slot(p)] = __float2bfloat16_rn(M[i]);
+    Mb[rest * 128 + tc_slot(p)] = __float2half_rn(M[i]);
+}
+
+// Total log-decay of every segment (sum of its chunks' 128-token totals), as seg_state_tc
+// computes it; one warp per (segment, b*h).
+__global__ void seg_decay_kernel(TcFwdArgs a, int segc) {
+    const Shape s = a.s;
+    const int seg = blockIdx.x, bh = blockIdx.y, b = bh / s.H, h = bh % s.H;
+    const int nct = s.T / CT, c_begin = seg * segc, nc = min(segc, nct - c_begin);
+    const int lane = threadIdx.x;
+    float tot = 0.f;
+    if (lane < nc) {
+        const int t0 = (c_begin + lane) * CT;
+        tot = cum128(s, a.g, b, h, t0, t0 + CT - 1);
+    }
+    // the same order as seg_state_tc: acc over chunks from last to first
+    float acc = 0.f;
+    for (int c = nc - 1; c >= 0; --c) acc += __shfl_sync(0xffffffffu, tot, c);
+    if (lane == 0) a.segG[(size_t)bh * a.nseg + seg] = acc;
 }
 
 constexpr int SEGC_DEFAULT = TC_SEGC;
@@ -529,33 +563,46 @@ bool tc_rows_map(CUtensorMap* map, const void* base, unsigned long long rows, bo
 }
 
 cudaError_t launch_fwd_segment_states(const TcFwdArgs& a, const void* k, const void* v,
-                                      const float* Mf, cudaStream_t st, bool f16) {
+                                      const float* Mf, cudaStream_t st) {
     const Shape& s = a.s;
     CUtensorMap mk, mv;
     if (!tc_qkv_maps(s, nullptr, k, v, nullptr, &mk, &mv)) return cudaErrorInvalidValue;
     const int n = s.H * 128 * 128;
     {
-        LaunchScope ls_("m_to_k16", st);
-        if (f16)
-            m_to_k16_kernel<__half><<<(n + 255) / 256, 256, 0, st>>>(Mf, (__half*)(a.Mb), s.H);
-        else
-            m_to_k16_kernel<__nv_bfloat16><<<(n + 255) / 256, 256, 0, st>>>(Mf, const_cast<__nv_bfloat16*>(a.Mb), s.H);
+        LaunchScope ls_("m_to_f16", st);
+        m_to_f16_kernel<<<(n + 255) / 256, 256, 0, st>>>(Mf, const_cast<__half*>(a.Mb), s.H);
     }
     const dim3 grid(a.nseg, s.B * s.H);
     const int smA = 1024 + 6 * TILE + 1024;
-    auto kA = f16 ? seg_state_tc<SEGC_DEFAULT, __half> : seg_state_tc<SEGC_DEFAULT, __nv_bfloat16>;
+    auto kA = seg_state_tc<SEGC_DEFAULT, __half>;
     cudaFuncSetAttribute(kA, cudaFuncAttributeMaxDynamicSharedMemorySize, smA);
     { LaunchScope ls_("tc_seg_state", st); kA<<<grid, 256, smA, st>>>(mk, mv, a); }
     { LaunchScope ls_("tc_seg_scan", st); seg_scan_kernel<<<dim3(128, s.B * s.H), 256, 0, st>>>(a); }
     return cudaGetLastError();
 }
 
+cudaError_t launch_m_and_segment_decay(const TcFwdArgs& a, const float* Mf, cudaStream_t st) {
+    const Shape& s = a.s;
+    const int n = s.H * 128 * 128;
+    {
+        LaunchScope ls_("m_to_f16", st);
+        m_to_f16_kernel<<<(n + 255) / 256, 256, 0, st>>>(Mf, const_cast<__half*>(a.Mb), s.H);
+    }
+    { LaunchScope ls_("tc_seg_decay", st); seg_decay_kernel<<<dim3(a.nseg, s.B * s.H), 32, 0, st>>>(a, SEGC_DEFAULT); }
+    return cudaGetLastError();
+}
+
 cudaError_t launch_fwd_tc(const TcFwdArgs& a, const void* q, const void* k, const void* v,
                           const float* Mf, cudaStream_t st) {
     const Shape& s = a.s;
-    CUtensorMap mq, mk, mv, mm;
+    const unsigned long long BH = (unsigned long long)s.B * s.H;
+    CUtensorMap mq, mk, mv, mm, msnap;
     if (!tc_qkv_maps(s, q, k, v, &mq, &mk, &mv) ||
-        !tc_rows_map(&mm, a.Mb, (unsigned long long)s.H * 128))
+        !tc_rows_map(&mm, a.Mb, (unsigned long long)s.H * 128, true))
+        return cudaErrorInvalidValue;
+    // without a snapshot buffer the map is a valid placeholder over M that is never used
+    if (!tc_rows_map(&msnap, a.snap ? (const void*)a.snap : (const void*)a.Mb,
+                     a.snap ? BH * (s.T / CT) * 2 * 128 : (unsigned long long)s.H * 128, true))
         return cudaErrorInvalidValue;
     cudaError_t e = launch_fwd_segment_states(a, k, v, Mf, st);
     if (e != cudaSuccess) return e;
@@ -563,7 +610,7 @@ cudaError_t launch_fwd_tc(const TcFwdArgs& a, const void* q, const void* k, cons
     const int smC = 2048 + 7 * TILE + 1024;
     auto kC = seg_out_tc<SEGC_DEFAULT>;
     cudaFuncSetAttribute(kC, cudaFuncAttributeMaxDynamicSharedMemorySize, smC);
-    { LaunchScope ls_("tc_seg_out", st); kC<<<grid, 512, smC, st>>>(mq, mk, mv, mm, a); }
+    { LaunchScope ls_("tc_seg_out", st); kC<<<grid, 512, smC, st>>>(mq, mk, mv, mm, msnap, a); }
     return cudaGetLastError();
 }
 

@@ -22,7 +22,7 @@ CYFA_WS_PREPARE, CYFA_WS_FWD, CYFA_WS_BWD = 0, 1, 2
 EXPORTS = ('cyfa_version', 'cyfa_error_string', 'cyfa_workspace_size', 'cyfa_prepare',
            'cyfa_chunk_fwd', 'cyfa_chunk_bwd', 'cyfa_step', 'cyfa_check', 'cyfa_stats_reset',
            'cyfa_stats_timing', 'cyfa_stats_get', 'cyfa_prepare_noalloc',
-           'cyfa_selftest_mma')
+           'cyfa_selftest_mma', 'cyfa_saved_size')
 
 
 class CyfaError(RuntimeError):
@@ -65,8 +65,9 @@ def load(path=LIB_PATH):
     lib.cyfa_error_string.argtypes = [ctypes.c_int]
     lib.cyfa_workspace_size.argtypes = [P, ctypes.c_int, ctypes.POINTER(ctypes.c_size_t)]
     lib.cyfa_prepare.argtypes = [P] + [_VP] * 9 + [_VP, ctypes.c_size_t, _VP]
-    lib.cyfa_chunk_fwd.argtypes = [P] + [_VP] * 13 + [ctypes.c_size_t, _VP]
-    lib.cyfa_chunk_bwd.argtypes = [P] + [_VP] * 20 + [ctypes.c_size_t, _VP]
+    lib.cyfa_saved_size.argtypes = [P, ctypes.POINTER(ctypes.c_size_t)]
+    lib.cyfa_chunk_fwd.argtypes = [P] + [_VP] * 14 + [ctypes.c_size_t, _VP]
+    lib.cyfa_chunk_bwd.argtypes = [P] + [_VP] * 21 + [ctypes.c_size_t, _VP]
     lib.cyfa_step.argtypes = [P] + [_VP] * 13
     lib.cyfa_check.argtypes = [_VP]
     lib.cyfa_selftest_mma.argtypes = [ctypes.c_int, _VP, _VP, _VP, _VP]
@@ -112,6 +113,18 @@ def workspace(d, which, device='cuda'):
     return torch.empty(max(1, cyfa_workspace_size(d, which)), dtype=torch.uint8, device=device)
 
 
+def cyfa_saved_size(d):
+    n = ctypes.c_size_t(0)
+    _ok(load().cyfa_saved_size(ctypes.byref(d), ctypes.byref(n)))
+    return n.value
+
+
+def saved_buffer(d, device='cuda'):
+    """Buffer for the forward's saved chunk-start states (None where nothing is saved)."""
+    n = cyfa_saved_size(d)
+    return torch.empty(n, dtype=torch.uint8, device=device) if n else None
+
+
 def cyfa_prepare(d, clock_logit, decay_logit, beta_logit, A, lambda0, lam_mod, g_cum, beta,
                  lambda_end, ws, stream=None):
     _ok(load().cyfa_prepare(ctypes.byref(d), _ptr(clock_logit), _ptr(decay_logit),
@@ -129,20 +142,22 @@ def cyfa_prepare_noalloc(d, clock_logit, decay_logit, beta_logit, A, lambda0, la
 
 
 def cyfa_chunk_fwd(d, q, k, v, lam_mod, g_cum, beta, R, Kbar0, Vbar0, o, Kbar_out, Vbar_out, ws,
-                   stream=None):
+                   stream=None, saved=None):
     _ok(load().cyfa_chunk_fwd(ctypes.byref(d), _ptr(q), _ptr(k), _ptr(v), _ptr(lam_mod),
                               _ptr(g_cum), _ptr(beta), _ptr(R), _ptr(Kbar0), _ptr(Vbar0), _ptr(o),
-                              _ptr(Kbar_out), _ptr(Vbar_out), _ptr(ws), ws.numel(),
+                              _ptr(Kbar_out), _ptr(Vbar_out), _ptr(saved), _ptr(ws), ws.numel(),
                               _stream(stream)))
 
 
 def cyfa_chunk_bwd(d, q, k, v, lam_mod, g_cum, beta, R, clock_logit, decay_logit, A, dO, dq, dk,
-                   dv, d_clock_logit, d_decay_logit, d_beta_logit, dR, dA, ws, stream=None):
+                   dv, d_clock_logit, d_decay_logit, d_beta_logit, dR, dA, ws, stream=None,
+                   saved=None):
     _ok(load().cyfa_chunk_bwd(ctypes.byref(d), _ptr(q), _ptr(k), _ptr(v), _ptr(lam_mod),
                               _ptr(g_cum), _ptr(beta), _ptr(R), _ptr(clock_logit),
                               _ptr(decay_logit), _ptr(A), _ptr(dO), _ptr(dq), _ptr(dk), _ptr(dv),
                               _ptr(d_clock_logit), _ptr(d_decay_logit), _ptr(d_beta_logit),
-                              _ptr(dR), _ptr(dA), _ptr(ws), ws.numel(), _stream(stream)))
+                              _ptr(dR), _ptr(dA), _ptr(saved), _ptr(ws), ws.numel(),
+                              _stream(stream)))
 
 
 def cyfa_step(d, q, k, v, clock_logit, decay_logit, beta_logit, A, R, Kbar, Vbar, lam, o,
@@ -196,7 +211,8 @@ def prepare(d, clock_logit, decay_logit, beta_logit, A, lambda0=None, want_lambd
     return lam, g, beta, lend
 
 
-def forward(d, q, k, v, lam, g, beta, R, Kbar0=None, Vbar0=None, want_state=False, ws=None):
+def forward(d, q, k, v, lam, g, beta, R, Kbar0=None, Vbar0=None, want_state=False, ws=None,
+            saved=None):
     o = torch.empty_like(v)
     B, T, H, D = v.shape
     Ko = Vo = None
@@ -205,5 +221,5 @@ def forward(d, q, k, v, lam, g, beta, R, Kbar0=None, Vbar0=None, want_state=Fals
         Vo = torch.empty_like(Ko)
     if ws is None:
         ws = workspace(d, CYFA_WS_FWD, v.device)
-    cyfa_chunk_fwd(d, q, k, v, lam, g, beta, R, Kbar0, Vbar0, o, Ko, Vo, ws)
+    cyfa_chunk_fwd(d, q, k, v, lam, g, beta, R, Kbar0, Vbar0, o, Ko, Vo, ws, saved=saved)
     return o, Ko, Vo

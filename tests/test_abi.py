@@ -5,6 +5,7 @@ import os
 import re
 
 import pytest
+import torch
 
 from paper_2609_36259_gb300 import cyfa
 
@@ -64,12 +65,24 @@ def test_bad_dims_rejected_on_host(lib, field, value, code):
 
 def test_null_and_misaligned_pointers_rejected_on_host(lib):
     d = cyfa.dims(1, 128, 1, 128)
-    nul = [None] * 13
+    nul = [None] * 14
     assert lib.cyfa_chunk_fwd(ctypes.byref(d), *nul, 0, None) == cyfa.CYFA_ERR_ARG
     bad = ctypes.c_void_p(0x1002)      # never dereferenced: rejected before any launch
     good = ctypes.c_void_p(0x1000)
-    args = [bad, good, good, good, good, good, good, None, None, good, None, None, good]
+    args = [bad, good, good, good, good, good, good, None, None, good, None, None, None, good]
     assert lib.cyfa_chunk_fwd(ctypes.byref(d), *args, 1 << 30, None) == cyfa.CYFA_ERR_ALIGN
-    args = [good] * 7 + [None, None, good, None, None, good]
+    args = [good] * 7 + [None, None, good, None, None, bad, good]   # misaligned saved buffer
+    assert lib.cyfa_chunk_fwd(ctypes.byref(d), *args, 1 << 30, None) == cyfa.CYFA_ERR_ALIGN
+    args = [good] * 7 + [None, None, good, None, None, None, good]
     assert lib.cyfa_chunk_fwd(ctypes.byref(d), *args, 16, None) == cyfa.CYFA_ERR_WORKSPACE
     assert lib.cyfa_step(ctypes.byref(d), *([None] * 13)) == cyfa.CYFA_ERR_ARG
+
+
+def test_saved_size(lib):
+    """The saved chunk-start states: fp16 [B*H][T/128][2][128][128] on the tensor-core path,
+    nothing on the CUDA-core kernels."""
+    B, T, H = 2, 1024, 3
+    assert cyfa.cyfa_saved_size(cyfa.dims(B, T, H, 128)) == B * H * (T // 128) * 2 * 128 * 128 * 2
+    assert cyfa.cyfa_saved_size(cyfa.dims(B, T, H, 128, cuda_cores=True)) == 0
+    assert cyfa.cyfa_saved_size(cyfa.dims(B, T, H, 64)) == 0
+    assert cyfa.cyfa_saved_size(cyfa.dims(B, T, H, 128, dtype=torch.float32)) == 0

@@ -15,9 +15,16 @@ GRADS = (('dq', 'dq'), ('dk', 'dk'), ('dv', 'dv'), ('d_clock', 'd_clock'),
          ('d_decay', 'd_decay'), ('d_beta', 'd_beta'))
 
 
-def gpu_backward(d, inp, want_dA=True):
+def gpu_backward(d, inp, want_dA=True, use_saved=False):
     lam, g, beta, _ = gpu_prepare(d, inp)
     q, k, v, dO = inp['q'], inp['k'], inp['v'], inp['dO']
+    saved = None
+    if use_saved:   # a forward that saves its chunk-start states for this backward
+        saved = cyfa.saved_buffer(d, q.device)
+        assert saved is not None
+        o_plain = cyfa.forward(d, q, k, v, lam, g, beta, inp['R'])[0]
+        o_saving = cyfa.forward(d, q, k, v, lam, g, beta, inp['R'], saved=saved)[0]
+        assert torch.equal(o_plain, o_saving)   # saving does not change the forward
     out = dict(dq=torch.empty_like(q), dk=torch.empty_like(k), dv=torch.empty_like(v),
                d_clock=torch.empty_like(inp['clock_logit']),
                d_decay=torch.empty_like(inp['clock_logit']),
@@ -26,7 +33,8 @@ def gpu_backward(d, inp, want_dA=True):
     ws = cyfa.workspace(d, cyfa.CYFA_WS_BWD, q.device)
     cyfa.cyfa_chunk_bwd(d, q, k, v, lam, g, beta, inp['R'], inp['clock_logit'],
                         inp['decay_logit'], inp['A'], dO, out['dq'], out['dk'], out['dv'],
-                        out['d_clock'], out['d_decay'], out['d_beta'], None, out['dA'], ws)
+                        out['d_clock'], out['d_decay'], out['d_beta'], None, out['dA'], ws,
+                        saved=saved)
     torch.cuda.synchronize()
     return out
 
@@ -83,3 +91,26 @@ def test_backward_full_size_sampled(B, T, H, C, cuda_cores):
     pairs = sample_pairs(B, H, 2)
     ref = oracle_backward(oracle_inputs(inp, pairs), pairs_np(inp['dO'], pairs))
     _compare(out, ref, pairs, assert_close_bf16, 'B%d T%d' % (B, T))
+
+
+@pytest.mark.parametrize('B,T,H', [(2, 256, 2), (1, 2304, 2), (2, 1152, 3)])
+def test_backward_saved_states(B, T, H):
+    """The backward reading the forward's saved chunk-start states instead of recomputing them
+    (one segment, several segments plus a partial one, odd head count)."""
+    inp = to_device(synth.make_inputs(B, T, H, 128, seed=11, with_dO=True))
+    d = cyfa.dims(B, T, H, 128, chunk=64)
+    out = gpu_backward(d, inp, use_saved=True)
+    pairs = [(b, h) for b in range(B) for h in range(H)]
+    ref = oracle_backward(oracle_inputs(inp, pairs), pairs_np(inp['dO'], pairs))
+    _compare(out, ref, pairs, assert_close_bf16, 'saved')
+
+
+def test_backward_saved_full_size_sampled():
+    """The 1.4B-shaped layer (B2 H16 T32768) with saved states, as the bench step runs it."""
+    B, T, H = 2, 32768, 16
+    inp = synth.make_inputs(B, T, H, 128, seed=1, device='cuda', with_dO=True)
+    d = cyfa.dims(B, T, H, 128, chunk=64)
+    out = gpu_backward(d, inp, want_dA=False, use_saved=True)
+    pairs = sample_pairs(B, H, 2)
+    ref = oracle_backward(oracle_inputs(inp, pairs), pairs_np(inp['dO'], pairs))
+    _compare(out, ref, pairs, assert_close_bf16, 'saved full')
