@@ -364,11 +364,12 @@ def load_traffic(kernel):
     ent = j.get(kernel)
     if not ent:
         return None
-    src = os.path.join(ROOT, ent['source'])
-    if not os.path.exists(src):
-        return None
-    sha = hashlib.sha256(open(src, 'rb').read()).hexdigest()
-    return ent['bytes_per_launch'] if sha == ent.get('source_sha256') else None
+    srcs = ent.get('sources') or {ent['source']: ent.get('source_sha256')}
+    for rel, want in srcs.items():
+        src = os.path.join(ROOT, rel)
+        if not os.path.exists(src) or hashlib.sha256(open(src, 'rb').read()).hexdigest() != want:
+            return None
+    return ent['bytes_per_launch']
 
 
 def run_decode(args, dev, peaks, rank):
@@ -485,12 +486,12 @@ def run_reference(args):
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument('--gpus', type=int, default=1)
-    ap.add_argument('--steps', type=int, default=5)
-    ap.add_argument('--warmup', type=int, default=3)
+    ap.add_argument('--steps', type=int, default=200)
+    ap.add_argument('--warmup', type=int, default=5)
     ap.add_argument('--impl', default='ours', choices=['ours', 'reference'])
     ap.add_argument('--chunk', type=int, default=64, choices=[64, 128])
     ap.add_argument('--decode-steps', type=int, default=1024)
-    ap.add_argument('--cpu-tokens', type=int, default=2048)
+    ap.add_argument('--cpu-tokens', type=int, default=32768)
     ap.add_argument('--shape', default=None,
                     help='B,T,H override of the layer shape (profiling runs on smaller cases)')
     ap.add_argument('--ref-tokens', type=int, default=256)
