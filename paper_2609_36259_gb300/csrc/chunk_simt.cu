@@ -18,22 +18,28 @@ namespace {
 // Phi is the real Fourier basis of App. A.1 Eq. app-real-fourier.
 __global__ void __launch_bounds__(128) readout_matrix_kernel(const float* R, float* M, float* MT) {
     const int h = blockIdx.y, i = blockIdx.x, col = threadIdx.x;
-    __shared__ float srow[128];
+    __shared__ float srow[128], s_ct[MA], s_st[MA];
     srow[col] = (i < MA && col < MA) ? R[((size_t)h * MA + i) * MA + col] : 0.f;
+    if (col < MA) {   // cos / sin of 2 pi x / m for x = 0 .. m-1 (the entries of Phi)
+        float sv, cv;
+        sincospif((float)col * (2.f / 127.f), &sv, &cv);
+        s_ct[col] = cv;
+        s_st[col] = sv;
+    }
     __syncthreads();
     float acc = 0.f;
     if (i < MA && col < MA) {
-        const int j = (col + 1) >> 1;
-        for (int r = 0; r < MA; ++r) {
-            float phi;
-            if (col == 0) {
-                phi = INV_SQRT_M;
-            } else {
-                float s, c;
-                sincospif((float)((j * r) % MA) * (2.f / 127.f), &s, &c);
-                phi = SQRT_2_OVER_M * ((col & 1) ? c : s);
+        if (col == 0) {
+            for (int r = 0; r < MA; ++r) acc = fmaf(srow[r], INV_SQRT_M, acc);
+        } else {
+            const int j = (col + 1) >> 1;
+            const float* tab = (col & 1) ? s_ct : s_st;
+            int idx = 0;   // (j r) mod m
+            for (int r = 0; r < MA; ++r) {
+                acc = fmaf(srow[r], SQRT_2_OVER_M * tab[idx], acc);
+                idx += j;
+                if (idx >= MA) idx -= MA;
             }
-            acc = fmaf(srow[r], phi, acc);
         }
     }
     M[((size_t)h * MS + i) * MS + col] = acc;

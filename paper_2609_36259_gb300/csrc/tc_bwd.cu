@@ -819,16 +819,16 @@ __global__ void __launch_bounds__(256) seg_scan_rev_kernel(TcBwdArgs a) {
     float* base = a.segD + (size_t)bh * a.nseg * 128 * 256 + e;
     const float* G = a.segG + (size_t)bh * a.nseg;
     float cur = 0.f;
-    for (int j1 = a.nseg - 1; j1 >= 0; j1 -= 8) {
-        float d[8], gj[8];
+    for (int j1 = a.nseg - 1; j1 >= 0; j1 -= 32) {
+        float d[32], gj[32];   // all loads first: the stores below may alias them
 #pragma unroll
-        for (int u = 0; u < 8; ++u) {
+        for (int u = 0; u < 32; ++u) {
             const int j = j1 - u;
             d[u] = j >= 0 ? base[(size_t)j * 128 * 256] : 0.f;
             gj[u] = j >= 0 ? G[j] : 0.f;
         }
 #pragma unroll
-        for (int u = 0; u < 8; ++u) {
+        for (int u = 0; u < 32; ++u) {
             const int j = j1 - u;
             if (j >= 0) {
                 base[(size_t)j * 128 * 256] = cur;

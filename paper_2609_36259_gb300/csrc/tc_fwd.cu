@@ -140,7 +140,7 @@ __global__ void __launch_bounds__(256, 1) seg_state_tc(const __grid_constant__ C
 
 // Segment-start states: S_start(0) = initial state, S_start(j+1) = exp(G_j) S_start(j) + dS(j),
 // in place over the dS buffer (tensor-core row order); the final state goes to Kout / Vout in
-// the paper's row order.  Eight segments are loaded before they are folded in.
+// the paper's row order.  Up to 32 segments are loaded before they are folded in.
 __global__ void __launch_bounds__(256) seg_scan_kernel(TcFwdArgs a) {
     const int bh = blockIdx.y;
     const int e = blockIdx.x * 256 + threadIdx.x;   // element of the [128 x 256] state block
@@ -153,16 +153,16 @@ __global__ void __launch_bounds__(256) seg_scan_kernel(TcFwdArgs a) {
     if (init) S = init[((size_t)bh * 128 + prow) * 128 + dcol];
     float* base = a.segS + (size_t)bh * a.nseg * 128 * 256 + e;
     const float* G = a.segG + (size_t)bh * a.nseg;
-    for (int j0 = 0; j0 < a.nseg; j0 += 8) {
-        float d[8], gj[8];
+    for (int j0 = 0; j0 < a.nseg; j0 += 32) {
+        float d[32], gj[32];   // all loads first: the stores below may alias them
 #pragma unroll
-        for (int u = 0; u < 8; ++u) {
+        for (int u = 0; u < 32; ++u) {
             const bool in = j0 + u < a.nseg;
             d[u] = in ? base[(size_t)(j0 + u) * 128 * 256] : 0.f;
             gj[u] = in ? G[j0 + u] : 0.f;
         }
 #pragma unroll
-        for (int u = 0; u < 8; ++u) {
+        for (int u = 0; u < 32; ++u) {
             if (j0 + u < a.nseg) {
                 base[(size_t)(j0 + u) * 128 * 256] = S;
                 S = expf(gj[u]) * S + d[u];
@@ -194,7 +194,7 @@ __global__ void __launch_bounds__(512, 1) seg_out_tc(const __grid_constant__ CUt
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                                ~uintptr_t(1023));
-    uint64_t* bars = reinterpret_cast<uint64_t*>(smem);          // tma, mma, m
+    uint64_t* bars = reinterpret_cast<uint64_t*>(smem);          // tma q k, mma, m, tma v
     uint32_t* s_taddr = reinterpret_cast<uint32_t*>(smem + 32);
     float* s_g2 = reinterpret_cast<float*>(smem + 64);            // [128] log2-domain decays
     uint8_t* T_Q = smem + 2048;        // Q, later A-> (state-update operand)
@@ -206,7 +206,7 @@ __global__ void __launch_bounds__(512, 1) seg_out_tc(const __grid_constant__ CUt
     uint8_t* T_M = T_Q + 6 * TILE;     // M = R Phi (rows = slots r, cols = Fourier index)
 
     if (tid == 0) {
-        for (int i = 0; i < 3; ++i) mbar_init(&bars[i], 1);
+        for (int i = 0; i < 4; ++i) mbar_init(&bars[i], 1);
         fence_mbar_init();
     }
     if (ro.warp == 0) tmem_alloc(s_taddr, 512);
@@ -217,21 +217,31 @@ __global__ void __launch_bounds__(512, 1) seg_out_tc(const __grid_constant__ CUt
     const uint32_t tl = taddr + ((uint32_t)(32 * ro.q) << 16) + c0;   // lane, column quarter
     const uint32_t SK = 0, SV = 128, X1 = 256, X2 = 384;
 
-    auto issue_qkv = [&](int c) {
+    // Q and K of a chunk are loaded as soon as the previous chunk's state update has read T_Q
+    // and T_K; V as soon as its P2 V product has read T_V.  (Thread 0 tracks what is in flight.)
+    bool qk_pending = false, v_pending = false;
+    auto issue_qk = [&](int c) {
         const int r0 = b * s.T + (c_begin + c) * CT;
-        mbar_expect_tx(&bars[0], 3 * TILE);
+        mbar_expect_tx(&bars[0], 2 * TILE);
         tma_load_3d(T_Q, &tq, 0, h, r0, &bars[0]);
         tma_load_3d(T_Q + TILE / 2, &tq, 64, h, r0, &bars[0]);
         tma_load_3d(T_K, &tk, 0, h, r0, &bars[0]);
         tma_load_3d(T_K + TILE / 2, &tk, 64, h, r0, &bars[0]);
-        tma_load_3d(T_V, &tv, 0, h, r0, &bars[0]);
-        tma_load_3d(T_V + TILE / 2, &tv, 64, h, r0, &bars[0]);
+        qk_pending = true;
+    };
+    auto issue_v = [&](int c) {
+        const int r0 = b * s.T + (c_begin + c) * CT;
+        mbar_expect_tx(&bars[3], TILE);
+        tma_load_3d(T_V, &tv, 0, h, r0, &bars[3]);
+        tma_load_3d(T_V + TILE / 2, &tv, 64, h, r0, &bars[3]);
+        v_pending = true;
     };
     if (tid == 0) {
         mbar_expect_tx(&bars[2], TILE);
         tma_load_2d(T_M, &tm, 0, h * 128, &bars[2]);
         tma_load_2d(T_M + TILE / 2, &tm, 64, h * 128, &bars[2]);
-        issue_qkv(0);
+        issue_qk(0);
+        issue_v(0);
     }
     // segment-start state into TMEM; Kbar snapshot into T_N (row = slot)
     {
@@ -254,7 +264,7 @@ __global__ void __launch_bounds__(512, 1) seg_out_tc(const __grid_constant__ CUt
     tc_fence_after();
     bool ok = mbar_wait(&bars[2], 0);
     ok = __syncthreads_and(ok);
-    uint32_t tma_ph = 0, mma_ph = 0;
+    uint32_t qk_ph = 0, v_ph = 0, mma_ph = 0;
     const float scale = s.scale;
     const uint32_t id_kk = idesc_f16(128, 128, 0, 0);
     const uint32_t id_kn = idesc_f16(128, 128, 0, 1);
@@ -304,36 +314,44 @@ __global__ void __launch_bounds__(512, 1) seg_out_tc(const __grid_constant__ CUt
         }
     };
 
-    // gates of the first chunk; later chunks are prefetched one chunk ahead
-    float n_lam, n_beta, n_g;
+    // Set-up of a chunk that needs no product of the previous one: its decays, its write vectors
+    // (T_A) and its Q, K tiles (waited for and converted to fp16).  For chunk c + 1 it runs while
+    // chunk c's last product (P2 V) is in flight.
+    auto chunk_setup = [&](float lam_, float beta_, float g2_) {
+        if (cq == 0) s_g2[row] = g2_;
+        write_vector_q<__half>(T_A, row, hf, u, lam_, beta_);
+        if (ok) ok = mbar_wait(&bars[0], qk_ph);
+        if (tid == 0 && ok) qk_pending = false;
+        qk_ph ^= 1;
+        if (ok) {
+            bf16_to_f16_q(T_Q, row, c0);
+            bf16_to_f16_q(T_K, row, c0);
+        }
+    };
+    // gates of the current and of the next chunk (prefetched one chunk ahead: the loads are
+    // issued a chunk before their values are combined, so their latency is never waited for)
+    float lam, beta, g2;
+    float n_lam = 0.f, n_beta = 0.f, n_ga = 0.f, n_gb = 0.f;
+    auto load_gates = [&](int c, float& l_, float& b_, float& ga, float& gb) {
+        const int t0 = (c_begin + c) * CT, t = t0 + row;
+        const size_t gi = ((size_t)b * s.T + t) * s.H + h;
+        l_ = a.lam[gi];
+        b_ = a.beta[gi];
+        // cum128 in two loads: g_cum is local to s.Cg-token chunks
+        ga = a.g[gi];
+        gb = (s.Cg == 64 && t - t0 >= 64) ? a.g[((size_t)b * s.T + t0 + 63) * s.H + h] : 0.f;
+    };
     {
-        const int t0 = c_begin * CT;
-        const size_t gi = ((size_t)b * s.T + t0 + row) * s.H + h;
-        n_lam = a.lam[gi];
-        n_beta = a.beta[gi];
-        n_g = cum128(s, a.g, b, h, t0, t0 + row);
+        float ga, gb;
+        load_gates(0, lam, beta, ga, gb);
+        g2 = (ga + gb) * LOG2E;
     }
+    chunk_setup(lam, beta, g2);
+    publish();
     for (int c = 0; c < nc && ok; ++c) {
         const int t0 = (c_begin + c) * CT;
         const size_t gi = ((size_t)b * s.T + t0 + row) * s.H + h;
-        const float lam = n_lam, beta = n_beta, g2 = n_g * LOG2E;
-        if (c + 1 < nc) {
-            const int t1 = t0 + CT;
-            const size_t g1 = ((size_t)b * s.T + t1 + row) * s.H + h;
-            n_lam = a.lam[g1];
-            n_beta = a.beta[g1];
-            n_g = cum128(s, a.g, b, h, t1, t1 + row);
-        }
-        if (cq == 0) s_g2[row] = g2;
-        write_vector_q<__half>(T_A, row, hf, u, lam, beta);
-        if (ok) ok = mbar_wait(&bars[0], tma_ph);
-        if (ok) {   // Q, K, V: bf16 -> fp16
-            bf16_to_f16_q(T_Q, row, c0);
-            bf16_to_f16_q(T_K, row, c0);
-            bf16_to_f16_q(T_V, row, c0);
-        }
-        publish();
-        if (!ok) break;
+        if (c + 1 < nc) load_gates(c + 1, n_lam, n_beta, n_ga, n_gb);
         const float g2C = s_g2[CT - 1];
         const float gam = ex2(g2);
         if (save && tid == 0) store_snap(c_begin + c, 0);
@@ -349,7 +367,6 @@ __global__ void __launch_bounds__(512, 1) seg_out_tc(const __grid_constant__ CUt
                 mma_commit(&bars[1]);
             }
         }
-        tma_ph ^= 1;
         wait_mma();
         {   // P1 = s (Q K^T) o Gamma
             float x[32];
@@ -381,6 +398,10 @@ __global__ void __launch_bounds__(512, 1) seg_out_tc(const __grid_constant__ CUt
             for (int i = 0; i < 32; ++i) x[i] *= gC;
             tmem_st16x2(tl + SV, x);
         }
+        if (ok) ok = mbar_wait(&bars[3], v_ph);   // V: the state update reads it next
+        if (tid == 0 && ok) v_pending = false;
+        v_ph ^= 1;
+        if (ok) bf16_to_f16_q(T_V, row, c0);
         publish();
         if (!ok) break;
         if (save && tid == 0) store_snap(c_begin + c, 1);
@@ -411,6 +432,7 @@ __global__ void __launch_bounds__(512, 1) seg_out_tc(const __grid_constant__ CUt
             mma_commit(&bars[1]);
         }
         wait_mma();   // also covers the state update issued before this commit
+        if (issuer() && c + 1 < nc) issue_qk(c + 1);   // T_Q (A->) and T_K are consumed
         {   // p = softmax over the 127 active slots of l = z M^T; the staging tile (z is
             // consumed) holds the row reductions over the four column quarters
             float* red = reinterpret_cast<float*>(T_S);
@@ -479,9 +501,15 @@ __global__ void __launch_bounds__(512, 1) seg_out_tc(const __grid_constant__ CUt
                 mma_bf16(taddr + X1, kmajor_desc(uS, 128, k), mnmajor_desc(uV, 128, k), id_kn, k > 0);
             mma_commit(&bars[1]);
         }
+        if (c + 1 < nc) {   // while P2 V runs: the next chunk's set-up (T_A, T_Q, T_K are free)
+            lam = n_lam;
+            beta = n_beta;
+            g2 = (n_ga + n_gb) * LOG2E;
+            chunk_setup(lam, beta, g2);
+        }
         wait_mma();
-        // next chunk's tiles (Q, K, V are consumed), then o = gamma_r (O'' Vbar) + P2 V
-        if (issuer() && c + 1 < nc) issue_qkv(c + 1);
+        // next chunk's V (T_V is consumed), then o = gamma_r (O'' Vbar) + P2 V
+        if (issuer() && c + 1 < nc) issue_v(c + 1);
         {
             float x[32], y[32];
             tmem_ld16x2(tl + X2, x);
@@ -499,7 +527,9 @@ __global__ void __launch_bounds__(512, 1) seg_out_tc(const __grid_constant__ CUt
     }
     if (!ok && tid == 0) {
         flag_error(CYFA_ERR_TIMEOUT);
-        mbar_wait(&bars[0], tma_ph);   // let copies still in flight land
+        // let copies still in flight land before the shared memory is released
+        if (qk_pending) mbar_wait(&bars[0], qk_ph);
+        if (v_pending) mbar_wait(&bars[3], v_ph);
     }
     if (save && tid == 0) bulk_wait_all();
     tc_fence_before();
