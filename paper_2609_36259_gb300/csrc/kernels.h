@@ -110,11 +110,12 @@ cudaError_t launch_fwd_tc(const TcFwdArgs& a, const void* q, const void* k, cons
 // Reads (and clears) the error word of the tensor-core kernels; synchronises the stream.
 cudaError_t tc_read_error(cudaStream_t st, int* err);
 cudaError_t tc_bwd_read_error(cudaStream_t st, int* err);
-// TMA maps of [B, T, H, 128] bf16 tensors (128-token boxes of one head) and of row-major
-// [rows x 128] bf16 arrays (128-row boxes); null outputs are skipped.
+// TMA maps of [B, T, H, 128] bf16 tensors (boxes of box_rows tokens of one head) and of
+// row-major [rows x 128] 16-bit arrays (box_rows-row boxes); null outputs are skipped.
 bool tc_qkv_maps(const Shape& s, const void* q, const void* k, const void* v, CUtensorMap* mq,
-                 CUtensorMap* mk, CUtensorMap* mv);
-bool tc_rows_map(CUtensorMap* map, const void* base, unsigned long long rows, bool f16 = false);
+                 CUtensorMap* mk, CUtensorMap* mv, unsigned box_rows = 128);
+bool tc_rows_map(CUtensorMap* map, const void* base, unsigned long long rows, bool f16 = false,
+                 unsigned box_rows = 128);
 // M -> fp16 (tensor-core order), segment state contributions, segment scan.
 cudaError_t launch_fwd_segment_states(const TcFwdArgs& a, const void* k, const void* v,
                                       const float* Mf, cudaStream_t st);

@@ -89,34 +89,6 @@ __device__ __forceinline__ void scale_half_smem(uint8_t* tile, int r, int hf, fl
     store_half_bf16<__half>(tile, r, hf, x);
 }
 
-// Fourier-axis write vector of a token on this thread's column half, in fp32 (tensor-core order).
-__device__ __forceinline__ void write_vector_vals(float (&x)[64], int hf, float lam, float w) {
-    HalfAngles ang(lam, hf);
-    const float wa = w * SQRT_2_OVER_M;
-#pragma unroll
-    for (int jj = 0; jj < 32; ++jj) {
-        if (jj > 0) ang.step(jj);
-        x[jj] = wa * ang.c;
-        x[jj + 32] = -wa * ang.s;
-    }
-    if (hf == 1) {
-        x[31] = w * INV_SQRT_M;
-        x[63] = 0.f;
-    }
-}
-
-// <x, Omega y> restricted to the pairs of this column half (tensor-core order):
-// sum_j (2 pi j / m) (x_sin,j y_cos,j - x_cos,j y_sin,j).
-__device__ __forceinline__ float omega_dot_half(const float (&x)[64], const float (&y)[64], int hf) {
-    float acc = 0.f;
-#pragma unroll
-    for (int jj = 0; jj < 32; ++jj) {
-        const int j = 32 * hf + jj + 1;
-        if (j <= NPAIR) acc += (6.283185307179586f * (float)j / 127.f) * (x[jj + 32] * y[jj] - x[jj] * y[jj + 32]);
-    }
-    return acc;
-}
-
 __device__ __forceinline__ float dot64(const float (&x)[64], const float (&y)[64]) {
     float acc = 0.f;
 #pragma unroll
@@ -130,7 +102,7 @@ __global__ void __launch_bounds__(256, 1) snap_fwd_tc(const __grid_constant__ CU
                                                        const __grid_constant__ CUtensorMap tv,
                                                        TcBwdArgs a) {
     const Shape s = a.s;
-    const int seg = blockIdx.x, bh = blockIdx.y, b = bh / s.H, h = bh % s.H;
+    const int bh = blockIdx.x, seg = blockIdx.y, b = bh / s.H, h = bh % s.H;
     const int nct = s.T / CT;
     const int c_begin = seg * TC_SEGC;
     const int nc = min(TC_SEGC, nct - c_begin);
@@ -250,7 +222,7 @@ __global__ void __launch_bounds__(512, 1) bwd_chunk1_tc(const __grid_constant__ 
                                                          const __grid_constant__ CUtensorMap tsf,
                                                          TcBwdArgs a) {
     const Shape s = a.s;
-    const int cg = blockIdx.x, bh = blockIdx.y, b = bh / s.H, h = bh % s.H;
+    const int bh = blockIdx.x, cg = blockIdx.y, b = bh / s.H, h = bh % s.H;
     const int nct = s.T / CT, t0 = cg * CT;
     const int tid = threadIdx.x;
     const QRole ro;
@@ -625,7 +597,7 @@ __global__ void __launch_bounds__(256, 1) adj_walk_tc(const __grid_constant__ CU
                                                        const __grid_constant__ CUtensorMap tsa,
                                                        TcBwdArgs a) {
     const Shape s = a.s;
-    const int seg = blockIdx.x, bh = blockIdx.y, b = bh / s.H, h = bh % s.H;
+    const int bh = blockIdx.x, seg = blockIdx.y, b = bh / s.H, h = bh % s.H;
     const int nct = s.T / CT;
     const int c_begin = seg * TC_SEGC;
     const int nc = min(TC_SEGC, nct - c_begin);
@@ -640,8 +612,13 @@ __global__ void __launch_bounds__(256, 1) adj_walk_tc(const __grid_constant__ CU
     float* s_tot = reinterpret_cast<float*>(smem + 128);   // [TC_SEGC]
     float* s_pre = s_tot + TC_SEGC;                         // [TC_SEGC]
     float* s_bnd = s_pre + TC_SEGC;                         // [TC_SEGC][2]
+    float* s_gs = reinterpret_cast<float*>(smem + 1024);    // [TC_SEGC * CT] chunk-local decays
     constexpr int NT = SNAP ? 3 : 2;                       // tiles per buffer
-    uint8_t* tiles = smem + 1024;                          // [buf][X | Y (| S)]
+    uint8_t* tiles = smem + 1024 + 4 * TC_SEGC * CT;       // [buf][X | Y (| S)]
+    for (int i = tid; i < nc * CT; i += 256) {   // every token's decay, loaded once
+        const int t0 = (c_begin + i / CT) * CT;
+        s_gs[i] = cum128(s, a.g, b, h, t0, t0 + (i % CT));
+    }
     if (tid == 0) {
         for (int i = 0; i < 4; ++i) mbar_init(&bars[i], 1);
         fence_mbar_init();
@@ -711,7 +688,7 @@ __global__ void __launch_bounds__(256, 1) adj_walk_tc(const __grid_constant__ CU
     const uint32_t id_nn = idesc_f16(128, 128, 1, 1);
     for (int it = 0; it < total; ++it) {
         const int part = it / nc, c = chunk_of(it), buf = it & 1;
-        const int cg = c_begin + c, t0 = cg * CT;
+        const int cg = c_begin + c;
         if (it >= 1 && ok) ok = mbar_wait(&bars[2 + ((it - 1) & 1)], ((it - 1) >> 1) & 1);
         tc_fence_after();
         if (tid == 0 && ok && it + 1 < total) {
@@ -719,7 +696,7 @@ __global__ void __launch_bounds__(256, 1) adj_walk_tc(const __grid_constant__ CU
             issue(it + 1);
         }
         if (ok) ok = mbar_wait(&bars[buf], (it >> 1) & 1);
-        const float g = cum128(s, a.g, b, h, t0, t0 + row);
+        const float g = s_gs[c * CT + row];
         uint8_t* tX = tiles + (NT * buf) * TILE;
         float w;
         if (SNAP) {
@@ -852,7 +829,7 @@ __global__ void __launch_bounds__(512, 1) bwd_chunk2_tc(const __grid_constant__ 
                                                          const __grid_constant__ CUtensorMap tsa,
                                                          TcBwdArgs a) {
     const Shape s = a.s;
-    const int cg = blockIdx.x, bh = blockIdx.y, b = bh / s.H, h = bh % s.H;
+    const int bh = blockIdx.x, cg = blockIdx.y, b = bh / s.H, h = bh % s.H;
     const int nct = s.T / CT, t0 = cg * CT;
     const int tid = threadIdx.x;
     const QRole ro;
@@ -1118,7 +1095,7 @@ __global__ void __launch_bounds__(512, 1) bwd_chunk2_tc(const __grid_constant__ 
 // state-level term of everything after the chunk, then the activation derivatives.
 __global__ void __launch_bounds__(128) tc_gate_kernel(TcBwdArgs a) {
     const Shape s = a.s;
-    const int cg = blockIdx.x, bh = blockIdx.y, b = bh / s.H, h = bh % s.H;
+    const int bh = blockIdx.x, cg = blockIdx.y, b = bh / s.H, h = bh % s.H;
     const int nct = s.T / CT, tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const size_t BTH = (size_t)s.B * s.T * s.H;
     const size_t gi = ((size_t)b * s.T + cg * CT + tid) * s.H + h;
@@ -1223,8 +1200,11 @@ cudaError_t launch_bwd_tc(const TcBwdArgs& a, const TcFwdArgs& f, const void* q,
     cudaError_t e = a.saved ? launch_m_and_segment_decay(f, Mf, st)
                             : launch_fwd_segment_states(f, k, v, Mf, st);
     if (e != cudaSuccess) return e;
-    const dim3 gseg(a.nseg, s.B * s.H), gchunk(nct, s.B * s.H);
-    const int sm_walk6 = 1024 + 6 * TILE + 1024, sm_walk4 = 1024 + 4 * TILE + 1024;
+    // heads fastest: the CTAs that read the same token rows of q, k, v, dO run together
+    const dim3 gseg(s.B * s.H, a.nseg), gchunk(s.B * s.H, nct);
+    const int sm_walk6 = 1024 + 6 * TILE + 1024;
+    const int sm_snap_adj = 1024 + 4 * TC_SEGC * CT + 6 * TILE + 1024;
+    const int sm_adj_seg = 1024 + 4 * TC_SEGC * CT + 4 * TILE + 1024;
     const int sm_chunk1 = 5120 + 6 * TILE + 1024, sm_chunk2 = 2048 + 7 * TILE + 1024;
     if (!a.saved) {
         cudaFuncSetAttribute(snap_fwd_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, sm_walk6);
@@ -1232,11 +1212,11 @@ cudaError_t launch_bwd_tc(const TcBwdArgs& a, const TcFwdArgs& f, const void* q,
     }
     cudaFuncSetAttribute(bwd_chunk1_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, sm_chunk1);
     { LaunchScope ls_("tc_bwd_chunk1", st); bwd_chunk1_tc<<<gchunk, 512, sm_chunk1, st>>>(mq, mk, mv, mdo, mm, msf, a); }
-    cudaFuncSetAttribute(adj_walk_tc<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, sm_walk4);
-    { LaunchScope ls_("tc_adj_segment", st); adj_walk_tc<false><<<gseg, 256, sm_walk4, st>>>(mdo1, mo2, mq, mdo, msf, msa, a); }
+    cudaFuncSetAttribute(adj_walk_tc<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, sm_adj_seg);
+    { LaunchScope ls_("tc_adj_segment", st); adj_walk_tc<false><<<gseg, 256, sm_adj_seg, st>>>(mdo1, mo2, mq, mdo, msf, msa, a); }
     { LaunchScope ls_("tc_adj_scan", st); seg_scan_rev_kernel<<<dim3(128, s.B * s.H), 256, 0, st>>>(a); }
-    cudaFuncSetAttribute(adj_walk_tc<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, sm_walk6);
-    { LaunchScope ls_("tc_snap_adj", st); adj_walk_tc<true><<<gseg, 256, sm_walk6, st>>>(mdo1, mo2, mq, mdo, msf, msa, a); }
+    cudaFuncSetAttribute(adj_walk_tc<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, sm_snap_adj);
+    { LaunchScope ls_("tc_snap_adj", st); adj_walk_tc<true><<<gseg, 256, sm_snap_adj, st>>>(mdo1, mo2, mq, mdo, msf, msa, a); }
     cudaFuncSetAttribute(bwd_chunk2_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, sm_chunk2);
     { LaunchScope ls_("tc_bwd_chunk2", st); bwd_chunk2_tc<<<gchunk, 512, sm_chunk2, st>>>(mq, mk, mv, mdo, mo2, mdo1, msa, a); }
     { LaunchScope ls_("tc_gate", st); tc_gate_kernel<<<gchunk, 128, 0, st>>>(a); }

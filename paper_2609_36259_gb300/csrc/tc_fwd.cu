@@ -25,7 +25,7 @@ __global__ void __launch_bounds__(256, 1) seg_state_tc(const __grid_constant__ C
                                                         const __grid_constant__ CUtensorMap tv,
                                                         TcFwdArgs a) {
     const Shape s = a.s;
-    const int seg = blockIdx.x, bh = blockIdx.y, b = bh / s.H, h = bh % s.H;
+    const int bh = blockIdx.x, seg = blockIdx.y, b = bh / s.H, h = bh % s.H;
     const int nct = s.T / CT;
     const int c_begin = seg * SEGC;
     const int nc = min(SEGC, nct - c_begin);
@@ -38,7 +38,17 @@ __global__ void __launch_bounds__(256, 1) seg_state_tc(const __grid_constant__ C
     uint32_t* s_taddr = reinterpret_cast<uint32_t*>(smem + 64);
     float* s_tot = reinterpret_cast<float*>(smem + 128);             // [SEGC]
     float* s_sfx = s_tot + SEGC;                                     // [SEGC]
-    uint8_t* tiles = smem + 1024;                                    // [buf][A | K | V]
+    float* s_lam = reinterpret_cast<float*>(smem + 1024);            // [SEGC * CT] per token
+    float* s_beta = s_lam + SEGC * CT;
+    float* s_gs = s_beta + SEGC * CT;                                // chunk-local decays
+    uint8_t* tiles = smem + 1024 + 12 * SEGC * CT;                   // [buf][A | K | V]
+    for (int i = tid; i < nc * CT; i += 256) {   // every token's gates, loaded once
+        const int t0 = (c_begin + i / CT) * CT, t = t0 + i % CT;
+        const size_t gi = ((size_t)b * s.T + t) * s.H + h;
+        s_lam[i] = a.lam[gi];
+        s_beta[i] = a.beta[gi];
+        s_gs[i] = cum128(s, a.g, b, h, t0, t);
+    }
 
     if (tid == 0) {
         for (int i = 0; i < 4; ++i) mbar_init(&bars[i], 1);
@@ -82,11 +92,9 @@ __global__ void __launch_bounds__(256, 1) seg_state_tc(const __grid_constant__ C
         if (tid == 0 && ok && c + 1 < nc) issue_kv(c + 1, (c + 1) & 1);
         // A-> rows of this chunk, scaled by the decay from the token to the segment end
         {
-            const int t0 = (c_begin + c) * CT, t = t0 + ro.row;
-            const size_t gi = ((size_t)b * s.T + t) * s.H + h;
-            const float w = a.beta[gi] *
-                            ex2((s_tot[c] - cum128(s, a.g, b, h, t0, t) + s_sfx[c]) * LOG2E);
-            write_vector_half<OT>(tiles + 3 * buf * TILE, ro.row, ro.hf, a.lam[gi], w);
+            const int i = c * CT + ro.row;
+            const float w = s_beta[i] * ex2((s_tot[c] - s_gs[i] + s_sfx[c]) * LOG2E);
+            write_vector_half<OT>(tiles + 3 * buf * TILE, ro.row, ro.hf, s_lam[i], w);
         }
         if (F16) {   // the bf16 K and V tiles become fp16 operands
             if (ok) ok = mbar_wait(&bars[buf], (c >> 1) & 1);
@@ -184,7 +192,7 @@ __global__ void __launch_bounds__(512, 1) seg_out_tc(const __grid_constant__ CUt
                                                       const __grid_constant__ CUtensorMap tsnap,
                                                       TcFwdArgs a) {
     const Shape s = a.s;
-    const int seg = blockIdx.x, bh = blockIdx.y, b = bh / s.H, h = bh % s.H;
+    const int bh = blockIdx.x, seg = blockIdx.y, b = bh / s.H, h = bh % s.H;
     const int nct = s.T / CT;
     const int c_begin = seg * SEGC;
     const int nc = min(SEGC, nct - c_begin);
@@ -575,20 +583,21 @@ int tc_fwd_segments(const Shape& s) {
 bool tc_fwd_supported(const Shape& s) { return s.bf16 && s.D == 128 && s.T % CT == 0; }
 
 bool tc_qkv_maps(const Shape& s, const void* q, const void* k, const void* v, CUtensorMap* mq,
-                 CUtensorMap* mk, CUtensorMap* mv) {
+                 CUtensorMap* mk, CUtensorMap* mv, unsigned box_rows) {
     const unsigned long long dims[3] = {128ull, (unsigned long long)s.H,
                                         (unsigned long long)s.B * s.T};
     const unsigned long long strides[2] = {128ull * 2, (unsigned long long)s.H * 128 * 2};
-    const unsigned box[3] = {64, 1, CT};
+    const unsigned box[3] = {64, 1, box_rows};
     return (!mq || make_tmap_bf16(mq, q, 3, dims, strides, box)) &&
            (!mk || make_tmap_bf16(mk, k, 3, dims, strides, box)) &&
            (!mv || make_tmap_bf16(mv, v, 3, dims, strides, box));
 }
 
-bool tc_rows_map(CUtensorMap* map, const void* base, unsigned long long rows, bool f16) {
+bool tc_rows_map(CUtensorMap* map, const void* base, unsigned long long rows, bool f16,
+                 unsigned box_rows) {
     const unsigned long long dims[2] = {128ull, rows};
     const unsigned long long str[1] = {256ull};
-    const unsigned box[2] = {64, 128};
+    const unsigned box[2] = {64, box_rows};
     return make_tmap_bf16(map, base, 2, dims, str, box, f16);
 }
 
@@ -602,8 +611,8 @@ cudaError_t launch_fwd_segment_states(const TcFwdArgs& a, const void* k, const v
         LaunchScope ls_("m_to_f16", st);
         m_to_f16_kernel<<<(n + 255) / 256, 256, 0, st>>>(Mf, const_cast<__half*>(a.Mb), s.H);
     }
-    const dim3 grid(a.nseg, s.B * s.H);
-    const int smA = 1024 + 6 * TILE + 1024;
+    const dim3 grid(s.B * s.H, a.nseg);   // heads fastest: CTAs that share token rows run together
+    const int smA = 1024 + 12 * SEGC_DEFAULT * CT + 6 * TILE + 1024;
     auto kA = seg_state_tc<SEGC_DEFAULT, __half>;
     cudaFuncSetAttribute(kA, cudaFuncAttributeMaxDynamicSharedMemorySize, smA);
     { LaunchScope ls_("tc_seg_state", st); kA<<<grid, 256, smA, st>>>(mk, mv, a); }
@@ -636,7 +645,7 @@ cudaError_t launch_fwd_tc(const TcFwdArgs& a, const void* q, const void* k, cons
         return cudaErrorInvalidValue;
     cudaError_t e = launch_fwd_segment_states(a, k, v, Mf, st);
     if (e != cudaSuccess) return e;
-    const dim3 grid(a.nseg, s.B * s.H);
+    const dim3 grid(s.B * s.H, a.nseg);   // heads fastest: CTAs that share token rows run together
     const int smC = 2048 + 7 * TILE + 1024;
     auto kC = seg_out_tc<SEGC_DEFAULT>;
     cudaFuncSetAttribute(kC, cudaFuncAttributeMaxDynamicSharedMemorySize, smC);
