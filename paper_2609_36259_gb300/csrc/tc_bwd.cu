@@ -213,7 +213,11 @@ __global__ void __launch_bounds__(256, 1) snap_fwd_tc(const __grid_constant__ CU
 
 // ---------------------------------------------------------------------------------------
 // Per chunk: recompute O', O''; dO''; middle-readout gradient; dO'; dq; per-token scalars.
-// 512 threads: one row and one column quarter each (QRole).
+// 512 threads: one row and one column quarter each (QRole).  Persistent: each CTA walks a
+// contiguous range of (b*h, chunk) items; the next item's dO, Vbar (and M on a new head) are
+// loaded into the tiles the current item has finished with after its dO' products, and its V
+// after the last product, so an item starts with its operands mostly in place.  The six tiles
+// change roles from item to item: (dO/Q, A, staging) <- (A, staging, dO/Q).
 __global__ void __launch_bounds__(512, 1) bwd_chunk1_tc(const __grid_constant__ CUtensorMap tq,
                                                          const __grid_constant__ CUtensorMap tk,
                                                          const __grid_constant__ CUtensorMap tv,
@@ -222,61 +226,72 @@ __global__ void __launch_bounds__(512, 1) bwd_chunk1_tc(const __grid_constant__ 
                                                          const __grid_constant__ CUtensorMap tsf,
                                                          TcBwdArgs a) {
     const Shape s = a.s;
-    const int bh = blockIdx.x, cg = blockIdx.y, b = bh / s.H, h = bh % s.H;
-    const int nct = s.T / CT, t0 = cg * CT;
+    const int nct = s.T / CT;
+    const int NI = s.B * s.H * nct;   // items (b*h, chunk), b*h-major
+    const int i0 = (int)((long long)NI * blockIdx.x / gridDim.x);
+    const int i1 = (int)((long long)NI * (blockIdx.x + 1) / gridDim.x);
     const int tid = threadIdx.x;
     const QRole ro;
     const int row = ro.row, hf = ro.hf, u = ro.u, c0 = ro.c0, cq = ro.cq;
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                                ~uintptr_t(1023));
-    uint64_t* bars = reinterpret_cast<uint64_t*>(smem);            // tma0, tma1, mma
+    // first operands (dO, Vbar, M), second operands (Q, K, Kbar), products, V
+    uint64_t* bars = reinterpret_cast<uint64_t*>(smem);
     uint32_t* s_taddr = reinterpret_cast<uint32_t*>(smem + 32);
     float* s_g2 = reinterpret_cast<float*>(smem + 64);              // [128]
     float* s_red = s_g2 + 128;                                      // [2][4][128]
-    uint8_t* T_K = smem + 5120;       // V (first), then K
-    uint8_t* T_KB = T_K + 1 * TILE;   // Kbar snapshot (rows = slots)
-    uint8_t* T_A = T_K + 2 * TILE;    // write vectors (rows = tokens)
-    uint8_t* T_M = T_K + 3 * TILE;    // M = R Phi
-    uint8_t* T_S = T_K + 4 * TILE;    // Vbar snapshot (first), then staging
-    uint8_t* T_L1 = T_K + 5 * TILE;   // dO, then Q
+    float* s_gate = s_red + 1024;                                   // [4][128] next item's gates
+    uint8_t* P = smem + 7168;                                       // six tiles
+    int rL1 = 0, rA = 3, rS = 4;                                    // rotating roles
+    uint8_t* T_K = P + 1 * TILE;      // V (first), then K
+    uint8_t* T_KB = P + 2 * TILE;     // Vbar snapshot (first), then Kbar snapshot
+    uint8_t* T_M = P + 5 * TILE;      // M = R Phi
     if (tid == 0) {
-        for (int i = 0; i < 3; ++i) mbar_init(&bars[i], 1);
+        for (int i = 0; i < 4; ++i) mbar_init(&bars[i], 1);
         fence_mbar_init();
     }
     if (ro.warp == 0) tmem_alloc(s_taddr, 512);
-    const size_t gi = ((size_t)b * s.T + t0 + row) * s.H + h;
-    const float lam = a.lam[gi], beta = a.beta[gi];
-    const float g2 = cum128(s, a.g, b, h, t0, t0 + row) * LOG2E;
-    if (cq == 0) s_g2[row] = g2;
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
     const uint32_t taddr = *s_taddr;
     const uint32_t tl = taddr + ((uint32_t)(32 * ro.q) << 16) + c0;
     const uint32_t X1 = 0, X2 = 128, X3 = 256, X4 = 384;
-    const int rowtok = b * s.T + t0;
-    const int snap_row = (bh * nct + cg) * 2 * 128;
-    if (tid == 0) {
-        mbar_expect_tx(&bars[0], 5 * TILE);
-        tma_load_3d(T_L1, &tdo, 0, h, rowtok, &bars[0]);
-        tma_load_3d(T_L1 + TILE / 2, &tdo, 64, h, rowtok, &bars[0]);
-        tma_load_3d(T_K, &tv, 0, h, rowtok, &bars[0]);
-        tma_load_3d(T_K + TILE / 2, &tv, 64, h, rowtok, &bars[0]);
-        tma_load_2d(T_S, &tsf, 0, snap_row + 128, &bars[0]);
-        tma_load_2d(T_S + TILE / 2, &tsf, 64, snap_row + 128, &bars[0]);
-        tma_load_2d(T_KB, &tsf, 0, snap_row, &bars[0]);
-        tma_load_2d(T_KB + TILE / 2, &tsf, 64, snap_row, &bars[0]);
-        tma_load_2d(T_M, &tm, 0, h * 128, &bars[0]);
-        tma_load_2d(T_M + TILE / 2, &tm, 64, h * 128, &bars[0]);
-    }
-    write_vector_q<__half>(T_A, row, hf, u, lam, beta);
-    bool ok = mbar_wait(&bars[0], 0);
-    if (ok) {   // dO and V: bf16 -> fp16
-        bf16_to_f16_q(T_L1, row, c0);
-        bf16_to_f16_q(T_K, row, c0);
-    }
+    const float scale = s.scale;
+    const uint32_t id_kk = idesc_f16(128, 128, 0, 0), id_kn = idesc_f16(128, 128, 0, 1);
+    bool ok = i0 < i1;
+    // loads in flight (thread 0), for a clean stop after a failed wait
+    // bits 0-2: a load on barrier 0 / 1 / 3 in flight; bits 4-6: the parity it completes
+    uint32_t pend = 0;
+    uint32_t ph = 0;                   // parity of the per-item barriers (0, 1, 3) of this item
     uint32_t mma_ph = 0;
+    float g2 = 0.f;                    // this thread's log2-domain decay in the current item
+    auto issue_first = [&](int item, uint8_t* tdO, uint8_t* tVb, bool with_m) {
+        const int ibh = item / nct, icg = item - ibh * nct, ib = ibh / s.H, ih = ibh - ib * s.H;
+        const int rtok = ib * s.T + icg * CT, srow = (ibh * nct + icg) * 2 * 128;
+        mbar_expect_tx(&bars[0], (with_m ? 3 : 2) * TILE);
+        tma_load_3d(tdO, &tdo, 0, ih, rtok, &bars[0]);
+        tma_load_3d(tdO + TILE / 2, &tdo, 64, ih, rtok, &bars[0]);
+        tma_load_2d(tVb, &tsf, 0, srow + 128, &bars[0]);
+        tma_load_2d(tVb + TILE / 2, &tsf, 64, srow + 128, &bars[0]);
+        if (with_m) {
+            tma_load_2d(T_M, &tm, 0, ih * 128, &bars[0]);
+            tma_load_2d(T_M + TILE / 2, &tm, 64, ih * 128, &bars[0]);
+        }
+        pend = (pend & ~0x11u) | 0x1u | ((uint32_t)((item - i0) & 1) << 4);
+    };
+    auto issue_v = [&](int item, uint8_t* tV) {
+        const int ibh = item / nct, icg = item - ibh * nct, ib = ibh / s.H, ih = ibh - ib * s.H;
+        mbar_expect_tx(&bars[3], TILE);
+        tma_load_3d(tV, &tv, 0, ih, ib * s.T + icg * CT, &bars[3]);
+        tma_load_3d(tV + TILE / 2, &tv, 64, ih, ib * s.T + icg * CT, &bars[3]);
+        pend = (pend & ~0x44u) | 0x4u | ((uint32_t)((item - i0) & 1) << 6);
+    };
+    if (tid == 0 && ok) {
+        issue_first(i0, P + rL1 * TILE, T_KB, true);
+        issue_v(i0, T_K);
+    }
     auto publish = [&]() {
         fence_async_smem();
         tc_fence_before();
@@ -289,6 +304,34 @@ __global__ void __launch_bounds__(512, 1) bwd_chunk1_tc(const __grid_constant__ 
         tc_fence_after();
     };
     auto issuer = [&]() { return tid == 0 && ok; };
+    // gates of the current item, and the next item's prefetched
+    auto gate_index = [&](int item) {
+        const int ibh = item / nct, icg = item - ibh * nct, ib = ibh / s.H, ih = ibh - ib * s.H;
+        return ((size_t)ib * s.T + icg * CT + row) * s.H + ih;
+    };
+    // the gates of an item (clock, write strength, the two terms of the chunk-local decay) go to
+    // s_gate by asynchronous copies, issued an epilogue ahead of their use (no registers held)
+    auto stage_gates = [&](int item) {
+        if (cq != 0) return;
+        const int ibh = item / nct, icg = item - ibh * nct, ib = ibh / s.H, ih = ibh - ib * s.H;
+        const size_t gi_ = ((size_t)ib * s.T + icg * CT + row) * s.H + ih;
+        const float* src[4] = {a.lam + gi_, a.beta + gi_, a.g + gi_,
+                               (s.Cg == 64 && row >= 64) ? a.g + ((size_t)ib * s.T + icg * CT + 63) * s.H + ih
+                                                         : nullptr};
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+            const uint32_t d = smem_u32(s_gate + 128 * k + row);
+            if (src[k])
+                asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"(d), "l"(src[k]) : "memory");
+            else
+                s_gate[128 * k + row] = 0.f;
+        }
+        asm volatile("cp.async.commit_group;" ::: "memory");
+    };
+    auto gates_landed = [&]() { asm volatile("cp.async.wait_group 0;" ::: "memory"); };
+    if (ok) stage_gates(i0);
+    gates_landed();
+    __syncthreads();
     // x o Gamma (times mul) with the causal mask; columns are tokens of this chunk
     auto mask_scores = [&](float (&x)[32], float mul) {
 #pragma unroll
@@ -317,262 +360,300 @@ __global__ void __launch_bounds__(512, 1) bwd_chunk1_tc(const __grid_constant__ 
         return is_max ? fmaxf(fmaxf(r[row], r[128 + row]), fmaxf(r[256 + row], r[384 + row]))
                       : (r[row] + r[128 + row]) + (r[256 + row] + r[384 + row]);
     };
-    const uint32_t id_kk = idesc_f16(128, 128, 0, 0), id_kn = idesc_f16(128, 128, 0, 1);
-    const uint32_t uK = smem_u32(T_K), uKB = smem_u32(T_KB), uA = smem_u32(T_A), uM = smem_u32(T_M),
-                   uS = smem_u32(T_S), uL1 = smem_u32(T_L1);
-    const float scale = s.scale;
-    const float gam = ex2(g2);
-    float s1 = 0.f, s2 = 0.f, s3 = 0.f, s4 = 0.f;
-    publish();
-    if (issuer()) {   // G1: X1 = dO V^T, X2 = dO Vbar^T
-#pragma unroll
-        for (int k = 0; k < 8; ++k) {
-            mma_bf16(taddr + X1, kmajor_desc(uL1, 128, k), kmajor_desc(uK, 128, k), id_kk, k > 0);
-            mma_bf16(taddr + X2, kmajor_desc(uL1, 128, k), kmajor_desc(uS, 128, k), id_kk, k > 0);
-        }
-        mma_commit(&bars[2]);
-    }
-    wait_mma();
-    if (issuer()) {   // dO and V are consumed: Q and K
-        mbar_expect_tx(&bars[1], 2 * TILE);
-        tma_load_3d(T_L1, &tq, 0, h, rowtok, &bars[1]);
-        tma_load_3d(T_L1 + TILE / 2, &tq, 64, h, rowtok, &bars[1]);
-        tma_load_3d(T_K, &tk, 0, h, rowtok, &bars[1]);
-        tma_load_3d(T_K + TILE / 2, &tk, 64, h, rowtok, &bars[1]);
-    }
-    {   // P4 = (dO V^T) o Gamma
-        float x[32];
-        tmem_ld16x2(tl + X1, x);
-        mask_scores(x, 1.f);
-        store_q<__half>(T_S, row, c0, x);
-    }
-    publish();
-    if (issuer()) {   // G2: X3 = P4 A
-#pragma unroll
-        for (int k = 0; k < 8; ++k)
-            mma_bf16(taddr + X3, kmajor_desc(uS, 128, k), mnmajor_desc(uA, 128, k), id_kn, k > 0);
-        mma_commit(&bars[2]);
-    }
-    wait_mma();
-    {   // do'' = gamma (dO Vbar^T) + P4 A, kept in X2
-        float x[32], y[32];
-        tmem_ld16x2(tl + X2, x);
-        tmem_ld16x2(tl + X3, y);
-#pragma unroll
-        for (int i = 0; i < 32; ++i) x[i] = fmaf(gam, x[i], y[i]);
-        tmem_st16x2(tl + X2, x);
-        if (ok) ok = mbar_wait(&bars[1], 0);
-        if (ok) {   // Q and K: bf16 -> fp16
+    for (int it = i0; it < i1 && ok; ++it) {
+        const int bh = it / nct, cg = it - bh * nct, b = bh / s.H, h = bh % s.H;
+        const int t0 = cg * CT;
+        const size_t gi = gate_index(it);
+        const float lam = s_gate[row], beta = s_gate[128 + row];
+        g2 = (s_gate[256 + row] + s_gate[384 + row]) * LOG2E;
+        uint8_t* T_L1 = P + rL1 * TILE;   // dO, then Q
+        uint8_t* T_A = P + rA * TILE;     // write vectors (rows = tokens)
+        uint8_t* T_S = P + rS * TILE;     // staging
+        const int rowtok = b * s.T + t0;
+        const int snap_row = (bh * nct + cg) * 2 * 128;
+        if (cq == 0) s_g2[row] = g2;
+        if (ok) ok = mbar_wait(&bars[0], ph);
+        if (tid == 0 && ok) pend &= ~0x1u;
+        if (ok) ok = mbar_wait(&bars[3], ph);
+        if (tid == 0 && ok) pend &= ~0x4u;
+        if (ok) {   // dO and V: bf16 -> fp16
             bf16_to_f16_q(T_L1, row, c0);
             bf16_to_f16_q(T_K, row, c0);
         }
-    }
-    publish();
-    if (issuer()) {   // G3: X1 = Q K^T, X3 = Q Kbar^T
-#pragma unroll
-        for (int k = 0; k < 8; ++k) {
-            mma_bf16(taddr + X1, kmajor_desc(uL1, 128, k), kmajor_desc(uK, 128, k), id_kk, k > 0);
-            mma_bf16(taddr + X3, kmajor_desc(uL1, 128, k), kmajor_desc(uKB, 128, k), id_kk, k > 0);
-        }
-        mma_commit(&bars[2]);
-    }
-    wait_mma();
-    {   // P1 = s (Q K^T) o Gamma
-        float x[32];
-        tmem_ld16x2(tl + X1, x);
-        mask_scores(x, scale);
-        store_q<__half>(T_S, row, c0, x);
-    }
-    publish();
-    if (issuer()) {   // G4: X4 = P1 A
-#pragma unroll
-        for (int k = 0; k < 8; ++k)
-            mma_bf16(taddr + X4, kmajor_desc(uS, 128, k), mnmajor_desc(uA, 128, k), id_kn, k > 0);
-        mma_commit(&bars[2]);
-    }
-    wait_mma();
-    {   // z = U(lam) o', kept in X3
-        float x[32], y[32];
-        tmem_ld16x2(tl + X3, x);
-        tmem_ld16x2(tl + X4, y);
-        const float f = scale * gam;
-#pragma unroll
-        for (int i = 0; i < 32; ++i) x[i] = fmaf(f, x[i], y[i]);
-        rotate_q<1>(x, hf, u, lam);
-        store_q<__half>(T_S, row, c0, x);
-        tmem_st16x2(tl + X3, x);
-    }
-    publish();
-    if (issuer()) {   // G5: X1 = z M^T
-#pragma unroll
-        for (int k = 0; k < 8; ++k)
-            mma_bf16(taddr + X1, kmajor_desc(uS, 128, k), kmajor_desc(uM, 128, k), id_kk, k > 0);
-        mma_commit(&bars[2]);
-    }
-    wait_mma();
-    {   // p = softmax(l) over the m valid entries (the padding column is out), kept in X1
-        float x[32];
-        tmem_ld16x2(tl + X1, x);
-        const bool pad = (hf == 1 && u == 1);
-        float mx = -INFINITY;
-#pragma unroll
-        for (int i = 0; i < 32; ++i)
-            if (!(pad && i == 31)) mx = fmaxf(mx, x[i]);
-        mx = row_reduce(mx, true);
-        float sum = 0.f;
-#pragma unroll
-        for (int i = 0; i < 32; ++i) {
-            x[i] = (pad && i == 31) ? 0.f : ex2((x[i] - mx) * LOG2E);
-            sum += x[i];
-        }
-        const float inv = 1.f / row_reduce(sum, false);
-#pragma unroll
-        for (int i = 0; i < 32; ++i) x[i] *= inv;
-        store_q<__half>(T_S, row, c0, x);
-        tmem_st16x2(tl + X1, x);
-    }
-    publish();
-    if (issuer()) {   // G6: X4 = p M
-#pragma unroll
-        for (int k = 0; k < 8; ++k)
-            mma_bf16(taddr + X4, kmajor_desc(uS, 128, k), mnmajor_desc(uM, 128, k), id_kn, k > 0);
-        mma_commit(&bars[2]);
-    }
-    wait_mma();
-    {   // o'' = U(-lam) (p M); scalars with do'' (o'' as stored in fp16); dy = U(lam) do''.
-        // Eight rotation pairs at a time: cosine entries, then sine entries.
-        QuarterAngles ang(lam, hf, u);
-        const bool dcq = (hf == 1 && u == 1);   // pair 15 of this quarter is the DC / padding
-        __half* o2row = a.O2 + ((size_t)bh * s.T + t0 + row) * 128;
-#pragma unroll
-        for (int p8 = 0; p8 < 2; ++p8) {
-            float o[16], gv[16];
-            tmem_ld8x2(tl + X4 + 8 * p8, o);
-            tmem_ld8x2(tl + X2 + 8 * p8, gv);
-#pragma unroll
-            for (int i = 0; i < 8; ++i) {
-                if (p8 + i > 0) ang.step();
-                const float c = ang.c, sn = ang.s;
-                const bool dc = dcq && p8 == 1 && i == 7;
-                const float xc = o[i], xs = o[8 + i];
-                o[i] = dc ? xc : c * xc + sn * xs;          // U(-lam)
-                o[8 + i] = dc ? 0.f : c * xs - sn * xc;
-                const float orc = round16<__half>(o[i]), ors = round16<__half>(o[8 + i]);
-                const float gc = gv[i], gs = gv[8 + i];
-                s1 = fmaf(orc, gc, fmaf(ors, gs, s1));
-                if (!dc) {   // <o'', Omega do''>
-                    const int j = 32 * hf + 16 * u + 8 * p8 + i + 1;
-                    s2 += (6.283185307179586f * (float)j / 127.f) * (ors * gc - orc * gs);
-                }
-                gv[i] = dc ? gc : c * gc - sn * gs;          // U(lam)
-                gv[8 + i] = dc ? 0.f : sn * gc + c * gs;
+        publish();
+        if (!ok) break;
+        const uint32_t uK = smem_u32(T_K), uKB = smem_u32(T_KB), uA = smem_u32(T_A), uM = smem_u32(T_M),
+                       uS = smem_u32(T_S), uL1 = smem_u32(T_L1);
+        const float gam = ex2(g2);
+        float s1 = 0.f, s2 = 0.f, s3 = 0.f, s4 = 0.f;
+        if (issuer()) {   // G1: X1 = dO V^T, X2 = dO Vbar^T
+    #pragma unroll
+            for (int k = 0; k < 8; ++k) {
+                mma_bf16(taddr + X1, kmajor_desc(uL1, 128, k), kmajor_desc(uK, 128, k), id_kk, k > 0);
+                mma_bf16(taddr + X2, kmajor_desc(uL1, 128, k), kmajor_desc(uKB, 128, k), id_kk, k > 0);
             }
-            store8x2_global(o2row, c0 + 8 * p8, o);
-            store8x2<__half>(T_S, row, c0 + 8 * p8, gv);
+            mma_commit(&bars[2]);
         }
-    }
-    publish();
-    if (issuer()) {   // G7: X4 = dy M^T = M dy
-#pragma unroll
-        for (int k = 0; k < 8; ++k)
-            mma_bf16(taddr + X4, kmajor_desc(uS, 128, k), kmajor_desc(uM, 128, k), id_kk, k > 0);
-        mma_commit(&bars[2]);
-    }
-    wait_mma();
-    {   // dl = p o (dp - <p, dp>)
-        float p[32], dp[32];
-        tmem_ld16x2(tl + X1, p);
-        tmem_ld16x2(tl + X4, dp);
-        const float pdp = row_reduce(dot32(p, dp), false);
-#pragma unroll
-        for (int i = 0; i < 32; ++i) p[i] = p[i] * (dp[i] - pdp);
-        store_q<__half>(T_S, row, c0, p);
-    }
-    publish();
-    if (issuer()) {   // G8: X2 = dl M = M^T dl
-#pragma unroll
-        for (int k = 0; k < 8; ++k)
-            mma_bf16(taddr + X2, kmajor_desc(uS, 128, k), mnmajor_desc(uM, 128, k), id_kn, k > 0);
-        mma_commit(&bars[2]);
-    }
-    wait_mma();
-    {   // do' = U(-lam) dz; <do', Omega o'> with do' as stored in fp16 (= <dz, Omega z> exactly)
-        QuarterAngles ang(lam, hf, u);
-        const bool dcq = (hf == 1 && u == 1);
-        __half* d1row = a.DO1 + ((size_t)bh * s.T + t0 + row) * 128;
-#pragma unroll
-        for (int p8 = 0; p8 < 2; ++p8) {
-            float dz[16], z[16];
-            tmem_ld8x2(tl + X2 + 8 * p8, dz);
-            tmem_ld8x2(tl + X3 + 8 * p8, z);
-#pragma unroll
-            for (int i = 0; i < 8; ++i) {
-                if (p8 + i > 0) ang.step();
-                const float c = ang.c, sn = ang.s;
-                const bool dc = dcq && p8 == 1 && i == 7;
-                const float xc = dz[i], xs = dz[8 + i];
-                dz[i] = dc ? xc : c * xc + sn * xs;         // U(-lam)
-                dz[8 + i] = dc ? 0.f : c * xs - sn * xc;
-                if (!dc) {   // o' = U(-lam) z
-                    const float zc = c * z[i] + sn * z[8 + i], zs = c * z[8 + i] - sn * z[i];
-                    const int j = 32 * hf + 16 * u + 8 * p8 + i + 1;
-                    s3 += (6.283185307179586f * (float)j / 127.f) *
-                          (round16<__half>(dz[8 + i]) * zc - round16<__half>(dz[i]) * zs);
-                }
+        write_vector_q<__half>(T_A, row, hf, u, lam, beta);   // while G1 runs
+        wait_mma();
+        if (issuer()) {   // dO, V and Vbar are consumed: Q, K and Kbar
+            mbar_expect_tx(&bars[1], 3 * TILE);
+            tma_load_3d(T_L1, &tq, 0, h, rowtok, &bars[1]);
+            tma_load_3d(T_L1 + TILE / 2, &tq, 64, h, rowtok, &bars[1]);
+            tma_load_3d(T_K, &tk, 0, h, rowtok, &bars[1]);
+            tma_load_3d(T_K + TILE / 2, &tk, 64, h, rowtok, &bars[1]);
+            tma_load_2d(T_KB, &tsf, 0, snap_row, &bars[1]);
+            tma_load_2d(T_KB + TILE / 2, &tsf, 64, snap_row, &bars[1]);
+            pend = (pend & ~0x22u) | 0x2u | (ph << 5);
+        }
+        {   // P4 = (dO V^T) o Gamma
+            float x[32];
+            tmem_ld16x2(tl + X1, x);
+            mask_scores(x, 1.f);
+            store_q<__half>(T_S, row, c0, x);
+        }
+        publish();
+        if (issuer()) {   // G2: X3 = P4 A
+    #pragma unroll
+            for (int k = 0; k < 8; ++k)
+                mma_bf16(taddr + X3, kmajor_desc(uS, 128, k), mnmajor_desc(uA, 128, k), id_kn, k > 0);
+            mma_commit(&bars[2]);
+        }
+        wait_mma();
+        {   // do'' = gamma (dO Vbar^T) + P4 A, kept in X2
+            float x[32], y[32];
+            tmem_ld16x2(tl + X2, x);
+            tmem_ld16x2(tl + X3, y);
+    #pragma unroll
+            for (int i = 0; i < 32; ++i) x[i] = fmaf(gam, x[i], y[i]);
+            tmem_st16x2(tl + X2, x);
+            if (ok) ok = mbar_wait(&bars[1], ph);
+            if (tid == 0 && ok) pend &= ~0x2u;
+            if (ok) {   // Q and K: bf16 -> fp16
+                bf16_to_f16_q(T_L1, row, c0);
+                bf16_to_f16_q(T_K, row, c0);
             }
-            store8x2<__half>(T_S, row, c0 + 8 * p8, dz);
-            store8x2_global(d1row, c0 + 8 * p8, dz);
         }
-    }
-    publish();
-    if (issuer()) {   // G9: X1 = dO' A^T, X3 = dO' Kbar
-#pragma unroll
-        for (int k = 0; k < 8; ++k) {
-            mma_bf16(taddr + X1, kmajor_desc(uS, 128, k), kmajor_desc(uA, 128, k), id_kk, k > 0);
-            mma_bf16(taddr + X3, kmajor_desc(uS, 128, k), mnmajor_desc(uKB, 128, k), id_kn, k > 0);
+        publish();
+        if (issuer()) {   // G3: X1 = Q K^T, X3 = Q Kbar^T
+    #pragma unroll
+            for (int k = 0; k < 8; ++k) {
+                mma_bf16(taddr + X1, kmajor_desc(uL1, 128, k), kmajor_desc(uK, 128, k), id_kk, k > 0);
+                mma_bf16(taddr + X3, kmajor_desc(uL1, 128, k), kmajor_desc(uKB, 128, k), id_kk, k > 0);
+            }
+            mma_commit(&bars[2]);
         }
-        mma_commit(&bars[2]);
-    }
-    wait_mma();
-    {   // P3 = s (dO' A^T) o Gamma
-        float x[32];
-        tmem_ld16x2(tl + X1, x);
-        mask_scores(x, scale);
-        store_q<__half>(T_S, row, c0, x);
-    }
-    publish();
-    if (issuer()) {   // G10: X4 = P3 K
-#pragma unroll
-        for (int k = 0; k < 8; ++k)
-            mma_bf16(taddr + X4, kmajor_desc(uS, 128, k), mnmajor_desc(uK, 128, k), id_kn, k > 0);
-        mma_commit(&bars[2]);
-    }
-    wait_mma();
-    if (ok) {   // dq = s gamma (dO' Kbar) + P3 K  (P3 carries s) ; <q, dq> = <q~, dq~>
-        float x[32], y[32];
-        tmem_ld16x2(tl + X3, x);
-        tmem_ld16x2(tl + X4, y);
-        const float f = scale * gam;
-#pragma unroll
-        for (int i = 0; i < 32; ++i) x[i] = fmaf(f, x[i], y[i]);
-        load_q(T_L1, row, c0, y);
-        s4 = dot32(y, x);
-        store_global_q(static_cast<__nv_bfloat16*>(a.dq) + gi * 128, c0, x);
-    }
-    {
-        const float dG = row_reduce(s1 + s4, false);
-        const float dL = row_reduce(s3 + s2, false);
-        if (cq == 0 && ok) {
-            const size_t BTH = (size_t)s.B * s.T * s.H;
-            a.tok[gi] = dG;
-            a.tok[BTH + gi] = dL;
+        wait_mma();
+        {   // P1 = s (Q K^T) o Gamma
+            float x[32];
+            tmem_ld16x2(tl + X1, x);
+            mask_scores(x, scale);
+            store_q<__half>(T_S, row, c0, x);
+        }
+        publish();
+        if (issuer()) {   // G4: X4 = P1 A
+    #pragma unroll
+            for (int k = 0; k < 8; ++k)
+                mma_bf16(taddr + X4, kmajor_desc(uS, 128, k), mnmajor_desc(uA, 128, k), id_kn, k > 0);
+            mma_commit(&bars[2]);
+        }
+        wait_mma();
+        {   // z = U(lam) o', kept in X3
+            float x[32], y[32];
+            tmem_ld16x2(tl + X3, x);
+            tmem_ld16x2(tl + X4, y);
+            const float f = scale * gam;
+    #pragma unroll
+            for (int i = 0; i < 32; ++i) x[i] = fmaf(f, x[i], y[i]);
+            rotate_q<1>(x, hf, u, lam);
+            store_q<__half>(T_S, row, c0, x);
+            tmem_st16x2(tl + X3, x);
+        }
+        publish();
+        if (issuer()) {   // G5: X1 = z M^T
+    #pragma unroll
+            for (int k = 0; k < 8; ++k)
+                mma_bf16(taddr + X1, kmajor_desc(uS, 128, k), kmajor_desc(uM, 128, k), id_kk, k > 0);
+            mma_commit(&bars[2]);
+        }
+        wait_mma();
+        {   // p = softmax(l) over the m valid entries (the padding column is out), kept in X1
+            float x[32];
+            tmem_ld16x2(tl + X1, x);
+            const bool pad = (hf == 1 && u == 1);
+            float mx = -INFINITY;
+    #pragma unroll
+            for (int i = 0; i < 32; ++i)
+                if (!(pad && i == 31)) mx = fmaxf(mx, x[i]);
+            mx = row_reduce(mx, true);
+            float sum = 0.f;
+    #pragma unroll
+            for (int i = 0; i < 32; ++i) {
+                x[i] = (pad && i == 31) ? 0.f : ex2((x[i] - mx) * LOG2E);
+                sum += x[i];
+            }
+            const float inv = 1.f / row_reduce(sum, false);
+    #pragma unroll
+            for (int i = 0; i < 32; ++i) x[i] *= inv;
+            store_q<__half>(T_S, row, c0, x);
+            tmem_st16x2(tl + X1, x);
+        }
+        publish();
+        if (issuer()) {   // G6: X4 = p M
+    #pragma unroll
+            for (int k = 0; k < 8; ++k)
+                mma_bf16(taddr + X4, kmajor_desc(uS, 128, k), mnmajor_desc(uM, 128, k), id_kn, k > 0);
+            mma_commit(&bars[2]);
+        }
+        wait_mma();
+        {   // o'' = U(-lam) (p M); scalars with do'' (o'' as stored in fp16); dy = U(lam) do''.
+            // Eight rotation pairs at a time: cosine entries, then sine entries.
+            QuarterAngles ang(lam, hf, u);
+            const bool dcq = (hf == 1 && u == 1);   // pair 15 of this quarter is the DC / padding
+            __half* o2row = a.O2 + ((size_t)bh * s.T + t0 + row) * 128;
+    #pragma unroll
+            for (int p8 = 0; p8 < 2; ++p8) {
+                float o[16], gv[16];
+                tmem_ld8x2(tl + X4 + 8 * p8, o);
+                tmem_ld8x2(tl + X2 + 8 * p8, gv);
+    #pragma unroll
+                for (int i = 0; i < 8; ++i) {
+                    if (p8 + i > 0) ang.step();
+                    const float c = ang.c, sn = ang.s;
+                    const bool dc = dcq && p8 == 1 && i == 7;
+                    const float xc = o[i], xs = o[8 + i];
+                    o[i] = dc ? xc : c * xc + sn * xs;          // U(-lam)
+                    o[8 + i] = dc ? 0.f : c * xs - sn * xc;
+                    const float orc = round16<__half>(o[i]), ors = round16<__half>(o[8 + i]);
+                    const float gc = gv[i], gs = gv[8 + i];
+                    s1 = fmaf(orc, gc, fmaf(ors, gs, s1));
+                    if (!dc) {   // <o'', Omega do''>
+                        const int j = 32 * hf + 16 * u + 8 * p8 + i + 1;
+                        s2 += (6.283185307179586f * (float)j / 127.f) * (ors * gc - orc * gs);
+                    }
+                    gv[i] = dc ? gc : c * gc - sn * gs;          // U(lam)
+                    gv[8 + i] = dc ? 0.f : sn * gc + c * gs;
+                }
+                store8x2_global(o2row, c0 + 8 * p8, o);
+                store8x2<__half>(T_S, row, c0 + 8 * p8, gv);
+            }
+        }
+        publish();
+        if (issuer()) {   // G7: X4 = dy M^T = M dy
+    #pragma unroll
+            for (int k = 0; k < 8; ++k)
+                mma_bf16(taddr + X4, kmajor_desc(uS, 128, k), kmajor_desc(uM, 128, k), id_kk, k > 0);
+            mma_commit(&bars[2]);
+        }
+        wait_mma();
+        {   // dl = p o (dp - <p, dp>)
+            float p[32], dp[32];
+            tmem_ld16x2(tl + X1, p);
+            tmem_ld16x2(tl + X4, dp);
+            const float pdp = row_reduce(dot32(p, dp), false);
+    #pragma unroll
+            for (int i = 0; i < 32; ++i) p[i] = p[i] * (dp[i] - pdp);
+            store_q<__half>(T_S, row, c0, p);
+        }
+        publish();
+        if (issuer()) {   // G8: X2 = dl M = M^T dl
+    #pragma unroll
+            for (int k = 0; k < 8; ++k)
+                mma_bf16(taddr + X2, kmajor_desc(uS, 128, k), mnmajor_desc(uM, 128, k), id_kn, k > 0);
+            mma_commit(&bars[2]);
+        }
+        wait_mma();
+        {   // do' = U(-lam) dz; <do', Omega o'> with do' as stored in fp16 (= <dz, Omega z> exactly)
+            QuarterAngles ang(lam, hf, u);
+            const bool dcq = (hf == 1 && u == 1);
+            __half* d1row = a.DO1 + ((size_t)bh * s.T + t0 + row) * 128;
+    #pragma unroll
+            for (int p8 = 0; p8 < 2; ++p8) {
+                float dz[16], z[16];
+                tmem_ld8x2(tl + X2 + 8 * p8, dz);
+                tmem_ld8x2(tl + X3 + 8 * p8, z);
+    #pragma unroll
+                for (int i = 0; i < 8; ++i) {
+                    if (p8 + i > 0) ang.step();
+                    const float c = ang.c, sn = ang.s;
+                    const bool dc = dcq && p8 == 1 && i == 7;
+                    const float xc = dz[i], xs = dz[8 + i];
+                    dz[i] = dc ? xc : c * xc + sn * xs;         // U(-lam)
+                    dz[8 + i] = dc ? 0.f : c * xs - sn * xc;
+                    if (!dc) {   // o' = U(-lam) z
+                        const float zc = c * z[i] + sn * z[8 + i], zs = c * z[8 + i] - sn * z[i];
+                        const int j = 32 * hf + 16 * u + 8 * p8 + i + 1;
+                        s3 += (6.283185307179586f * (float)j / 127.f) *
+                              (round16<__half>(dz[8 + i]) * zc - round16<__half>(dz[i]) * zs);
+                    }
+                }
+                store8x2<__half>(T_S, row, c0 + 8 * p8, dz);
+                store8x2_global(d1row, c0 + 8 * p8, dz);
+            }
+        }
+        publish();
+        if (issuer()) {   // G9: X1 = dO' A^T, X3 = dO' Kbar
+    #pragma unroll
+            for (int k = 0; k < 8; ++k) {
+                mma_bf16(taddr + X1, kmajor_desc(uS, 128, k), kmajor_desc(uA, 128, k), id_kk, k > 0);
+                mma_bf16(taddr + X3, kmajor_desc(uS, 128, k), mnmajor_desc(uKB, 128, k), id_kn, k > 0);
+            }
+            mma_commit(&bars[2]);
+        }
+        wait_mma();
+        if (issuer() && it + 1 < i1) issue_first(it + 1, T_A, T_KB, (it + 1) / nct % s.H != h);
+        if (it + 1 < i1) stage_gates(it + 1);   // the next item's gates, an epilogue ahead
+        {   // P3 = s (dO' A^T) o Gamma
+            float x[32];
+            tmem_ld16x2(tl + X1, x);
+            mask_scores(x, scale);
+            store_q<__half>(T_S, row, c0, x);
+        }
+        publish();
+        if (issuer()) {   // G10: X4 = P3 K
+    #pragma unroll
+            for (int k = 0; k < 8; ++k)
+                mma_bf16(taddr + X4, kmajor_desc(uS, 128, k), mnmajor_desc(uK, 128, k), id_kn, k > 0);
+            mma_commit(&bars[2]);
+        }
+        wait_mma();
+        if (issuer() && it + 1 < i1) issue_v(it + 1, T_K);
+        if (ok) {   // dq = s gamma (dO' Kbar) + P3 K  (P3 carries s) ; <q, dq> = <q~, dq~>
+            float x[32], y[32];
+            tmem_ld16x2(tl + X3, x);
+            tmem_ld16x2(tl + X4, y);
+            const float f = scale * gam;
+    #pragma unroll
+            for (int i = 0; i < 32; ++i) x[i] = fmaf(f, x[i], y[i]);
+            load_q(T_L1, row, c0, y);
+            s4 = dot32(y, x);
+            store_global_q(static_cast<__nv_bfloat16*>(a.dq) + gi * 128, c0, x);
+        }
+        gates_landed();   // the next item's gates, visible after the barriers below
+        {
+            const float dG = row_reduce(s1 + s4, false);
+            const float dL = row_reduce(s3 + s2, false);
+            if (cq == 0 && ok) {
+                const size_t BTH = (size_t)s.B * s.T * s.H;
+                a.tok[gi] = dG;
+                a.tok[BTH + gi] = dL;
+            }
+        }
+        ph ^= 1;
+        {   // roles of the next item
+            const int l1 = rL1;
+            rL1 = rA;
+            rA = rS;
+            rS = l1;
         }
     }
     ok = __syncthreads_and(ok);
     if (!ok && tid == 0) {
         flag_error(CYFA_ERR_TIMEOUT);
-        mbar_wait(&bars[0], 0);
-        mbar_wait(&bars[1], 0);
+        // let copies still in flight land before the shared memory is released
+        if (pend & 0x1u) mbar_wait(&bars[0], (pend >> 4) & 1);
+        if (pend & 0x2u) mbar_wait(&bars[1], (pend >> 5) & 1);
+        if (pend & 0x4u) mbar_wait(&bars[3], (pend >> 6) & 1);
     }
     tc_fence_before();
     __syncthreads();
@@ -1205,13 +1286,22 @@ cudaError_t launch_bwd_tc(const TcBwdArgs& a, const TcFwdArgs& f, const void* q,
     const int sm_walk6 = 1024 + 6 * TILE + 1024;
     const int sm_snap_adj = 1024 + 4 * TC_SEGC * CT + 6 * TILE + 1024;
     const int sm_adj_seg = 1024 + 4 * TC_SEGC * CT + 4 * TILE + 1024;
-    const int sm_chunk1 = 5120 + 6 * TILE + 1024, sm_chunk2 = 2048 + 7 * TILE + 1024;
+    const int sm_chunk1 = 7168 + 6 * TILE + 1024, sm_chunk2 = 2048 + 7 * TILE + 1024;
     if (!a.saved) {
         cudaFuncSetAttribute(snap_fwd_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, sm_walk6);
         { LaunchScope ls_("tc_snap_fwd", st); snap_fwd_tc<<<gseg, 256, sm_walk6, st>>>(mk, mv, a); }
     }
     cudaFuncSetAttribute(bwd_chunk1_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, sm_chunk1);
-    { LaunchScope ls_("tc_bwd_chunk1", st); bwd_chunk1_tc<<<gchunk, 512, sm_chunk1, st>>>(mq, mk, mv, mdo, mm, msf, a); }
+    {   // persistent: one CTA per SM walks a contiguous range of (b*h, chunk) items
+        int dev = 0, sms = 0;
+        if (cudaGetDevice(&dev) != cudaSuccess ||
+            cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+            return cudaErrorInvalidValue;
+        const long long items = (long long)s.B * s.H * nct;
+        const int grid1 = (int)(items < sms ? items : sms);
+        LaunchScope ls_("tc_bwd_chunk1", st);
+        bwd_chunk1_tc<<<grid1, 512, sm_chunk1, st>>>(mq, mk, mv, mdo, mm, msf, a);
+    }
     cudaFuncSetAttribute(adj_walk_tc<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, sm_adj_seg);
     { LaunchScope ls_("tc_adj_segment", st); adj_walk_tc<false><<<gseg, 256, sm_adj_seg, st>>>(mdo1, mo2, mq, mdo, msf, msa, a); }
     { LaunchScope ls_("tc_adj_scan", st); seg_scan_rev_kernel<<<dim3(128, s.B * s.H), 256, 0, st>>>(a); }
