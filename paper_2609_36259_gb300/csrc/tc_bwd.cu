@@ -900,7 +900,10 @@ __global__ void __launch_bounds__(256) seg_scan_rev_kernel(TcBwdArgs a) {
 // Per chunk: dK, dV, dA (both passes) and the column-side gate scalars, from the adjoint
 // snapshot.  The intra-chunk and the inter-chunk parts of dA are kept apart (X3 / X4) so that
 // the gate kernel can pair every intra-chunk term with its row-side twin from bwd_chunk1_tc,
-// which uses bit-identical score matrices and roundings.  512 threads (QRole).
+// which uses bit-identical score matrices and roundings.  512 threads (QRole).  Persistent over
+// (b*h, chunk) items like bwd_chunk1_tc: the next item's V goes into the write-vector tile once
+// dO' A^T has read it, its dO into the Q tile after Q K^T, its O'' and D^V after the last
+// products; the write-vector tile and the V / K tile swap roles from item to item.
 __global__ void __launch_bounds__(512, 1) bwd_chunk2_tc(const __grid_constant__ CUtensorMap tq,
                                                          const __grid_constant__ CUtensorMap tk,
                                                          const __grid_constant__ CUtensorMap tv,
@@ -910,61 +913,86 @@ __global__ void __launch_bounds__(512, 1) bwd_chunk2_tc(const __grid_constant__ 
                                                          const __grid_constant__ CUtensorMap tsa,
                                                          TcBwdArgs a) {
     const Shape s = a.s;
-    const int bh = blockIdx.x, cg = blockIdx.y, b = bh / s.H, h = bh % s.H;
-    const int nct = s.T / CT, t0 = cg * CT;
+    const int nct = s.T / CT;
+    const int NI = s.B * s.H * nct;
+    const int i0 = (int)((long long)NI * blockIdx.x / gridDim.x);
+    const int i1 = (int)((long long)NI * (blockIdx.x + 1) / gridDim.x);
     const int tid = threadIdx.x;
     const QRole ro;
     const int row = ro.row, hf = ro.hf, u = ro.u, c0 = ro.c0, cq = ro.cq;
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                                ~uintptr_t(1023));
-    uint64_t* bars = reinterpret_cast<uint64_t*>(smem);   // tma0..tma3, mma
+    // 0: O'' + D^V, 1: K, 2: dO', 3: Q + D^K, 4: products, 5: V, 6: dO
+    uint64_t* bars = reinterpret_cast<uint64_t*>(smem);
     uint32_t* s_taddr = reinterpret_cast<uint32_t*>(smem + 64);
     float* s_g2 = reinterpret_cast<float*>(smem + 128);
-    uint8_t* T_A = smem + 2048;       // write vectors a (fp16)
-    uint8_t* T_AS = T_A + 1 * TILE;   // write vectors scaled by gamma^C / gamma^s
-    uint8_t* T_S = T_A + 2 * TILE;    // staging
-    uint8_t* L1 = T_A + 3 * TILE;     // dO, then Q
-    uint8_t* L2 = T_A + 4 * TILE;     // V (-> V->), then K (-> K->)
-    uint8_t* L3 = T_A + 5 * TILE;     // O'', then dO'
-    uint8_t* L4 = T_A + 6 * TILE;     // D^V, then D^K
+    uint8_t* P = smem + 2048;
+    int rA = 0, rL2 = 4;              // the write-vector tile and the V / K tile swap each item
+    uint8_t* T_AS = P + 1 * TILE;     // write vectors scaled by gamma^C / gamma^s
+    uint8_t* T_S = P + 2 * TILE;      // staging
+    uint8_t* L1 = P + 3 * TILE;       // dO, then Q
+    uint8_t* L3 = P + 5 * TILE;       // O'', then dO'
+    uint8_t* L4 = P + 6 * TILE;       // D^V, then D^K
     if (tid == 0) {
-        for (int i = 0; i < 5; ++i) mbar_init(&bars[i], 1);
+        for (int i = 0; i < 7; ++i) mbar_init(&bars[i], 1);
         fence_mbar_init();
     }
     if (ro.warp == 0) tmem_alloc(s_taddr, 512);
-    const size_t gi = ((size_t)b * s.T + t0 + row) * s.H + h;
-    const float lam = a.lam[gi], beta = a.beta[gi];
-    const float g2 = cum128(s, a.g, b, h, t0, t0 + row) * LOG2E;
-    if (cq == 0) s_g2[row] = g2;
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
     const uint32_t taddr = *s_taddr;
     const uint32_t tl = taddr + ((uint32_t)(32 * ro.q) << 16) + c0;
     const uint32_t X1 = 0, X2 = 128, X3 = 256, X4 = 384;
-    const int rowtok = b * s.T + t0, rowbh = bh * s.T + t0;
-    const int snap_row = (bh * nct + cg) * 2 * 128;
-    if (tid == 0) {
-        mbar_expect_tx(&bars[0], 4 * TILE);
-        tma_load_3d(L1, &tdo, 0, h, rowtok, &bars[0]);
-        tma_load_3d(L1 + TILE / 2, &tdo, 64, h, rowtok, &bars[0]);
-        tma_load_3d(L2, &tv, 0, h, rowtok, &bars[0]);
-        tma_load_3d(L2 + TILE / 2, &tv, 64, h, rowtok, &bars[0]);
-        tma_load_2d(L3, &to2, 0, rowbh, &bars[0]);
-        tma_load_2d(L3 + TILE / 2, &to2, 64, rowbh, &bars[0]);
-        tma_load_2d(L4, &tsa, 0, snap_row + 128, &bars[0]);
-        tma_load_2d(L4 + TILE / 2, &tsa, 64, snap_row + 128, &bars[0]);
-    }
-    const float g2C = cum128(s, a.g, b, h, t0, t0 + CT - 1) * LOG2E;
-    const float fw = ex2(g2C - g2);
-    write_vector_q<__half>(T_A, row, hf, u, lam, beta);
-    write_vector_q<__half>(T_AS, row, hf, u, lam, beta * fw);
-    uint32_t mma_ph = 0;
-    bool ok = mbar_wait(&bars[0], 0);
-    if (ok) {   // dO and V: bf16 -> fp16
-        bf16_to_f16_q(L1, row, c0);
-        bf16_to_f16_q(L2, row, c0);
+    const float scale = s.scale;
+    const uint32_t id_kk = idesc_f16(128, 128, 0, 0), id_kn = idesc_f16(128, 128, 0, 1),
+                   id_nn = idesc_f16(128, 128, 1, 1);
+    bool ok = i0 < i1;
+    // thread 0: bit k set = a load on barrier k in flight (its parity in bit 8 + k)
+    uint32_t pend = 0;
+    uint32_t ph = 0, mma_ph = 0;
+    float g2 = 0.f;
+    auto item_rows = [&](int item, int& ih, int& rtok, int& rbh, int& srow) {
+        const int ibh = item / nct, icg = item - ibh * nct, ib = ibh / s.H;
+        ih = ibh - ib * s.H;
+        rtok = ib * s.T + icg * CT;
+        rbh = ibh * s.T + icg * CT;
+        srow = (ibh * nct + icg) * 2 * 128;
+    };
+    auto mark = [&](int k, int item) {
+        pend = (pend & ~((1u << k) | (1u << (8 + k)))) | (1u << k) | ((uint32_t)((item - i0) & 1) << (8 + k));
+    };
+    auto issue_first = [&](int item, uint8_t* tO2, uint8_t* tDV) {
+        int ih, rtok, rbh, srow;
+        item_rows(item, ih, rtok, rbh, srow);
+        mbar_expect_tx(&bars[0], 2 * TILE);
+        tma_load_2d(tO2, &to2, 0, rbh, &bars[0]);
+        tma_load_2d(tO2 + TILE / 2, &to2, 64, rbh, &bars[0]);
+        tma_load_2d(tDV, &tsa, 0, srow + 128, &bars[0]);
+        tma_load_2d(tDV + TILE / 2, &tsa, 64, srow + 128, &bars[0]);
+        mark(0, item);
+    };
+    auto issue_v = [&](int item, uint8_t* tV) {
+        int ih, rtok, rbh, srow;
+        item_rows(item, ih, rtok, rbh, srow);
+        mbar_expect_tx(&bars[5], TILE);
+        tma_load_3d(tV, &tv, 0, ih, rtok, &bars[5]);
+        tma_load_3d(tV + TILE / 2, &tv, 64, ih, rtok, &bars[5]);
+        mark(5, item);
+    };
+    auto issue_do = [&](int item, uint8_t* tD) {
+        int ih, rtok, rbh, srow;
+        item_rows(item, ih, rtok, rbh, srow);
+        mbar_expect_tx(&bars[6], TILE);
+        tma_load_3d(tD, &tdo, 0, ih, rtok, &bars[6]);
+        tma_load_3d(tD + TILE / 2, &tdo, 64, ih, rtok, &bars[6]);
+        mark(6, item);
+    };
+    if (tid == 0 && ok) {
+        issue_first(i0, L3, L4);
+        issue_v(i0, P + rL2 * TILE);
+        issue_do(i0, L1);
     }
     auto publish = [&]() {
         fence_async_smem();
@@ -994,178 +1022,217 @@ __global__ void __launch_bounds__(512, 1) bwd_chunk2_tc(const __grid_constant__ 
             }
         }
     };
-    const uint32_t id_kk = idesc_f16(128, 128, 0, 0), id_kn = idesc_f16(128, 128, 0, 1),
-                   id_nn = idesc_f16(128, 128, 1, 1);
-    const uint32_t uA = smem_u32(T_A), uAS = smem_u32(T_AS), uS = smem_u32(T_S),
-                   u1 = smem_u32(L1), u2 = smem_u32(L2), u3 = smem_u32(L3), u4 = smem_u32(L4);
-    const float scale = s.scale;
-    float cG = 0.f;
-    publish();
-    if (issuer()) {   // X1 = dO V^T
-#pragma unroll
-        for (int k = 0; k < 8; ++k)
-            mma_bf16(taddr + X1, kmajor_desc(u1, 128, k), kmajor_desc(u2, 128, k), id_kk, k > 0);
-        mma_commit(&bars[4]);
-    }
-    wait_mma();
-    {   // P4 = (dO V^T) o Gamma ; V -> V-> (rows scaled by gamma^C / gamma^s)
-        float x[32];
-        tmem_ld16x2(tl + X1, x);
-        mask_scores(x, 1.f);
-        store_q<__half>(T_S, row, c0, x);
-        if (ok) scale_q(L2, row, c0, fw);
-    }
-    publish();
-    if (issuer()) {   // X3 = P4^T O'' ; X4 = V-> D^V^T ; X1 = O'' A^T
-#pragma unroll
-        for (int k = 0; k < 8; ++k) {
-            mma_bf16(taddr + X3, mnmajor_desc(uS, 128, k), mnmajor_desc(u3, 128, k), id_nn, k > 0);
-            mma_bf16(taddr + X4, kmajor_desc(u2, 128, k), kmajor_desc(u4, 128, k), id_kk, k > 0);
-            mma_bf16(taddr + X1, kmajor_desc(u3, 128, k), kmajor_desc(uA, 128, k), id_kk, k > 0);
-        }
-        mma_commit(&bars[4]);
-    }
-    wait_mma();
-    if (issuer()) {   // V and O'' are consumed: K, dO'
-        mbar_expect_tx(&bars[1], TILE);
-        tma_load_3d(L2, &tk, 0, h, rowtok, &bars[1]);
-        tma_load_3d(L2 + TILE / 2, &tk, 64, h, rowtok, &bars[1]);
-        mbar_expect_tx(&bars[2], TILE);
-        tma_load_2d(L3, &tdo1, 0, rowbh, &bars[2]);
-        tma_load_2d(L3 + TILE / 2, &tdo1, 64, rowbh, &bars[2]);
-    }
-    {   // <a, (P4^T O'')_t> ; P2 = (O'' A^T) o Gamma
-        float x[32], av[32];
-        tmem_ld16x2(tl + X3, x);
-        load_q(T_A, row, c0, av);   // the fp16 write vector entries, as the MMAs see them
-        cG = dot32(av, x);
-        tmem_ld16x2(tl + X1, x);
-        mask_scores(x, 1.f);
-        store_q<__half>(T_S, row, c0, x);
-    }
-    publish();
-    if (issuer()) {   // X2 = P2^T dO + A-> D^V  (dv)
-#pragma unroll
-        for (int k = 0; k < 8; ++k)
-            mma_bf16(taddr + X2, mnmajor_desc(uS, 128, k), mnmajor_desc(u1, 128, k), id_nn, k > 0);
-#pragma unroll
-        for (int k = 0; k < 8; ++k)
-            mma_bf16(taddr + X2, kmajor_desc(uAS, 128, k), mnmajor_desc(u4, 128, k), id_kn, 1u);
-        mma_commit(&bars[4]);
-    }
-    wait_mma();
-    if (issuer()) {   // dO and D^V are consumed: Q, D^K
-        mbar_expect_tx(&bars[3], 2 * TILE);
-        tma_load_3d(L1, &tq, 0, h, rowtok, &bars[3]);
-        tma_load_3d(L1 + TILE / 2, &tq, 64, h, rowtok, &bars[3]);
-        tma_load_2d(L4, &tsa, 0, snap_row, &bars[3]);
-        tma_load_2d(L4 + TILE / 2, &tsa, 64, snap_row, &bars[3]);
-    }
-    if (ok) {   // dv
-        float x[32];
-        tmem_ld16x2(tl + X2, x);
-        store_global_q(static_cast<__nv_bfloat16*>(a.dv) + gi * 128, c0, x);
-    }
-    publish();
-    if (issuer()) {   // X1 = dO' A^T
-        ok = mbar_wait(&bars[2], 0);
-        if (ok) {
-            tc_fence_after();
-#pragma unroll
-            for (int k = 0; k < 8; ++k)
-                mma_bf16(taddr + X1, kmajor_desc(u3, 128, k), kmajor_desc(uA, 128, k), id_kk, k > 0);
-            mma_commit(&bars[4]);
-        }
-    }
-    wait_mma();
-    {   // P3 = s (dO' A^T) o Gamma (the s of q~ = s q folded in, exactly as bwd_chunk1_tc does)
-        float x[32];
-        tmem_ld16x2(tl + X1, x);
-        mask_scores(x, scale);
-        store_q<__half>(T_S, row, c0, x);
-        if (ok) ok = mbar_wait(&bars[3], 0) && mbar_wait(&bars[1], 0);
-        if (ok) {   // Q and K: bf16 -> fp16
+    for (int it = i0; it < i1 && ok; ++it) {
+        const int bh = it / nct, cg = it - bh * nct, b = bh / s.H, h = bh % s.H;
+        const int t0 = cg * CT;
+        const size_t gi = ((size_t)b * s.T + t0 + row) * s.H + h;
+        // gates: loaded while this item's first tiles land
+        const float lam = a.lam[gi], beta = a.beta[gi];
+        g2 = cum128(s, a.g, b, h, t0, t0 + row) * LOG2E;
+        const float g2C = cum128(s, a.g, b, h, t0, t0 + CT - 1) * LOG2E;
+        const float fw = ex2(g2C - g2);
+        uint8_t* T_A = P + rA * TILE;     // write vectors a (fp16)
+        uint8_t* L2 = P + rL2 * TILE;     // V (-> V->), then K (-> K->)
+        const int rowtok = b * s.T + t0, rowbh = bh * s.T + t0;
+        const int snap_row = (bh * nct + cg) * 2 * 128;
+        if (cq == 0) s_g2[row] = g2;
+        if (ok) ok = mbar_wait(&bars[0], ph) && mbar_wait(&bars[5], ph) && mbar_wait(&bars[6], ph);
+        if (tid == 0 && ok) pend &= ~0x61u;
+        if (ok) {   // dO and V: bf16 -> fp16
             bf16_to_f16_q(L1, row, c0);
             bf16_to_f16_q(L2, row, c0);
         }
-    }
-    publish();
-    if (issuer()) {   // X2 = P3^T Q (intra part of dk) ;  X1 = Q K^T
-#pragma unroll
-        for (int k = 0; k < 8; ++k) {
-            mma_bf16(taddr + X2, mnmajor_desc(uS, 128, k), mnmajor_desc(u1, 128, k), id_nn, k > 0);
-            mma_bf16(taddr + X1, kmajor_desc(u1, 128, k), kmajor_desc(u2, 128, k), id_kk, k > 0);
+        publish();
+        if (!ok) break;
+        const uint32_t uA = smem_u32(T_A), uAS = smem_u32(T_AS), uS = smem_u32(T_S),
+                       u1 = smem_u32(L1), u2 = smem_u32(L2), u3 = smem_u32(L3), u4 = smem_u32(L4);
+        float cG = 0.f;
+        if (issuer()) {   // X1 = dO V^T
+    #pragma unroll
+            for (int k = 0; k < 8; ++k)
+                mma_bf16(taddr + X1, kmajor_desc(u1, 128, k), kmajor_desc(u2, 128, k), id_kk, k > 0);
+            mma_commit(&bars[4]);
         }
-        mma_commit(&bars[4]);
-    }
-    wait_mma();
-    {   // <k, (P3^T Q)_t> ; P1 = s (Q K^T) o Gamma ; K -> K->
-        float x[32], kv[32];
-        tmem_ld16x2(tl + X2, x);
-        load_q(L2, row, c0, kv);
-        cG += dot32(kv, x);
-        tmem_ld16x2(tl + X1, x);
-        mask_scores(x, scale);
-        store_q<__half>(T_S, row, c0, x);
-        __syncthreads();   // the Q K^T product has read K; rows are rescaled in place below
-        if (ok) scale_q(L2, row, c0, fw);
-    }
-    publish();
-    if (issuer()) {   // X1 = A-> D^K (inter part of dk) ; X3 += P1^T dO' ; X4 += K-> D^K^T
-#pragma unroll
-        for (int k = 0; k < 8; ++k) {
-            mma_bf16(taddr + X1, kmajor_desc(uAS, 128, k), mnmajor_desc(u4, 128, k), id_kn, k > 0);
-            mma_bf16(taddr + X3, mnmajor_desc(uS, 128, k), mnmajor_desc(u3, 128, k), id_nn, 1u);
-            mma_bf16(taddr + X4, kmajor_desc(u2, 128, k), kmajor_desc(u4, 128, k), id_kk, 1u);
+        // while it runs: the write vectors and their copies scaled by gamma^C / gamma^s
+        write_vector_q<__half>(T_A, row, hf, u, lam, beta);
+        write_vector_q<__half>(T_AS, row, hf, u, lam, beta * fw);
+        wait_mma();
+        {   // P4 = (dO V^T) o Gamma ; V -> V-> (rows scaled by gamma^C / gamma^s)
+            float x[32];
+            tmem_ld16x2(tl + X1, x);
+            mask_scores(x, 1.f);
+            store_q<__half>(T_S, row, c0, x);
+            if (ok) scale_q(L2, row, c0, fw);
         }
-        mma_commit(&bars[4]);
+        publish();
+        if (issuer()) {   // X3 = P4^T O'' ; X4 = V-> D^V^T ; X1 = O'' A^T
+    #pragma unroll
+            for (int k = 0; k < 8; ++k) {
+                mma_bf16(taddr + X3, mnmajor_desc(uS, 128, k), mnmajor_desc(u3, 128, k), id_nn, k > 0);
+                mma_bf16(taddr + X4, kmajor_desc(u2, 128, k), kmajor_desc(u4, 128, k), id_kk, k > 0);
+                mma_bf16(taddr + X1, kmajor_desc(u3, 128, k), kmajor_desc(uA, 128, k), id_kk, k > 0);
+            }
+            mma_commit(&bars[4]);
+        }
+        wait_mma();
+        if (issuer()) {   // V and O'' are consumed: K, dO'
+            mbar_expect_tx(&bars[1], TILE);
+            tma_load_3d(L2, &tk, 0, h, rowtok, &bars[1]);
+            tma_load_3d(L2 + TILE / 2, &tk, 64, h, rowtok, &bars[1]);
+            mbar_expect_tx(&bars[2], TILE);
+            tma_load_2d(L3, &tdo1, 0, rowbh, &bars[2]);
+            tma_load_2d(L3 + TILE / 2, &tdo1, 64, rowbh, &bars[2]);
+            mark(1, it);
+            mark(2, it);
+        }
+        {   // <a, (P4^T O'')_t> ; P2 = (O'' A^T) o Gamma
+            float x[32], av[32];
+            tmem_ld16x2(tl + X3, x);
+            load_q(T_A, row, c0, av);   // the fp16 write vector entries, as the MMAs see them
+            cG = dot32(av, x);
+            tmem_ld16x2(tl + X1, x);
+            mask_scores(x, 1.f);
+            store_q<__half>(T_S, row, c0, x);
+        }
+        publish();
+        if (issuer()) {   // X2 = P2^T dO + A-> D^V  (dv)
+    #pragma unroll
+            for (int k = 0; k < 8; ++k)
+                mma_bf16(taddr + X2, mnmajor_desc(uS, 128, k), mnmajor_desc(u1, 128, k), id_nn, k > 0);
+    #pragma unroll
+            for (int k = 0; k < 8; ++k)
+                mma_bf16(taddr + X2, kmajor_desc(uAS, 128, k), mnmajor_desc(u4, 128, k), id_kn, 1u);
+            mma_commit(&bars[4]);
+        }
+        wait_mma();
+        if (issuer()) {   // dO and D^V are consumed: Q, D^K
+            mbar_expect_tx(&bars[3], 2 * TILE);
+            tma_load_3d(L1, &tq, 0, h, rowtok, &bars[3]);
+            tma_load_3d(L1 + TILE / 2, &tq, 64, h, rowtok, &bars[3]);
+            tma_load_2d(L4, &tsa, 0, snap_row, &bars[3]);
+            tma_load_2d(L4 + TILE / 2, &tsa, 64, snap_row, &bars[3]);
+            mark(3, it);
+        }
+        if (ok) {   // dv
+            float x[32];
+            tmem_ld16x2(tl + X2, x);
+            store_global_q(static_cast<__nv_bfloat16*>(a.dv) + gi * 128, c0, x);
+        }
+        publish();
+        if (issuer()) {   // X1 = dO' A^T
+            ok = mbar_wait(&bars[2], ph);
+            if (ok) pend &= ~0x4u;
+            if (ok) {
+                tc_fence_after();
+    #pragma unroll
+                for (int k = 0; k < 8; ++k)
+                    mma_bf16(taddr + X1, kmajor_desc(u3, 128, k), kmajor_desc(uA, 128, k), id_kk, k > 0);
+                mma_commit(&bars[4]);
+            }
+        }
+        wait_mma();
+        if (issuer() && it + 1 < i1) issue_v(it + 1, T_A);   // A is consumed: the next item's V
+        {   // P3 = s (dO' A^T) o Gamma (the s of q~ = s q folded in, exactly as bwd_chunk1_tc does)
+            float x[32];
+            tmem_ld16x2(tl + X1, x);
+            mask_scores(x, scale);
+            store_q<__half>(T_S, row, c0, x);
+            if (ok) ok = mbar_wait(&bars[3], ph) && mbar_wait(&bars[1], ph);
+            if (tid == 0 && ok) pend &= ~0xAu;
+            if (ok) {   // Q and K: bf16 -> fp16
+                bf16_to_f16_q(L1, row, c0);
+                bf16_to_f16_q(L2, row, c0);
+            }
+        }
+        publish();
+        if (issuer()) {   // X2 = P3^T Q (intra part of dk) ;  X1 = Q K^T
+    #pragma unroll
+            for (int k = 0; k < 8; ++k) {
+                mma_bf16(taddr + X2, mnmajor_desc(uS, 128, k), mnmajor_desc(u1, 128, k), id_nn, k > 0);
+                mma_bf16(taddr + X1, kmajor_desc(u1, 128, k), kmajor_desc(u2, 128, k), id_kk, k > 0);
+            }
+            mma_commit(&bars[4]);
+        }
+        wait_mma();
+        if (issuer() && it + 1 < i1) issue_do(it + 1, L1);   // Q is consumed: the next item's dO
+        {   // <k, (P3^T Q)_t> ; P1 = s (Q K^T) o Gamma ; K -> K->
+            float x[32], kv[32];
+            tmem_ld16x2(tl + X2, x);
+            load_q(L2, row, c0, kv);
+            cG += dot32(kv, x);
+            tmem_ld16x2(tl + X1, x);
+            mask_scores(x, scale);
+            store_q<__half>(T_S, row, c0, x);
+            __syncthreads();   // the Q K^T product has read K; rows are rescaled in place below
+            if (ok) scale_q(L2, row, c0, fw);
+        }
+        publish();
+        if (issuer()) {   // X1 = A-> D^K (inter part of dk) ; X3 += P1^T dO' ; X4 += K-> D^K^T
+    #pragma unroll
+            for (int k = 0; k < 8; ++k) {
+                mma_bf16(taddr + X1, kmajor_desc(uAS, 128, k), mnmajor_desc(u4, 128, k), id_kn, k > 0);
+                mma_bf16(taddr + X3, mnmajor_desc(uS, 128, k), mnmajor_desc(u3, 128, k), id_nn, 1u);
+                mma_bf16(taddr + X4, kmajor_desc(u2, 128, k), kmajor_desc(u4, 128, k), id_kk, 1u);
+            }
+            mma_commit(&bars[4]);
+        }
+        wait_mma();
+        if (issuer() && it + 1 < i1) issue_first(it + 1, L3, L4);   // the next item's O'', D^V
+        float cIG = 0.f, cL = 0.f, cIL = 0.f, db = 0.f;
+        if (ok) {
+            float x[32], y[32];
+            tmem_ld16x2(tl + X2, x);          // dk = P3^T Q + A-> D^K
+            tmem_ld16x2(tl + X1, y);
+    #pragma unroll
+            for (int i = 0; i < 32; ++i) x[i] += y[i];
+            store_global_q(static_cast<__nv_bfloat16*>(a.dk) + gi * 128, c0, x);
+            float av[32];
+            write_vector_q_vals(av, hf, u, lam, beta);   // unrounded a
+            tmem_ld16x2(tl + X3, x);          // intra-chunk da (both passes)
+            tmem_ld16x2(tl + X4, y);          // inter-chunk da (both passes)
+    #pragma unroll
+            for (int i = 0; i < 32; ++i) db = fmaf(x[i] + y[i], av[i], db);
+    #pragma unroll
+            for (int i = 0; i < 32; ++i) av[i] = round16<__half>(av[i]);   // a as the MMAs saw it
+            cL = -omega_dot_q(x, av, hf, u);
+            cIG = dot32(av, y);
+            cIL = -omega_dot_q(y, av, hf, u);
+        }
+        // row sums over the four column quarters, staged in the (now idle) staging tile
+        float* s_fin = reinterpret_cast<float*>(T_S);   // [5][4][128]
+        s_fin[(0 * 4 + cq) * 128 + row] = cG;
+        s_fin[(1 * 4 + cq) * 128 + row] = cL;
+        s_fin[(2 * 4 + cq) * 128 + row] = db;
+        s_fin[(3 * 4 + cq) * 128 + row] = cIG;
+        s_fin[(4 * 4 + cq) * 128 + row] = cIL;
+        ok = __syncthreads_and(ok);
+        if (cq == 0 && ok) {
+            float v[5];
+    #pragma unroll
+            for (int k = 0; k < 5; ++k) {
+                const float* r = s_fin + 4 * 128 * k + row;
+                v[k] = (r[0] + r[128]) + (r[256] + r[384]);
+            }
+            const size_t BTH = (size_t)s.B * s.T * s.H;
+            a.tok[2 * BTH + gi] = v[0];
+            a.tok[3 * BTH + gi] = v[1];
+            a.tok[4 * BTH + gi] = v[2] / beta;
+            a.tok[5 * BTH + gi] = v[3];
+            a.tok[6 * BTH + gi] = v[4];
+        }
+        ph ^= 1;
+        {
+            const int t = rA;
+            rA = rL2;
+            rL2 = t;
+        }
     }
-    wait_mma();
-    float cIG = 0.f, cL = 0.f, cIL = 0.f, db = 0.f;
-    if (ok) {
-        float x[32], y[32];
-        tmem_ld16x2(tl + X2, x);          // dk = P3^T Q + A-> D^K
-        tmem_ld16x2(tl + X1, y);
-#pragma unroll
-        for (int i = 0; i < 32; ++i) x[i] += y[i];
-        store_global_q(static_cast<__nv_bfloat16*>(a.dk) + gi * 128, c0, x);
-        float av[32];
-        load_q(T_A, row, c0, av);
-        tmem_ld16x2(tl + X3, x);          // intra-chunk da (both passes)
-        tmem_ld16x2(tl + X4, y);          // inter-chunk da (both passes)
-        cL = -omega_dot_q(x, av, hf, u);
-        cIG = dot32(av, y);
-        cIL = -omega_dot_q(y, av, hf, u);
-#pragma unroll
-        for (int i = 0; i < 32; ++i) x[i] += y[i];
-        write_vector_q_vals(av, hf, u, lam, beta);   // unrounded a
-        db = dot32(x, av);
-    }
-    // row sums over the four column quarters, staged in the (now idle) staging tile
-    float* s_fin = reinterpret_cast<float*>(T_S);   // [5][4][128]
-    s_fin[(0 * 4 + cq) * 128 + row] = cG;
-    s_fin[(1 * 4 + cq) * 128 + row] = cL;
-    s_fin[(2 * 4 + cq) * 128 + row] = db;
-    s_fin[(3 * 4 + cq) * 128 + row] = cIG;
-    s_fin[(4 * 4 + cq) * 128 + row] = cIL;
     ok = __syncthreads_and(ok);
-    if (cq == 0 && ok) {
-        float v[5];
-#pragma unroll
-        for (int k = 0; k < 5; ++k) {
-            const float* r = s_fin + 4 * 128 * k + row;
-            v[k] = (r[0] + r[128]) + (r[256] + r[384]);
-        }
-        const size_t BTH = (size_t)s.B * s.T * s.H;
-        a.tok[2 * BTH + gi] = v[0];
-        a.tok[3 * BTH + gi] = v[1];
-        a.tok[4 * BTH + gi] = v[2] / beta;
-        a.tok[5 * BTH + gi] = v[3];
-        a.tok[6 * BTH + gi] = v[4];
-    }
     if (!ok && tid == 0) {
         flag_error(CYFA_ERR_TIMEOUT);
-        for (int i = 0; i < 4; ++i) mbar_wait(&bars[i], 0);
+        // let copies still in flight land before the shared memory is released
+        for (int k = 0; k < 7; ++k)
+            if (pend & (1u << k)) mbar_wait(&bars[k], (pend >> (8 + k)) & 1);
     }
     tc_fence_before();
     __syncthreads();
@@ -1308,7 +1375,16 @@ cudaError_t launch_bwd_tc(const TcBwdArgs& a, const TcFwdArgs& f, const void* q,
     cudaFuncSetAttribute(adj_walk_tc<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, sm_snap_adj);
     { LaunchScope ls_("tc_snap_adj", st); adj_walk_tc<true><<<gseg, 256, sm_snap_adj, st>>>(mdo1, mo2, mq, mdo, msf, msa, a); }
     cudaFuncSetAttribute(bwd_chunk2_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, sm_chunk2);
-    { LaunchScope ls_("tc_bwd_chunk2", st); bwd_chunk2_tc<<<gchunk, 512, sm_chunk2, st>>>(mq, mk, mv, mdo, mo2, mdo1, msa, a); }
+    {
+        int dev = 0, sms = 0;
+        if (cudaGetDevice(&dev) != cudaSuccess ||
+            cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+            return cudaErrorInvalidValue;
+        const long long items = (long long)s.B * s.H * nct;
+        const int grid2 = (int)(items < sms ? items : sms);
+        LaunchScope ls_("tc_bwd_chunk2", st);
+        bwd_chunk2_tc<<<grid2, 512, sm_chunk2, st>>>(mq, mk, mv, mdo, mo2, mdo1, msa, a);
+    }
     { LaunchScope ls_("tc_gate", st); tc_gate_kernel<<<gchunk, 128, 0, st>>>(a); }
     if (a.dA) { LaunchScope ls_("tc_dA", st); tc_dA_kernel<<<s.H, 256, 0, st>>>(a); }
     return cudaGetLastError();
