@@ -240,9 +240,10 @@ __global__ void __launch_bounds__(512, 1) bwd_chunk1_tc(const __grid_constant__ 
     uint64_t* bars = reinterpret_cast<uint64_t*>(smem);
     uint32_t* s_taddr = reinterpret_cast<uint32_t*>(smem + 32);
     float* s_g2 = reinterpret_cast<float*>(smem + 64);              // [128]
-    float* s_red = s_g2 + 128;                                      // [2][4][128]
-    float* s_gate = s_red + 1024;                                   // [4][128] next item's gates
-    uint8_t* P = smem + 7168;                                       // six tiles
+    float* s_b = s_g2 + 128;                                        // [128] in-block decay factors
+    float* s_red = s_b + 128;                                       // [2][4][128]
+    float* s_gate = s_red + 1024;                                   // [5][128] next item's gates
+    uint8_t* P = smem + 8192;                                       // six tiles
     int rL1 = 0, rA = 3, rS = 4;                                    // rotating roles
     uint8_t* T_K = P + 1 * TILE;      // V (first), then K
     uint8_t* T_KB = P + 2 * TILE;     // Vbar snapshot (first), then Kbar snapshot
@@ -315,11 +316,12 @@ __global__ void __launch_bounds__(512, 1) bwd_chunk1_tc(const __grid_constant__ 
         if (cq != 0) return;
         const int ibh = item / nct, icg = item - ibh * nct, ib = ibh / s.H, ih = ibh - ib * s.H;
         const size_t gi_ = ((size_t)ib * s.T + icg * CT + row) * s.H + ih;
-        const float* src[4] = {a.lam + gi_, a.beta + gi_, a.g + gi_,
+        const float* src[5] = {a.lam + gi_, a.beta + gi_, a.g + gi_,
                                (s.Cg == 64 && row >= 64) ? a.g + ((size_t)ib * s.T + icg * CT + 63) * s.H + ih
-                                                         : nullptr};
+                                                         : nullptr,
+                               a.g + ((size_t)ib * s.T + icg * CT + (row | 15)) * s.H + ih};
 #pragma unroll
-        for (int k = 0; k < 4; ++k) {
+        for (int k = 0; k < 5; ++k) {
             const uint32_t d = smem_u32(s_gate + 128 * k + row);
             if (src[k])
                 asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"(d), "l"(src[k]) : "memory");
@@ -334,20 +336,7 @@ __global__ void __launch_bounds__(512, 1) bwd_chunk1_tc(const __grid_constant__ 
     __syncthreads();
     // x o Gamma (times mul) with the causal mask; columns are tokens of this chunk
     auto mask_scores = [&](float (&x)[32], float mul) {
-#pragma unroll
-        for (int blk = 0; blk < 2; ++blk) {
-            const int tb = c0 + 32 * blk;
-            if (tb >= 32 * (ro.q + 1)) {   // every token of the block is after every row of the warp
-#pragma unroll
-                for (int i = 0; i < 16; ++i) x[16 * blk + i] = 0.f;
-            } else {
-#pragma unroll
-                for (int i = 0; i < 16; ++i) {
-                    const int t = tb + i;
-                    x[16 * blk + i] = (t <= row) ? mul * x[16 * blk + i] * ex2(g2 - s_g2[t]) : 0.f;
-                }
-            }
-        }
+        mask_decay_q(x, mul, row, ro.q, c0, g2, s_g2, s_b);
     };
     // sum / max of a per-thread partial over the four column quarters of this row (the same
     // order on every quarter, so all four get bit-identical results)
@@ -366,12 +355,16 @@ __global__ void __launch_bounds__(512, 1) bwd_chunk1_tc(const __grid_constant__ 
         const size_t gi = gate_index(it);
         const float lam = s_gate[row], beta = s_gate[128 + row];
         g2 = (s_gate[256 + row] + s_gate[384 + row]) * LOG2E;
+        const float g2e = (s_gate[512 + row] + s_gate[384 + row]) * LOG2E;   // token row | 15
         uint8_t* T_L1 = P + rL1 * TILE;   // dO, then Q
         uint8_t* T_A = P + rA * TILE;     // write vectors (rows = tokens)
         uint8_t* T_S = P + rS * TILE;     // staging
         const int rowtok = b * s.T + t0;
         const int snap_row = (bh * nct + cg) * 2 * 128;
-        if (cq == 0) s_g2[row] = g2;
+        if (cq == 0) {
+            s_g2[row] = g2;
+            s_b[row] = ex2(g2e - g2);
+        }
         if (ok) ok = mbar_wait(&bars[0], ph);
         if (tid == 0 && ok) pend &= ~0x1u;
         if (ok) ok = mbar_wait(&bars[3], ph);
@@ -927,6 +920,7 @@ __global__ void __launch_bounds__(512, 1) bwd_chunk2_tc(const __grid_constant__ 
     uint64_t* bars = reinterpret_cast<uint64_t*>(smem);
     uint32_t* s_taddr = reinterpret_cast<uint32_t*>(smem + 64);
     float* s_g2 = reinterpret_cast<float*>(smem + 128);
+    float* s_b = s_g2 + 128;          // [128] in-block decay factors
     uint8_t* P = smem + 2048;
     int rA = 0, rL2 = 4;              // the write-vector tile and the V / K tile swap each item
     uint8_t* T_AS = P + 1 * TILE;     // write vectors scaled by gamma^C / gamma^s
@@ -1007,20 +1001,7 @@ __global__ void __launch_bounds__(512, 1) bwd_chunk2_tc(const __grid_constant__ 
     };
     auto issuer = [&]() { return tid == 0 && ok; };
     auto mask_scores = [&](float (&x)[32], float mul) {
-#pragma unroll
-        for (int blk = 0; blk < 2; ++blk) {
-            const int tb = c0 + 32 * blk;
-            if (tb >= 32 * (ro.q + 1)) {
-#pragma unroll
-                for (int i = 0; i < 16; ++i) x[16 * blk + i] = 0.f;
-            } else {
-#pragma unroll
-                for (int i = 0; i < 16; ++i) {
-                    const int t = tb + i;
-                    x[16 * blk + i] = (t <= row) ? mul * x[16 * blk + i] * ex2(g2 - s_g2[t]) : 0.f;
-                }
-            }
-        }
+        mask_decay_q(x, mul, row, ro.q, c0, g2, s_g2, s_b);
     };
     for (int it = i0; it < i1 && ok; ++it) {
         const int bh = it / nct, cg = it - bh * nct, b = bh / s.H, h = bh % s.H;
@@ -1029,13 +1010,17 @@ __global__ void __launch_bounds__(512, 1) bwd_chunk2_tc(const __grid_constant__ 
         // gates: loaded while this item's first tiles land
         const float lam = a.lam[gi], beta = a.beta[gi];
         g2 = cum128(s, a.g, b, h, t0, t0 + row) * LOG2E;
+        const float g2e = cum128(s, a.g, b, h, t0, t0 + (row | 15)) * LOG2E;
         const float g2C = cum128(s, a.g, b, h, t0, t0 + CT - 1) * LOG2E;
         const float fw = ex2(g2C - g2);
         uint8_t* T_A = P + rA * TILE;     // write vectors a (fp16)
         uint8_t* L2 = P + rL2 * TILE;     // V (-> V->), then K (-> K->)
         const int rowtok = b * s.T + t0, rowbh = bh * s.T + t0;
         const int snap_row = (bh * nct + cg) * 2 * 128;
-        if (cq == 0) s_g2[row] = g2;
+        if (cq == 0) {
+            s_g2[row] = g2;
+            s_b[row] = ex2(g2e - g2);
+        }
         if (ok) ok = mbar_wait(&bars[0], ph) && mbar_wait(&bars[5], ph) && mbar_wait(&bars[6], ph);
         if (tid == 0 && ok) pend &= ~0x61u;
         if (ok) {   // dO and V: bf16 -> fp16
@@ -1353,7 +1338,7 @@ cudaError_t launch_bwd_tc(const TcBwdArgs& a, const TcFwdArgs& f, const void* q,
     const int sm_walk6 = 1024 + 6 * TILE + 1024;
     const int sm_snap_adj = 1024 + 4 * TC_SEGC * CT + 6 * TILE + 1024;
     const int sm_adj_seg = 1024 + 4 * TC_SEGC * CT + 4 * TILE + 1024;
-    const int sm_chunk1 = 7168 + 6 * TILE + 1024, sm_chunk2 = 2048 + 7 * TILE + 1024;
+    const int sm_chunk1 = 8192 + 6 * TILE + 1024, sm_chunk2 = 2048 + 7 * TILE + 1024;
     if (!a.saved) {
         cudaFuncSetAttribute(snap_fwd_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, sm_walk6);
         { LaunchScope ls_("tc_snap_fwd", st); snap_fwd_tc<<<gseg, 256, sm_walk6, st>>>(mk, mv, a); }

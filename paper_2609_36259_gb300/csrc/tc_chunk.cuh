@@ -376,6 +376,35 @@ __device__ __forceinline__ float omega_dot_q(const float (&x)[32], const float (
     return acc;
 }
 
+// Causal decay mask on the thread's 32 columns (tokens t = c0 + 32 blk + i of this chunk) of
+// row `row` (lane quarter q): x <- mul x 2^(g2 - g2_t) for t <= row, 0 otherwise, with g2 the
+// row's log2-domain cumulative decay and s_g2[t] the column's.  A 16-token block wholly before the
+// row uses 2^(g2 - g2_e) 2^(g2_e - g2_t), e the block's last token: both factors are <= 1 (no
+// overflow for any gate values), the first is one ex2 per thread and block, the second
+// (s_b[t] = 2^(s_g2[t | 15] - s_g2[t])) is shared by all rows.  Blocks that hold the diagonal
+// take one ex2 per entry.  Every kernel pairing score matrices across the backward uses this.
+__device__ __forceinline__ void mask_decay_q(float (&x)[32], float mul, int row, int q, int c0,
+                                             float g2, const float* s_g2, const float* s_b) {
+#pragma unroll
+    for (int blk = 0; blk < 2; ++blk) {
+        const int tb = c0 + 32 * blk, te = tb + 15;
+        if (tb >= 32 * (q + 1)) {   // every token of the block is after every row of the warp
+#pragma unroll
+            for (int i = 0; i < 16; ++i) x[16 * blk + i] = 0.f;
+        } else if (te < row) {
+            const float ar = mul * ex2(g2 - s_g2[te]);
+#pragma unroll
+            for (int i = 0; i < 16; ++i) x[16 * blk + i] = x[16 * blk + i] * ar * s_b[tb + i];
+        } else {
+#pragma unroll
+            for (int i = 0; i < 16; ++i) {
+                const int t = tb + i;
+                x[16 * blk + i] = (t <= row) ? mul * x[16 * blk + i] * ex2(g2 - s_g2[t]) : 0.f;
+            }
+        }
+    }
+}
+
 __device__ __forceinline__ float dot32(const float (&x)[32], const float (&y)[32]) {
     float acc = 0.f;
 #pragma unroll

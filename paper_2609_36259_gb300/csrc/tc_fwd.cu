@@ -205,6 +205,7 @@ __global__ void __launch_bounds__(512, 1) seg_out_tc(const __grid_constant__ CUt
     uint64_t* bars = reinterpret_cast<uint64_t*>(smem);          // tma q k, mma, m, tma v
     uint32_t* s_taddr = reinterpret_cast<uint32_t*>(smem + 32);
     float* s_g2 = reinterpret_cast<float*>(smem + 64);            // [128] log2-domain decays
+    float* s_b = s_g2 + 128;                                      // [128] in-block decay factors
     uint8_t* T_Q = smem + 2048;        // Q, later A-> (state-update operand)
     uint8_t* T_K = T_Q + 1 * TILE;
     uint8_t* T_V = T_Q + 2 * TILE;
@@ -303,30 +304,18 @@ __global__ void __launch_bounds__(512, 1) seg_out_tc(const __grid_constant__ CUt
         tc_fence_after();
     };
     auto issuer = [&]() { return tid == 0 && ok; };
-    // masked decay of the intra-chunk scores for this thread's 32 columns (t <= row only);
-    // 16-column blocks wholly above the diagonal of this warp's rows are skipped
-    auto mask_scores = [&](float (&x)[32], float g2, float mul) {
-#pragma unroll
-        for (int blk = 0; blk < 2; ++blk) {
-            const int tb = c0 + 32 * blk;
-            if (tb >= 32 * (ro.q + 1)) {
-#pragma unroll
-                for (int i = 0; i < 16; ++i) x[16 * blk + i] = 0.f;
-            } else {
-#pragma unroll
-                for (int i = 0; i < 16; ++i) {
-                    const int t = tb + i;
-                    x[16 * blk + i] = (t <= row) ? mul * x[16 * blk + i] * ex2(g2 - s_g2[t]) : 0.f;
-                }
-            }
-        }
+    auto mask_scores = [&](float (&x)[32], float g2_, float mul) {
+        mask_decay_q(x, mul, row, ro.q, c0, g2_, s_g2, s_b);
     };
 
     // Set-up of a chunk that needs no product of the previous one: its decays, its write vectors
     // (T_A) and its Q, K tiles (waited for and converted to fp16).  For chunk c + 1 it runs while
     // chunk c's last product (P2 V) is in flight.
-    auto chunk_setup = [&](float lam_, float beta_, float g2_) {
-        if (cq == 0) s_g2[row] = g2_;
+    auto chunk_setup = [&](float lam_, float beta_, float g2_, float g2e_) {
+        if (cq == 0) {
+            s_g2[row] = g2_;
+            s_b[row] = ex2(g2e_ - g2_);   // from this row's token to the end of its 16-block
+        }
         write_vector_q<__half>(T_A, row, hf, u, lam_, beta_);
         if (ok) ok = mbar_wait(&bars[0], qk_ph);
         if (tid == 0 && ok) qk_pending = false;
@@ -339,27 +328,29 @@ __global__ void __launch_bounds__(512, 1) seg_out_tc(const __grid_constant__ CUt
     // gates of the current and of the next chunk (prefetched one chunk ahead: the loads are
     // issued a chunk before their values are combined, so their latency is never waited for)
     float lam, beta, g2;
-    float n_lam = 0.f, n_beta = 0.f, n_ga = 0.f, n_gb = 0.f;
-    auto load_gates = [&](int c, float& l_, float& b_, float& ga, float& gb) {
+    float n_lam = 0.f, n_beta = 0.f, n_ga = 0.f, n_gb = 0.f, n_ge = 0.f;
+    auto load_gates = [&](int c, float& l_, float& b_, float& ga, float& gb, float& ge) {
         const int t0 = (c_begin + c) * CT, t = t0 + row;
         const size_t gi = ((size_t)b * s.T + t) * s.H + h;
         l_ = a.lam[gi];
         b_ = a.beta[gi];
-        // cum128 in two loads: g_cum is local to s.Cg-token chunks
+        // cum128 in two loads: g_cum is local to s.Cg-token chunks (row and row | 15 share the
+        // second term)
         ga = a.g[gi];
         gb = (s.Cg == 64 && t - t0 >= 64) ? a.g[((size_t)b * s.T + t0 + 63) * s.H + h] : 0.f;
+        ge = a.g[((size_t)b * s.T + t0 + (row | 15)) * s.H + h];
     };
     {
-        float ga, gb;
-        load_gates(0, lam, beta, ga, gb);
+        float ga, gb, ge;
+        load_gates(0, lam, beta, ga, gb, ge);
         g2 = (ga + gb) * LOG2E;
+        chunk_setup(lam, beta, g2, (ge + gb) * LOG2E);
     }
-    chunk_setup(lam, beta, g2);
     publish();
     for (int c = 0; c < nc && ok; ++c) {
         const int t0 = (c_begin + c) * CT;
         const size_t gi = ((size_t)b * s.T + t0 + row) * s.H + h;
-        if (c + 1 < nc) load_gates(c + 1, n_lam, n_beta, n_ga, n_gb);
+        if (c + 1 < nc) load_gates(c + 1, n_lam, n_beta, n_ga, n_gb, n_ge);
         const float g2C = s_g2[CT - 1];
         const float gam = ex2(g2);
         if (save && tid == 0) store_snap(c_begin + c, 0);
@@ -513,7 +504,7 @@ __global__ void __launch_bounds__(512, 1) seg_out_tc(const __grid_constant__ CUt
             lam = n_lam;
             beta = n_beta;
             g2 = (n_ga + n_gb) * LOG2E;
-            chunk_setup(lam, beta, g2);
+            chunk_setup(lam, beta, g2, (n_ge + n_gb) * LOG2E);
         }
         wait_mma();
         // next chunk's V (T_V is consumed), then o = gamma_r (O'' Vbar) + P2 V
