@@ -763,12 +763,18 @@ __global__ void __launch_bounds__(256, 1) adj_walk_tc(const __grid_constant__ CU
     for (int it = 0; it < total; ++it) {
         const int part = it / nc, c = chunk_of(it), buf = it & 1;
         const int cg = c_begin + c;
-        if (it >= 1 && ok) ok = mbar_wait(&bars[2 + ((it - 1) & 1)], ((it - 1) >> 1) & 1);
-        tc_fence_after();
-        if (tid == 0 && ok && it + 1 < total) {
-            if (SNAP) bulk_wait_read_all();   // the other buffer's S tile may be a store's source
-            issue(it + 1);
-        }
+        // product it - 1 must be complete before the other buffer is refilled (and, in the SNAP
+        // walk, before D is read); the refill goes out as early as possible: the walks are bound
+        // by how far ahead their loads run
+        auto refill = [&]() {
+            if (it >= 1 && ok) ok = mbar_wait(&bars[2 + ((it - 1) & 1)], ((it - 1) >> 1) & 1);
+            tc_fence_after();
+            if (tid == 0 && ok && it + 1 < total) {
+                if (SNAP) bulk_wait_read_all();   // the other buffer's S tile may be a store's source
+                issue(it + 1);
+            }
+        };
+        refill();
         if (ok) ok = mbar_wait(&bars[buf], (it >> 1) & 1);
         const float g = s_gs[c * CT + row];
         uint8_t* tX = tiles + (NT * buf) * TILE;
@@ -812,6 +818,7 @@ __global__ void __launch_bounds__(256, 1) adj_walk_tc(const __grid_constant__ CU
             scale_half_smem(tX, row, hf, w);
             bf16_to_f16_half(tX + TILE, row, hf);   // q or dO
         }
+
         fence_async_smem();
         tc_fence_before();
         ok = __syncthreads_and(ok);

@@ -88,14 +88,15 @@ __global__ void __launch_bounds__(256, 1) seg_state_tc(const __grid_constant__ C
     const uint32_t idesc = idesc_k16<OT>(128, 128, 1, 1);
     for (int c = 0; c < nc; ++c) {
         const int buf = c & 1;
-        if (c >= 1 && ok) ok = mbar_wait(&bars[2 + ((c - 1) & 1)], ((c - 1) >> 1) & 1);
-        if (tid == 0 && ok && c + 1 < nc) issue_kv(c + 1, (c + 1) & 1);
-        // A-> rows of this chunk, scaled by the decay from the token to the segment end
+        // A-> rows of this chunk, scaled by the decay from the token to the segment end (its
+        // buffer's last reader, product c - 2, is complete; product c - 1 runs meanwhile)
         {
             const int i = c * CT + ro.row;
             const float w = s_beta[i] * ex2((s_tot[c] - s_gs[i] + s_sfx[c]) * LOG2E);
             write_vector_half<OT>(tiles + 3 * buf * TILE, ro.row, ro.hf, s_lam[i], w);
         }
+        if (c >= 1 && ok) ok = mbar_wait(&bars[2 + ((c - 1) & 1)], ((c - 1) >> 1) & 1);
+        if (tid == 0 && ok && c + 1 < nc) issue_kv(c + 1, (c + 1) & 1);
         if (F16) {   // the bf16 K and V tiles become fp16 operands
             if (ok) ok = mbar_wait(&bars[buf], (c >> 1) & 1);
             if (ok) {
