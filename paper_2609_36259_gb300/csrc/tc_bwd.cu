@@ -415,8 +415,7 @@ __global__ void __launch_bounds__(512, 1) bwd_chunk1_tc(const __grid_constant__ 
         wait_mma();
         {   // do'' = gamma (dO Vbar^T) + P4 A, kept in X2
             float x[32], y[32];
-            tmem_ld16x2(tl + X2, x);
-            tmem_ld16x2(tl + X3, y);
+            tmem_ld16x2_pair(tl + X2, x, tl + X3, y);
     #pragma unroll
             for (int i = 0; i < 32; ++i) x[i] = fmaf(gam, x[i], y[i]);
             tmem_st16x2(tl + X2, x);
@@ -453,8 +452,7 @@ __global__ void __launch_bounds__(512, 1) bwd_chunk1_tc(const __grid_constant__ 
         wait_mma();
         {   // z = U(lam) o', kept in X3
             float x[32], y[32];
-            tmem_ld16x2(tl + X3, x);
-            tmem_ld16x2(tl + X4, y);
+            tmem_ld16x2_pair(tl + X3, x, tl + X4, y);
             const float f = scale * gam;
     #pragma unroll
             for (int i = 0; i < 32; ++i) x[i] = fmaf(f, x[i], y[i]);
@@ -507,8 +505,7 @@ __global__ void __launch_bounds__(512, 1) bwd_chunk1_tc(const __grid_constant__ 
     #pragma unroll
             for (int p8 = 0; p8 < 2; ++p8) {
                 float o[16], gv[16];
-                tmem_ld8x2(tl + X4 + 8 * p8, o);
-                tmem_ld8x2(tl + X2 + 8 * p8, gv);
+                tmem_ld8x2_pair(tl + X4 + 8 * p8, o, tl + X2 + 8 * p8, gv);
     #pragma unroll
                 for (int i = 0; i < 8; ++i) {
                     if (p8 + i > 0) ang.step();
@@ -541,8 +538,7 @@ __global__ void __launch_bounds__(512, 1) bwd_chunk1_tc(const __grid_constant__ 
         wait_mma();
         {   // dl = p o (dp - <p, dp>)
             float p[32], dp[32];
-            tmem_ld16x2(tl + X1, p);
-            tmem_ld16x2(tl + X4, dp);
+            tmem_ld16x2_pair(tl + X1, p, tl + X4, dp);
             const float pdp = row_reduce(dot32(p, dp), false);
     #pragma unroll
             for (int i = 0; i < 32; ++i) p[i] = p[i] * (dp[i] - pdp);
@@ -563,8 +559,7 @@ __global__ void __launch_bounds__(512, 1) bwd_chunk1_tc(const __grid_constant__ 
     #pragma unroll
             for (int p8 = 0; p8 < 2; ++p8) {
                 float dz[16], z[16];
-                tmem_ld8x2(tl + X2 + 8 * p8, dz);
-                tmem_ld8x2(tl + X3 + 8 * p8, z);
+                tmem_ld8x2_pair(tl + X2 + 8 * p8, dz, tl + X3 + 8 * p8, z);
     #pragma unroll
                 for (int i = 0; i < 8; ++i) {
                     if (p8 + i > 0) ang.step();
@@ -613,8 +608,7 @@ __global__ void __launch_bounds__(512, 1) bwd_chunk1_tc(const __grid_constant__ 
         if (issuer() && it + 1 < i1) issue_v(it + 1, T_K);
         if (ok) {   // dq = s gamma (dO' Kbar) + P3 K  (P3 carries s) ; <q, dq> = <q~, dq~>
             float x[32], y[32];
-            tmem_ld16x2(tl + X3, x);
-            tmem_ld16x2(tl + X4, y);
+            tmem_ld16x2_pair(tl + X3, x, tl + X4, y);
             const float f = scale * gam;
     #pragma unroll
             for (int i = 0; i < 32; ++i) x[i] = fmaf(f, x[i], y[i]);
@@ -1173,15 +1167,13 @@ __global__ void __launch_bounds__(512, 1) bwd_chunk2_tc(const __grid_constant__ 
         float cIG = 0.f, cL = 0.f, cIL = 0.f, db = 0.f;
         if (ok) {
             float x[32], y[32];
-            tmem_ld16x2(tl + X2, x);          // dk = P3^T Q + A-> D^K
-            tmem_ld16x2(tl + X1, y);
+            tmem_ld16x2_pair(tl + X2, x, tl + X1, y);   // dk = P3^T Q + A-> D^K
     #pragma unroll
             for (int i = 0; i < 32; ++i) x[i] += y[i];
             store_global_q(static_cast<__nv_bfloat16*>(a.dk) + gi * 128, c0, x);
             float av[32];
             write_vector_q_vals(av, hf, u, lam, beta);   // unrounded a
-            tmem_ld16x2(tl + X3, x);          // intra-chunk da (both passes)
-            tmem_ld16x2(tl + X4, y);          // inter-chunk da (both passes)
+            tmem_ld16x2_pair(tl + X3, x, tl + X4, y);   // intra- / inter-chunk da (both passes)
     #pragma unroll
             for (int i = 0; i < 32; ++i) db = fmaf(x[i] + y[i], av[i], db);
     #pragma unroll

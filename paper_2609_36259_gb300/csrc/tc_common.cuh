@@ -200,6 +200,48 @@ __device__ __forceinline__ void tmem_ld16x2(uint32_t taddr, float (&v)[32]) {
 #pragma unroll
     for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
 }
+// Two accumulators' blocks at once (tmem_ld16x2 at ta into a, at tb into b), one wait.
+__device__ __forceinline__ void tmem_ld16x2_pair(uint32_t ta, float (&a)[32], uint32_t tb, float (&b)[32]) {
+    uint32_t r[64];
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+        const uint32_t addr = (k < 2 ? ta : tb) + 32 * (k & 1);
+        uint32_t* o = r + 16 * k;
+        asm volatile(
+            "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, "
+            "%11, %12, %13, %14, %15}, [%16];"
+            : "=r"(o[0]), "=r"(o[1]), "=r"(o[2]), "=r"(o[3]), "=r"(o[4]), "=r"(o[5]), "=r"(o[6]),
+              "=r"(o[7]), "=r"(o[8]), "=r"(o[9]), "=r"(o[10]), "=r"(o[11]), "=r"(o[12]),
+              "=r"(o[13]), "=r"(o[14]), "=r"(o[15])
+            : "r"(addr));
+    }
+    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+    for (int i = 0; i < 32; ++i) {
+        a[i] = __uint_as_float(r[i]);
+        b[i] = __uint_as_float(r[32 + i]);
+    }
+}
+// Same with 8-column blocks (tmem_ld8x2 at ta into a, at tb into b), one wait.
+__device__ __forceinline__ void tmem_ld8x2_pair(uint32_t ta, float (&a)[16], uint32_t tb, float (&b)[16]) {
+    uint32_t r[32];
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+        const uint32_t addr = (k < 2 ? ta : tb) + 32 * (k & 1);
+        uint32_t* o = r + 8 * k;
+        asm volatile(
+            "tcgen05.ld.sync.aligned.32x32b.x8.b32 {%0, %1, %2, %3, %4, %5, %6, %7}, [%8];"
+            : "=r"(o[0]), "=r"(o[1]), "=r"(o[2]), "=r"(o[3]), "=r"(o[4]), "=r"(o[5]), "=r"(o[6]),
+              "=r"(o[7])
+            : "r"(addr));
+    }
+    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+    for (int i = 0; i < 16; ++i) {
+        a[i] = __uint_as_float(r[i]);
+        b[i] = __uint_as_float(r[16 + i]);
+    }
+}
 __device__ __forceinline__ void tmem_st16x2(uint32_t taddr, const float (&v)[32]) {
 #pragma unroll
     for (int blk = 0; blk < 2; ++blk) {

@@ -415,8 +415,7 @@ __global__ void __launch_bounds__(512, 1) seg_out_tc(const __grid_constant__ CUt
         wait_mma();   // P1 A
         {   // z = U(lam) o',  o' = s gamma_r (Q Kbar^T) + P1 A
             float x[32], y[32];
-            tmem_ld16x2(tl + X2, x);
-            tmem_ld16x2(tl + X1, y);
+            tmem_ld16x2_pair(tl + X2, x, tl + X1, y);
             const float f = scale * gam;
 #pragma unroll
             for (int i = 0; i < 32; ++i) x[i] = fmaf(f, x[i], y[i]);
@@ -512,8 +511,7 @@ __global__ void __launch_bounds__(512, 1) seg_out_tc(const __grid_constant__ CUt
         if (issuer() && c + 1 < nc) issue_v(c + 1);
         {
             float x[32], y[32];
-            tmem_ld16x2(tl + X2, x);
-            tmem_ld16x2(tl + X1, y);
+            tmem_ld16x2_pair(tl + X2, x, tl + X1, y);
 #pragma unroll
             for (int i = 0; i < 32; ++i) x[i] = fmaf(gam, x[i], y[i]);
             store_global_q(static_cast<__nv_bfloat16*>(a.o) + gi * 128, c0, x);
