@@ -682,13 +682,14 @@ __global__ void __launch_bounds__(256, 1) adj_walk_tc(const __grid_constant__ CU
     float* s_bnd = s_pre + TC_SEGC;                         // [TC_SEGC][2]
     float* s_gs = reinterpret_cast<float*>(smem + 1024);    // [TC_SEGC * CT] chunk-local decays
     constexpr int NT = SNAP ? 3 : 2;                       // tiles per buffer
+    constexpr int NB = SNAP ? 2 : 3;                       // buffers: loads run NB - 1 chunks ahead
     uint8_t* tiles = smem + 1024 + 4 * TC_SEGC * CT;       // [buf][X | Y (| S)]
     for (int i = tid; i < nc * CT; i += 256) {   // every token's decay, loaded once
         const int t0 = (c_begin + i / CT) * CT;
         s_gs[i] = cum128(s, a.g, b, h, t0, t0 + (i % CT));
     }
     if (tid == 0) {
-        for (int i = 0; i < 4; ++i) mbar_init(&bars[i], 1);
+        for (int i = 0; i < 2 * NB; ++i) mbar_init(&bars[i], 1);   // tma[NB], mma[NB]
         fence_mbar_init();
     }
     if (ro.warp == 0) tmem_alloc(s_taddr, 256);
@@ -728,8 +729,10 @@ __global__ void __launch_bounds__(256, 1) adj_walk_tc(const __grid_constant__ CU
         const int i = it % nc;
         return SNAP ? nc - 1 - i : i;
     };
+    int issued = 0, landed = 0;   // thread 0: loads issued / seen complete
     auto issue = [&](int it) {
-        const int part = it / nc, c = chunk_of(it), buf = it & 1;
+        const int part = it / nc, c = chunk_of(it), buf = it % NB;
+        ++issued;
         uint8_t* tX = tiles + (NT * buf) * TILE;
         uint8_t* tY = tX + TILE;
         const int t0 = (c_begin + c) * CT;
@@ -748,28 +751,30 @@ __global__ void __launch_bounds__(256, 1) adj_walk_tc(const __grid_constant__ CU
             tma_load_2d(tS + TILE / 2, &tsf, 64, srow, &bars[buf]);
         }
     };
-    if (tid == 0) issue(0);
+    if (tid == 0)
+        for (int i = 0; i < NB - 1 && i < total; ++i) issue(i);
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
     bool ok = true;
     const uint32_t id_nn = idesc_f16(128, 128, 1, 1);
     for (int it = 0; it < total; ++it) {
-        const int part = it / nc, c = chunk_of(it), buf = it & 1;
+        const int part = it / nc, c = chunk_of(it), buf = it % NB;
         const int cg = c_begin + c;
         // product it - 1 must be complete before the other buffer is refilled (and, in the SNAP
         // walk, before D is read); the refill goes out as early as possible: the walks are bound
         // by how far ahead their loads run
         auto refill = [&]() {
-            if (it >= 1 && ok) ok = mbar_wait(&bars[2 + ((it - 1) & 1)], ((it - 1) >> 1) & 1);
+            if (it >= 1 && ok) ok = mbar_wait(&bars[NB + (it - 1) % NB], ((it - 1) / NB) & 1);
             tc_fence_after();
-            if (tid == 0 && ok && it + 1 < total) {
+            if (tid == 0 && ok && it + NB - 1 < total) {
                 if (SNAP) bulk_wait_read_all();   // the other buffer's S tile may be a store's source
-                issue(it + 1);
+                issue(it + NB - 1);
             }
         };
         refill();
-        if (ok) ok = mbar_wait(&bars[buf], (it >> 1) & 1);
+        if (ok) ok = mbar_wait(&bars[buf], (it / NB) & 1);
+        if (tid == 0 && ok) ++landed;
         const float g = s_gs[c * CT + row];
         uint8_t* tX = tiles + (NT * buf) * TILE;
         float w;
@@ -832,10 +837,10 @@ __global__ void __launch_bounds__(256, 1) adj_walk_tc(const __grid_constant__ CU
             for (int k = 0; k < 8; ++k)
                 mma_bf16(taddr + 128 * part, mnmajor_desc(uX, 128, k), mnmajor_desc(uY, 128, k),
                          id_nn, (first && k == 0) ? 0u : 1u);
-            mma_commit(&bars[2 + buf]);
+            mma_commit(&bars[NB + buf]);
         }
     }
-    if (ok) ok = mbar_wait(&bars[2 + ((total - 1) & 1)], ((total - 1) >> 1) & 1);
+    if (ok) ok = mbar_wait(&bars[NB + (total - 1) % NB], ((total - 1) / NB) & 1);
     tc_fence_after();
     ok = __syncthreads_and(ok);
     if (SNAP && ok && tid < nc) {
@@ -856,7 +861,8 @@ __global__ void __launch_bounds__(256, 1) adj_walk_tc(const __grid_constant__ CU
     }
     if (!ok && tid == 0) {
         flag_error(CYFA_ERR_TIMEOUT);
-        for (int i = 0; i < 2; ++i) mbar_wait(&bars[i], 0);
+        // let every copy issued so far land before the shared memory is released
+        for (int i = landed; i < issued; ++i) mbar_wait(&bars[i % NB], (i / NB) & 1);
     }
     if (SNAP && tid == 0) bulk_wait_all();
     tc_fence_before();
@@ -1336,7 +1342,7 @@ cudaError_t launch_bwd_tc(const TcBwdArgs& a, const TcFwdArgs& f, const void* q,
     const dim3 gseg(s.B * s.H, a.nseg), gchunk(s.B * s.H, nct);
     const int sm_walk6 = 1024 + 6 * TILE + 1024;
     const int sm_snap_adj = 1024 + 4 * TC_SEGC * CT + 6 * TILE + 1024;
-    const int sm_adj_seg = 1024 + 4 * TC_SEGC * CT + 4 * TILE + 1024;
+    const int sm_adj_seg = 1024 + 4 * TC_SEGC * CT + 6 * TILE + 1024;
     const int sm_chunk1 = 8192 + 6 * TILE + 1024, sm_chunk2 = 2048 + 7 * TILE + 1024;
     if (!a.saved) {
         cudaFuncSetAttribute(snap_fwd_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, sm_walk6);
