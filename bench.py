@@ -52,12 +52,13 @@ def kernel_flops_per_token_head(name, C, d=128, ms=MS):
         'tc_adj_segment': 4 * d * ms,
         'tc_snap_adj': 4 * d * ms,
         'tc_bwd_chunk2': 12 * 2 * 128 * 128,
+        'tc_dm_reduce': 2 * 2 * 128 * 128,                         # dl z^T + p dy^T for dR
     }
     return table.get(name)
 
 
 TENSOR_KERNELS = ('tc_seg_state', 'tc_seg_out', 'tc_snap_fwd', 'tc_bwd_chunk1', 'tc_adj_segment',
-                  'tc_snap_adj', 'tc_bwd_chunk2')
+                  'tc_snap_adj', 'tc_bwd_chunk2', 'tc_dm_reduce')
 
 
 def operator_flops_per_token_head(C, d=128, ms=MS):
@@ -221,6 +222,9 @@ def run_ours(args):
     dq, dk, dv = torch.empty_like(inp['q']), torch.empty_like(inp['k']), torch.empty_like(inp['v'])
     dc, dd, db = torch.empty_like(lam), torch.empty_like(lam), torch.empty_like(lam)
     dA = torch.empty(H, **f32)
+    # the readout's gradient (the tensor-core kernels give it; a training step needs it)
+    dR = (torch.empty(H, 127, 127, **f32)
+          if cyfa.cyfa_saved_size(d) > 0 and not args.no_dR else None)
     ws_p = cyfa.workspace(d, cyfa.CYFA_WS_PREPARE, dev)
     ws_f = cyfa.workspace(d, cyfa.CYFA_WS_FWD, dev)
     ws_b = cyfa.workspace(d, cyfa.CYFA_WS_BWD, dev)
@@ -237,7 +241,7 @@ def run_ours(args):
         if args.no_bwd:
             return
         cyfa.cyfa_chunk_bwd(d, x['q'], x['k'], x['v'], lam, g, beta, x['R'], x['clock_logit'],
-                            x['decay_logit'], x['A'], x['dO'], dq, dk, dv, dc, dd, db, None, dA,
+                            x['decay_logit'], x['A'], x['dO'], dq, dk, dv, dc, dd, db, dR, dA,
                             ws_b, saved=saved)
 
     for _ in range(args.warmup):
@@ -322,7 +326,7 @@ def run_ours(args):
     # end to end through the public API with host buffers
     e2e = None
     if not args.no_e2e:
-        e2e = run_e2e(args, d, inp, dev, step_outputs=(o, dq, dk, dv, dc, dd, db),
+        e2e = run_e2e(args, d, inp, dev, step_outputs=tuple(x for x in (o, dq, dk, dv, dc, dd, db, dA, dR) if x is not None),
                       step=step)
 
     del ws_f, ws_b
@@ -338,6 +342,7 @@ def run_ours(args):
                    'arithmetic': ('tcgen05 fp16 operands, fp32 accumulate' if tc_path
                                   else 'fp32 CUDA cores'),
                    'saved_states': saved is not None,
+                   'grads': 'q, k, v, clock, decay, beta logits, A' + (', R' if dR is not None else ''),
                    'global_batch': B * world, 'seq_len': T,
                    'parallelism': 'dp%d' % world,
                    'l2': 'inputs larger than L2 (q,k,v,dO %.0f MB)' % (4 * B * T * H * D * 2 / 1e6)},
@@ -497,6 +502,8 @@ def main():
     ap.add_argument('--ref-tokens', type=int, default=256)
     ap.add_argument('--no-decode', action='store_true')
     ap.add_argument('--no-e2e', action='store_true')
+    ap.add_argument('--no-dR', action='store_true',
+                    help='leave the readout gradient dR out of the backward')
     ap.add_argument('--no-saved', action='store_true',
                     help='backward recomputes the chunk-start states instead of reading the '
                          'ones the forward saved')

@@ -88,6 +88,9 @@ struct BwdLayout {
     __half *Mb, *snapF, *snapA, *O2b, *DO1b;   // tensor-core path (fp16 operands)
     float *segS, *segG, *segD, *bnd;
     double* dA_chunk;
+    __half *mZ, *mP, *mDY, *mDL;     // middle-readout vectors for dR
+    float* dMp;
+    int dm_split;
     int nseg;
     size_t bytes;
 };
@@ -116,6 +119,13 @@ BwdLayout bwd_layout(const Shape& s0, bool tc_path, void* ws) {
         L.DO1b = c.take<__half>(BH * s.T * MS);
         L.bnd = c.take<float>(BH * nct * 2);
         L.dA_chunk = c.take<double>(BH * nct);
+        L.mZ = c.take<__half>(BH * s.T * MS);
+        L.mP = c.take<__half>(BH * s.T * MS);
+        L.mDY = c.take<__half>(BH * s.T * MS);
+        L.mDL = c.take<__half>(BH * s.T * MS);
+        const size_t nch = (size_t)s.B * nct;
+        L.dm_split = (int)(nch < 32 ? nch : 32);
+        L.dMp = c.take<float>((size_t)s.H * L.dm_split * MS * MS);
     } else {
         L.states = c.take<float>(BH * s.nchunk() * MS * 2 * s.D);
         L.adj = c.take<float>(BH * s.nchunk() * MS * 2 * s.D);
@@ -273,10 +283,10 @@ int cyfa_chunk_bwd(const cyfa_dims_t* dims, const void* q, const void* k, const 
     if (!aligned16(q) || !aligned16(k) || !aligned16(v) || !aligned16(dO) || !aligned16(dq) ||
         !aligned16(dk) || !aligned16(dv))
         return CYFA_ERR_ALIGN;
-    if (dR) return CYFA_ERR_UNSUPPORTED;
     if (saved && !aligned16(saved)) return CYFA_ERR_ALIGN;
     const Shape s = shape_of(dims);
     const bool tc_path = use_tc(dims, s);
+    if (dR && !tc_path) return CYFA_ERR_UNSUPPORTED;
     const BwdLayout need = bwd_layout(s, tc_path, nullptr);
     if (!workspace || workspace_bytes < need.bytes) return CYFA_ERR_WORKSPACE;
     if (!aligned16(workspace)) return CYFA_ERR_ALIGN;
@@ -354,6 +364,13 @@ int cyfa_chunk_bwd(const cyfa_dims_t* dims, const void* q, const void* k, const 
         t.d_beta = d_beta_logit;
         t.dA = dA;
         t.dA_part = L.dA_chunk;
+        t.dR = dR;
+        t.mZ = dR ? L.mZ : nullptr;
+        t.mP = dR ? L.mP : nullptr;
+        t.mDY = dR ? L.mDY : nullptr;
+        t.mDL = dR ? L.mDL : nullptr;
+        t.dMp = L.dMp;
+        t.dm_split = L.dm_split;
         return cuda_status(launch_bwd_tc(t, f, q, k, v, dO, L.M, st));
     }
     return cuda_status(launch_bwd_simt(a, st));

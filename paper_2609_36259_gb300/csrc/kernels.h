@@ -144,6 +144,12 @@ struct TcBwdArgs {
     const float *clock_logit, *decay_logit, *A;
     float *d_clock, *d_decay, *d_beta, *dA;
     double* dA_part;             // [B*H][T/128]
+    // dR (nullable): per-token z, p, dy, dl of the middle readout (fp16 [B*H][T][128]: z, dy in
+    // the kernels' Fourier order, p, dl over the slots), per-head partial dM and the output
+    __half *mZ, *mP, *mDY, *mDL;
+    float* dMp;                  // [H][dm_split][128][128]
+    int dm_split;
+    float* dR;                   // [H][127][127]
 };
 cudaError_t launch_bwd_tc(const TcBwdArgs& a, const TcFwdArgs& f, const void* q, const void* k,
                           const void* v, const void* dO, const float* Mf, cudaStream_t st);

@@ -224,6 +224,10 @@ __global__ void __launch_bounds__(512, 1) bwd_chunk1_tc(const __grid_constant__ 
                                                          const __grid_constant__ CUtensorMap tdo,
                                                          const __grid_constant__ CUtensorMap tm,
                                                          const __grid_constant__ CUtensorMap tsf,
+                                                         const __grid_constant__ CUtensorMap tmz,
+                                                         const __grid_constant__ CUtensorMap tmp,
+                                                         const __grid_constant__ CUtensorMap tmdy,
+                                                         const __grid_constant__ CUtensorMap tmdl,
                                                          TcBwdArgs a) {
     const Shape s = a.s;
     const int nct = s.T / CT;
@@ -305,6 +309,18 @@ __global__ void __launch_bounds__(512, 1) bwd_chunk1_tc(const __grid_constant__ 
         tc_fence_after();
     };
     auto issuer = [&]() { return tid == 0 && ok; };
+    // the staging tile (rows = the item's tokens) out to a [B*H*T][128] fp16 array by a TMA store
+    // that runs beside the product reading the same tile; after the product, a barrier behind
+    // thread 0's wait for the store's read guards the tile's next writes
+    auto store_staged = [&](const CUtensorMap* map, const uint8_t* tile, int rowbh) {
+        tma_store_2d(map, tile, 0, rowbh);
+        tma_store_2d(map, tile + TILE / 2, 64, rowbh);
+        bulk_commit();
+    };
+    auto staged_read = [&]() {   // every thread, after the product: the store has read the tile
+        if (tid == 0) bulk_wait_read_all();
+        __syncthreads();
+    };
     // gates of the current item, and the next item's prefetched
     auto gate_index = [&](int item) {
         const int ibh = item / nct, icg = item - ibh * nct, ib = ibh / s.H, ih = ibh - ib * s.H;
@@ -359,7 +375,7 @@ __global__ void __launch_bounds__(512, 1) bwd_chunk1_tc(const __grid_constant__ 
         uint8_t* T_L1 = P + rL1 * TILE;   // dO, then Q
         uint8_t* T_A = P + rA * TILE;     // write vectors (rows = tokens)
         uint8_t* T_S = P + rS * TILE;     // staging
-        const int rowtok = b * s.T + t0;
+        const int rowtok = b * s.T + t0, rowbh = bh * s.T + t0;
         const int snap_row = (bh * nct + cg) * 2 * 128;
         if (cq == 0) {
             s_g2[row] = g2;
@@ -462,12 +478,14 @@ __global__ void __launch_bounds__(512, 1) bwd_chunk1_tc(const __grid_constant__ 
         }
         publish();
         if (issuer()) {   // G5: X1 = z M^T
+            if (a.mZ) store_staged(&tmz, T_S, rowbh);
     #pragma unroll
             for (int k = 0; k < 8; ++k)
                 mma_bf16(taddr + X1, kmajor_desc(uS, 128, k), kmajor_desc(uM, 128, k), id_kk, k > 0);
             mma_commit(&bars[2]);
         }
         wait_mma();
+        if (a.mZ) staged_read();   // the staging tile is rewritten below (uniform branch)
         {   // p = softmax(l) over the m valid entries (the padding column is out), kept in X1
             float x[32];
             tmem_ld16x2(tl + X1, x);
@@ -491,12 +509,14 @@ __global__ void __launch_bounds__(512, 1) bwd_chunk1_tc(const __grid_constant__ 
         }
         publish();
         if (issuer()) {   // G6: X4 = p M
+            if (a.mP) store_staged(&tmp, T_S, rowbh);
     #pragma unroll
             for (int k = 0; k < 8; ++k)
                 mma_bf16(taddr + X4, kmajor_desc(uS, 128, k), mnmajor_desc(uM, 128, k), id_kn, k > 0);
             mma_commit(&bars[2]);
         }
         wait_mma();
+        if (a.mZ) staged_read();   // the staging tile is rewritten below (uniform branch)
         {   // o'' = U(-lam) (p M); scalars with do'' (o'' as stored in fp16); dy = U(lam) do''.
             // Eight rotation pairs at a time: cosine entries, then sine entries.
             QuarterAngles ang(lam, hf, u);
@@ -530,12 +550,14 @@ __global__ void __launch_bounds__(512, 1) bwd_chunk1_tc(const __grid_constant__ 
         }
         publish();
         if (issuer()) {   // G7: X4 = dy M^T = M dy
+            if (a.mDY) store_staged(&tmdy, T_S, rowbh);
     #pragma unroll
             for (int k = 0; k < 8; ++k)
                 mma_bf16(taddr + X4, kmajor_desc(uS, 128, k), kmajor_desc(uM, 128, k), id_kk, k > 0);
             mma_commit(&bars[2]);
         }
         wait_mma();
+        if (a.mZ) staged_read();   // the staging tile is rewritten below (uniform branch)
         {   // dl = p o (dp - <p, dp>)
             float p[32], dp[32];
             tmem_ld16x2_pair(tl + X1, p, tl + X4, dp);
@@ -546,12 +568,14 @@ __global__ void __launch_bounds__(512, 1) bwd_chunk1_tc(const __grid_constant__ 
         }
         publish();
         if (issuer()) {   // G8: X2 = dl M = M^T dl
+            if (a.mDL) store_staged(&tmdl, T_S, rowbh);
     #pragma unroll
             for (int k = 0; k < 8; ++k)
                 mma_bf16(taddr + X2, kmajor_desc(uS, 128, k), mnmajor_desc(uM, 128, k), id_kn, k > 0);
             mma_commit(&bars[2]);
         }
         wait_mma();
+        if (a.mZ) staged_read();   // the staging tile is rewritten below (uniform branch)
         {   // do' = U(-lam) dz; <do', Omega o'> with do' as stored in fp16 (= <dz, Omega z> exactly)
             QuarterAngles ang(lam, hf, u);
             const bool dcq = (hf == 1 && u == 1);
@@ -642,6 +666,7 @@ __global__ void __launch_bounds__(512, 1) bwd_chunk1_tc(const __grid_constant__ 
         if (pend & 0x2u) mbar_wait(&bars[1], (pend >> 5) & 1);
         if (pend & 0x4u) mbar_wait(&bars[3], (pend >> 6) & 1);
     }
+    if (tid == 0) bulk_wait_all();
     tc_fence_before();
     __syncthreads();
     if (ro.warp == 0) tmem_dealloc(taddr, 512);
@@ -1229,6 +1254,131 @@ __global__ void __launch_bounds__(512, 1) bwd_chunk2_tc(const __grid_constant__ 
     if (ro.warp == 0) tmem_dealloc(taddr, 512);
 }
 
+// ---------------------------------------------------------------------------------------
+// dR (Sec. 3.3: the middle readout l = M z, p = softmax(l), y = M^T p with M = R Phi): the
+// gradient of M is dM = sum_t (dl_t z_t^T + p_t dy_t^T), summed over the batch; then
+// dR = dM Phi^T.  dm_reduce_tc: CTA (h, split) runs over its share of the head's 128-token
+// chunks (all batch rows) and accumulates DL^T Z + P^T DY on tcgen05 in TMEM (the vectors were
+// written in fp16 by bwd_chunk1_tc), streaming pairs of tiles through a three-stage TMA ring.
+constexpr int DM_NS = 3;
+
+__global__ void __launch_bounds__(256, 1) dm_reduce_tc(const __grid_constant__ CUtensorMap tz,
+                                                        const __grid_constant__ CUtensorMap tp,
+                                                        const __grid_constant__ CUtensorMap tdy,
+                                                        const __grid_constant__ CUtensorMap tdl,
+                                                        TcBwdArgs a) {
+    const Shape s = a.s;
+    const int h = blockIdx.x, split = blockIdx.y;
+    const int nct = s.T / CT, nch = s.B * nct;   // the head's chunks over the batch
+    const int c0i = (int)((long long)nch * split / a.dm_split);
+    const int c1i = (int)((long long)nch * (split + 1) / a.dm_split);
+    const int NT = 2 * (c1i - c0i);              // steps: (DL, Z) then (P, DY) per chunk
+    const int tid = threadIdx.x, warp = tid >> 5;
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                               ~uintptr_t(1023));
+    uint64_t* bar_tma = reinterpret_cast<uint64_t*>(smem);
+    uint64_t* bar_mma = bar_tma + DM_NS;
+    uint32_t* s_taddr = reinterpret_cast<uint32_t*>(smem + 128);
+    uint8_t* tiles = smem + 1024;   // [stage][X | Y]
+    if (tid == 0) {
+        for (int i = 0; i < 2 * DM_NS; ++i) mbar_init(&bar_tma[i], 1);
+        fence_mbar_init();
+    }
+    if (warp == 0) tmem_alloc(s_taddr, 128);
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t taddr = *s_taddr;
+    int issued = 0, landed = 0;
+    auto issue = [&](int it) {
+        const int st = it % DM_NS, ch = c0i + it / 2, b = ch / nct, c = ch - b * nct;
+        const int rowbh = (b * s.H + h) * s.T + c * CT;
+        uint8_t* tX = tiles + (2 * st) * TILE;
+        const CUtensorMap* mx = (it & 1) ? &tp : &tdl;
+        const CUtensorMap* my = (it & 1) ? &tdy : &tz;
+        mbar_expect_tx(&bar_tma[st], 2 * TILE);
+        tma_load_2d(tX, mx, 0, rowbh, &bar_tma[st]);
+        tma_load_2d(tX + TILE / 2, mx, 64, rowbh, &bar_tma[st]);
+        tma_load_2d(tX + TILE, my, 0, rowbh, &bar_tma[st]);
+        tma_load_2d(tX + TILE + TILE / 2, my, 64, rowbh, &bar_tma[st]);
+        ++issued;
+    };
+    if (tid == 0)
+        for (int i = 0; i < DM_NS - 1 && i < NT; ++i) issue(i);
+    bool ok = true;
+    const uint32_t id_nn = idesc_f16(128, 128, 1, 1);
+    if (tid == 0) {   // one thread runs the ring: the tiles need no touch-up
+        for (int it = 0; it < NT && ok; ++it) {
+            const int st = it % DM_NS;
+            if (it >= 1) ok = mbar_wait(&bar_mma[(it - 1) % DM_NS], ((it - 1) / DM_NS) & 1);
+            if (ok && it + DM_NS - 1 < NT) issue(it + DM_NS - 1);
+            if (ok) ok = mbar_wait(&bar_tma[st], (it / DM_NS) & 1);
+            if (!ok) break;
+            ++landed;
+            tc_fence_after();
+            const uint32_t uX = smem_u32(tiles + (2 * st) * TILE), uY = uX + TILE;
+#pragma unroll
+            for (int k = 0; k < 8; ++k)
+                mma_bf16(taddr, mnmajor_desc(uX, 128, k), mnmajor_desc(uY, 128, k), id_nn,
+                         (it == 0 && k == 0) ? 0u : 1u);
+            mma_commit(&bar_mma[st]);
+        }
+        if (ok && NT > 0) ok = mbar_wait(&bar_mma[(NT - 1) % DM_NS], ((NT - 1) / DM_NS) & 1);
+    }
+    tc_fence_after();
+    ok = __syncthreads_and(ok);
+    float* dst = a.dMp + ((size_t)h * a.dm_split + split) * 128 * 128;
+    const int q = warp & 3, hf = warp >> 2, lrow = 32 * q + (tid & 31);
+    if (ok && NT > 0) {
+        float x[64];
+        tmem_ld64(taddr + ((uint32_t)(32 * q) << 16) + 64 * hf, x);
+#pragma unroll
+        for (int i = 0; i < 64; i += 4)
+            *reinterpret_cast<float4*>(dst + lrow * 128 + 64 * hf + i) = make_float4(x[i], x[i + 1], x[i + 2], x[i + 3]);
+    } else if (ok) {   // no chunk in this split
+        for (int i = 0; i < 64; ++i) dst[lrow * 128 + 64 * hf + i] = 0.f;
+    } else if (tid == 0) {
+        flag_error(CYFA_ERR_TIMEOUT);
+        for (int i = landed; i < issued; ++i) mbar_wait(&bar_tma[i % DM_NS], (i / DM_NS) & 1);
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 0) tmem_dealloc(taddr, 128);
+}
+
+// dR[h][i][k] = sum_j dM[h][i][j] Phi[k][j] for the m active slots i, k (dM summed over the
+// splits; its column j is in the kernels' Fourier order).  One block per (h, i).
+__global__ void __launch_bounds__(128) dr_finalize_kernel(TcBwdArgs a) {
+    const int h = blockIdx.x, i = blockIdx.y, t = threadIdx.x;
+    __shared__ float s_dm[128], s_ct[MA], s_st[MA];
+    {
+        float acc = 0.f;
+        const float* src = a.dMp + (size_t)h * a.dm_split * 128 * 128 + i * 128 + t;
+        for (int sp = 0; sp < a.dm_split; ++sp) acc += src[(size_t)sp * 128 * 128];
+        s_dm[paper_slot(t)] = acc;   // paper order: DC, cos_1, sin_1, ..., pad
+    }
+    if (t < MA) {
+        float sv, cv;
+        sincospif((float)t * (2.f / 127.f), &sv, &cv);
+        s_ct[t] = cv;
+        s_st[t] = sv;
+    }
+    __syncthreads();
+    if (t < MA) {   // k = t: Phi[k][0] = 1/sqrt(m), Phi[k][2j-1] = sqrt(2/m) cos(2 pi j k / m), ...
+        float acc = s_dm[0] * INV_SQRT_M;
+        float ac = 0.f, as = 0.f;
+        int idx = 0;
+        for (int j = 1; j <= NPAIR; ++j) {
+            idx += t;
+            if (idx >= MA) idx -= MA;
+            ac = fmaf(s_dm[2 * j - 1], s_ct[idx], ac);
+            as = fmaf(s_dm[2 * j], s_st[idx], as);
+        }
+        a.dR[((size_t)h * MA + i) * MA + t] = acc + SQRT_2_OVER_M * (ac + as);
+    }
+}
+
 // Gate gradients of one chunk: chunk-local suffix sums of the per-token scalars plus the
 // state-level term of everything after the chunk, then the activation derivatives.
 __global__ void __launch_bounds__(128) tc_gate_kernel(TcBwdArgs a) {
@@ -1356,8 +1506,17 @@ cudaError_t launch_bwd_tc(const TcBwdArgs& a, const TcFwdArgs& f, const void* q,
             return cudaErrorInvalidValue;
         const long long items = (long long)s.B * s.H * nct;
         const int grid1 = (int)(items < sms ? items : sms);
+        // the staged vectors of dR go out by TMA store; without dR the maps are unused stand-ins
+        CUtensorMap mz, mpp, mdy, mdl;
+        const void* bz = a.mZ ? (const void*)a.mZ : (const void*)a.DO1;
+        const void* bp = a.mP ? (const void*)a.mP : (const void*)a.DO1;
+        const void* bdy = a.mDY ? (const void*)a.mDY : (const void*)a.DO1;
+        const void* bdl = a.mDL ? (const void*)a.mDL : (const void*)a.DO1;
+        if (!tc_rows_map(&mz, bz, BH * s.T, true) || !tc_rows_map(&mpp, bp, BH * s.T, true) ||
+            !tc_rows_map(&mdy, bdy, BH * s.T, true) || !tc_rows_map(&mdl, bdl, BH * s.T, true))
+            return cudaErrorInvalidValue;
         LaunchScope ls_("tc_bwd_chunk1", st);
-        bwd_chunk1_tc<<<grid1, 512, sm_chunk1, st>>>(mq, mk, mv, mdo, mm, msf, a);
+        bwd_chunk1_tc<<<grid1, 512, sm_chunk1, st>>>(mq, mk, mv, mdo, mm, msf, mz, mpp, mdy, mdl, a);
     }
     cudaFuncSetAttribute(adj_walk_tc<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, sm_adj_seg);
     { LaunchScope ls_("tc_adj_segment", st); adj_walk_tc<false><<<gseg, 256, sm_adj_seg, st>>>(mdo1, mo2, mq, mdo, msf, msa, a); }
@@ -1376,6 +1535,16 @@ cudaError_t launch_bwd_tc(const TcBwdArgs& a, const TcFwdArgs& f, const void* q,
         bwd_chunk2_tc<<<grid2, 512, sm_chunk2, st>>>(mq, mk, mv, mdo, mo2, mdo1, msa, a);
     }
     { LaunchScope ls_("tc_gate", st); tc_gate_kernel<<<gchunk, 128, 0, st>>>(a); }
+    if (a.dR) {   // dR from the middle-readout vectors bwd_chunk1_tc wrote
+        CUtensorMap mz, mp, mdy, mdl;
+        if (!tc_rows_map(&mz, a.mZ, BH * s.T, true) || !tc_rows_map(&mp, a.mP, BH * s.T, true) ||
+            !tc_rows_map(&mdy, a.mDY, BH * s.T, true) || !tc_rows_map(&mdl, a.mDL, BH * s.T, true))
+            return cudaErrorInvalidValue;
+        const int sm_dm = 1024 + 2 * DM_NS * TILE + 1024;
+        cudaFuncSetAttribute(dm_reduce_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, sm_dm);
+        { LaunchScope ls_("tc_dm_reduce", st); dm_reduce_tc<<<dim3(s.H, a.dm_split), 256, sm_dm, st>>>(mz, mp, mdy, mdl, a); }
+        { LaunchScope ls_("tc_dr_finalize", st); dr_finalize_kernel<<<dim3(s.H, MA), 128, 0, st>>>(a); }
+    }
     if (a.dA) { LaunchScope ls_("tc_dA", st); tc_dA_kernel<<<s.H, 256, 0, st>>>(a); }
     return cudaGetLastError();
 }

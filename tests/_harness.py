@@ -38,6 +38,19 @@ def assert_close_sum(got, want, l1, what=''):
     return err
 
 
+def assert_close_rel(got, want, what=''):
+    """A matrix of sums over every token (dR): rel-L2 within the bf16 bar, and max-abs within
+    the bf16 max-abs bar relative to the largest entry."""
+    got = np.asarray(got, dtype=np.float64)
+    want = np.asarray(want, dtype=np.float64)
+    scale = max(1.0, float(np.max(np.abs(want))))
+    err = float(np.max(np.abs(got - want))) / scale
+    rl = rel_l2(got, want)
+    assert err <= BF16_MAX_ABS and rl <= BF16_REL_L2, \
+        '%s: max-abs/max %.3e (bar %.0e), rel-L2 %.3e (bar %.0e)' % (what, err, BF16_MAX_ABS, rl, BF16_REL_L2)
+    return err, rl
+
+
 def assert_close_fp32(got, want, what=''):
     err = float(np.max(np.abs(np.asarray(got, np.float64) - np.asarray(want, np.float64))))
     assert err <= FP32_MAX_ABS, '%s: max-abs %.3e (bar %.0e)' % (what, err, FP32_MAX_ABS)

@@ -5,7 +5,8 @@ import torch
 
 from paper_2609_36259_gb300 import cyfa, synth
 
-from _harness import (assert_close_bf16, assert_close_fp32, assert_close_sum, gpu_prepare,
+from _harness import (assert_close_bf16, assert_close_fp32, assert_close_rel, assert_close_sum,
+                      gpu_prepare,
                       oracle_backward,
                       oracle_inputs, pairs_np, sample_pairs, to_device)
 
@@ -15,7 +16,7 @@ GRADS = (('dq', 'dq'), ('dk', 'dk'), ('dv', 'dv'), ('d_clock', 'd_clock'),
          ('d_decay', 'd_decay'), ('d_beta', 'd_beta'))
 
 
-def gpu_backward(d, inp, want_dA=True, use_saved=False):
+def gpu_backward(d, inp, want_dA=True, use_saved=False, want_dR=False):
     lam, g, beta, _ = gpu_prepare(d, inp)
     q, k, v, dO = inp['q'], inp['k'], inp['v'], inp['dO']
     saved = None
@@ -29,11 +30,12 @@ def gpu_backward(d, inp, want_dA=True, use_saved=False):
                d_clock=torch.empty_like(inp['clock_logit']),
                d_decay=torch.empty_like(inp['clock_logit']),
                d_beta=torch.empty_like(inp['clock_logit']),
-               dA=torch.empty_like(inp['A']) if want_dA else None)
+               dA=torch.empty_like(inp['A']) if want_dA else None,
+               dR=torch.empty_like(inp['R']) if want_dR else None)
     ws = cyfa.workspace(d, cyfa.CYFA_WS_BWD, q.device)
     cyfa.cyfa_chunk_bwd(d, q, k, v, lam, g, beta, inp['R'], inp['clock_logit'],
                         inp['decay_logit'], inp['A'], dO, out['dq'], out['dk'], out['dv'],
-                        out['d_clock'], out['d_decay'], out['d_beta'], None, out['dA'], ws,
+                        out['d_clock'], out['d_decay'], out['d_beta'], out['dR'], out['dA'], ws,
                         saved=saved)
     torch.cuda.synchronize()
     return out
@@ -52,10 +54,16 @@ def test_backward_small_bf16(B, T, H, D, C, cuda_cores):
     T = 2304 spans several 1024-token segments plus a partial one."""
     inp = to_device(synth.make_inputs(B, T, H, D, seed=8, with_dO=True))
     d = cyfa.dims(B, T, H, D, chunk=C, cuda_cores=cuda_cores)
-    out = gpu_backward(d, inp)
+    tc = cyfa.cyfa_saved_size(d) > 0   # the tensor-core kernels (they also give dR)
+    out = gpu_backward(d, inp, want_dR=tc)
     pairs = [(b, h) for b in range(B) for h in range(H)]
     ref = oracle_backward(oracle_inputs(inp, pairs), pairs_np(inp['dO'], pairs))
     _compare(out, ref, pairs, assert_close_bf16)
+    if tc:
+        dR_ref = np.zeros((H, 127, 127))
+        for n, (b, h) in enumerate(pairs):
+            dR_ref[h] += ref['dR'][n]
+        assert_close_rel(out['dR'].double().cpu().numpy(), dR_ref, 'dR')
     dA_ref, l1 = np.zeros(H), np.zeros(H)
     f = pairs_np(inp['decay_logit'], pairs)
     softplus = np.logaddexp(0.0, f)
@@ -114,3 +122,12 @@ def test_backward_saved_full_size_sampled():
     pairs = sample_pairs(B, H, 2)
     ref = oracle_backward(oracle_inputs(inp, pairs), pairs_np(inp['dO'], pairs))
     _compare(out, ref, pairs, assert_close_bf16, 'saved full')
+
+
+def test_backward_dR_unsupported_on_cuda_cores():
+    """dR comes from the tensor-core kernels; the CUDA-core kernels refuse it before launching."""
+    B, T, H, D = 1, 256, 2, 64
+    inp = to_device(synth.make_inputs(B, T, H, D, seed=3, with_dO=True))
+    d = cyfa.dims(B, T, H, D, chunk=64)
+    with pytest.raises(cyfa.CyfaError):
+        gpu_backward(d, inp, want_dR=True)
