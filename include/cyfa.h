@@ -154,9 +154,8 @@ int cyfa_chunk_fwd(const cyfa_dims_t* dims, const void* q, const void* k, const 
  * the reverse cumulative sum dL/d delta_s = sum_{t>=s} dL/d lambda_t of App. D.1 Eq.
  * app-clock-gradient-accumulation; the decay gradient is the reverse cumulative sum of
  * the per-token gradient of the cumulative log-decay.  dR [H,m,m] and dA [H] are sums
- * over the batch; dR (through M = R Phi of the middle readout, Sec. 3.3 Eq. cyfa-two-pass) is
- * computed by the tensor-core kernels only: on the CUDA-core kernels a non-null dR returns
- * CYFA_ERR_UNSUPPORTED.  Inputs are those of cyfa_chunk_fwd plus the raw clock / decay logits
+ * over the batch (dR through M = R Phi of the middle readout, Sec. 3.3 Eq. cyfa-two-pass).
+ * Inputs are those of cyfa_chunk_fwd plus the raw clock / decay logits
  * and A (for the activation derivatives).  saved (nullable): the buffer a cyfa_chunk_fwd call
  * with the same dims, inputs and no initial state filled; the chunk-start states are then
  * read from it instead of being recomputed.  Ignored where cyfa_saved_size is 0.

@@ -42,11 +42,13 @@ __device__ __forceinline__ float warp_omega_dot(const float* x, const float* y, 
 
 // Gradient of the middle readout, one warp per row:
 // given o' (sO1), o'' (sO2) and dL/do'' (sD), writes dL/do' into sD and the row scalars
-// sdG[r] = <o'', do''> and sdL[r] = <dz, Omega z> - <do'', Omega o''>.
+// sdG[r] = <o'', do''> and sdL[r] = <dz, Omega z> - <do'', Omega o''>.  With gz non-null the
+// row's z, p, dy, dl (for dR) go to gz / gp / gdy / gdl + 128 r.
 __device__ __noinline__ void middle_rows_bwd(const float* sO1, const float* sO2, float* sD,
                                              const float* slam, int C, const float* M,
                                              const float* MT, float* swarp, float* sdG,
-                                             float* sdL) {
+                                             float* sdL, float* gz, float* gp, float* gdy,
+                                             float* gdl) {
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     float* z = swarp + warp * 640;
     float* p = z + 128;
@@ -116,6 +118,16 @@ __device__ __noinline__ void middle_rows_bwd(const float* sO1, const float* sO2,
         pdp = warp_sum(pdp);
 #pragma unroll
         for (int u = 0; u < 4; ++u) dl[lane + 32 * u] = e[u] * (dp[u] - pdp);
+        if (gz) {
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+                const int k = lane + 32 * u;
+                gz[r * 128 + k] = z[k];
+                gp[r * 128 + k] = e[u];
+                gdy[r * 128 + k] = dy[k];
+                gdl[r * 128 + k] = e[u] * (dp[u] - pdp);
+            }
+        }
         __syncwarp();
         float g[4] = {0.f, 0.f, 0.f, 0.f};                   // dz = M^T dl
         for (int i = 0; i < MA; ++i) {
@@ -317,7 +329,13 @@ __global__ void __launch_bounds__(256) bwd_intra1_kernel(BwdArgs a) {
             for (int j = 0; j < 8; ++j) sD[(ty + 16 * i) * LD + tx + 16 * j] = g2[i][j];
     }
     __syncthreads();
-    middle_rows_bwd(sO1, sO2, sD, slam, CB, Mh, MTh, swarp, sdG, sdL);
+    {
+        const size_t rowbase = ((size_t)bh * s.T + t0) * MS;
+        const bool dr = a.mZ != nullptr;
+        middle_rows_bwd(sO1, sO2, sD, slam, CB, Mh, MTh, swarp, sdG, sdL,
+                        dr ? a.mZ + rowbase : nullptr, dr ? a.mP + rowbase : nullptr,
+                        dr ? a.mDY + rowbase : nullptr, dr ? a.mDL + rowbase : nullptr);
+    }
     __syncthreads();
 
     // dQ~ = gamma o (dO' Kbar) + (dO' A^T o Gamma) K ;  dq = s dQ~
@@ -704,6 +722,23 @@ __global__ void dA_final_kernel(BwdArgs a, int nseg) {
     a.dA[h] = (float)t;
 }
 
+// dM[h][i][j] = sum over the batch and the tokens of dl[i] z[j] + p[i] dy[j] (paper order), one
+// block per (h, i), one thread per j.
+__global__ void __launch_bounds__(128) dm_reduce_simt(BwdArgs a) {
+    const Shape s = a.s;
+    const int h = blockIdx.x, i = blockIdx.y, j = threadIdx.x;
+    float acc = 0.f;
+    for (int b = 0; b < s.B; ++b) {
+        const size_t base = ((size_t)b * s.H + h) * s.T * MS;
+        for (int t = 0; t < s.T; ++t) {
+            const size_t o = base + (size_t)t * MS;
+            acc = fmaf(a.mDL[o + i], a.mZ[o + j], acc);
+            acc = fmaf(a.mP[o + i], a.mDY[o + j], acc);
+        }
+    }
+    a.dM[((size_t)h * MS + i) * MS + j] = acc;
+}
+
 template <int D, typename TI>
 cudaError_t bwd_dispatch(const BwdArgs& a, cudaStream_t st) {
     const Shape& s = a.s;
@@ -731,6 +766,11 @@ cudaError_t bwd_dispatch(const BwdArgs& a, cudaStream_t st) {
     auto k2 = bwd_intra2_kernel<D, TI>;
     cudaFuncSetAttribute(k2, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm2);
     { LaunchScope ls_("bwd_intra2", st); k2<<<gchunk, 256, sm2, st>>>(a); }
+    if (a.dR) {
+        { LaunchScope ls_("bwd_dm_reduce", st); dm_reduce_simt<<<dim3(s.H, MS), 128, 0, st>>>(a); }
+        e = launch_dr_finalize(a.dM, 1, s.H, false, a.dR, st);
+        if (e != cudaSuccess) return e;
+    }
     return launch_bwd_gates(a, st);
 }
 

@@ -89,6 +89,7 @@ struct BwdLayout {
     float *segS, *segG, *segD, *bnd;
     double* dA_chunk;
     __half *mZ, *mP, *mDY, *mDL;     // middle-readout vectors for dR
+    float *fZ, *fP, *fDY, *fDL, *fdM;   // the same on the CUDA-core path (fp32)
     float* dMp;
     int dm_split;
     int nseg;
@@ -131,6 +132,11 @@ BwdLayout bwd_layout(const Shape& s0, bool tc_path, void* ws) {
         L.adj = c.take<float>(BH * s.nchunk() * MS * 2 * s.D);
         L.o2 = c.take<float>(BH * s.T * MS);
         L.do1 = c.take<float>(BH * s.T * MS);
+        L.fZ = c.take<float>(BH * s.T * MS);
+        L.fP = c.take<float>(BH * s.T * MS);
+        L.fDY = c.take<float>(BH * s.T * MS);
+        L.fDL = c.take<float>(BH * s.T * MS);
+        L.fdM = c.take<float>((size_t)s.H * MS * MS);
     }
     L.bytes = c.off;
     return L;
@@ -286,7 +292,6 @@ int cyfa_chunk_bwd(const cyfa_dims_t* dims, const void* q, const void* k, const 
     if (saved && !aligned16(saved)) return CYFA_ERR_ALIGN;
     const Shape s = shape_of(dims);
     const bool tc_path = use_tc(dims, s);
-    if (dR && !tc_path) return CYFA_ERR_UNSUPPORTED;
     const BwdLayout need = bwd_layout(s, tc_path, nullptr);
     if (!workspace || workspace_bytes < need.bytes) return CYFA_ERR_WORKSPACE;
     if (!aligned16(workspace)) return CYFA_ERR_ALIGN;
@@ -323,6 +328,12 @@ int cyfa_chunk_bwd(const cyfa_dims_t* dims, const void* q, const void* k, const 
     a.tok = L.tok;
     a.seg = L.seg;
     a.dA_part = L.dA_part;
+    a.dR = tc_path ? nullptr : dR;
+    a.mZ = (dR && !tc_path) ? L.fZ : nullptr;
+    a.mP = (dR && !tc_path) ? L.fP : nullptr;
+    a.mDY = (dR && !tc_path) ? L.fDY : nullptr;
+    a.mDL = (dR && !tc_path) ? L.fDL : nullptr;
+    a.dM = L.fdM;
     if (tc_path) {
         TcFwdArgs f{};
         f.s = s;

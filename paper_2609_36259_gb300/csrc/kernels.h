@@ -75,7 +75,15 @@ struct BwdArgs {
     float* tok;         // [4][B*T*H]: dG part 1, d lambda part 1, dG part 2 / d lambda part 2 / d beta
     double* seg;        // [2][B*H][nseg] reverse-scan partials
     double* dA_part;    // [B*H*nseg]
+    // dR (nullable): per-token z, p, dy, dl of the middle readout (fp32 [B*H][T][128], paper
+    // order), the per-head dM and the output [H][127][127]
+    float *mZ, *mP, *mDY, *mDL;
+    float *dM, *dR;
 };
+// dR[h] = dM[h] Phi^T over the m active slots from dm_split partial dM blocks [H][split][128][128]
+// whose Fourier (column) index is in the tensor-core order (tc_order) or in the paper's order.
+cudaError_t launch_dr_finalize(const float* dMp, int dm_split, int H, bool tc_order, float* dR,
+                               cudaStream_t st);
 constexpr int BWD_C = 64;       // chunk length used by the SIMT backward
 cudaError_t launch_bwd_simt(const BwdArgs& a, cudaStream_t st);
 // reverse cumulative sums of the per-token scalars in a.tok and the logit gradients

@@ -1348,15 +1348,17 @@ __global__ void __launch_bounds__(256, 1) dm_reduce_tc(const __grid_constant__ C
 }
 
 // dR[h][i][k] = sum_j dM[h][i][j] Phi[k][j] for the m active slots i, k (dM summed over the
-// splits; its column j is in the kernels' Fourier order).  One block per (h, i).
-__global__ void __launch_bounds__(128) dr_finalize_kernel(TcBwdArgs a) {
+// splits; its column j in the kernels' Fourier order when tc_order, else in the paper's).  One
+// block per (h, i).
+__global__ void __launch_bounds__(128) dr_finalize_kernel(const float* dMp, int dm_split,
+                                                          bool tc_order, float* dR) {
     const int h = blockIdx.x, i = blockIdx.y, t = threadIdx.x;
     __shared__ float s_dm[128], s_ct[MA], s_st[MA];
     {
         float acc = 0.f;
-        const float* src = a.dMp + (size_t)h * a.dm_split * 128 * 128 + i * 128 + t;
-        for (int sp = 0; sp < a.dm_split; ++sp) acc += src[(size_t)sp * 128 * 128];
-        s_dm[paper_slot(t)] = acc;   // paper order: DC, cos_1, sin_1, ..., pad
+        const float* src = dMp + (size_t)h * dm_split * 128 * 128 + i * 128 + t;
+        for (int sp = 0; sp < dm_split; ++sp) acc += src[(size_t)sp * 128 * 128];
+        s_dm[tc_order ? paper_slot(t) : t] = acc;   // paper order: DC, cos_1, sin_1, ..., pad
     }
     if (t < MA) {
         float sv, cv;
@@ -1375,7 +1377,7 @@ __global__ void __launch_bounds__(128) dr_finalize_kernel(TcBwdArgs a) {
             ac = fmaf(s_dm[2 * j - 1], s_ct[idx], ac);
             as = fmaf(s_dm[2 * j], s_st[idx], as);
         }
-        a.dR[((size_t)h * MA + i) * MA + t] = acc + SQRT_2_OVER_M * (ac + as);
+        dR[((size_t)h * MA + i) * MA + t] = acc + SQRT_2_OVER_M * (ac + as);
     }
 }
 
@@ -1543,9 +1545,16 @@ cudaError_t launch_bwd_tc(const TcBwdArgs& a, const TcFwdArgs& f, const void* q,
         const int sm_dm = 1024 + 2 * DM_NS * TILE + 1024;
         cudaFuncSetAttribute(dm_reduce_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, sm_dm);
         { LaunchScope ls_("tc_dm_reduce", st); dm_reduce_tc<<<dim3(s.H, a.dm_split), 256, sm_dm, st>>>(mz, mp, mdy, mdl, a); }
-        { LaunchScope ls_("tc_dr_finalize", st); dr_finalize_kernel<<<dim3(s.H, MA), 128, 0, st>>>(a); }
+        e = launch_dr_finalize(a.dMp, a.dm_split, s.H, true, a.dR, st);
+        if (e != cudaSuccess) return e;
     }
     if (a.dA) { LaunchScope ls_("tc_dA", st); tc_dA_kernel<<<s.H, 256, 0, st>>>(a); }
+    return cudaGetLastError();
+}
+
+cudaError_t launch_dr_finalize(const float* dMp, int dm_split, int H, bool tc_order, float* dR,
+                               cudaStream_t st) {
+    { LaunchScope ls_("dr_finalize", st); dr_finalize_kernel<<<dim3(H, MA), 128, 0, st>>>(dMp, dm_split, tc_order, dR); }
     return cudaGetLastError();
 }
 

@@ -54,16 +54,14 @@ def test_backward_small_bf16(B, T, H, D, C, cuda_cores):
     T = 2304 spans several 1024-token segments plus a partial one."""
     inp = to_device(synth.make_inputs(B, T, H, D, seed=8, with_dO=True))
     d = cyfa.dims(B, T, H, D, chunk=C, cuda_cores=cuda_cores)
-    tc = cyfa.cyfa_saved_size(d) > 0   # the tensor-core kernels (they also give dR)
-    out = gpu_backward(d, inp, want_dR=tc)
+    out = gpu_backward(d, inp, want_dR=True)
     pairs = [(b, h) for b in range(B) for h in range(H)]
     ref = oracle_backward(oracle_inputs(inp, pairs), pairs_np(inp['dO'], pairs))
     _compare(out, ref, pairs, assert_close_bf16)
-    if tc:
-        dR_ref = np.zeros((H, 127, 127))
-        for n, (b, h) in enumerate(pairs):
-            dR_ref[h] += ref['dR'][n]
-        assert_close_rel(out['dR'].double().cpu().numpy(), dR_ref, 'dR')
+    dR_ref = np.zeros((H, 127, 127))
+    for n, (b, h) in enumerate(pairs):
+        dR_ref[h] += ref['dR'][n]
+    assert_close_rel(out['dR'].double().cpu().numpy(), dR_ref, 'dR')
     dA_ref, l1 = np.zeros(H), np.zeros(H)
     f = pairs_np(inp['decay_logit'], pairs)
     softplus = np.logaddexp(0.0, f)
@@ -77,7 +75,7 @@ def test_backward_fp32():
     B, T, H, D = 1, 256, 2, 64
     inp = to_device(synth.make_inputs(B, T, H, D, seed=9, with_dO=True, dtype=torch.float32))
     d = cyfa.dims(B, T, H, D, chunk=64, dtype=torch.float32)
-    out = gpu_backward(d, inp)
+    out = gpu_backward(d, inp, want_dR=True)
     pairs = [(0, 0), (0, 1)]
     ref = oracle_backward(oracle_inputs(inp, pairs), pairs_np(inp['dO'], pairs))
     for gk, rk in GRADS:
@@ -85,6 +83,10 @@ def test_backward_fp32():
         scale = max(1.0, float(np.abs(ref[rk]).max()))
         err = float(np.abs(got - ref[rk]).max())
         assert err <= 1e-4 * scale, (gk, err, scale)
+    got = out['dR'].double().cpu().numpy()   # both heads of the single batch row
+    scale = max(1.0, float(np.abs(ref['dR']).max()))
+    err = float(np.abs(got - ref['dR']).max())
+    assert err <= 1e-4 * scale, ('dR', err, scale)
 
 
 @pytest.mark.parametrize('B,T,H,C,cuda_cores', [(4, 8192, 16, 64, False), (4, 8192, 16, 64, True),
@@ -122,12 +124,3 @@ def test_backward_saved_full_size_sampled():
     pairs = sample_pairs(B, H, 2)
     ref = oracle_backward(oracle_inputs(inp, pairs), pairs_np(inp['dO'], pairs))
     _compare(out, ref, pairs, assert_close_bf16, 'saved full')
-
-
-def test_backward_dR_unsupported_on_cuda_cores():
-    """dR comes from the tensor-core kernels; the CUDA-core kernels refuse it before launching."""
-    B, T, H, D = 1, 256, 2, 64
-    inp = to_device(synth.make_inputs(B, T, H, D, seed=3, with_dO=True))
-    d = cyfa.dims(B, T, H, D, chunk=64)
-    with pytest.raises(cyfa.CyfaError):
-        gpu_backward(d, inp, want_dR=True)
