@@ -326,8 +326,7 @@ def run_ours(args):
     # end to end through the public API with host buffers
     e2e = None
     if not args.no_e2e:
-        e2e = run_e2e(args, d, inp, dev, step_outputs=tuple(x for x in (o, dq, dk, dv, dc, dd, db, dA, dR) if x is not None),
-                      step=step)
+        e2e = run_e2e(args, inp, dev, want_dR=dR is not None)
 
     del ws_f, ws_b
     line = {
@@ -418,40 +417,82 @@ def run_decode(args, dev, peaks, rank):
             'frac_hbm_8TBs': gbs / 8000.0}
 
 
-def run_e2e(args, d, inp, dev, step_outputs, step):
-    """The same step through the public API with pinned host buffers: every step copies its
-    inputs host->device and reads every output back."""
+def run_e2e(args, inp, dev, want_dR):
+    """The step through the public API with pinned host buffers: every step copies all its inputs
+    host->device and reads every output back.  The batch rows go as micro-batches on their own
+    CUDA streams (each with its own workspaces), so one row's copies overlap another row's
+    kernels and the two copy directions overlap each other; the per-row dA / dR partials are
+    read back and summed on the host."""
     import torch
+    from paper_2609_36259_gb300 import cyfa
+    B, T, H, D = inp['q'].shape
     keys = ('q', 'k', 'v', 'clock_logit', 'decay_logit', 'beta_logit', 'dO')
-    host = {k: inp[k].cpu().pin_memory() for k in keys}
-    outs_h = [t.new_empty(t.shape, device='cpu').pin_memory() for t in step_outputs]
-    dev_in = {k: torch.empty_like(inp[k]) for k in keys}
-    x = dict(inp)
-    x.update(dev_in)
-    h2d = sum(t.numel() * t.element_size() for t in host.values())
-    d2h = sum(t.numel() * t.element_size() for t in outs_h)
+    d1 = cyfa.dims(1, T, H, D, chunk=args.chunk, cuda_cores=args.cuda_cores)
+    rows = []
+    for b in range(B):
+        r = {'stream': torch.cuda.Stream(device=dev)}
+        r['host'] = {k: inp[k][b:b + 1].cpu().pin_memory() for k in keys}
+        r['x'] = {k: torch.empty_like(inp[k][b:b + 1]) for k in keys}
+        r['x'].update({k: inp[k] for k in ('A', 'R')})
+        f32 = dict(dtype=torch.float32, device=dev)
+        lam = torch.empty(1, T, H, **f32)
+        r['gates'] = (lam, torch.empty_like(lam), torch.empty_like(lam))
+        r['out'] = dict(o=torch.empty_like(r['x']['v']), dq=torch.empty_like(r['x']['q']),
+                        dk=torch.empty_like(r['x']['k']), dv=torch.empty_like(r['x']['v']),
+                        dc=torch.empty_like(lam), dd=torch.empty_like(lam), db=torch.empty_like(lam),
+                        dA=torch.empty(H, **f32))
+        if want_dR:
+            r['out']['dR'] = torch.empty(H, 127, 127, **f32)
+        r['host_out'] = {k: t.new_empty(t.shape, device='cpu').pin_memory() for k, t in r['out'].items()}
+        r['ws'] = [cyfa.workspace(d1, w, dev) for w in (cyfa.CYFA_WS_PREPARE, cyfa.CYFA_WS_FWD, cyfa.CYFA_WS_BWD)]
+        r['saved'] = None if args.no_saved else cyfa.saved_buffer(d1, dev)
+        rows.append(r)
+    h2d = sum(t.numel() * t.element_size() for r in rows for t in r['host'].values())
+    d2h = sum(t.numel() * t.element_size() for r in rows for t in r['host_out'].values())
 
     def one():
-        for k in keys:
-            dev_in[k].copy_(host[k], non_blocking=True)
-        step(x)
-        for hb, t in zip(outs_h, step_outputs):
-            hb.copy_(t, non_blocking=True)
+        main = torch.cuda.current_stream(dev)
+        ev = main.record_event()
+        for r in rows:
+            st, x, o = r['stream'], r['x'], r['out']
+            st.wait_event(ev)
+            with torch.cuda.stream(st):
+                for k in keys:
+                    x[k].copy_(r['host'][k], non_blocking=True)
+                lam, g, beta = r['gates']
+                cyfa.cyfa_prepare(d1, x['clock_logit'], x['decay_logit'], x['beta_logit'], x['A'],
+                                  None, lam, g, beta, None, r['ws'][0], stream=st)
+                cyfa.cyfa_chunk_fwd(d1, x['q'], x['k'], x['v'], lam, g, beta, x['R'], None, None,
+                                    o['o'], None, None, r['ws'][1], stream=st, saved=r['saved'])
+                cyfa.cyfa_chunk_bwd(d1, x['q'], x['k'], x['v'], lam, g, beta, x['R'],
+                                    x['clock_logit'], x['decay_logit'], x['A'], x['dO'], o['dq'],
+                                    o['dk'], o['dv'], o['dc'], o['dd'], o['db'], o.get('dR'), o['dA'],
+                                    r['ws'][2], stream=st, saved=r['saved'])
+                for k, t in o.items():
+                    r['host_out'][k].copy_(t, non_blocking=True)
+        for r in rows:
+            main.wait_stream(r['stream'])
+
     for _ in range(2):
         one()
     torch.cuda.synchronize()
     n = max(1, min(args.steps, 3))
-    t0 = time.perf_counter()
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    t0 = time.perf_counter()
     e0.record()
     for _ in range(n):
         one()
     e1.record()
     torch.cuda.synchronize()
+    # the batch sums of dA and dR from the rows' partials (host side, inside the wall clock)
+    dA = sum(r['host_out']['dA'] for r in rows)
+    if want_dR:
+        dR = sum(r['host_out']['dR'] for r in rows)
+    wall = (time.perf_counter() - t0) / n
     ms = e0.elapsed_time(e1) / n
-    B, T = inp['q'].shape[0], inp['q'].shape[1]
     return {'value': B * T / (ms / 1e3), 'unit': 'tokens/s', 'h2d_bytes_per_step': h2d,
-            'd2h_bytes_per_step': d2h, 'ms_per_step': ms}
+            'd2h_bytes_per_step': d2h, 'ms_per_step': ms, 'wall_ms_per_step': wall * 1e3,
+            'micro_batches': B}
 
 
 # ---------------------------------------------------------------------------- reference
