@@ -21,7 +21,7 @@ using namespace tc;
 
 // ---------------------------------------------------------------------------------------
 template <int SEGC, typename OT>
-__global__ void __launch_bounds__(256, 1) seg_state_tc(const __grid_constant__ CUtensorMap tk,
+__global__ void __launch_bounds__(512, 1) seg_state_tc(const __grid_constant__ CUtensorMap tk,
                                                         const __grid_constant__ CUtensorMap tv,
                                                         TcFwdArgs a) {
     const Shape s = a.s;
@@ -30,7 +30,7 @@ __global__ void __launch_bounds__(256, 1) seg_state_tc(const __grid_constant__ C
     const int c_begin = seg * SEGC;
     const int nc = min(SEGC, nct - c_begin);
     const int tid = threadIdx.x;
-    const Role ro;
+    const QRole ro;   // 512 threads: one row and one column quarter each
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                                ~uintptr_t(1023));
@@ -42,7 +42,7 @@ __global__ void __launch_bounds__(256, 1) seg_state_tc(const __grid_constant__ C
     float* s_beta = s_lam + SEGC * CT;
     float* s_gs = s_beta + SEGC * CT;                                // chunk-local decays
     uint8_t* tiles = smem + 1024 + 12 * SEGC * CT;                   // [buf][A | K | V]
-    for (int i = tid; i < nc * CT; i += 256) {   // every token's gates, loaded once
+    for (int i = tid; i < nc * CT; i += 512) {   // every token's gates, loaded once
         const int t0 = (c_begin + i / CT) * CT, t = t0 + i % CT;
         const size_t gi = ((size_t)b * s.T + t) * s.H + h;
         s_lam[i] = a.lam[gi];
@@ -93,15 +93,15 @@ __global__ void __launch_bounds__(256, 1) seg_state_tc(const __grid_constant__ C
         {
             const int i = c * CT + ro.row;
             const float w = s_beta[i] * ex2((s_tot[c] - s_gs[i] + s_sfx[c]) * LOG2E);
-            write_vector_half<OT>(tiles + 3 * buf * TILE, ro.row, ro.hf, s_lam[i], w);
+            write_vector_q<OT>(tiles + 3 * buf * TILE, ro.row, ro.hf, ro.u, s_lam[i], w);
         }
         if (c >= 1 && ok) ok = mbar_wait(&bars[2 + ((c - 1) & 1)], ((c - 1) >> 1) & 1);
         if (tid == 0 && ok && c + 1 < nc) issue_kv(c + 1, (c + 1) & 1);
         if (F16) {   // the bf16 K and V tiles become fp16 operands
             if (ok) ok = mbar_wait(&bars[buf], (c >> 1) & 1);
             if (ok) {
-                bf16_to_f16_half(tiles + (3 * buf + 1) * TILE, ro.row, ro.hf);
-                bf16_to_f16_half(tiles + (3 * buf + 2) * TILE, ro.row, ro.hf);
+                bf16_to_f16_q(tiles + (3 * buf + 1) * TILE, ro.row, ro.c0);
+                bf16_to_f16_q(tiles + (3 * buf + 2) * TILE, ro.row, ro.c0);
             }
         }
         fence_async_smem();
@@ -127,10 +127,10 @@ __global__ void __launch_bounds__(256, 1) seg_state_tc(const __grid_constant__ C
     if (ok) ok = mbar_wait(&bars[2 + ((nc - 1) & 1)], ((nc - 1) >> 1) & 1);
     tc_fence_after();
     ok = __syncthreads_and(ok);
-    if (ok) {
-        float* dst = a.segS + (((size_t)bh * a.nseg + seg) * 128 + ro.row) * 256 + 128 * ro.hf;
-        const uint32_t tl = taddr + ((uint32_t)(32 * ro.q) << 16) + 128 * ro.hf;
-        for (int c0 = 0; c0 < 128; c0 += 32) {
+    if (ok) {   // [Kbar | Vbar] delta out: each thread 64 of the row's 256 columns
+        float* dst = a.segS + (((size_t)bh * a.nseg + seg) * 128 + ro.row) * 256 + 64 * ro.cq;
+        const uint32_t tl = taddr + ((uint32_t)(32 * ro.q) << 16) + 64 * ro.cq;
+        for (int c0 = 0; c0 < 64; c0 += 32) {
             float v[32];
             tmem_ld32(tl + c0, v);
 #pragma unroll
@@ -605,7 +605,7 @@ cudaError_t launch_fwd_segment_states(const TcFwdArgs& a, const void* k, const v
     const int smA = 1024 + 12 * SEGC_DEFAULT * CT + 6 * TILE + 1024;
     auto kA = seg_state_tc<SEGC_DEFAULT, __half>;
     cudaFuncSetAttribute(kA, cudaFuncAttributeMaxDynamicSharedMemorySize, smA);
-    { LaunchScope ls_("tc_seg_state", st); kA<<<grid, 256, smA, st>>>(mk, mv, a); }
+    { LaunchScope ls_("tc_seg_state", st); kA<<<grid, 512, smA, st>>>(mk, mv, a); }
     { LaunchScope ls_("tc_seg_scan", st); seg_scan_kernel<<<dim3(128, s.B * s.H), 256, 0, st>>>(a); }
     return cudaGetLastError();
 }
