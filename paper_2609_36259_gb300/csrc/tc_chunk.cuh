@@ -56,25 +56,33 @@ __host__ __device__ __forceinline__ int paper_slot(int t) {
     return (l >= 32) ? 2 * j : 2 * j - 1;
 }
 
+// sin(pi x), cos(pi x) for a phase x in [0, 2) (a phase_pi value) on the special-function unit.
+// The argument is first reduced to [-1, 1), where the unit's absolute error is about 2^-21: far
+// below the fp16 rounding (2^-11 relative) of every tensor-core operand these angles feed.
+__device__ __forceinline__ void sincospi_fast(float x, float* s, float* c) {
+    if (x >= 1.f) x -= 2.f;
+    __sincosf(3.14159265358979f * x, s, c);
+}
+
 // Rotation angles theta_j = 2 pi j lam / m for the 32 pairs of one column half, produced in
 // order by angle addition from theta_1 (cos(x + y) = cos x cos y - sin x sin y,
-// sin(x + y) = sin x cos y + cos x sin y), re-seeded from sincospif every 16 steps.
+// sin(x + y) = sin x cos y + cos x sin y), re-seeded from sincospi_fast every 16 steps.
 struct HalfAngles {
     float c1, s1, c, s, lam;
     int j0;
     __device__ __forceinline__ HalfAngles(float lam_, int hf) : lam(lam_), j0(32 * hf + 1) {
-        sincospif(phase_pi(lam, 1), &s1, &c1);
+        sincospi_fast(phase_pi(lam, 1), &s1, &c1);
         if (j0 == 1) {
             c = c1;
             s = s1;
         } else {
-            sincospif(phase_pi(lam, j0), &s, &c);
+            sincospi_fast(phase_pi(lam, j0), &s, &c);
         }
     }
     // advance to local pair jj (1..31)
     __device__ __forceinline__ void step(int jj) {
         if (jj == 16) {
-            sincospif(phase_pi(lam, j0 + 16), &s, &c);
+            sincospi_fast(phase_pi(lam, j0 + 16), &s, &c);
         } else {
             const float cn = c * c1 - s * s1;
             const float sn = s * c1 + c * s1;
@@ -208,18 +216,18 @@ struct QRole {
     }
 };
 
-// Angles of the 16 pairs of a quarter by angle addition from theta_1, seeded with sincospif at
+// Angles of the 16 pairs of a quarter by angle addition from theta_1, seeded with sincospi_fast at
 // the quarter's first pair (the same seeds as HalfAngles).
 struct QuarterAngles {
     float c1, s1, c, s;
     __device__ __forceinline__ QuarterAngles(float lam, int hf, int u) {
         const int j0 = 32 * hf + 16 * u + 1;
-        sincospif(phase_pi(lam, 1), &s1, &c1);
+        sincospi_fast(phase_pi(lam, 1), &s1, &c1);
         if (j0 == 1) {
             c = c1;
             s = s1;
         } else {
-            sincospif(phase_pi(lam, j0), &s, &c);
+            sincospi_fast(phase_pi(lam, j0), &s, &c);
         }
     }
     __device__ __forceinline__ void step() {
@@ -378,28 +386,47 @@ __device__ __forceinline__ float omega_dot_q(const float (&x)[32], const float (
 
 // Causal decay mask on the thread's 32 columns (tokens t = c0 + 32 blk + i of this chunk) of
 // row `row` (lane quarter q): x <- mul x 2^(g2 - g2_t) for t <= row, 0 otherwise, with g2 the
-// row's log2-domain cumulative decay and s_g2[t] the column's.  A 16-token block wholly before the
-// row uses 2^(g2 - g2_e) 2^(g2_e - g2_t), e the block's last token: both factors are <= 1 (no
-// overflow for any gate values), the first is one ex2 per thread and block, the second
-// (s_b[t] = 2^(s_g2[t | 15] - s_g2[t])) is shared by all rows.  Blocks that hold the diagonal
-// take one ex2 per entry.  Every kernel pairing score matrices across the backward uses this.
+// row's log2-domain cumulative decay and s_g2[t] the column's.  Each 16-token block is classed
+// for the whole warp (rows 32q .. 32q + 31), so no warp runs two paths:
+//  * after every row of the warp: zero;
+//  * before every row of the warp: 2^(g2 - g2_e) 2^(g2_e - g2_t), e the block's last token; both
+//    factors are <= 1 (no overflow for any gate values), the first is one ex2 per thread and
+//    block, the second (s_b[t] = 2^(s_g2[t | 15] - s_g2[t])) is shared by all rows;
+//  * holding the diagonal of some row of the warp: one ex2 per entry.
+// s_g2 and s_b are 16-byte aligned.  Every kernel pairing score matrices across the backward uses
+// this with the same thread roles, so their score matrices agree bit for bit.
 __device__ __forceinline__ void mask_decay_q(float (&x)[32], float mul, int row, int q, int c0,
                                              float g2, const float* s_g2, const float* s_b) {
 #pragma unroll
     for (int blk = 0; blk < 2; ++blk) {
         const int tb = c0 + 32 * blk, te = tb + 15;
-        if (tb >= 32 * (q + 1)) {   // every token of the block is after every row of the warp
+        float* xb = x + 16 * blk;
+        if (tb >= 32 * (q + 1)) {
 #pragma unroll
-            for (int i = 0; i < 16; ++i) x[16 * blk + i] = 0.f;
-        } else if (te < row) {
+            for (int i = 0; i < 16; ++i) xb[i] = 0.f;
+        } else if (te < 32 * q) {
             const float ar = mul * ex2(g2 - s_g2[te]);
+            const float4* b4 = reinterpret_cast<const float4*>(s_b + tb);
 #pragma unroll
-            for (int i = 0; i < 16; ++i) x[16 * blk + i] = x[16 * blk + i] * ar * s_b[tb + i];
+            for (int k = 0; k < 4; ++k) {
+                const float4 f = b4[k];
+                xb[4 * k + 0] *= ar * f.x;
+                xb[4 * k + 1] *= ar * f.y;
+                xb[4 * k + 2] *= ar * f.z;
+                xb[4 * k + 3] *= ar * f.w;
+            }
         } else {
+            const float4* g4 = reinterpret_cast<const float4*>(s_g2 + tb);
 #pragma unroll
-            for (int i = 0; i < 16; ++i) {
-                const int t = tb + i;
-                x[16 * blk + i] = (t <= row) ? mul * x[16 * blk + i] * ex2(g2 - s_g2[t]) : 0.f;
+            for (int k = 0; k < 4; ++k) {
+                const float4 f = g4[k];
+                const float gt[4] = {f.x, f.y, f.z, f.w};
+#pragma unroll
+                for (int m = 0; m < 4; ++m) {
+                    const int t = tb + 4 * k + m;
+                    const float e = ex2(g2 - gt[m]);
+                    xb[4 * k + m] = (t <= row) ? mul * xb[4 * k + m] * e : 0.f;
+                }
             }
         }
     }

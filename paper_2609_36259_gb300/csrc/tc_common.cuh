@@ -54,6 +54,17 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
         : "memory");
     return ok != 0;
 }
+// Non-blocking test of the phase with the given parity (never suspends the thread).
+__device__ __forceinline__ bool mbar_test_wait(uint64_t* bar, uint32_t parity) {
+    uint32_t ok;
+    asm volatile(
+        "{\n .reg .pred p;\n mbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n"
+        " selp.b32 %0, 1, 0, p;\n}\n"
+        : "=r"(ok)
+        : "r"(smem_u32(bar)), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
 // Bounded wait for the phase with the given parity; false if it never completed.
 __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity) {
     for (uint32_t i = 0; i < SPIN_LIMIT; ++i)
@@ -96,6 +107,13 @@ __device__ __forceinline__ void tma_store_2d(const CUtensorMap* map, const void*
         "cp.async.bulk.tensor.2d.global.shared::cta.bulk_group [%0, {%1, %2}], [%3];" ::"l"(
             reinterpret_cast<uint64_t>(map)),
         "r"(c0), "r"(c1), "r"(smem_u32(src))
+        : "memory");
+}
+__device__ __forceinline__ void tma_store_3d(const CUtensorMap* map, const void* src, int c0, int c1, int c2) {
+    asm volatile(
+        "cp.async.bulk.tensor.3d.global.shared::cta.bulk_group [%0, {%1, %2, %3}], [%4];" ::"l"(
+            reinterpret_cast<uint64_t>(map)),
+        "r"(c0), "r"(c1), "r"(c2), "r"(smem_u32(src))
         : "memory");
 }
 __device__ __forceinline__ void bulk_commit() {
@@ -259,6 +277,37 @@ __device__ __forceinline__ void tmem_st16x2(uint32_t taddr, const float (&v)[32]
     }
     asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
 }
+
+// Asynchronous halves of tmem_ld16x2 / tmem_st16x2: the loads or stores are issued and completed
+// later by tmem_wait_ld / tmem_wait_st, so several can be in flight at once.
+__device__ __forceinline__ void tmem_ld16x2_async(uint32_t taddr, uint32_t (&r)[32]) {
+#pragma unroll
+    for (int blk = 0; blk < 2; ++blk) {
+        uint32_t* o = r + 16 * blk;
+        asm volatile(
+            "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, "
+            "%11, %12, %13, %14, %15}, [%16];"
+            : "=r"(o[0]), "=r"(o[1]), "=r"(o[2]), "=r"(o[3]), "=r"(o[4]), "=r"(o[5]), "=r"(o[6]),
+              "=r"(o[7]), "=r"(o[8]), "=r"(o[9]), "=r"(o[10]), "=r"(o[11]), "=r"(o[12]),
+              "=r"(o[13]), "=r"(o[14]), "=r"(o[15])
+            : "r"(taddr + 32 * blk));
+    }
+}
+__device__ __forceinline__ void tmem_wait_ld() { asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory"); }
+__device__ __forceinline__ void tmem_st16x2_async(uint32_t taddr, const uint32_t (&w)[32]) {
+#pragma unroll
+    for (int blk = 0; blk < 2; ++blk) {
+        const uint32_t* v = w + 16 * blk;
+        asm volatile(
+            "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8, %9, "
+            "%10, %11, %12, %13, %14, %15, %16};" ::"r"(taddr + 32 * blk),
+            "r"(v[0]), "r"(v[1]), "r"(v[2]), "r"(v[3]), "r"(v[4]), "r"(v[5]), "r"(v[6]), "r"(v[7]),
+            "r"(v[8]), "r"(v[9]), "r"(v[10]), "r"(v[11]), "r"(v[12]), "r"(v[13]), "r"(v[14]),
+            "r"(v[15])
+            : "memory");
+    }
+}
+__device__ __forceinline__ void tmem_wait_st() { asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory"); }
 
 // Two blocks of 8 consecutive fp32 columns (at taddr and taddr + 32), one wait.
 __device__ __forceinline__ void tmem_ld8x2(uint32_t taddr, float (&v)[16]) {

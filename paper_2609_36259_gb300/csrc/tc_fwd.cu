@@ -183,103 +183,96 @@ __global__ void __launch_bounds__(256) seg_scan_kernel(TcFwdArgs a) {
 }
 
 // ---------------------------------------------------------------------------------------
-// Chunk walk of one (b, h, segment).  512 threads: thread (row, quarter) owns TMEM lane `row`
-// and the column quarter of QRole in each 128-column accumulator; thread 0 issues TMA and MMA.
+// Chunk walk of one (b, h, segment), warp-specialised.  640 threads in two groups:
+//  * chain (warps 0-15, 512 threads): thread (row, quarter) owns TMEM lane `row` and the column
+//    quarter of QRole in the two product accumulators X1, X2; it runs the epilogues of the
+//    output chain Q K^T, Q Kbar^T -> P1 -> P1 A -> z -> z M^T -> softmax -> p M -> o'' ->
+//    O'' A^T, O'' Vbar -> P2 -> P2 V -> o.  Thread 0 issues the chain's MMAs.
+//  * state (warps 16-19, 128 threads): thread r owns row r of every tile and TMEM lane r of the
+//    state accumulators [Kbar | Vbar]; it builds the write vectors a (T_A) and A-> (T_Q), takes
+//    the fp16 state snapshots (T_N), scales the state by gamma^C, converts the bf16 inputs to
+//    fp16 and issues the TMA loads, the state-update MMAs and the snapshot stores.  Thread 512
+//    leads.
+// The state work of chunk c (snapshot of Vbar, A->, scaling, V) runs under the chain's products
+// and epilogues; the state update [Kbar | Vbar] += A->^T [K | V] is issued by the state leader as
+// soon as its operands are ready, so the chain's commits never wait for it.  The groups meet on
+// mbarriers only:
+//   F1 / F5 / F6  chain products 1, 5, 6 of the chunk complete (tiles they read are free)
+//   SR            state ready: Vbar snapshot in T_N, A-> in T_Q, state scaled, V converted
+//   SU            state update (issued by the state leader) complete
+//   NX            next chunk's a and Kbar snapshot in place (the chain converts its Q, K)
+enum { OB_QK, OB_V, OB_M, OB_MMA, OB_F1, OB_F5, OB_F6, OB_SU, OB_SR, OB_NX, OB_END, OB_ENDS, OB_N };
+constexpr int OUT_CHAIN = 512, OUT_THREADS = 640;
+
+// Bounded wait that also gives up once the other group has flagged an abort.
+__device__ __forceinline__ bool mbar_wait_ab(uint64_t* bar, uint32_t parity, volatile int* abort_) {
+    for (uint32_t i = 0; i < SPIN_LIMIT; ++i) {
+        if (mbar_try_wait(bar, parity)) return true;
+        if ((i & 255u) == 255u && *abort_) return false;
+    }
+    return false;
+}
+__device__ __forceinline__ void named_sync(uint32_t id, uint32_t n) {
+    asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(n) : "memory");
+}
+// Barrier `id` over n threads that also ANDs a predicate across them.
+__device__ __forceinline__ bool named_and(uint32_t id, uint32_t n, bool v) {
+    uint32_t r;
+    asm volatile(
+        "{\n .reg .pred p, q;\n setp.ne.u32 p, %1, 0;\n bar.red.and.pred q, %2, %3, p;\n"
+        " selp.u32 %0, 1, 0, q;\n}\n"
+        : "=r"(r)
+        : "r"((uint32_t)v), "r"(id), "r"(n)
+        : "memory");
+    return r != 0;
+}
+
 template <int SEGC>
-__global__ void __launch_bounds__(512, 1) seg_out_tc(const __grid_constant__ CUtensorMap tq,
-                                                      const __grid_constant__ CUtensorMap tk,
-                                                      const __grid_constant__ CUtensorMap tv,
-                                                      const __grid_constant__ CUtensorMap tm,
-                                                      const __grid_constant__ CUtensorMap tsnap,
-                                                      TcFwdArgs a) {
+__global__ void __launch_bounds__(OUT_THREADS, 1) seg_out_tc(const __grid_constant__ CUtensorMap tq,
+                                                              const __grid_constant__ CUtensorMap tk,
+                                                              const __grid_constant__ CUtensorMap tv,
+                                                              const __grid_constant__ CUtensorMap tm,
+                                                              const __grid_constant__ CUtensorMap tsnap,
+                                                              const __grid_constant__ CUtensorMap to,
+                                                              TcFwdArgs a) {
     const Shape s = a.s;
     const int bh = blockIdx.x, seg = blockIdx.y, b = bh / s.H, h = bh % s.H;
     const int nct = s.T / CT;
     const int c_begin = seg * SEGC;
     const int nc = min(SEGC, nct - c_begin);
     const int tid = threadIdx.x;
-    const QRole ro;
-    const int row = ro.row, hf = ro.hf, u = ro.u, c0 = ro.c0, cq = ro.cq;
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                                ~uintptr_t(1023));
-    uint64_t* bars = reinterpret_cast<uint64_t*>(smem);          // tma q k, mma, m, tma v
-    uint32_t* s_taddr = reinterpret_cast<uint32_t*>(smem + 32);
-    float* s_g2 = reinterpret_cast<float*>(smem + 64);            // [128] log2-domain decays
+    uint64_t* bars = reinterpret_cast<uint64_t*>(smem);          // OB_N mbarriers
+    static_assert(OB_N * 8 <= 112, "mbarriers overlap the TMEM address word");
+    uint32_t* s_taddr = reinterpret_cast<uint32_t*>(smem + 112);
+    volatile int* s_abort = reinterpret_cast<volatile int*>(smem + 116);
+    float* s_g2 = reinterpret_cast<float*>(smem + 128);           // [128] log2-domain decays
     float* s_b = s_g2 + 128;                                      // [128] in-block decay factors
-    uint8_t* T_Q = smem + 2048;        // Q, later A-> (state-update operand)
+    uint8_t* T_Q = smem + 2048;        // Q, then A-> (state-update operand)
     uint8_t* T_K = T_Q + 1 * TILE;
     uint8_t* T_V = T_Q + 2 * TILE;
     uint8_t* T_A = T_Q + 3 * TILE;     // write vectors a_s (rows = tokens)
-    uint8_t* T_S = T_Q + 4 * TILE;     // staging: P1, z, p, O'', P2 (rows = tokens)
+    uint8_t* T_S = T_Q + 4 * TILE;     // chain staging: P1, z, p, O'', P2 (rows = tokens)
     uint8_t* T_N = T_Q + 5 * TILE;     // state snapshot: Kbar, then Vbar (rows = slots)
     uint8_t* T_M = T_Q + 6 * TILE;     // M = R Phi (rows = slots r, cols = Fourier index)
 
     if (tid == 0) {
-        for (int i = 0; i < 4; ++i) mbar_init(&bars[i], 1);
+        for (int i = 0; i < OB_N; ++i) mbar_init(&bars[i], 1);
+        *s_abort = 0;
         fence_mbar_init();
     }
-    if (ro.warp == 0) tmem_alloc(s_taddr, 512);
+    if (tid < 32) tmem_alloc(s_taddr, 512);
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
     const uint32_t taddr = *s_taddr;
-    const uint32_t tl = taddr + ((uint32_t)(32 * ro.q) << 16) + c0;   // lane, column quarter
     const uint32_t SK = 0, SV = 128, X1 = 256, X2 = 384;
-
-    // Q and K of a chunk are loaded as soon as the previous chunk's state update has read T_Q
-    // and T_K; V as soon as its P2 V product has read T_V.  (Thread 0 tracks what is in flight.)
-    bool qk_pending = false, v_pending = false;
-    auto issue_qk = [&](int c) {
-        const int r0 = b * s.T + (c_begin + c) * CT;
-        mbar_expect_tx(&bars[0], 2 * TILE);
-        tma_load_3d(T_Q, &tq, 0, h, r0, &bars[0]);
-        tma_load_3d(T_Q + TILE / 2, &tq, 64, h, r0, &bars[0]);
-        tma_load_3d(T_K, &tk, 0, h, r0, &bars[0]);
-        tma_load_3d(T_K + TILE / 2, &tk, 64, h, r0, &bars[0]);
-        qk_pending = true;
-    };
-    auto issue_v = [&](int c) {
-        const int r0 = b * s.T + (c_begin + c) * CT;
-        mbar_expect_tx(&bars[3], TILE);
-        tma_load_3d(T_V, &tv, 0, h, r0, &bars[3]);
-        tma_load_3d(T_V + TILE / 2, &tv, 64, h, r0, &bars[3]);
-        v_pending = true;
-    };
-    if (tid == 0) {
-        mbar_expect_tx(&bars[2], TILE);
-        tma_load_2d(T_M, &tm, 0, h * 128, &bars[2]);
-        tma_load_2d(T_M + TILE / 2, &tm, 64, h * 128, &bars[2]);
-        issue_qk(0);
-        issue_v(0);
-    }
-    // segment-start state into TMEM; Kbar snapshot into T_N (row = slot)
-    {
-        const float* src = a.segS + (((size_t)bh * a.nseg + seg) * 128 + row) * 256 + c0;
-#pragma unroll
-        for (int part = 0; part < 2; ++part) {
-            float x[32];
-#pragma unroll
-            for (int i = 0; i < 32; i += 4) {
-                const float4 f = *reinterpret_cast<const float4*>(src + 128 * part + (i & 15) + 32 * (i >> 4));
-                x[i] = f.x; x[i + 1] = f.y; x[i + 2] = f.z; x[i + 3] = f.w;
-            }
-            tmem_st16x2(tl + 128 * part, x);
-            if (part == 0) store_q<__half>(T_N, row, c0, x);
-        }
-    }
-    fence_async_smem();
-    tc_fence_before();
-    __syncthreads();
-    tc_fence_after();
-    bool ok = mbar_wait(&bars[2], 0);
-    ok = __syncthreads_and(ok);
-    uint32_t qk_ph = 0, v_ph = 0, mma_ph = 0;
-    const float scale = s.scale;
-    const uint32_t id_kk = idesc_f16(128, 128, 0, 0);
-    const uint32_t id_kn = idesc_f16(128, 128, 0, 1);
-    const uint32_t id_nn = idesc_f16(128, 128, 1, 1);
     const bool save = a.snap != nullptr;
+    const uint32_t uQ = smem_u32(T_Q), uK = smem_u32(T_K), uV = smem_u32(T_V),
+                   uA = smem_u32(T_A), uS = smem_u32(T_S), uN = smem_u32(T_N),
+                   uM = smem_u32(T_M);
     // the snapshot in T_N (part 0: Kbar, 1: Vbar) of chunk cg leaves by a TMA store
     auto store_snap = [&](int cg, int part) {
         const int r = ((bh * nct + cg) * 2 + part) * 128;
@@ -287,252 +280,451 @@ __global__ void __launch_bounds__(512, 1) seg_out_tc(const __grid_constant__ CUt
         tma_store_2d(&tsnap, T_N + TILE / 2, 64, r);
         bulk_commit();
     };
-    const uint32_t uQ = smem_u32(T_Q), uK = smem_u32(T_K), uV = smem_u32(T_V),
-                   uA = smem_u32(T_A), uS = smem_u32(T_S), uN = smem_u32(T_N),
-                   uM = smem_u32(T_M);
+    bool ok = true;
 
-    auto wait_mma = [&]() {
-        if (ok) ok = mbar_wait(&bars[1], mma_ph);
-        mma_ph ^= 1;
-        tc_fence_after();
-    };
-    // publish shared-memory operand writes / TMEM stores to the MMA issuer; the block agrees
-    // on `ok`, so every later branch on it is uniform
-    auto publish = [&]() {
+    if (tid >= OUT_CHAIN) {
+        // ================================================================ state group
+        const int r = tid - OUT_CHAIN;                 // row of every tile / TMEM lane
+        const uint32_t tlane = taddr + ((uint32_t)(32 * ((tid >> 5) & 3)) << 16);
+        const bool leader = tid == OUT_CHAIN;
+        const uint32_t id_nn = idesc_f16(128, 128, 1, 1);
+        bool su_issued = false;   // leader: a state update that nobody has waited for
+        bool qk_pending = false, v_pending = false;
+        uint32_t qk_par = 0, v_par = 0;   // parity of the pending loads' phases
+        auto issue_qk = [&](int c) {
+            const int r0 = b * s.T + (c_begin + c) * CT;
+            mbar_expect_tx(&bars[OB_QK], 2 * TILE);
+            tma_load_3d(T_Q, &tq, 0, h, r0, &bars[OB_QK]);
+            tma_load_3d(T_Q + TILE / 2, &tq, 64, h, r0, &bars[OB_QK]);
+            tma_load_3d(T_K, &tk, 0, h, r0, &bars[OB_QK]);
+            tma_load_3d(T_K + TILE / 2, &tk, 64, h, r0, &bars[OB_QK]);
+            qk_pending = true;
+            qk_par = c & 1;
+        };
+        auto issue_v = [&](int c) {
+            const int r0 = b * s.T + (c_begin + c) * CT;
+            mbar_expect_tx(&bars[OB_V], TILE);
+            tma_load_3d(T_V, &tv, 0, h, r0, &bars[OB_V]);
+            tma_load_3d(T_V + TILE / 2, &tv, 64, h, r0, &bars[OB_V]);
+            v_pending = true;
+            v_par = c & 1;
+        };
+        // gates of this row's token in chunk c: clock, write strength, log2 decay from the chunk
+        // start, and the log2 decay of the whole chunk
+        auto gates = [&](int c, float& lam_, float& beta_, float& g2_, float& g2C_) {
+            const int t0 = (c_begin + c) * CT;
+            const size_t gi = ((size_t)b * s.T + t0 + r) * s.H + h;
+            lam_ = a.lam[gi];
+            beta_ = a.beta[gi];
+            g2_ = cum128(s, a.g, b, h, t0, t0 + r) * LOG2E;
+            g2C_ = cum128(s, a.g, b, h, t0, t0 + CT - 1) * LOG2E;
+        };
+        if (leader) {
+            mbar_expect_tx(&bars[OB_M], TILE);
+            tma_load_2d(T_M, &tm, 0, h * 128, &bars[OB_M]);
+            tma_load_2d(T_M + TILE / 2, &tm, 64, h * 128, &bars[OB_M]);
+            issue_qk(0);
+            issue_v(0);
+        }
+        float lam, beta, g2, g2C;
+        gates(0, lam, beta, g2, g2C);
+#pragma unroll 1
+        for (int qq = 0; qq < 4; ++qq) write_vector_q<__half>(T_A, r, qq >> 1, qq & 1, lam, beta);
+        if (ok) ok = mbar_wait(&bars[OB_QK], 0);
+        if (leader && ok) qk_pending = false;
+        if (ok) {
+            bf16_to_f16_half(T_Q, r, 0);
+            bf16_to_f16_half(T_Q, r, 1);
+            bf16_to_f16_half(T_K, r, 0);
+            bf16_to_f16_half(T_K, r, 1);
+        }
+        // the chain group has put the segment-start state into TMEM and the Kbar snapshot
+        // into T_N before this barrier
         fence_async_smem();
         tc_fence_before();
         ok = __syncthreads_and(ok);
         tc_fence_after();
-    };
-    auto issuer = [&]() { return tid == 0 && ok; };
-    auto mask_scores = [&](float (&x)[32], float g2_, float mul) {
-        mask_decay_q(x, mul, row, ro.q, c0, g2_, s_g2, s_b);
-    };
-
-    // Set-up of a chunk that needs no product of the previous one: its decays, its write vectors
-    // (T_A) and its Q, K tiles (waited for and converted to fp16).  For chunk c + 1 it runs while
-    // chunk c's last product (P2 V) is in flight.
-    auto chunk_setup = [&](float lam_, float beta_, float g2_, float g2e_) {
-        if (cq == 0) {
-            s_g2[row] = g2_;
-            s_b[row] = ex2(g2e_ - g2_);   // from this row's token to the end of its 16-block
+        if (ok && leader) {
+            if (save) store_snap(c_begin, 0);
+            mbar_arrive(&bars[OB_NX]);
         }
-        write_vector_q<__half>(T_A, row, hf, u, lam_, beta_);
-        if (ok) ok = mbar_wait(&bars[0], qk_ph);
-        if (tid == 0 && ok) qk_pending = false;
-        qk_ph ^= 1;
-        if (ok) {
-            bf16_to_f16_q(T_Q, row, c0);
-            bf16_to_f16_q(T_K, row, c0);
-        }
-    };
-    // gates of the current and of the next chunk (prefetched one chunk ahead: the loads are
-    // issued a chunk before their values are combined, so their latency is never waited for)
-    float lam, beta, g2;
-    float n_lam = 0.f, n_beta = 0.f, n_ga = 0.f, n_gb = 0.f, n_ge = 0.f;
-    auto load_gates = [&](int c, float& l_, float& b_, float& ga, float& gb, float& ge) {
-        const int t0 = (c_begin + c) * CT, t = t0 + row;
-        const size_t gi = ((size_t)b * s.T + t) * s.H + h;
-        l_ = a.lam[gi];
-        b_ = a.beta[gi];
-        // cum128 in two loads: g_cum is local to s.Cg-token chunks (row and row | 15 share the
-        // second term)
-        ga = a.g[gi];
-        gb = (s.Cg == 64 && t - t0 >= 64) ? a.g[((size_t)b * s.T + t0 + 63) * s.H + h] : 0.f;
-        ge = a.g[((size_t)b * s.T + t0 + (row | 15)) * s.H + h];
-    };
-    {
-        float ga, gb, ge;
-        load_gates(0, lam, beta, ga, gb, ge);
-        g2 = (ga + gb) * LOG2E;
-        chunk_setup(lam, beta, g2, (ge + gb) * LOG2E);
-    }
-    publish();
-    for (int c = 0; c < nc && ok; ++c) {
-        const int t0 = (c_begin + c) * CT;
-        const size_t gi = ((size_t)b * s.T + t0 + row) * s.H + h;
-        if (c + 1 < nc) load_gates(c + 1, n_lam, n_beta, n_ga, n_gb, n_ge);
-        const float g2C = s_g2[CT - 1];
-        const float gam = ex2(g2);
-        if (save && tid == 0) store_snap(c_begin + c, 0);
-
-        // X1 = Q K^T, X2 = Q Kbar^T
-        if (issuer()) {
+        for (int c = 0; c < nc && ok; ++c) {
+            const bool last = c + 1 == nc;
+            float n_lam = 0.f, n_beta = 0.f, n_g2 = 0.f, n_g2C = 0.f;
+            if (!last) gates(c + 1, n_lam, n_beta, n_g2, n_g2C);
+            // S1: product 1 has read Q and the Kbar snapshot
+            if (ok) ok = mbar_wait_ab(&bars[OB_F1], c & 1, s_abort);
+            if (save && leader) bulk_wait_read_all();   // the Kbar snapshot store has read T_N
+            tc_fence_after();
+            ok = named_and(2, 128, ok);
+            if (!ok) break;
+            // S2: Vbar snapshot (before scaling), state scaled by gamma^C, A-> rows
             {
+                const float gC = ex2(g2C);
+#pragma unroll 1
+                for (int qq = 0; qq < 4; ++qq) {   // column quarters c0 = 64 (qq / 2) + 16 (qq % 2)
+                    const int cc = 64 * (qq >> 1) + 16 * (qq & 1);
+                    uint32_t xv[32], xk[32];
+                    tmem_ld16x2_async(tlane + SV + cc, xv);
+                    if (!last) tmem_ld16x2_async(tlane + SK + cc, xk);
+                    tmem_wait_ld();
+                    float x[32];
+#pragma unroll
+                    for (int i = 0; i < 32; ++i) x[i] = __uint_as_float(xv[i]);
+                    store_q<__half>(T_N, r, cc, x);
+                    if (!last) {   // loads and stores of the quarters overlap; one wait at the end
+#pragma unroll
+                        for (int i = 0; i < 32; ++i) {
+                            xv[i] = __float_as_uint(x[i] * gC);
+                            xk[i] = __float_as_uint(__uint_as_float(xk[i]) * gC);
+                        }
+                        tmem_st16x2_async(tlane + SV + cc, xv);
+                        tmem_st16x2_async(tlane + SK + cc, xk);
+                    }
+                }
+                if (!last) {
+                    tmem_wait_st();
+                    // A-> rows: the fp16 write vector a of the row (T_A) times beta gamma^C / gamma_r
+                    const __half2 w2 = __float2half2_rn(ex2(g2C - g2));
+#pragma unroll 4
+                    for (int j = 0; j < 16; ++j) {
+                        const uint32_t off = swz_off(r, 8 * j, 128);
+                        uint4 v = *reinterpret_cast<const uint4*>(T_A + off);
+                        __half2* e = reinterpret_cast<__half2*>(&v);
+#pragma unroll
+                        for (int i = 0; i < 4; ++i) e[i] = __hmul2(e[i], w2);
+                        *reinterpret_cast<uint4*>(T_Q + off) = v;
+                    }
+                }
+            }
+            // S3: V of this chunk
+            if (ok) ok = mbar_wait_ab(&bars[OB_V], c & 1, s_abort);
+            if (leader && ok) v_pending = false;
+            if (ok) {
+                bf16_to_f16_half(T_V, r, 0);
+                bf16_to_f16_half(T_V, r, 1);
+            }
+            // S4: publish to the MMA issuer
+            fence_async_smem();
+            tc_fence_before();
+            ok = named_and(2, 128, ok);
+            if (!ok) break;
+            if (leader) {
+                if (save) store_snap(c_begin + c, 1);
+                mbar_arrive(&bars[OB_SR]);
+                if (!last) {   // state update [Kbar | Vbar] += A->^T [K | V], issued from here so
+                               // that the chain's own commits never wait for it
+                    tc_fence_after();
+#pragma unroll
+                    for (int k = 0; k < 8; ++k) {
+                        mma_bf16(taddr + SK, mnmajor_desc(uQ, 128, k), mnmajor_desc(uK, 128, k), id_nn, 1u);
+                        mma_bf16(taddr + SV, mnmajor_desc(uQ, 128, k), mnmajor_desc(uV, 128, k), id_nn, 1u);
+                    }
+                    mma_commit(&bars[OB_SU]);
+                    su_issued = true;
+                }
+            }
+            if (last) break;
+            // S5: the state update has read A->, K and V: next Q, K may come in
+            if (ok) ok = mbar_wait_ab(&bars[OB_SU], c & 1, s_abort);
+            if (ok && leader) {
+                su_issued = false;
+                issue_qk(c + 1);   // stays pending for the failure path: the chain waits for it
+            }
+            // S6: product 5 has read a and the Vbar snapshot: next a and the Kbar snapshot
+            if (ok) ok = mbar_wait_ab(&bars[OB_F5], c & 1, s_abort);
+            if (save && leader) bulk_wait_read_all();   // the Vbar snapshot store has read T_N
+            tc_fence_after();
+            ok = named_and(2, 128, ok);
+            if (!ok) break;
+            lam = n_lam;
+            beta = n_beta;
+            g2 = n_g2;
+            g2C = n_g2C;
+#pragma unroll 1
+            for (int qq = 0; qq < 4; ++qq) {
+                const int cc = 64 * (qq >> 1) + 16 * (qq & 1);
+                float x[32];
+                tmem_ld16x2(tlane + SK + cc, x);
+                store_q<__half>(T_N, r, cc, x);
+            }
+#pragma unroll 1
+            for (int qq = 0; qq < 4; ++qq) write_vector_q<__half>(T_A, r, qq >> 1, qq & 1, lam, beta);
+            // S8: the next chunk's a and Kbar snapshot are ready (its Q and K are converted to
+            // fp16 by the chain group, which is idle at that point)
+            fence_async_smem();
+            tc_fence_before();
+            ok = named_and(2, 128, ok);
+            if (!ok) break;
+            if (leader) {
+                if (save) store_snap(c_begin + c + 1, 0);
+                mbar_arrive(&bars[OB_NX]);
+            }
+            // S9: product 6 has read V: next V may come in
+            if (ok) ok = mbar_wait_ab(&bars[OB_F6], c & 1, s_abort);
+            if (ok && leader) issue_v(c + 1);
+        }
+        if (!ok) *s_abort = 1;
+        if (leader) {
+            if (!ok) {
+                flag_error(CYFA_ERR_TIMEOUT);
+                if (su_issued) {   // the state update may still be running: let it finish
+                    mma_commit(&bars[OB_ENDS]);
+                    mbar_wait(&bars[OB_ENDS], 0);
+                }
+                // copies still in flight land before the shared memory is released
+                if (qk_pending) mbar_wait(&bars[OB_QK], qk_par);
+                if (v_pending) mbar_wait(&bars[OB_V], v_par);
+            }
+            if (save) bulk_wait_all();
+        }
+    } else {
+        // ================================================================ chain group
+        const QRole ro;
+        const int row = ro.row, hf = ro.hf, u = ro.u, c0 = ro.c0, cq = ro.cq;
+        const uint32_t tl = taddr + ((uint32_t)(32 * ro.q) << 16) + c0;   // lane, column quarter
+        // segment-start state into TMEM; Kbar snapshot into T_N (row = slot)
+        {
+            const float* src = a.segS + (((size_t)bh * a.nseg + seg) * 128 + row) * 256 + c0;
+#pragma unroll
+            for (int part = 0; part < 2; ++part) {
+                float x[32];
+#pragma unroll
+                for (int i = 0; i < 32; i += 4) {
+                    const float4 f = *reinterpret_cast<const float4*>(src + 128 * part + (i & 15) + 32 * (i >> 4));
+                    x[i] = f.x; x[i + 1] = f.y; x[i + 2] = f.z; x[i + 3] = f.w;
+                }
+                tmem_st16x2(tl + 128 * part, x);
+                if (part == 0) store_q<__half>(T_N, row, c0, x);
+            }
+        }
+        fence_async_smem();
+        tc_fence_before();
+        ok = __syncthreads_and(ok);
+        tc_fence_after();
+        if (tid == 0 && ok) ok = mbar_wait(&bars[OB_M], 0);
+        uint32_t mma_ph = 0;
+        const float scale = s.scale;
+        const uint32_t id_kk = idesc_f16(128, 128, 0, 0);
+        const uint32_t id_kn = idesc_f16(128, 128, 0, 1);
+        bool issued = false;   // thread 0: an MMA commit that nobody waited for may be in flight
+
+        auto wait_mma = [&]() {
+            if (ok) ok = mbar_wait_ab(&bars[OB_MMA], mma_ph, s_abort);
+            mma_ph ^= 1;
+            tc_fence_after();
+        };
+        auto publish = [&]() {
+            fence_async_smem();
+            tc_fence_before();
+            ok = named_and(1, OUT_CHAIN, ok);
+            tc_fence_after();
+        };
+        auto issuer = [&]() { return tid == 0 && ok; };
+        auto mask_scores = [&](float (&x)[32], float g2_, float mul) {
+            mask_decay_q(x, mul, row, ro.q, c0, g2_, s_g2, s_b);
+        };
+        // gates of this row's token: prefetched a chunk ahead
+        float lam, g2, g2e;
+        float n_lam = 0.f, n_ga = 0.f, n_gb = 0.f, n_ge = 0.f;
+        auto load_gates = [&](int c, float& l_, float& ga, float& gb, float& ge) {
+            const int t0 = (c_begin + c) * CT, t = t0 + row;
+            const size_t gi = ((size_t)b * s.T + t) * s.H + h;
+            l_ = a.lam[gi];
+            // cum128 in two loads: g_cum is local to s.Cg-token chunks (row and row | 15 share
+            // the second term)
+            ga = a.g[gi];
+            gb = (s.Cg == 64 && t - t0 >= 64) ? a.g[((size_t)b * s.T + t0 + 63) * s.H + h] : 0.f;
+            ge = a.g[((size_t)b * s.T + t0 + (row | 15)) * s.H + h];
+        };
+        {
+            float ga, gb, ge;
+            load_gates(0, lam, ga, gb, ge);
+            g2 = (ga + gb) * LOG2E;
+            g2e = (ge + gb) * LOG2E;
+        }
+        for (int c = 0; c < nc && ok; ++c) {
+            const bool last = c + 1 == nc;
+            if (!last) load_gates(c + 1, n_lam, n_ga, n_gb, n_ge);
+            if (cq == 0) {
+                s_g2[row] = g2;
+                s_b[row] = ex2(g2e - g2);   // from this row's token to the end of its 16-block
+            }
+            if (ok) ok = mbar_wait_ab(&bars[OB_NX], c & 1, s_abort);
+            fence_async_smem();
+            tc_fence_before();
+            ok = named_and(1, OUT_CHAIN, ok);
+            tc_fence_after();
+            if (!ok) break;
+            const float gam = ex2(g2);
+
+            // product 1: X1 = Q K^T, X2 = Q Kbar^T
+            if (issuer()) {
 #pragma unroll
                 for (int k = 0; k < 8; ++k) {
                     mma_bf16(taddr + X1, kmajor_desc(uQ, 128, k), kmajor_desc(uK, 128, k), id_kk, k > 0);
                     mma_bf16(taddr + X2, kmajor_desc(uQ, 128, k), kmajor_desc(uN, 128, k), id_kk, k > 0);
                 }
-                mma_commit(&bars[1]);
+                // E1 rewrites T_S once this product completes: the previous chunk's output
+                // store must have read it (the commit below is only issued after that)
+                bulk_wait_read_all();
+                mma_commit(&bars[OB_MMA]);
+                mma_commit(&bars[OB_F1]);
+                issued = true;
+            }
+            wait_mma();
+            {   // P1 = s (Q K^T) o Gamma
+                float x[32];
+                tmem_ld16x2(tl + X1, x);
+                mask_scores(x, g2, scale);
+                store_q<__half>(T_S, row, c0, x);
+            }
+            publish();
+            if (!ok) break;
+            // product 2: X1 = P1 A
+            if (issuer()) {
+#pragma unroll
+                for (int k = 0; k < 8; ++k)
+                    mma_bf16(taddr + X1, kmajor_desc(uS, 128, k), mnmajor_desc(uA, 128, k), id_kn, k > 0);
+                mma_commit(&bars[OB_MMA]);
+            }
+            wait_mma();
+            {   // z = U(lam) o',  o' = s gamma_r (Q Kbar^T) + P1 A
+                float x[32], y[32];
+                tmem_ld16x2_pair(tl + X2, x, tl + X1, y);
+                const float f = scale * gam;
+#pragma unroll
+                for (int i = 0; i < 32; ++i) x[i] = fmaf(f, x[i], y[i]);
+                rotate_q<1>(x, hf, u, lam);
+                store_q<__half>(T_S, row, c0, x);
+            }
+            publish();
+            if (!ok) break;
+            // product 3: X1 = z M^T
+            if (issuer()) {
+#pragma unroll
+                for (int k = 0; k < 8; ++k)
+                    mma_bf16(taddr + X1, kmajor_desc(uS, 128, k), kmajor_desc(uM, 128, k), id_kk, k > 0);
+                mma_commit(&bars[OB_MMA]);
+            }
+            wait_mma();
+            {   // p = softmax over the 127 active slots of l = z M^T; the staging tile (z is
+                // consumed) holds the row reductions over the four column quarters
+                float* red = reinterpret_cast<float*>(T_S);
+                float x[32];
+                tmem_ld16x2(tl + X1, x);
+                const bool pad = (hf == 1 && u == 1);       // its element 31 is the padding slot
+                float mx = -INFINITY;
+#pragma unroll
+                for (int i = 0; i < 32; ++i)
+                    if (!(pad && i == 31)) mx = fmaxf(mx, x[i]);
+                red[128 * cq + row] = mx;
+                named_sync(1, OUT_CHAIN);
+                mx = fmaxf(fmaxf(red[row], red[128 + row]), fmaxf(red[256 + row], red[384 + row]));
+                float sum = 0.f;
+#pragma unroll
+                for (int i = 0; i < 32; ++i) {
+                    x[i] = (pad && i == 31) ? 0.f : ex2((x[i] - mx) * LOG2E);
+                    sum += x[i];
+                }
+                red[512 + 128 * cq + row] = sum;
+                named_sync(1, OUT_CHAIN);
+                const float inv = 1.f / ((red[512 + row] + red[640 + row]) + (red[768 + row] + red[896 + row]));
+#pragma unroll
+                for (int i = 0; i < 32; ++i) x[i] *= inv;
+                named_sync(1, OUT_CHAIN);   // every quarter has read its sums before p overwrites them
+                store_q<__half>(T_S, row, c0, x);
+            }
+            publish();
+            if (!ok) break;
+            // product 4: X2 = p M
+            if (issuer()) {
+#pragma unroll
+                for (int k = 0; k < 8; ++k)
+                    mma_bf16(taddr + X2, kmajor_desc(uS, 128, k), mnmajor_desc(uM, 128, k), id_kn, k > 0);
+                mma_commit(&bars[OB_MMA]);
+            }
+            wait_mma();
+            {   // o'' = U(-lam) (p M)
+                float x[32];
+                tmem_ld16x2(tl + X2, x);
+                rotate_q<-1>(x, hf, u, lam);
+                store_q<__half>(T_S, row, c0, x);
+            }
+            publish();
+            if (!ok) break;
+            // product 5: X1 = O'' A^T, X2 = O'' Vbar (needs the Vbar snapshot: state ready)
+            if (issuer()) {
+                ok = mbar_wait_ab(&bars[OB_SR], c & 1, s_abort);
+                if (ok) {
+                    tc_fence_after();
+#pragma unroll
+                    for (int k = 0; k < 8; ++k) {
+                        mma_bf16(taddr + X1, kmajor_desc(uS, 128, k), kmajor_desc(uA, 128, k), id_kk, k > 0);
+                        mma_bf16(taddr + X2, kmajor_desc(uS, 128, k), mnmajor_desc(uN, 128, k), id_kn, k > 0);
+                    }
+                    mma_commit(&bars[OB_MMA]);
+                    mma_commit(&bars[OB_F5]);
+                }
+            }
+            wait_mma();
+            {   // P2 = (O'' A^T) o Gamma
+                float x[32];
+                tmem_ld16x2(tl + X1, x);
+                mask_scores(x, g2, 1.f);
+                store_q<__half>(T_S, row, c0, x);
+            }
+            publish();
+            if (!ok) break;
+            // product 6: X1 = P2 V
+            if (issuer()) {
+#pragma unroll
+                for (int k = 0; k < 8; ++k)
+                    mma_bf16(taddr + X1, kmajor_desc(uS, 128, k), mnmajor_desc(uV, 128, k), id_kn, k > 0);
+                mma_commit(&bars[OB_MMA]);
+                mma_commit(&bars[OB_F6]);
+            }
+            wait_mma();
+            {   // o = gamma_r (O'' Vbar) + P2 V, staged in T_S (P2 is consumed) for a TMA store
+                float x[32], y[32];
+                tmem_ld16x2_pair(tl + X2, x, tl + X1, y);
+#pragma unroll
+                for (int i = 0; i < 32; ++i) x[i] = fmaf(gam, x[i], y[i]);
+                store_q<__nv_bfloat16>(T_S, row, c0, x);
+            }
+            publish();
+            if (tid == 0) {
+                issued = false;   // every product of the chunk has been waited for
+                if (ok) {
+                    const int r0 = b * s.T + (c_begin + c) * CT;
+                    tma_store_3d(&to, T_S, 0, h, r0);
+                    tma_store_3d(&to, T_S + TILE / 2, 64, h, r0);
+                    bulk_commit();
+                }
+            }
+            if (!last) {
+                lam = n_lam;
+                g2 = (n_ga + n_gb) * LOG2E;
+                g2e = (n_ge + n_gb) * LOG2E;
+                // the next chunk's Q and K (loaded once the state update had read T_Q, T_K)
+                // become fp16 operands
+                if (ok) ok = mbar_wait_ab(&bars[OB_QK], (c + 1) & 1, s_abort);
+                if (ok) {
+                    bf16_to_f16_q(T_Q, row, c0);
+                    bf16_to_f16_q(T_K, row, c0);
+                }
             }
         }
-        wait_mma();
-        {   // P1 = s (Q K^T) o Gamma
-            float x[32];
-            tmem_ld16x2(tl + X1, x);
-            mask_scores(x, g2, scale);
-            store_q<__half>(T_S, row, c0, x);
+        if (!ok) *s_abort = 1;
+        if (tid == 0 && issued) {   // a product may still be running: let it finish
+            mma_commit(&bars[OB_END]);
+            mbar_wait(&bars[OB_END], 0);
         }
-        if (save && tid == 0) bulk_wait_read_all();   // T_N is rewritten after this barrier
-        publish();
-        if (!ok) break;
-        if (issuer()) {
-#pragma unroll
-            for (int k = 0; k < 8; ++k)
-                mma_bf16(taddr + X1, kmajor_desc(uS, 128, k), mnmajor_desc(uA, 128, k), id_kn, k > 0);
-            mma_commit(&bars[1]);
-        }
-        // A-> rows into T_Q (Q is consumed), Vbar snapshot into T_N, state scaled by gamma^C
-        write_vector_q<__half>(T_Q, row, hf, u, lam, beta * ex2(g2C - g2));
-        {
-            const float gC = ex2(g2C);
-            float x[32];
-            tmem_ld16x2(tl + SK, x);
-#pragma unroll
-            for (int i = 0; i < 32; ++i) x[i] *= gC;
-            tmem_st16x2(tl + SK, x);
-            tmem_ld16x2(tl + SV, x);
-            store_q<__half>(T_N, row, c0, x);
-#pragma unroll
-            for (int i = 0; i < 32; ++i) x[i] *= gC;
-            tmem_st16x2(tl + SV, x);
-        }
-        if (ok) ok = mbar_wait(&bars[3], v_ph);   // V: the state update reads it next
-        if (tid == 0 && ok) v_pending = false;
-        v_ph ^= 1;
-        if (ok) bf16_to_f16_q(T_V, row, c0);
-        publish();
-        if (!ok) break;
-        if (save && tid == 0) store_snap(c_begin + c, 1);
-        if (issuer()) {   // state update: [Kbar | Vbar] += A->^T [K | V]
-#pragma unroll
-            for (int k = 0; k < 8; ++k) {
-                mma_bf16(taddr + SK, mnmajor_desc(uQ, 128, k), mnmajor_desc(uK, 128, k), id_nn, 1u);
-                mma_bf16(taddr + SV, mnmajor_desc(uQ, 128, k), mnmajor_desc(uV, 128, k), id_nn, 1u);
-            }
-        }
-        wait_mma();   // P1 A
-        {   // z = U(lam) o',  o' = s gamma_r (Q Kbar^T) + P1 A
-            float x[32], y[32];
-            tmem_ld16x2_pair(tl + X2, x, tl + X1, y);
-            const float f = scale * gam;
-#pragma unroll
-            for (int i = 0; i < 32; ++i) x[i] = fmaf(f, x[i], y[i]);
-            rotate_q<1>(x, hf, u, lam);
-            store_q<__half>(T_S, row, c0, x);
-        }
-        publish();
-        if (!ok) break;
-        if (issuer()) {
-#pragma unroll
-            for (int k = 0; k < 8; ++k)
-                mma_bf16(taddr + X1, kmajor_desc(uS, 128, k), kmajor_desc(uM, 128, k), id_kk, k > 0);
-            mma_commit(&bars[1]);
-        }
-        wait_mma();   // also covers the state update issued before this commit
-        if (issuer() && c + 1 < nc) issue_qk(c + 1);   // T_Q (A->) and T_K are consumed
-        {   // p = softmax over the 127 active slots of l = z M^T; the staging tile (z is
-            // consumed) holds the row reductions over the four column quarters
-            float* red = reinterpret_cast<float*>(T_S);
-            float x[32];
-            tmem_ld16x2(tl + X1, x);
-            const bool pad = (hf == 1 && u == 1);       // its element 31 is the padding slot
-            float mx = -INFINITY;
-#pragma unroll
-            for (int i = 0; i < 32; ++i)
-                if (!(pad && i == 31)) mx = fmaxf(mx, x[i]);
-            red[128 * cq + row] = mx;
-            __syncthreads();
-            mx = fmaxf(fmaxf(red[row], red[128 + row]), fmaxf(red[256 + row], red[384 + row]));
-            float sum = 0.f;
-#pragma unroll
-            for (int i = 0; i < 32; ++i) {
-                x[i] = (pad && i == 31) ? 0.f : ex2((x[i] - mx) * LOG2E);
-                sum += x[i];
-            }
-            red[512 + 128 * cq + row] = sum;
-            __syncthreads();
-            const float inv = 1.f / ((red[512 + row] + red[640 + row]) + (red[768 + row] + red[896 + row]));
-#pragma unroll
-            for (int i = 0; i < 32; ++i) x[i] *= inv;
-            __syncthreads();   // every quarter has read its sums before p overwrites them
-            store_q<__half>(T_S, row, c0, x);
-        }
-        publish();
-        if (!ok) break;
-        if (issuer()) {
-#pragma unroll
-            for (int k = 0; k < 8; ++k)
-                mma_bf16(taddr + X2, kmajor_desc(uS, 128, k), mnmajor_desc(uM, 128, k), id_kn, k > 0);
-            mma_commit(&bars[1]);
-        }
-        wait_mma();
-        {   // o'' = U(-lam) (p M)
-            float x[32];
-            tmem_ld16x2(tl + X2, x);
-            rotate_q<-1>(x, hf, u, lam);
-            store_q<__half>(T_S, row, c0, x);
-        }
-        publish();
-        if (!ok) break;
-        if (issuer()) {
-#pragma unroll
-            for (int k = 0; k < 8; ++k) {
-                mma_bf16(taddr + X1, kmajor_desc(uS, 128, k), kmajor_desc(uA, 128, k), id_kk, k > 0);
-                mma_bf16(taddr + X2, kmajor_desc(uS, 128, k), mnmajor_desc(uN, 128, k), id_kn, k > 0);
-            }
-            mma_commit(&bars[1]);
-        }
-        wait_mma();
-        {   // P2 = (O'' A^T) o Gamma
-            float x[32];
-            tmem_ld16x2(tl + X1, x);
-            mask_scores(x, g2, 1.f);
-            store_q<__half>(T_S, row, c0, x);
-        }
-        if (save && tid == 0) bulk_wait_read_all();   // T_N is rewritten after this barrier
-        publish();
-        if (!ok) break;
-        if (issuer()) {
-#pragma unroll
-            for (int k = 0; k < 8; ++k)
-                mma_bf16(taddr + X1, kmajor_desc(uS, 128, k), mnmajor_desc(uV, 128, k), id_kn, k > 0);
-            mma_commit(&bars[1]);
-        }
-        if (c + 1 < nc) {   // while P2 V runs: the next chunk's set-up (T_A, T_Q, T_K are free)
-            lam = n_lam;
-            beta = n_beta;
-            g2 = (n_ga + n_gb) * LOG2E;
-            chunk_setup(lam, beta, g2, (n_ge + n_gb) * LOG2E);
-        }
-        wait_mma();
-        // next chunk's V (T_V is consumed), then o = gamma_r (O'' Vbar) + P2 V
-        if (issuer() && c + 1 < nc) issue_v(c + 1);
-        {
-            float x[32], y[32];
-            tmem_ld16x2_pair(tl + X2, x, tl + X1, y);
-#pragma unroll
-            for (int i = 0; i < 32; ++i) x[i] = fmaf(gam, x[i], y[i]);
-            store_global_q(static_cast<__nv_bfloat16*>(a.o) + gi * 128, c0, x);
-        }
-        {   // Kbar snapshot of the next chunk's start state
-            float x[32];
-            tmem_ld16x2(tl + SK, x);
-            store_q<__half>(T_N, row, c0, x);
-        }
-        publish();
+        if (tid == 0) bulk_wait_all();
     }
-    if (!ok && tid == 0) {
-        flag_error(CYFA_ERR_TIMEOUT);
-        // let copies still in flight land before the shared memory is released
-        if (qk_pending) mbar_wait(&bars[0], qk_ph);
-        if (v_pending) mbar_wait(&bars[3], v_ph);
-    }
-    if (save && tid == 0) bulk_wait_all();
     tc_fence_before();
     __syncthreads();
-    if (ro.warp == 0) tmem_dealloc(taddr, 512);
+    if (tid < 32) tmem_dealloc(taddr, 512);
 }
 
 // M (fp32, paper order) -> fp16 with its Fourier (column) index in the tensor-core order.
@@ -625,8 +817,9 @@ cudaError_t launch_fwd_tc(const TcFwdArgs& a, const void* q, const void* k, cons
                           const float* Mf, cudaStream_t st) {
     const Shape& s = a.s;
     const unsigned long long BH = (unsigned long long)s.B * s.H;
-    CUtensorMap mq, mk, mv, mm, msnap;
+    CUtensorMap mq, mk, mv, mm, msnap, mo;
     if (!tc_qkv_maps(s, q, k, v, &mq, &mk, &mv) ||
+        !tc_qkv_maps(s, a.o, nullptr, nullptr, &mo, nullptr, nullptr) ||
         !tc_rows_map(&mm, a.Mb, (unsigned long long)s.H * 128, true))
         return cudaErrorInvalidValue;
     // without a snapshot buffer the map is a valid placeholder over M that is never used
@@ -639,7 +832,7 @@ cudaError_t launch_fwd_tc(const TcFwdArgs& a, const void* q, const void* k, cons
     const int smC = 2048 + 7 * TILE + 1024;
     auto kC = seg_out_tc<SEGC_DEFAULT>;
     cudaFuncSetAttribute(kC, cudaFuncAttributeMaxDynamicSharedMemorySize, smC);
-    { LaunchScope ls_("tc_seg_out", st); kC<<<grid, 512, smC, st>>>(mq, mk, mv, mm, msnap, a); }
+    { LaunchScope ls_("tc_seg_out", st); kC<<<grid, OUT_THREADS, smC, st>>>(mq, mk, mv, mm, msnap, mo, a); }
     return cudaGetLastError();
 }
 
