@@ -26,7 +26,7 @@ constexpr int CB = BWD_C;          // 64
 constexpr int LPB = CB + 1;
 constexpr int TMB = CB / 16;       // 4 rows per thread
 
-__device__ __forceinline__ float freq(int j) { return 6.283185307179586f * (float)j / 127.f; }
+__device__ __forceinline__ float freq(int j) { return (6.283185307179586f / 127.f) * (float)j; }
 
 // <x, Omega y> for 128-vectors in shared memory, summed over the warp (pairs j = lane+1, lane+33).
 __device__ __forceinline__ float warp_omega_dot(const float* x, const float* y, int lane) {

@@ -228,6 +228,7 @@ __global__ void __launch_bounds__(512, 1) bwd_chunk1_tc(const __grid_constant__ 
                                                          const __grid_constant__ CUtensorMap tmp,
                                                          const __grid_constant__ CUtensorMap tmdy,
                                                          const __grid_constant__ CUtensorMap tmdl,
+                                                         const __grid_constant__ CUtensorMap tdq,
                                                          TcBwdArgs a) {
     const Shape s = a.s;
     const int nct = s.T / CT;
@@ -389,6 +390,9 @@ __global__ void __launch_bounds__(512, 1) bwd_chunk1_tc(const __grid_constant__ 
             bf16_to_f16_q(T_L1, row, c0);
             bf16_to_f16_q(T_K, row, c0);
         }
+        // the previous item's dq store has read its staging tile, this item's T_A (written
+        // after this barrier)
+        if (tid == 0) bulk_wait_read_all();
         publish();
         if (!ok) break;
         const uint32_t uK = smem_u32(T_K), uKB = smem_u32(T_KB), uA = smem_u32(T_A), uM = smem_u32(T_M),
@@ -520,8 +524,10 @@ __global__ void __launch_bounds__(512, 1) bwd_chunk1_tc(const __grid_constant__ 
         {   // o'' = U(-lam) (p M); scalars with do'' (o'' as stored in fp16); dy = U(lam) do''.
             // Eight rotation pairs at a time: cosine entries, then sine entries.
             QuarterAngles ang(lam, hf, u);
+            const float wb = OMEGA1 * (float)(32 * hf + 16 * u + 1);   // pair frequency, first pair
             const bool dcq = (hf == 1 && u == 1);   // pair 15 of this quarter is the DC / padding
             __half* o2row = a.O2 + ((size_t)bh * s.T + t0 + row) * 128;
+            uint32_t pc[8], ps[8];   // o'' packed: columns c0 .. c0 + 15 and c0 + 32 .. c0 + 47
     #pragma unroll
             for (int p8 = 0; p8 < 2; ++p8) {
                 float o[16], gv[16];
@@ -537,16 +543,20 @@ __global__ void __launch_bounds__(512, 1) bwd_chunk1_tc(const __grid_constant__ 
                     const float orc = round16<__half>(o[i]), ors = round16<__half>(o[8 + i]);
                     const float gc = gv[i], gs = gv[8 + i];
                     s1 = fmaf(orc, gc, fmaf(ors, gs, s1));
-                    if (!dc) {   // <o'', Omega do''>
-                        const int j = 32 * hf + 16 * u + 8 * p8 + i + 1;
-                        s2 += (6.283185307179586f * (float)j / 127.f) * (ors * gc - orc * gs);
-                    }
+                    if (!dc)   // <o'', Omega do''>
+                        s2 += (wb + OMEGA1 * (float)(8 * p8 + i)) * (ors * gc - orc * gs);
                     gv[i] = dc ? gc : c * gc - sn * gs;          // U(lam)
                     gv[8 + i] = dc ? 0.f : sn * gc + c * gs;
                 }
-                store8x2_global(o2row, c0 + 8 * p8, o);
+    #pragma unroll
+                for (int k = 0; k < 4; ++k) {
+                    pc[4 * p8 + k] = pack_f16(o[2 * k], o[2 * k + 1]);
+                    ps[4 * p8 + k] = pack_f16(o[8 + 2 * k], o[9 + 2 * k]);
+                }
                 store8x2<__half>(T_S, row, c0 + 8 * p8, gv);
             }
+            st_global_v8(o2row + c0, pc);
+            st_global_v8(o2row + c0 + 32, ps);
         }
         publish();
         if (issuer()) {   // G7: X4 = dy M^T = M dy
@@ -578,8 +588,10 @@ __global__ void __launch_bounds__(512, 1) bwd_chunk1_tc(const __grid_constant__ 
         if (a.mZ) staged_read();   // the staging tile is rewritten below (uniform branch)
         {   // do' = U(-lam) dz; <do', Omega o'> with do' as stored in fp16 (= <dz, Omega z> exactly)
             QuarterAngles ang(lam, hf, u);
+            const float wb = OMEGA1 * (float)(32 * hf + 16 * u + 1);   // pair frequency, first pair
             const bool dcq = (hf == 1 && u == 1);
             __half* d1row = a.DO1 + ((size_t)bh * s.T + t0 + row) * 128;
+            uint32_t pc[8], ps[8];   // do' packed: columns c0 .. c0 + 15 and c0 + 32 .. c0 + 47
     #pragma unroll
             for (int p8 = 0; p8 < 2; ++p8) {
                 float dz[16], z[16];
@@ -594,14 +606,19 @@ __global__ void __launch_bounds__(512, 1) bwd_chunk1_tc(const __grid_constant__ 
                     dz[8 + i] = dc ? 0.f : c * xs - sn * xc;
                     if (!dc) {   // o' = U(-lam) z
                         const float zc = c * z[i] + sn * z[8 + i], zs = c * z[8 + i] - sn * z[i];
-                        const int j = 32 * hf + 16 * u + 8 * p8 + i + 1;
-                        s3 += (6.283185307179586f * (float)j / 127.f) *
+                        s3 += (wb + OMEGA1 * (float)(8 * p8 + i)) *
                               (round16<__half>(dz[8 + i]) * zc - round16<__half>(dz[i]) * zs);
                     }
                 }
                 store8x2<__half>(T_S, row, c0 + 8 * p8, dz);
-                store8x2_global(d1row, c0 + 8 * p8, dz);
+    #pragma unroll
+                for (int k = 0; k < 4; ++k) {
+                    pc[4 * p8 + k] = pack_f16(dz[2 * k], dz[2 * k + 1]);
+                    ps[4 * p8 + k] = pack_f16(dz[8 + 2 * k], dz[9 + 2 * k]);
+                }
             }
+            st_global_v8(d1row + c0, pc);
+            st_global_v8(d1row + c0 + 32, ps);
         }
         publish();
         if (issuer()) {   // G9: X1 = dO' A^T, X3 = dO' Kbar
@@ -638,11 +655,18 @@ __global__ void __launch_bounds__(512, 1) bwd_chunk1_tc(const __grid_constant__ 
             for (int i = 0; i < 32; ++i) x[i] = fmaf(f, x[i], y[i]);
             load_q(T_L1, row, c0, y);
             s4 = dot32(y, x);
-            store_global_q(static_cast<__nv_bfloat16*>(a.dq) + gi * 128, c0, x);
+            // dq leaves through the staging tile (P3 is consumed) by a TMA store
+            store_q<__nv_bfloat16>(T_S, row, c0, x);
+            fence_async_smem();
         }
         gates_landed();   // the next item's gates, visible after the barriers below
         {
             const float dG = row_reduce(s1 + s4, false);
+            if (issuer()) {   // the staged dq rows are complete after the reduction's barrier
+                tma_store_3d(&tdq, T_S, 0, h, rowtok);
+                tma_store_3d(&tdq, T_S + TILE / 2, 64, h, rowtok);
+                bulk_commit();
+            }
             const float dL = row_reduce(s3 + s2, false);
             if (cq == 0 && ok) {
                 const size_t BTH = (size_t)s.B * s.T * s.H;
@@ -816,7 +840,7 @@ __global__ void __launch_bounds__(256, 1) adj_walk_tc(const __grid_constant__ CU
                 const int l = row & 63, jj = l & 31, j = 32 * (row >> 6) + jj + 1;
                 const bool paired = j <= NPAIR;
                 const int partner = (l >= 32) ? row - 32 : row + 32;
-                const float f = paired ? ((l >= 32) ? 1.f : -1.f) * 6.283185307179586f * (float)j / 127.f : 0.f;
+                const float f = paired ? ((l >= 32) ? 1.f : -1.f) * OMEGA1 * (float)j : 0.f;
                 float sr[64], sp[64];
                 load_half_smem(tS, row, hf, sr);
                 load_half_smem(tS, paired ? partner : row, hf, sp);
@@ -1478,8 +1502,9 @@ cudaError_t launch_bwd_tc(const TcBwdArgs& a, const TcFwdArgs& f, const void* q,
     const Shape& s = a.s;
     const int nct = s.T / CT;
     const unsigned long long BH = (unsigned long long)s.B * s.H;
-    CUtensorMap mq, mk, mv, mdo, mm, msf, msa, mo2, mdo1;
+    CUtensorMap mq, mk, mv, mdo, mm, msf, msa, mo2, mdo1, mdq;
     if (!tc_qkv_maps(s, q, k, v, &mq, &mk, &mv) || !tc_qkv_maps(s, dO, nullptr, nullptr, &mdo, nullptr, nullptr) ||
+        !tc_qkv_maps(s, a.dq, nullptr, nullptr, &mdq, nullptr, nullptr) ||
         !tc_rows_map(&mm, a.Mb, (unsigned long long)s.H * 128, true) ||
         !tc_rows_map(&msf, a.snapF, BH * nct * 2 * 128, true) ||
         !tc_rows_map(&msa, a.snapA, BH * nct * 2 * 128, true) ||
@@ -1518,7 +1543,7 @@ cudaError_t launch_bwd_tc(const TcBwdArgs& a, const TcFwdArgs& f, const void* q,
             !tc_rows_map(&mdy, bdy, BH * s.T, true) || !tc_rows_map(&mdl, bdl, BH * s.T, true))
             return cudaErrorInvalidValue;
         LaunchScope ls_("tc_bwd_chunk1", st);
-        bwd_chunk1_tc<<<grid1, 512, sm_chunk1, st>>>(mq, mk, mv, mdo, mm, msf, mz, mpp, mdy, mdl, a);
+        bwd_chunk1_tc<<<grid1, 512, sm_chunk1, st>>>(mq, mk, mv, mdo, mm, msf, mz, mpp, mdy, mdl, mdq, a);
     }
     cudaFuncSetAttribute(adj_walk_tc<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, sm_adj_seg);
     { LaunchScope ls_("tc_adj_segment", st); adj_walk_tc<false><<<gseg, 256, sm_adj_seg, st>>>(mdo1, mo2, mq, mdo, msf, msa, a); }

@@ -17,6 +17,7 @@ constexpr int CT = 128;              // tokens per chunk on this path
 constexpr int TC_SEGC = 8;           // chunks per segment (1024 tokens)
 constexpr int TILE = CT * 128 * 2;   // one 128 x 128 bf16 tile (32 KiB)
 constexpr float LOG2E = 1.4426950408889634f;
+constexpr float OMEGA1 = 6.283185307179586f / 127.f;   // 2 pi / m: frequency of rotation pair 1
 
 // error word of the including translation unit (each has its own copy)
 static __device__ int g_tc_err;
@@ -289,18 +290,16 @@ __device__ __forceinline__ void scale_q(uint8_t* tile, int r, int c0, float w) {
     for (int i = 0; i < 32; ++i) x[i] *= w;
     store_q<__half>(tile, r, c0, x);
 }
-// The thread's 32 values -> a plain row-major 16-bit row at dst (columns c0.. and c0 + 32..).
+// The thread's 32 values -> a plain row-major 16-bit row at dst (columns c0.. and c0 + 32..), as
+// two 32-byte stores (dst + c0 is 32-byte aligned: rows of 128 16-bit values, c0 a multiple of 16).
 template <typename OT>
 __device__ __forceinline__ void store_global_q(OT* dst, int c0, const float (&x)[32]) {
 #pragma unroll
-    for (int k = 0; k < 4; ++k) {
-        const float* v = x + 8 * k;
-        uint4 w;
-        w.x = pack2<OT>(v[0], v[1]);
-        w.y = pack2<OT>(v[2], v[3]);
-        w.z = pack2<OT>(v[4], v[5]);
-        w.w = pack2<OT>(v[6], v[7]);
-        *reinterpret_cast<uint4*>(dst + c0 + 32 * (k >> 1) + 8 * (k & 1)) = w;
+    for (int hb = 0; hb < 2; ++hb) {
+        uint32_t w[8];
+#pragma unroll
+        for (int k = 0; k < 8; ++k) w[k] = pack2<OT>(x[16 * hb + 2 * k], x[16 * hb + 2 * k + 1]);
+        st_global_v8(dst + c0 + 32 * hb, w);
     }
 }
 
@@ -376,10 +375,11 @@ __device__ __forceinline__ void rotate_q(float (&x)[32], int hf, int u, float la
 // <x, Omega y> over the quarter's pairs: sum_j (2 pi j / m) (x_sin,j y_cos,j - x_cos,j y_sin,j).
 __device__ __forceinline__ float omega_dot_q(const float (&x)[32], const float (&y)[32], int hf, int u) {
     float acc = 0.f;
+    const int jb = 32 * hf + 16 * u + 1;
+    const float wb = OMEGA1 * (float)jb;
 #pragma unroll
     for (int i = 0; i < 16; ++i) {
-        const int j = 32 * hf + 16 * u + i + 1;
-        if (j <= NPAIR) acc += (6.283185307179586f * (float)j / 127.f) * (x[16 + i] * y[i] - x[i] * y[16 + i]);
+        if (jb + i <= NPAIR) acc += (wb + OMEGA1 * (float)i) * (x[16 + i] * y[i] - x[i] * y[16 + i]);
     }
     return acc;
 }
