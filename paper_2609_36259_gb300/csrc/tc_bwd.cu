@@ -960,6 +960,8 @@ __global__ void __launch_bounds__(512, 1) bwd_chunk2_tc(const __grid_constant__ 
                                                          const __grid_constant__ CUtensorMap to2,
                                                          const __grid_constant__ CUtensorMap tdo1,
                                                          const __grid_constant__ CUtensorMap tsa,
+                                                         const __grid_constant__ CUtensorMap tdk,
+                                                         const __grid_constant__ CUtensorMap tdv,
                                                          TcBwdArgs a) {
     const Shape s = a.s;
     const int nct = s.T / CT;
@@ -1092,6 +1094,9 @@ __global__ void __launch_bounds__(512, 1) bwd_chunk2_tc(const __grid_constant__ 
     #pragma unroll
             for (int k = 0; k < 8; ++k)
                 mma_bf16(taddr + X1, kmajor_desc(u1, 128, k), kmajor_desc(u2, 128, k), id_kk, k > 0);
+            // the P4 epilogue rewrites T_S once this completes: the previous item's dk store must
+            // have read it first (the commit is only issued after that)
+            bulk_wait_read_all();
             mma_commit(&bars[4]);
         }
         // while it runs: the write vectors and their copies scaled by gamma^C / gamma^s
@@ -1154,12 +1159,17 @@ __global__ void __launch_bounds__(512, 1) bwd_chunk2_tc(const __grid_constant__ 
             tma_load_2d(L4 + TILE / 2, &tsa, 64, snap_row, &bars[3]);
             mark(3, it);
         }
-        if (ok) {   // dv
+        if (ok) {   // dv, staged in T_S (P2 is consumed) for a TMA store
             float x[32];
             tmem_ld16x2(tl + X2, x);
-            store_global_q(static_cast<__nv_bfloat16*>(a.dv) + gi * 128, c0, x);
+            store_q<__nv_bfloat16>(T_S, row, c0, x);
         }
         publish();
+        if (issuer()) {
+            tma_store_3d(&tdv, T_S, 0, h, rowtok);
+            tma_store_3d(&tdv, T_S + TILE / 2, 64, h, rowtok);
+            bulk_commit();
+        }
         if (issuer()) {   // X1 = dO' A^T
             ok = mbar_wait(&bars[2], ph);
             if (ok) pend &= ~0x4u;
@@ -1168,6 +1178,7 @@ __global__ void __launch_bounds__(512, 1) bwd_chunk2_tc(const __grid_constant__ 
     #pragma unroll
                 for (int k = 0; k < 8; ++k)
                     mma_bf16(taddr + X1, kmajor_desc(u3, 128, k), kmajor_desc(uA, 128, k), id_kk, k > 0);
+                bulk_wait_read_all();   // the dv store has read T_S before the P3 epilogue rewrites it
                 mma_commit(&bars[4]);
             }
         }
@@ -1225,7 +1236,7 @@ __global__ void __launch_bounds__(512, 1) bwd_chunk2_tc(const __grid_constant__ 
             tmem_ld16x2_pair(tl + X2, x, tl + X1, y);   // dk = P3^T Q + A-> D^K
     #pragma unroll
             for (int i = 0; i < 32; ++i) x[i] += y[i];
-            store_global_q(static_cast<__nv_bfloat16*>(a.dk) + gi * 128, c0, x);
+            store_q<__nv_bfloat16>(T_S, row, c0, x);   // dk, staged (P1 is consumed) for a TMA store
             float av[32];
             write_vector_q_vals(av, hf, u, lam, beta);   // unrounded a
             tmem_ld16x2_pair(tl + X3, x, tl + X4, y);   // intra- / inter-chunk da (both passes)
@@ -1237,14 +1248,21 @@ __global__ void __launch_bounds__(512, 1) bwd_chunk2_tc(const __grid_constant__ 
             cIG = dot32(av, y);
             cIL = -omega_dot_q(y, av, hf, u);
         }
-        // row sums over the four column quarters, staged in the (now idle) staging tile
-        float* s_fin = reinterpret_cast<float*>(T_S);   // [5][4][128]
+        // row sums over the four column quarters, staged in the scaled write-vector tile (its last
+        // product is complete; the next item rewrites it after its first barrier)
+        float* s_fin = reinterpret_cast<float*>(T_AS);   // [5][4][128]
+        fence_async_smem();   // the staged dk rows, for the TMA store after the barrier below
         s_fin[(0 * 4 + cq) * 128 + row] = cG;
         s_fin[(1 * 4 + cq) * 128 + row] = cL;
         s_fin[(2 * 4 + cq) * 128 + row] = db;
         s_fin[(3 * 4 + cq) * 128 + row] = cIG;
         s_fin[(4 * 4 + cq) * 128 + row] = cIL;
         ok = __syncthreads_and(ok);
+        if (issuer()) {
+            tma_store_3d(&tdk, T_S, 0, h, rowtok);
+            tma_store_3d(&tdk, T_S + TILE / 2, 64, h, rowtok);
+            bulk_commit();
+        }
         if (cq == 0 && ok) {
             float v[5];
     #pragma unroll
@@ -1273,6 +1291,7 @@ __global__ void __launch_bounds__(512, 1) bwd_chunk2_tc(const __grid_constant__ 
         for (int k = 0; k < 7; ++k)
             if (pend & (1u << k)) mbar_wait(&bars[k], (pend >> (8 + k)) & 1);
     }
+    if (tid == 0) bulk_wait_all();
     tc_fence_before();
     __syncthreads();
     if (ro.warp == 0) tmem_dealloc(taddr, 512);
@@ -1559,7 +1578,9 @@ cudaError_t launch_bwd_tc(const TcBwdArgs& a, const TcFwdArgs& f, const void* q,
         const long long items = (long long)s.B * s.H * nct;
         const int grid2 = (int)(items < sms ? items : sms);
         LaunchScope ls_("tc_bwd_chunk2", st);
-        bwd_chunk2_tc<<<grid2, 512, sm_chunk2, st>>>(mq, mk, mv, mdo, mo2, mdo1, msa, a);
+        CUtensorMap mdk, mdv;
+        if (!tc_qkv_maps(s, a.dk, a.dv, nullptr, &mdk, &mdv, nullptr)) return cudaErrorInvalidValue;
+        bwd_chunk2_tc<<<grid2, 512, sm_chunk2, st>>>(mq, mk, mv, mdo, mo2, mdo1, msa, mdk, mdv, a);
     }
     { LaunchScope ls_("tc_gate", st); tc_gate_kernel<<<gchunk, 128, 0, st>>>(a); }
     if (a.dR) {   // dR from the middle-readout vectors bwd_chunk1_tc wrote
