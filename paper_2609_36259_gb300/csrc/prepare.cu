@@ -98,15 +98,22 @@ __global__ void __launch_bounds__(256) prep_scan_kernel(PrepareArgs a, int nseg)
     double wex = 0.0;
     for (int w = 0; w < warp; ++w) wex += s_wtot[w];
     const double excl = s_base + wex + (incl - pref);
+    // clock mod m: the clock before this thread's first token is reduced once in fp64 (one
+    // multiply by 1/m, no divide); its four tokens add their increments in fp64 (together < 4,
+    // so at most one wrap) and are rounded to fp32 once
+    double bm = fma(-127.0, floor(excl * (1.0 / 127.0)), excl);
+    if (bm < 0.0) bm += 127.0;
+    else if (bm >= 127.0) bm -= 127.0;
 #pragma unroll
     for (int u = 0; u < 4; ++u) {
         const int i = 4 * threadIdx.x + u;
         if (i < len) {
             const size_t gi = ((size_t)b * T + t0 + i) * H + h;
-            const double lam = excl + loc[u];
-            a.lam_mod[gi] = (float)(lam - 127.0 * floor(lam / 127.0));
+            double lm = bm + loc[u];
+            if (lm >= 127.0) lm -= 127.0;
+            a.lam_mod[gi] = (float)lm;
             a.g_cum[gi] = gex + lp[u];
-            if (a.lambda_end && t0 + i == T - 1) a.lambda_end[bh] = lam;
+            if (a.lambda_end && t0 + i == T - 1) a.lambda_end[bh] = excl + loc[u];
         }
     }
 }

@@ -733,9 +733,19 @@ __global__ void __launch_bounds__(256, 1) adj_walk_tc(const __grid_constant__ CU
     constexpr int NT = SNAP ? 3 : 2;                       // tiles per buffer
     constexpr int NB = SNAP ? 2 : 3;                       // buffers: loads run NB - 1 chunks ahead
     uint8_t* tiles = smem + 1024 + 4 * TC_SEGC * CT;       // [buf][X | Y (| S)]
-    for (int i = tid; i < nc * CT; i += 256) {   // every token's decay, loaded once
-        const int t0 = (c_begin + i / CT) * CT;
-        s_gs[i] = cum128(s, a.g, b, h, t0, t0 + (i % CT));
+    {   // every token's decay, loaded once: all of a thread's loads in flight together
+        constexpr int NPT = TC_SEGC * CT / 256;
+        float v[NPT], w[NPT];
+#pragma unroll
+        for (int k = 0; k < NPT; ++k) {
+            const int i = tid + 256 * k;
+            const int t0 = (c_begin + i / CT) * CT, t = t0 + i % CT;
+            v[k] = i < nc * CT ? a.g[((size_t)b * s.T + t) * s.H + h] : 0.f;
+            w[k] = (i < nc * CT && s.Cg == 64 && t - t0 >= 64) ? a.g[((size_t)b * s.T + t0 + 63) * s.H + h] : 0.f;
+        }
+#pragma unroll
+        for (int k = 0; k < NPT; ++k)
+            if (tid + 256 * k < nc * CT) s_gs[tid + 256 * k] = v[k] + w[k];   // cum128
     }
     if (tid == 0) {
         for (int i = 0; i < 2 * NB; ++i) mbar_init(&bars[i], 1);   // tma[NB], mma[NB]
@@ -810,9 +820,9 @@ __global__ void __launch_bounds__(256, 1) adj_walk_tc(const __grid_constant__ CU
     for (int it = 0; it < total; ++it) {
         const int part = it / nc, c = chunk_of(it), buf = it % NB;
         const int cg = c_begin + c;
-        // product it - 1 must be complete before the other buffer is refilled (and, in the SNAP
-        // walk, before D is read); the refill goes out as early as possible: the walks are bound
-        // by how far ahead their loads run
+        // product it - 1 must be complete before its buffer is refilled (and, in the SNAP walk,
+        // before D is read); the refill goes out right after this chunk's operand rows are
+        // prepared, which overlaps product it - 1
         auto refill = [&]() {
             if (it >= 1 && ok) ok = mbar_wait(&bars[NB + (it - 1) % NB], ((it - 1) / NB) & 1);
             tc_fence_after();
@@ -821,12 +831,18 @@ __global__ void __launch_bounds__(256, 1) adj_walk_tc(const __grid_constant__ CU
                 issue(it + NB - 1);
             }
         };
-        refill();
         if (ok) ok = mbar_wait(&bars[buf], (it / NB) & 1);
         if (tid == 0 && ok) ++landed;
         const float g = s_gs[c * CT + row];
         uint8_t* tX = tiles + (NT * buf) * TILE;
-        float w;
+        // this chunk's operand rows (its own buffer) are prepared while product it - 1 runs
+        float w = SNAP ? ex2(g * LOG2E) : ex2((s_pre[c] + g) * LOG2E);
+        if (part == 0) w *= s.scale;   // q~ = s q
+        if (ok) {
+            scale_half_smem(tX, row, hf, w);
+            bf16_to_f16_half(tX + TILE, row, hf);   // q or dO
+        }
+        refill();
         if (SNAP) {
             // adjoint of this chunk's end state, then D <- gamma^C D (this part's 128 columns)
             uint8_t* tS = tX + 2 * TILE;
@@ -857,14 +873,6 @@ __global__ void __launch_bounds__(256, 1) adj_walk_tc(const __grid_constant__ CU
 #pragma unroll
             for (int i = 0; i < 64; ++i) x[i] *= dC;
             tmem_st64(tl + 128 * part + 64 * hf, x);
-            w = ex2(g * LOG2E);
-        } else {
-            w = ex2((s_pre[c] + g) * LOG2E);
-        }
-        if (part == 0) w *= s.scale;   // q~ = s q
-        if (ok) {
-            scale_half_smem(tX, row, hf, w);
-            bf16_to_f16_half(tX + TILE, row, hf);   // q or dO
         }
 
         fence_async_smem();

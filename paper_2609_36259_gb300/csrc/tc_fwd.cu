@@ -42,12 +42,29 @@ __global__ void __launch_bounds__(512, 1) seg_state_tc(const __grid_constant__ C
     float* s_beta = s_lam + SEGC * CT;
     float* s_gs = s_beta + SEGC * CT;                                // chunk-local decays
     uint8_t* tiles = smem + 1024 + 12 * SEGC * CT;                   // [buf][A | K | V]
-    for (int i = tid; i < nc * CT; i += 512) {   // every token's gates, loaded once
-        const int t0 = (c_begin + i / CT) * CT, t = t0 + i % CT;
-        const size_t gi = ((size_t)b * s.T + t) * s.H + h;
-        s_lam[i] = a.lam[gi];
-        s_beta[i] = a.beta[gi];
-        s_gs[i] = cum128(s, a.g, b, h, t0, t);
+    {   // every token's gates, loaded once: all of a thread's loads in flight together
+        constexpr int NPT = SEGC * CT / 512;
+        float l[NPT], be[NPT], v[NPT], w[NPT];
+#pragma unroll
+        for (int k = 0; k < NPT; ++k) {
+            const int i = tid + 512 * k;
+            const int t0 = (c_begin + i / CT) * CT, t = t0 + i % CT;
+            const size_t gi = ((size_t)b * s.T + t) * s.H + h;
+            const bool in = i < nc * CT;
+            l[k] = in ? a.lam[gi] : 0.f;
+            be[k] = in ? a.beta[gi] : 0.f;
+            v[k] = in ? a.g[gi] : 0.f;
+            w[k] = (in && s.Cg == 64 && t - t0 >= 64) ? a.g[((size_t)b * s.T + t0 + 63) * s.H + h] : 0.f;
+        }
+#pragma unroll
+        for (int k = 0; k < NPT; ++k) {
+            const int i = tid + 512 * k;
+            if (i < nc * CT) {
+                s_lam[i] = l[k];
+                s_beta[i] = be[k];
+                s_gs[i] = v[k] + w[k];   // cum128
+            }
+        }
     }
 
     if (tid == 0) {
@@ -85,7 +102,9 @@ __global__ void __launch_bounds__(512, 1) seg_state_tc(const __grid_constant__ C
     __syncthreads();
     bool ok = true;
     constexpr bool F16 = std::is_same<OT, __half>::value;
-    const uint32_t idesc = idesc_k16<OT>(128, 128, 1, 1);
+    // one N = 256 product per K-step: B = [K | V] (adjacent tiles, 64-column blocks 16 KiB apart),
+    // D = [Kbar | Vbar] (TMEM columns 0 .. 255), the A-> operand read once
+    const uint32_t idesc = idesc_k16<OT>(128, 256, 1, 1);
     for (int c = 0; c < nc; ++c) {
         const int buf = c & 1;
         // A-> rows of this chunk, scaled by the decay from the token to the segment end (its
@@ -112,14 +131,10 @@ __global__ void __launch_bounds__(512, 1) seg_state_tc(const __grid_constant__ C
                 tc_fence_after();
                 const uint32_t tA = smem_u32(tiles + 3 * buf * TILE);
                 const uint32_t tK = smem_u32(tiles + (3 * buf + 1) * TILE);
-                const uint32_t tV = smem_u32(tiles + (3 * buf + 2) * TILE);
 #pragma unroll
-                for (int k = 0; k < 8; ++k) {
+                for (int k = 0; k < 8; ++k)
                     mma_bf16(taddr, mnmajor_desc(tA, 128, k), mnmajor_desc(tK, 128, k), idesc,
                              (c > 0 || k > 0) ? 1u : 0u);
-                    mma_bf16(taddr + 128, mnmajor_desc(tA, 128, k), mnmajor_desc(tV, 128, k),
-                             idesc, (c > 0 || k > 0) ? 1u : 0u);
-                }
                 mma_commit(&bars[2 + buf]);
             }
         }
@@ -287,7 +302,8 @@ __global__ void __launch_bounds__(OUT_THREADS, 1) seg_out_tc(const __grid_consta
         const int r = tid - OUT_CHAIN;                 // row of every tile / TMEM lane
         const uint32_t tlane = taddr + ((uint32_t)(32 * ((tid >> 5) & 3)) << 16);
         const bool leader = tid == OUT_CHAIN;
-        const uint32_t id_nn = idesc_f16(128, 128, 1, 1);
+        const uint32_t id_nn2 = idesc_f16(128, 256, 1, 1);
+        static_assert(SV == SK + 128, "the state update writes [Kbar | Vbar] as one accumulator");
         bool su_issued = false;   // leader: a state update that nobody has waited for
         bool qk_pending = false, v_pending = false;
         uint32_t qk_par = 0, v_par = 0;   // parity of the pending loads' phases
@@ -413,13 +429,12 @@ __global__ void __launch_bounds__(OUT_THREADS, 1) seg_out_tc(const __grid_consta
                 if (save) store_snap(c_begin + c, 1);
                 mbar_arrive(&bars[OB_SR]);
                 if (!last) {   // state update [Kbar | Vbar] += A->^T [K | V], issued from here so
-                               // that the chain's own commits never wait for it
+                               // that the chain's own commits never wait for it; one N = 256
+                               // product (T_K, T_V adjacent; SK, SV adjacent)
                     tc_fence_after();
 #pragma unroll
-                    for (int k = 0; k < 8; ++k) {
-                        mma_bf16(taddr + SK, mnmajor_desc(uQ, 128, k), mnmajor_desc(uK, 128, k), id_nn, 1u);
-                        mma_bf16(taddr + SV, mnmajor_desc(uQ, 128, k), mnmajor_desc(uV, 128, k), id_nn, 1u);
-                    }
+                    for (int k = 0; k < 8; ++k)
+                        mma_bf16(taddr + SK, mnmajor_desc(uQ, 128, k), mnmajor_desc(uK, 128, k), id_nn2, 1u);
                     mma_commit(&bars[OB_SU]);
                     su_issued = true;
                 }
