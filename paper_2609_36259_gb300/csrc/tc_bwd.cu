@@ -905,16 +905,19 @@ __global__ void __launch_bounds__(256, 1) adj_walk_tc(const __grid_constant__ CU
         dst[0] = s_bnd[2 * tid];
         dst[1] = s_bnd[2 * tid + 1];
     }
-    if (ok && !SNAP) {
-        float* dst = a.segD + (((size_t)bh * a.nseg + seg) * 128 + row) * 256 + 128 * hf;
+    if (ok && !SNAP) {   // the segment's contribution out through the (now idle) tiles, coalesced
+        float* stage = reinterpret_cast<float*>(tiles);
 #pragma unroll
         for (int q2 = 0; q2 < 2; ++q2) {
             float x[64];
             tmem_ld64(tl + 128 * hf + 64 * q2, x);
 #pragma unroll
             for (int i = 0; i < 64; i += 4)
-                *reinterpret_cast<float4*>(dst + 64 * q2 + i) = make_float4(x[i], x[i + 1], x[i + 2], x[i + 3]);
+                *reinterpret_cast<float4*>(stage + row * STAGE_LD + 128 * hf + 64 * q2 + i) =
+                    make_float4(x[i], x[i + 1], x[i + 2], x[i + 3]);
         }
+        __syncthreads();
+        stage_to_global_128x256(a.segD + ((size_t)bh * a.nseg + seg) * 128 * 256, stage, tid, 256);
     }
     if (!ok && tid == 0) {
         flag_error(CYFA_ERR_TIMEOUT);

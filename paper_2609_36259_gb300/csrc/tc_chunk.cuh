@@ -432,6 +432,20 @@ __device__ __forceinline__ void mask_decay_q(float (&x)[32], float mul, int row,
     }
 }
 
+// A [128][256] fp32 block staged in shared memory with rows padded to STAGE_LD floats (so that a
+// warp's 16-byte stores to 32 different rows hit distinct banks) -> a contiguous global
+// [128][256] block, every warp writing 512 contiguous bytes per instruction.  The caller has
+// filled the stage and synchronised the block.
+constexpr int STAGE_LD = 260;
+__device__ __forceinline__ void stage_to_global_128x256(float* dst, const float* stage, int tid,
+                                                        int nthreads) {
+    for (int i = tid; i < 128 * 64; i += nthreads) {
+        const int r = i >> 6, c4 = i & 63;
+        *reinterpret_cast<float4*>(dst + r * 256 + 4 * c4) =
+            *reinterpret_cast<const float4*>(stage + r * STAGE_LD + 4 * c4);
+    }
+}
+
 __device__ __forceinline__ float dot32(const float (&x)[32], const float (&y)[32]) {
     float acc = 0.f;
 #pragma unroll

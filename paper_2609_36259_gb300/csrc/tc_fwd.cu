@@ -42,6 +42,21 @@ __global__ void __launch_bounds__(512, 1) seg_state_tc(const __grid_constant__ C
     float* s_beta = s_lam + SEGC * CT;
     float* s_gs = s_beta + SEGC * CT;                                // chunk-local decays
     uint8_t* tiles = smem + 1024 + 12 * SEGC * CT;                   // [buf][A | K | V]
+    auto issue_kv = [&](int c, int buf) {
+        uint8_t* tK = tiles + (3 * buf + 1) * TILE;
+        uint8_t* tV = tiles + (3 * buf + 2) * TILE;
+        const int row = b * s.T + (c_begin + c) * CT;
+        mbar_expect_tx(&bars[buf], 2 * TILE);
+        tma_load_3d(tK, &tk, 0, h, row, &bars[buf]);
+        tma_load_3d(tK + TILE / 2, &tk, 64, h, row, &bars[buf]);
+        tma_load_3d(tV, &tv, 0, h, row, &bars[buf]);
+        tma_load_3d(tV + TILE / 2, &tv, 64, h, row, &bars[buf]);
+    };
+    if (tid == 0) {   // chunk 0's K and V are on their way while the gates load
+        for (int i = 0; i < 4; ++i) mbar_init(&bars[i], 1);
+        fence_mbar_init();
+        issue_kv(0, 0);
+    }
     {   // every token's gates, loaded once: all of a thread's loads in flight together
         constexpr int NPT = SEGC * CT / 512;
         float l[NPT], be[NPT], v[NPT], w[NPT];
@@ -67,10 +82,6 @@ __global__ void __launch_bounds__(512, 1) seg_state_tc(const __grid_constant__ C
         }
     }
 
-    if (tid == 0) {
-        for (int i = 0; i < 4; ++i) mbar_init(&bars[i], 1);
-        fence_mbar_init();
-    }
     if (ro.warp == 0) tmem_alloc(s_taddr, 256);
     if (tid < nc) {
         const int t0 = (c_begin + tid) * CT;
@@ -88,17 +99,6 @@ __global__ void __launch_bounds__(512, 1) seg_state_tc(const __grid_constant__ C
         }
         a.segG[(size_t)bh * a.nseg + seg] = acc;
     }
-    auto issue_kv = [&](int c, int buf) {
-        uint8_t* tK = tiles + (3 * buf + 1) * TILE;
-        uint8_t* tV = tiles + (3 * buf + 2) * TILE;
-        const int row = b * s.T + (c_begin + c) * CT;
-        mbar_expect_tx(&bars[buf], 2 * TILE);
-        tma_load_3d(tK, &tk, 0, h, row, &bars[buf]);
-        tma_load_3d(tK + TILE / 2, &tk, 64, h, row, &bars[buf]);
-        tma_load_3d(tV, &tv, 0, h, row, &bars[buf]);
-        tma_load_3d(tV + TILE / 2, &tv, 64, h, row, &bars[buf]);
-    };
-    if (tid == 0) issue_kv(0, 0);
     __syncthreads();
     bool ok = true;
     constexpr bool F16 = std::is_same<OT, __half>::value;
@@ -142,16 +142,19 @@ __global__ void __launch_bounds__(512, 1) seg_state_tc(const __grid_constant__ C
     if (ok) ok = mbar_wait(&bars[2 + ((nc - 1) & 1)], ((nc - 1) >> 1) & 1);
     tc_fence_after();
     ok = __syncthreads_and(ok);
-    if (ok) {   // [Kbar | Vbar] delta out: each thread 64 of the row's 256 columns
-        float* dst = a.segS + (((size_t)bh * a.nseg + seg) * 128 + ro.row) * 256 + 64 * ro.cq;
+    if (ok) {   // [Kbar | Vbar] delta out through the (now idle) tiles, coalesced
+        float* stage = reinterpret_cast<float*>(tiles);
         const uint32_t tl = taddr + ((uint32_t)(32 * ro.q) << 16) + 64 * ro.cq;
         for (int c0 = 0; c0 < 64; c0 += 32) {
             float v[32];
             tmem_ld32(tl + c0, v);
 #pragma unroll
             for (int i = 0; i < 32; i += 4)
-                *reinterpret_cast<float4*>(dst + c0 + i) = make_float4(v[i], v[i + 1], v[i + 2], v[i + 3]);
+                *reinterpret_cast<float4*>(stage + ro.row * STAGE_LD + 64 * ro.cq + c0 + i) =
+                    make_float4(v[i], v[i + 1], v[i + 2], v[i + 3]);
         }
+        __syncthreads();
+        stage_to_global_128x256(a.segS + ((size_t)bh * a.nseg + seg) * 128 * 256, stage, tid, 512);
     } else if (tid == 0) {
         flag_error(CYFA_ERR_TIMEOUT);
         // let copies still in flight land before the shared memory is released
