@@ -733,6 +733,38 @@ __global__ void __launch_bounds__(256, 1) adj_walk_tc(const __grid_constant__ CU
     constexpr int NT = SNAP ? 3 : 2;                       // tiles per buffer
     constexpr int NB = SNAP ? 2 : 3;                       // buffers: loads run NB - 1 chunks ahead
     uint8_t* tiles = smem + 1024 + 4 * TC_SEGC * CT;       // [buf][X | Y (| S)]
+    const int total = 2 * nc;   // iterations: part 0 (K) chunks, then part 1 (V) chunks
+    auto chunk_of = [&](int it) {
+        const int i = it % nc;
+        return SNAP ? nc - 1 - i : i;
+    };
+    int issued = 0, landed = 0;   // thread 0: loads issued / seen complete
+    auto issue = [&](int it) {
+        const int part = it / nc, c = chunk_of(it), buf = it % NB;
+        ++issued;
+        uint8_t* tX = tiles + (NT * buf) * TILE;
+        uint8_t* tY = tX + TILE;
+        const int t0 = (c_begin + c) * CT;
+        const int xrow = bh * s.T + t0, yrow = b * s.T + t0;
+        const CUtensorMap* mx = part == 0 ? &tdo1 : &to2;
+        const CUtensorMap* my = part == 0 ? &tq : &tdo;
+        mbar_expect_tx(&bars[buf], NT * TILE);
+        tma_load_2d(tX, mx, 0, xrow, &bars[buf]);
+        tma_load_2d(tX + TILE / 2, mx, 64, xrow, &bars[buf]);
+        tma_load_3d(tY, my, 0, h, yrow, &bars[buf]);
+        tma_load_3d(tY + TILE / 2, my, 64, h, yrow, &bars[buf]);
+        if (SNAP) {
+            uint8_t* tS = tX + 2 * TILE;
+            const int srow = ((bh * nct + c_begin + c) * 2 + part) * 128;
+            tma_load_2d(tS, &tsf, 0, srow, &bars[buf]);
+            tma_load_2d(tS + TILE / 2, &tsf, 64, srow, &bars[buf]);
+        }
+    };
+    if (tid == 0) {   // the first operand tiles are on their way while the decays load
+        for (int i = 0; i < 2 * NB; ++i) mbar_init(&bars[i], 1);   // tma[NB], mma[NB]
+        fence_mbar_init();
+        for (int i = 0; i < NB - 1 && i < total; ++i) issue(i);
+    }
     {   // every token's decay, loaded once: all of a thread's loads in flight together
         constexpr int NPT = TC_SEGC * CT / 256;
         float v[NPT], w[NPT];
@@ -746,10 +778,6 @@ __global__ void __launch_bounds__(256, 1) adj_walk_tc(const __grid_constant__ CU
 #pragma unroll
         for (int k = 0; k < NPT; ++k)
             if (tid + 256 * k < nc * CT) s_gs[tid + 256 * k] = v[k] + w[k];   // cum128
-    }
-    if (tid == 0) {
-        for (int i = 0; i < 2 * NB; ++i) mbar_init(&bars[i], 1);   // tma[NB], mma[NB]
-        fence_mbar_init();
     }
     if (ro.warp == 0) tmem_alloc(s_taddr, 256);
     if (tid < nc) {
@@ -783,35 +811,6 @@ __global__ void __launch_bounds__(256, 1) adj_walk_tc(const __grid_constant__ CU
             tmem_st64(tl + 128 * hf + 64 * q2, x);
         }
     }
-    const int total = 2 * nc;   // iterations: part 0 (K) chunks, then part 1 (V) chunks
-    auto chunk_of = [&](int it) {
-        const int i = it % nc;
-        return SNAP ? nc - 1 - i : i;
-    };
-    int issued = 0, landed = 0;   // thread 0: loads issued / seen complete
-    auto issue = [&](int it) {
-        const int part = it / nc, c = chunk_of(it), buf = it % NB;
-        ++issued;
-        uint8_t* tX = tiles + (NT * buf) * TILE;
-        uint8_t* tY = tX + TILE;
-        const int t0 = (c_begin + c) * CT;
-        const int xrow = bh * s.T + t0, yrow = b * s.T + t0;
-        const CUtensorMap* mx = part == 0 ? &tdo1 : &to2;
-        const CUtensorMap* my = part == 0 ? &tq : &tdo;
-        mbar_expect_tx(&bars[buf], NT * TILE);
-        tma_load_2d(tX, mx, 0, xrow, &bars[buf]);
-        tma_load_2d(tX + TILE / 2, mx, 64, xrow, &bars[buf]);
-        tma_load_3d(tY, my, 0, h, yrow, &bars[buf]);
-        tma_load_3d(tY + TILE / 2, my, 64, h, yrow, &bars[buf]);
-        if (SNAP) {
-            uint8_t* tS = tX + 2 * TILE;
-            const int srow = ((bh * nct + c_begin + c) * 2 + part) * 128;
-            tma_load_2d(tS, &tsf, 0, srow, &bars[buf]);
-            tma_load_2d(tS + TILE / 2, &tsf, 64, srow, &bars[buf]);
-        }
-    };
-    if (tid == 0)
-        for (int i = 0; i < NB - 1 && i < total; ++i) issue(i);
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
