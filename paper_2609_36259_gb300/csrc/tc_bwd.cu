@@ -760,10 +760,24 @@ __global__ void __launch_bounds__(256, 1) adj_walk_tc(const __grid_constant__ CU
             tma_load_2d(tS + TILE / 2, &tsf, 64, srow, &bars[buf]);
         }
     };
+    auto prefetch = [&](int it) {   // the tiles of iteration it into L2
+        const int part = it / nc, c = chunk_of(it);
+        const int t0 = (c_begin + c) * CT;
+        const int xrow = bh * s.T + t0, yrow = b * s.T + t0;
+        const CUtensorMap* mx = part == 0 ? &tdo1 : &to2;
+        const CUtensorMap* my = part == 0 ? &tq : &tdo;
+#pragma unroll
+        for (int x = 0; x < 128; x += 64) {
+            tma_prefetch_2d(mx, x, xrow);
+            tma_prefetch_3d(my, x, h, yrow);
+            if (SNAP) tma_prefetch_2d(&tsf, x, ((bh * nct + c_begin + c) * 2 + part) * 128);
+        }
+    };
     if (tid == 0) {   // the first operand tiles are on their way while the decays load
         for (int i = 0; i < 2 * NB; ++i) mbar_init(&bars[i], 1);   // tma[NB], mma[NB]
         fence_mbar_init();
         for (int i = 0; i < NB - 1 && i < total; ++i) issue(i);
+        if (NB - 1 < total) prefetch(NB - 1);
     }
     {   // every token's decay, loaded once: all of a thread's loads in flight together
         constexpr int NPT = TC_SEGC * CT / 256;
@@ -828,6 +842,7 @@ __global__ void __launch_bounds__(256, 1) adj_walk_tc(const __grid_constant__ CU
             if (tid == 0 && ok && it + NB - 1 < total) {
                 if (SNAP) bulk_wait_read_all();   // the other buffer's S tile may be a store's source
                 issue(it + NB - 1);
+                if (it + NB < total) prefetch(it + NB);
             }
         };
         if (ok) ok = mbar_wait(&bars[buf], (it / NB) & 1);

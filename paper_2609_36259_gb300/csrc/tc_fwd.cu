@@ -116,6 +116,13 @@ __global__ void __launch_bounds__(512, 1) seg_state_tc(const __grid_constant__ C
         }
         if (c >= 1 && ok) ok = mbar_wait(&bars[2 + ((c - 1) & 1)], ((c - 1) >> 1) & 1);
         if (tid == 0 && ok && c + 1 < nc) issue_kv(c + 1, (c + 1) & 1);
+        if (tid == 0 && c + 2 < nc) {   // the chunk after into L2: its load then comes from there
+            const int r2 = b * s.T + (c_begin + c + 2) * CT;
+            tma_prefetch_3d(&tk, 0, h, r2);
+            tma_prefetch_3d(&tk, 64, h, r2);
+            tma_prefetch_3d(&tv, 0, h, r2);
+            tma_prefetch_3d(&tv, 64, h, r2);
+        }
         if (F16) {   // the bf16 K and V tiles become fp16 operands
             if (ok) ok = mbar_wait(&bars[buf], (c >> 1) & 1);
             if (ok) {
@@ -371,6 +378,15 @@ __global__ void __launch_bounds__(OUT_THREADS, 1) seg_out_tc(const __grid_consta
             const bool last = c + 1 == nc;
             float n_lam = 0.f, n_beta = 0.f, n_g2 = 0.f, n_g2C = 0.f;
             if (!last) gates(c + 1, n_lam, n_beta, n_g2, n_g2C);
+            if (leader && !last) {   // the next chunk's Q, K, V into L2: their loads wait for tiles
+                const int r1 = b * s.T + (c_begin + c + 1) * CT;
+#pragma unroll
+                for (int x = 0; x < 128; x += 64) {
+                    tma_prefetch_3d(&tq, x, h, r1);
+                    tma_prefetch_3d(&tk, x, h, r1);
+                    tma_prefetch_3d(&tv, x, h, r1);
+                }
+            }
             // S1: product 1 has read Q and the Kbar snapshot
             if (ok) ok = mbar_wait_ab(&bars[OB_F1], c & 1, s_abort);
             if (save && leader) bulk_wait_read_all();   // the Kbar snapshot store has read T_N
