@@ -276,7 +276,7 @@ def run_ours(args):
     # per-kernel times and the forward / backward split
     per_kernel = {k: {'launches': n, 'ms_per_launch': t / n if n else 0.0}
                   for k, (n, t) in stats.items()}
-    fwd_names = ('readout_matrix', 'fwd_state', 'fwd_out', 'm_to_f16', 'tc_seg_state',
+    fwd_names = ('readout_matrix', 'readout_f16', 'fwd_state', 'fwd_out', 'tc_seg_state',
                  'tc_seg_scan', 'tc_seg_out')
     # the forward's kernels are launched again inside the backward (recomputation): split by
     # launch count, one forward's worth per step belongs to cyfa_chunk_fwd

@@ -236,7 +236,8 @@ int cyfa_chunk_fwd(const cyfa_dims_t* dims, const void* q, const void* k, const 
     if (!aligned16(workspace)) return CYFA_ERR_ALIGN;
     const FwdLayout L = fwd_layout(s, tc_path, workspace);
     cudaStream_t st = static_cast<cudaStream_t>(stream);
-    rc = cuda_status(launch_readout_matrix(s.H, R, L.M, L.MT, st));
+    rc = cuda_status(tc_path ? launch_readout_f16(s.H, R, L.Mb, st)
+                             : launch_readout_matrix(s.H, R, L.M, L.MT, st));
     if (rc) return rc;
     if (tc_path) {
         TcFwdArgs t;
@@ -254,7 +255,7 @@ int cyfa_chunk_fwd(const cyfa_dims_t* dims, const void* q, const void* k, const 
         t.Mb = L.Mb;
         t.snap = static_cast<__half*>(saved);
         t.nseg = L.nseg;
-        return cuda_status(launch_fwd_tc(t, q, k, v, L.M, st));
+        return cuda_status(launch_fwd_tc(t, q, k, v, st));
     }
     FwdArgs a;
     a.s = s;
@@ -297,7 +298,8 @@ int cyfa_chunk_bwd(const cyfa_dims_t* dims, const void* q, const void* k, const 
     if (!aligned16(workspace)) return CYFA_ERR_ALIGN;
     const BwdLayout L = bwd_layout(s, tc_path, workspace);
     cudaStream_t st = static_cast<cudaStream_t>(stream);
-    rc = cuda_status(launch_readout_matrix(s.H, R, L.M, L.MT, st));
+    rc = cuda_status(tc_path ? launch_readout_f16(s.H, R, L.Mb, st)
+                             : launch_readout_matrix(s.H, R, L.M, L.MT, st));
     if (rc) return rc;
     BwdArgs a;
     a.s = s;
@@ -382,7 +384,7 @@ int cyfa_chunk_bwd(const cyfa_dims_t* dims, const void* q, const void* k, const 
         t.mDL = dR ? L.mDL : nullptr;
         t.dMp = L.dMp;
         t.dm_split = L.dm_split;
-        return cuda_status(launch_bwd_tc(t, f, q, k, v, dO, L.M, st));
+        return cuda_status(launch_bwd_tc(t, f, q, k, v, dO, st));
     }
     return cuda_status(launch_bwd_simt(a, st));
 }

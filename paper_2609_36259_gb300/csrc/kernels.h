@@ -114,7 +114,9 @@ struct TcFwdArgs {
 bool tc_fwd_supported(const Shape& s);
 int tc_fwd_segments(const Shape& s);
 cudaError_t launch_fwd_tc(const TcFwdArgs& a, const void* q, const void* k, const void* v,
-                          const float* Mf, cudaStream_t st);
+                          cudaStream_t st);
+// M = R Phi as fp16 in the tensor-core column order ([H][128][128], padding row / column zero).
+cudaError_t launch_readout_f16(int H, const float* R, __half* Mb, cudaStream_t st);
 // Reads (and clears) the error word of the tensor-core kernels; synchronises the stream.
 cudaError_t tc_read_error(cudaStream_t st, int* err);
 cudaError_t tc_bwd_read_error(cudaStream_t st, int* err);
@@ -124,11 +126,11 @@ bool tc_qkv_maps(const Shape& s, const void* q, const void* k, const void* v, CU
                  CUtensorMap* mk, CUtensorMap* mv, unsigned box_rows = 128);
 bool tc_rows_map(CUtensorMap* map, const void* base, unsigned long long rows, bool f16 = false,
                  unsigned box_rows = 128);
-// M -> fp16 (tensor-core order), segment state contributions, segment scan.
+// Segment state contributions and the segment scan.
 cudaError_t launch_fwd_segment_states(const TcFwdArgs& a, const void* k, const void* v,
-                                      const float* Mf, cudaStream_t st);
-// M -> fp16 (tensor-core order) and the total log-decay of every segment, without the states.
-cudaError_t launch_m_and_segment_decay(const TcFwdArgs& a, const float* Mf, cudaStream_t st);
+                                      cudaStream_t st);
+// The total log-decay of every segment, without the states.
+cudaError_t launch_segment_decay(const TcFwdArgs& a, cudaStream_t st);
 
 struct TcBwdArgs {
     Shape s;
@@ -160,7 +162,7 @@ struct TcBwdArgs {
     float* dR;                   // [H][127][127]
 };
 cudaError_t launch_bwd_tc(const TcBwdArgs& a, const TcFwdArgs& f, const void* q, const void* k,
-                          const void* v, const void* dO, const float* Mf, cudaStream_t st);
+                          const void* v, const void* dO, cudaStream_t st);
 
 // ---- decode (decode.cu) ----
 struct StepArgs {

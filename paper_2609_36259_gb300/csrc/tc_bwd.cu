@@ -1542,7 +1542,7 @@ __global__ void __launch_bounds__(256) tc_dA_kernel(TcBwdArgs a) {
 }  // namespace
 
 cudaError_t launch_bwd_tc(const TcBwdArgs& a, const TcFwdArgs& f, const void* q, const void* k,
-                          const void* v, const void* dO, const float* Mf, cudaStream_t st) {
+                          const void* v, const void* dO, cudaStream_t st) {
     const Shape& s = a.s;
     const int nct = s.T / CT;
     const unsigned long long BH = (unsigned long long)s.B * s.H;
@@ -1556,8 +1556,7 @@ cudaError_t launch_bwd_tc(const TcBwdArgs& a, const TcFwdArgs& f, const void* q,
         return cudaErrorInvalidValue;
     // chunk-start states: the forward's saved snapshots, or recomputed (segment states, then a
     // walk of every segment)
-    cudaError_t e = a.saved ? launch_m_and_segment_decay(f, Mf, st)
-                            : launch_fwd_segment_states(f, k, v, Mf, st);
+    cudaError_t e = a.saved ? launch_segment_decay(f, st) : launch_fwd_segment_states(f, k, v, st);
     if (e != cudaSuccess) return e;
     // heads fastest: the CTAs that read the same token rows of q, k, v, dO run together
     const dim3 gseg(s.B * s.H, a.nseg), gchunk(s.B * s.H, nct);

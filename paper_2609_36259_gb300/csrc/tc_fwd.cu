@@ -761,12 +761,50 @@ __global__ void __launch_bounds__(OUT_THREADS, 1) seg_out_tc(const __grid_consta
     if (tid < 32) tmem_dealloc(taddr, 512);
 }
 
-// M (fp32, paper order) -> fp16 with its Fourier (column) index in the tensor-core order.
-__global__ void m_to_f16_kernel(const float* M, __half* Mb, int H) {
-    const int i = blockIdx.x * blockDim.x + threadIdx.x;
-    if (i >= H * 128 * 128) return;
-    const int p = i & 127, rest = i >> 7;
-    Mb[rest * 128 + tc_slot(p)] = __float2half_rn(M[i]);
+// M = R Phi (App. A.1 Eq. app-real-fourier: Phi[r][0] = 1/sqrt(m), Phi[r][2j-1] =
+// sqrt(2/m) cos(2 pi j r / m), Phi[r][2j] = sqrt(2/m) sin(2 pi j r / m)) straight into fp16 with
+// its Fourier (column) index in the tensor-core order; the padding row and column are zero.
+// Block (group of 8 rows i, h), 128 threads: thread p owns Fourier column p and accumulates its 8
+// rows over r in fp32, in the same order as the CUDA-core path's readout matrix.
+__global__ void __launch_bounds__(128) readout_f16_kernel(const float* R, __half* Mb) {
+    const int h = blockIdx.y, i0 = 8 * blockIdx.x, p = threadIdx.x;
+    __shared__ float s_r[8][MA];
+    __shared__ float s_c[MA], s_s[MA];   // cos / sin of 2 pi x / m, x = 0 .. m - 1
+    for (int e = p; e < 8 * MA; e += 128) {
+        const int ii = e / MA, r = e - ii * MA;
+        s_r[ii][r] = (i0 + ii < MA) ? R[((size_t)h * MA + i0 + ii) * MA + r] : 0.f;
+    }
+    if (p < MA) {
+        float sv, cv;
+        sincospif((float)p * (2.f / 127.f), &sv, &cv);
+        s_c[p] = cv;
+        s_s[p] = sv;
+    }
+    __syncthreads();
+    float acc[8];
+#pragma unroll
+    for (int ii = 0; ii < 8; ++ii) acc[ii] = 0.f;
+    if (p == 0) {
+        for (int r = 0; r < MA; ++r)
+#pragma unroll
+            for (int ii = 0; ii < 8; ++ii) acc[ii] = fmaf(s_r[ii][r], INV_SQRT_M, acc[ii]);
+    } else if (p < MA) {
+        const int j = (p + 1) >> 1;
+        const float* tab = (p & 1) ? s_c : s_s;
+        int idx = 0;   // (j r) mod m
+        for (int r = 0; r < MA; ++r) {
+            const float phi = SQRT_2_OVER_M * tab[idx];
+#pragma unroll
+            for (int ii = 0; ii < 8; ++ii) acc[ii] = fmaf(s_r[ii][r], phi, acc[ii]);
+            idx += j;
+            if (idx >= MA) idx -= MA;
+        }
+    }
+#pragma unroll
+    for (int ii = 0; ii < 8; ++ii) {
+        const int i = i0 + ii;
+        Mb[((size_t)h * MS + i) * MS + tc_slot(p)] = __float2half_rn(i < MA ? acc[ii] : 0.f);
+    }
 }
 
 // Total log-decay of every segment (sum of its chunks' 128-token totals), as seg_state_tc
@@ -817,16 +855,16 @@ bool tc_rows_map(CUtensorMap* map, const void* base, unsigned long long rows, bo
     return make_tmap_bf16(map, base, 2, dims, str, box, f16);
 }
 
+cudaError_t launch_readout_f16(int H, const float* R, __half* Mb, cudaStream_t st) {
+    { LaunchScope ls_("readout_f16", st); readout_f16_kernel<<<dim3(MS / 8, H), 128, 0, st>>>(R, Mb); }
+    return cudaGetLastError();
+}
+
 cudaError_t launch_fwd_segment_states(const TcFwdArgs& a, const void* k, const void* v,
-                                      const float* Mf, cudaStream_t st) {
+                                      cudaStream_t st) {
     const Shape& s = a.s;
     CUtensorMap mk, mv;
     if (!tc_qkv_maps(s, nullptr, k, v, nullptr, &mk, &mv)) return cudaErrorInvalidValue;
-    const int n = s.H * 128 * 128;
-    {
-        LaunchScope ls_("m_to_f16", st);
-        m_to_f16_kernel<<<(n + 255) / 256, 256, 0, st>>>(Mf, const_cast<__half*>(a.Mb), s.H);
-    }
     const dim3 grid(s.B * s.H, a.nseg);   // heads fastest: CTAs that share token rows run together
     const int smA = 1024 + 12 * SEGC_DEFAULT * CT + 6 * TILE + 1024;
     auto kA = seg_state_tc<SEGC_DEFAULT, __half>;
@@ -836,19 +874,14 @@ cudaError_t launch_fwd_segment_states(const TcFwdArgs& a, const void* k, const v
     return cudaGetLastError();
 }
 
-cudaError_t launch_m_and_segment_decay(const TcFwdArgs& a, const float* Mf, cudaStream_t st) {
+cudaError_t launch_segment_decay(const TcFwdArgs& a, cudaStream_t st) {
     const Shape& s = a.s;
-    const int n = s.H * 128 * 128;
-    {
-        LaunchScope ls_("m_to_f16", st);
-        m_to_f16_kernel<<<(n + 255) / 256, 256, 0, st>>>(Mf, const_cast<__half*>(a.Mb), s.H);
-    }
     { LaunchScope ls_("tc_seg_decay", st); seg_decay_kernel<<<dim3(a.nseg, s.B * s.H), 32, 0, st>>>(a, SEGC_DEFAULT); }
     return cudaGetLastError();
 }
 
 cudaError_t launch_fwd_tc(const TcFwdArgs& a, const void* q, const void* k, const void* v,
-                          const float* Mf, cudaStream_t st) {
+                          cudaStream_t st) {
     const Shape& s = a.s;
     const unsigned long long BH = (unsigned long long)s.B * s.H;
     CUtensorMap mq, mk, mv, mm, msnap, mo;
@@ -860,7 +893,7 @@ cudaError_t launch_fwd_tc(const TcFwdArgs& a, const void* q, const void* k, cons
     if (!tc_rows_map(&msnap, a.snap ? (const void*)a.snap : (const void*)a.Mb,
                      a.snap ? BH * (s.T / CT) * 2 * 128 : (unsigned long long)s.H * 128, true))
         return cudaErrorInvalidValue;
-    cudaError_t e = launch_fwd_segment_states(a, k, v, Mf, st);
+    cudaError_t e = launch_fwd_segment_states(a, k, v, st);
     if (e != cudaSuccess) return e;
     const dim3 grid(s.B * s.H, a.nseg);   // heads fastest: CTAs that share token rows run together
     const int smC = 2048 + 7 * TILE + 1024;
