@@ -67,10 +67,12 @@ def test_fp32_config_parity():
 @pytest.mark.parametrize('cuda_cores', [False, True])
 @pytest.mark.parametrize('B,T,H,D,C', [(2, 384, 3, 128, 64), (1, 512, 2, 128, 128),
                                        (3, 256, 1, 64, 128), (1, 64, 1, 128, 64),
-                                       (1, 2304, 2, 128, 64)])
+                                       (1, 2304, 2, 128, 64), (1, 128, 2, 128, 64),
+                                       (2, 1152, 2, 128, 64)])
 def test_bf16_forward_small(B, T, H, D, C, cuda_cores):
     """Tensor-core kernels (bf16, d = 128, T a multiple of 128) and the CUDA-core kernels;
-    T = 2304 spans several 1024-token segments plus a partial one."""
+    T = 2304 spans several 1024-token segments plus a partial one, T = 128 is a single chunk
+    (its first chunk is its last), T = 1152 ends with a one-chunk segment."""
     inp = to_device(synth.make_inputs(B, T, H, D, seed=2))
     d = cyfa.dims(B, T, H, D, chunk=C, cuda_cores=cuda_cores)
     o, Ko, Vo, _ = gpu_forward(d, inp, want_state=True)
