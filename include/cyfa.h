@@ -197,6 +197,18 @@ int cyfa_check(void* stream);
 int cyfa_selftest_mma(int variant, const void* X, const void* Y, float* D, void* stream);
 
 /*
+ * cyfa_selftest_timeout -- self-check of failure detection; the paper has no counterpart.  One
+ * device thread waits on an mbarrier that nothing ever completes, with the same bounded wait the
+ * kernels use (which gives up after 2 s) but a limit of `limit_us` microseconds (1 .. 10^6).
+ * When the wait gives up the kernel records CYFA_ERR_TIMEOUT and returns normally, exactly as the
+ * chunk kernels do, so the CUDA context stays usable.  `elapsed_ns` (device pointer to one
+ * unsigned 64-bit value, or NULL) receives the time the wait took.  Synchronises `stream`.
+ * Returns CYFA_ERR_TIMEOUT when the wait expired (the expected outcome), CYFA_OK if it did not,
+ * CYFA_ERR_ARG for a limit out of range, CYFA_ERR_CUDA on a launch failure.
+ */
+int cyfa_selftest_timeout(unsigned int limit_us, unsigned long long* elapsed_ns, void* stream);
+
+/*
  * Launch accounting (host side, process-wide).  Every kernel launch of the library increments
  * a counter kept per kernel name.  With cyfa_stats_timing(1) each launch is also bracketed by
  * CUDA events recorded on its own stream; the elapsed times are summed per kernel when read.

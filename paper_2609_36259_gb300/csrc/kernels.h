@@ -97,6 +97,10 @@ bool make_tmap_bf16(CUtensorMap* map, const void* base, int rank, const unsigned
                     const unsigned long long* strides_bytes, const unsigned* box, bool f16 = false);
 cudaError_t launch_selftest_mma(int variant, const void* X, const void* Y, float* D,
                                 cudaStream_t st, int* host_err);
+// One thread waits on an mbarrier nothing arrives on with the kernels' own bounded wait, given a
+// limit of limit_us; *host_err = CYFA_ERR_TIMEOUT when it gave up (synchronises st).
+cudaError_t launch_timeout_probe(unsigned limit_us, unsigned long long* elapsed_ns,
+                                 cudaStream_t st, int* host_err);
 
 struct TcFwdArgs {
     Shape s;

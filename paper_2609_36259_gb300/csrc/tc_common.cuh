@@ -9,7 +9,8 @@
 //  * MN-major operand (M or N index contiguous): sub-tile j holds MN columns [64j, 64j+64); rows
 //    are the K index; 64-column blocks LBO = R * 128 B apart; 8-row K groups SBO = 1024 B apart;
 //    an MMA K-step (16 rows) advances the start address by 2048 B.
-// Every wait is bounded: on expiry the kernel records an error code and the caller bails out.
+// Every wait is bounded (WAIT_LIMIT_NS): on expiry the kernel records an error code and the
+// caller bails out.
 #pragma once
 
 #include <cuda.h>
@@ -23,7 +24,16 @@
 namespace cyfa {
 namespace tc {
 
-constexpr uint32_t SPIN_LIMIT = 1u << 26;   // ~ tens of ms of polling before giving up
+// A wait on an mbarrier gives up after this long (read from %globaltimer).  An unsatisfied
+// try_wait suspends the thread for about 3.75 us on GB300, so a poll count alone would be a poor
+// bound (2^26 polls were about 250 s); every kernel of the library finishes in milliseconds.
+constexpr unsigned long long WAIT_LIMIT_NS = 2000000000ull;   // 2 s
+
+__device__ __forceinline__ unsigned long long globaltimer_ns() {
+    unsigned long long t;
+    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+    return t;
+}
 
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
     return static_cast<uint32_t>(__cvta_generic_to_shared(p));
@@ -65,11 +75,20 @@ __device__ __forceinline__ bool mbar_test_wait(uint64_t* bar, uint32_t parity) {
         : "memory");
     return ok != 0;
 }
-// Bounded wait for the phase with the given parity; false if it never completed.
-__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity) {
-    for (uint32_t i = 0; i < SPIN_LIMIT; ++i)
+// Wait for the phase with the given parity, giving up after `limit_ns` nanoseconds; false if it
+// never completed.
+__device__ __forceinline__ bool mbar_wait_for(uint64_t* bar, uint32_t parity,
+                                              unsigned long long limit_ns) {
+    if (mbar_try_wait(bar, parity)) return true;
+    const unsigned long long t0 = globaltimer_ns();
+    for (;;) {
         if (mbar_try_wait(bar, parity)) return true;
-    return false;
+        if (globaltimer_ns() - t0 > limit_ns) return false;
+    }
+}
+// Bounded wait of the kernels (WAIT_LIMIT_NS).
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity) {
+    return mbar_wait_for(bar, parity, WAIT_LIMIT_NS);
 }
 
 // ---------------------------------------------------------------------------- fences

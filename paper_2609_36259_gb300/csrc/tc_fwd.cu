@@ -229,13 +229,14 @@ __global__ void __launch_bounds__(256) seg_scan_kernel(TcFwdArgs a) {
 enum { OB_QK, OB_V, OB_M, OB_MMA, OB_F1, OB_F5, OB_F6, OB_SU, OB_SR, OB_NX, OB_END, OB_ENDS, OB_N };
 constexpr int OUT_CHAIN = 512, OUT_THREADS = 640;
 
-// Bounded wait that also gives up once the other group has flagged an abort.
+// Bounded wait (WAIT_LIMIT_NS) that also gives up once the other group has flagged an abort.
 __device__ __forceinline__ bool mbar_wait_ab(uint64_t* bar, uint32_t parity, volatile int* abort_) {
-    for (uint32_t i = 0; i < SPIN_LIMIT; ++i) {
+    if (mbar_try_wait(bar, parity)) return true;
+    const unsigned long long t0 = globaltimer_ns();
+    for (;;) {
         if (mbar_try_wait(bar, parity)) return true;
-        if ((i & 255u) == 255u && *abort_) return false;
+        if (*abort_ || globaltimer_ns() - t0 > WAIT_LIMIT_NS) return false;
     }
-    return false;
 }
 __device__ __forceinline__ void named_sync(uint32_t id, uint32_t n) {
     asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(n) : "memory");

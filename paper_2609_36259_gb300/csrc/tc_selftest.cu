@@ -84,7 +84,43 @@ __global__ void __launch_bounds__(128) selftest_kernel(const __grid_constant__ C
     if (warp == 0) tmem_dealloc(taddr, 128);
 }
 
+// Expiry of a bounded wait: one thread waits on an mbarrier that nothing ever arrives on, with
+// the kernels' own wait (mbar_wait_for) given a limit of `limit_us`; when it gives up, the error
+// word is set and the kernel returns normally (no trap, no fault: the context stays usable).
+static __device__ int g_timeout_err;
+
+__global__ void timeout_probe_kernel(uint32_t limit_us, unsigned long long* elapsed_ns) {
+    using namespace tc;
+    __shared__ __align__(8) uint64_t bar;
+    if (threadIdx.x == 0) {
+        mbar_init(&bar, 1);
+        fence_mbar_init();
+        const unsigned long long t0 = globaltimer_ns();
+        const bool done = mbar_wait_for(&bar, 0, 1000ull * limit_us);
+        if (elapsed_ns) *elapsed_ns = globaltimer_ns() - t0;
+        if (!done) atomicExch(&g_timeout_err, CYFA_ERR_TIMEOUT);
+    }
+}
+
 }  // namespace
+
+cudaError_t launch_timeout_probe(unsigned limit_us, unsigned long long* elapsed_ns,
+                                 cudaStream_t st, int* host_err) {
+    int zero = 0;
+    cudaError_t e = cudaMemcpyToSymbolAsync(g_timeout_err, &zero, sizeof(int), 0,
+                                            cudaMemcpyHostToDevice, st);
+    if (e != cudaSuccess) return e;
+    {
+        LaunchScope ls_("selftest_timeout", st);
+        timeout_probe_kernel<<<1, 32, 0, st>>>(limit_us, elapsed_ns);
+    }
+    e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    e = cudaMemcpyFromSymbolAsync(host_err, g_timeout_err, sizeof(int), 0, cudaMemcpyDeviceToHost,
+                                  st);
+    if (e != cudaSuccess) return e;
+    return cudaStreamSynchronize(st);
+}
 
 cudaError_t launch_selftest_mma(int variant, const void* X, const void* Y, float* D,
                                 cudaStream_t st, int* host_err) {
@@ -121,6 +157,16 @@ extern "C" int cyfa_selftest_mma(int variant, const void* X, const void* Y, floa
     int err = 0;
     const cudaError_t e =
         cyfa::launch_selftest_mma(variant, X, Y, D, static_cast<cudaStream_t>(stream), &err);
+    if (e != cudaSuccess) return CYFA_ERR_CUDA;
+    return err ? CYFA_ERR_TIMEOUT : CYFA_OK;
+}
+
+extern "C" int cyfa_selftest_timeout(unsigned int limit_us, unsigned long long* elapsed_ns,
+                                     void* stream) {
+    if (limit_us == 0 || limit_us > 1000000u) return CYFA_ERR_ARG;
+    int err = 0;
+    const cudaError_t e =
+        cyfa::launch_timeout_probe(limit_us, elapsed_ns, static_cast<cudaStream_t>(stream), &err);
     if (e != cudaSuccess) return CYFA_ERR_CUDA;
     return err ? CYFA_ERR_TIMEOUT : CYFA_OK;
 }

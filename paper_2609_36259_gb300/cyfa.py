@@ -22,7 +22,7 @@ CYFA_WS_PREPARE, CYFA_WS_FWD, CYFA_WS_BWD = 0, 1, 2
 EXPORTS = ('cyfa_version', 'cyfa_error_string', 'cyfa_workspace_size', 'cyfa_prepare',
            'cyfa_chunk_fwd', 'cyfa_chunk_bwd', 'cyfa_step', 'cyfa_check', 'cyfa_stats_reset',
            'cyfa_stats_timing', 'cyfa_stats_get', 'cyfa_prepare_noalloc',
-           'cyfa_selftest_mma', 'cyfa_saved_size')
+           'cyfa_selftest_mma', 'cyfa_saved_size', 'cyfa_selftest_timeout')
 
 
 class CyfaError(RuntimeError):
@@ -71,6 +71,7 @@ def load(path=LIB_PATH):
     lib.cyfa_step.argtypes = [P] + [_VP] * 13
     lib.cyfa_check.argtypes = [_VP]
     lib.cyfa_selftest_mma.argtypes = [ctypes.c_int, _VP, _VP, _VP, _VP]
+    lib.cyfa_selftest_timeout.argtypes = [ctypes.c_uint, _VP, _VP]
     lib.cyfa_prepare_noalloc.argtypes = [P] + [_VP] * 9 + [_VP]
     lib.cyfa_stats_timing.argtypes = [ctypes.c_int]
     lib.cyfa_stats_get.argtypes = [ctypes.c_int, ctypes.c_char_p, ctypes.c_int,
@@ -173,6 +174,12 @@ def cyfa_check(stream=None):
 
 def cyfa_selftest_mma(variant, X, Y, D, stream=None):
     _ok(load().cyfa_selftest_mma(variant, _ptr(X), _ptr(Y), _ptr(D), _stream(stream)))
+
+
+def cyfa_selftest_timeout(limit_us, elapsed_ns=None, stream=None):
+    """Run the bounded-wait expiry self-check with a wait limit of limit_us microseconds;
+    returns the library's status code (not raised: CYFA_ERR_TIMEOUT is the expected outcome)."""
+    return load().cyfa_selftest_timeout(limit_us, _ptr(elapsed_ns), _stream(stream))
 
 
 def cyfa_stats_reset():
