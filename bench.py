@@ -185,6 +185,23 @@ def oracle_baseline(T_sample, H_full, cores=None):
     return value, cores, sample, wall, max(per)
 
 
+# ------------------------------------------------------------------------- multi-rank
+def job_step_ms(ms, dist=None, device=None):
+    """The job's step time: the max over ranks of each rank's own step time (every rank must call
+    this; a rank on its own returns its time)."""
+    if dist is None:
+        return ms
+    import torch
+    t = torch.tensor([ms], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_tokens_per_s(tokens_per_rank, world, ms):
+    """Whole-job throughput: every rank processes its own batch (weak scaling)."""
+    return tokens_per_rank * world / (ms / 1e3)
+
+
 # --------------------------------------------------------------------------------- ours
 def run_ours(args):
     import numpy as np
@@ -265,12 +282,8 @@ def run_ours(args):
     ms = e0.elapsed_time(e1) / args.steps
     stats = cyfa.cyfa_stats_get()
     cyfa.cyfa_stats_timing(False)
-    if dist:
-        t = torch.tensor([ms], dtype=torch.float64, device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms = float(t.item())
-    tokens = B * T * world
-    value = tokens / (ms / 1e3)
+    ms = job_step_ms(ms, dist, dev)
+    value = job_tokens_per_s(B * T, world, ms)
     launches = sum(n for n, _ in stats.values())
 
     # per-kernel times and the forward / backward split
