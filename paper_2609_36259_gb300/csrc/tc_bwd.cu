@@ -1124,9 +1124,14 @@ __global__ void __launch_bounds__(512, 1) bwd_chunk2_tc(const __grid_constant__ 
             bulk_wait_read_all();
             mma_commit(&bars[4]);
         }
-        // while it runs: the write vectors and their copies scaled by gamma^C / gamma^s
-        write_vector_q<__half>(T_A, row, hf, u, lam, beta);
-        write_vector_q<__half>(T_AS, row, hf, u, lam, beta * fw);
+        {   // while it runs: the write vectors and their copies scaled by gamma^C / gamma^s
+            float x[32];
+            write_vector_q_vals(x, hf, u, lam, beta);
+            store_q<__half>(T_A, row, c0, x);
+#pragma unroll
+            for (int i = 0; i < 32; ++i) x[i] *= fw;
+            store_q<__half>(T_AS, row, c0, x);
+        }
         wait_mma();
         {   // P4 = (dO V^T) o Gamma ; V -> V-> (rows scaled by gamma^C / gamma^s)
             float x[32];

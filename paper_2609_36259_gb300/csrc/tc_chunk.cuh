@@ -144,24 +144,6 @@ __device__ __forceinline__ void bf16_to_f16_half(uint8_t* tile, int r, int hf) {
     }
 }
 
-// x <- U(sign lam) x on one column half (tensor-core row order); DC kept, padding zeroed.
-template <int SIGN>
-__device__ __forceinline__ void rotate_half(float (&x)[64], int hf, float lam) {
-    HalfAngles ang(lam, hf);
-    const float dc = x[31];
-#pragma unroll
-    for (int jj = 0; jj < 32; ++jj) {
-        if (jj > 0) ang.step(jj);
-        const float c = ang.c, s = SIGN * ang.s;
-        const float xc = x[jj], xs = x[jj + 32];
-        x[jj] = c * xc - s * xs;
-        x[jj + 32] = s * xc + c * xs;
-    }
-    if (hf == 1) {
-        x[31] = dc;
-        x[63] = 0.f;
-    }
-}
 
 __device__ __forceinline__ void tmem_ld64(uint32_t taddr, float (&x)[64]) {
     float v[32];
@@ -290,20 +272,8 @@ __device__ __forceinline__ void scale_q(uint8_t* tile, int r, int c0, float w) {
     for (int i = 0; i < 32; ++i) x[i] *= w;
     store_q<__half>(tile, r, c0, x);
 }
-// The thread's 32 values -> a plain row-major 16-bit row at dst (columns c0.. and c0 + 32..), as
-// two 32-byte stores (dst + c0 is 32-byte aligned: rows of 128 16-bit values, c0 a multiple of 16).
-template <typename OT>
-__device__ __forceinline__ void store_global_q(OT* dst, int c0, const float (&x)[32]) {
-#pragma unroll
-    for (int hb = 0; hb < 2; ++hb) {
-        uint32_t w[8];
-#pragma unroll
-        for (int k = 0; k < 8; ++k) w[k] = pack2<OT>(x[16 * hb + 2 * k], x[16 * hb + 2 * k + 1]);
-        st_global_v8(dst + c0 + 32 * hb, w);
-    }
-}
 
-// 16 values (8 at column col, 8 at col + 32) -> row r of a swizzled 16-bit tile / a plain row.
+// 16 values (8 at column col, 8 at col + 32) -> row r of a swizzled 16-bit tile.
 template <typename OT>
 __device__ __forceinline__ void store8x2(uint8_t* tile, int r, int col, const float (&x)[16]) {
 #pragma unroll
@@ -315,19 +285,6 @@ __device__ __forceinline__ void store8x2(uint8_t* tile, int r, int col, const fl
         w.z = pack2<OT>(v[4], v[5]);
         w.w = pack2<OT>(v[6], v[7]);
         *reinterpret_cast<uint4*>(tile + swz_off(r, col + 32 * k, 128)) = w;
-    }
-}
-template <typename OT>
-__device__ __forceinline__ void store8x2_global(OT* rowp, int col, const float (&x)[16]) {
-#pragma unroll
-    for (int k = 0; k < 2; ++k) {
-        const float* v = x + 8 * k;
-        uint4 w;
-        w.x = pack2<OT>(v[0], v[1]);
-        w.y = pack2<OT>(v[2], v[3]);
-        w.z = pack2<OT>(v[4], v[5]);
-        w.w = pack2<OT>(v[6], v[7]);
-        *reinterpret_cast<uint4*>(rowp + col + 32 * k) = w;
     }
 }
 
