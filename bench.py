@@ -93,7 +93,9 @@ class ClockSampler:
     def __init__(self, device_index):
         self.idx = device_index
         self.proc = None
-        self.path = os.path.join(ROOT, 'gpurun_out', 'bench_clocks_%d.csv' % device_index)
+        import tempfile
+        self.path = os.path.join(tempfile.gettempdir(),
+                                 'cyfa_bench_clocks_%d_%d.csv' % (os.getpid(), device_index))
 
     def start(self):
         try:
@@ -129,6 +131,10 @@ class ClockSampler:
             for nm, val in zip(names, parts[5:9]):
                 if val.lower() == 'active':
                     reasons.add(nm)
+        try:
+            os.remove(self.path)
+        except OSError:
+            pass
         if not sm:
             return None
         sm.sort()
