@@ -630,7 +630,13 @@ __global__ void __launch_bounds__(512, 1) bwd_chunk1_tc(const __grid_constant__ 
             mma_commit(&bars[2]);
         }
         wait_mma();
-        if (issuer() && it + 1 < i1) issue_first(it + 1, T_A, T_KB, (it + 1) / nct % s.H != h);
+        if (issuer() && it + 1 < i1) {
+            issue_first(it + 1, T_A, T_KB, (it + 1) / nct % s.H != h);
+            // the next item's V into L2: its load waits for this item's last product
+            const int nbh = (it + 1) / nct, ncg = (it + 1) - nbh * nct, nb = nbh / s.H;
+            tma_prefetch_3d(&tv, 0, nbh - nb * s.H, nb * s.T + ncg * CT);
+            tma_prefetch_3d(&tv, 64, nbh - nb * s.H, nb * s.T + ncg * CT);
+        }
         if (it + 1 < i1) stage_gates(it + 1);   // the next item's gates, an epilogue ahead
         {   // P3 = s (dO' A^T) o Gamma
             float x[32];
