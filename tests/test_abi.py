@@ -86,3 +86,10 @@ def test_saved_size(lib):
     assert cyfa.cyfa_saved_size(cyfa.dims(B, T, H, 128, cuda_cores=True)) == 0
     assert cyfa.cyfa_saved_size(cyfa.dims(B, T, H, 64)) == 0
     assert cyfa.cyfa_saved_size(cyfa.dims(B, T, H, 128, dtype=torch.float32)) == 0
+
+
+def test_timeout_selftest_rejects_bad_limits_on_host(lib):
+    """The failure-detection self-check refuses a wait limit outside 1 us .. 1 s before any CUDA
+    call (its GPU behaviour is tested in test_gpu_failure_detection.py)."""
+    for limit in (0, 1000001, 2 ** 32 - 1):
+        assert lib.cyfa_selftest_timeout(limit, None, None) == cyfa.CYFA_ERR_ARG
