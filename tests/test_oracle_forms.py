@@ -151,3 +151,21 @@ def test_clock_is_order_preserving():
         for j in range(i + 1, 50, 5):
             gap = lam[j] - lam[i]
             assert 0 < gap < j - i
+
+
+@pytest.mark.parametrize('m', [7, 127])
+def test_chunk_form_over_128_token_chunks(m):
+    """App. B at the blocking of the tensor-core path: two full 128-token chunks and a ragged
+    tail, with slow decay (A = 0.02) so the state carried across chunk boundaries matters."""
+    q, k, v, delta, alpha, beta, R = _case(1, 300, 4, m, seed=300 + m, A=0.02)
+    s = 0.7
+    o_rel = F.relative_time(q, k, v, delta, alpha, beta, R, s)[0]
+    o_abs, Kb, Vb, _ = F.absolute_clock(q, k, v, delta, alpha, beta, R, s)
+    o_ch, Kc, Vc = F.chunkwise(q, k, v, delta, alpha, beta, R, s, 128)
+    np.testing.assert_allclose(o_ch, o_rel, atol=1e-10, rtol=0)
+    np.testing.assert_allclose(o_ch, o_abs, atol=1e-10, rtol=0)
+    np.testing.assert_allclose(Kc, Kb, atol=1e-10, rtol=0)
+    np.testing.assert_allclose(Vc, Vb, atol=1e-10, rtol=0)
+    # the state carried into the last chunk still weighs: its decay over the first two chunks
+    decay = np.prod(alpha[0, :256])
+    assert decay > 1e-3, decay
