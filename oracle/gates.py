@@ -6,8 +6,12 @@
 * beta_t  = sigmoid(beta_logit_t)                     Sec. 3.1 states only beta in (0,1);
   the sigmoid is this library's reading (the paper names no activation).
 
-Pins: lambda is checked against the closed form of a constant-rate clock and
-Prop. 5 (order preservation); the activations are elementwise definitions.
+Pins (tests/test_oracle_gates.py): sigmoid(0) = 1/2, the symmetry sigmoid(x) +
+sigmoid(-x) = 1, the exact rationals sigmoid(+-ln n) and the logistic definition at
+sample points; softplus(0) = ln 2, softplus(x) - softplus(-x) = x, its limits and
+its derivative (sigmoid); forget_gate(0, A) = 2^-A, its limits 1 and 0, its range
+(0, 1] and monotonicity, and additivity in A; write_strength in (0, 1); lambda
+against the closed form of a constant-rate clock and Prop. 5 (order preservation).
 """
 import numpy as np
 
