@@ -30,7 +30,8 @@
  *   stream            a cudaStream_t passed as void*; every call is asynchronous on it.
  *
  * Shapes supported: m = 127 (128 storage rows), dk = dv in {64, 128}, chunk in {64, 128},
- * T a positive multiple of chunk (for cyfa_prepare / cyfa_chunk_fwd / cyfa_chunk_bwd).
+ * T a positive multiple of chunk (for cyfa_prepare / cyfa_chunk_fwd / cyfa_chunk_bwd),
+ * B * H <= 65535.
  *
  * Errors: every entry point returns CYFA_OK (0) or a negative code.  Argument errors are
  * found on the host before anything is launched.  CYFA_ERR_TIMEOUT is raised on the device
@@ -112,9 +113,12 @@ int cyfa_prepare(const cyfa_dims_t* dims, const float* clock_logit, const float*
  * the process exits), which limits B * H * ceil(T / 1024) to 32768; larger shapes return
  * CYFA_ERR_WORKSPACE before anything is launched.  The first call made on a device looks up
  * the array's device address (cudaGetSymbolAddress) with that device current; make that first
- * call before any stream capture.  All calls share the array and each call overwrites it
- * entirely before reading it, so nothing needs clearing, but calls that may run concurrently
- * on the GPU (on different streams, or different host threads) race on it and must not overlap.
+ * call before any stream capture.  The looked-up address is kept for the life of the process:
+ * do not use this entry point after a cudaDeviceReset (or any other reset of the device's
+ * primary context) in the same process, since the kept address may then be stale.  All calls
+ * share the array and each call overwrites it entirely before reading it, so nothing needs
+ * clearing, but calls that may run concurrently on the GPU (on different streams, or different
+ * host threads) race on it and must not overlap.  Argument errors are those of cyfa_prepare.
  */
 int cyfa_prepare_noalloc(const cyfa_dims_t* dims, const float* clock_logit,
                          const float* decay_logit, const float* beta_logit, const float* A,

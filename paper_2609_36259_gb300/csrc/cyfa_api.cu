@@ -27,19 +27,27 @@ struct Carver {
 
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
-int check_dims(const cyfa_dims_t* d, bool need_T) {
+}  // namespace
+
+// The (b, h) sequences go on gridDim.y of the per-sequence launches, whose limit is 65535.
+constexpr long long kMaxSequences = 65535;
+
+int cyfa::check_dims(const cyfa_dims_t* d, bool need_T) {
     if (!d) return CYFA_ERR_ARG;
     if (d->B <= 0 || d->H <= 0 || d->dk <= 0 || d->dv <= 0 || (need_T && d->T <= 0))
         return CYFA_ERR_ARG;
+    if (d->dtype != CYFA_DTYPE_BF16 && d->dtype != CYFA_DTYPE_FP32) return CYFA_ERR_ARG;
     if (d->m != 127) return CYFA_ERR_SHAPE;
     if (d->dk != d->dv || (d->dk != 64 && d->dk != 128)) return CYFA_ERR_SHAPE;
-    if (d->dtype != CYFA_DTYPE_BF16 && d->dtype != CYFA_DTYPE_FP32) return CYFA_ERR_ARG;
+    if ((long long)d->B * d->H > kMaxSequences) return CYFA_ERR_SHAPE;
     if (need_T) {
         if (d->chunk != 64 && d->chunk != 128) return CYFA_ERR_SHAPE;
         if (d->T % d->chunk != 0) return CYFA_ERR_SHAPE;
     }
     return CYFA_OK;
 }
+
+namespace {
 
 Shape shape_of(const cyfa_dims_t* d) {
     Shape s;

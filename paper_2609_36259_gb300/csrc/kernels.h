@@ -7,7 +7,13 @@
 #include <cuda_runtime.h>
 #include <stddef.h>
 
+struct cyfa_dims;
+
 namespace cyfa {
+
+// Host-side check of a dims struct shared by every entry point: CYFA_OK, or the error code the
+// entry point returns before launching anything (need_T: T and chunk are used by the call).
+int check_dims(const ::cyfa_dims* d, bool need_T);
 
 // Counts one launch of the named kernel and, when timing is on (cyfa_stats_timing), brackets it
 // with CUDA events on its stream.  Construct immediately before the <<<>>> launch.

@@ -183,10 +183,8 @@ extern "C" int cyfa_prepare_noalloc(const cyfa_dims_t* dims, const float* clock_
                                     const float* A, const double* lambda0, float* lam_mod,
                                     float* g_cum, float* beta, double* lambda_end, void* stream) {
     using namespace cyfa;
-    if (!dims || dims->B <= 0 || dims->T <= 0 || dims->H <= 0) return CYFA_ERR_ARG;
-    if (dims->m != 127 || dims->dk != dims->dv || (dims->dk != 64 && dims->dk != 128) ||
-        (dims->chunk != 64 && dims->chunk != 128) || dims->T % dims->chunk != 0)
-        return CYFA_ERR_SHAPE;
+    const int rc = check_dims(dims, true);   // the same argument checks as cyfa_prepare
+    if (rc) return rc;
     if (!clock_logit || !decay_logit || !beta_logit || !A || !lam_mod || !g_cum || !beta)
         return CYFA_ERR_ARG;
     const long long nseg = (dims->T + PREP_SEG - 1) / PREP_SEG;

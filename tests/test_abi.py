@@ -55,7 +55,8 @@ def test_workspace_sizes(lib):
 
 @pytest.mark.parametrize('field,value,code', [
     ('m', 63, cyfa.CYFA_ERR_SHAPE), ('dk', 96, cyfa.CYFA_ERR_SHAPE), ('chunk', 32, cyfa.CYFA_ERR_SHAPE),
-    ('T', 100, cyfa.CYFA_ERR_SHAPE), ('B', 0, cyfa.CYFA_ERR_ARG), ('dtype', 7, cyfa.CYFA_ERR_ARG)])
+    ('T', 100, cyfa.CYFA_ERR_SHAPE), ('B', 0, cyfa.CYFA_ERR_ARG), ('dtype', 7, cyfa.CYFA_ERR_ARG),
+    ('B', 65536, cyfa.CYFA_ERR_SHAPE)])
 def test_bad_dims_rejected_on_host(lib, field, value, code):
     d = cyfa.dims(1, 128, 1, 128)
     setattr(d, field, value)
@@ -93,3 +94,16 @@ def test_timeout_selftest_rejects_bad_limits_on_host(lib):
     call (its GPU behaviour is tested in test_gpu_failure_detection.py)."""
     for limit in (0, 1000001, 2 ** 32 - 1):
         assert lib.cyfa_selftest_timeout(limit, None, None) == cyfa.CYFA_ERR_ARG
+
+
+@pytest.mark.parametrize('field,value,code', [
+    ('dtype', 7, cyfa.CYFA_ERR_ARG), ('m', 63, cyfa.CYFA_ERR_SHAPE), ('T', 100, cyfa.CYFA_ERR_SHAPE),
+    ('B', 65536, cyfa.CYFA_ERR_SHAPE)])
+def test_noalloc_prepare_checks_dims_like_prepare(lib, field, value, code):
+    """cyfa_prepare_noalloc applies cyfa_prepare's argument checks, before any CUDA call."""
+    d = cyfa.dims(1, 128, 1, 128)
+    setattr(d, field, value)
+    good = ctypes.c_void_p(0x1000)      # never dereferenced: rejected before any launch
+    args = [good] * 4 + [None] + [good] * 3 + [None, None]
+    assert lib.cyfa_prepare_noalloc(ctypes.byref(d), *args) == code
+    assert lib.cyfa_prepare(ctypes.byref(d), *args[:9], good, 1 << 30, None) == code
