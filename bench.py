@@ -32,8 +32,10 @@ LAYER = dict(B=2, T=32768, H=16, d=128)          # 1.4B-shaped layer
 DECODE = dict(B=256, H=16, d=128, prefill=2048)   # decode workload
 MS = 128
 
-# Algorithmic flops per (token, head) of each kernel (d = 128, m* = 128, chunk C): the
-# products each kernel's equations call for, counted 2 per multiply-add, full C x C blocks.
+# Issued flops per (token, head) of each kernel (d = 128, m* = 128, chunk C): the products each
+# kernel's equations call for, counted 2 per multiply-add, full C x C blocks.  On the CUDA-core
+# kernels these are also their share of the work; the tensor-core kernels are charged by the
+# counting rule below instead.
 def kernel_flops_per_token_head(name, C, d=128, ms=MS):
     table = {
         'fwd_state': 4 * d * ms,                                    # Kbar, Vbar updates
@@ -44,29 +46,59 @@ def kernel_flops_per_token_head(name, C, d=128, ms=MS):
                       + (2 * C * ms + 2 * C * d + 2 * d * ms),
         'bwd_adjoint': 4 * d * ms,
         'bwd_intra2': 4 * (2 * C * ms + 2 * C * d + 2 * d * ms),
-        # tensor-core kernels (128-token chunks; every product a 128 x 128 x 128 tcgen05 GEMM)
-        'tc_seg_state': 4 * d * ms,
-        'tc_seg_out': 4 * 128 * d + 4 * 128 * ms + 8 * d * ms + 4 * ms * ms,
-        'tc_snap_fwd': 4 * d * ms,
-        'tc_bwd_chunk1': 13 * 2 * 128 * 128,
-        'tc_adj_segment': 4 * d * ms,
-        'tc_snap_adj': 4 * d * ms,
-        'tc_bwd_chunk2': 12 * 2 * 128 * 128,
-        'tc_dm_reduce': 2 * 2 * 128 * 128,                         # dl z^T + p dy^T for dR
     }
+    if name in TC_PRODUCTS:
+        return TC_PRODUCTS[name] * TC_PRODUCT_FLOPS
     return table.get(name)
 
 
-TENSOR_KERNELS = ('tc_seg_state', 'tc_seg_out', 'tc_snap_fwd', 'tc_bwd_chunk1', 'tc_adj_segment',
-                  'tc_snap_adj', 'tc_bwd_chunk2', 'tc_dm_reduce')
+# Tensor-core kernels: 128 x 128 x 128 products (an N = 256 product counts as two) each issues
+# per 128-token chunk, and the flops one such product per chunk costs per (token, head).
+TC_PRODUCTS = {'tc_seg_state': 2, 'tc_seg_out': 10, 'tc_snap_fwd': 2, 'tc_bwd_chunk1': 13,
+               'tc_adj_segment': 2, 'tc_snap_adj': 2, 'tc_bwd_chunk2': 12, 'tc_dm_reduce': 2}
+TC_PRODUCT_FLOPS = 2 * 128 * 128 * 128 // 128
+TENSOR_KERNELS = tuple(TC_PRODUCTS)
+FWD_TC = ('tc_seg_state', 'tc_seg_out')      # launched once per step by cyfa_chunk_fwd
 
 
 def operator_flops_per_token_head(C, d=128, ms=MS):
-    """Forward count of the chunk equations (state updates, intra-chunk, inter-chunk, middle)."""
+    """Forward count of the chunk equations (state updates, intra-chunk, inter-chunk, middle):
+    key pass 2Cd + 2Cm* + 4dm*, middle 4m*^2, value pass 2Cm* + 2Cd + 4m*d (262,144 at C = 64);
+    the backward counts as twice the forward."""
     key = 2 * C * d + 2 * C * ms + 4 * d * ms
     middle = 4 * ms * ms
     value = 2 * C * ms + 2 * C * d + 4 * ms * d
     return key + middle + value
+
+
+def tc_algorithmic_shares(launches_per_step, C=64):
+    """Algorithmic flops per (token, head) charged to each tensor-core kernel per launch.
+
+    Rule: the forward's algorithmic count (operator_flops_per_token_head at the caller's chunk C)
+    is split over the forward's tensor-core launches, and the backward's (twice the forward) over
+    the backward's, in proportion to the 128^3 products each launch issues.  Recomputation and the
+    masked halves of causal blocks are therefore not credited: a kernel's share is what the
+    operator's equations need of it, not what it issues."""
+    fwd_alg = operator_flops_per_token_head(C)
+    bwd_alg = 2 * fwd_alg
+    fwd_issued, bwd_issued = {}, {}
+    for k, n in launches_per_step.items():
+        if k not in TC_PRODUCTS:
+            continue
+        nf = 1 if k in FWD_TC else 0               # the forward's own launch of this kernel
+        if nf:
+            fwd_issued[k] = TC_PRODUCTS[k]
+        if n - nf > 0:
+            bwd_issued[k] = TC_PRODUCTS[k] * (n - nf)
+    tf, tb = sum(fwd_issued.values()), sum(bwd_issued.values())
+    share = {}
+    for k, n in launches_per_step.items():
+        if k not in TC_PRODUCTS:
+            continue
+        total = (fwd_alg * fwd_issued.get(k, 0) / tf if tf else 0.0) + \
+                (bwd_alg * bwd_issued.get(k, 0) / tb if tb else 0.0)
+        share[k] = total / n                         # per launch
+    return share, tf * TC_PRODUCT_FLOPS, tb * TC_PRODUCT_FLOPS
 
 
 def load_peaks():
@@ -160,9 +192,10 @@ def _oracle_warm(_):
     return 0
 
 
-def oracle_baseline(T_sample, H_full, cores=None):
-    """Time the oracle on `cores` (b, h) sequences of T_sample tokens of the layer's shape,
-    one process per core; returns (tokens/s of the full layer, cores, sample text, seconds)."""
+def oracle_baseline(T_sample, H_full, cores=None, reps=1):
+    """Time the oracle on `cores` (b, h) sequences of T_sample tokens of the layer's shape, one
+    process per core, `reps` times over; returns (tokens/s of the full layer, cores, sample text,
+    seconds per rep, slowest sequence)."""
     import multiprocessing as mp
     import numpy as np
     import torch
@@ -182,13 +215,25 @@ def oracle_baseline(T_sample, H_full, cores=None):
     with ctx.Pool(cores) as pool:
         pool.map(_oracle_warm, range(cores))          # start the workers and import the oracle
         t0 = time.perf_counter()
-        per = pool.map(_oracle_pair_worker, jobs)
-        wall = time.perf_counter() - t0
+        for _ in range(reps):
+            per = pool.map(_oracle_pair_worker, jobs)
+        wall = (time.perf_counter() - t0) / reps
     token_heads = cores * T_sample
     value = token_heads / H_full / wall
-    sample = ('%d (b,h) sequences x %d tokens, fwd+bwd, d=128, m=127, one process per core; '
-              'tokens/s = token-heads / H(=%d) / wall' % (cores, T_sample, H_full))
+    sample = ('%d (b,h) sequences x %d tokens of the layer, fwd+bwd, d=128, m=127, one process '
+              'per core; tokens/s = token-heads / H(=%d) / wall' % (cores, T_sample, H_full))
     return value, cores, sample, wall, max(per)
+
+
+def workload_config(world, C, with_dR):
+    """The workload both arms run (one line of each names the same one)."""
+    B, T, H, D = LAYER['B'], LAYER['T'], LAYER['H'], LAYER['d']
+    return {'workload': 'cyfa-1.4B-layer prepare+fwd+bwd', 'model': 'CyFA core operator',
+            'B': B, 'T': T, 'H': H, 'dk': D, 'dv': D, 'm': 127, 'm_store': MS, 'chunk': C,
+            'io_dtype': 'bf16',
+            'grads': 'q, k, v, clock, decay, beta logits, A' + (', R' if with_dR else ''),
+            'global_batch': B * world, 'seq_len': T, 'parallelism': 'dp%d' % world,
+            'l2': 'inputs larger than L2 (q,k,v,dO %.0f MB)' % (4 * B * T * H * D * 2 / 1e6)}
 
 
 # ------------------------------------------------------------------------- multi-rank
@@ -230,9 +275,11 @@ def run_ours(args):
     # CPU baseline first: its process pool is spawned before any GPU work of this process
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        v, cores, sample, wall, _ = oracle_baseline(args.cpu_tokens, LAYER['H'])
+        v, cores, sample, wall, _ = oracle_baseline(args.oracle_tokens, LAYER['H'],
+                                                    reps=args.cpu_reps)
         cpu = {'value': v, 'unit': 'tokens/s', 'cores': cores, 'kind': 'oracle',
-               'sample': sample, 'seconds': round(wall, 2)}
+               'sample': sample + ', mean of %d repetitions' % args.cpu_reps,
+               'seconds': round(wall * args.cpu_reps, 2)}
 
     B, T, H, D, C = LAYER['B'], LAYER['T'], LAYER['H'], LAYER['d'], args.chunk
     d = cyfa.dims(B, T, H, D, chunk=C, cuda_cores=args.cuda_cores)
@@ -306,31 +353,48 @@ def run_ours(args):
     prep_ms = sum(stats[k][1] for k in stats if k.startswith('prep')) / args.steps
     bwd_ms = (sum(stats[k][1] for k in stats if not k.startswith('prep')) / args.steps) - fwd_ms
     token_heads = B * T * H
-    op_flops = operator_flops_per_token_head(64) * token_heads      # counting rule at C = 64
+    op_flops = operator_flops_per_token_head(C) * token_heads      # counting rule at the chunk C
+    step_ms_kernels = fwd_ms + bwd_ms + prep_ms
     fwd = {'ms': fwd_ms, 'tokens_per_s': B * T / (fwd_ms / 1e3) if fwd_ms else None,
-           'tflops_rule_c64': op_flops / (fwd_ms / 1e3) / 1e12 if fwd_ms else None}
-    fwd['frac_bf16_peak'] = fwd['tflops_rule_c64'] / peaks['bf16'] if fwd_ms else None
+           'tflops_rule': op_flops / (fwd_ms / 1e3) / 1e12 if fwd_ms else None}
     bwd = {'ms': bwd_ms, 'tokens_per_s': B * T / (bwd_ms / 1e3) if bwd_ms else None,
-           'tflops_rule_2x_fwd': 2 * op_flops / (bwd_ms / 1e3) / 1e12 if bwd_ms else None}
+           'tflops_rule': 2 * op_flops / (bwd_ms / 1e3) / 1e12 if bwd_ms else None}
+    for ph in (fwd, bwd):
+        ph['frac_bf16_peak'] = ph['tflops_rule'] / peaks['bf16'] if ph['tflops_rule'] else None
+    step_tf = (3 * op_flops if not args.no_bwd else op_flops) / (ms / 1e3) / 1e12
+    tensor_frac = {'rule': 'fwd %d, bwd 2x fwd flops per token-head (chunk %d); '
+                           'of the measured bf16 burst peak %.1f TFLOP/s'
+                           % (operator_flops_per_token_head(C), C, peaks['bf16']),
+                   'fwd': fwd['frac_bf16_peak'], 'bwd': bwd['frac_bf16_peak'],
+                   'step': step_tf / peaks['bf16'], 'step_tflops': step_tf}
 
-    # roofline of every chunk kernel, and of the dominant one
+    # roofline of every kernel, and of the dominant one.  Tensor-core kernels are charged their
+    # share of the counting rule (tc_algorithmic_shares) against the bf16 burst peak: the timed
+    # region is a sub-second run of millisecond steps, not a seconds-long loop under the power cap.
+    per_step = {k: n / args.steps for k, (n, _) in stats.items()}
+    shares, _, _ = tc_algorithmic_shares(per_step, C)
     def roofline_of(name):
         n_k, t_k = stats[name]
-        C_k = 64 if name.startswith('bwd') or name == 'state_pass' else C
-        fl = kernel_flops_per_token_head(name, C_k)
-        if fl is None or n_k == 0 or t_k <= 0:
+        if n_k == 0 or t_k <= 0:
             return None
-        achieved = fl * token_heads / (t_k / n_k / 1e3) / 1e12
         if name in TENSOR_KERNELS:
-            peak, bound = peaks['bf16_sus'], 'tensor'
-            src = '%s bf16 sustained (kernel timed inside the step)' % peaks['src']
+            fl = shares.get(name)
+            issued = kernel_flops_per_token_head(name, C) * token_heads
+            peak, bound = peaks['bf16'], 'tensor'
+            src = '%s bf16 burst (fp16 operands: the same tensor rate)' % peaks['src']
         else:
+            C_k = 64 if name.startswith('bwd') or name == 'state_pass' else C
+            fl = kernel_flops_per_token_head(name, C_k)
+            issued = None
             peak, bound = fp32_alu_peak_tflops(peaks['sm_max_mhz']), 'alu'
             src = 'fp32 FMA: 152 SMs x 128 lanes x 2 x %.0f MHz' % peaks['sm_max_mhz']
+        if fl is None:
+            return None
+        achieved = fl * token_heads / (t_k / n_k / 1e3) / 1e12
         r = {'kernel': name, 'bound': bound, 'achieved': round(achieved, 3),
              'peak': round(peak, 2), 'unit': 'TFLOP/s', 'frac': round(achieved / peak, 4),
              'traffic': load_traffic(name), 'flops_per_launch': fl * token_heads,
-             'ms_per_launch': t_k / n_k, 'peak_source': src}
+             'issued_flops': issued, 'ms_per_launch': t_k / n_k, 'peak_source': src}
         return r
     rooflines = {k: roofline_of(k) for k in stats}
     rooflines = {k: v for k, v in rooflines.items() if v is not None}
@@ -354,18 +418,14 @@ def run_ours(args):
         'higher_is_better': True, 'scaling': 'weak', 'vs_baseline': None,
         'dtype': 'fp16' if tc_path else 'fp32',
         'data': 'synthetic',
-        'config': {'workload': 'cyfa-1.4B-layer prepare+fwd+bwd', 'model': 'CyFA core operator',
-                   'B': B, 'T': T, 'H': H, 'dk': D, 'dv': D, 'm': 127, 'm_store': MS,
-                   'chunk': 128 if tc_path else C, 'io_dtype': 'bf16',
-                   'arithmetic': ('tcgen05 fp16 operands, fp32 accumulate' if tc_path
-                                  else 'fp32 CUDA cores'),
-                   'saved_states': saved is not None,
-                   'grads': 'q, k, v, clock, decay, beta logits, A' + (', R' if dR is not None else ''),
-                   'global_batch': B * world, 'seq_len': T,
-                   'parallelism': 'dp%d' % world,
-                   'l2': 'inputs larger than L2 (q,k,v,dO %.0f MB)' % (4 * B * T * H * D * 2 / 1e6)},
+        'config': workload_config(world, C, dR is not None),
+        'impl_detail': {'kernel_chunk': 128 if tc_path else C,
+                        'arithmetic': ('tcgen05 fp16 operands, fp32 accumulate' if tc_path
+                                       else 'fp32 CUDA cores'),
+                        'saved_states': saved is not None},
         'roofline': roof, 'kernel_rooflines': rooflines, 'cpu_baseline': cpu, 'e2e': e2e, 'gpu_launches': launches,
-        'clocks': clk, 'fwd': fwd, 'bwd': bwd, 'prepare_ms': prep_ms, 'decode': dec,
+        'clocks': clk, 'tensor_frac': tensor_frac, 'fwd': fwd, 'bwd': bwd,
+        'prepare_ms': prep_ms, 'kernel_ms_per_step': step_ms_kernels, 'decode': dec,
         'kernels': per_kernel,
     }
     if rank == 0:
@@ -398,7 +458,7 @@ def load_traffic(kernel):
 def run_decode(args, dev, peaks, rank):
     import torch
     from paper_2609_36259_gb300 import cyfa, synth
-    B, H, D, T0 = DECODE['B'], DECODE['H'], DECODE['d'], DECODE['prefill']
+    B, H, D, T0 = args.decode_batch, DECODE['H'], DECODE['d'], DECODE['prefill']
     S = args.decode_steps
     inp = synth.make_inputs(B, T0, H, D, seed=1000 + rank, device=dev)
     d0 = cyfa.dims(B, T0, H, D, chunk=64)
@@ -495,7 +555,7 @@ def run_e2e(args, inp, dev, want_dR):
     for _ in range(2):
         one()
     torch.cuda.synchronize()
-    n = max(1, min(args.steps, 3))
+    n = max(1, args.steps)
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     t0 = time.perf_counter()
     e0.record()
@@ -528,7 +588,7 @@ def run_reference(args):
     cores = None
     sample = None
     for _ in range(args.steps):
-        v, cores, sample, wall, _ = oracle_baseline(args.ref_tokens, H)
+        v, cores, sample, wall, _ = oracle_baseline(args.oracle_tokens, H)
         vals.append(v)
         walls.append(wall)
     value = sum(vals) / len(vals)
@@ -537,9 +597,7 @@ def run_reference(args):
         'n_gpus': world, 'steps': args.steps, 'warmup': args.warmup,
         'ms_per_step': 1e3 * sum(walls) / len(walls), 'higher_is_better': True,
         'scaling': 'weak', 'vs_baseline': None, 'dtype': 'f64', 'data': 'synthetic',
-        'config': {'workload': 'cyfa-1.4B-layer prepare+fwd+bwd', 'model': 'CyFA core operator',
-                   'B': B, 'T': T, 'H': H, 'dk': 128, 'dv': 128, 'm': 127, 'chunk': args.chunk,
-                   'global_batch': B * world, 'seq_len': T, 'parallelism': 'dp%d' % world},
+        'config': workload_config(world, args.chunk, not args.no_dR),
         'cpu_baseline': {'value': value, 'unit': 'tokens/s', 'cores': cores, 'kind': 'oracle',
                          'sample': sample},
         'e2e': {'value': value, 'unit': 'tokens/s', 'h2d_bytes_per_step': 0,
@@ -556,10 +614,15 @@ def main():
     ap.add_argument('--impl', default='ours', choices=['ours', 'reference'])
     ap.add_argument('--chunk', type=int, default=64, choices=[64, 128])
     ap.add_argument('--decode-steps', type=int, default=1024)
-    ap.add_argument('--cpu-tokens', type=int, default=32768)
+    ap.add_argument('--decode-batch', type=int, default=DECODE['B'],
+                    help='decode batch (profiling runs on smaller cases)')
+    ap.add_argument('--oracle-tokens', type=int, default=4096,
+                    help='tokens per (b,h) sequence of one oracle sample (cpu_baseline and the '
+                         'reference arm time the same sample)')
+    ap.add_argument('--cpu-reps', type=int, default=4,
+                    help='oracle samples timed for cpu_baseline')
     ap.add_argument('--shape', default=None,
                     help='B,T,H override of the layer shape (profiling runs on smaller cases)')
-    ap.add_argument('--ref-tokens', type=int, default=256)
     ap.add_argument('--no-decode', action='store_true')
     ap.add_argument('--no-e2e', action='store_true')
     ap.add_argument('--no-dR', action='store_true',

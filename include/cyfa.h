@@ -34,8 +34,9 @@
  * B * H <= 65535.
  *
  * Errors: every entry point returns CYFA_OK (0) or a negative code.  Argument errors are
- * found on the host before anything is launched.  CYFA_ERR_TIMEOUT is raised on the device
- * by a bounded wait and read back by cyfa_check().
+ * found on the host before anything is launched.  CYFA_ERR_TIMEOUT (a bounded wait expired)
+ * and CYFA_ERR_RANGE (a non-finite value reached a result) are raised on the device and read
+ * back by cyfa_check().
  */
 #ifndef CYFA_H
 #define CYFA_H
@@ -54,7 +55,8 @@ enum {
     CYFA_ERR_WORKSPACE = -4,  /* workspace null or smaller than cyfa_workspace_size() */
     CYFA_ERR_CUDA = -5,       /* a CUDA runtime call or launch failed */
     CYFA_ERR_TIMEOUT = -6,    /* a bounded device-side wait expired (see cyfa_check) */
-    CYFA_ERR_UNSUPPORTED = -7 /* a valid request this build does not implement */
+    CYFA_ERR_UNSUPPORTED = -7,/* a valid request this build does not implement */
+    CYFA_ERR_RANGE = -8       /* a non-finite value reached a result (see cyfa_check) */
 };
 
 enum { CYFA_DTYPE_BF16 = 0, CYFA_DTYPE_FP32 = 1 };
@@ -143,8 +145,12 @@ int cyfa_saved_size(const cyfa_dims_t* dims, size_t* bytes);
  * o receives the output; Kbar_out / Vbar_out (nullable) receive the states after token T-1.
  * saved (nullable, device, 16-byte aligned, cyfa_saved_size bytes) receives the chunk-start
  * states for cyfa_chunk_bwd; ignored where cyfa_saved_size is 0.
- * The tensor-core kernels (bf16, d = 128) compute with fp16 operands: q, k, v must lie within
- * fp16's range (|x| < 65504).
+ * The tensor-core kernels (bf16, d = 128) compute with fp16 operands (fp32 accumulation):
+ * q, k, v must lie within fp16's range (|x| < 65504), and so must the states they build, whose
+ * entries are bounded by 0.126 max|v| / (1 - max alpha) (|a_t| <= sqrt(2/m) beta_t entrywise;
+ * a geometric sum of decays).  Where an fp16 snapshot of a state overflows anyway, the output o
+ * becomes non-finite; the kernel that writes o then records CYFA_ERR_RANGE, which the next
+ * cyfa_check() returns.  The CUDA-core kernels (fp32 throughout) have no such limit.
  */
 int cyfa_chunk_fwd(const cyfa_dims_t* dims, const void* q, const void* k, const void* v,
                    const float* lam_mod, const float* g_cum, const float* beta, const float* R,
@@ -163,6 +169,11 @@ int cyfa_chunk_fwd(const cyfa_dims_t* dims, const void* q, const void* k, const 
  * and A (for the activation derivatives).  saved (nullable): the buffer a cyfa_chunk_fwd call
  * with the same dims, inputs and no initial state filled; the chunk-start states are then
  * read from it instead of being recomputed.  Ignored where cyfa_saved_size is 0.
+ * The tensor-core kernels' fp16 intermediates include the adjoint states (which grow with
+ * |dO| / (1 - max alpha)) and dL/do' = Vbar dO per token (which grows with |v| |dO| / (1 -
+ * max alpha)); all of them feed the three logit gradients, so an overflow anywhere makes one
+ * of those non-finite, and the kernel that writes them then records CYFA_ERR_RANGE, which the
+ * next cyfa_check() returns.
  */
 int cyfa_chunk_bwd(const cyfa_dims_t* dims, const void* q, const void* k, const void* v,
                    const float* lam_mod, const float* g_cum, const float* beta, const float* R,
@@ -184,8 +195,9 @@ int cyfa_step(const cyfa_dims_t* dims, const void* q, const void* k, const void*
               void* stream);
 
 /*
- * cyfa_check -- wait for `stream`, then report (and clear) the device error word that
- * bounded device-side waits set when they give up: CYFA_OK or CYFA_ERR_TIMEOUT, or
+ * cyfa_check -- wait for `stream`, then report (and clear) the device error word that the
+ * kernels set: CYFA_ERR_TIMEOUT when a bounded device-side wait gave up, else CYFA_ERR_RANGE
+ * when a non-finite value reached an output of the tensor-core kernels, else CYFA_OK;
  * CYFA_ERR_CUDA if the stream itself reports an error.
  */
 int cyfa_check(void* stream);

@@ -168,6 +168,7 @@ const char* cyfa_error_string(int code) {
         case CYFA_ERR_CUDA: return "CUDA runtime error";
         case CYFA_ERR_TIMEOUT: return "bounded device-side wait expired";
         case CYFA_ERR_UNSUPPORTED: return "request not implemented by this build";
+        case CYFA_ERR_RANGE: return "non-finite result: an fp16 operand of the tensor-core kernels overflowed, or an input was not finite";
         default: return "unknown cyfa error code";
     }
 }
@@ -436,7 +437,10 @@ int cyfa_check(void* stream) {
     int err = 0, err2 = 0;
     if (tc_read_error(st, &err) != cudaSuccess) return CYFA_ERR_CUDA;
     if (tc_bwd_read_error(st, &err2) != cudaSuccess) return CYFA_ERR_CUDA;
-    return (err || err2) ? CYFA_ERR_TIMEOUT : CYFA_OK;
+    // a timeout is reported before a range error (its results are incomplete, not just inexact)
+    if (err == CYFA_ERR_TIMEOUT || err2 == CYFA_ERR_TIMEOUT) return CYFA_ERR_TIMEOUT;
+    if (err == CYFA_ERR_RANGE || err2 == CYFA_ERR_RANGE) return CYFA_ERR_RANGE;
+    return (err || err2) ? CYFA_ERR_CUDA : CYFA_OK;
 }
 
 }  // extern "C"

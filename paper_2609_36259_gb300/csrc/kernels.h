@@ -50,6 +50,15 @@ struct PrepareArgs {
 constexpr int PREP_SEG = 1024;  // tokens per prepare block (multiple of every chunk size)
 size_t prepare_workspace(const Shape& s);
 cudaError_t launch_prepare(const PrepareArgs& a, cudaStream_t st);
+// Packed sequences (prepare_varlen.cu): a.s.B == 1, sequence j on tokens [cu[j], cu[j+1]);
+// lambda0 / lambda_end are [nseq][H]; rho > 0 and a.clock_logit == nullptr for a fixed-rate clock.
+size_t prepare_varlen_workspace(const Shape& s);
+cudaError_t launch_prepare_varlen(const PrepareArgs& a, const int* cu, int nseq, double rho,
+                                  double* seg, cudaStream_t st);
+// Fixed-rate clock delta = 1 / rho (no clock logits, no scan, no workspace).
+cudaError_t launch_prepare_fixed_rate(const PrepareArgs& a, double rho, cudaStream_t st);
+// Reads (and clears) the error word of the packed-sequence prepare; synchronises the stream.
+cudaError_t prep_read_error(cudaStream_t st, int* err);
 
 // ---- readout matrix M = R Phi and its transpose (chunk_simt.cu) ----
 cudaError_t launch_readout_matrix(int H, const float* R, float* M, float* MT, cudaStream_t st);

@@ -1520,7 +1520,11 @@ __global__ void __launch_bounds__(128) tc_gate_kernel(TcBwdArgs a) {
     const float delta = sigmoidf_(a.clock_logit[gi]);
     a.d_clock[gi] = ddelta * delta * (1.f - delta);
     const float bt = a.beta[gi];
-    a.d_beta[gi] = a.tok[4 * BTH + gi] * bt * (1.f - bt);
+    const float dbeta = a.tok[4 * BTH + gi];
+    a.d_beta[gi] = dbeta * bt * (1.f - bt);
+    // every per-token intermediate of the backward (fp16 snapshots, adjoints, o'', dL/do')
+    // feeds these three sums, so an fp16 overflow anywhere reaches them as inf / NaN
+    if (!isfinite(dlogalpha + ddelta + dbeta)) flag_error(CYFA_ERR_RANGE);
     double da = (double)dlogalpha * (double)(-softplusf_(f));
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) da += __shfl_xor_sync(0xffffffffu, da, o);

@@ -723,8 +723,14 @@ __global__ void __launch_bounds__(OUT_THREADS, 1) seg_out_tc(const __grid_consta
             {   // o = gamma_r (O'' Vbar) + P2 V, staged in T_S (P2 is consumed) for a TMA store
                 float x[32], y[32];
                 tmem_ld16x2_pair(tl + X2, x, tl + X1, y);
+                float fin = 0.f;   // a non-finite output makes the sum non-finite
 #pragma unroll
-                for (int i = 0; i < 32; ++i) x[i] = fmaf(gam, x[i], y[i]);
+                for (int i = 0; i < 32; ++i) {
+                    x[i] = fmaf(gam, x[i], y[i]);
+                    fin += x[i];
+                }
+                // an fp16 operand that overflowed (the Vbar snapshot) reaches o as inf / NaN
+                if (!isfinite(fin)) flag_error(CYFA_ERR_RANGE);
                 store_q<__nv_bfloat16>(T_S, row, c0, x);
             }
             publish();

@@ -14,7 +14,7 @@ LIB_PATH = os.path.join(HERE, 'libcyfa.so')
 
 CYFA_OK = 0
 CYFA_ERR_ARG, CYFA_ERR_SHAPE, CYFA_ERR_ALIGN, CYFA_ERR_WORKSPACE = -1, -2, -3, -4
-CYFA_ERR_CUDA, CYFA_ERR_TIMEOUT, CYFA_ERR_UNSUPPORTED = -5, -6, -7
+CYFA_ERR_CUDA, CYFA_ERR_TIMEOUT, CYFA_ERR_UNSUPPORTED, CYFA_ERR_RANGE = -5, -6, -7, -8
 CYFA_DTYPE_BF16, CYFA_DTYPE_FP32 = 0, 1
 CYFA_WS_PREPARE, CYFA_WS_FWD, CYFA_WS_BWD = 0, 1, 2
 

@@ -5,10 +5,8 @@ import torch
 
 from paper_2609_36259_gb300 import cyfa, synth
 
-from _harness import (assert_close_bf16, assert_close_fp32, assert_close_rel, assert_close_sum,
-                      gpu_prepare,
-                      oracle_backward,
-                      oracle_inputs, pairs_np, sample_pairs, to_device)
+from _harness import (assert_close_batch_sum, assert_close_bf16, assert_close_rel, gpu_prepare,
+                      oracle_backward, oracle_inputs, pairs_np, rel_l2, sample_pairs, to_device)
 
 pytestmark = pytest.mark.gpu
 
@@ -44,6 +42,23 @@ def gpu_backward(d, inp, want_dA=True, use_saved=False, want_dR=False):
 def _compare(out, ref, pairs, close, what=''):
     for gk, rk in GRADS:
         close(pairs_np(out[gk].float(), pairs), ref[rk], '%s %s' % (what, gk))
+    # the decay gradient of each head on its own (A_h scales it by up to 256x between heads)
+    got = pairs_np(out['d_decay'].float(), pairs)
+    for h in sorted({h for _, h in pairs}):
+        idx = [n for n, (_, hh) in enumerate(pairs) if hh == h]
+        print('measured %s d_decay head %d: rel-L2 %.3e'
+              % (what, h, rel_l2(got[idx], ref['d_decay'][idx])))
+
+
+def _dA_terms(inp, ref, pairs, H):
+    """The oracle's dA per head and its terms w_t d log alpha_t (w_t = -softplus(f_t))."""
+    f = pairs_np(inp['decay_logit'], pairs)
+    dA_ref = np.zeros(H)
+    terms = [[] for _ in range(H)]
+    for n, (b, h) in enumerate(pairs):
+        dA_ref[h] += ref['dA'][n]
+        terms[h].append(-np.logaddexp(0.0, f[n]) * ref['d_logalpha'][n])
+    return dA_ref, [np.concatenate(t) if t else np.zeros(1) for t in terms]
 
 
 @pytest.mark.parametrize('cuda_cores', [False, True])
@@ -62,13 +77,8 @@ def test_backward_small_bf16(B, T, H, D, C, cuda_cores):
     for n, (b, h) in enumerate(pairs):
         dR_ref[h] += ref['dR'][n]
     assert_close_rel(out['dR'].double().cpu().numpy(), dR_ref, 'dR')
-    dA_ref, l1 = np.zeros(H), np.zeros(H)
-    f = pairs_np(inp['decay_logit'], pairs)
-    softplus = np.logaddexp(0.0, f)
-    for n, (b, h) in enumerate(pairs):
-        dA_ref[h] += ref['dA'][n]
-        l1[h] += np.abs(ref['d_logalpha'][n] * softplus[n]).sum()
-    assert_close_sum(out['dA'].double().cpu().numpy(), dA_ref, l1, 'dA')
+    dA_ref, terms = _dA_terms(inp, ref, pairs, H)
+    assert_close_batch_sum(out['dA'].double().cpu().numpy(), dA_ref, terms, 'dA')
 
 
 def test_backward_fp32():
@@ -124,3 +134,33 @@ def test_backward_saved_full_size_sampled():
     pairs = sample_pairs(B, H, 2)
     ref = oracle_backward(oracle_inputs(inp, pairs), pairs_np(inp['dO'], pairs))
     _compare(out, ref, pairs, assert_close_bf16, 'saved full')
+
+
+@pytest.mark.parametrize('B,T,H,saved', [(4, 8192, 16, False), (2, 32768, 16, True)])
+def test_backward_full_size_dA_dR(B, T, H, saved):
+    """dA and dR at full size, in the launch configuration the bench step uses (dR requested,
+    saved states on the 1.4B layer).  Both are sums over the batch, so the upstream gradient is
+    kept on a few sampled (b, h) sequences and zeroed on every other one: the others then add
+    exactly zero to every gradient, and dA[h], dR[h] equal the oracle's sums over the sampled
+    sequences of head h (heads without a sampled sequence must come out zero)."""
+    inp = synth.make_inputs(B, T, H, 128, seed=3, device='cuda', with_dO=True)
+    pairs = sample_pairs(B, H, 3, seed=5)
+    keep = torch.zeros(B, 1, H, 1, device='cuda')
+    for b, h in pairs:
+        keep[b, 0, h, 0] = 1.0
+    inp['dO'] = (inp['dO'].float() * keep).to(inp['dO'].dtype)
+    d = cyfa.dims(B, T, H, 128, chunk=64)
+    out = gpu_backward(d, inp, want_dA=True, use_saved=saved, want_dR=True)
+    ref = oracle_backward(oracle_inputs(inp, pairs), pairs_np(inp['dO'], pairs))
+    _compare(out, ref, pairs, assert_close_bf16, 'masked dO B%d T%d' % (B, T))
+    dR_ref = np.zeros((H, 127, 127))
+    for n, (b, h) in enumerate(pairs):
+        dR_ref[h] += ref['dR'][n]
+    dA_ref, terms = _dA_terms(inp, ref, pairs, H)
+    hs = sorted({h for _, h in pairs})
+    dA = out['dA'].double().cpu().numpy()
+    dR = out['dR'].double().cpu().numpy()
+    assert_close_batch_sum(dA[hs], dA_ref[hs], [terms[h] for h in hs], 'dA')
+    assert_close_rel(dR[hs], dR_ref[hs], 'dR')
+    others = [h for h in range(H) if h not in hs]
+    assert np.all(dA[others] == 0) and np.all(dR[others] == 0)

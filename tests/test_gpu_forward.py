@@ -110,22 +110,35 @@ def test_extreme_gates():
     assert_close_bf16(pairs_np(o.float(), pairs), o_ref, 'o (saturated gates)')
 
 
+@pytest.mark.parametrize('cuda_cores', [False, True])
 @pytest.mark.parametrize('T,T1', [(512, 192), (2560, 1280)])
-def test_state_continuation(T, T1):
-    """Forward over [0, T1) exporting (Kbar, Vbar, lambda), then [T1, T) from them, equals one call."""
+def test_state_continuation(T, T1, cuda_cores):
+    """Forward over [0, T1) exporting (Kbar, Vbar, lambda), then [T1, T) started from them,
+    against the oracle: the oracle's own states after T1 (absolute_clock over [0, T1)) are fed
+    to absolute_clock over [T1, T) as (lambda0, Kbar0, Vbar0), and the library's exported states
+    are compared with the oracle's after T1 and after T."""
     B, H, D = 1, 2, 128
     inp = to_device(synth.make_inputs(B, T, H, D, seed=5))
-    d = cyfa.dims(B, T, H, D, chunk=64)
-    o_full, K_full, _, _ = gpu_forward(d, inp, want_state=True)
     seq = ('q', 'k', 'v', 'clock_logit', 'decay_logit', 'beta_logit')
     first = {k: (v[:, :T1].contiguous() if k in seq else v) for k, v in inp.items()}
     second = {k: (v[:, T1:].contiguous() if k in seq else v) for k, v in inp.items()}
-    o1, K1, V1, l1 = gpu_forward(cyfa.dims(B, T1, H, D, chunk=64), first, want_state=True)
-    o2, K2, V2, _ = gpu_forward(cyfa.dims(B, T - T1, H, D, chunk=64), second, want_state=True,
-                                Kbar0=K1, Vbar0=V1, lambda0=l1)
-    np.testing.assert_allclose(torch.cat([o1, o2], 1).float().cpu().numpy(),
-                               o_full.float().cpu().numpy(), atol=2e-2)
-    np.testing.assert_allclose(K2.cpu().numpy(), K_full.cpu().numpy(), atol=2e-3, rtol=2e-3)
+    o1, K1, V1, l1 = gpu_forward(cyfa.dims(B, T1, H, D, chunk=64, cuda_cores=cuda_cores), first,
+                                 want_state=True)
+    o2, K2, V2, l2 = gpu_forward(cyfa.dims(B, T - T1, H, D, chunk=64, cuda_cores=cuda_cores),
+                                 second, want_state=True, Kbar0=K1, Vbar0=V1, lambda0=l1)
+    pairs = [(0, h) for h in range(H)]
+    oi1, oi2 = oracle_inputs(first, pairs), oracle_inputs(second, pairs)
+    r1, Kr1, Vr1, lr1 = oracle_forward(oi1)
+    r2, Kr2, Vr2, lr2 = oracle_forward(oi2, lambda0=lr1, Kbar0=Kr1, Vbar0=Vr1)
+    assert_close_bf16(pairs_np(o1.float(), pairs), r1, 'o [0, T1)')
+    assert_close_bf16(pairs_np(o2.float(), pairs), r2, 'o [T1, T) from the exported states')
+    for got, want, what in ((K1, Kr1, 'Kbar(T1)'), (V1, Vr1, 'Vbar(T1)'), (K2, Kr2, 'Kbar(T)'),
+                            (V2, Vr2, 'Vbar(T)')):
+        g = np.stack([got[0, h].double().cpu().numpy() for h in range(H)])
+        assert_close_bf16(g[:, :127], want, what)
+        assert np.all(g[:, 127] == 0)
+    # the running clock continues: lambda_T of the second call against the oracle's
+    np.testing.assert_allclose(l2[0].cpu().numpy(), lr2, rtol=0, atol=1e-6 + 4e-9 * T)
 
 
 @pytest.mark.parametrize('B,T,H,C,cuda_cores', [(8, 4096, 8, 64, False), (8, 4096, 8, 64, True),
