@@ -13,6 +13,7 @@ batch (the (b, h) sequences are independent): weak scaling with no data-path col
 step time is the max over ranks.  --impl reference times the fp64 CPU oracle on the host cores.
 """
 import argparse
+import itertools
 import json
 import math
 import os
@@ -406,6 +407,16 @@ def run_ours(args):
     if not args.no_decode:
         dec = run_decode(args, dev, peaks, rank)
 
+    # packed variable-length sequences and the fixed-rate clock on the same layer
+    varlen = None
+    if not args.no_varlen:
+        varlen = run_varlen(args, dev, rank)
+
+    # the paper's own kernel shape (H = 4, d = 256, T = 2048, B = 32)
+    paper = None
+    if not args.no_paper_shape:
+        paper = run_paper_shape(args, dev, rank, peaks)
+
     # end to end through the public API with host buffers
     e2e = None
     if not args.no_e2e:
@@ -426,6 +437,7 @@ def run_ours(args):
         'roofline': roof, 'kernel_rooflines': rooflines, 'cpu_baseline': cpu, 'e2e': e2e, 'gpu_launches': launches,
         'clocks': clk, 'tensor_frac': tensor_frac, 'fwd': fwd, 'bwd': bwd,
         'prepare_ms': prep_ms, 'kernel_ms_per_step': step_ms_kernels, 'decode': dec,
+        'varlen': varlen, 'paper_shape': paper,
         'kernels': per_kernel,
     }
     if rank == 0:
@@ -493,7 +505,129 @@ def run_decode(args, dev, peaks, rank):
     return {'workload': 'B=%d H=%d d=%d fp32 states, %d-token prefill, %d steps' % (B, H, D, T0, S),
             'ms_per_step': ms, 'tokens_per_s': B / (ms / 1e3), 'GB_per_s': gbs,
             'bytes_per_step': bytes_step, 'frac_hbm_measured': gbs / peaks['hbm_gbs'],
+            'traffic': load_traffic('decode_step') if B == DECODE['B'] else None,
             'frac_hbm_8TBs': gbs / 8000.0}
+
+
+def run_paper_shape(args, dev, rank, peaks):
+    """prepare + forward + backward (every gradient) at the shape of the paper's kernel-latency
+    figure: B = 32, T = 2048, H = 4, d_k = d_v = 256, m = 127, bf16 inputs."""
+    import torch
+    from paper_2609_36259_gb300 import cyfa, synth
+    B, T, H, D, C = 32, 2048, 4, 256, 64
+    inp = synth.make_inputs(B, T, H, D, seed=4000 + rank, device=dev, with_dO=True)
+    d = cyfa.dims(B, T, H, D, chunk=C)
+    f32 = dict(dtype=torch.float32, device=dev)
+    lam, g, beta = (torch.empty(B, T, H, **f32) for _ in range(3))
+    o = torch.empty_like(inp['v'])
+    dq, dk, dv = (torch.empty_like(inp[x]) for x in ('q', 'k', 'v'))
+    dc, dd, db = (torch.empty_like(lam) for _ in range(3))
+    dA, dR = torch.empty(H, **f32), torch.empty(H, 127, 127, **f32)
+    ws = [cyfa.workspace(d, w, dev) for w in (cyfa.CYFA_WS_PREPARE, cyfa.CYFA_WS_FWD,
+                                               cyfa.CYFA_WS_BWD)]
+
+    def fwd():
+        cyfa.cyfa_prepare(d, inp['clock_logit'], inp['decay_logit'], inp['beta_logit'], inp['A'],
+                          None, lam, g, beta, None, ws[0])
+        cyfa.cyfa_chunk_fwd(d, inp['q'], inp['k'], inp['v'], lam, g, beta, inp['R'], None, None,
+                            o, None, None, ws[1])
+
+    def step():
+        fwd()
+        cyfa.cyfa_chunk_bwd(d, inp['q'], inp['k'], inp['v'], lam, g, beta, inp['R'],
+                            inp['clock_logit'], inp['decay_logit'], inp['A'], inp['dO'], dq, dk,
+                            dv, dc, dd, db, dR, dA, ws[2])
+
+    def timed(fn, n):
+        for _ in range(3):
+            fn()
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        for _ in range(n):
+            fn()
+        e1.record()
+        torch.cuda.synchronize()
+        return e0.elapsed_time(e1) / n
+
+    n = max(1, min(args.steps, 20))
+    ms = timed(step, n)
+    ms_fwd = timed(fwd, n)
+    cyfa.cyfa_check()
+    th = B * T * H
+    fl = operator_flops_per_token_head(C, d=D) * th
+    alu = fp32_alu_peak_tflops(peaks['sm_max_mhz'])
+    return {'workload': 'B=%d T=%d H=%d d=%d chunk %d (the paper\'s kernel-latency shape), '
+                        'prepare + fwd + bwd with every gradient' % (B, T, H, D, C),
+            'path': 'fp32 CUDA-core kernels (the tensor-core kernels take d = 128)',
+            'ms_per_step': ms, 'tokens_per_s': B * T / (ms / 1e3),
+            'fwd_ms': ms_fwd, 'fwd_tokens_per_s': B * T / (ms_fwd / 1e3),
+            'tflops_rule': 3 * fl / (ms / 1e3) / 1e12,
+            'frac_fp32_alu_peak': 3 * fl / (ms / 1e3) / 1e12 / alu, 'alu_peak_tflops': alu}
+
+
+def run_varlen(args, dev, rank):
+    """The layer's B*T tokens as one packed stream of sequences of mixed length around 2,048
+    tokens (cyfa_prepare_varlen + forward + backward with every gradient, saved states), and the
+    prepare of the fixed-rate clock (cyfa_prepare_fixed_rate, no scan) beside the learned one."""
+    import torch
+    from paper_2609_36259_gb300 import cyfa, synth
+    B, T, H, D = LAYER['B'], LAYER['T'], LAYER['H'], LAYER['d']
+    N = B * T
+    lengths = synth.varlen_lengths(N, 2048, seed=rank)
+    inp = synth.make_inputs(1, N, H, D, seed=3000 + rank, device=dev, with_dO=True)
+    cu = torch.tensor([0] + list(itertools.accumulate(lengths)), dtype=torch.int32, device=dev)
+    d = cyfa.dims(1, N, H, D, chunk=args.chunk)
+    f32 = dict(dtype=torch.float32, device=dev)
+    lam, g, beta = (torch.empty(1, N, H, **f32) for _ in range(3))
+    o = torch.empty_like(inp['v'])
+    dq, dk, dv = (torch.empty_like(inp[x]) for x in ('q', 'k', 'v'))
+    dc, dd, db = (torch.empty_like(lam) for _ in range(3))
+    dA, dR = torch.empty(H, **f32), torch.empty(H, 127, 127, **f32)
+    ws_v = cyfa.workspace(d, cyfa.CYFA_WS_PREPARE_VARLEN, dev)
+    ws_f = cyfa.workspace(d, cyfa.CYFA_WS_FWD, dev)
+    ws_b = cyfa.workspace(d, cyfa.CYFA_WS_BWD, dev)
+    saved = cyfa.saved_buffer(d, dev)
+
+    def step():
+        cyfa.cyfa_prepare_varlen(d, cu, len(lengths), inp['clock_logit'], 0.0, inp['decay_logit'],
+                                 inp['beta_logit'], inp['A'], None, lam, g, beta, None, ws_v)
+        cyfa.cyfa_chunk_fwd(d, inp['q'], inp['k'], inp['v'], lam, g, beta, inp['R'], None, None,
+                            o, None, None, ws_f, saved=saved)
+        cyfa.cyfa_chunk_bwd(d, inp['q'], inp['k'], inp['v'], lam, g, beta, inp['R'],
+                            inp['clock_logit'], inp['decay_logit'], inp['A'], inp['dO'], dq, dk,
+                            dv, dc, dd, db, dR, dA, ws_b, saved=saved)
+
+    def timed(fn, n):
+        for _ in range(3):
+            fn()
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        for _ in range(n):
+            fn()
+        e1.record()
+        torch.cuda.synchronize()
+        return e0.elapsed_time(e1) / n
+
+    ms = timed(step, max(1, args.steps))
+    cyfa.cyfa_check()
+    ws_p = cyfa.workspace(d, cyfa.CYFA_WS_PREPARE, dev)
+    ms_prep = timed(lambda: cyfa.cyfa_prepare(d, inp['clock_logit'], inp['decay_logit'],
+                                              inp['beta_logit'], inp['A'], None, lam, g, beta,
+                                              None, ws_p), 20)
+    ms_prepv = timed(lambda: cyfa.cyfa_prepare_varlen(d, cu, len(lengths), inp['clock_logit'],
+                                                      0.0, inp['decay_logit'], inp['beta_logit'],
+                                                      inp['A'], None, lam, g, beta, None, ws_v), 20)
+    ms_fixed = timed(lambda: cyfa.cyfa_prepare_fixed_rate(d, 2.0, inp['decay_logit'],
+                                                          inp['beta_logit'], inp['A'], None, lam,
+                                                          g, beta, None), 20)
+    return {'workload': '%d tokens H=%d d=%d as %d packed sequences (log-normal lengths, mean '
+                        '2048, %d..%d), prepare_varlen + fwd + bwd with every gradient'
+                        % (N, H, D, len(lengths), min(lengths), max(lengths)),
+            'ms_per_step': ms, 'tokens_per_s': N / (ms / 1e3),
+            'prepare_ms': ms_prep, 'prepare_varlen_ms': ms_prepv,
+            'prepare_fixed_rate_ms': ms_fixed}
 
 
 def run_e2e(args, inp, dev, want_dR):
@@ -625,6 +759,8 @@ def main():
                     help='B,T,H override of the layer shape (profiling runs on smaller cases)')
     ap.add_argument('--no-decode', action='store_true')
     ap.add_argument('--no-e2e', action='store_true')
+    ap.add_argument('--no-varlen', action='store_true')
+    ap.add_argument('--no-paper-shape', action='store_true')
     ap.add_argument('--no-dR', action='store_true',
                     help='leave the readout gradient dR out of the backward')
     ap.add_argument('--no-saved', action='store_true',

@@ -62,7 +62,7 @@ enum {
 enum { CYFA_DTYPE_BF16 = 0, CYFA_DTYPE_FP32 = 1 };
 
 /* Which call a workspace is sized for. */
-enum { CYFA_WS_PREPARE = 0, CYFA_WS_FWD = 1, CYFA_WS_BWD = 2 };
+enum { CYFA_WS_PREPARE = 0, CYFA_WS_FWD = 1, CYFA_WS_BWD = 2, CYFA_WS_PREPARE_VARLEN = 3 };
 
 typedef struct cyfa_dims {
     int B, T, H;   /* batch, sequence length, heads */
@@ -103,6 +103,50 @@ int cyfa_prepare(const cyfa_dims_t* dims, const float* clock_logit, const float*
                  const float* beta_logit, const float* A, const double* lambda0,
                  float* lam_mod, float* g_cum, float* beta, double* lambda_end,
                  void* workspace, size_t workspace_bytes, void* stream);
+
+/*
+ * cyfa_prepare_fixed_rate -- cyfa_prepare for the fixed-rate clock delta_t = 1 / rho (App. A,
+ * Fixed-Rate Specialization and Relation to BLA, Eq. app-constant-rate-profile: with a constant
+ * increment the relative-time profile is the Fourier-Dirichlet profile of Blurry Window
+ * Attention).  lambda_t = lambda0[b,h] + t / rho (t = 1..T) in fp64 closed form, reduced mod m:
+ * there are no clock logits and no prefix sum, so no workspace.  g_cum, beta and lambda_end as in
+ * cyfa_prepare.  rho > 0 (CYFA_ERR_ARG otherwise).  The chunk calls take the results unchanged;
+ * cyfa_chunk_bwd then gets clock_logit = d_clock_logit = NULL.  A decode step of the same model
+ * is cyfa_step with clock logit -ln(rho - 1) (+inf for rho = 1), whose sigmoid is 1 / rho.
+ */
+int cyfa_prepare_fixed_rate(const cyfa_dims_t* dims, double rho, const float* decay_logit,
+                            const float* beta_logit, const float* A, const double* lambda0,
+                            float* lam_mod, float* g_cum, float* beta, double* lambda_end,
+                            void* stream);
+
+/*
+ * cyfa_prepare_varlen -- cyfa_prepare for variable-length sequences packed into one stream:
+ * dims.B = 1, dims.T the total token count, and sequence j (0 <= j < nseq) on tokens
+ * [cu_seqlens[j], cu_seqlens[j+1]) (cu_seqlens: device int32 [nseq + 1], non-decreasing, from 0
+ * to T; empty sequences are allowed).  Each sequence is the operator on its own: its clock
+ * starts at lambda0[j,h] (lambda0 [nseq, H] fp64, nullable for 0) and its states at zero.
+ *   lam_mod, beta  as in cyfa_prepare, the clock restarting at every sequence start.
+ *   g_cum          as in cyfa_prepare, minus 64 for every sequence start s > 0 with
+ *                  chunk_start(t) <= s <= t: every decay factor exp(g_t - g_s) of the chunk
+ *                  form (App. B Eq. app-chunk-decay) that spans a start then carries exp(-64),
+ *                  which removes every contribution of an earlier sequence in fp32, while the
+ *                  factors inside a sequence keep their value (one extra fp32 rounding of g).
+ *   lambda_end     [nseq, H] fp64 (nullable): each sequence's final clock.
+ * clock_logit may be NULL: the fixed-rate clock delta = 1 / rho of cyfa_prepare_fixed_rate.
+ * cyfa_chunk_fwd and cyfa_chunk_bwd take the results as they are (B = 1, T the total) and give
+ * each sequence's outputs and gradients; the decay and clock gradients need no change because
+ * every term that spans a sequence start vanishes with its decay factor.  Kbar0 / Vbar0 give the
+ * first sequence's initial states; Kbar_out / Vbar_out receive the last sequence's final states
+ * (the chunk calls export no per-sequence states).  T must still be a multiple of the chunk
+ * (pad with one more sequence).  Needs cyfa_workspace_size(CYFA_WS_PREPARE_VARLEN) bytes.
+ * Offsets that are not a non-decreasing cover of [0, T] are detected on the device: the next
+ * cyfa_check() returns CYFA_ERR_ARG (the results are then meaningless).
+ */
+int cyfa_prepare_varlen(const cyfa_dims_t* dims, const int* cu_seqlens, int nseq,
+                        const float* clock_logit, double rho, const float* decay_logit,
+                        const float* beta_logit, const float* A, const double* lambda0,
+                        float* lam_mod, float* g_cum, float* beta, double* lambda_end,
+                        void* workspace, size_t workspace_bytes, void* stream);
 
 /*
  * cyfa_prepare_noalloc -- cyfa_prepare for callers that cannot provide any device memory of
@@ -166,7 +210,8 @@ int cyfa_chunk_fwd(const cyfa_dims_t* dims, const void* q, const void* k, const 
  * the per-token gradient of the cumulative log-decay.  dR [H,m,m] and dA [H] are sums
  * over the batch (dR through M = R Phi of the middle readout, Sec. 3.3 Eq. cyfa-two-pass).
  * Inputs are those of cyfa_chunk_fwd plus the raw clock / decay logits
- * and A (for the activation derivatives).  saved (nullable): the buffer a cyfa_chunk_fwd call
+ * and A (for the activation derivatives).  clock_logit and d_clock_logit are both NULL for a
+ * fixed-rate clock (cyfa_prepare_fixed_rate): the clock gradient is then not formed.  saved (nullable): the buffer a cyfa_chunk_fwd call
  * with the same dims, inputs and no initial state filled; the chunk-start states are then
  * read from it instead of being recomputed.  Ignored where cyfa_saved_size is 0.
  * The tensor-core kernels' fp16 intermediates include the adjoint states (which grow with
@@ -195,10 +240,11 @@ int cyfa_step(const cyfa_dims_t* dims, const void* q, const void* k, const void*
               void* stream);
 
 /*
- * cyfa_check -- wait for `stream`, then report (and clear) the device error word that the
- * kernels set: CYFA_ERR_TIMEOUT when a bounded device-side wait gave up, else CYFA_ERR_RANGE
- * when a non-finite value reached an output of the tensor-core kernels, else CYFA_OK;
- * CYFA_ERR_CUDA if the stream itself reports an error.
+ * cyfa_check -- wait for `stream`, then report (and clear) the device error words that the
+ * kernels set: CYFA_ERR_TIMEOUT when a bounded device-side wait gave up, else CYFA_ERR_ARG when
+ * cyfa_prepare_varlen found invalid sequence offsets, else CYFA_ERR_RANGE when a non-finite
+ * value reached an output of the tensor-core kernels, else CYFA_OK; CYFA_ERR_CUDA if the stream
+ * itself reports an error.
  */
 int cyfa_check(void* stream);
 

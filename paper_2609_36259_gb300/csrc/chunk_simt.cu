@@ -282,6 +282,7 @@ cudaError_t launch_fwd_simt(const FwdArgs& a, cudaStream_t st) {
     CYFA_FWD(64, 128)
     CYFA_FWD(128, 64)
     CYFA_FWD(128, 128)
+    CYFA_FWD(64, 256)
 #undef CYFA_FWD
     return cudaErrorInvalidValue;
 }

@@ -697,8 +697,10 @@ __global__ void __launch_bounds__(256) gate_scan_kernel(BwdArgs a, int nseg) {
             const float dlogalpha = (float)rg;
             a.d_decay[gi] = dlogalpha * (-Ah * sigmoidf_(f));
             dA_acc += (double)dlogalpha * (double)(-softplusf_(f));
-            const float delta = sigmoidf_(a.clock_logit[gi]);
-            a.d_clock[gi] = (float)rl * delta * (1.f - delta);
+            if (a.d_clock) {   // no clock logits (fixed-rate clock): no clock gradient
+                const float delta = sigmoidf_(a.clock_logit[gi]);
+                a.d_clock[gi] = (float)rl * delta * (1.f - delta);
+            }
             const float bt = a.beta[gi];
             a.d_beta[gi] = a.tok[4 * BTH + gi] * bt * (1.f - bt);
         }
@@ -790,6 +792,7 @@ cudaError_t launch_bwd_simt(const BwdArgs& a, cudaStream_t st) {
     if (s.C != CB) return cudaErrorInvalidValue;
     if (s.D == 128) return s.bf16 ? bwd_dispatch<128, __nv_bfloat16>(a, st) : bwd_dispatch<128, float>(a, st);
     if (s.D == 64) return s.bf16 ? bwd_dispatch<64, __nv_bfloat16>(a, st) : bwd_dispatch<64, float>(a, st);
+    if (s.D == 256) return s.bf16 ? bwd_dispatch<256, __nv_bfloat16>(a, st) : bwd_dispatch<256, float>(a, st);
     return cudaErrorInvalidValue;
 }
 

@@ -38,7 +38,7 @@ int cyfa::check_dims(const cyfa_dims_t* d, bool need_T) {
         return CYFA_ERR_ARG;
     if (d->dtype != CYFA_DTYPE_BF16 && d->dtype != CYFA_DTYPE_FP32) return CYFA_ERR_ARG;
     if (d->m != 127) return CYFA_ERR_SHAPE;
-    if (d->dk != d->dv || (d->dk != 64 && d->dk != 128)) return CYFA_ERR_SHAPE;
+    if (d->dk != d->dv || (d->dk != 64 && d->dk != 128 && d->dk != 256)) return CYFA_ERR_SHAPE;
     if ((long long)d->B * d->H > kMaxSequences) return CYFA_ERR_SHAPE;
     if (need_T) {
         if (d->chunk != 64 && d->chunk != 128) return CYFA_ERR_SHAPE;
@@ -66,6 +66,14 @@ bool use_tc(const cyfa_dims_t* d, const Shape& s) {
     return !(d->flags & CYFA_FLAG_CUDA_CORES) && tc_fwd_supported(s);
 }
 
+// The CUDA-core forward walks the caller's chunk, except at d = 256, where it walks 64-token
+// chunks (its register tiles of a 128-token chunk would not fit); g_cum stays local to the
+// caller's chunk (Cg) and the kernels rebase it.
+Shape simt_fwd_shape(Shape s) {
+    if (s.D == 256) s.C = 64;
+    return s;
+}
+
 struct FwdLayout {
     float *M, *MT, *states;          // CUDA-core path
     float *segS, *segG;              // tensor-core path
@@ -73,7 +81,8 @@ struct FwdLayout {
     int nseg;
     size_t bytes;
 };
-FwdLayout fwd_layout(const Shape& s, bool tc_path, void* ws) {
+FwdLayout fwd_layout(const Shape& s0, bool tc_path, void* ws) {
+    const Shape s = tc_path ? s0 : simt_fwd_shape(s0);
     Carver c{static_cast<char*>(ws)};
     FwdLayout L{};
     L.M = c.take<float>((size_t)s.H * MS * MS);
@@ -162,7 +171,7 @@ const char* cyfa_error_string(int code) {
     switch (code) {
         case CYFA_OK: return "ok";
         case CYFA_ERR_ARG: return "invalid argument (null pointer or non-positive size)";
-        case CYFA_ERR_SHAPE: return "unsupported shape (m must be 127, dk == dv in {64,128}, chunk in {64,128}, T % chunk == 0)";
+        case CYFA_ERR_SHAPE: return "unsupported shape (m must be 127, dk == dv in {64,128,256}, chunk in {64,128}, T % chunk == 0, B*H <= 65535)";
         case CYFA_ERR_ALIGN: return "tensor pointer not 16-byte aligned";
         case CYFA_ERR_WORKSPACE: return "workspace missing or too small";
         case CYFA_ERR_CUDA: return "CUDA runtime error";
@@ -180,6 +189,7 @@ int cyfa_workspace_size(const cyfa_dims_t* dims, int which, size_t* bytes) {
     const Shape s = shape_of(dims);
     switch (which) {
         case CYFA_WS_PREPARE: *bytes = up(prepare_workspace(s)); return CYFA_OK;
+        case CYFA_WS_PREPARE_VARLEN: *bytes = up(prepare_varlen_workspace(s)); return CYFA_OK;
         case CYFA_WS_FWD: *bytes = fwd_layout(s, use_tc(dims, s), nullptr).bytes; return CYFA_OK;
         case CYFA_WS_BWD: *bytes = bwd_layout(s, use_tc(dims, s), nullptr).bytes; return CYFA_OK;
         default: return CYFA_ERR_ARG;
@@ -221,6 +231,56 @@ int cyfa_prepare(const cyfa_dims_t* dims, const float* clock_logit, const float*
     a.lambda_end = lambda_end;
     a.seg_sum = static_cast<double*>(workspace);
     return cuda_status(launch_prepare(a, static_cast<cudaStream_t>(stream)));
+}
+
+int cyfa_prepare_fixed_rate(const cyfa_dims_t* dims, double rho, const float* decay_logit,
+                            const float* beta_logit, const float* A, const double* lambda0,
+                            float* lam_mod, float* g_cum, float* beta, double* lambda_end,
+                            void* stream) {
+    int rc = check_dims(dims, true);
+    if (rc) return rc;
+    if (!(rho > 0.0) || !decay_logit || !beta_logit || !A || !lam_mod || !g_cum || !beta)
+        return CYFA_ERR_ARG;
+    PrepareArgs a{};
+    a.s = shape_of(dims);
+    a.clock_logit = nullptr;
+    a.decay_logit = decay_logit;
+    a.beta_logit = beta_logit;
+    a.A = A;
+    a.lambda0 = lambda0;
+    a.lam_mod = lam_mod;
+    a.g_cum = g_cum;
+    a.beta = beta;
+    a.lambda_end = lambda_end;
+    return cuda_status(launch_prepare_fixed_rate(a, rho, static_cast<cudaStream_t>(stream)));
+}
+
+int cyfa_prepare_varlen(const cyfa_dims_t* dims, const int* cu_seqlens, int nseq,
+                        const float* clock_logit, double rho, const float* decay_logit,
+                        const float* beta_logit, const float* A, const double* lambda0,
+                        float* lam_mod, float* g_cum, float* beta, double* lambda_end,
+                        void* workspace, size_t workspace_bytes, void* stream) {
+    int rc = check_dims(dims, true);
+    if (rc) return rc;
+    if (dims->B != 1 || nseq <= 0 || !cu_seqlens) return CYFA_ERR_ARG;
+    if (!clock_logit && !(rho > 0.0)) return CYFA_ERR_ARG;
+    if (!decay_logit || !beta_logit || !A || !lam_mod || !g_cum || !beta) return CYFA_ERR_ARG;
+    const Shape s = shape_of(dims);
+    if (!workspace || workspace_bytes < prepare_varlen_workspace(s)) return CYFA_ERR_WORKSPACE;
+    PrepareArgs a{};
+    a.s = s;
+    a.clock_logit = clock_logit;
+    a.decay_logit = decay_logit;
+    a.beta_logit = beta_logit;
+    a.A = A;
+    a.lambda0 = lambda0;
+    a.lam_mod = lam_mod;
+    a.g_cum = g_cum;
+    a.beta = beta;
+    a.lambda_end = lambda_end;
+    return cuda_status(launch_prepare_varlen(a, cu_seqlens, nseq, clock_logit ? 1.0 : rho,
+                                             static_cast<double*>(workspace),
+                                             static_cast<cudaStream_t>(stream)));
 }
 
 int cyfa_chunk_fwd(const cyfa_dims_t* dims, const void* q, const void* k, const void* v,
@@ -267,7 +327,7 @@ int cyfa_chunk_fwd(const cyfa_dims_t* dims, const void* q, const void* k, const 
         return cuda_status(launch_fwd_tc(t, q, k, v, st));
     }
     FwdArgs a;
-    a.s = s;
+    a.s = simt_fwd_shape(s);
     a.q = q;
     a.k = k;
     a.v = v;
@@ -293,9 +353,11 @@ int cyfa_chunk_bwd(const cyfa_dims_t* dims, const void* q, const void* k, const 
                    const void* saved, void* workspace, size_t workspace_bytes, void* stream) {
     int rc = check_dims(dims, true);
     if (rc) return rc;
-    if (!q || !k || !v || !lam_mod || !g_cum || !beta || !R || !clock_logit || !decay_logit ||
-        !A || !dO || !dq || !dk || !dv || !d_clock_logit || !d_decay_logit || !d_beta_logit)
+    if (!q || !k || !v || !lam_mod || !g_cum || !beta || !R || !decay_logit || !A || !dO || !dq ||
+        !dk || !dv || !d_decay_logit || !d_beta_logit)
         return CYFA_ERR_ARG;
+    // both or neither: a fixed-rate clock has no clock logits and no clock gradient
+    if ((clock_logit == nullptr) != (d_clock_logit == nullptr)) return CYFA_ERR_ARG;
     if (!aligned16(q) || !aligned16(k) || !aligned16(v) || !aligned16(dO) || !aligned16(dq) ||
         !aligned16(dk) || !aligned16(dv))
         return CYFA_ERR_ALIGN;
@@ -434,13 +496,16 @@ int cyfa_step(const cyfa_dims_t* dims, const void* q, const void* k, const void*
 int cyfa_check(void* stream) {
     cudaStream_t st = static_cast<cudaStream_t>(stream);
     if (cudaStreamSynchronize(st) != cudaSuccess) return CYFA_ERR_CUDA;
-    int err = 0, err2 = 0;
+    int err = 0, err2 = 0, err3 = 0;
     if (tc_read_error(st, &err) != cudaSuccess) return CYFA_ERR_CUDA;
     if (tc_bwd_read_error(st, &err2) != cudaSuccess) return CYFA_ERR_CUDA;
-    // a timeout is reported before a range error (its results are incomplete, not just inexact)
+    if (prep_read_error(st, &err3) != cudaSuccess) return CYFA_ERR_CUDA;
+    // a timeout is reported first (its results are incomplete), then invalid sequence offsets
+    // (every result after them is meaningless), then a range error (results inexact)
     if (err == CYFA_ERR_TIMEOUT || err2 == CYFA_ERR_TIMEOUT) return CYFA_ERR_TIMEOUT;
+    if (err3 == CYFA_ERR_ARG) return CYFA_ERR_ARG;
     if (err == CYFA_ERR_RANGE || err2 == CYFA_ERR_RANGE) return CYFA_ERR_RANGE;
-    return (err || err2) ? CYFA_ERR_CUDA : CYFA_OK;
+    return (err || err2 || err3) ? CYFA_ERR_CUDA : CYFA_OK;
 }
 
 }  // extern "C"

@@ -677,6 +677,9 @@ cudaError_t launch_step(const StepArgs& a, cudaStream_t st) {
     } else if (a.D == 64) {
         if (a.bf16) { LaunchScope ls_("decode_step", st); step_kernel<64, __nv_bfloat16><<<grid, 256, 0, st>>>(a); }
         else { LaunchScope ls_("decode_step", st); step_kernel<64, float><<<grid, 256, 0, st>>>(a); }
+    } else if (a.D == 256) {
+        if (a.bf16) { LaunchScope ls_("decode_step", st); step_kernel<256, __nv_bfloat16><<<grid, 256, 0, st>>>(a); }
+        else { LaunchScope ls_("decode_step", st); step_kernel<256, float><<<grid, 256, 0, st>>>(a); }
     } else {
         return cudaErrorInvalidValue;
     }

@@ -1517,8 +1517,10 @@ __global__ void __launch_bounds__(128) tc_gate_kernel(TcBwdArgs a) {
     const float ddelta = sl - ql + bd[1];
     const float f = a.decay_logit[gi];
     a.d_decay[gi] = dlogalpha * (-a.A[h] * sigmoidf_(f));
-    const float delta = sigmoidf_(a.clock_logit[gi]);
-    a.d_clock[gi] = ddelta * delta * (1.f - delta);
+    if (a.d_clock) {   // no clock logits (fixed-rate clock): no clock gradient
+        const float delta = sigmoidf_(a.clock_logit[gi]);
+        a.d_clock[gi] = ddelta * delta * (1.f - delta);
+    }
     const float bt = a.beta[gi];
     const float dbeta = a.tok[4 * BTH + gi];
     a.d_beta[gi] = dbeta * bt * (1.f - bt);

@@ -16,13 +16,14 @@ CYFA_OK = 0
 CYFA_ERR_ARG, CYFA_ERR_SHAPE, CYFA_ERR_ALIGN, CYFA_ERR_WORKSPACE = -1, -2, -3, -4
 CYFA_ERR_CUDA, CYFA_ERR_TIMEOUT, CYFA_ERR_UNSUPPORTED, CYFA_ERR_RANGE = -5, -6, -7, -8
 CYFA_DTYPE_BF16, CYFA_DTYPE_FP32 = 0, 1
-CYFA_WS_PREPARE, CYFA_WS_FWD, CYFA_WS_BWD = 0, 1, 2
+CYFA_WS_PREPARE, CYFA_WS_FWD, CYFA_WS_BWD, CYFA_WS_PREPARE_VARLEN = 0, 1, 2, 3
 
 # Every symbol include/cyfa.h declares (checked by tests/test_abi.py).
 EXPORTS = ('cyfa_version', 'cyfa_error_string', 'cyfa_workspace_size', 'cyfa_prepare',
            'cyfa_chunk_fwd', 'cyfa_chunk_bwd', 'cyfa_step', 'cyfa_check', 'cyfa_stats_reset',
            'cyfa_stats_timing', 'cyfa_stats_get', 'cyfa_prepare_noalloc',
-           'cyfa_selftest_mma', 'cyfa_saved_size', 'cyfa_selftest_timeout')
+           'cyfa_selftest_mma', 'cyfa_saved_size', 'cyfa_selftest_timeout',
+           'cyfa_prepare_fixed_rate', 'cyfa_prepare_varlen')
 
 
 class CyfaError(RuntimeError):
@@ -73,6 +74,9 @@ def load(path=LIB_PATH):
     lib.cyfa_selftest_mma.argtypes = [ctypes.c_int, _VP, _VP, _VP, _VP]
     lib.cyfa_selftest_timeout.argtypes = [ctypes.c_uint, _VP, _VP]
     lib.cyfa_prepare_noalloc.argtypes = [P] + [_VP] * 9 + [_VP]
+    lib.cyfa_prepare_fixed_rate.argtypes = [P, ctypes.c_double] + [_VP] * 8 + [_VP]
+    lib.cyfa_prepare_varlen.argtypes = ([P, _VP, ctypes.c_int, _VP, ctypes.c_double] + [_VP] * 8
+                                        + [_VP, ctypes.c_size_t, _VP])
     lib.cyfa_stats_timing.argtypes = [ctypes.c_int]
     lib.cyfa_stats_get.argtypes = [ctypes.c_int, ctypes.c_char_p, ctypes.c_int,
                                    ctypes.POINTER(ctypes.c_longlong), ctypes.POINTER(ctypes.c_double)]
@@ -140,6 +144,22 @@ def cyfa_prepare_noalloc(d, clock_logit, decay_logit, beta_logit, A, lambda0, la
     _ok(load().cyfa_prepare_noalloc(ctypes.byref(d), _ptr(clock_logit), _ptr(decay_logit),
                                     _ptr(beta_logit), _ptr(A), _ptr(lambda0), _ptr(lam_mod),
                                     _ptr(g_cum), _ptr(beta), _ptr(lambda_end), _stream(stream)))
+
+
+def cyfa_prepare_fixed_rate(d, rho, decay_logit, beta_logit, A, lambda0, lam_mod, g_cum, beta,
+                            lambda_end, stream=None):
+    _ok(load().cyfa_prepare_fixed_rate(ctypes.byref(d), float(rho), _ptr(decay_logit),
+                                       _ptr(beta_logit), _ptr(A), _ptr(lambda0), _ptr(lam_mod),
+                                       _ptr(g_cum), _ptr(beta), _ptr(lambda_end), _stream(stream)))
+
+
+def cyfa_prepare_varlen(d, cu_seqlens, nseq, clock_logit, rho, decay_logit, beta_logit, A,
+                        lambda0, lam_mod, g_cum, beta, lambda_end, ws, stream=None):
+    _ok(load().cyfa_prepare_varlen(ctypes.byref(d), _ptr(cu_seqlens), int(nseq),
+                                   _ptr(clock_logit), float(rho), _ptr(decay_logit),
+                                   _ptr(beta_logit), _ptr(A), _ptr(lambda0), _ptr(lam_mod),
+                                   _ptr(g_cum), _ptr(beta), _ptr(lambda_end), _ptr(ws),
+                                   ws.numel(), _stream(stream)))
 
 
 def cyfa_chunk_fwd(d, q, k, v, lam_mod, g_cum, beta, R, Kbar0, Vbar0, o, Kbar_out, Vbar_out, ws,
@@ -215,6 +235,32 @@ def prepare(d, clock_logit, decay_logit, beta_logit, A, lambda0=None, want_lambd
     lend = torch.empty(B, H, dtype=torch.float64, device=dev) if want_lambda_end else None
     ws = workspace(d, CYFA_WS_PREPARE, dev)
     cyfa_prepare(d, clock_logit, decay_logit, beta_logit, A, lambda0, lam, g, beta, lend, ws)
+    return lam, g, beta, lend
+
+
+def prepare_varlen(d, cu_seqlens, decay_logit, beta_logit, A, clock_logit=None, rho=0.0,
+                   lambda0=None, want_lambda_end=False):
+    B, T, H = decay_logit.shape
+    dev = decay_logit.device
+    nseq = cu_seqlens.numel() - 1
+    lam = torch.empty(B, T, H, dtype=torch.float32, device=dev)
+    g = torch.empty_like(lam)
+    beta = torch.empty_like(lam)
+    lend = torch.empty(nseq, H, dtype=torch.float64, device=dev) if want_lambda_end else None
+    ws = workspace(d, CYFA_WS_PREPARE_VARLEN, dev)
+    cyfa_prepare_varlen(d, cu_seqlens, nseq, clock_logit, rho, decay_logit, beta_logit, A,
+                        lambda0, lam, g, beta, lend, ws)
+    return lam, g, beta, lend
+
+
+def prepare_fixed_rate(d, rho, decay_logit, beta_logit, A, lambda0=None, want_lambda_end=False):
+    B, T, H = decay_logit.shape
+    dev = decay_logit.device
+    lam = torch.empty(B, T, H, dtype=torch.float32, device=dev)
+    g = torch.empty_like(lam)
+    beta = torch.empty_like(lam)
+    lend = torch.empty(B, H, dtype=torch.float64, device=dev) if want_lambda_end else None
+    cyfa_prepare_fixed_rate(d, rho, decay_logit, beta_logit, A, lambda0, lam, g, beta, lend)
     return lam, g, beta, lend
 
 

@@ -73,3 +73,21 @@ def make_inputs(B, T, H, d, *, seed=0, dtype=torch.bfloat16, device='cpu', with_
 def pair_view(x, b, h):
     """Slice one (batch, head) sequence out of a [B, T, H, ...] tensor as float64 numpy."""
     return x[b, :, h].detach().to('cpu', torch.float64).numpy()
+
+
+def varlen_lengths(total, mean, *, seed=0, sigma=0.75, max_len=None):
+    """Lengths of the sequences of one packed stream of `total` tokens: log-normal around `mean`
+    (log-space spread sigma), each at least 1 and at most max_len, the last one taking what is
+    left so that they sum to `total`.  A stand-in for a batch of documents of mixed length."""
+    g = torch.Generator(device='cpu').manual_seed(seed + 104729)
+    mu = math.log(mean) - 0.5 * sigma * sigma
+    out, used = [], 0
+    while used < total:
+        x = math.exp(mu + sigma * float(torch.randn(1, generator=g)))
+        n = max(1, int(round(x)))
+        if max_len:
+            n = min(n, max_len)
+        n = min(n, total - used)
+        out.append(n)
+        used += n
+    return out

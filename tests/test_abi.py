@@ -107,3 +107,36 @@ def test_noalloc_prepare_checks_dims_like_prepare(lib, field, value, code):
     args = [good] * 4 + [None] + [good] * 3 + [None, None]
     assert lib.cyfa_prepare_noalloc(ctypes.byref(d), *args) == code
     assert lib.cyfa_prepare(ctypes.byref(d), *args[:9], good, 1 << 30, None) == code
+
+
+def test_fixed_rate_and_varlen_prepare_check_arguments_on_host(lib):
+    """Host-side refusals of cyfa_prepare_fixed_rate and cyfa_prepare_varlen (nothing launched)."""
+    good = ctypes.c_void_p(0x1000)      # never dereferenced: rejected before any launch
+    d = cyfa.dims(1, 128, 1, 128)
+    for rho in (0.0, -1.0, float('nan')):
+        assert lib.cyfa_prepare_fixed_rate(ctypes.byref(d), rho, *([good] * 3), None,
+                                           *([good] * 3), None, None) == cyfa.CYFA_ERR_ARG
+    n = ctypes.c_size_t()
+    assert lib.cyfa_workspace_size(ctypes.byref(d), cyfa.CYFA_WS_PREPARE_VARLEN,
+                                   ctypes.byref(n)) == 0 and n.value > 0
+
+    def varlen(dd, nseq=2, clock=good, rho=0.0, ws_bytes=1 << 20):
+        return lib.cyfa_prepare_varlen(ctypes.byref(dd), good, nseq, clock, rho, good, good, good,
+                                       None, good, good, good, None, good, ws_bytes, None)
+    assert varlen(cyfa.dims(2, 128, 1, 128)) == cyfa.CYFA_ERR_ARG          # B must be 1
+    assert varlen(d, nseq=0) == cyfa.CYFA_ERR_ARG
+    assert varlen(d, clock=None, rho=0.0) == cyfa.CYFA_ERR_ARG              # no clock, no rate
+    assert varlen(d, ws_bytes=8) == cyfa.CYFA_ERR_WORKSPACE
+    assert varlen(cyfa.dims(1, 100, 1, 128)) == cyfa.CYFA_ERR_SHAPE
+
+
+def test_backward_clock_gradient_both_or_neither(lib):
+    """cyfa_chunk_bwd takes no clock logits only together with no clock gradient."""
+    good = ctypes.c_void_p(0x1000)
+    d = cyfa.dims(1, 128, 1, 128)
+    args = [good] * 21
+    args[7] = None      # clock_logit missing, d_clock_logit given
+    assert lib.cyfa_chunk_bwd(ctypes.byref(d), *args, 1 << 30, None) == cyfa.CYFA_ERR_ARG
+    args = [good] * 21
+    args[14] = None     # d_clock_logit missing, clock_logit given
+    assert lib.cyfa_chunk_bwd(ctypes.byref(d), *args, 1 << 30, None) == cyfa.CYFA_ERR_ARG

@@ -63,7 +63,8 @@ def _dA_terms(inp, ref, pairs, H):
 
 @pytest.mark.parametrize('cuda_cores', [False, True])
 @pytest.mark.parametrize('B,T,H,D,C', [(2, 256, 2, 128, 64), (1, 384, 3, 64, 64),
-                                       (1, 512, 2, 128, 128), (1, 2304, 2, 128, 64)])
+                                       (1, 512, 2, 128, 128), (1, 2304, 2, 128, 64),
+                                       (1, 256, 2, 256, 64)])
 def test_backward_small_bf16(B, T, H, D, C, cuda_cores):
     """Tensor-core kernels (bf16, d = 128, T a multiple of 128) and the CUDA-core kernels;
     T = 2304 spans several 1024-token segments plus a partial one."""
@@ -164,3 +165,15 @@ def test_backward_full_size_dA_dR(B, T, H, saved):
     assert_close_rel(dR[hs], dR_ref[hs], 'dR')
     others = [h for h in range(H) if h not in hs]
     assert np.all(dA[others] == 0) and np.all(dR[others] == 0)
+
+
+def test_backward_paper_kernel_shape_sampled():
+    """The paper's kernel-latency shape (H = 4, d_k = d_v = 256, T = 2048, B = 32): all
+    gradients of sampled (b, h) sequences against the oracle."""
+    B, T, H = 32, 2048, 4
+    inp = synth.make_inputs(B, T, H, 256, seed=0, device='cuda', with_dO=True)
+    d = cyfa.dims(B, T, H, 256, chunk=64)
+    out = gpu_backward(d, inp, want_dA=False)
+    pairs = sample_pairs(B, H, 2)
+    ref = oracle_backward(oracle_inputs(inp, pairs), pairs_np(inp['dO'], pairs))
+    _compare(out, ref, pairs, assert_close_bf16, 'paper shape')

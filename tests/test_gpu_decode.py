@@ -29,7 +29,8 @@ def _decode(inp, T0, steps, d_prefill, d_step):
     return torch.stack(outs, 1), K, V, lam
 
 
-@pytest.mark.parametrize('dtype,D', [(torch.bfloat16, 128), (torch.float32, 64)])
+@pytest.mark.parametrize('dtype,D', [(torch.bfloat16, 128), (torch.float32, 64),
+                                     (torch.bfloat16, 256), (torch.float32, 256)])
 def test_decode_small(dtype, D):
     B, H, T0, steps = 2, 3, 128, 24
     inp = synth.make_inputs(B, T0 + steps, H, D, seed=6, dtype=dtype, device='cuda')

@@ -68,7 +68,8 @@ def test_fp32_config_parity():
 @pytest.mark.parametrize('B,T,H,D,C', [(2, 384, 3, 128, 64), (1, 512, 2, 128, 128),
                                        (3, 256, 1, 64, 128), (1, 64, 1, 128, 64),
                                        (1, 2304, 2, 128, 64), (1, 128, 2, 128, 64),
-                                       (2, 1152, 2, 128, 64)])
+                                       (2, 1152, 2, 128, 64), (2, 256, 2, 256, 64),
+                                       (1, 384, 2, 256, 128)])
 def test_bf16_forward_small(B, T, H, D, C, cuda_cores):
     """Tensor-core kernels (bf16, d = 128, T a multiple of 128) and the CUDA-core kernels;
     T = 2304 spans several 1024-token segments plus a partial one, T = 128 is a single chunk
@@ -83,6 +84,29 @@ def test_bf16_forward_small(B, T, H, D, C, cuda_cores):
     Kg = np.stack([Ko[b, h].double().cpu().numpy() for b, h in pairs])
     assert_close_bf16(Kg[:, :127], Kb, 'Kbar')
     assert np.all(Kg[:, 127] == 0)
+
+
+def test_fp32_d256_parity():
+    """fp32 at d = 256 (the paper's head size), 128-token caller chunks: within 1e-4."""
+    inp = to_device(synth.make_inputs(1, 384, 2, 256, seed=12, dtype=torch.float32))
+    d = cyfa.dims(1, 384, 2, 256, chunk=128, dtype=torch.float32)
+    o, Ko, Vo, _ = gpu_forward(d, inp, want_state=True)
+    pairs = [(0, 0), (0, 1)]
+    o_ref, Kb, Vb, _ = oracle_forward(oracle_inputs(inp, pairs))
+    assert_close_fp32(pairs_np(o, pairs), o_ref, 'o')
+    assert_close_fp32(Vo[0].double().cpu().numpy()[:, :127], Vb, 'Vbar')
+
+
+def test_paper_kernel_shape_forward_sampled():
+    """The paper's kernel-latency shape (H = 4, d_k = d_v = 256, T = 2048, B = 32): every output
+    of sampled (b, h) sequences against the oracle."""
+    B, T, H, D = 32, 2048, 4, 256
+    inp = synth.make_inputs(B, T, H, D, seed=0, device='cuda')
+    d = cyfa.dims(B, T, H, D, chunk=64)
+    o, _, _, _ = gpu_forward(d, inp)
+    pairs = sample_pairs(B, H, 3)
+    o_ref = oracle_forward(oracle_inputs(inp, pairs))[0]
+    assert_close_bf16(pairs_np(o.float(), pairs), o_ref, 'o')
 
 
 def test_stress_scale_and_identity_readout():
