@@ -413,9 +413,10 @@ def run_ours(args):
         varlen = run_varlen(args, dev, rank)
 
     # the paper's own kernel shape (H = 4, d = 256, T = 2048, B = 32)
-    paper = None
+    paper = slots = None
     if not args.no_paper_shape:
         paper = run_paper_shape(args, dev, rank, peaks)
+        slots = run_slots_variant(args, dev, rank, peaks)
 
     # end to end through the public API with host buffers
     e2e = None
@@ -437,7 +438,7 @@ def run_ours(args):
         'roofline': roof, 'kernel_rooflines': rooflines, 'cpu_baseline': cpu, 'e2e': e2e, 'gpu_launches': launches,
         'clocks': clk, 'tensor_frac': tensor_frac, 'fwd': fwd, 'bwd': bwd,
         'prepare_ms': prep_ms, 'kernel_ms_per_step': step_ms_kernels, 'decode': dec,
-        'varlen': varlen, 'paper_shape': paper,
+        'varlen': varlen, 'paper_shape': paper, 'slots_m63': slots,
         'kernels': per_kernel,
     }
     if rank == 0:
@@ -512,17 +513,28 @@ def run_decode(args, dev, peaks, rank):
 def run_paper_shape(args, dev, rank, peaks):
     """prepare + forward + backward (every gradient) at the shape of the paper's kernel-latency
     figure: B = 32, T = 2048, H = 4, d_k = d_v = 256, m = 127, bf16 inputs."""
+    return run_extra_shape(args, dev, rank, peaks, 32, 2048, 4, 256, 127,
+                           "the paper's kernel-latency shape")
+
+
+def run_slots_variant(args, dev, rank, peaks):
+    """The same step on the 1.4B-shaped layer with m = 63 slots (the paper's slot ablation)."""
+    return run_extra_shape(args, dev, rank, peaks, LAYER['B'], LAYER['T'], LAYER['H'],
+                           LAYER['d'], 63, 'the 1.4B layer with m = 63 (slot ablation)')
+
+
+def run_extra_shape(args, dev, rank, peaks, B, T, H, D, m, what):
     import torch
     from paper_2609_36259_gb300 import cyfa, synth
-    B, T, H, D, C = 32, 2048, 4, 256, 64
-    inp = synth.make_inputs(B, T, H, D, seed=4000 + rank, device=dev, with_dO=True)
-    d = cyfa.dims(B, T, H, D, chunk=C)
+    C = 64
+    inp = synth.make_inputs(B, T, H, D, seed=4000 + rank, device=dev, with_dO=True, m=m)
+    d = cyfa.dims(B, T, H, D, chunk=C, m=m)
     f32 = dict(dtype=torch.float32, device=dev)
     lam, g, beta = (torch.empty(B, T, H, **f32) for _ in range(3))
     o = torch.empty_like(inp['v'])
     dq, dk, dv = (torch.empty_like(inp[x]) for x in ('q', 'k', 'v'))
     dc, dd, db = (torch.empty_like(lam) for _ in range(3))
-    dA, dR = torch.empty(H, **f32), torch.empty(H, 127, 127, **f32)
+    dA, dR = torch.empty(H, **f32), torch.empty(H, m, m, **f32)
     ws = [cyfa.workspace(d, w, dev) for w in (cyfa.CYFA_WS_PREPARE, cyfa.CYFA_WS_FWD,
                                                cyfa.CYFA_WS_BWD)]
 
@@ -555,11 +567,11 @@ def run_paper_shape(args, dev, rank, peaks):
     ms_fwd = timed(fwd, n)
     cyfa.cyfa_check()
     th = B * T * H
-    fl = operator_flops_per_token_head(C, d=D) * th
+    fl = operator_flops_per_token_head(C, d=D, ms=m + 1) * th
     alu = fp32_alu_peak_tflops(peaks['sm_max_mhz'])
-    return {'workload': 'B=%d T=%d H=%d d=%d chunk %d (the paper\'s kernel-latency shape), '
-                        'prepare + fwd + bwd with every gradient' % (B, T, H, D, C),
-            'path': 'fp32 CUDA-core kernels (the tensor-core kernels take d = 128)',
+    return {'workload': 'B=%d T=%d H=%d d=%d m=%d chunk %d (%s), prepare + fwd + bwd with every '
+                        'gradient' % (B, T, H, D, m, C, what),
+            'path': 'fp32 CUDA-core kernels (the tensor-core kernels take d = 128, m = 127)',
             'ms_per_step': ms, 'tokens_per_s': B * T / (ms / 1e3),
             'fwd_ms': ms_fwd, 'fwd_tokens_per_s': B * T / (ms_fwd / 1e3),
             'tflops_rule': 3 * fl / (ms / 1e3) / 1e12,

@@ -14,31 +14,33 @@ namespace cyfa {
 namespace {
 
 // ---------------------------------------------------------------------------------------
-// M = R Phi (padded to 128 x 128 with a zero last row and column) and its transpose.
-// Phi is the real Fourier basis of App. A.1 Eq. app-real-fourier.
-__global__ void __launch_bounds__(128) readout_matrix_kernel(const float* R, float* M, float* MT) {
+// M = R Phi (padded to 128 x 128 with zero rows and columns m..127) and its transpose.
+// Phi is the real Fourier basis of App. A.1 Eq. app-real-fourier; R is [H, m, m].
+__global__ void __launch_bounds__(128) readout_matrix_kernel(const float* R, float* M, float* MT,
+                                                             Slots sl) {
     const int h = blockIdx.y, i = blockIdx.x, col = threadIdx.x;
+    const int m = sl.m;
     __shared__ float srow[128], s_ct[MA], s_st[MA];
-    srow[col] = (i < MA && col < MA) ? R[((size_t)h * MA + i) * MA + col] : 0.f;
-    if (col < MA) {   // cos / sin of 2 pi x / m for x = 0 .. m-1 (the entries of Phi)
+    srow[col] = (i < m && col < m) ? R[((size_t)h * m + i) * m + col] : 0.f;
+    if (col < m) {   // cos / sin of 2 pi x / m for x = 0 .. m-1 (the entries of Phi)
         float sv, cv;
-        sincospif((float)col * (2.f / 127.f), &sv, &cv);
+        sincospif((float)col * sl.two_over_m, &sv, &cv);
         s_ct[col] = cv;
         s_st[col] = sv;
     }
     __syncthreads();
     float acc = 0.f;
-    if (i < MA && col < MA) {
+    if (i < m && col < m) {
         if (col == 0) {
-            for (int r = 0; r < MA; ++r) acc = fmaf(srow[r], INV_SQRT_M, acc);
+            for (int r = 0; r < m; ++r) acc = fmaf(srow[r], sl.inv_sqrt_m, acc);
         } else {
             const int j = (col + 1) >> 1;
             const float* tab = (col & 1) ? s_ct : s_st;
             int idx = 0;   // (j r) mod m
-            for (int r = 0; r < MA; ++r) {
-                acc = fmaf(srow[r], SQRT_2_OVER_M * tab[idx], acc);
+            for (int r = 0; r < m; ++r) {
+                acc = fmaf(srow[r], sl.sqrt2_over_m * tab[idx], acc);
                 idx += j;
-                if (idx >= MA) idx -= MA;
+                if (idx >= m) idx -= m;
             }
         }
     }
@@ -85,7 +87,7 @@ __global__ void __launch_bounds__(256) fwd_state_kernel(FwdArgs a) {
         stage_tok(sX, X, s, b, h, t0, C, xc0, 1.f);
         __syncthreads();
         const float gC = sg[C - 1];
-        build_write_rows(sA, LD, slam, sbeta, C, [&](int r) { return expf(gC - sg[r]); });
+        build_write_rows(sA, LD, slam, sbeta, C, s.sl, [&](int r) { return expf(gC - sg[r]); });
         __syncthreads();
         const float decay = expf(gC);
 #pragma unroll
@@ -133,7 +135,7 @@ __global__ void __launch_bounds__(256) fwd_out_kernel(FwdArgs a) {
     load_gates(s, a.lam, a.g, a.beta, b, h, t0, C, slam, sg, sbeta);
     __syncthreads();
     for (int r = threadIdx.x; r < C; r += blockDim.x) seg[r] = expf(sg[r]);
-    build_write_rows(sA, LD, slam, sbeta, C, [](int) { return 1.f; });
+    build_write_rows(sA, LD, slam, sbeta, C, s.sl, [](int) { return 1.f; });
 
     // P = (s Q K^T) o Gamma
     float acc[TM][TM];
@@ -181,7 +183,7 @@ __global__ void __launch_bounds__(256) fwd_out_kernel(FwdArgs a) {
         for (int j = 0; j < 8; ++j) sX[(ty + 16 * i) * LD + tx + 16 * j] = o1[i][j];
     __syncthreads();
 
-    middle_rows(sX, slam, C, a.M + (size_t)h * MS * MS, a.MT + (size_t)h * MS * MS, swarp);
+    middle_rows(sX, slam, C, a.M + (size_t)h * MS * MS, a.MT + (size_t)h * MS * MS, swarp, s.sl);
     __syncthreads();
 
     // P = (O'' A^T) o Gamma
@@ -251,8 +253,9 @@ cudaError_t fwd_dispatch(const FwdArgs& a, cudaStream_t st) {
 
 }  // namespace
 
-cudaError_t launch_readout_matrix(int H, const float* R, float* M, float* MT, cudaStream_t st) {
-    { LaunchScope ls_("readout_matrix", st); readout_matrix_kernel<<<dim3(MS, H), 128, 0, st>>>(R, M, MT); }
+cudaError_t launch_readout_matrix(int H, const float* R, float* M, float* MT, const Slots& sl,
+                                  cudaStream_t st) {
+    { LaunchScope ls_("readout_matrix", st); readout_matrix_kernel<<<dim3(MS, H), 128, 0, st>>>(R, M, MT, sl); }
     return cudaGetLastError();
 }
 

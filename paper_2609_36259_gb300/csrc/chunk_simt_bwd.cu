@@ -26,16 +26,20 @@ constexpr int CB = BWD_C;          // 64
 constexpr int LPB = CB + 1;
 constexpr int TMB = CB / 16;       // 4 rows per thread
 
-__device__ __forceinline__ float freq(int j) { return (6.283185307179586f / 127.f) * (float)j; }
+// 2 pi j / m, the rotation rate of pair j
+__device__ __forceinline__ float freq(int j, const Slots& sl) {
+    return (6.283185307179586f * sl.inv_m) * (float)j;
+}
 
 // <x, Omega y> for 128-vectors in shared memory, summed over the warp (pairs j = lane+1, lane+33).
-__device__ __forceinline__ float warp_omega_dot(const float* x, const float* y, int lane) {
+__device__ __forceinline__ float warp_omega_dot(const float* x, const float* y, int lane,
+                                                const Slots& sl) {
     float acc = 0.f;
 #pragma unroll
     for (int u = 0; u < 2; ++u) {
         const int j = lane + 1 + 32 * u;
-        if (j <= NPAIR)
-            acc += freq(j) * (x[2 * j] * y[2 * j - 1] - x[2 * j - 1] * y[2 * j]);
+        if (j <= sl.npair)
+            acc += freq(j, sl) * (x[2 * j] * y[2 * j - 1] - x[2 * j - 1] * y[2 * j]);
     }
     return warp_sum(acc);
 }
@@ -48,7 +52,7 @@ __device__ __noinline__ void middle_rows_bwd(const float* sO1, const float* sO2,
                                              const float* slam, int C, const float* M,
                                              const float* MT, float* swarp, float* sdG,
                                              float* sdL, float* gz, float* gp, float* gdy,
-                                             float* gdl) {
+                                             float* gdl, const Slots& sl) {
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     float* z = swarp + warp * 640;
     float* p = z + 128;
@@ -66,14 +70,17 @@ __device__ __noinline__ void middle_rows_bwd(const float* sO1, const float* sO2,
             const int j = lane + 1 + 32 * u;
             cs[u] = 1.f;
             sn[u] = 0.f;
-            if (j <= NPAIR) {
-                sincospif(phase_pi(lam, j), &sn[u], &cs[u]);
+            if (j <= sl.npair) {
+                sincospif(phase_pi_m(lam, j, sl), &sn[u], &cs[u]);
                 const float xc = x1[2 * j - 1], xs = x1[2 * j];
                 z[2 * j - 1] = cs[u] * xc - sn[u] * xs;
                 z[2 * j] = sn[u] * xc + cs[u] * xs;
                 const float gc = xd[2 * j - 1], gs = xd[2 * j];
                 dy[2 * j - 1] = cs[u] * gc - sn[u] * gs;     // dy = U(lam) do''
                 dy[2 * j] = sn[u] * gc + cs[u] * gs;
+            } else if (j <= NPAIR) {   // padding slots (zero)
+                z[2 * j - 1] = z[2 * j] = 0.f;
+                dy[2 * j - 1] = dy[2 * j] = 0.f;
             }
         }
         if (lane == 0) {
@@ -87,7 +94,7 @@ __device__ __noinline__ void middle_rows_bwd(const float* sO1, const float* sO2,
 #pragma unroll
         for (int u = 0; u < 4; ++u) g1 += x2[lane + 32 * u] * xd[lane + 32 * u];
         g1 = warp_sum(g1);
-        const float om2 = warp_omega_dot(xd, x2, lane);      // <do'', Omega o''>
+        const float om2 = warp_omega_dot(xd, x2, lane, sl);  // <do'', Omega o''>
         // logits and softmax
         float l[4] = {0.f, 0.f, 0.f, 0.f}, dp[4] = {0.f, 0.f, 0.f, 0.f};
         for (int k = 0; k < MS; ++k) {
@@ -99,7 +106,9 @@ __device__ __noinline__ void middle_rows_bwd(const float* sO1, const float* sO2,
                 dp[u] = fmaf(mt, dyk, dp[u]);           // dp = M dy
             }
         }
-        if (lane == 31) l[3] = -INFINITY;
+#pragma unroll
+        for (int u = 0; u < 4; ++u)
+            if (lane + 32 * u >= sl.m) l[u] = -INFINITY;
         float mx = warp_max(fmaxf(fmaxf(l[0], l[1]), fmaxf(l[2], l[3])));
         float e[4], sum = 0.f;
 #pragma unroll
@@ -130,7 +139,7 @@ __device__ __noinline__ void middle_rows_bwd(const float* sO1, const float* sO2,
         }
         __syncwarp();
         float g[4] = {0.f, 0.f, 0.f, 0.f};                   // dz = M^T dl
-        for (int i = 0; i < MA; ++i) {
+        for (int i = 0; i < sl.m; ++i) {
             const float di = dl[i];
 #pragma unroll
             for (int u = 0; u < 4; ++u) g[u] = fmaf(M[i * MS + lane + 32 * u], di, g[u]);
@@ -138,7 +147,7 @@ __device__ __noinline__ void middle_rows_bwd(const float* sO1, const float* sO2,
 #pragma unroll
         for (int u = 0; u < 4; ++u) dz[lane + 32 * u] = g[u];
         __syncwarp();
-        const float om1 = warp_omega_dot(dz, z, lane);       // <dz, Omega z>
+        const float om1 = warp_omega_dot(dz, z, lane, sl);   // <dz, Omega z>
         // do' = U(-lam) dz
 #pragma unroll
         for (int u = 0; u < 2; ++u) {
@@ -286,7 +295,7 @@ __global__ void __launch_bounds__(256) bwd_intra1_kernel(BwdArgs a) {
     load_gates(s, a.lam, a.g, a.beta, b, h, t0, CB, slam, sg, sbeta);
     __syncthreads();
     for (int r = threadIdx.x; r < CB; r += blockDim.x) seg[r] = expf(sg[r]);
-    build_write_rows(sA, LD, slam, sbeta, CB, [](int) { return 1.f; });
+    build_write_rows(sA, LD, slam, sbeta, CB, s.sl, [](int) { return 1.f; });
 
     // O' = s gamma o (Q Kbar^T) + (s Q K^T o Gamma) A
     masked_scores_tok(sP, sS, sg, Q, K, s, b, h, t0, s.scale);
@@ -309,7 +318,7 @@ __global__ void __launch_bounds__(256) bwd_intra1_kernel(BwdArgs a) {
             }
     }
     __syncthreads();
-    middle_rows(sO2, slam, CB, Mh, MTh, swarp);
+    middle_rows(sO2, slam, CB, Mh, MTh, swarp, s.sl);
 
     // dO'' = gamma o (dO Vbar^T) + (dO V^T o Gamma) A
     masked_scores_tok(sP, sS, sg, dO, V, s, b, h, t0, 1.f);
@@ -334,7 +343,7 @@ __global__ void __launch_bounds__(256) bwd_intra1_kernel(BwdArgs a) {
         const bool dr = a.mZ != nullptr;
         middle_rows_bwd(sO1, sO2, sD, slam, CB, Mh, MTh, swarp, sdG, sdL,
                         dr ? a.mZ + rowbase : nullptr, dr ? a.mP + rowbase : nullptr,
-                        dr ? a.mDY + rowbase : nullptr, dr ? a.mDL + rowbase : nullptr);
+                        dr ? a.mDY + rowbase : nullptr, dr ? a.mDL + rowbase : nullptr, s.sl);
     }
     __syncthreads();
 
@@ -474,7 +483,7 @@ __global__ void __launch_bounds__(256) bwd_intra2_kernel(BwdArgs a) {
         sfw[r] = expf(sg[CB - 1] - sg[r]);
         sdG[r] = 0.f;
     }
-    build_write_rows(sA, LD, slam, sbeta, CB, [](int) { return 1.f; });
+    build_write_rows(sA, LD, slam, sbeta, CB, s.sl, [](int) { return 1.f; });
     __syncthreads();
 
     // dK = P3^T (s Q) + diag(fw) A D^K,  P3 = (dO' A^T) o Gamma
@@ -579,7 +588,7 @@ __global__ void __launch_bounds__(256) bwd_intra2_kernel(BwdArgs a) {
 #pragma unroll
         for (int u = 0; u < 4; ++u) db += da[lane + 32 * u] * av[lane + 32 * u];
         db = warp_sum(db);
-        const float om = warp_omega_dot(da, av, lane);       // <da, Omega a>
+        const float om = warp_omega_dot(da, av, lane, s.sl); // <da, Omega a>
         if (lane == 0) {
             const size_t gi = tokbase + (size_t)t * s.H;
             a.tok[2 * BTH + gi] = sdG[t];
@@ -770,7 +779,7 @@ cudaError_t bwd_dispatch(const BwdArgs& a, cudaStream_t st) {
     { LaunchScope ls_("bwd_intra2", st); k2<<<gchunk, 256, sm2, st>>>(a); }
     if (a.dR) {
         { LaunchScope ls_("bwd_dm_reduce", st); dm_reduce_simt<<<dim3(s.H, MS), 128, 0, st>>>(a); }
-        e = launch_dr_finalize(a.dM, 1, s.H, false, a.dR, st);
+        e = launch_dr_finalize(a.dM, 1, s.H, false, a.dR, s.sl, st);
         if (e != cudaSuccess) return e;
     }
     return launch_bwd_gates(a, st);

@@ -5,6 +5,8 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include "kernels.h"
+
 namespace cyfa {
 
 constexpr int MS = 128;        // storage rows per state (m* = m + 1)
@@ -33,26 +35,44 @@ __device__ __forceinline__ float phase_pi(float lam, int j) {
     return r * (2.f / 127.f);
 }
 
+// phase_pi for m active slots (the same arithmetic with m in place of 127; identical values at
+// m = 127): lam in [0, m), theta_j = 2 pi j lam / m = pi * phase_pi_m(lam, j, sl).
+__device__ __forceinline__ float phase_pi_m(float lam, int j, const Slots& sl) {
+    const float hi = rintf(lam * 256.f) * (1.f / 256.f);
+    const float lo = lam - hi;
+    const float jh = (float)j * hi;
+    const float qn = floorf(jh * sl.inv_m);
+    float r = fmaf(-qn, sl.fm, jh);
+    if (r < 0.f) r += sl.fm;
+    else if (r >= sl.fm) r -= sl.fm;
+    r = fmaf((float)j, lo, r);
+    return r * sl.two_over_m;
+}
+
 // Temporal write-vector entries for one token: a = beta * U(-lam) b (Sec. 3.2), with
 // b = [1/sqrt(m), sqrt(2/m), 0, sqrt(2/m), 0, ...] (App. A.1 Eq. app-b-explicit), so
-// a[0] = beta/sqrt(m), a[2j-1] = beta sqrt(2/m) cos(theta_j), a[2j] = -beta sqrt(2/m) sin(theta_j),
-// and the padding entry a[127] = 0 (App. A.7).
+// a[0] = beta/sqrt(m), a[2j-1] = beta sqrt(2/m) cos(theta_j), a[2j] = -beta sqrt(2/m) sin(theta_j)
+// for j <= (m-1)/2, and the padding entries a[m..127] = 0 (App. A.7).
 // Fills rows r < C of a row-major [C][ld] shared array; row r is scaled by sc[r] * beta[r].
 template <class ScaleFn>
 __device__ __forceinline__ void build_write_rows(float* sA, int ld, const float* slam,
-                                                 const float* sbeta, int C, ScaleFn scale_of) {
+                                                 const float* sbeta, int C, const Slots& sl,
+                                                 ScaleFn scale_of) {
     for (int e = threadIdx.x; e < C * 64; e += blockDim.x) {
         const int r = e >> 6, j = e & 63;
         const float sc = sbeta[r] * scale_of(r);
         if (j == 0) {
-            sA[r * ld] = sc * INV_SQRT_M;
+            sA[r * ld] = sc * sl.inv_sqrt_m;
             sA[r * ld + 127] = 0.f;
-        } else {
+        } else if (j <= sl.npair) {
             float s, c;
-            sincospif(phase_pi(slam[r], j), &s, &c);
-            const float w = sc * SQRT_2_OVER_M;
+            sincospif(phase_pi_m(slam[r], j, sl), &s, &c);
+            const float w = sc * sl.sqrt2_over_m;
             sA[r * ld + 2 * j - 1] = w * c;
             sA[r * ld + 2 * j] = -w * s;
+        } else {
+            sA[r * ld + 2 * j - 1] = 0.f;
+            sA[r * ld + 2 * j] = 0.f;
         }
     }
 }

@@ -37,7 +37,10 @@ int cyfa::check_dims(const cyfa_dims_t* d, bool need_T) {
     if (d->B <= 0 || d->H <= 0 || d->dk <= 0 || d->dv <= 0 || (need_T && d->T <= 0))
         return CYFA_ERR_ARG;
     if (d->dtype != CYFA_DTYPE_BF16 && d->dtype != CYFA_DTYPE_FP32) return CYFA_ERR_ARG;
-    if (d->m != 127) return CYFA_ERR_SHAPE;
+    // m: odd, 1..127 (128 storage rows); the paper's m = 255 needs 256 rows, which this build
+    // does not implement
+    if (d->m == 255) return CYFA_ERR_UNSUPPORTED;
+    if (d->m < 1 || d->m > 127 || d->m % 2 == 0) return CYFA_ERR_SHAPE;
     if (d->dk != d->dv || (d->dk != 64 && d->dk != 128 && d->dk != 256)) return CYFA_ERR_SHAPE;
     if ((long long)d->B * d->H > kMaxSequences) return CYFA_ERR_SHAPE;
     if (need_T) {
@@ -59,6 +62,7 @@ Shape shape_of(const cyfa_dims_t* d) {
     s.Cg = d->chunk;
     s.scale = d->scale;
     s.bf16 = d->dtype == CYFA_DTYPE_BF16;
+    s.sl = make_slots(d->m);
     return s;
 }
 
@@ -171,7 +175,7 @@ const char* cyfa_error_string(int code) {
     switch (code) {
         case CYFA_OK: return "ok";
         case CYFA_ERR_ARG: return "invalid argument (null pointer or non-positive size)";
-        case CYFA_ERR_SHAPE: return "unsupported shape (m must be 127, dk == dv in {64,128,256}, chunk in {64,128}, T % chunk == 0, B*H <= 65535)";
+        case CYFA_ERR_SHAPE: return "unsupported shape (m odd in 1..127, dk == dv in {64,128,256}, chunk in {64,128}, T % chunk == 0, B*H <= 65535)";
         case CYFA_ERR_ALIGN: return "tensor pointer not 16-byte aligned";
         case CYFA_ERR_WORKSPACE: return "workspace missing or too small";
         case CYFA_ERR_CUDA: return "CUDA runtime error";
@@ -306,7 +310,7 @@ int cyfa_chunk_fwd(const cyfa_dims_t* dims, const void* q, const void* k, const 
     const FwdLayout L = fwd_layout(s, tc_path, workspace);
     cudaStream_t st = static_cast<cudaStream_t>(stream);
     rc = cuda_status(tc_path ? launch_readout_f16(s.H, R, L.Mb, st)
-                             : launch_readout_matrix(s.H, R, L.M, L.MT, st));
+                             : launch_readout_matrix(s.H, R, L.M, L.MT, s.sl, st));
     if (rc) return rc;
     if (tc_path) {
         TcFwdArgs t;
@@ -370,7 +374,7 @@ int cyfa_chunk_bwd(const cyfa_dims_t* dims, const void* q, const void* k, const 
     const BwdLayout L = bwd_layout(s, tc_path, workspace);
     cudaStream_t st = static_cast<cudaStream_t>(stream);
     rc = cuda_status(tc_path ? launch_readout_f16(s.H, R, L.Mb, st)
-                             : launch_readout_matrix(s.H, R, L.M, L.MT, st));
+                             : launch_readout_matrix(s.H, R, L.M, L.MT, s.sl, st));
     if (rc) return rc;
     BwdArgs a;
     a.s = s;
@@ -478,6 +482,7 @@ int cyfa_step(const cyfa_dims_t* dims, const void* q, const void* k, const void*
     a.D = dims->dk;
     a.scale = dims->scale;
     a.bf16 = dims->dtype == CYFA_DTYPE_BF16;
+    a.sl = make_slots(dims->m);
     a.q = q;
     a.k = k;
     a.v = v;

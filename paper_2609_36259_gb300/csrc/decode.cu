@@ -19,12 +19,39 @@ namespace {
 constexpr int G = 4;          // batch rows per block
 constexpr int BATCH = 8;      // rows loaded per warp before they are used
 
+// A lane's VPL consecutive floats of a state row (VPL = 2, 4 or 8), by 8- or 16-byte accesses.
+template <int VPL>
+__device__ __forceinline__ void load_row(float (&x)[VPL], const float* p) {
+    if constexpr (VPL == 2) {
+        const float2 t = *reinterpret_cast<const float2*>(p);
+        x[0] = t.x; x[1] = t.y;
+    } else {
+#pragma unroll
+        for (int u = 0; u < VPL; u += 4) {
+            const float4 t = *reinterpret_cast<const float4*>(p + u);
+            x[u] = t.x; x[u + 1] = t.y; x[u + 2] = t.z; x[u + 3] = t.w;
+        }
+    }
+}
+template <int VPL>
+__device__ __forceinline__ void store_row(float* p, const float (&x)[VPL]) {
+    if constexpr (VPL == 2) {
+        *reinterpret_cast<float2*>(p) = make_float2(x[0], x[1]);
+    } else {
+#pragma unroll
+        for (int u = 0; u < VPL; u += 4)
+            *reinterpret_cast<float4*>(p + u) = make_float4(x[u], x[u + 1], x[u + 2], x[u + 3]);
+    }
+}
+
 template <int D, typename TI>
 __global__ void __launch_bounds__(256) step_kernel(StepArgs a) {
     constexpr int VPL = D / 32;   // floats per lane per state row
     const int h = blockIdx.y, b0 = blockIdx.x * G;
     const int ng = min(G, a.B - b0);
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const Slots sl = a.sl;
+    const int m = sl.m;
     __shared__ float s_ct[MA], s_st[MA];
     __shared__ float s_q[G][D], s_k[G][D], s_v[G][D];
     __shared__ float s_a[G][MS], s_o1[G][MS], s_z[G][MS], s_u[G][MS], s_l[G][MS], s_y[G][MS];
@@ -36,9 +63,9 @@ __global__ void __launch_bounds__(256) step_kernel(StepArgs a) {
     const TI* Q = (const TI*)a.q;
     const TI* K = (const TI*)a.k;
     const TI* V = (const TI*)a.v;
-    if (tid < MA) {
+    if (tid < m) {
         float s, c;
-        sincospif((float)tid * (2.f / 127.f), &s, &c);
+        sincospif((float)tid * sl.two_over_m, &s, &c);
         s_ct[tid] = c;
         s_st[tid] = s;
     }
@@ -57,22 +84,27 @@ __global__ void __launch_bounds__(256) step_kernel(StepArgs a) {
         if (g < ng) {
             const size_t bh = (size_t)(b0 + g) * a.H + h;
             const double lam_new = a.lambda[bh] + (double)sigmoidf_(a.clock_logit[bh]);
-            const float lam = (float)(lam_new - 127.0 * floor(lam_new / 127.0));
+            const float lam = (float)(lam_new - (double)m * floor(lam_new / (double)m));
             const float beta = sigmoidf_(a.beta_logit[bh]);
             if (j == 0) {
                 s_alpha[g] = expf(-a.A[h] * softplusf_(a.decay_logit[bh]));
                 s_lam[g] = lam_new;
-                s_a[g][0] = beta * INV_SQRT_M;
+                s_a[g][0] = beta * sl.inv_sqrt_m;
                 s_a[g][127] = 0.f;
                 s_cs[g][0] = 1.f;
                 s_sn[g][0] = 0.f;
-            } else {
+            } else if (j <= sl.npair) {
                 float s, c;
-                sincospif(phase_pi(lam, j), &s, &c);
+                sincospif(phase_pi_m(lam, j, sl), &s, &c);
                 s_cs[g][j] = c;
                 s_sn[g][j] = s;
-                s_a[g][2 * j - 1] = beta * SQRT_2_OVER_M * c;
-                s_a[g][2 * j] = -beta * SQRT_2_OVER_M * s;
+                s_a[g][2 * j - 1] = beta * sl.sqrt2_over_m * c;
+                s_a[g][2 * j] = -beta * sl.sqrt2_over_m * s;
+            } else {   // padding slots: no write, no rotation
+                s_cs[g][j] = 1.f;
+                s_sn[g][j] = 0.f;
+                s_a[g][2 * j - 1] = 0.f;
+                s_a[g][2 * j] = 0.f;
             }
         }
     }
@@ -96,13 +128,7 @@ __global__ void __launch_bounds__(256) step_kernel(StepArgs a) {
 #pragma unroll
             for (int bb = 0; bb < BATCH; ++bb) {
                 const int r = half + 2 * (i0 + bb);
-                if constexpr (VPL == 4) {
-                    const float4 t = *reinterpret_cast<const float4*>(Kb + r * D + lane * 4);
-                    x[bb][0] = t.x; x[bb][1] = t.y; x[bb][2] = t.z; x[bb][3] = t.w;
-                } else {
-                    const float2 t = *reinterpret_cast<const float2*>(Kb + r * D + lane * 2);
-                    x[bb][0] = t.x; x[bb][1] = t.y;
-                }
+                load_row<VPL>(x[bb], Kb + r * D + lane * VPL);
             }
 #pragma unroll
             for (int bb = 0; bb < BATCH; ++bb) {
@@ -114,12 +140,7 @@ __global__ void __launch_bounds__(256) step_kernel(StepArgs a) {
                     x[bb][u] = fmaf(alpha, x[bb][u], ar * kv[u]);
                     dot = fmaf(x[bb][u], qv[u], dot);
                 }
-                if constexpr (VPL == 4) {
-                    *reinterpret_cast<float4*>(Kb + r * D + lane * 4) =
-                        make_float4(x[bb][0], x[bb][1], x[bb][2], x[bb][3]);
-                } else {
-                    *reinterpret_cast<float2*>(Kb + r * D + lane * 2) = make_float2(x[bb][0], x[bb][1]);
-                }
+                store_row<VPL>(Kb + r * D + lane * VPL, x[bb]);
                 dot = warp_sum(dot);
                 if (lane == 0) s_o1[g][r] = dot;
             }
@@ -135,7 +156,7 @@ __global__ void __launch_bounds__(256) step_kernel(StepArgs a) {
             if (j == 0) {
                 s_z[g][0] = s_o1[g][0];
                 s_z[g][127] = 0.f;
-            } else {
+            } else {   // padding pairs have c = 1, sn = 0 and zero entries
                 const float c = s_cs[g][j], sn = s_sn[g][j];
                 const float xc = s_o1[g][2 * j - 1], xs = s_o1[g][2 * j];
                 s_z[g][2 * j - 1] = c * xc - sn * xs;
@@ -146,33 +167,33 @@ __global__ void __launch_bounds__(256) step_kernel(StepArgs a) {
     __syncthreads();
     for (int e = tid; e < G * MS; e += 256) {   // u_r = z_0/sqrt(m) + sqrt(2/m) sum_j (...)
         const int g = e >> 7, r = e & 127;
-        if (g < ng && r < MA) {
+        if (g < ng && r < m) {
             float acc = 0.f;
             int idx = 0;
-            for (int j = 1; j <= NPAIR; ++j) {
+            for (int j = 1; j <= sl.npair; ++j) {
                 idx += r;
-                if (idx >= MA) idx -= MA;
+                if (idx >= m) idx -= m;
                 acc = fmaf(s_z[g][2 * j - 1], s_ct[idx], acc);
                 acc = fmaf(s_z[g][2 * j], s_st[idx], acc);
             }
-            s_u[g][r] = s_z[g][0] * INV_SQRT_M + SQRT_2_OVER_M * acc;
+            s_u[g][r] = s_z[g][0] * sl.inv_sqrt_m + sl.sqrt2_over_m * acc;
         }
     }
     __syncthreads();
-    const float* Rh = a.R + (size_t)h * MA * MA;
-    for (int i = warp; i < MA; i += 8) {   // l_i = sum_r R[i][r] u_r, one R row per warp
+    const float* Rh = a.R + (size_t)h * m * m;
+    for (int i = warp; i < m; i += 8) {   // l_i = sum_r R[i][r] u_r, one R row per warp
         float rv[4];
 #pragma unroll
         for (int k = 0; k < 4; ++k) {
             const int r = lane + 32 * k;
-            rv[k] = r < MA ? Rh[i * MA + r] : 0.f;
+            rv[k] = r < m ? Rh[i * m + r] : 0.f;
         }
         for (int g = 0; g < ng; ++g) {
             float acc = 0.f;
 #pragma unroll
             for (int k = 0; k < 4; ++k) {
                 const int r = lane + 32 * k;
-                if (r < MA) acc = fmaf(rv[k], s_u[g][r], acc);
+                if (r < m) acc = fmaf(rv[k], s_u[g][r], acc);
             }
             acc = warp_sum(acc);
             if (lane == 0) s_l[g][i] = acc;
@@ -182,10 +203,10 @@ __global__ void __launch_bounds__(256) step_kernel(StepArgs a) {
     if (warp < ng) {
         const int g = warp;
         float mx = -INFINITY;
-        for (int i = lane; i < MA; i += 32) mx = fmaxf(mx, s_l[g][i]);
+        for (int i = lane; i < m; i += 32) mx = fmaxf(mx, s_l[g][i]);
         mx = warp_max(mx);
         float sum = 0.f;
-        for (int i = lane; i < MA; i += 32) {
+        for (int i = lane; i < m; i += 32) {
             const float e = expf(s_l[g][i] - mx);
             s_l[g][i] = e;
             sum += e;
@@ -196,11 +217,11 @@ __global__ void __launch_bounds__(256) step_kernel(StepArgs a) {
     __syncthreads();
     {   // y'_r = sum_i R[i][r] p_i, thread (r, half): rows g = half, half + 2
         const int r = tid & 127, half = tid >> 7;
-        if (r < MA) {
+        if (r < m) {
             float acc0 = 0.f, acc1 = 0.f;
             const int g0 = half, g1 = half + 2;
-            for (int i = 0; i < MA; ++i) {
-                const float rv = Rh[i * MA + r];
+            for (int i = 0; i < m; ++i) {
+                const float rv = Rh[i * m + r];
                 acc0 = fmaf(rv, s_l[g0][i], acc0);
                 acc1 = fmaf(rv, s_l[g1][i], acc1);
             }
@@ -214,19 +235,22 @@ __global__ void __launch_bounds__(256) step_kernel(StepArgs a) {
         if (g < ng) {
             if (j == 0) {
                 float ac = 0.f;
-                for (int r = 0; r < MA; ++r) ac += s_u[g][r];
-                s_y[g][0] = ac * INV_SQRT_M;
+                for (int r = 0; r < m; ++r) ac += s_u[g][r];
+                s_y[g][0] = ac * sl.inv_sqrt_m;
                 s_y[g][127] = 0.f;
+            } else if (j > sl.npair) {   // padding slots
+                s_y[g][2 * j - 1] = 0.f;
+                s_y[g][2 * j] = 0.f;
             } else {
                 float ac = 0.f, as = 0.f;
                 int idx = 0;
-                for (int r = 0; r < MA; ++r) {
+                for (int r = 0; r < m; ++r) {
                     ac = fmaf(s_u[g][r], s_ct[idx], ac);
                     as = fmaf(s_u[g][r], s_st[idx], as);
                     idx += j;
-                    if (idx >= MA) idx -= MA;
+                    if (idx >= m) idx -= m;
                 }
-                const float yc = SQRT_2_OVER_M * ac, ys = SQRT_2_OVER_M * as;
+                const float yc = sl.sqrt2_over_m * ac, ys = sl.sqrt2_over_m * as;
                 const float c = s_cs[g][j], sn = s_sn[g][j];
                 s_y[g][2 * j - 1] = c * yc + sn * ys;
                 s_y[g][2 * j] = -sn * yc + c * ys;
@@ -251,13 +275,7 @@ __global__ void __launch_bounds__(256) step_kernel(StepArgs a) {
 #pragma unroll
             for (int bb = 0; bb < BATCH; ++bb) {
                 const int r = half + 2 * (i0 + bb);
-                if constexpr (VPL == 4) {
-                    const float4 t = *reinterpret_cast<const float4*>(Vb + r * D + lane * 4);
-                    x[bb][0] = t.x; x[bb][1] = t.y; x[bb][2] = t.z; x[bb][3] = t.w;
-                } else {
-                    const float2 t = *reinterpret_cast<const float2*>(Vb + r * D + lane * 2);
-                    x[bb][0] = t.x; x[bb][1] = t.y;
-                }
+                load_row<VPL>(x[bb], Vb + r * D + lane * VPL);
             }
 #pragma unroll
             for (int bb = 0; bb < BATCH; ++bb) {
@@ -268,12 +286,7 @@ __global__ void __launch_bounds__(256) step_kernel(StepArgs a) {
                     x[bb][u] = fmaf(alpha, x[bb][u], ar * vv[u]);
                     oacc[u] = fmaf(x[bb][u], yr, oacc[u]);
                 }
-                if constexpr (VPL == 4) {
-                    *reinterpret_cast<float4*>(Vb + r * D + lane * 4) =
-                        make_float4(x[bb][0], x[bb][1], x[bb][2], x[bb][3]);
-                } else {
-                    *reinterpret_cast<float2*>(Vb + r * D + lane * 2) = make_float2(x[bb][0], x[bb][1]);
-                }
+                store_row<VPL>(Vb + r * D + lane * VPL, x[bb]);
             }
         }
 #pragma unroll
@@ -655,7 +668,7 @@ __global__ void __launch_bounds__(P_THREADS, 1) step_pipe_kernel(StepArgs a) {
 
 cudaError_t launch_step(const StepArgs& a, cudaStream_t st) {
     const dim3 grid((a.B + G - 1) / G, a.H);
-    if (a.D == 128) {
+    if (a.D == 128 && a.sl.m == 127) {
         int dev = 0, sms = 0;
         cudaError_t e = cudaGetDevice(&dev);
         if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
@@ -677,6 +690,9 @@ cudaError_t launch_step(const StepArgs& a, cudaStream_t st) {
     } else if (a.D == 64) {
         if (a.bf16) { LaunchScope ls_("decode_step", st); step_kernel<64, __nv_bfloat16><<<grid, 256, 0, st>>>(a); }
         else { LaunchScope ls_("decode_step", st); step_kernel<64, float><<<grid, 256, 0, st>>>(a); }
+    } else if (a.D == 128) {   // m != 127: the generic kernel
+        if (a.bf16) { LaunchScope ls_("decode_step", st); step_kernel<128, __nv_bfloat16><<<grid, 256, 0, st>>>(a); }
+        else { LaunchScope ls_("decode_step", st); step_kernel<128, float><<<grid, 256, 0, st>>>(a); }
     } else if (a.D == 256) {
         if (a.bf16) { LaunchScope ls_("decode_step", st); step_kernel<256, __nv_bfloat16><<<grid, 256, 0, st>>>(a); }
         else { LaunchScope ls_("decode_step", st); step_kernel<256, float><<<grid, 256, 0, st>>>(a); }

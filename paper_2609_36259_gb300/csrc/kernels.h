@@ -30,11 +30,32 @@ class LaunchScope {
     cudaEvent_t start_ = nullptr;
 };
 
+// Slot geometry: m active relative-time slots (odd, 1 <= m <= 127) in 128 storage rows; the
+// real Fourier basis of App. A.1 Eq. app-real-fourier has the DC row and (m-1)/2 cosine-sine
+// pairs, b = [1/sqrt(m), sqrt(2/m), 0, sqrt(2/m), 0, ...] (Eq. app-b-explicit), and rows m..127
+// stay zero.  The constants are formed once on the host.
+struct Slots {
+    int m, npair;
+    float fm, inv_m, two_over_m, inv_sqrt_m, sqrt2_over_m;
+};
+inline Slots make_slots(int m) {
+    Slots s;
+    s.m = m;
+    s.npair = (m - 1) / 2;
+    s.fm = (float)m;
+    s.inv_m = 1.f / (float)m;
+    s.two_over_m = 2.f / (float)m;
+    s.inv_sqrt_m = (float)(1.0 / __builtin_sqrt((double)m));
+    s.sqrt2_over_m = (float)__builtin_sqrt(2.0 / (double)m);
+    return s;
+}
+
 struct Shape {
     int B, T, H, D, C;      // batch, tokens, heads, head dim (dk == dv), chunk walked by a kernel
     int Cg;                 // chunk length the g_cum input is local to (the caller's chunk)
     float scale;
     bool bf16;
+    Slots sl;               // active slots
     __host__ __device__ int nchunk() const { return T / C; }
 };
 
@@ -61,7 +82,9 @@ cudaError_t launch_prepare_fixed_rate(const PrepareArgs& a, double rho, cudaStre
 cudaError_t prep_read_error(cudaStream_t st, int* err);
 
 // ---- readout matrix M = R Phi and its transpose (chunk_simt.cu) ----
-cudaError_t launch_readout_matrix(int H, const float* R, float* M, float* MT, cudaStream_t st);
+// R [H, m, m]; M, MT [H, 128, 128] with the rows and columns m..127 zero.
+cudaError_t launch_readout_matrix(int H, const float* R, float* M, float* MT, const Slots& sl,
+                                  cudaStream_t st);
 
 // ---- chunk forward / backward ----
 struct FwdArgs {
@@ -98,7 +121,7 @@ struct BwdArgs {
 // dR[h] = dM[h] Phi^T over the m active slots from dm_split partial dM blocks [H][split][128][128]
 // whose Fourier (column) index is in the tensor-core order (tc_order) or in the paper's order.
 cudaError_t launch_dr_finalize(const float* dMp, int dm_split, int H, bool tc_order, float* dR,
-                               cudaStream_t st);
+                               const Slots& sl, cudaStream_t st);
 constexpr int BWD_C = 64;       // chunk length used by the SIMT backward
 cudaError_t launch_bwd_simt(const BwdArgs& a, cudaStream_t st);
 // reverse cumulative sums of the per-token scalars in a.tok and the logit gradients
@@ -186,6 +209,7 @@ cudaError_t launch_bwd_tc(const TcBwdArgs& a, const TcFwdArgs& f, const void* q,
 // ---- decode (decode.cu) ----
 struct StepArgs {
     int B, H, D;
+    Slots sl;
     float scale;
     bool bf16;
     const void *q, *k, *v;

@@ -101,16 +101,17 @@ __global__ void __launch_bounds__(256) prep_scan_kernel(PrepareArgs a, int nseg)
     // clock mod m: the clock before this thread's first token is reduced once in fp64 (one
     // multiply by 1/m, no divide); its four tokens add their increments in fp64 (together < 4,
     // so at most one wrap) and are rounded to fp32 once
-    double bm = fma(-127.0, floor(excl * (1.0 / 127.0)), excl);
-    if (bm < 0.0) bm += 127.0;
-    else if (bm >= 127.0) bm -= 127.0;
+    const double fm = (double)a.s.sl.m, inv_m = 1.0 / fm;
+    double bm = fma(-fm, floor(excl * inv_m), excl);
+    if (bm < 0.0) bm += fm;
+    else if (bm >= fm) bm -= fm;
 #pragma unroll
     for (int u = 0; u < 4; ++u) {
         const int i = 4 * threadIdx.x + u;
         if (i < len) {
             const size_t gi = ((size_t)b * T + t0 + i) * H + h;
             double lm = bm + loc[u];
-            if (lm >= 127.0) lm -= 127.0;
+            if (lm >= fm) lm -= fm;
             a.lam_mod[gi] = (float)lm;
             a.g_cum[gi] = gex + lp[u];
             if (a.lambda_end && t0 + i == T - 1) a.lambda_end[bh] = excl + loc[u];
@@ -200,6 +201,7 @@ extern "C" int cyfa_prepare_noalloc(const cyfa_dims_t* dims, const float* clock_
     a.s.Cg = dims->chunk;
     a.s.scale = dims->scale;
     a.s.bf16 = dims->dtype == CYFA_DTYPE_BF16;
+    a.s.sl = make_slots(dims->m);
     a.clock_logit = clock_logit;
     a.decay_logit = decay_logit;
     a.beta_logit = beta_logit;

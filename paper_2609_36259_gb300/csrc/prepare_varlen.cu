@@ -257,10 +257,11 @@ __global__ void __launch_bounds__(256) prepv_scan_kernel(VarArgs a, int nseg) {
         rex += nres[u];
         if (i < len) {
             const size_t gi = ((size_t)b * T + t0 + i) * H + h;
+            const double fm = (double)a.p.s.sl.m;
             double lm = lamv[u];
-            lm = fma(-127.0, floor(lm * (1.0 / 127.0)), lm);
-            if (lm < 0.0) lm += 127.0;
-            else if (lm >= 127.0) lm -= 127.0;
+            lm = fma(-fm, floor(lm * (1.0 / fm)), lm);
+            if (lm < 0.0) lm += fm;
+            else if (lm >= fm) lm -= fm;
             a.p.lam_mod[gi] = (float)lm;
             a.p.g_cum[gi] = (gex + lp[u]) - RESET * (float)rex;
             if (VARLEN) {

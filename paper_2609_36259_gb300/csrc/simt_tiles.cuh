@@ -10,10 +10,10 @@ constexpr int LD = 129;   // padded row stride of [C][128] shared tiles
 
 // ---------------------------------------------------------------------------------------
 // Token-wise middle readout for rows r < C of sX (in place): o'' = U(-lam) M^T softmax(M U(lam) o')
-// with M = R Phi; the padding logit is excluded from the softmax and o''[127] = 0.
-// One warp per row; swarp holds 2 x 128 floats of scratch per warp.
+// with M = R Phi; the padding logits (slots m..127) are excluded from the softmax and o''[m..127]
+// stay 0.  One warp per row; swarp holds 2 x 128 floats of scratch per warp.
 static __device__ __noinline__ void middle_rows(float* sX, const float* slam, int C, const float* M, const float* MT,
-                            float* swarp) {
+                            float* swarp, const Slots& sl) {
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     float* z = swarp + warp * 256;
     float* p = z + 128;
@@ -26,11 +26,14 @@ static __device__ __noinline__ void middle_rows(float* sX, const float* slam, in
             const int j = lane + 1 + 32 * u;
             cs[u] = 1.f;
             sn[u] = 0.f;
-            if (j <= NPAIR) {
-                sincospif(phase_pi(lam, j), &sn[u], &cs[u]);
+            if (j <= sl.npair) {
+                sincospif(phase_pi_m(lam, j, sl), &sn[u], &cs[u]);
                 const float xc = x[2 * j - 1], xs = x[2 * j];
                 z[2 * j - 1] = cs[u] * xc - sn[u] * xs;
                 z[2 * j] = sn[u] * xc + cs[u] * xs;
+            } else if (j <= NPAIR) {   // padding slots (zero)
+                z[2 * j - 1] = 0.f;
+                z[2 * j] = 0.f;
             }
         }
         if (lane == 0) {
@@ -44,7 +47,9 @@ static __device__ __noinline__ void middle_rows(float* sX, const float* slam, in
 #pragma unroll
             for (int u = 0; u < 4; ++u) l[u] = fmaf(MT[k * MS + lane + 32 * u], zk, l[u]);
         }
-        if (lane == 31) l[3] = -INFINITY;
+#pragma unroll
+        for (int u = 0; u < 4; ++u)
+            if (lane + 32 * u >= sl.m) l[u] = -INFINITY;
         float mx = fmaxf(fmaxf(l[0], l[1]), fmaxf(l[2], l[3]));
         mx = warp_max(mx);
         float e[4], sum = 0.f;
@@ -59,7 +64,7 @@ static __device__ __noinline__ void middle_rows(float* sX, const float* slam, in
         for (int u = 0; u < 4; ++u) p[lane + 32 * u] = e[u] * inv;
         __syncwarp();
         float y[4] = {0.f, 0.f, 0.f, 0.f};
-        for (int i = 0; i < MA; ++i) {
+        for (int i = 0; i < sl.m; ++i) {
             const float pi = p[i];
 #pragma unroll
             for (int u = 0; u < 4; ++u) y[u] = fmaf(M[i * MS + lane + 32 * u], pi, y[u]);
@@ -71,7 +76,7 @@ static __device__ __noinline__ void middle_rows(float* sX, const float* slam, in
 #pragma unroll
         for (int u = 0; u < 2; ++u) {
             const int j = lane + 1 + 32 * u;
-            if (j <= NPAIR) {
+            if (j <= sl.npair) {
                 const float yc = z[2 * j - 1], ys = z[2 * j];
                 x[2 * j - 1] = cs[u] * yc + sn[u] * ys;
                 x[2 * j] = -sn[u] * yc + cs[u] * ys;

@@ -1430,8 +1430,9 @@ __global__ void __launch_bounds__(256, 1) dm_reduce_tc(const __grid_constant__ C
 // splits; its column j in the kernels' Fourier order when tc_order, else in the paper's).  One
 // block per (h, i).
 __global__ void __launch_bounds__(128) dr_finalize_kernel(const float* dMp, int dm_split,
-                                                          bool tc_order, float* dR) {
+                                                          bool tc_order, float* dR, Slots sl) {
     const int h = blockIdx.x, i = blockIdx.y, t = threadIdx.x;
+    const int m = sl.m;
     __shared__ float s_dm[128], s_ct[MA], s_st[MA];
     {
         float acc = 0.f;
@@ -1439,24 +1440,24 @@ __global__ void __launch_bounds__(128) dr_finalize_kernel(const float* dMp, int 
         for (int sp = 0; sp < dm_split; ++sp) acc += src[(size_t)sp * 128 * 128];
         s_dm[tc_order ? paper_slot(t) : t] = acc;   // paper order: DC, cos_1, sin_1, ..., pad
     }
-    if (t < MA) {
+    if (t < m) {
         float sv, cv;
-        sincospif((float)t * (2.f / 127.f), &sv, &cv);
+        sincospif((float)t * sl.two_over_m, &sv, &cv);
         s_ct[t] = cv;
         s_st[t] = sv;
     }
     __syncthreads();
-    if (t < MA) {   // k = t: Phi[k][0] = 1/sqrt(m), Phi[k][2j-1] = sqrt(2/m) cos(2 pi j k / m), ...
-        float acc = s_dm[0] * INV_SQRT_M;
+    if (t < m) {   // k = t: Phi[k][0] = 1/sqrt(m), Phi[k][2j-1] = sqrt(2/m) cos(2 pi j k / m), ...
+        float acc = s_dm[0] * sl.inv_sqrt_m;
         float ac = 0.f, as = 0.f;
         int idx = 0;
-        for (int j = 1; j <= NPAIR; ++j) {
+        for (int j = 1; j <= sl.npair; ++j) {
             idx += t;
-            if (idx >= MA) idx -= MA;
+            if (idx >= m) idx -= m;
             ac = fmaf(s_dm[2 * j - 1], s_ct[idx], ac);
             as = fmaf(s_dm[2 * j], s_st[idx], as);
         }
-        dR[((size_t)h * MA + i) * MA + t] = acc + SQRT_2_OVER_M * (ac + as);
+        dR[((size_t)h * m + i) * m + t] = acc + sl.sqrt2_over_m * (ac + as);
     }
 }
 
@@ -1632,7 +1633,7 @@ cudaError_t launch_bwd_tc(const TcBwdArgs& a, const TcFwdArgs& f, const void* q,
         const int sm_dm = 1024 + 2 * DM_NS * TILE + 1024;
         cudaFuncSetAttribute(dm_reduce_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, sm_dm);
         { LaunchScope ls_("tc_dm_reduce", st); dm_reduce_tc<<<dim3(s.H, a.dm_split), 256, sm_dm, st>>>(mz, mp, mdy, mdl, a); }
-        e = launch_dr_finalize(a.dMp, a.dm_split, s.H, true, a.dR, st);
+        e = launch_dr_finalize(a.dMp, a.dm_split, s.H, true, a.dR, s.sl, st);
         if (e != cudaSuccess) return e;
     }
     if (a.dA) { LaunchScope ls_("tc_dA", st); tc_dA_kernel<<<s.H, 256, 0, st>>>(a); }
@@ -1640,8 +1641,8 @@ cudaError_t launch_bwd_tc(const TcBwdArgs& a, const TcFwdArgs& f, const void* q,
 }
 
 cudaError_t launch_dr_finalize(const float* dMp, int dm_split, int H, bool tc_order, float* dR,
-                               cudaStream_t st) {
-    { LaunchScope ls_("dr_finalize", st); dr_finalize_kernel<<<dim3(H, MA), 128, 0, st>>>(dMp, dm_split, tc_order, dR); }
+                               const Slots& sl, cudaStream_t st) {
+    { LaunchScope ls_("dr_finalize", st); dr_finalize_kernel<<<dim3(H, sl.m), 128, 0, st>>>(dMp, dm_split, tc_order, dR, sl); }
     return cudaGetLastError();
 }
 

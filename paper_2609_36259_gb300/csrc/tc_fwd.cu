@@ -841,7 +841,9 @@ int tc_fwd_segments(const Shape& s) {
     return (nct + SEGC_DEFAULT - 1) / SEGC_DEFAULT;
 }
 
-bool tc_fwd_supported(const Shape& s) { return s.bf16 && s.D == 128 && s.T % CT == 0; }
+bool tc_fwd_supported(const Shape& s) {
+    return s.bf16 && s.D == 128 && s.sl.m == 127 && s.T % CT == 0;
+}
 
 bool tc_qkv_maps(const Shape& s, const void* q, const void* k, const void* v, CUtensorMap* mq,
                  CUtensorMap* mk, CUtensorMap* mv, unsigned box_rows) {

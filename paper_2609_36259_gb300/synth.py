@@ -47,7 +47,7 @@ def _unit(x):
 
 
 def make_inputs(B, T, H, d, *, seed=0, dtype=torch.bfloat16, device='cpu', with_dO=False,
-                identity_R=False):
+                identity_R=False, m=M_ACTIVE):
     """Draw one workload.  Returns a dict of tensors on ``device``.
 
     Draw order: q, k, v, clock_logit, decay_logit, beta_logit, dO (if asked).
@@ -64,7 +64,7 @@ def make_inputs(B, T, H, d, *, seed=0, dtype=torch.bfloat16, device='cpu', with_
     out = dict(q=q, k=k, v=v, clock_logit=clock, decay_logit=decay, beta_logit=beta)
     if with_dO:
         out['dO'] = torch.randn(B, T, H, d, **kw).to(dtype)
-    out['R'] = readout_init(H, seed=seed, identity=identity_R).to(device)
+    out['R'] = readout_init(H, m=m, seed=seed, identity=identity_R).to(device)
     out['A'] = decay_scales(H).to(device)
     out['scale'] = 1.0 / math.sqrt(d)
     return out

@@ -54,9 +54,10 @@ def test_workspace_sizes(lib):
 
 
 @pytest.mark.parametrize('field,value,code', [
-    ('m', 63, cyfa.CYFA_ERR_SHAPE), ('dk', 96, cyfa.CYFA_ERR_SHAPE), ('chunk', 32, cyfa.CYFA_ERR_SHAPE),
-    ('T', 100, cyfa.CYFA_ERR_SHAPE), ('B', 0, cyfa.CYFA_ERR_ARG), ('dtype', 7, cyfa.CYFA_ERR_ARG),
-    ('B', 65536, cyfa.CYFA_ERR_SHAPE)])
+    ('m', 64, cyfa.CYFA_ERR_SHAPE), ('m', 129, cyfa.CYFA_ERR_SHAPE), ('m', 0, cyfa.CYFA_ERR_SHAPE),
+    ('m', 255, cyfa.CYFA_ERR_UNSUPPORTED), ('dk', 96, cyfa.CYFA_ERR_SHAPE),
+    ('chunk', 32, cyfa.CYFA_ERR_SHAPE), ('T', 100, cyfa.CYFA_ERR_SHAPE), ('B', 0, cyfa.CYFA_ERR_ARG),
+    ('dtype', 7, cyfa.CYFA_ERR_ARG), ('B', 65536, cyfa.CYFA_ERR_SHAPE)])
 def test_bad_dims_rejected_on_host(lib, field, value, code):
     d = cyfa.dims(1, 128, 1, 128)
     setattr(d, field, value)
@@ -81,9 +82,11 @@ def test_null_and_misaligned_pointers_rejected_on_host(lib):
 
 def test_saved_size(lib):
     """The saved chunk-start states: fp16 [B*H][T/128][2][128][128] on the tensor-core path,
-    nothing on the CUDA-core kernels."""
+    nothing on the CUDA-core kernels (which also take every m other than 127 and d = 256)."""
     B, T, H = 2, 1024, 3
     assert cyfa.cyfa_saved_size(cyfa.dims(B, T, H, 128)) == B * H * (T // 128) * 2 * 128 * 128 * 2
+    assert cyfa.cyfa_saved_size(cyfa.dims(B, T, H, 128, m=63)) == 0
+    assert cyfa.cyfa_saved_size(cyfa.dims(B, T, H, 256)) == 0
     assert cyfa.cyfa_saved_size(cyfa.dims(B, T, H, 128, cuda_cores=True)) == 0
     assert cyfa.cyfa_saved_size(cyfa.dims(B, T, H, 64)) == 0
     assert cyfa.cyfa_saved_size(cyfa.dims(B, T, H, 128, dtype=torch.float32)) == 0
@@ -97,7 +100,7 @@ def test_timeout_selftest_rejects_bad_limits_on_host(lib):
 
 
 @pytest.mark.parametrize('field,value,code', [
-    ('dtype', 7, cyfa.CYFA_ERR_ARG), ('m', 63, cyfa.CYFA_ERR_SHAPE), ('T', 100, cyfa.CYFA_ERR_SHAPE),
+    ('dtype', 7, cyfa.CYFA_ERR_ARG), ('m', 64, cyfa.CYFA_ERR_SHAPE), ('T', 100, cyfa.CYFA_ERR_SHAPE),
     ('B', 65536, cyfa.CYFA_ERR_SHAPE)])
 def test_noalloc_prepare_checks_dims_like_prepare(lib, field, value, code):
     """cyfa_prepare_noalloc applies cyfa_prepare's argument checks, before any CUDA call."""
