@@ -418,6 +418,8 @@ def run_ours(args):
         paper = run_paper_shape(args, dev, rank, peaks)
         slots = run_slots_variant(args, dev, rank, peaks)
 
+    mixer = None if args.no_mixer else run_mixer(args, dev, rank, peaks)
+
     # end to end through the public API with host buffers
     e2e = None
     if not args.no_e2e:
@@ -438,7 +440,7 @@ def run_ours(args):
         'roofline': roof, 'kernel_rooflines': rooflines, 'cpu_baseline': cpu, 'e2e': e2e, 'gpu_launches': launches,
         'clocks': clk, 'tensor_frac': tensor_frac, 'fwd': fwd, 'bwd': bwd,
         'prepare_ms': prep_ms, 'kernel_ms_per_step': step_ms_kernels, 'decode': dec,
-        'varlen': varlen, 'paper_shape': paper, 'slots_m63': slots,
+        'varlen': varlen, 'paper_shape': paper, 'slots_m63': slots, 'mixer': mixer,
         'kernels': per_kernel,
     }
     if rank == 0:
@@ -576,6 +578,54 @@ def run_extra_shape(args, dev, rank, peaks, B, T, H, D, m, what):
             'fwd_ms': ms_fwd, 'fwd_tokens_per_s': B * T / (ms_fwd / 1e3),
             'tflops_rule': 3 * fl / (ms / 1e3) / 1e12,
             'frac_fp32_alu_peak': 3 * fl / (ms / 1e3) / 1e12 / alu, 'alu_peak_tflops': alu}
+
+
+def run_mixer(args, dev, rank, peaks):
+    """The mixer's neighbours on the layer's activations (bf16 [B, T, H, d]): ShortConv + SiLU +
+    QK RMSNorm before the operator and head RMSNorm + sigmoid gate after it, forward and backward.
+    HBM-bound: algorithmic bytes are each call's tensors read and written once (parameters and
+    their partial sums are under 0.1%)."""
+    import torch
+    from paper_2609_36259_gb300 import cyfa
+    B, T, H, D = LAYER['B'], LAYER['T'], LAYER['H'], LAYER['d']
+    g = torch.Generator(device=dev).manual_seed(5000 + rank)
+    mk = lambda: torch.randn(B, T, H, D, generator=g, device=dev).to(torch.bfloat16)
+    x = [mk() for _ in range(3)]
+    dy = [mk() for _ in range(3)]
+    y = [torch.empty_like(t) for t in x]
+    dx = [torch.empty_like(t) for t in x]
+    w = [torch.randn(H * D, 4, generator=g, device=dev) for _ in range(3)]
+    dw = [torch.empty_like(t) for t in w]
+    gains = [torch.ones(D, device=dev) for _ in range(3)]
+    dgs = [torch.empty_like(t) for t in gains]
+    d = cyfa.dims(B, T, H, D, chunk=args.chunk)
+    ws = cyfa.workspace(d, cyfa.CYFA_WS_MIXER, dev)
+    calls = {
+        'pre_fwd': (lambda: cyfa.cyfa_mixer_pre(d, *x, *w, gains[0], gains[1], 1e-6, *y), 6),
+        'pre_bwd': (lambda: cyfa.cyfa_mixer_pre_bwd(d, *x, *w, gains[0], gains[1], 1e-6, *dy,
+                                                    *dx, *dw, dgs[0], dgs[1], ws), 9),
+        'post_fwd': (lambda: cyfa.cyfa_mixer_post(d, x[0], x[1], gains[2], 1e-6, y[0]), 3),
+        'post_bwd': (lambda: cyfa.cyfa_mixer_post_bwd(d, x[0], x[1], gains[2], 1e-6, dy[0], dx[0],
+                                                      dx[1], dgs[2], ws), 5),
+    }
+    out = {'workload': 'B=%d T=%d H=%d d=%d bf16' % (B, T, H, D)}
+    for name, (fn, ntens) in calls.items():
+        for _ in range(3):
+            fn()
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        n = 20
+        e0.record()
+        for _ in range(n):
+            fn()
+        e1.record()
+        torch.cuda.synchronize()
+        ms = e0.elapsed_time(e1) / n
+        nbytes = ntens * B * T * H * D * 2
+        out[name] = {'ms': ms, 'bytes': nbytes, 'GB_per_s': nbytes / (ms / 1e3) / 1e9,
+                     'frac_hbm_measured': nbytes / (ms / 1e3) / 1e9 / peaks['hbm_gbs']}
+    cyfa.cyfa_check()
+    return out
 
 
 def run_varlen(args, dev, rank):
@@ -773,6 +823,7 @@ def main():
     ap.add_argument('--no-e2e', action='store_true')
     ap.add_argument('--no-varlen', action='store_true')
     ap.add_argument('--no-paper-shape', action='store_true')
+    ap.add_argument('--no-mixer', action='store_true')
     ap.add_argument('--no-dR', action='store_true',
                     help='leave the readout gradient dR out of the backward')
     ap.add_argument('--no-saved', action='store_true',

@@ -62,7 +62,8 @@ enum {
 enum { CYFA_DTYPE_BF16 = 0, CYFA_DTYPE_FP32 = 1 };
 
 /* Which call a workspace is sized for. */
-enum { CYFA_WS_PREPARE = 0, CYFA_WS_FWD = 1, CYFA_WS_BWD = 2, CYFA_WS_PREPARE_VARLEN = 3 };
+enum { CYFA_WS_PREPARE = 0, CYFA_WS_FWD = 1, CYFA_WS_BWD = 2, CYFA_WS_PREPARE_VARLEN = 3,
+       CYFA_WS_MIXER = 4 };
 
 typedef struct cyfa_dims {
     int B, T, H;   /* batch, sequence length, heads */
@@ -238,6 +239,39 @@ int cyfa_step(const cyfa_dims_t* dims, const void* q, const void* k, const void*
               const float* clock_logit, const float* decay_logit, const float* beta_logit,
               const float* A, const float* R, float* Kbar, float* Vbar, double* lambda, void* o,
               void* stream);
+
+/*
+ * The mixer's neighbours of the operator (Sec. 3.4, Mixer and backbone: ShortConv on q, k, v,
+ * RMSNorm of the queries and keys, head-wise RMSNorm of the output and a sigmoid output gate).
+ * The paper gives no formulas for them; this library's reading, with every tensor [B, T, H, d]
+ * in dims.dtype (channel c = h d + i), filters [H d][4] fp32 and gains [d] fp32 shared by the
+ * heads:
+ *   cyfa_mixer_pre:   a_t = silu(sum_{i<4} w[c][i] x_{t-3+i}[c])  (causal depthwise ShortConv,
+ *                     width 4, zero before token 0, per batch row), then for q and k
+ *                     q_t = a_t / sqrt(mean_d(a_t^2) + eps) * g per (token, head); v = a.
+ *   cyfa_mixer_post:  y_t = o_t / sqrt(mean_d(o_t^2) + eps) * g * sigmoid(z_t), z the gate
+ *                     logits of the mixer's low-rank gate projection.
+ * The *_bwd calls give the gradients of sum(out * d_out) with respect to every input and
+ * parameter (filter and gain gradients summed over the batch and, for gains, the heads);
+ * they need cyfa_workspace_size(CYFA_WS_MIXER) bytes of workspace.  Tensor pointers must be
+ * 16-byte aligned (CYFA_ERR_ALIGN otherwise).  The projections around
+ * them are plain matrix products left to the caller.  dims is that of the operator call (T, H,
+ * dk and dtype are used; m and chunk are checked as for the other calls).
+ */
+int cyfa_mixer_pre(const cyfa_dims_t* dims, const void* xq, const void* xk, const void* xv,
+                   const float* wq, const float* wk, const float* wv, const float* gq,
+                   const float* gk, float eps, void* q, void* k, void* v, void* stream);
+int cyfa_mixer_pre_bwd(const cyfa_dims_t* dims, const void* xq, const void* xk, const void* xv,
+                       const float* wq, const float* wk, const float* wv, const float* gq,
+                       const float* gk, float eps, const void* dq, const void* dk, const void* dv,
+                       void* dxq, void* dxk, void* dxv, float* dwq, float* dwk, float* dwv,
+                       float* dgq, float* dgk, void* workspace, size_t workspace_bytes,
+                       void* stream);
+int cyfa_mixer_post(const cyfa_dims_t* dims, const void* o, const void* z, const float* g,
+                    float eps, void* y, void* stream);
+int cyfa_mixer_post_bwd(const cyfa_dims_t* dims, const void* o, const void* z, const float* g,
+                        float eps, const void* dy, void* d_o, void* dz, float* dg,
+                        void* workspace, size_t workspace_bytes, void* stream);
 
 /*
  * cyfa_check -- wait for `stream`, then report (and clear) the device error words that the

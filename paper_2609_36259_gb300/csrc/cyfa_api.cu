@@ -194,6 +194,7 @@ int cyfa_workspace_size(const cyfa_dims_t* dims, int which, size_t* bytes) {
     switch (which) {
         case CYFA_WS_PREPARE: *bytes = up(prepare_workspace(s)); return CYFA_OK;
         case CYFA_WS_PREPARE_VARLEN: *bytes = up(prepare_varlen_workspace(s)); return CYFA_OK;
+        case CYFA_WS_MIXER: *bytes = up(mixer_workspace(s)); return CYFA_OK;
         case CYFA_WS_FWD: *bytes = fwd_layout(s, use_tc(dims, s), nullptr).bytes; return CYFA_OK;
         case CYFA_WS_BWD: *bytes = bwd_layout(s, use_tc(dims, s), nullptr).bytes; return CYFA_OK;
         default: return CYFA_ERR_ARG;
@@ -496,6 +497,75 @@ int cyfa_step(const cyfa_dims_t* dims, const void* q, const void* k, const void*
     a.lambda = lambda;
     a.o = o;
     return cuda_status(launch_step(a, static_cast<cudaStream_t>(stream)));
+}
+
+int cyfa_mixer_pre(const cyfa_dims_t* dims, const void* xq, const void* xk, const void* xv,
+                   const float* wq, const float* wk, const float* wv, const float* gq,
+                   const float* gk, float eps, void* q, void* k, void* v, void* stream) {
+    int rc = check_dims(dims, true);
+    if (rc) return rc;
+    if (!xq || !xk || !xv || !wq || !wk || !wv || !gq || !gk || !q || !k || !v) return CYFA_ERR_ARG;
+    if (!(eps >= 0.f)) return CYFA_ERR_ARG;
+    for (const void* p : {xq, xk, xv, (const void*)q, (const void*)k, (const void*)v})
+        if (!aligned16(p)) return CYFA_ERR_ALIGN;
+    const void* x[3] = {xq, xk, xv};
+    const float* w[3] = {wq, wk, wv};
+    const float* g[2] = {gq, gk};
+    void* y[3] = {q, k, v};
+    return cuda_status(launch_mixer_pre(shape_of(dims), x, w, g, eps, y,
+                                        static_cast<cudaStream_t>(stream)));
+}
+
+int cyfa_mixer_pre_bwd(const cyfa_dims_t* dims, const void* xq, const void* xk, const void* xv,
+                       const float* wq, const float* wk, const float* wv, const float* gq,
+                       const float* gk, float eps, const void* dq, const void* dk, const void* dv,
+                       void* dxq, void* dxk, void* dxv, float* dwq, float* dwk, float* dwv,
+                       float* dgq, float* dgk, void* workspace, size_t workspace_bytes,
+                       void* stream) {
+    int rc = check_dims(dims, true);
+    if (rc) return rc;
+    if (!xq || !xk || !xv || !wq || !wk || !wv || !gq || !gk || !dq || !dk || !dv || !dxq ||
+        !dxk || !dxv || !dwq || !dwk || !dwv || !dgq || !dgk)
+        return CYFA_ERR_ARG;
+    if (!(eps >= 0.f)) return CYFA_ERR_ARG;
+    for (const void* p : {xq, xk, xv, dq, dk, dv, (const void*)dxq, (const void*)dxk,
+                          (const void*)dxv})
+        if (!aligned16(p)) return CYFA_ERR_ALIGN;
+    const Shape s = shape_of(dims);
+    if (!workspace || workspace_bytes < mixer_workspace(s)) return CYFA_ERR_WORKSPACE;
+    const void* x[3] = {xq, xk, xv};
+    const float* w[3] = {wq, wk, wv};
+    const float* g[2] = {gq, gk};
+    const void* dy[3] = {dq, dk, dv};
+    void* dx[3] = {dxq, dxk, dxv};
+    float* dw[3] = {dwq, dwk, dwv};
+    float* dg[2] = {dgq, dgk};
+    return cuda_status(launch_mixer_pre_bwd(s, x, w, g, eps, dy, dx, dw, dg, workspace,
+                                            static_cast<cudaStream_t>(stream)));
+}
+
+int cyfa_mixer_post(const cyfa_dims_t* dims, const void* o, const void* z, const float* g,
+                    float eps, void* y, void* stream) {
+    int rc = check_dims(dims, true);
+    if (rc) return rc;
+    if (!o || !z || !g || !y || !(eps >= 0.f)) return CYFA_ERR_ARG;
+    if (!aligned16(o) || !aligned16(z) || !aligned16(y)) return CYFA_ERR_ALIGN;
+    return cuda_status(launch_mixer_post(shape_of(dims), o, z, g, eps, y,
+                                         static_cast<cudaStream_t>(stream)));
+}
+
+int cyfa_mixer_post_bwd(const cyfa_dims_t* dims, const void* o, const void* z, const float* g,
+                        float eps, const void* dy, void* d_o, void* dz, float* dg,
+                        void* workspace, size_t workspace_bytes, void* stream) {
+    int rc = check_dims(dims, true);
+    if (rc) return rc;
+    if (!o || !z || !g || !dy || !d_o || !dz || !dg || !(eps >= 0.f)) return CYFA_ERR_ARG;
+    if (!aligned16(o) || !aligned16(z) || !aligned16(dy) || !aligned16(d_o) || !aligned16(dz))
+        return CYFA_ERR_ALIGN;
+    const Shape s = shape_of(dims);
+    if (!workspace || workspace_bytes < mixer_workspace(s)) return CYFA_ERR_WORKSPACE;
+    return cuda_status(launch_mixer_post_bwd(s, o, z, g, eps, dy, d_o, dz, dg, workspace,
+                                             static_cast<cudaStream_t>(stream)));
 }
 
 int cyfa_check(void* stream) {

@@ -206,6 +206,21 @@ struct TcBwdArgs {
 cudaError_t launch_bwd_tc(const TcBwdArgs& a, const TcFwdArgs& f, const void* q, const void* k,
                           const void* v, const void* dO, cudaStream_t st);
 
+// ---- mixer neighbours (mixer.cu) ----
+// Arrays of three are (q, k, v); of two (q, k).
+size_t mixer_workspace(const Shape& s);
+cudaError_t launch_mixer_pre(const Shape& s, const void* const* x, const float* const* w,
+                             const float* const* g, float eps, void* const* y, cudaStream_t st);
+cudaError_t launch_mixer_pre_bwd(const Shape& s, const void* const* x, const float* const* w,
+                                 const float* const* g, float eps, const void* const* dy,
+                                 void* const* dx, float* const* dw, float* const* dg, void* ws,
+                                 cudaStream_t st);
+cudaError_t launch_mixer_post(const Shape& s, const void* o, const void* z, const float* g,
+                              float eps, void* y, cudaStream_t st);
+cudaError_t launch_mixer_post_bwd(const Shape& s, const void* o, const void* z, const float* g,
+                                  float eps, const void* dy, void* dO, void* dz, float* dg,
+                                  void* ws, cudaStream_t st);
+
 // ---- decode (decode.cu) ----
 struct StepArgs {
     int B, H, D;

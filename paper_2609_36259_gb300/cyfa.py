@@ -16,14 +16,15 @@ CYFA_OK = 0
 CYFA_ERR_ARG, CYFA_ERR_SHAPE, CYFA_ERR_ALIGN, CYFA_ERR_WORKSPACE = -1, -2, -3, -4
 CYFA_ERR_CUDA, CYFA_ERR_TIMEOUT, CYFA_ERR_UNSUPPORTED, CYFA_ERR_RANGE = -5, -6, -7, -8
 CYFA_DTYPE_BF16, CYFA_DTYPE_FP32 = 0, 1
-CYFA_WS_PREPARE, CYFA_WS_FWD, CYFA_WS_BWD, CYFA_WS_PREPARE_VARLEN = 0, 1, 2, 3
+CYFA_WS_PREPARE, CYFA_WS_FWD, CYFA_WS_BWD, CYFA_WS_PREPARE_VARLEN, CYFA_WS_MIXER = 0, 1, 2, 3, 4
 
 # Every symbol include/cyfa.h declares (checked by tests/test_abi.py).
 EXPORTS = ('cyfa_version', 'cyfa_error_string', 'cyfa_workspace_size', 'cyfa_prepare',
            'cyfa_chunk_fwd', 'cyfa_chunk_bwd', 'cyfa_step', 'cyfa_check', 'cyfa_stats_reset',
            'cyfa_stats_timing', 'cyfa_stats_get', 'cyfa_prepare_noalloc',
            'cyfa_selftest_mma', 'cyfa_saved_size', 'cyfa_selftest_timeout',
-           'cyfa_prepare_fixed_rate', 'cyfa_prepare_varlen')
+           'cyfa_prepare_fixed_rate', 'cyfa_prepare_varlen', 'cyfa_mixer_pre',
+           'cyfa_mixer_pre_bwd', 'cyfa_mixer_post', 'cyfa_mixer_post_bwd')
 
 
 class CyfaError(RuntimeError):
@@ -77,6 +78,13 @@ def load(path=LIB_PATH):
     lib.cyfa_prepare_fixed_rate.argtypes = [P, ctypes.c_double] + [_VP] * 8 + [_VP]
     lib.cyfa_prepare_varlen.argtypes = ([P, _VP, ctypes.c_int, _VP, ctypes.c_double] + [_VP] * 8
                                         + [_VP, ctypes.c_size_t, _VP])
+    F = ctypes.c_float
+    lib.cyfa_mixer_pre.argtypes = [P] + [_VP] * 8 + [F] + [_VP] * 3 + [_VP]
+    lib.cyfa_mixer_pre_bwd.argtypes = ([P] + [_VP] * 8 + [F] + [_VP] * 11 + [_VP, ctypes.c_size_t,
+                                                                             _VP])
+    lib.cyfa_mixer_post.argtypes = [P, _VP, _VP, _VP, F, _VP, _VP]
+    lib.cyfa_mixer_post_bwd.argtypes = [P, _VP, _VP, _VP, F, _VP, _VP, _VP, _VP, _VP,
+                                        ctypes.c_size_t, _VP]
     lib.cyfa_stats_timing.argtypes = [ctypes.c_int]
     lib.cyfa_stats_get.argtypes = [ctypes.c_int, ctypes.c_char_p, ctypes.c_int,
                                    ctypes.POINTER(ctypes.c_longlong), ctypes.POINTER(ctypes.c_double)]
@@ -186,6 +194,30 @@ def cyfa_step(d, q, k, v, clock_logit, decay_logit, beta_logit, A, R, Kbar, Vbar
     _ok(load().cyfa_step(ctypes.byref(d), _ptr(q), _ptr(k), _ptr(v), _ptr(clock_logit),
                          _ptr(decay_logit), _ptr(beta_logit), _ptr(A), _ptr(R), _ptr(Kbar),
                          _ptr(Vbar), _ptr(lam), _ptr(o), _stream(stream)))
+
+
+def cyfa_mixer_pre(d, xq, xk, xv, wq, wk, wv, gq, gk, eps, q, k, v, stream=None):
+    _ok(load().cyfa_mixer_pre(ctypes.byref(d), *map(_ptr, (xq, xk, xv, wq, wk, wv, gq, gk)),
+                              float(eps), _ptr(q), _ptr(k), _ptr(v), _stream(stream)))
+
+
+def cyfa_mixer_pre_bwd(d, xq, xk, xv, wq, wk, wv, gq, gk, eps, dq, dk, dv, dxq, dxk, dxv, dwq, dwk,
+                       dwv, dgq, dgk, ws, stream=None):
+    _ok(load().cyfa_mixer_pre_bwd(ctypes.byref(d), *map(_ptr, (xq, xk, xv, wq, wk, wv, gq, gk)),
+                                  float(eps), *map(_ptr, (dq, dk, dv, dxq, dxk, dxv, dwq, dwk,
+                                                          dwv, dgq, dgk)),
+                                  _ptr(ws), ws.numel(), _stream(stream)))
+
+
+def cyfa_mixer_post(d, o, z, g, eps, y, stream=None):
+    _ok(load().cyfa_mixer_post(ctypes.byref(d), _ptr(o), _ptr(z), _ptr(g), float(eps), _ptr(y),
+                               _stream(stream)))
+
+
+def cyfa_mixer_post_bwd(d, o, z, g, eps, dy, d_o, dz, dg, ws, stream=None):
+    _ok(load().cyfa_mixer_post_bwd(ctypes.byref(d), _ptr(o), _ptr(z), _ptr(g), float(eps),
+                                   _ptr(dy), _ptr(d_o), _ptr(dz), _ptr(dg), _ptr(ws), ws.numel(),
+                                   _stream(stream)))
 
 
 def cyfa_check(stream=None):

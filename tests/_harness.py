@@ -27,6 +27,27 @@ def assert_close_bf16(got, want, what=''):
     return err, rl
 
 
+def assert_close_rounded(got, want, what=''):
+    """Outputs of the mixer kernels, which compute in fp32 and round once to bf16: a bf16 value
+    x carries up to half a unit in the last place, at most 2^-8 |x| (8 significant bits), which
+    no kernel can avoid, and the normalised outputs reach |x| ~ 10, where that alone is the
+    operator's 2e-2 max-abs bar.  Bar derived from that arithmetic: elementwise
+    |got - want| <= 2^-8 |want| + 1e-3 (the 1e-3 for the fp32 arithmetic before the rounding),
+    and rel-L2 within the stated 5e-3."""
+    got = np.asarray(got, dtype=np.float64)
+    want = np.asarray(want, dtype=np.float64)
+    err = np.abs(got - want)
+    bar = 2.0 ** -8 * np.abs(want) + 1e-3
+    rl = rel_l2(got, want)
+    worst = float(np.max(err / bar)) if err.size else 0.0
+    print('measured %s: max-abs %.3e, max err/bar %.3f, rel-L2 %.3e'
+          % (what, float(err.max()) if err.size else 0.0, worst, rl))
+    assert worst <= 1.0 and rl <= BF16_REL_L2, \
+        '%s: max err/bar %.3f (bar 2^-8|x| + 1e-3), rel-L2 %.3e (bar %.0e)' % (what, worst, rl,
+                                                                          BF16_REL_L2)
+    return worst, rl
+
+
 def assert_close_batch_sum(got, want, terms, what=''):
     """dA[h] = sum over the batch's tokens of w_t d log alpha_t (w_t = -softplus(f_t)), a sum of
     many terms that cancel: its size says nothing about the error its terms carry.  Reading: each
