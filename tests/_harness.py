@@ -126,16 +126,64 @@ def to_device(inp, device='cuda'):
     return {k: (v.to(device) if torch.is_tensor(v) else v) for k, v in inp.items()}
 
 
-def gpu_prepare(d, inp, lambda0=None, want_lambda_end=False):
-    return cyfa.prepare(d, inp['clock_logit'], inp['decay_logit'], inp['beta_logit'], inp['A'],
-                        lambda0=lambda0, want_lambda_end=want_lambda_end)
+GUARD_BYTES = 256      # canary bytes on each side of every guarded output (keeps 256-B alignment)
+CANARY = 0xA5
+
+
+class Guards:
+    """Output tensors with canary bytes on both sides, checked on the host after the calls that
+    wrote them: a kernel writing past either end of an output (which the compute-sanitizer
+    closed on this pool would otherwise catch) changes a canary and fails the test."""
+
+    def __init__(self):
+        self.bufs = []
+
+    def empty(self, shape, dtype, device='cuda'):
+        n = int(np.prod(shape)) * torch.empty(0, dtype=dtype).element_size()
+        raw = torch.full((n + 2 * GUARD_BYTES,), CANARY, dtype=torch.uint8, device=device)
+        self.bufs.append((raw, n))
+        return raw[GUARD_BYTES:GUARD_BYTES + n].view(dtype).view(*shape)
+
+    def empty_like(self, t):
+        return self.empty(tuple(t.shape), t.dtype, t.device)
+
+    def check(self, what=''):
+        if any(raw.is_cuda for raw, _ in self.bufs):
+            torch.cuda.synchronize()
+        for raw, n in self.bufs:
+            head, tail = raw[:GUARD_BYTES], raw[GUARD_BYTES + n:]
+            assert bool((head == CANARY).all()) and bool((tail == CANARY).all()), \
+                '%s: a canary next to an output of %d bytes was overwritten' % (what, n)
+
+
+def gpu_prepare(d, inp, lambda0=None, want_lambda_end=False, guards=None):
+    gd = guards or Guards()
+    B, T, H = inp['clock_logit'].shape
+    dev = inp['clock_logit'].device
+    lam, g, beta = (gd.empty((B, T, H), torch.float32, dev) for _ in range(3))
+    lend = gd.empty((B, H), torch.float64, dev) if want_lambda_end else None
+    ws = cyfa.workspace(d, cyfa.CYFA_WS_PREPARE, dev)
+    cyfa.cyfa_prepare(d, inp['clock_logit'], inp['decay_logit'], inp['beta_logit'], inp['A'],
+                      lambda0, lam, g, beta, lend, ws)
+    if guards is None:
+        gd.check('cyfa_prepare')
+    return lam, g, beta, lend
 
 
 def gpu_forward(d, inp, want_state=False, Kbar0=None, Vbar0=None, lambda0=None):
-    lam, g, beta, lend = gpu_prepare(d, inp, lambda0=lambda0, want_lambda_end=True)
-    o, Ko, Vo = cyfa.forward(d, inp['q'], inp['k'], inp['v'], lam, g, beta, inp['R'],
-                             Kbar0=Kbar0, Vbar0=Vbar0, want_state=want_state)
-    torch.cuda.synchronize()
+    gd = Guards()
+    lam, g, beta, lend = gpu_prepare(d, inp, lambda0=lambda0, want_lambda_end=True, guards=gd)
+    v = inp['v']
+    B, T, H, D = v.shape
+    o = gd.empty_like(v)
+    Ko = Vo = None
+    if want_state:
+        Ko = gd.empty((B, H, 128, D), torch.float32, v.device)
+        Vo = gd.empty((B, H, 128, D), torch.float32, v.device)
+    ws = cyfa.workspace(d, cyfa.CYFA_WS_FWD, v.device)
+    cyfa.cyfa_chunk_fwd(d, inp['q'], inp['k'], v, lam, g, beta, inp['R'], Kbar0, Vbar0, o, Ko, Vo,
+                        ws)
+    gd.check('cyfa_prepare + cyfa_chunk_fwd')
     return o, Ko, Vo, lend
 
 

@@ -5,8 +5,9 @@ import torch
 
 from paper_2609_36259_gb300 import cyfa, synth
 
-from _harness import (assert_close_batch_sum, assert_close_bf16, assert_close_rel, gpu_prepare,
-                      oracle_backward, oracle_inputs, pairs_np, rel_l2, sample_pairs, to_device)
+from _harness import (Guards, assert_close_batch_sum, assert_close_bf16, assert_close_rel,
+                      gpu_prepare, oracle_backward, oracle_inputs, pairs_np, rel_l2, sample_pairs,
+                      to_device)
 
 pytestmark = pytest.mark.gpu
 
@@ -19,23 +20,27 @@ def gpu_backward(d, inp, want_dA=True, use_saved=False, want_dR=False):
     q, k, v, dO = inp['q'], inp['k'], inp['v'], inp['dO']
     saved = None
     if use_saved:   # a forward that saves its chunk-start states for this backward
-        saved = cyfa.saved_buffer(d, q.device)
-        assert saved is not None
+        n = cyfa.cyfa_saved_size(d)
+        assert n > 0
+        sg = Guards()
+        saved = sg.empty((n,), torch.uint8, q.device)
         o_plain = cyfa.forward(d, q, k, v, lam, g, beta, inp['R'])[0]
         o_saving = cyfa.forward(d, q, k, v, lam, g, beta, inp['R'], saved=saved)[0]
         assert torch.equal(o_plain, o_saving)   # saving does not change the forward
-    out = dict(dq=torch.empty_like(q), dk=torch.empty_like(k), dv=torch.empty_like(v),
-               d_clock=torch.empty_like(inp['clock_logit']),
-               d_decay=torch.empty_like(inp['clock_logit']),
-               d_beta=torch.empty_like(inp['clock_logit']),
-               dA=torch.empty_like(inp['A']) if want_dA else None,
-               dR=torch.empty_like(inp['R']) if want_dR else None)
+        sg.check('cyfa_chunk_fwd saved states')
+    gd = Guards()
+    out = dict(dq=gd.empty_like(q), dk=gd.empty_like(k), dv=gd.empty_like(v),
+               d_clock=gd.empty_like(inp['clock_logit']),
+               d_decay=gd.empty_like(inp['clock_logit']),
+               d_beta=gd.empty_like(inp['clock_logit']),
+               dA=gd.empty_like(inp['A']) if want_dA else None,
+               dR=gd.empty_like(inp['R']) if want_dR else None)
     ws = cyfa.workspace(d, cyfa.CYFA_WS_BWD, q.device)
     cyfa.cyfa_chunk_bwd(d, q, k, v, lam, g, beta, inp['R'], inp['clock_logit'],
                         inp['decay_logit'], inp['A'], dO, out['dq'], out['dk'], out['dv'],
                         out['d_clock'], out['d_decay'], out['d_beta'], out['dR'], out['dA'], ws,
                         saved=saved)
-    torch.cuda.synchronize()
+    gd.check('cyfa_chunk_bwd')
     return out
 
 

@@ -5,8 +5,8 @@ import torch
 
 from paper_2609_36259_gb300 import cyfa, synth
 
-from _harness import (assert_close_bf16, gpu_forward, oracle_forward, oracle_inputs, pairs_np,
-                      sample_pairs)
+from _harness import (Guards, assert_close_bf16, gpu_forward, oracle_forward, oracle_inputs,
+                      pairs_np, sample_pairs)
 
 pytestmark = pytest.mark.gpu
 
@@ -18,14 +18,15 @@ def _decode(inp, T0, steps, d_prefill, d_step):
     _, K, V, lam = gpu_forward(d_prefill, pre, want_state=True)
     B, _, H, D = inp['q'].shape
     outs = []
+    gd = Guards()
     for t in range(T0, T0 + steps):
-        o = torch.empty(B, H, D, dtype=inp['v'].dtype, device='cuda')
+        o = gd.empty((B, H, D), inp['v'].dtype)
         cyfa.cyfa_step(d_step, inp['q'][:, t].contiguous(), inp['k'][:, t].contiguous(),
                        inp['v'][:, t].contiguous(), inp['clock_logit'][:, t].contiguous(),
                        inp['decay_logit'][:, t].contiguous(), inp['beta_logit'][:, t].contiguous(),
                        inp['A'], inp['R'], K, V, lam, o)
         outs.append(o)
-    torch.cuda.synchronize()
+    gd.check('cyfa_step')
     return torch.stack(outs, 1), K, V, lam
 
 
