@@ -694,80 +694,91 @@ def run_varlen(args, dev, rank):
 
 def run_e2e(args, inp, dev, want_dR):
     """The step through the public API with pinned host buffers: every step copies all its inputs
-    host->device and reads every output back.  The batch rows go as micro-batches on their own
-    CUDA streams (each with its own workspaces), so one row's copies overlap another row's
-    kernels and the two copy directions overlap each other; the per-row dA / dR partials are
-    read back and summed on the host."""
+    host->device and reads every output back.  The (b, h) sequences are independent, so the step
+    runs as micro-batches of one batch row and a group of heads (host buffers laid out per
+    micro-batch), spread round-robin over a few CUDA streams with a workspace each: one
+    micro-batch's copies run under another's kernels, the two copy directions overlap, and the
+    next step's uploads start while this step's last results come back (a stream's micro-batches
+    run in order, so its device buffers are never reused early).  The per-micro-batch dA / dR
+    partials are read back and summed on the host."""
     import torch
     from paper_2609_36259_gb300 import cyfa
     B, T, H, D = inp['q'].shape
+    hg = args.e2e_heads if H % args.e2e_heads == 0 else H
     keys = ('q', 'k', 'v', 'clock_logit', 'decay_logit', 'beta_logit', 'dO')
-    d1 = cyfa.dims(1, T, H, D, chunk=args.chunk, cuda_cores=args.cuda_cores)
-    rows = []
+    d1 = cyfa.dims(1, T, hg, D, chunk=args.chunk, cuda_cores=args.cuda_cores)
+    nstream = max(1, min(args.e2e_streams, B * (H // hg)))
+    streams = [torch.cuda.Stream(device=dev) for _ in range(nstream)]
+    ws = [[cyfa.workspace(d1, w, dev) for w in (cyfa.CYFA_WS_PREPARE, cyfa.CYFA_WS_FWD,
+                                                 cyfa.CYFA_WS_BWD)] for _ in range(nstream)]
+    saved = [None if args.no_saved else cyfa.saved_buffer(d1, dev) for _ in range(nstream)]
+    f32 = dict(dtype=torch.float32, device=dev)
+    mbs = []
     for b in range(B):
-        r = {'stream': torch.cuda.Stream(device=dev)}
-        r['host'] = {k: inp[k][b:b + 1].cpu().pin_memory() for k in keys}
-        r['x'] = {k: torch.empty_like(inp[k][b:b + 1]) for k in keys}
-        r['x'].update({k: inp[k] for k in ('A', 'R')})
-        f32 = dict(dtype=torch.float32, device=dev)
-        lam = torch.empty(1, T, H, **f32)
-        r['gates'] = (lam, torch.empty_like(lam), torch.empty_like(lam))
-        r['out'] = dict(o=torch.empty_like(r['x']['v']), dq=torch.empty_like(r['x']['q']),
-                        dk=torch.empty_like(r['x']['k']), dv=torch.empty_like(r['x']['v']),
-                        dc=torch.empty_like(lam), dd=torch.empty_like(lam), db=torch.empty_like(lam),
-                        dA=torch.empty(H, **f32))
-        if want_dR:
-            r['out']['dR'] = torch.empty(H, 127, 127, **f32)
-        r['host_out'] = {k: t.new_empty(t.shape, device='cpu').pin_memory() for k, t in r['out'].items()}
-        r['ws'] = [cyfa.workspace(d1, w, dev) for w in (cyfa.CYFA_WS_PREPARE, cyfa.CYFA_WS_FWD, cyfa.CYFA_WS_BWD)]
-        r['saved'] = None if args.no_saved else cyfa.saved_buffer(d1, dev)
-        rows.append(r)
-    h2d = sum(t.numel() * t.element_size() for r in rows for t in r['host'].values())
-    d2h = sum(t.numel() * t.element_size() for r in rows for t in r['host_out'].values())
+        for h0 in range(0, H, hg):
+            sl = slice(h0, h0 + hg)
+            m = {'stream': len(mbs) % nstream}
+            m['host'] = {k: inp[k][b:b + 1, :, sl].contiguous().cpu().pin_memory() for k in keys}
+            m['x'] = {k: torch.empty(m['host'][k].shape, dtype=m['host'][k].dtype, device=dev)
+                      for k in keys}
+            m['x']['A'] = inp['A'][sl].contiguous()
+            m['x']['R'] = inp['R'][sl].contiguous()
+            lam = torch.empty(1, T, hg, **f32)
+            m['gates'] = (lam, torch.empty_like(lam), torch.empty_like(lam))
+            m['out'] = dict(o=torch.empty_like(m['x']['v']), dq=torch.empty_like(m['x']['q']),
+                            dk=torch.empty_like(m['x']['k']), dv=torch.empty_like(m['x']['v']),
+                            dc=torch.empty_like(lam), dd=torch.empty_like(lam),
+                            db=torch.empty_like(lam), dA=torch.empty(hg, **f32))
+            if want_dR:
+                m['out']['dR'] = torch.empty(hg, 127, 127, **f32)
+            m['host_out'] = {k: t.new_empty(t.shape, device='cpu').pin_memory()
+                             for k, t in m['out'].items()}
+            m['h0'] = h0
+            mbs.append(m)
+    h2d = sum(t.numel() * t.element_size() for m in mbs for t in m['host'].values())
+    d2h = sum(t.numel() * t.element_size() for m in mbs for t in m['host_out'].values())
 
     def one():
-        main = torch.cuda.current_stream(dev)
-        ev = main.record_event()
-        for r in rows:
-            st, x, o = r['stream'], r['x'], r['out']
-            st.wait_event(ev)
+        for m in mbs:
+            si = m['stream']
+            st, x, o = streams[si], m['x'], m['out']
             with torch.cuda.stream(st):
                 for k in keys:
-                    x[k].copy_(r['host'][k], non_blocking=True)
-                lam, g, beta = r['gates']
+                    x[k].copy_(m['host'][k], non_blocking=True)
+                lam, g, beta = m['gates']
+                w = ws[si]
                 cyfa.cyfa_prepare(d1, x['clock_logit'], x['decay_logit'], x['beta_logit'], x['A'],
-                                  None, lam, g, beta, None, r['ws'][0], stream=st)
+                                  None, lam, g, beta, None, w[0], stream=st)
                 cyfa.cyfa_chunk_fwd(d1, x['q'], x['k'], x['v'], lam, g, beta, x['R'], None, None,
-                                    o['o'], None, None, r['ws'][1], stream=st, saved=r['saved'])
+                                    o['o'], None, None, w[1], stream=st, saved=saved[si])
                 cyfa.cyfa_chunk_bwd(d1, x['q'], x['k'], x['v'], lam, g, beta, x['R'],
                                     x['clock_logit'], x['decay_logit'], x['A'], x['dO'], o['dq'],
-                                    o['dk'], o['dv'], o['dc'], o['dd'], o['db'], o.get('dR'), o['dA'],
-                                    r['ws'][2], stream=st, saved=r['saved'])
+                                    o['dk'], o['dv'], o['dc'], o['dd'], o['db'], o.get('dR'),
+                                    o['dA'], w[2], stream=st, saved=saved[si])
                 for k, t in o.items():
-                    r['host_out'][k].copy_(t, non_blocking=True)
-        for r in rows:
-            main.wait_stream(r['stream'])
+                    m['host_out'][k].copy_(t, non_blocking=True)
 
     for _ in range(2):
         one()
     torch.cuda.synchronize()
     n = max(1, args.steps)
-    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     t0 = time.perf_counter()
-    e0.record()
     for _ in range(n):
         one()
-    e1.record()
     torch.cuda.synchronize()
-    # the batch sums of dA and dR from the rows' partials (host side, inside the wall clock)
-    dA = sum(r['host_out']['dA'] for r in rows)
+    # the batch sums of dA and dR from the micro-batches' partials (host side, inside the clock)
+    dA = torch.zeros(H)
+    for m in mbs:
+        dA[m['h0']:m['h0'] + hg] += m['host_out']['dA']
     if want_dR:
-        dR = sum(r['host_out']['dR'] for r in rows)
+        dR = torch.zeros(H, 127, 127)
+        for m in mbs:
+            dR[m['h0']:m['h0'] + hg] += m['host_out']['dR']
     wall = (time.perf_counter() - t0) / n
-    ms = e0.elapsed_time(e1) / n
-    return {'value': B * T / (ms / 1e3), 'unit': 'tokens/s', 'h2d_bytes_per_step': h2d,
-            'd2h_bytes_per_step': d2h, 'ms_per_step': ms, 'wall_ms_per_step': wall * 1e3,
-            'micro_batches': B}
+    return {'value': B * T / wall, 'unit': 'tokens/s', 'h2d_bytes_per_step': h2d,
+            'd2h_bytes_per_step': d2h, 'ms_per_step': wall * 1e3,
+            'micro_batches': len(mbs), 'heads_per_micro_batch': hg, 'streams': nstream,
+            'timing': 'host wall clock over %d back-to-back steps, synchronised at both ends' % n}
 
 
 # ---------------------------------------------------------------------------- reference
@@ -821,6 +832,9 @@ def main():
                     help='B,T,H override of the layer shape (profiling runs on smaller cases)')
     ap.add_argument('--no-decode', action='store_true')
     ap.add_argument('--no-e2e', action='store_true')
+    ap.add_argument('--e2e-heads', type=int, default=8,
+                    help='heads per micro-batch of the end-to-end step')
+    ap.add_argument('--e2e-streams', type=int, default=4)
     ap.add_argument('--no-varlen', action='store_true')
     ap.add_argument('--no-paper-shape', action='store_true')
     ap.add_argument('--no-mixer', action='store_true')
