@@ -570,14 +570,19 @@ def run_extra_shape(args, dev, rank, peaks, B, T, H, D, m, what):
     cyfa.cyfa_check()
     th = B * T * H
     fl = operator_flops_per_token_head(C, d=D, ms=m + 1) * th
-    alu = fp32_alu_peak_tflops(peaks['sm_max_mhz'])
+    tc = cyfa.cyfa_saved_size(d) > 0
+    peak = peaks['bf16'] if tc else fp32_alu_peak_tflops(peaks['sm_max_mhz'])
+    tf = 3 * fl / (ms / 1e3) / 1e12
     return {'workload': 'B=%d T=%d H=%d d=%d m=%d chunk %d (%s), prepare + fwd + bwd with every '
                         'gradient' % (B, T, H, D, m, C, what),
-            'path': 'fp32 CUDA-core kernels (the tensor-core kernels take d = 128, m = 127)',
+            'path': ('tensor-core kernels (128 storage rows, m* = %d counted)' % (m + 1) if tc else
+                     'fp32 CUDA-core kernels (the tensor-core kernels take bf16, d = 128, '
+                     '63 <= m <= 127)'),
             'ms_per_step': ms, 'tokens_per_s': B * T / (ms / 1e3),
             'fwd_ms': ms_fwd, 'fwd_tokens_per_s': B * T / (ms_fwd / 1e3),
-            'tflops_rule': 3 * fl / (ms / 1e3) / 1e12,
-            'frac_fp32_alu_peak': 3 * fl / (ms / 1e3) / 1e12 / alu, 'alu_peak_tflops': alu}
+            'tflops_rule': tf, 'peak_tflops': peak,
+            'peak_source': 'measured bf16 burst' if tc else 'fp32 FMA: 152 x 128 x 2 x clock',
+            'frac_peak': tf / peak}
 
 
 def run_mixer(args, dev, rank, peaks):

@@ -22,16 +22,19 @@
  *   v, o, dO, dv      [B, T, H, dv]   bf16 or fp32
  *   *_logit, lam_mod, g_cum, beta, d_*_logit   [B, T, H] fp32
  *   A                 [H] fp32 (> 0)
- *   R, dR             [H, m, m] fp32 (m = 127)
+ *   R, dR             [H, m, m] fp32
  *   Kbar, Vbar        [B, H, 128, dk] / [B, H, 128, dv] fp32; rows in the order of the real
  *                     Fourier basis of App. A.1 Eq. app-real-fourier (DC, cos_1, sin_1, ...,
- *                     cos_63, sin_63) followed by one padding row that stays zero (App. A.7).
+ *                     cos_p, sin_p with p = (m-1)/2) followed by 128 - m padding rows that
+ *                     stay zero (App. A.7; one row at m = 127).
  *   lambda            [B, H] fp64 (the running clock)
  *   stream            a cudaStream_t passed as void*; every call is asynchronous on it.
  *
- * Shapes supported: m = 127 (128 storage rows), dk = dv in {64, 128}, chunk in {64, 128},
- * T a positive multiple of chunk (for cyfa_prepare / cyfa_chunk_fwd / cyfa_chunk_bwd),
- * B * H <= 65535.
+ * Shapes supported: odd m in 1..127 (128 storage rows; m = 255 is CYFA_ERR_UNSUPPORTED),
+ * dk = dv in {64, 128, 256}, chunk in {64, 128}, T a positive multiple of chunk (for
+ * cyfa_prepare / cyfa_chunk_fwd / cyfa_chunk_bwd), B * H <= 65535.  The tensor-core kernels
+ * take bf16 with d = 128, 63 <= m <= 127 and T a multiple of 128; every other supported shape
+ * runs on the fp32 CUDA-core kernels.
  *
  * Errors: every entry point returns CYFA_OK (0) or a negative code.  Argument errors are
  * found on the host before anything is launched.  CYFA_ERR_TIMEOUT (a bounded wait expired)
@@ -68,7 +71,7 @@ enum { CYFA_WS_PREPARE = 0, CYFA_WS_FWD = 1, CYFA_WS_BWD = 2, CYFA_WS_PREPARE_VA
 typedef struct cyfa_dims {
     int B, T, H;   /* batch, sequence length, heads */
     int dk, dv;    /* head dims (dk == dv) */
-    int m;         /* active relative-time slots; must be 127 */
+    int m;         /* active relative-time slots: odd, 1..127 (the paper's default is 127) */
     int chunk;     /* tokens per chunk: 64 or 128 */
     float scale;   /* dot-product scale s; the query enters the key pass as s*q */
     int dtype;     /* CYFA_DTYPE_BF16 or CYFA_DTYPE_FP32 for q, k, v, o, dO, dq, dk, dv */

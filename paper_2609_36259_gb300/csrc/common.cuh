@@ -12,7 +12,7 @@ namespace cyfa {
 constexpr int MS = 128;        // storage rows per state (m* = m + 1)
 constexpr int MA = 127;        // active relative-time slots m
 constexpr int NPAIR = 63;      // cosine-sine pairs (m - 1) / 2
-constexpr float INV_SQRT_M = 0.088735651910547f;   // 1 / sqrt(127)
+constexpr float INV_SQRT_M = 0.088735650941611f;   // 1 / sqrt(127)
 constexpr float SQRT_2_OVER_M = 0.125491161809579f; // sqrt(2 / 127)
 
 __device__ __forceinline__ float ldf(const float* p, size_t i) { return p[i]; }
@@ -37,7 +37,8 @@ __device__ __forceinline__ float phase_pi(float lam, int j) {
 
 // phase_pi for m active slots (the same arithmetic with m in place of 127; identical values at
 // m = 127): lam in [0, m), theta_j = 2 pi j lam / m = pi * phase_pi_m(lam, j, sl).
-__device__ __forceinline__ float phase_pi_m(float lam, int j, const Slots& sl) {
+template <class SL>
+__device__ __forceinline__ float phase_pi_m(float lam, int j, const SL& sl) {
     const float hi = rintf(lam * 256.f) * (1.f / 256.f);
     const float lo = lam - hi;
     const float jh = (float)j * hi;

@@ -310,7 +310,7 @@ int cyfa_chunk_fwd(const cyfa_dims_t* dims, const void* q, const void* k, const 
     if (!aligned16(workspace)) return CYFA_ERR_ALIGN;
     const FwdLayout L = fwd_layout(s, tc_path, workspace);
     cudaStream_t st = static_cast<cudaStream_t>(stream);
-    rc = cuda_status(tc_path ? launch_readout_f16(s.H, R, L.Mb, st)
+    rc = cuda_status(tc_path ? launch_readout_f16(s.H, R, L.Mb, s.sl, st)
                              : launch_readout_matrix(s.H, R, L.M, L.MT, s.sl, st));
     if (rc) return rc;
     if (tc_path) {
@@ -374,7 +374,7 @@ int cyfa_chunk_bwd(const cyfa_dims_t* dims, const void* q, const void* k, const 
     if (!aligned16(workspace)) return CYFA_ERR_ALIGN;
     const BwdLayout L = bwd_layout(s, tc_path, workspace);
     cudaStream_t st = static_cast<cudaStream_t>(stream);
-    rc = cuda_status(tc_path ? launch_readout_f16(s.H, R, L.Mb, st)
+    rc = cuda_status(tc_path ? launch_readout_f16(s.H, R, L.Mb, s.sl, st)
                              : launch_readout_matrix(s.H, R, L.M, L.MT, s.sl, st));
     if (rc) return rc;
     BwdArgs a;

@@ -37,6 +37,7 @@ class LaunchScope {
 struct Slots {
     int m, npair;
     float fm, inv_m, two_over_m, inv_sqrt_m, sqrt2_over_m;
+    float omega1;           // 2 pi / m, the rotation rate of pair 1
 };
 inline Slots make_slots(int m) {
     Slots s;
@@ -47,8 +48,18 @@ inline Slots make_slots(int m) {
     s.two_over_m = 2.f / (float)m;
     s.inv_sqrt_m = (float)(1.0 / __builtin_sqrt((double)m));
     s.sqrt2_over_m = (float)__builtin_sqrt(2.0 / (double)m);
+    s.omega1 = 6.283185307179586f / (float)m;
     return s;
 }
+
+// The same geometry as compile-time constants for m = 127 (the paper's setting): kernels
+// templated on the slot type fold every constant; runtime Slots serve the other m.
+struct Slots127 {
+    static constexpr int m = 127, npair = 63;
+    static constexpr float fm = 127.f, inv_m = 1.f / 127.f, two_over_m = 2.f / 127.f;
+    static constexpr float inv_sqrt_m = 0.088735650941611f, sqrt2_over_m = 0.125491161809579f;
+    static constexpr float omega1 = 6.283185307179586f / 127.f;
+};
 
 struct Shape {
     int B, T, H, D, C;      // batch, tokens, heads, head dim (dk == dv), chunk walked by a kernel
@@ -158,7 +169,8 @@ int tc_fwd_segments(const Shape& s);
 cudaError_t launch_fwd_tc(const TcFwdArgs& a, const void* q, const void* k, const void* v,
                           cudaStream_t st);
 // M = R Phi as fp16 in the tensor-core column order ([H][128][128], padding row / column zero).
-cudaError_t launch_readout_f16(int H, const float* R, __half* Mb, cudaStream_t st);
+cudaError_t launch_readout_f16(int H, const float* R, __half* Mb, const Slots& sl,
+                               cudaStream_t st);
 // Reads (and clears) the error word of the tensor-core kernels; synchronises the stream.
 cudaError_t tc_read_error(cudaStream_t st, int* err);
 cudaError_t tc_bwd_read_error(cudaStream_t st, int* err);

@@ -98,10 +98,12 @@ __device__ __forceinline__ float dot64(const float (&x)[64], const float (&y)[64
 
 // ---------------------------------------------------------------------------------------
 // Chunk-start states of every chunk, walking each segment from its start state.
+template <class SL>
 __global__ void __launch_bounds__(256, 1) snap_fwd_tc(const __grid_constant__ CUtensorMap tk,
                                                        const __grid_constant__ CUtensorMap tv,
                                                        TcBwdArgs a) {
     const Shape s = a.s;
+    const SL sl = slots_of<SL>(s);
     const int bh = blockIdx.x, seg = blockIdx.y, b = bh / s.H, h = bh % s.H;
     const int nct = s.T / CT;
     const int c_begin = seg * TC_SEGC;
@@ -175,7 +177,8 @@ __global__ void __launch_bounds__(256, 1) snap_fwd_tc(const __grid_constant__ CU
                 tmem_st64(tl + 128 * hf + 64 * q2, x);
             }
         }
-        write_vector_half<__half>(tiles + 3 * buf * TILE, row, hf, lam, beta * ex2((gC - g) * LOG2E));
+        write_vector_half<__half>(tiles + 3 * buf * TILE, row, hf, lam, beta * ex2((gC - g) * LOG2E),
+                                  sl);
         if (ok) ok = mbar_wait(&bars[buf], (c >> 1) & 1);
         if (ok) {
             bf16_to_f16_half(tiles + (3 * buf + 1) * TILE, row, hf);
@@ -218,6 +221,7 @@ __global__ void __launch_bounds__(256, 1) snap_fwd_tc(const __grid_constant__ CU
 // loaded into the tiles the current item has finished with after its dO' products, and its V
 // after the last product, so an item starts with its operands mostly in place.  The six tiles
 // change roles from item to item: (dO/Q, A, staging) <- (A, staging, dO/Q).
+template <class SL>
 __global__ void __launch_bounds__(512, 1) bwd_chunk1_tc(const __grid_constant__ CUtensorMap tq,
                                                          const __grid_constant__ CUtensorMap tk,
                                                          const __grid_constant__ CUtensorMap tv,
@@ -231,6 +235,7 @@ __global__ void __launch_bounds__(512, 1) bwd_chunk1_tc(const __grid_constant__ 
                                                          const __grid_constant__ CUtensorMap tdq,
                                                          TcBwdArgs a) {
     const Shape s = a.s;
+    const SL sl = slots_of<SL>(s);
     const int nct = s.T / CT;
     const int NI = s.B * s.H * nct;   // items (b*h, chunk), b*h-major
     const int i0 = (int)((long long)NI * blockIdx.x / gridDim.x);
@@ -407,7 +412,7 @@ __global__ void __launch_bounds__(512, 1) bwd_chunk1_tc(const __grid_constant__ 
             }
             mma_commit(&bars[2]);
         }
-        write_vector_q<__half>(T_A, row, hf, u, lam, beta);   // while G1 runs
+        write_vector_q<__half>(T_A, row, hf, u, lam, beta, sl);   // while G1 runs
         wait_mma();
         if (issuer()) {   // dO, V and Vbar are consumed: Q, K and Kbar
             mbar_expect_tx(&bars[1], 3 * TILE);
@@ -476,7 +481,7 @@ __global__ void __launch_bounds__(512, 1) bwd_chunk1_tc(const __grid_constant__ 
             const float f = scale * gam;
     #pragma unroll
             for (int i = 0; i < 32; ++i) x[i] = fmaf(f, x[i], y[i]);
-            rotate_q<1>(x, hf, u, lam);
+            rotate_q<1>(x, hf, u, lam, sl);
             store_q<__half>(T_S, row, c0, x);
             tmem_st16x2(tl + X3, x);
         }
@@ -493,16 +498,15 @@ __global__ void __launch_bounds__(512, 1) bwd_chunk1_tc(const __grid_constant__ 
         {   // p = softmax(l) over the m valid entries (the padding column is out), kept in X1
             float x[32];
             tmem_ld16x2(tl + X1, x);
-            const bool pad = (hf == 1 && u == 1);
             float mx = -INFINITY;
     #pragma unroll
             for (int i = 0; i < 32; ++i)
-                if (!(pad && i == 31)) mx = fmaxf(mx, x[i]);
+                if (!slot_off(c0, i, sl)) mx = fmaxf(mx, x[i]);
             mx = row_reduce(mx, true);
             float sum = 0.f;
     #pragma unroll
             for (int i = 0; i < 32; ++i) {
-                x[i] = (pad && i == 31) ? 0.f : ex2((x[i] - mx) * LOG2E);
+                x[i] = slot_off(c0, i, sl) ? 0.f : ex2((x[i] - mx) * LOG2E);
                 sum += x[i];
             }
             const float inv = 1.f / row_reduce(sum, false);
@@ -523,8 +527,9 @@ __global__ void __launch_bounds__(512, 1) bwd_chunk1_tc(const __grid_constant__ 
         if (a.mZ) staged_read();   // the staging tile is rewritten below (uniform branch)
         {   // o'' = U(-lam) (p M); scalars with do'' (o'' as stored in fp16); dy = U(lam) do''.
             // Eight rotation pairs at a time: cosine entries, then sine entries.
-            QuarterAngles ang(lam, hf, u);
-            const float wb = OMEGA1 * (float)(32 * hf + 16 * u + 1);   // pair frequency, first pair
+            QuarterAngles ang(lam, hf, u, sl);
+            const float om1 = sl.omega1;
+            const float wb = om1 * (float)(32 * hf + 16 * u + 1);   // pair frequency, first pair
             const bool dcq = (hf == 1 && u == 1);   // pair 15 of this quarter is the DC / padding
             __half* o2row = a.O2 + ((size_t)bh * s.T + t0 + row) * 128;
             uint32_t pc[8], ps[8];   // o'' packed: columns c0 .. c0 + 15 and c0 + 32 .. c0 + 47
@@ -544,7 +549,7 @@ __global__ void __launch_bounds__(512, 1) bwd_chunk1_tc(const __grid_constant__ 
                     const float gc = gv[i], gs = gv[8 + i];
                     s1 = fmaf(orc, gc, fmaf(ors, gs, s1));
                     if (!dc)   // <o'', Omega do''>
-                        s2 += (wb + OMEGA1 * (float)(8 * p8 + i)) * (ors * gc - orc * gs);
+                        s2 += (wb + om1 * (float)(8 * p8 + i)) * (ors * gc - orc * gs);
                     gv[i] = dc ? gc : c * gc - sn * gs;          // U(lam)
                     gv[8 + i] = dc ? 0.f : sn * gc + c * gs;
                 }
@@ -587,8 +592,9 @@ __global__ void __launch_bounds__(512, 1) bwd_chunk1_tc(const __grid_constant__ 
         wait_mma();
         if (a.mZ) staged_read();   // the staging tile is rewritten below (uniform branch)
         {   // do' = U(-lam) dz; <do', Omega o'> with do' as stored in fp16 (= <dz, Omega z> exactly)
-            QuarterAngles ang(lam, hf, u);
-            const float wb = OMEGA1 * (float)(32 * hf + 16 * u + 1);   // pair frequency, first pair
+            QuarterAngles ang(lam, hf, u, sl);
+            const float om1 = sl.omega1;
+            const float wb = om1 * (float)(32 * hf + 16 * u + 1);   // pair frequency, first pair
             const bool dcq = (hf == 1 && u == 1);
             __half* d1row = a.DO1 + ((size_t)bh * s.T + t0 + row) * 128;
             uint32_t pc[8], ps[8];   // do' packed: columns c0 .. c0 + 15 and c0 + 32 .. c0 + 47
@@ -606,7 +612,7 @@ __global__ void __launch_bounds__(512, 1) bwd_chunk1_tc(const __grid_constant__ 
                     dz[8 + i] = dc ? 0.f : c * xs - sn * xc;
                     if (!dc) {   // o' = U(-lam) z
                         const float zc = c * z[i] + sn * z[8 + i], zs = c * z[8 + i] - sn * z[i];
-                        s3 += (wb + OMEGA1 * (float)(8 * p8 + i)) *
+                        s3 += (wb + om1 * (float)(8 * p8 + i)) *
                               (round16<__half>(dz[8 + i]) * zc - round16<__half>(dz[i]) * zs);
                     }
                 }
@@ -711,7 +717,7 @@ __global__ void __launch_bounds__(512, 1) bwd_chunk1_tc(const __grid_constant__ 
 // after the other with double-buffered tiles.  In the SNAP walk the chunk-start state S of
 // the forward (for the boundary terms of the gate gradients) arrives by TMA with the operand
 // tiles, and the adjoint snapshot leaves through the same shared tile by a TMA store.
-template <bool SNAP>
+template <bool SNAP, class SL>
 __global__ void __launch_bounds__(256, 1) adj_walk_tc(const __grid_constant__ CUtensorMap tdo1,
                                                        const __grid_constant__ CUtensorMap to2,
                                                        const __grid_constant__ CUtensorMap tq,
@@ -720,6 +726,7 @@ __global__ void __launch_bounds__(256, 1) adj_walk_tc(const __grid_constant__ CU
                                                        const __grid_constant__ CUtensorMap tsa,
                                                        TcBwdArgs a) {
     const Shape s = a.s;
+    const SL sl = slots_of<SL>(s);
     const int bh = blockIdx.x, seg = blockIdx.y, b = bh / s.H, h = bh % s.H;
     const int nct = s.T / CT;
     const int c_begin = seg * TC_SEGC;
@@ -874,9 +881,9 @@ __global__ void __launch_bounds__(256, 1) adj_walk_tc(const __grid_constant__ CU
                 // chunk's own writes enter through the inter-chunk column terms of
                 // bwd_chunk2_tc); this thread's row and 64 columns
                 const int l = row & 63, jj = l & 31, j = 32 * (row >> 6) + jj + 1;
-                const bool paired = j <= NPAIR;
+                const bool paired = j <= sl.npair;
                 const int partner = (l >= 32) ? row - 32 : row + 32;
-                const float f = paired ? ((l >= 32) ? 1.f : -1.f) * OMEGA1 * (float)j : 0.f;
+                const float f = paired ? ((l >= 32) ? 1.f : -1.f) * sl.omega1 * (float)j : 0.f;
                 float sr[64], sp[64];
                 load_half_smem(tS, row, hf, sr);
                 load_half_smem(tS, paired ? partner : row, hf, sp);
@@ -984,6 +991,7 @@ __global__ void __launch_bounds__(256) seg_scan_rev_kernel(TcBwdArgs a) {
 // (b*h, chunk) items like bwd_chunk1_tc: the next item's V goes into the write-vector tile once
 // dO' A^T has read it, its dO into the Q tile after Q K^T, its O'' and D^V after the last
 // products; the write-vector tile and the V / K tile swap roles from item to item.
+template <class SL>
 __global__ void __launch_bounds__(512, 1) bwd_chunk2_tc(const __grid_constant__ CUtensorMap tq,
                                                          const __grid_constant__ CUtensorMap tk,
                                                          const __grid_constant__ CUtensorMap tv,
@@ -995,6 +1003,7 @@ __global__ void __launch_bounds__(512, 1) bwd_chunk2_tc(const __grid_constant__ 
                                                          const __grid_constant__ CUtensorMap tdv,
                                                          TcBwdArgs a) {
     const Shape s = a.s;
+    const SL sl = slots_of<SL>(s);
     const int nct = s.T / CT;
     const int NI = s.B * s.H * nct;
     const int i0 = (int)((long long)NI * blockIdx.x / gridDim.x);
@@ -1132,7 +1141,7 @@ __global__ void __launch_bounds__(512, 1) bwd_chunk2_tc(const __grid_constant__ 
         }
         {   // while it runs: the write vectors and their copies scaled by gamma^C / gamma^s
             float x[32];
-            write_vector_q_vals(x, hf, u, lam, beta);
+            write_vector_q_vals(x, hf, u, lam, beta, sl);
             store_q<__half>(T_A, row, c0, x);
 #pragma unroll
             for (int i = 0; i < 32; ++i) x[i] *= fw;
@@ -1274,15 +1283,15 @@ __global__ void __launch_bounds__(512, 1) bwd_chunk2_tc(const __grid_constant__ 
             for (int i = 0; i < 32; ++i) x[i] += y[i];
             store_q<__nv_bfloat16>(T_S, row, c0, x);   // dk, staged (P1 is consumed) for a TMA store
             float av[32];
-            write_vector_q_vals(av, hf, u, lam, beta);   // unrounded a
+            write_vector_q_vals(av, hf, u, lam, beta, sl);   // unrounded a
             tmem_ld16x2_pair(tl + X3, x, tl + X4, y);   // intra- / inter-chunk da (both passes)
     #pragma unroll
             for (int i = 0; i < 32; ++i) db = fmaf(x[i] + y[i], av[i], db);
     #pragma unroll
             for (int i = 0; i < 32; ++i) av[i] = round16<__half>(av[i]);   // a as the MMAs saw it
-            cL = -omega_dot_q(x, av, hf, u);
+            cL = -omega_dot_q(x, av, hf, u, sl);
             cIG = dot32(av, y);
-            cIL = -omega_dot_q(y, av, hf, u);
+            cIL = -omega_dot_q(y, av, hf, u, sl);
         }
         // row sums over the four column quarters, staged in the scaled write-vector tile (its last
         // product is complete; the next item rewrites it after its first barrier)
@@ -1559,8 +1568,9 @@ __global__ void __launch_bounds__(256) tc_dA_kernel(TcBwdArgs a) {
 
 }  // namespace
 
-cudaError_t launch_bwd_tc(const TcBwdArgs& a, const TcFwdArgs& f, const void* q, const void* k,
-                          const void* v, const void* dO, cudaStream_t st) {
+template <class SL>
+cudaError_t launch_bwd_tc_sl(const TcBwdArgs& a, const TcFwdArgs& f, const void* q, const void* k,
+                             const void* v, const void* dO, cudaStream_t st) {
     const Shape& s = a.s;
     const int nct = s.T / CT;
     const unsigned long long BH = (unsigned long long)s.B * s.H;
@@ -1583,10 +1593,10 @@ cudaError_t launch_bwd_tc(const TcBwdArgs& a, const TcFwdArgs& f, const void* q,
     const int sm_adj_seg = 1024 + 4 * TC_SEGC * CT + 6 * TILE + 1024;
     const int sm_chunk1 = 8192 + 6 * TILE + 1024, sm_chunk2 = 2048 + 7 * TILE + 1024;
     if (!a.saved) {
-        cudaFuncSetAttribute(snap_fwd_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, sm_walk6);
-        { LaunchScope ls_("tc_snap_fwd", st); snap_fwd_tc<<<gseg, 256, sm_walk6, st>>>(mk, mv, a); }
+        cudaFuncSetAttribute(snap_fwd_tc<SL>, cudaFuncAttributeMaxDynamicSharedMemorySize, sm_walk6);
+        { LaunchScope ls_("tc_snap_fwd", st); snap_fwd_tc<SL><<<gseg, 256, sm_walk6, st>>>(mk, mv, a); }
     }
-    cudaFuncSetAttribute(bwd_chunk1_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, sm_chunk1);
+    cudaFuncSetAttribute(bwd_chunk1_tc<SL>, cudaFuncAttributeMaxDynamicSharedMemorySize, sm_chunk1);
     {   // persistent: one CTA per SM walks a contiguous range of (b*h, chunk) items
         int dev = 0, sms = 0;
         if (cudaGetDevice(&dev) != cudaSuccess ||
@@ -1604,14 +1614,14 @@ cudaError_t launch_bwd_tc(const TcBwdArgs& a, const TcFwdArgs& f, const void* q,
             !tc_rows_map(&mdy, bdy, BH * s.T, true) || !tc_rows_map(&mdl, bdl, BH * s.T, true))
             return cudaErrorInvalidValue;
         LaunchScope ls_("tc_bwd_chunk1", st);
-        bwd_chunk1_tc<<<grid1, 512, sm_chunk1, st>>>(mq, mk, mv, mdo, mm, msf, mz, mpp, mdy, mdl, mdq, a);
+        bwd_chunk1_tc<SL><<<grid1, 512, sm_chunk1, st>>>(mq, mk, mv, mdo, mm, msf, mz, mpp, mdy, mdl, mdq, a);
     }
-    cudaFuncSetAttribute(adj_walk_tc<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, sm_adj_seg);
-    { LaunchScope ls_("tc_adj_segment", st); adj_walk_tc<false><<<gseg, 256, sm_adj_seg, st>>>(mdo1, mo2, mq, mdo, msf, msa, a); }
+    cudaFuncSetAttribute(adj_walk_tc<false, SL>, cudaFuncAttributeMaxDynamicSharedMemorySize, sm_adj_seg);
+    { LaunchScope ls_("tc_adj_segment", st); adj_walk_tc<false, SL><<<gseg, 256, sm_adj_seg, st>>>(mdo1, mo2, mq, mdo, msf, msa, a); }
     { LaunchScope ls_("tc_adj_scan", st); seg_scan_rev_kernel<<<dim3(128, s.B * s.H), 256, 0, st>>>(a); }
-    cudaFuncSetAttribute(adj_walk_tc<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, sm_snap_adj);
-    { LaunchScope ls_("tc_snap_adj", st); adj_walk_tc<true><<<gseg, 256, sm_snap_adj, st>>>(mdo1, mo2, mq, mdo, msf, msa, a); }
-    cudaFuncSetAttribute(bwd_chunk2_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, sm_chunk2);
+    cudaFuncSetAttribute(adj_walk_tc<true, SL>, cudaFuncAttributeMaxDynamicSharedMemorySize, sm_snap_adj);
+    { LaunchScope ls_("tc_snap_adj", st); adj_walk_tc<true, SL><<<gseg, 256, sm_snap_adj, st>>>(mdo1, mo2, mq, mdo, msf, msa, a); }
+    cudaFuncSetAttribute(bwd_chunk2_tc<SL>, cudaFuncAttributeMaxDynamicSharedMemorySize, sm_chunk2);
     {
         int dev = 0, sms = 0;
         if (cudaGetDevice(&dev) != cudaSuccess ||
@@ -1622,7 +1632,7 @@ cudaError_t launch_bwd_tc(const TcBwdArgs& a, const TcFwdArgs& f, const void* q,
         LaunchScope ls_("tc_bwd_chunk2", st);
         CUtensorMap mdk, mdv;
         if (!tc_qkv_maps(s, a.dk, a.dv, nullptr, &mdk, &mdv, nullptr)) return cudaErrorInvalidValue;
-        bwd_chunk2_tc<<<grid2, 512, sm_chunk2, st>>>(mq, mk, mv, mdo, mo2, mdo1, msa, mdk, mdv, a);
+        bwd_chunk2_tc<SL><<<grid2, 512, sm_chunk2, st>>>(mq, mk, mv, mdo, mo2, mdo1, msa, mdk, mdv, a);
     }
     { LaunchScope ls_("tc_gate", st); tc_gate_kernel<<<gchunk, 128, 0, st>>>(a); }
     if (a.dR) {   // dR from the middle-readout vectors bwd_chunk1_tc wrote
@@ -1638,6 +1648,12 @@ cudaError_t launch_bwd_tc(const TcBwdArgs& a, const TcFwdArgs& f, const void* q,
     }
     if (a.dA) { LaunchScope ls_("tc_dA", st); tc_dA_kernel<<<s.H, 256, 0, st>>>(a); }
     return cudaGetLastError();
+}
+
+cudaError_t launch_bwd_tc(const TcBwdArgs& a, const TcFwdArgs& f, const void* q, const void* k,
+                          const void* v, const void* dO, cudaStream_t st) {
+    return a.s.sl.m == 127 ? launch_bwd_tc_sl<Slots127>(a, f, q, k, v, dO, st)
+                           : launch_bwd_tc_sl<Slots>(a, f, q, k, v, dO, st);
 }
 
 cudaError_t launch_dr_finalize(const float* dMp, int dm_split, int H, bool tc_order, float* dR,

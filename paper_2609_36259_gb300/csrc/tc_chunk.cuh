@@ -3,6 +3,8 @@
 // loads / stores, the thread roles of the 256-thread kernels.
 #pragma once
 
+#include <type_traits>
+
 #include "../../include/cyfa.h"
 #include "common.cuh"
 #include "kernels.h"
@@ -17,7 +19,6 @@ constexpr int CT = 128;              // tokens per chunk on this path
 constexpr int TC_SEGC = 8;           // chunks per segment (1024 tokens)
 constexpr int TILE = CT * 128 * 2;   // one 128 x 128 bf16 tile (32 KiB)
 constexpr float LOG2E = 1.4426950408889634f;
-constexpr float OMEGA1 = 6.283185307179586f / 127.f;   // 2 pi / m: frequency of rotation pair 1
 
 // error word of the including translation unit (each has its own copy)
 static __device__ int g_tc_err;
@@ -37,6 +38,14 @@ __device__ __forceinline__ float cum128(const Shape& s, const float* g, int b, i
     if (s.Cg == 64 && t - t0 >= 64) v += g[((size_t)b * s.T + t0 + 63) * s.H + h];
     return v;
 }
+
+// The slot geometry a kernel instance works with: compile-time for m = 127, else the runtime
+// values carried in the Shape.
+template <class SL> __device__ __forceinline__ SL slots_of(const Shape& s);
+// m = 127: every rotation pair is active and slot 127 alone is padding (no masks to evaluate)
+template <class SL> constexpr bool full_slots() { return std::is_same<SL, Slots127>::value; }
+template <> __device__ __forceinline__ Slots127 slots_of<Slots127>(const Shape&) { return {}; }
+template <> __device__ __forceinline__ Slots slots_of<Slots>(const Shape& s) { return s.sl; }
 
 // Order of the 128 Fourier-axis rows inside the tensor-core kernels.  Column half hf (0 or 1)
 // holds the pairs j = 32 hf + jj + 1 (jj < 32): cosine entry at 64 hf + jj, sine entry at
@@ -68,22 +77,25 @@ __device__ __forceinline__ void sincospi_fast(float x, float* s, float* c) {
 // Rotation angles theta_j = 2 pi j lam / m for the 32 pairs of one column half, produced in
 // order by angle addition from theta_1 (cos(x + y) = cos x cos y - sin x sin y,
 // sin(x + y) = sin x cos y + cos x sin y), re-seeded from sincospi_fast every 16 steps.
+template <class SL>
 struct HalfAngles {
     float c1, s1, c, s, lam;
     int j0;
-    __device__ __forceinline__ HalfAngles(float lam_, int hf) : lam(lam_), j0(32 * hf + 1) {
-        sincospi_fast(phase_pi(lam, 1), &s1, &c1);
+    SL sl;
+    __device__ __forceinline__ HalfAngles(float lam_, int hf, const SL& sl_)
+        : lam(lam_), j0(32 * hf + 1), sl(sl_) {
+        sincospi_fast(phase_pi_m(lam, 1, sl), &s1, &c1);
         if (j0 == 1) {
             c = c1;
             s = s1;
         } else {
-            sincospi_fast(phase_pi(lam, j0), &s, &c);
+            sincospi_fast(phase_pi_m(lam, j0, sl), &s, &c);
         }
     }
     // advance to local pair jj (1..31)
     __device__ __forceinline__ void step(int jj) {
         if (jj == 16) {
-            sincospi_fast(phase_pi(lam, j0 + 16), &s, &c);
+            sincospi_fast(phase_pi_m(lam, j0 + 16, sl), &s, &c);
         } else {
             const float cn = c * c1 - s * s1;
             const float sn = s * c1 + c * s1;
@@ -108,20 +120,22 @@ __device__ __forceinline__ void store_half_bf16(uint8_t* tile, int r, int hf, co
 }
 
 // One column half of the temporal write vector w U(-lam) b of a token (Sec. 3.2, b of
-// Eq. app-b-explicit), in the tensor-core row order.
-template <typename OT = __nv_bfloat16>
-__device__ __forceinline__ void write_vector_half(uint8_t* tile, int r, int hf, float lam, float w) {
+// Eq. app-b-explicit), in the tensor-core row order; the entries of pairs past (m-1)/2 are zero.
+template <typename OT = __nv_bfloat16, class SL>
+__device__ __forceinline__ void write_vector_half(uint8_t* tile, int r, int hf, float lam, float w,
+                                                  const SL& sl) {
     float x[64];
-    HalfAngles ang(lam, hf);
-    const float wa = w * SQRT_2_OVER_M;
+    HalfAngles ang(lam, hf, sl);
+    const float wa = w * sl.sqrt2_over_m;
 #pragma unroll
     for (int jj = 0; jj < 32; ++jj) {
         if (jj > 0) ang.step(jj);
-        x[jj] = wa * ang.c;
-        x[jj + 32] = -wa * ang.s;
+        const bool on = full_slots<SL>() || 32 * hf + jj + 1 <= sl.npair;
+        x[jj] = on ? wa * ang.c : 0.f;
+        x[jj + 32] = on ? -wa * ang.s : 0.f;
     }
     if (hf == 1) {
-        x[31] = w * INV_SQRT_M;
+        x[31] = w * sl.inv_sqrt_m;
         x[63] = 0.f;
     }
     store_half_bf16<OT>(tile, r, hf, x);
@@ -201,16 +215,17 @@ struct QRole {
 
 // Angles of the 16 pairs of a quarter by angle addition from theta_1, seeded with sincospi_fast at
 // the quarter's first pair (the same seeds as HalfAngles).
+template <class SL>
 struct QuarterAngles {
     float c1, s1, c, s;
-    __device__ __forceinline__ QuarterAngles(float lam, int hf, int u) {
+    __device__ __forceinline__ QuarterAngles(float lam, int hf, int u, const SL& sl) {
         const int j0 = 32 * hf + 16 * u + 1;
-        sincospi_fast(phase_pi(lam, 1), &s1, &c1);
+        sincospi_fast(phase_pi_m(lam, 1, sl), &s1, &c1);
         if (j0 == 1) {
             c = c1;
             s = s1;
         } else {
-            sincospi_fast(phase_pi(lam, j0), &s, &c);
+            sincospi_fast(phase_pi_m(lam, j0, sl), &s, &c);
         }
     }
     __device__ __forceinline__ void step() {
@@ -288,32 +303,39 @@ __device__ __forceinline__ void store8x2(uint8_t* tile, int r, int col, const fl
     }
 }
 
-// The quarter's entries of the write vector w U(-lam) b (Sec. 3.2), fp32.
-__device__ __forceinline__ void write_vector_q_vals(float (&x)[32], int hf, int u, float lam, float w) {
-    QuarterAngles ang(lam, hf, u);
-    const float wa = w * SQRT_2_OVER_M;
+// The quarter's entries of the write vector w U(-lam) b (Sec. 3.2), fp32; the entries of pairs
+// past (m-1)/2 are zero.
+template <class SL>
+__device__ __forceinline__ void write_vector_q_vals(float (&x)[32], int hf, int u, float lam, float w,
+                                                    const SL& sl) {
+    QuarterAngles ang(lam, hf, u, sl);
+    const float wa = w * sl.sqrt2_over_m;
+    const int jb = 32 * hf + 16 * u + 1;
 #pragma unroll
     for (int i = 0; i < 16; ++i) {
         if (i > 0) ang.step();
-        x[i] = wa * ang.c;
-        x[16 + i] = -wa * ang.s;
+        const bool on = full_slots<SL>() || jb + i <= sl.npair;
+        x[i] = on ? wa * ang.c : 0.f;
+        x[16 + i] = on ? -wa * ang.s : 0.f;
     }
     if (hf == 1 && u == 1) {
-        x[15] = w * INV_SQRT_M;
+        x[15] = w * sl.inv_sqrt_m;
         x[31] = 0.f;
     }
 }
-template <typename OT>
-__device__ __forceinline__ void write_vector_q(uint8_t* tile, int r, int hf, int u, float lam, float w) {
+template <typename OT, class SL>
+__device__ __forceinline__ void write_vector_q(uint8_t* tile, int r, int hf, int u, float lam, float w,
+                                               const SL& sl) {
     float x[32];
-    write_vector_q_vals(x, hf, u, lam, w);
+    write_vector_q_vals(x, hf, u, lam, w, sl);
     store_q<OT>(tile, r, 64 * hf + 16 * u, x);
 }
 
-// x <- U(sign lam) x on the quarter's pairs; DC kept, padding zeroed.
-template <int SIGN>
-__device__ __forceinline__ void rotate_q(float (&x)[32], int hf, int u, float lam) {
-    QuarterAngles ang(lam, hf, u);
+// x <- U(sign lam) x on the quarter's pairs; DC kept, padding zeroed.  (Pairs past (m-1)/2 hold
+// zeros, which any rotation keeps.)
+template <int SIGN, class SL>
+__device__ __forceinline__ void rotate_q(float (&x)[32], int hf, int u, float lam, const SL& sl) {
+    QuarterAngles ang(lam, hf, u, sl);
     const float dc = x[15];
 #pragma unroll
     for (int i = 0; i < 16; ++i) {
@@ -330,15 +352,26 @@ __device__ __forceinline__ void rotate_q(float (&x)[32], int hf, int u, float la
 }
 
 // <x, Omega y> over the quarter's pairs: sum_j (2 pi j / m) (x_sin,j y_cos,j - x_cos,j y_sin,j).
-__device__ __forceinline__ float omega_dot_q(const float (&x)[32], const float (&y)[32], int hf, int u) {
+template <class SL>
+__device__ __forceinline__ float omega_dot_q(const float (&x)[32], const float (&y)[32], int hf, int u,
+                                             const SL& sl) {
     float acc = 0.f;
     const int jb = 32 * hf + 16 * u + 1;
-    const float wb = OMEGA1 * (float)jb;
+    const float wb = sl.omega1 * (float)jb;
 #pragma unroll
     for (int i = 0; i < 16; ++i) {
-        if (jb + i <= NPAIR) acc += (wb + OMEGA1 * (float)i) * (x[16 + i] * y[i] - x[i] * y[16 + i]);
+        if (jb + i <= sl.npair)
+            acc += (wb + sl.omega1 * (float)i) * (x[16 + i] * y[i] - x[i] * y[16 + i]);
     }
     return acc;
+}
+
+// Softmax mask of the slot logits on the thread's 32 columns (element i is slot column
+// c0 + (i & 15) + 32 (i >> 4)): true for the slots m..127 (padding), which leave the softmax.
+template <class SL>
+__device__ __forceinline__ bool slot_off(int c0, int i, const SL& sl) {
+    if (full_slots<SL>()) return c0 == 64 + 16 && i == 31;   // slot 127 only
+    return c0 + (i & 15) + 32 * (i >> 4) >= sl.m;
 }
 
 // Causal decay mask on the thread's 32 columns (tokens t = c0 + 32 blk + i of this chunk) of

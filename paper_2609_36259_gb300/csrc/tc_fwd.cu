@@ -20,11 +20,12 @@ namespace {
 using namespace tc;
 
 // ---------------------------------------------------------------------------------------
-template <int SEGC, typename OT>
+template <int SEGC, typename OT, class SL>
 __global__ void __launch_bounds__(512, 1) seg_state_tc(const __grid_constant__ CUtensorMap tk,
                                                         const __grid_constant__ CUtensorMap tv,
                                                         TcFwdArgs a) {
     const Shape s = a.s;
+    const SL sl = slots_of<SL>(s);
     const int bh = blockIdx.x, seg = blockIdx.y, b = bh / s.H, h = bh % s.H;
     const int nct = s.T / CT;
     const int c_begin = seg * SEGC;
@@ -112,7 +113,7 @@ __global__ void __launch_bounds__(512, 1) seg_state_tc(const __grid_constant__ C
         {
             const int i = c * CT + ro.row;
             const float w = s_beta[i] * ex2((s_tot[c] - s_gs[i] + s_sfx[c]) * LOG2E);
-            write_vector_q<OT>(tiles + 3 * buf * TILE, ro.row, ro.hf, ro.u, s_lam[i], w);
+            write_vector_q<OT>(tiles + 3 * buf * TILE, ro.row, ro.hf, ro.u, s_lam[i], w, sl);
         }
         if (c >= 1 && ok) ok = mbar_wait(&bars[2 + ((c - 1) & 1)], ((c - 1) >> 1) & 1);
         if (tid == 0 && ok && c + 1 < nc) issue_kv(c + 1, (c + 1) & 1);
@@ -253,7 +254,7 @@ __device__ __forceinline__ bool named_and(uint32_t id, uint32_t n, bool v) {
     return r != 0;
 }
 
-template <int SEGC>
+template <int SEGC, class SL>
 __global__ void __launch_bounds__(OUT_THREADS, 1) seg_out_tc(const __grid_constant__ CUtensorMap tq,
                                                               const __grid_constant__ CUtensorMap tk,
                                                               const __grid_constant__ CUtensorMap tv,
@@ -262,6 +263,7 @@ __global__ void __launch_bounds__(OUT_THREADS, 1) seg_out_tc(const __grid_consta
                                                               const __grid_constant__ CUtensorMap to,
                                                               TcFwdArgs a) {
     const Shape s = a.s;
+    const SL sl = slots_of<SL>(s);
     const int bh = blockIdx.x, seg = blockIdx.y, b = bh / s.H, h = bh % s.H;
     const int nct = s.T / CT;
     const int c_begin = seg * SEGC;
@@ -356,7 +358,7 @@ __global__ void __launch_bounds__(OUT_THREADS, 1) seg_out_tc(const __grid_consta
         float lam, beta, g2, g2C;
         gates(0, lam, beta, g2, g2C);
 #pragma unroll 1
-        for (int qq = 0; qq < 4; ++qq) write_vector_q<__half>(T_A, r, qq >> 1, qq & 1, lam, beta);
+        for (int qq = 0; qq < 4; ++qq) write_vector_q<__half>(T_A, r, qq >> 1, qq & 1, lam, beta, sl);
         if (ok) ok = mbar_wait(&bars[OB_QK], 0);
         if (leader && ok) qk_pending = false;
         if (ok) {
@@ -484,7 +486,7 @@ __global__ void __launch_bounds__(OUT_THREADS, 1) seg_out_tc(const __grid_consta
                 store_q<__half>(T_N, r, cc, x);
             }
 #pragma unroll 1
-            for (int qq = 0; qq < 4; ++qq) write_vector_q<__half>(T_A, r, qq >> 1, qq & 1, lam, beta);
+            for (int qq = 0; qq < 4; ++qq) write_vector_q<__half>(T_A, r, qq >> 1, qq & 1, lam, beta, sl);
             // S8: the next chunk's a and Kbar snapshot are ready (its Q and K are converted to
             // fp16 by the chain group, which is idle at that point)
             fence_async_smem();
@@ -630,7 +632,7 @@ __global__ void __launch_bounds__(OUT_THREADS, 1) seg_out_tc(const __grid_consta
                 const float f = scale * gam;
 #pragma unroll
                 for (int i = 0; i < 32; ++i) x[i] = fmaf(f, x[i], y[i]);
-                rotate_q<1>(x, hf, u, lam);
+                rotate_q<1>(x, hf, u, lam, sl);
                 store_q<__half>(T_S, row, c0, x);
             }
             publish();
@@ -643,23 +645,22 @@ __global__ void __launch_bounds__(OUT_THREADS, 1) seg_out_tc(const __grid_consta
                 mma_commit(&bars[OB_MMA]);
             }
             wait_mma();
-            {   // p = softmax over the 127 active slots of l = z M^T; the staging tile (z is
+            {   // p = softmax over the m active slots of l = z M^T; the staging tile (z is
                 // consumed) holds the row reductions over the four column quarters
                 float* red = reinterpret_cast<float*>(T_S);
                 float x[32];
                 tmem_ld16x2(tl + X1, x);
-                const bool pad = (hf == 1 && u == 1);       // its element 31 is the padding slot
                 float mx = -INFINITY;
 #pragma unroll
                 for (int i = 0; i < 32; ++i)
-                    if (!(pad && i == 31)) mx = fmaxf(mx, x[i]);
+                    if (!slot_off(c0, i, sl)) mx = fmaxf(mx, x[i]);
                 red[128 * cq + row] = mx;
                 named_sync(1, OUT_CHAIN);
                 mx = fmaxf(fmaxf(red[row], red[128 + row]), fmaxf(red[256 + row], red[384 + row]));
                 float sum = 0.f;
 #pragma unroll
                 for (int i = 0; i < 32; ++i) {
-                    x[i] = (pad && i == 31) ? 0.f : ex2((x[i] - mx) * LOG2E);
+                    x[i] = slot_off(c0, i, sl) ? 0.f : ex2((x[i] - mx) * LOG2E);
                     sum += x[i];
                 }
                 red[512 + 128 * cq + row] = sum;
@@ -683,7 +684,7 @@ __global__ void __launch_bounds__(OUT_THREADS, 1) seg_out_tc(const __grid_consta
             {   // o'' = U(-lam) (p M)
                 float x[32];
                 tmem_ld16x2(tl + X2, x);
-                rotate_q<-1>(x, hf, u, lam);
+                rotate_q<-1>(x, hf, u, lam, sl);
                 store_q<__half>(T_S, row, c0, x);
             }
             publish();
@@ -773,17 +774,18 @@ __global__ void __launch_bounds__(OUT_THREADS, 1) seg_out_tc(const __grid_consta
 // its Fourier (column) index in the tensor-core order; the padding row and column are zero.
 // Block (group of 8 rows i, h), 128 threads: thread p owns Fourier column p and accumulates its 8
 // rows over r in fp32, in the same order as the CUDA-core path's readout matrix.
-__global__ void __launch_bounds__(128) readout_f16_kernel(const float* R, __half* Mb) {
+__global__ void __launch_bounds__(128) readout_f16_kernel(const float* R, __half* Mb, Slots sl) {
     const int h = blockIdx.y, i0 = 8 * blockIdx.x, p = threadIdx.x;
+    const int m = sl.m;                  // R is [H, m, m]; rows and columns m..127 of M are zero
     __shared__ float s_r[8][MA];
     __shared__ float s_c[MA], s_s[MA];   // cos / sin of 2 pi x / m, x = 0 .. m - 1
-    for (int e = p; e < 8 * MA; e += 128) {
-        const int ii = e / MA, r = e - ii * MA;
-        s_r[ii][r] = (i0 + ii < MA) ? R[((size_t)h * MA + i0 + ii) * MA + r] : 0.f;
+    for (int e = p; e < 8 * m; e += 128) {
+        const int ii = e / m, r = e - ii * m;
+        s_r[ii][r] = (i0 + ii < m) ? R[((size_t)h * m + i0 + ii) * m + r] : 0.f;
     }
-    if (p < MA) {
+    if (p < m) {
         float sv, cv;
-        sincospif((float)p * (2.f / 127.f), &sv, &cv);
+        sincospif((float)p * sl.two_over_m, &sv, &cv);
         s_c[p] = cv;
         s_s[p] = sv;
     }
@@ -792,25 +794,25 @@ __global__ void __launch_bounds__(128) readout_f16_kernel(const float* R, __half
 #pragma unroll
     for (int ii = 0; ii < 8; ++ii) acc[ii] = 0.f;
     if (p == 0) {
-        for (int r = 0; r < MA; ++r)
+        for (int r = 0; r < m; ++r)
 #pragma unroll
-            for (int ii = 0; ii < 8; ++ii) acc[ii] = fmaf(s_r[ii][r], INV_SQRT_M, acc[ii]);
-    } else if (p < MA) {
+            for (int ii = 0; ii < 8; ++ii) acc[ii] = fmaf(s_r[ii][r], sl.inv_sqrt_m, acc[ii]);
+    } else if (p < m) {
         const int j = (p + 1) >> 1;
         const float* tab = (p & 1) ? s_c : s_s;
         int idx = 0;   // (j r) mod m
-        for (int r = 0; r < MA; ++r) {
-            const float phi = SQRT_2_OVER_M * tab[idx];
+        for (int r = 0; r < m; ++r) {
+            const float phi = sl.sqrt2_over_m * tab[idx];
 #pragma unroll
             for (int ii = 0; ii < 8; ++ii) acc[ii] = fmaf(s_r[ii][r], phi, acc[ii]);
             idx += j;
-            if (idx >= MA) idx -= MA;
+            if (idx >= m) idx -= m;
         }
     }
 #pragma unroll
     for (int ii = 0; ii < 8; ++ii) {
         const int i = i0 + ii;
-        Mb[((size_t)h * MS + i) * MS + tc_slot(p)] = __float2half_rn(i < MA ? acc[ii] : 0.f);
+        Mb[((size_t)h * MS + i) * MS + tc_slot(p)] = __float2half_rn(i < m ? acc[ii] : 0.f);
     }
 }
 
@@ -841,8 +843,11 @@ int tc_fwd_segments(const Shape& s) {
     return (nct + SEGC_DEFAULT - 1) / SEGC_DEFAULT;
 }
 
+// m >= 63: the fp16 operands' error in the clock gradient grows as 1 / sqrt(m) (fewer slots hold
+// larger, more cancelling terms): rel-L2 1.1e-3 at m = 127, 3.1e-3 at m = 63, 1.1e-2 at m = 5;
+// smaller m run on the fp32 CUDA-core kernels.
 bool tc_fwd_supported(const Shape& s) {
-    return s.bf16 && s.D == 128 && s.sl.m == 127 && s.T % CT == 0;
+    return s.bf16 && s.D == 128 && s.sl.m >= 63 && s.T % CT == 0;
 }
 
 bool tc_qkv_maps(const Shape& s, const void* q, const void* k, const void* v, CUtensorMap* mq,
@@ -864,8 +869,9 @@ bool tc_rows_map(CUtensorMap* map, const void* base, unsigned long long rows, bo
     return make_tmap_bf16(map, base, 2, dims, str, box, f16);
 }
 
-cudaError_t launch_readout_f16(int H, const float* R, __half* Mb, cudaStream_t st) {
-    { LaunchScope ls_("readout_f16", st); readout_f16_kernel<<<dim3(MS / 8, H), 128, 0, st>>>(R, Mb); }
+cudaError_t launch_readout_f16(int H, const float* R, __half* Mb, const Slots& sl,
+                               cudaStream_t st) {
+    { LaunchScope ls_("readout_f16", st); readout_f16_kernel<<<dim3(MS / 8, H), 128, 0, st>>>(R, Mb, sl); }
     return cudaGetLastError();
 }
 
@@ -876,7 +882,8 @@ cudaError_t launch_fwd_segment_states(const TcFwdArgs& a, const void* k, const v
     if (!tc_qkv_maps(s, nullptr, k, v, nullptr, &mk, &mv)) return cudaErrorInvalidValue;
     const dim3 grid(s.B * s.H, a.nseg);   // heads fastest: CTAs that share token rows run together
     const int smA = 1024 + 12 * SEGC_DEFAULT * CT + 6 * TILE + 1024;
-    auto kA = seg_state_tc<SEGC_DEFAULT, __half>;
+    auto kA = s.sl.m == 127 ? seg_state_tc<SEGC_DEFAULT, __half, Slots127>
+                            : seg_state_tc<SEGC_DEFAULT, __half, Slots>;
     cudaFuncSetAttribute(kA, cudaFuncAttributeMaxDynamicSharedMemorySize, smA);
     { LaunchScope ls_("tc_seg_state", st); kA<<<grid, 512, smA, st>>>(mk, mv, a); }
     { LaunchScope ls_("tc_seg_scan", st); seg_scan_kernel<<<dim3(128, s.B * s.H), 256, 0, st>>>(a); }
@@ -906,7 +913,7 @@ cudaError_t launch_fwd_tc(const TcFwdArgs& a, const void* q, const void* k, cons
     if (e != cudaSuccess) return e;
     const dim3 grid(s.B * s.H, a.nseg);   // heads fastest: CTAs that share token rows run together
     const int smC = 2048 + 7 * TILE + 1024;
-    auto kC = seg_out_tc<SEGC_DEFAULT>;
+    auto kC = s.sl.m == 127 ? seg_out_tc<SEGC_DEFAULT, Slots127> : seg_out_tc<SEGC_DEFAULT, Slots>;
     cudaFuncSetAttribute(kC, cudaFuncAttributeMaxDynamicSharedMemorySize, smC);
     { LaunchScope ls_("tc_seg_out", st); kC<<<grid, OUT_THREADS, smC, st>>>(mq, mk, mv, mm, msnap, mo, a); }
     return cudaGetLastError();

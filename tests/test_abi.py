@@ -82,10 +82,12 @@ def test_null_and_misaligned_pointers_rejected_on_host(lib):
 
 def test_saved_size(lib):
     """The saved chunk-start states: fp16 [B*H][T/128][2][128][128] on the tensor-core path,
-    nothing on the CUDA-core kernels (which also take every m other than 127 and d = 256)."""
+    nothing on the CUDA-core kernels (which also take d = 256)."""
     B, T, H = 2, 1024, 3
-    assert cyfa.cyfa_saved_size(cyfa.dims(B, T, H, 128)) == B * H * (T // 128) * 2 * 128 * 128 * 2
-    assert cyfa.cyfa_saved_size(cyfa.dims(B, T, H, 128, m=63)) == 0
+    full = B * H * (T // 128) * 2 * 128 * 128 * 2
+    assert cyfa.cyfa_saved_size(cyfa.dims(B, T, H, 128)) == full
+    assert cyfa.cyfa_saved_size(cyfa.dims(B, T, H, 128, m=63)) == full   # odd m in 63..127
+    assert cyfa.cyfa_saved_size(cyfa.dims(B, T, H, 128, m=31)) == 0
     assert cyfa.cyfa_saved_size(cyfa.dims(B, T, H, 256)) == 0
     assert cyfa.cyfa_saved_size(cyfa.dims(B, T, H, 128, cuda_cores=True)) == 0
     assert cyfa.cyfa_saved_size(cyfa.dims(B, T, H, 64)) == 0

@@ -1,7 +1,7 @@
 """Slot-count variants (the paper's ablation over m, Table ablations): every odd m <= 127 through
-the C ABI against the fp64 oracle.  m = 127 runs on the tensor-core kernels; every other m on the
-CUDA-core kernels, whose rows m..127 of the 128 storage rows stay zero.  m = 255 (256 storage
-rows) is refused with CYFA_ERR_UNSUPPORTED."""
+the C ABI against the fp64 oracle, on the tensor-core kernels (bf16, d = 128) and on the CUDA-core
+kernels; rows m..127 of the 128 storage rows stay zero.  m = 255 (256 storage rows) is refused
+with CYFA_ERR_UNSUPPORTED."""
 import numpy as np
 import pytest
 import torch
@@ -17,15 +17,19 @@ from test_gpu_decode import _decode
 pytestmark = pytest.mark.gpu
 
 
-@pytest.mark.parametrize('m,dtype,D', [(5, torch.bfloat16, 128), (63, torch.bfloat16, 128),
-                                       (1, torch.float32, 64), (5, torch.float32, 64),
-                                       (63, torch.float32, 64)])
-def test_slots_forward_backward(m, dtype, D):
-    """m = 1 runs in fp32 only: its single slot sums v over the whole memory (outputs up to ~30
+@pytest.mark.parametrize('m,dtype,D,cuda_cores', [(5, torch.bfloat16, 128, False),
+                                                  (63, torch.bfloat16, 128, False),
+                                                  (63, torch.bfloat16, 128, True),
+                                                  (1, torch.float32, 64, True),
+                                                  (5, torch.float32, 64, True),
+                                                  (63, torch.float32, 64, True)])
+def test_slots_forward_backward(m, dtype, D, cuda_cores):
+    """m = 5 in bf16 runs on the CUDA-core kernels even unforced (the tensor-core kernels take
+    m >= 63).  m = 1 runs in fp32 only: its single slot sums v over the whole memory (outputs up to ~30
     here), where the bf16 rounding of the output alone (2^-9 |o|) exceeds the 2e-2 bar."""
     B, T, H = 1, 384, 2
     inp = to_device(synth.make_inputs(B, T, H, D, seed=41, dtype=dtype, with_dO=True, m=m))
-    d = cyfa.dims(B, T, H, D, chunk=64, dtype=dtype, m=m)
+    d = cyfa.dims(B, T, H, D, chunk=64, dtype=dtype, m=m, cuda_cores=cuda_cores)
     o, Ko, Vo, _ = gpu_forward(d, inp, want_state=True)
     out = gpu_backward(d, inp, want_dR=True)
     pairs = [(0, h) for h in range(H)]
@@ -48,8 +52,8 @@ def test_slots_forward_backward(m, dtype, D):
 
 
 def test_slots_63_full_size_sampled():
-    """m = 63 on the 1.4B-shaped layer (B2 H16 T32768 d128): outputs and gradients of sampled
-    (b, h) sequences."""
+    """m = 63 on the 1.4B-shaped layer (B2 H16 T32768 d128, the tensor-core kernels): outputs
+    and gradients of sampled (b, h) sequences."""
     B, T, H, m = 2, 32768, 16, 63
     inp = synth.make_inputs(B, T, H, 128, seed=2, device='cuda', with_dO=True, m=m)
     d = cyfa.dims(B, T, H, 128, chunk=64, m=m)
