@@ -413,10 +413,11 @@ def run_ours(args):
         varlen = run_varlen(args, dev, rank)
 
     # the paper's own kernel shape (H = 4, d = 256, T = 2048, B = 32)
-    paper = slots = None
+    paper = slots = slots255 = None
     if not args.no_paper_shape:
         paper = run_paper_shape(args, dev, rank, peaks)
         slots = run_slots_variant(args, dev, rank, peaks)
+        slots255 = run_slots_255(args, dev, rank, peaks)
 
     mixer = None if args.no_mixer else run_mixer(args, dev, rank, peaks)
 
@@ -440,7 +441,8 @@ def run_ours(args):
         'roofline': roof, 'kernel_rooflines': rooflines, 'cpu_baseline': cpu, 'e2e': e2e, 'gpu_launches': launches,
         'clocks': clk, 'tensor_frac': tensor_frac, 'fwd': fwd, 'bwd': bwd,
         'prepare_ms': prep_ms, 'kernel_ms_per_step': step_ms_kernels, 'decode': dec,
-        'varlen': varlen, 'paper_shape': paper, 'slots_m63': slots, 'mixer': mixer,
+        'varlen': varlen, 'paper_shape': paper, 'slots_m63': slots, 'slots_m255': slots255,
+        'mixer': mixer,
         'kernels': per_kernel,
     }
     if rank == 0:
@@ -523,6 +525,13 @@ def run_slots_variant(args, dev, rank, peaks):
     """The same step on the 1.4B-shaped layer with m = 63 slots (the paper's slot ablation)."""
     return run_extra_shape(args, dev, rank, peaks, LAYER['B'], LAYER['T'], LAYER['H'],
                            LAYER['d'], 63, 'the 1.4B layer with m = 63 (slot ablation)')
+
+
+def run_slots_255(args, dev, rank, peaks):
+    """m = 255 slots (256 storage rows) at the shape of the paper's ablation model (400M:
+    B = 32, T = 2048, H = 4, d = 256), the slot ablation's best variant."""
+    return run_extra_shape(args, dev, rank, peaks, 32, 2048, 4, 256, 255,
+                           'the 400M ablation shape with m = 255 (slot ablation)')
 
 
 def run_extra_shape(args, dev, rank, peaks, B, T, H, D, m, what):

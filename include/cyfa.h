@@ -23,18 +23,19 @@
  *   *_logit, lam_mod, g_cum, beta, d_*_logit   [B, T, H] fp32
  *   A                 [H] fp32 (> 0)
  *   R, dR             [H, m, m] fp32
- *   Kbar, Vbar        [B, H, 128, dk] / [B, H, 128, dv] fp32; rows in the order of the real
- *                     Fourier basis of App. A.1 Eq. app-real-fourier (DC, cos_1, sin_1, ...,
- *                     cos_p, sin_p with p = (m-1)/2) followed by 128 - m padding rows that
- *                     stay zero (App. A.7; one row at m = 127).
+ *   Kbar, Vbar        [B, H, ms, dk] / [B, H, ms, dv] fp32 with ms = 128 storage rows for
+ *                     m <= 127 and 256 above; rows in the order of the real Fourier basis of
+ *                     App. A.1 Eq. app-real-fourier (DC, cos_1, sin_1, ..., cos_p, sin_p with
+ *                     p = (m-1)/2) followed by ms - m padding rows that stay zero (App. A.7;
+ *                     one row at m = 127 and at m = 255).
  *   lambda            [B, H] fp64 (the running clock)
  *   stream            a cudaStream_t passed as void*; every call is asynchronous on it.
  *
- * Shapes supported: odd m in 1..127 (128 storage rows; m = 255 is CYFA_ERR_UNSUPPORTED),
- * dk = dv in {64, 128, 256}, chunk in {64, 128}, T a positive multiple of chunk (for
- * cyfa_prepare / cyfa_chunk_fwd / cyfa_chunk_bwd), B * H <= 65535.  The tensor-core kernels
- * take bf16 with d = 128, 63 <= m <= 127 and T a multiple of 128; every other supported shape
- * runs on the fp32 CUDA-core kernels.
+ * Shapes supported: odd m in 1..255 (128 storage rows up to m = 127, 256 above), dk = dv in
+ * {64, 128, 256}, chunk in {64, 128}, T a positive multiple of chunk (for cyfa_prepare /
+ * cyfa_chunk_fwd / cyfa_chunk_bwd), B * H <= 65535.  The tensor-core kernels take bf16 with
+ * d = 128, 63 <= m <= 127 and T a multiple of 128; every other supported shape runs on the fp32
+ * CUDA-core kernels.
  *
  * Errors: every entry point returns CYFA_OK (0) or a negative code.  Argument errors are
  * found on the host before anything is launched.  CYFA_ERR_TIMEOUT (a bounded wait expired)
@@ -71,7 +72,7 @@ enum { CYFA_WS_PREPARE = 0, CYFA_WS_FWD = 1, CYFA_WS_BWD = 2, CYFA_WS_PREPARE_VA
 typedef struct cyfa_dims {
     int B, T, H;   /* batch, sequence length, heads */
     int dk, dv;    /* head dims (dk == dv) */
-    int m;         /* active relative-time slots: odd, 1..127 (the paper's default is 127) */
+    int m;         /* active relative-time slots: odd, 1..255 (the paper's default is 127) */
     int chunk;     /* tokens per chunk: 64 or 128 */
     float scale;   /* dot-product scale s; the query enters the key pass as s*q */
     int dtype;     /* CYFA_DTYPE_BF16 or CYFA_DTYPE_FP32 for q, k, v, o, dO, dq, dk, dv */
@@ -79,7 +80,8 @@ typedef struct cyfa_dims {
 } cyfa_dims_t;
 
 /* dims.flags: run the chunk calls on the fp32 CUDA-core kernels even where the tensor-core
- * kernels apply (bf16, d = 128, T a multiple of 128).  Slower; exact fp32 intermediates. */
+ * kernels apply (bf16, d = 128, 63 <= m <= 127, T a multiple of 128).  Slower; exact fp32
+ * intermediates. */
 enum { CYFA_FLAG_CUDA_CORES = 1 };
 
 /* Library version as 10000*major + 100*minor + patch. */
@@ -235,7 +237,8 @@ int cyfa_chunk_bwd(const cyfa_dims_t* dims, const void* q, const void* k, const 
  * cyfa_step -- one decode token for every (b, h), in place on the persistent state
  * (Sec. 3.2 Eq. cyfa-absolute-recurrence and Eq. cyfa-absolute-readout, one step).
  * q, k, v, o are [B, H, d] (dims.T is ignored); the logits are [B, H] fp32.
- * Kbar, Vbar [B, H, 128, d] fp32 and lambda [B, H] fp64 are read and overwritten.
+ * Kbar, Vbar [B, H, ms, d] fp32 (ms = 128 for m <= 127, 256 above) and lambda [B, H] fp64 are
+ * read and overwritten.
  * Needs no workspace.
  */
 int cyfa_step(const cyfa_dims_t* dims, const void* q, const void* k, const void* v,

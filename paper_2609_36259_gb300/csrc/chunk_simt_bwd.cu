@@ -1,4 +1,4 @@
-// fp32 SIMT backward of the CyFA operator (chunk length 64).
+// fp32 SIMT backward of the CyFA operator (chunk length 64 with 128 storage rows, 32 with 256).
 //
 // The forward (App. B Eqs. app-cyfa-key-chunk / app-cyfa-value-chunk with the middle line of
 // Sec. 3.3 Eq. cyfa-two-pass) is differentiated chunk by chunk:
@@ -22,21 +22,34 @@ namespace cyfa {
 
 namespace {
 
-constexpr int CB = BWD_C;          // 64
-constexpr int LPB = CB + 1;
-constexpr int TMB = CB / 16;       // 4 rows per thread
+// Tile geometry for MSZ storage rows: chunks of CB tokens (64 with 128 rows; 32 with 256, so
+// that five [CB][MSZ + 1] tiles still fit in shared memory); TMB rows per thread.
+template <int MSZ>
+struct Geo {
+    static constexpr int CB = MSZ == 128 ? BWD_C : BWD_C256;
+    static constexpr int LPB = CB + 1, TMB = CB / 16, LDM = MSZ + 1, NJ = MSZ / 16;
+    static constexpr int NP = MSZ / 64, NE = MSZ / 32, NPAIRS = MSZ / 2 - 1;
+};
+// Floats of the staging tile: the larger of a [CB][MSZ + 1] tile, the Q / Kbar column staging
+// ((CB + MSZ) x 33) and the state-row staging (32 x (D + 1)).
+template <int D, int MSZ>
+__host__ __device__ constexpr int staging_floats() {
+    constexpr int a = Geo<MSZ>::CB * Geo<MSZ>::LDM, b = (Geo<MSZ>::CB + MSZ) * 33, c = 32 * (D + 1);
+    return a > b ? (a > c ? a : c) : (b > c ? b : c);
+}
 
 // 2 pi j / m, the rotation rate of pair j
 __device__ __forceinline__ float freq(int j, const Slots& sl) {
     return (6.283185307179586f * sl.inv_m) * (float)j;
 }
 
-// <x, Omega y> for 128-vectors in shared memory, summed over the warp (pairs j = lane+1, lane+33).
+// <x, Omega y> for MSZ-vectors in shared memory, summed over the warp (pairs j = lane+1+32u).
+template <int MSZ>
 __device__ __forceinline__ float warp_omega_dot(const float* x, const float* y, int lane,
                                                 const Slots& sl) {
     float acc = 0.f;
 #pragma unroll
-    for (int u = 0; u < 2; ++u) {
+    for (int u = 0; u < Geo<MSZ>::NP; ++u) {
         const int j = lane + 1 + 32 * u;
         if (j <= sl.npair)
             acc += freq(j, sl) * (x[2 * j] * y[2 * j - 1] - x[2 * j - 1] * y[2 * j]);
@@ -47,26 +60,30 @@ __device__ __forceinline__ float warp_omega_dot(const float* x, const float* y, 
 // Gradient of the middle readout, one warp per row:
 // given o' (sO1), o'' (sO2) and dL/do'' (sD), writes dL/do' into sD and the row scalars
 // sdG[r] = <o'', do''> and sdL[r] = <dz, Omega z> - <do'', Omega o''>.  With gz non-null the
-// row's z, p, dy, dl (for dR) go to gz / gp / gdy / gdl + 128 r.
+// row's z, p, dy, dl (for dR) go to gz / gp / gdy / gdl + MSZ r.  Rows have stride MSZ + 1;
+// swarp holds 5 x MSZ floats per warp.
+template <int MSZ>
 __device__ __noinline__ void middle_rows_bwd(const float* sO1, const float* sO2, float* sD,
                                              const float* slam, int C, const float* M,
                                              const float* MT, float* swarp, float* sdG,
                                              float* sdL, float* gz, float* gp, float* gdy,
                                              float* gdl, const Slots& sl) {
+    using G = Geo<MSZ>;
+    constexpr int NP = G::NP, NE = G::NE;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    float* z = swarp + warp * 640;
-    float* p = z + 128;
-    float* dy = p + 128;
-    float* dl = dy + 128;
-    float* dz = dl + 128;
+    float* z = swarp + warp * 5 * MSZ;
+    float* p = z + MSZ;
+    float* dy = p + MSZ;
+    float* dl = dy + MSZ;
+    float* dz = dl + MSZ;
     for (int r = warp; r < C; r += 8) {
-        const float* x1 = sO1 + r * LD;
-        const float* x2 = sO2 + r * LD;
-        float* xd = sD + r * LD;
+        const float* x1 = sO1 + r * G::LDM;
+        const float* x2 = sO2 + r * G::LDM;
+        float* xd = sD + r * G::LDM;
         const float lam = slam[r];
-        float cs[2], sn[2];
+        float cs[NP], sn[NP];
 #pragma unroll
-        for (int u = 0; u < 2; ++u) {
+        for (int u = 0; u < NP; ++u) {
             const int j = lane + 1 + 32 * u;
             cs[u] = 1.f;
             sn[u] = 0.f;
@@ -78,41 +95,46 @@ __device__ __noinline__ void middle_rows_bwd(const float* sO1, const float* sO2,
                 const float gc = xd[2 * j - 1], gs = xd[2 * j];
                 dy[2 * j - 1] = cs[u] * gc - sn[u] * gs;     // dy = U(lam) do''
                 dy[2 * j] = sn[u] * gc + cs[u] * gs;
-            } else if (j <= NPAIR) {   // padding slots (zero)
+            } else if (j <= G::NPAIRS) {   // padding slots (zero)
                 z[2 * j - 1] = z[2 * j] = 0.f;
                 dy[2 * j - 1] = dy[2 * j] = 0.f;
             }
         }
         if (lane == 0) {
             z[0] = x1[0];
-            z[127] = 0.f;
+            z[MSZ - 1] = 0.f;
             dy[0] = xd[0];
-            dy[127] = 0.f;
+            dy[MSZ - 1] = 0.f;
         }
         __syncwarp();
         float g1 = 0.f;
 #pragma unroll
-        for (int u = 0; u < 4; ++u) g1 += x2[lane + 32 * u] * xd[lane + 32 * u];
+        for (int u = 0; u < NE; ++u) g1 += x2[lane + 32 * u] * xd[lane + 32 * u];
         g1 = warp_sum(g1);
-        const float om2 = warp_omega_dot(xd, x2, lane, sl);  // <do'', Omega o''>
+        const float om2 = warp_omega_dot<MSZ>(xd, x2, lane, sl);  // <do'', Omega o''>
         // logits and softmax
-        float l[4] = {0.f, 0.f, 0.f, 0.f}, dp[4] = {0.f, 0.f, 0.f, 0.f};
-        for (int k = 0; k < MS; ++k) {
+        float l[NE], dp[NE];
+#pragma unroll
+        for (int u = 0; u < NE; ++u) l[u] = dp[u] = 0.f;
+        for (int k = 0; k < MSZ; ++k) {
             const float zk = z[k], dyk = dy[k];
 #pragma unroll
-            for (int u = 0; u < 4; ++u) {
-                const float mt = MT[k * MS + lane + 32 * u];
+            for (int u = 0; u < NE; ++u) {
+                const float mt = MT[k * MSZ + lane + 32 * u];
                 l[u] = fmaf(mt, zk, l[u]);
                 dp[u] = fmaf(mt, dyk, dp[u]);           // dp = M dy
             }
         }
+        float mx = -INFINITY;
 #pragma unroll
-        for (int u = 0; u < 4; ++u)
+        for (int u = 0; u < NE; ++u) {
             if (lane + 32 * u >= sl.m) l[u] = -INFINITY;
-        float mx = warp_max(fmaxf(fmaxf(l[0], l[1]), fmaxf(l[2], l[3])));
-        float e[4], sum = 0.f;
+            mx = fmaxf(mx, l[u]);
+        }
+        mx = warp_max(mx);
+        float e[NE], sum = 0.f;
 #pragma unroll
-        for (int u = 0; u < 4; ++u) {
+        for (int u = 0; u < NE; ++u) {
             e[u] = expf(l[u] - mx);
             sum += e[u];
         }
@@ -120,39 +142,41 @@ __device__ __noinline__ void middle_rows_bwd(const float* sO1, const float* sO2,
         const float inv = 1.f / sum;
         float pdp = 0.f;
 #pragma unroll
-        for (int u = 0; u < 4; ++u) {
+        for (int u = 0; u < NE; ++u) {
             e[u] *= inv;
             pdp += e[u] * dp[u];
         }
         pdp = warp_sum(pdp);
 #pragma unroll
-        for (int u = 0; u < 4; ++u) dl[lane + 32 * u] = e[u] * (dp[u] - pdp);
+        for (int u = 0; u < NE; ++u) dl[lane + 32 * u] = e[u] * (dp[u] - pdp);
         if (gz) {
 #pragma unroll
-            for (int u = 0; u < 4; ++u) {
+            for (int u = 0; u < NE; ++u) {
                 const int k = lane + 32 * u;
-                gz[r * 128 + k] = z[k];
-                gp[r * 128 + k] = e[u];
-                gdy[r * 128 + k] = dy[k];
-                gdl[r * 128 + k] = e[u] * (dp[u] - pdp);
+                gz[r * MSZ + k] = z[k];
+                gp[r * MSZ + k] = e[u];
+                gdy[r * MSZ + k] = dy[k];
+                gdl[r * MSZ + k] = e[u] * (dp[u] - pdp);
             }
         }
         __syncwarp();
-        float g[4] = {0.f, 0.f, 0.f, 0.f};                   // dz = M^T dl
+        float g[NE];                                         // dz = M^T dl
+#pragma unroll
+        for (int u = 0; u < NE; ++u) g[u] = 0.f;
         for (int i = 0; i < sl.m; ++i) {
             const float di = dl[i];
 #pragma unroll
-            for (int u = 0; u < 4; ++u) g[u] = fmaf(M[i * MS + lane + 32 * u], di, g[u]);
+            for (int u = 0; u < NE; ++u) g[u] = fmaf(M[i * MSZ + lane + 32 * u], di, g[u]);
         }
 #pragma unroll
-        for (int u = 0; u < 4; ++u) dz[lane + 32 * u] = g[u];
+        for (int u = 0; u < NE; ++u) dz[lane + 32 * u] = g[u];
         __syncwarp();
-        const float om1 = warp_omega_dot(dz, z, lane, sl);   // <dz, Omega z>
+        const float om1 = warp_omega_dot<MSZ>(dz, z, lane, sl);   // <dz, Omega z>
         // do' = U(-lam) dz
 #pragma unroll
-        for (int u = 0; u < 2; ++u) {
+        for (int u = 0; u < NP; ++u) {
             const int j = lane + 1 + 32 * u;
-            if (j <= NPAIR) {
+            if (j <= G::NPAIRS) {
                 const float gc = dz[2 * j - 1], gs = dz[2 * j];
                 xd[2 * j - 1] = cs[u] * gc + sn[u] * gs;
                 xd[2 * j] = -sn[u] * gc + cs[u] * gs;
@@ -160,7 +184,7 @@ __device__ __noinline__ void middle_rows_bwd(const float* sO1, const float* sO2,
         }
         if (lane == 0) {
             xd[0] = dz[0];
-            xd[127] = 0.f;
+            xd[MSZ - 1] = 0.f;
             sdG[r] = g1;
             sdL[r] = om1 - om2;
         }
@@ -168,10 +192,12 @@ __device__ __noinline__ void middle_rows_bwd(const float* sO1, const float* sO2,
     }
 }
 
-// sP[r][t] = mul * (sum_k X(r,k) Y(t,k)) * exp(g_r - g_t) for t <= r, else 0
-template <class FX, class FY>
+// sP[r][t] = mul * (sum_k X(r,k) Y(t,k)) * exp(g_r - g_t) for t <= r, else 0  (r, t < CB)
+template <int MSZ, class FX, class FY>
 __device__ __forceinline__ void masked_scores(float* sP, const float* sg, int K, float mul,
                                               const FX& fx, const FY& fy) {
+    using G = Geo<MSZ>;
+    constexpr int TMB = G::TMB;
     const int tx = threadIdx.x & 15, ty = threadIdx.x >> 4;
     float acc[TMB][TMB];
     zero_acc(acc);
@@ -181,15 +207,17 @@ __device__ __forceinline__ void masked_scores(float* sP, const float* sg, int K,
 #pragma unroll
         for (int j = 0; j < TMB; ++j) {
             const int r = ty + 16 * i, t = tx + 16 * j;
-            sP[r * LPB + t] = (t <= r) ? acc[i][j] * mul * expf(sg[r] - sg[t]) : 0.f;
+            sP[r * G::LPB + t] = (t <= r) ? acc[i][j] * mul * expf(sg[r] - sg[t]) : 0.f;
         }
 }
 
 // masked scores from two token tensors staged 32 columns at a time through sS
-template <typename TI>
+template <int MSZ, typename TI>
 __device__ __forceinline__ void masked_scores_tok(float* sP, float* sS, const float* sg,
                                                   const TI* X, const TI* Y, const Shape& s, int b,
                                                   int h, int t0, float mul) {
+    using G = Geo<MSZ>;
+    constexpr int TMB = G::TMB, CB = G::CB;
     const int tx = threadIdx.x & 15, ty = threadIdx.x >> 4;
     float acc[TMB][TMB];
     zero_acc(acc);
@@ -206,87 +234,94 @@ __device__ __forceinline__ void masked_scores_tok(float* sP, float* sS, const fl
 #pragma unroll
         for (int j = 0; j < TMB; ++j) {
             const int r = ty + 16 * i, t = tx + 16 * j;
-            sP[r * LPB + t] = (t <= r) ? acc[i][j] * mul * expf(sg[r] - sg[t]) : 0.f;
+            sP[r * G::LPB + t] = (t <= r) ? acc[i][j] * mul * expf(sg[r] - sg[t]) : 0.f;
         }
 }
 
-// acc[r][i] += sum_d X[r][d] * Sst[i][coff + d]  (X a token tensor, Sst a [128][2D] state block)
-template <typename TI>
-__device__ __forceinline__ void tok_times_stateT(float (&acc)[TMB][8], float* sS, const TI* X,
-                                                 const float* Sst, int coff, const Shape& s,
-                                                 int b, int h, int t0) {
+// acc[r][i] += sum_d X[r][d] * Sst[i][coff + d]  (X a token tensor, Sst a [MSZ][2D] state block)
+template <int MSZ, typename TI>
+__device__ __forceinline__ void tok_times_stateT(float (&acc)[Geo<MSZ>::TMB][Geo<MSZ>::NJ],
+                                                 float* sS, const TI* X, const float* Sst,
+                                                 int coff, const Shape& s, int b, int h, int t0) {
+    using G = Geo<MSZ>;
+    constexpr int CB = G::CB;
     for (int d0 = 0; d0 < s.D; d0 += 32) {
         __syncthreads();
         stage_tok(sS, X, s, b, h, t0, CB, d0, 1.f);
-        for (int e = threadIdx.x; e < MS * 32; e += blockDim.x) {
+        for (int e = threadIdx.x; e < MSZ * 32; e += blockDim.x) {
             const int i = e >> 5, dd = e & 31;
             sS[CB * 33 + i * 33 + dd] = Sst[i * (2 * s.D) + coff + d0 + dd];
         }
         __syncthreads();
-        simt_mm<TMB, 8>(acc, 32, [&](int r, int kk) { return sS[r * 33 + kk]; },
-                        [&](int kk, int i) { return sS[CB * 33 + i * 33 + kk]; });
+        simt_mm<G::TMB, G::NJ>(acc, 32, [&](int r, int kk) { return sS[r * 33 + kk]; },
+                               [&](int kk, int i) { return sS[CB * 33 + i * 33 + kk]; });
     }
 }
 
-// acc[r][dd] += sum_i Y(r, i) * Sst[i][coff + dd]  (Y rows in shared memory with stride LD)
-template <int TN>
-__device__ __forceinline__ void rows_times_state(float (&acc)[TMB][TN], float* sS, const float* Y,
-                                                 const float* Sst, int coff, int D) {
-    for (int i0 = 0; i0 < MS; i0 += 32) {
+// acc[r][dd] += sum_i Y(r, i) * Sst[i][coff + dd]  (Y rows in shared memory with stride MSZ + 1)
+template <int MSZ, int TN>
+__device__ __forceinline__ void rows_times_state(float (&acc)[Geo<MSZ>::TMB][TN], float* sS,
+                                                 const float* Y, const float* Sst, int coff,
+                                                 int D) {
+    using G = Geo<MSZ>;
+    for (int i0 = 0; i0 < MSZ; i0 += 32) {
         __syncthreads();
         for (int e = threadIdx.x; e < 32 * D; e += blockDim.x) {
             const int ii = e / D, dd = e % D;
             sS[ii * (D + 1) + dd] = Sst[(i0 + ii) * (2 * D) + coff + dd];
         }
         __syncthreads();
-        simt_mm<TMB, TN>(acc, 32, [&](int r, int ii) { return Y[r * LD + i0 + ii]; },
-                         [&](int ii, int dd) { return sS[ii * (D + 1) + dd]; });
+        simt_mm<G::TMB, TN>(acc, 32, [&](int r, int ii) { return Y[r * G::LDM + i0 + ii]; },
+                            [&](int ii, int dd) { return sS[ii * (D + 1) + dd]; });
     }
 }
 
 // acc[r][dd] += sum_t P(r, t) * X[t][dd]  with P given by an accessor (K = CB tokens)
-template <int TN, typename TI, class FP>
-__device__ __forceinline__ void scores_times_tok(float (&acc)[TMB][TN], float* sS, const FP& fp,
-                                                 const TI* X, const Shape& s, int b, int h,
-                                                 int t0, float mul) {
+template <int MSZ, int TN, typename TI, class FP>
+__device__ __forceinline__ void scores_times_tok(float (&acc)[Geo<MSZ>::TMB][TN], float* sS,
+                                                 const FP& fp, const TI* X, const Shape& s,
+                                                 int b, int h, int t0, float mul) {
+    using G = Geo<MSZ>;
     const int D = s.D;
-    for (int s0 = 0; s0 < CB; s0 += 32) {
+    for (int s0 = 0; s0 < G::CB; s0 += 32) {
         __syncthreads();
         for (int e = threadIdx.x; e < 32 * D; e += blockDim.x) {
             const int ss = e / D, dd = e % D;
             sS[ss * (D + 1) + dd] = mul * ldf(X, (((size_t)b * s.T + t0 + s0 + ss) * s.H + h) * D + dd);
         }
         __syncthreads();
-        simt_mm<TMB, TN>(acc, 32, [&](int r, int ss) { return fp(r, s0 + ss); },
-                         [&](int ss, int dd) { return sS[ss * (D + 1) + dd]; });
+        simt_mm<G::TMB, TN>(acc, 32, [&](int r, int ss) { return fp(r, s0 + ss); },
+                            [&](int ss, int dd) { return sS[ss * (D + 1) + dd]; });
     }
 }
 
 // ---------------------------------------------------------------------------------------
-template <int D, typename TI>
+template <int D, int MSZ, typename TI>
 __global__ void __launch_bounds__(256) bwd_intra1_kernel(BwdArgs a) {
+    using G = Geo<MSZ>;
+    constexpr int CB = G::CB, LDM = G::LDM, LPB = G::LPB, TMB = G::TMB, NJ = G::NJ;
     const Shape s = a.s;
     constexpr int TN = D / 16;
     const int c = blockIdx.x, bh = blockIdx.y, b = bh / s.H, h = bh % s.H;
     const int nchunk = s.nchunk(), t0 = c * CB;
     extern __shared__ float smem[];
     float* sA = smem;
-    float* sO1 = sA + CB * LD;
-    float* sO2 = sO1 + CB * LD;
-    float* sD = sO2 + CB * LD;
-    float* sS = sD + CB * LD;
-    float* sP = sS + CB * LD;
+    float* sO1 = sA + CB * LDM;
+    float* sO2 = sO1 + CB * LDM;
+    float* sD = sO2 + CB * LDM;
+    float* sS = sD + CB * LDM;                      // staging
+    float* sP = sS + staging_floats<D, MSZ>();
     float* sg = sP + CB * LPB;
     float* seg = sg + CB;
     float* slam = seg + CB;
     float* sbeta = slam + CB;
     float* sdG = sbeta + CB;
     float* sdL = sdG + CB;
-    float* swarp = sdL + CB;     // [8][640]
+    float* swarp = sdL + CB;     // [8][5 MSZ]
     const int tx = threadIdx.x & 15, ty = threadIdx.x >> 4;
-    const float* Sst = a.states + ((size_t)bh * nchunk + c) * MS * (2 * D);
-    const float* Mh = a.M + (size_t)h * MS * MS;
-    const float* MTh = a.MT + (size_t)h * MS * MS;
+    const float* Sst = a.states + ((size_t)bh * nchunk + c) * MSZ * (2 * D);
+    const float* Mh = a.M + (size_t)h * MSZ * MSZ;
+    const float* MTh = a.MT + (size_t)h * MSZ * MSZ;
     const TI* Q = (const TI*)a.q;
     const TI* K = (const TI*)a.k;
     const TI* V = (const TI*)a.v;
@@ -295,71 +330,71 @@ __global__ void __launch_bounds__(256) bwd_intra1_kernel(BwdArgs a) {
     load_gates(s, a.lam, a.g, a.beta, b, h, t0, CB, slam, sg, sbeta);
     __syncthreads();
     for (int r = threadIdx.x; r < CB; r += blockDim.x) seg[r] = expf(sg[r]);
-    build_write_rows(sA, LD, slam, sbeta, CB, s.sl, [](int) { return 1.f; });
+    build_write_rows(sA, LDM, slam, sbeta, CB, s.sl, [](int) { return 1.f; });
 
     // O' = s gamma o (Q Kbar^T) + (s Q K^T o Gamma) A
-    masked_scores_tok(sP, sS, sg, Q, K, s, b, h, t0, s.scale);
+    masked_scores_tok<MSZ>(sP, sS, sg, Q, K, s, b, h, t0, s.scale);
     {
-        float o1[TMB][8];
+        float o1[TMB][NJ];
         zero_acc(o1);
-        tok_times_stateT(o1, sS, Q, Sst, 0, s, b, h, t0);
+        tok_times_stateT<MSZ>(o1, sS, Q, Sst, 0, s, b, h, t0);
 #pragma unroll
         for (int i = 0; i < TMB; ++i)
 #pragma unroll
-            for (int j = 0; j < 8; ++j) o1[i][j] *= s.scale * seg[ty + 16 * i];
-        simt_mm<TMB, 8>(o1, CB, [&](int r, int t) { return sP[r * LPB + t]; },
-                        [&](int t, int i) { return sA[t * LD + i]; });
+            for (int j = 0; j < NJ; ++j) o1[i][j] *= s.scale * seg[ty + 16 * i];
+        simt_mm<TMB, NJ>(o1, CB, [&](int r, int t) { return sP[r * LPB + t]; },
+                         [&](int t, int i) { return sA[t * LDM + i]; });
 #pragma unroll
         for (int i = 0; i < TMB; ++i)
 #pragma unroll
-            for (int j = 0; j < 8; ++j) {
-                sO1[(ty + 16 * i) * LD + tx + 16 * j] = o1[i][j];
-                sO2[(ty + 16 * i) * LD + tx + 16 * j] = o1[i][j];
+            for (int j = 0; j < NJ; ++j) {
+                sO1[(ty + 16 * i) * LDM + tx + 16 * j] = o1[i][j];
+                sO2[(ty + 16 * i) * LDM + tx + 16 * j] = o1[i][j];
             }
     }
     __syncthreads();
-    middle_rows(sO2, slam, CB, Mh, MTh, swarp, s.sl);
+    middle_rows<MSZ>(sO2, slam, CB, Mh, MTh, swarp, s.sl);
 
     // dO'' = gamma o (dO Vbar^T) + (dO V^T o Gamma) A
-    masked_scores_tok(sP, sS, sg, dO, V, s, b, h, t0, 1.f);
+    masked_scores_tok<MSZ>(sP, sS, sg, dO, V, s, b, h, t0, 1.f);
     {
-        float g2[TMB][8];
+        float g2[TMB][NJ];
         zero_acc(g2);
-        tok_times_stateT(g2, sS, dO, Sst, D, s, b, h, t0);
+        tok_times_stateT<MSZ>(g2, sS, dO, Sst, D, s, b, h, t0);
 #pragma unroll
         for (int i = 0; i < TMB; ++i)
 #pragma unroll
-            for (int j = 0; j < 8; ++j) g2[i][j] *= seg[ty + 16 * i];
-        simt_mm<TMB, 8>(g2, CB, [&](int r, int t) { return sP[r * LPB + t]; },
-                        [&](int t, int i) { return sA[t * LD + i]; });
+            for (int j = 0; j < NJ; ++j) g2[i][j] *= seg[ty + 16 * i];
+        simt_mm<TMB, NJ>(g2, CB, [&](int r, int t) { return sP[r * LPB + t]; },
+                         [&](int t, int i) { return sA[t * LDM + i]; });
 #pragma unroll
         for (int i = 0; i < TMB; ++i)
 #pragma unroll
-            for (int j = 0; j < 8; ++j) sD[(ty + 16 * i) * LD + tx + 16 * j] = g2[i][j];
+            for (int j = 0; j < NJ; ++j) sD[(ty + 16 * i) * LDM + tx + 16 * j] = g2[i][j];
     }
     __syncthreads();
     {
-        const size_t rowbase = ((size_t)bh * s.T + t0) * MS;
+        const size_t rowbase = ((size_t)bh * s.T + t0) * MSZ;
         const bool dr = a.mZ != nullptr;
-        middle_rows_bwd(sO1, sO2, sD, slam, CB, Mh, MTh, swarp, sdG, sdL,
+        middle_rows_bwd<MSZ>(sO1, sO2, sD, slam, CB, Mh, MTh, swarp, sdG, sdL,
                         dr ? a.mZ + rowbase : nullptr, dr ? a.mP + rowbase : nullptr,
                         dr ? a.mDY + rowbase : nullptr, dr ? a.mDL + rowbase : nullptr, s.sl);
     }
     __syncthreads();
 
     // dQ~ = gamma o (dO' Kbar) + (dO' A^T o Gamma) K ;  dq = s dQ~
-    masked_scores(sP, sg, MS, 1.f, [&](int r, int kk) { return sD[r * LD + kk]; },
-                  [&](int kk, int t) { return sA[t * LD + kk]; });
+    masked_scores<MSZ>(sP, sg, MSZ, 1.f, [&](int r, int kk) { return sD[r * LDM + kk]; },
+                       [&](int kk, int t) { return sA[t * LDM + kk]; });
     {
         float dqa[TMB][TN];
         zero_acc(dqa);
-        rows_times_state<TN>(dqa, sS, sD, Sst, 0, D);
+        rows_times_state<MSZ, TN>(dqa, sS, sD, Sst, 0, D);
 #pragma unroll
         for (int i = 0; i < TMB; ++i)
 #pragma unroll
             for (int j = 0; j < TN; ++j) dqa[i][j] *= seg[ty + 16 * i];
-        scores_times_tok<TN>(dqa, sS, [&](int r, int t) { return sP[r * LPB + t]; }, K, s, b, h,
-                             t0, 1.f);
+        scores_times_tok<MSZ, TN>(dqa, sS, [&](int r, int t) { return sP[r * LPB + t]; }, K, s,
+                                  b, h, t0, 1.f);
         TI* dQ = (TI*)a.dq;
 #pragma unroll
         for (int i = 0; i < TMB; ++i) {
@@ -377,12 +412,12 @@ __global__ void __launch_bounds__(256) bwd_intra1_kernel(BwdArgs a) {
     }
     __syncthreads();
     // stash o'' and dL/do' for the adjoint scan and the second intra-chunk pass
-    float* o2 = a.o2 + ((size_t)bh * s.T + t0) * MS;
-    float* do1 = a.do1 + ((size_t)bh * s.T + t0) * MS;
-    for (int e = threadIdx.x; e < CB * MS; e += blockDim.x) {
-        const int r = e >> 7, i = e & 127;
-        o2[e] = sO2[r * LD + i];
-        do1[e] = sD[r * LD + i];
+    float* o2 = a.o2 + ((size_t)bh * s.T + t0) * MSZ;
+    float* do1 = a.do1 + ((size_t)bh * s.T + t0) * MSZ;
+    for (int e = threadIdx.x; e < CB * MSZ; e += blockDim.x) {
+        const int r = e / MSZ, i = e % MSZ;
+        o2[e] = sO2[r * LDM + i];
+        do1[e] = sD[r * LDM + i];
     }
     const size_t BTH = (size_t)s.B * s.T * s.H;
     for (int r = threadIdx.x; r < CB; r += blockDim.x) {
@@ -392,33 +427,37 @@ __global__ void __launch_bounds__(256) bwd_intra1_kernel(BwdArgs a) {
     }
 }
 
-// Reverse scan of the state adjoints, one block per (b, h, 32-column tile of [D^K | D^V]).
-// Stores, for every chunk c, the adjoint of the state at the end of chunk c.
-template <typename TI>
+// Reverse scan of the state adjoints, one block per (b, h, 32-column tile of [D^K | D^V], 128
+// of the MSZ storage rows).  Stores, for every chunk c, the adjoint of the state at the end of
+// chunk c.
+template <int MSZ, typename TI>
 __global__ void __launch_bounds__(256) adj_state_kernel(BwdArgs a) {
+    using G = Geo<MSZ>;
+    constexpr int CB = G::CB, LDM = G::LDM;
     const Shape s = a.s;
     const int D = s.D, W = 2 * s.D;
     const int bh = blockIdx.y, b = bh / s.H, h = bh % s.H;
     const int col0 = blockIdx.x * 32;
+    const int rz = 128 * blockIdx.z;   // first storage row of this block
     const bool isK = col0 < D;
     const int xc0 = isK ? col0 : col0 - D;
     const TI* X = (const TI*)(isK ? a.q : a.dO);
     const float* Y = isK ? a.do1 : a.o2;
     const float xmul = isK ? s.scale : 1.f;
     extern __shared__ float smem[];
-    float* sY = smem;            // [CB][LD]
-    float* sX = sY + CB * LD;    // [CB][33]
+    float* sY = smem;            // [CB][LDM]
+    float* sX = sY + CB * LDM;   // [CB][33]
     float* sg = sX + CB * 33;
     const int tx = threadIdx.x & 15, ty = threadIdx.x >> 4;
     float S[8][2];
     zero_acc(S);
     const int nchunk = s.nchunk();
     for (int c = nchunk - 1; c >= 0; --c) {
-        float* dst = a.adj + ((size_t)bh * nchunk + c) * MS * W;
+        float* dst = a.adj + ((size_t)bh * nchunk + c) * MSZ * W;
 #pragma unroll
         for (int i = 0; i < 8; ++i)
 #pragma unroll
-            for (int j = 0; j < 2; ++j) dst[(ty + 16 * i) * W + col0 + tx + 16 * j] = S[i][j];
+            for (int j = 0; j < 2; ++j) dst[(rz + ty + 16 * i) * W + col0 + tx + 16 * j] = S[i][j];
         const int t0 = c * CB;
         __syncthreads();
         const float gb = g_base(s, a.g, b, h, t0, CB);
@@ -426,10 +465,10 @@ __global__ void __launch_bounds__(256) adj_state_kernel(BwdArgs a) {
             sg[r] = a.g[((size_t)b * s.T + t0 + r) * s.H + h] - gb;
         stage_tok(sX, X, s, b, h, t0, CB, xc0, xmul);
         __syncthreads();
-        const float* Yc = Y + ((size_t)bh * s.T + t0) * MS;
-        for (int e = threadIdx.x; e < CB * MS; e += blockDim.x) {
-            const int r = e >> 7, i = e & 127;
-            sY[r * LD + i] = Yc[e] * expf(sg[r]);
+        const float* Yc = Y + ((size_t)bh * s.T + t0) * MSZ;
+        for (int e = threadIdx.x; e < CB * MSZ; e += blockDim.x) {
+            const int r = e / MSZ, i = e % MSZ;
+            sY[r * LDM + i] = Yc[e] * expf(sg[r]);
         }
         __syncthreads();
         const float decay = expf(sg[CB - 1]);
@@ -437,31 +476,33 @@ __global__ void __launch_bounds__(256) adj_state_kernel(BwdArgs a) {
         for (int i = 0; i < 8; ++i)
 #pragma unroll
             for (int j = 0; j < 2; ++j) S[i][j] *= decay;
-        simt_mm<8, 2>(S, CB, [&](int row, int t) { return sY[t * LD + row]; },
+        simt_mm<8, 2>(S, CB, [&](int row, int t) { return sY[t * LDM + rz + row]; },
                       [&](int t, int col) { return sX[t * 33 + col]; });
     }
 }
 
-template <int D, typename TI>
+template <int D, int MSZ, typename TI>
 __global__ void __launch_bounds__(256) bwd_intra2_kernel(BwdArgs a) {
+    using G = Geo<MSZ>;
+    constexpr int CB = G::CB, LDM = G::LDM, LPB = G::LPB, TMB = G::TMB, NJ = G::NJ;
     const Shape s = a.s;
     constexpr int TN = D / 16;
     const int c = blockIdx.x, bh = blockIdx.y, b = bh / s.H, h = bh % s.H;
     const int nchunk = s.nchunk(), t0 = c * CB;
     extern __shared__ float smem[];
     float* sA = smem;
-    float* sY1 = sA + CB * LD;     // dL/do'
-    float* sY2 = sY1 + CB * LD;    // o''
-    float* sDA = sY2 + CB * LD;    // dL/da
-    float* sS = sDA + CB * LD;
-    float* sP = sS + CB * LD;
+    float* sY1 = sA + CB * LDM;    // dL/do'
+    float* sY2 = sY1 + CB * LDM;   // o''
+    float* sDA = sY2 + CB * LDM;   // dL/da
+    float* sS = sDA + CB * LDM;    // staging
+    float* sP = sS + staging_floats<D, MSZ>();
     float* sg = sP + CB * LPB;
     float* sfw = sg + CB;
     float* slam = sfw + CB;
     float* sbeta = slam + CB;
     float* sdG = sbeta + CB;
     const int tx = threadIdx.x & 15, ty = threadIdx.x >> 4;
-    const float* Dst = a.adj + ((size_t)bh * nchunk + c) * MS * (2 * D);
+    const float* Dst = a.adj + ((size_t)bh * nchunk + c) * MSZ * (2 * D);
     const TI* Q = (const TI*)a.q;
     const TI* K = (const TI*)a.k;
     const TI* V = (const TI*)a.v;
@@ -470,12 +511,12 @@ __global__ void __launch_bounds__(256) bwd_intra2_kernel(BwdArgs a) {
 
     load_gates(s, a.lam, a.g, a.beta, b, h, t0, CB, slam, sg, sbeta);
     {
-        const float* y1 = a.do1 + ((size_t)bh * s.T + t0) * MS;
-        const float* y2 = a.o2 + ((size_t)bh * s.T + t0) * MS;
-        for (int e = threadIdx.x; e < CB * MS; e += blockDim.x) {
-            const int r = e >> 7, i = e & 127;
-            sY1[r * LD + i] = y1[e];
-            sY2[r * LD + i] = y2[e];
+        const float* y1 = a.do1 + ((size_t)bh * s.T + t0) * MSZ;
+        const float* y2 = a.o2 + ((size_t)bh * s.T + t0) * MSZ;
+        for (int e = threadIdx.x; e < CB * MSZ; e += blockDim.x) {
+            const int r = e / MSZ, i = e % MSZ;
+            sY1[r * LDM + i] = y1[e];
+            sY2[r * LDM + i] = y2[e];
         }
     }
     __syncthreads();
@@ -483,22 +524,22 @@ __global__ void __launch_bounds__(256) bwd_intra2_kernel(BwdArgs a) {
         sfw[r] = expf(sg[CB - 1] - sg[r]);
         sdG[r] = 0.f;
     }
-    build_write_rows(sA, LD, slam, sbeta, CB, s.sl, [](int) { return 1.f; });
+    build_write_rows(sA, LDM, slam, sbeta, CB, s.sl, [](int) { return 1.f; });
     __syncthreads();
 
     // dK = P3^T (s Q) + diag(fw) A D^K,  P3 = (dO' A^T) o Gamma
-    masked_scores(sP, sg, MS, 1.f, [&](int r, int kk) { return sY1[r * LD + kk]; },
-                  [&](int kk, int t) { return sA[t * LD + kk]; });
+    masked_scores<MSZ>(sP, sg, MSZ, 1.f, [&](int r, int kk) { return sY1[r * LDM + kk]; },
+                       [&](int kk, int t) { return sA[t * LDM + kk]; });
     {
         float acc[TMB][TN];
         zero_acc(acc);
-        rows_times_state<TN>(acc, sS, sA, Dst, 0, D);
+        rows_times_state<MSZ, TN>(acc, sS, sA, Dst, 0, D);
 #pragma unroll
         for (int i = 0; i < TMB; ++i)
 #pragma unroll
             for (int j = 0; j < TN; ++j) acc[i][j] *= sfw[ty + 16 * i];
-        scores_times_tok<TN>(acc, sS, [&](int t, int r) { return sP[r * LPB + t]; }, Q, s, b, h,
-                             t0, s.scale);
+        scores_times_tok<MSZ, TN>(acc, sS, [&](int t, int r) { return sP[r * LPB + t]; }, Q, s,
+                                  b, h, t0, s.scale);
         TI* dK = (TI*)a.dk;
 #pragma unroll
         for (int i = 0; i < TMB; ++i) {
@@ -516,18 +557,18 @@ __global__ void __launch_bounds__(256) bwd_intra2_kernel(BwdArgs a) {
     }
     // dV = P2^T dO + diag(fw) A D^V,  P2 = (O'' A^T) o Gamma
     __syncthreads();
-    masked_scores(sP, sg, MS, 1.f, [&](int r, int kk) { return sY2[r * LD + kk]; },
-                  [&](int kk, int t) { return sA[t * LD + kk]; });
+    masked_scores<MSZ>(sP, sg, MSZ, 1.f, [&](int r, int kk) { return sY2[r * LDM + kk]; },
+                       [&](int kk, int t) { return sA[t * LDM + kk]; });
     {
         float acc[TMB][TN];
         zero_acc(acc);
-        rows_times_state<TN>(acc, sS, sA, Dst, D, D);
+        rows_times_state<MSZ, TN>(acc, sS, sA, Dst, D, D);
 #pragma unroll
         for (int i = 0; i < TMB; ++i)
 #pragma unroll
             for (int j = 0; j < TN; ++j) acc[i][j] *= sfw[ty + 16 * i];
-        scores_times_tok<TN>(acc, sS, [&](int t, int r) { return sP[r * LPB + t]; }, dO, s, b, h,
-                             t0, 1.f);
+        scores_times_tok<MSZ, TN>(acc, sS, [&](int t, int r) { return sP[r * LPB + t]; }, dO, s,
+                                  b, h, t0, 1.f);
         TI* dV = (TI*)a.dv;
 #pragma unroll
         for (int i = 0; i < TMB; ++i)
@@ -536,59 +577,59 @@ __global__ void __launch_bounds__(256) bwd_intra2_kernel(BwdArgs a) {
                 stf(dV, (tokbase + (size_t)(ty + 16 * i) * s.H) * D + tx + 16 * j, acc[i][j]);
     }
     // dA^V = P4^T O'' + diag(fw) V (D^V)^T,  P4 = (dO V^T) o Gamma
-    masked_scores_tok(sP, sS, sg, dO, V, s, b, h, t0, 1.f);
+    masked_scores_tok<MSZ>(sP, sS, sg, dO, V, s, b, h, t0, 1.f);
     {
-        float acc[TMB][8];
+        float acc[TMB][NJ];
         zero_acc(acc);
-        tok_times_stateT(acc, sS, V, Dst, D, s, b, h, t0);
+        tok_times_stateT<MSZ>(acc, sS, V, Dst, D, s, b, h, t0);
 #pragma unroll
         for (int i = 0; i < TMB; ++i)
 #pragma unroll
-            for (int j = 0; j < 8; ++j) acc[i][j] *= sfw[ty + 16 * i];
-        simt_mm<TMB, 8>(acc, CB, [&](int t, int r) { return sP[r * LPB + t]; },
-                        [&](int r, int i) { return sY2[r * LD + i]; });
+            for (int j = 0; j < NJ; ++j) acc[i][j] *= sfw[ty + 16 * i];
+        simt_mm<TMB, NJ>(acc, CB, [&](int t, int r) { return sP[r * LPB + t]; },
+                         [&](int r, int i) { return sY2[r * LDM + i]; });
 #pragma unroll
         for (int i = 0; i < TMB; ++i) {
             const int t = ty + 16 * i;
             float part = 0.f;
 #pragma unroll
-            for (int j = 0; j < 8; ++j) {
-                sDA[t * LD + tx + 16 * j] = acc[i][j];
-                part += sA[t * LD + tx + 16 * j] * acc[i][j];
+            for (int j = 0; j < NJ; ++j) {
+                sDA[t * LDM + tx + 16 * j] = acc[i][j];
+                part += sA[t * LDM + tx + 16 * j] * acc[i][j];
             }
             part = half_warp_sum(part);
             if (tx == 0) sdG[t] -= part;
         }
     }
     // dA^K = P1^T dO' + diag(fw) K (D^K)^T,  P1 = (s Q K^T) o Gamma
-    masked_scores_tok(sP, sS, sg, Q, K, s, b, h, t0, s.scale);
+    masked_scores_tok<MSZ>(sP, sS, sg, Q, K, s, b, h, t0, s.scale);
     {
-        float acc[TMB][8];
+        float acc[TMB][NJ];
         zero_acc(acc);
-        tok_times_stateT(acc, sS, K, Dst, 0, s, b, h, t0);
+        tok_times_stateT<MSZ>(acc, sS, K, Dst, 0, s, b, h, t0);
 #pragma unroll
         for (int i = 0; i < TMB; ++i)
 #pragma unroll
-            for (int j = 0; j < 8; ++j) acc[i][j] *= sfw[ty + 16 * i];
-        simt_mm<TMB, 8>(acc, CB, [&](int t, int r) { return sP[r * LPB + t]; },
-                        [&](int r, int i) { return sY1[r * LD + i]; });
+            for (int j = 0; j < NJ; ++j) acc[i][j] *= sfw[ty + 16 * i];
+        simt_mm<TMB, NJ>(acc, CB, [&](int t, int r) { return sP[r * LPB + t]; },
+                         [&](int r, int i) { return sY1[r * LDM + i]; });
 #pragma unroll
         for (int i = 0; i < TMB; ++i)
 #pragma unroll
-            for (int j = 0; j < 8; ++j) sDA[(ty + 16 * i) * LD + tx + 16 * j] += acc[i][j];
+            for (int j = 0; j < NJ; ++j) sDA[(ty + 16 * i) * LDM + tx + 16 * j] += acc[i][j];
     }
     __syncthreads();
     // per token: d beta, d lambda from the write vector, dG
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const size_t BTH = (size_t)s.B * s.T * s.H;
     for (int t = warp; t < CB; t += 8) {
-        const float* da = sDA + t * LD;
-        const float* av = sA + t * LD;
+        const float* da = sDA + t * LDM;
+        const float* av = sA + t * LDM;
         float db = 0.f;
 #pragma unroll
-        for (int u = 0; u < 4; ++u) db += da[lane + 32 * u] * av[lane + 32 * u];
+        for (int u = 0; u < G::NE; ++u) db += da[lane + 32 * u] * av[lane + 32 * u];
         db = warp_sum(db);
-        const float om = warp_omega_dot(da, av, lane, s.sl); // <da, Omega a>
+        const float om = warp_omega_dot<MSZ>(da, av, lane, s.sl); // <da, Omega a>
         if (lane == 0) {
             const size_t gi = tokbase + (size_t)t * s.H;
             a.tok[2 * BTH + gi] = sdG[t];
@@ -734,24 +775,56 @@ __global__ void dA_final_kernel(BwdArgs a, int nseg) {
 }
 
 // dM[h][i][j] = sum over the batch and the tokens of dl[i] z[j] + p[i] dy[j] (paper order), one
-// block per (h, i), one thread per j.
-__global__ void __launch_bounds__(128) dm_reduce_simt(BwdArgs a) {
+// block per (h, i), one thread per j (ms threads).
+__global__ void __launch_bounds__(MS_MAX) dm_reduce_simt(BwdArgs a) {
     const Shape s = a.s;
+    const int ms = s.sl.ms;
     const int h = blockIdx.x, i = blockIdx.y, j = threadIdx.x;
     float acc = 0.f;
     for (int b = 0; b < s.B; ++b) {
-        const size_t base = ((size_t)b * s.H + h) * s.T * MS;
+        const size_t base = ((size_t)b * s.H + h) * s.T * ms;
         for (int t = 0; t < s.T; ++t) {
-            const size_t o = base + (size_t)t * MS;
+            const size_t o = base + (size_t)t * ms;
             acc = fmaf(a.mDL[o + i], a.mZ[o + j], acc);
             acc = fmaf(a.mP[o + i], a.mDY[o + j], acc);
         }
     }
-    a.dM[((size_t)h * MS + i) * MS + j] = acc;
+    a.dM[((size_t)h * ms + i) * ms + j] = acc;
 }
 
-template <int D, typename TI>
+// dR[h][i][k] = sum_j dM[h][i][j] Phi[k][j] for the m active slots i, k (App. A.1
+// Eq. app-real-fourier: Phi[k][0] = 1/sqrt(m), Phi[k][2j-1] = sqrt(2/m) cos(2 pi j k / m),
+// Phi[k][2j] = sqrt(2/m) sin(2 pi j k / m)); dM [H][ms][ms] in the paper's order.  Block (h, i)
+// of ms threads.
+__global__ void __launch_bounds__(MS_MAX) dr_finalize_simt(const float* dM, float* dR, Slots sl) {
+    const int h = blockIdx.x, i = blockIdx.y, t = threadIdx.x;
+    const int m = sl.m, ms = sl.ms;
+    __shared__ float s_dm[MS_MAX], s_ct[MS_MAX], s_st[MS_MAX];
+    s_dm[t] = dM[((size_t)h * ms + i) * ms + t];
+    if (t < m) {
+        float sv, cv;
+        sincospif((float)t * sl.two_over_m, &sv, &cv);
+        s_ct[t] = cv;
+        s_st[t] = sv;
+    }
+    __syncthreads();
+    if (t < m) {
+        float ac = 0.f, as = 0.f;
+        int idx = 0;   // (j t) mod m
+        for (int j = 1; j <= sl.npair; ++j) {
+            idx += t;
+            if (idx >= m) idx -= m;
+            ac = fmaf(s_dm[2 * j - 1], s_ct[idx], ac);
+            as = fmaf(s_dm[2 * j], s_st[idx], as);
+        }
+        dR[((size_t)h * m + i) * m + t] = s_dm[0] * sl.inv_sqrt_m + sl.sqrt2_over_m * (ac + as);
+    }
+}
+
+template <int D, int MSZ, typename TI>
 cudaError_t bwd_dispatch(const BwdArgs& a, cudaStream_t st) {
+    using G = Geo<MSZ>;
+    constexpr int CB = G::CB, LDM = G::LDM;
     const Shape& s = a.s;
     FwdArgs f{};
     f.s = s;
@@ -765,24 +838,36 @@ cudaError_t bwd_dispatch(const BwdArgs& a, cudaStream_t st) {
     cudaError_t e = launch_state_simt(f, st);
     if (e != cudaSuccess) return e;
     const dim3 gchunk(s.nchunk(), s.B * s.H);
-    const size_t sm1 = (size_t)(5 * CB * LD + CB * LPB + 6 * CB + 8 * 640) * sizeof(float);
-    auto k1 = bwd_intra1_kernel<D, TI>;
+    constexpr int SSZ = staging_floats<D, MSZ>();
+    const size_t sm1 =
+        (size_t)(4 * CB * LDM + SSZ + CB * G::LPB + 6 * CB + 8 * 5 * MSZ) * sizeof(float);
+    auto k1 = bwd_intra1_kernel<D, MSZ, TI>;
     cudaFuncSetAttribute(k1, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm1);
     { LaunchScope ls_("bwd_intra1", st); k1<<<gchunk, 256, sm1, st>>>(a); }
-    const size_t sma = (size_t)(CB * LD + CB * 33 + CB) * sizeof(float);
-    auto ka = adj_state_kernel<TI>;
+    const size_t sma = (size_t)(CB * LDM + CB * 33 + CB) * sizeof(float);
+    auto ka = adj_state_kernel<MSZ, TI>;
     cudaFuncSetAttribute(ka, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sma);
-    { LaunchScope ls_("bwd_adjoint", st); ka<<<dim3(2 * D / 32, s.B * s.H), 256, sma, st>>>(a); }
-    const size_t sm2 = (size_t)(5 * CB * LD + CB * LPB + 5 * CB) * sizeof(float);
-    auto k2 = bwd_intra2_kernel<D, TI>;
+    { LaunchScope ls_("bwd_adjoint", st); ka<<<dim3(2 * D / 32, s.B * s.H, MSZ / 128), 256, sma, st>>>(a); }
+    const size_t sm2 = (size_t)(4 * CB * LDM + SSZ + CB * G::LPB + 5 * CB) * sizeof(float);
+    auto k2 = bwd_intra2_kernel<D, MSZ, TI>;
     cudaFuncSetAttribute(k2, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm2);
     { LaunchScope ls_("bwd_intra2", st); k2<<<gchunk, 256, sm2, st>>>(a); }
     if (a.dR) {
-        { LaunchScope ls_("bwd_dm_reduce", st); dm_reduce_simt<<<dim3(s.H, MS), 128, 0, st>>>(a); }
-        e = launch_dr_finalize(a.dM, 1, s.H, false, a.dR, s.sl, st);
+        { LaunchScope ls_("bwd_dm_reduce", st); dm_reduce_simt<<<dim3(s.H, MSZ), MSZ, 0, st>>>(a); }
+        { LaunchScope ls_("bwd_dr_finalize", st); dr_finalize_simt<<<dim3(s.H, s.sl.m), MSZ, 0, st>>>(a.dM, a.dR, s.sl); }
+        e = cudaGetLastError();
         if (e != cudaSuccess) return e;
     }
     return launch_bwd_gates(a, st);
+}
+
+template <int MSZ>
+cudaError_t bwd_dispatch_d(const BwdArgs& a, cudaStream_t st) {
+    const Shape& s = a.s;
+    if (s.D == 128) return s.bf16 ? bwd_dispatch<128, MSZ, __nv_bfloat16>(a, st) : bwd_dispatch<128, MSZ, float>(a, st);
+    if (s.D == 64) return s.bf16 ? bwd_dispatch<64, MSZ, __nv_bfloat16>(a, st) : bwd_dispatch<64, MSZ, float>(a, st);
+    if (s.D == 256) return s.bf16 ? bwd_dispatch<256, MSZ, __nv_bfloat16>(a, st) : bwd_dispatch<256, MSZ, float>(a, st);
+    return cudaErrorInvalidValue;
 }
 
 }  // namespace
@@ -798,10 +883,9 @@ cudaError_t launch_bwd_gates(const BwdArgs& a, cudaStream_t st) {
 
 cudaError_t launch_bwd_simt(const BwdArgs& a, cudaStream_t st) {
     const Shape& s = a.s;
-    if (s.C != CB) return cudaErrorInvalidValue;
-    if (s.D == 128) return s.bf16 ? bwd_dispatch<128, __nv_bfloat16>(a, st) : bwd_dispatch<128, float>(a, st);
-    if (s.D == 64) return s.bf16 ? bwd_dispatch<64, __nv_bfloat16>(a, st) : bwd_dispatch<64, float>(a, st);
-    if (s.D == 256) return s.bf16 ? bwd_dispatch<256, __nv_bfloat16>(a, st) : bwd_dispatch<256, float>(a, st);
+    if (s.C != bwd_chunk(s.sl)) return cudaErrorInvalidValue;
+    if (s.sl.ms == 128) return bwd_dispatch_d<128>(a, st);
+    if (s.sl.ms == 256) return bwd_dispatch_d<256>(a, st);
     return cudaErrorInvalidValue;
 }
 

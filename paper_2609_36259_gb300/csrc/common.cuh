@@ -53,18 +53,21 @@ __device__ __forceinline__ float phase_pi_m(float lam, int j, const SL& sl) {
 // Temporal write-vector entries for one token: a = beta * U(-lam) b (Sec. 3.2), with
 // b = [1/sqrt(m), sqrt(2/m), 0, sqrt(2/m), 0, ...] (App. A.1 Eq. app-b-explicit), so
 // a[0] = beta/sqrt(m), a[2j-1] = beta sqrt(2/m) cos(theta_j), a[2j] = -beta sqrt(2/m) sin(theta_j)
-// for j <= (m-1)/2, and the padding entries a[m..127] = 0 (App. A.7).
-// Fills rows r < C of a row-major [C][ld] shared array; row r is scaled by sc[r] * beta[r].
+// for j <= (m-1)/2, and the padding entries a[m..ms-1] = 0 (App. A.7).
+// Fills the ms entries of rows r < C of a row-major [C][ld] shared array; row r is scaled by
+// sc[r] * beta[r].
 template <class ScaleFn>
 __device__ __forceinline__ void build_write_rows(float* sA, int ld, const float* slam,
                                                  const float* sbeta, int C, const Slots& sl,
                                                  ScaleFn scale_of) {
-    for (int e = threadIdx.x; e < C * 64; e += blockDim.x) {
-        const int r = e >> 6, j = e & 63;
+    const int lg = sl.ms == 256 ? 7 : 6;   // log2 of the entry pairs per row (ms / 2)
+    const int hp = 1 << lg;
+    for (int e = threadIdx.x; e < C * hp; e += blockDim.x) {
+        const int r = e >> lg, j = e & (hp - 1);
         const float sc = sbeta[r] * scale_of(r);
         if (j == 0) {
             sA[r * ld] = sc * sl.inv_sqrt_m;
-            sA[r * ld + 127] = 0.f;
+            sA[r * ld + 2 * hp - 1] = 0.f;
         } else if (j <= sl.npair) {
             float s, c;
             sincospif(phase_pi_m(slam[r], j, sl), &s, &c);

@@ -37,10 +37,8 @@ int cyfa::check_dims(const cyfa_dims_t* d, bool need_T) {
     if (d->B <= 0 || d->H <= 0 || d->dk <= 0 || d->dv <= 0 || (need_T && d->T <= 0))
         return CYFA_ERR_ARG;
     if (d->dtype != CYFA_DTYPE_BF16 && d->dtype != CYFA_DTYPE_FP32) return CYFA_ERR_ARG;
-    // m: odd, 1..127 (128 storage rows); the paper's m = 255 needs 256 rows, which this build
-    // does not implement
-    if (d->m == 255) return CYFA_ERR_UNSUPPORTED;
-    if (d->m < 1 || d->m > 127 || d->m % 2 == 0) return CYFA_ERR_SHAPE;
+    // m: odd, 1..255 (128 storage rows up to 127, 256 above)
+    if (d->m < 1 || d->m > 255 || d->m % 2 == 0) return CYFA_ERR_SHAPE;
     if (d->dk != d->dv || (d->dk != 64 && d->dk != 128 && d->dk != 256)) return CYFA_ERR_SHAPE;
     if ((long long)d->B * d->H > kMaxSequences) return CYFA_ERR_SHAPE;
     if (need_T) {
@@ -66,15 +64,16 @@ Shape shape_of(const cyfa_dims_t* d) {
     return s;
 }
 
+// The tensor-core kernels hold 128 storage rows.
 bool use_tc(const cyfa_dims_t* d, const Shape& s) {
-    return !(d->flags & CYFA_FLAG_CUDA_CORES) && tc_fwd_supported(s);
+    return !(d->flags & CYFA_FLAG_CUDA_CORES) && s.sl.ms == 128 && tc_fwd_supported(s);
 }
 
-// The CUDA-core forward walks the caller's chunk, except at d = 256, where it walks 64-token
-// chunks (its register tiles of a 128-token chunk would not fit); g_cum stays local to the
-// caller's chunk (Cg) and the kernels rebase it.
+// The CUDA-core forward walks the caller's chunk, except at d = 256 or with 256 storage rows,
+// where it walks 64-token chunks (its register and shared tiles of a 128-token chunk would not
+// fit); g_cum stays local to the caller's chunk (Cg) and the kernels rebase it.
 Shape simt_fwd_shape(Shape s) {
-    if (s.D == 256) s.C = 64;
+    if (s.D == 256 || s.sl.ms == 256) s.C = 64;
     return s;
 }
 
@@ -87,17 +86,18 @@ struct FwdLayout {
 };
 FwdLayout fwd_layout(const Shape& s0, bool tc_path, void* ws) {
     const Shape s = tc_path ? s0 : simt_fwd_shape(s0);
+    const size_t ms = s.sl.ms;
     Carver c{static_cast<char*>(ws)};
     FwdLayout L{};
-    L.M = c.take<float>((size_t)s.H * MS * MS);
-    L.MT = c.take<float>((size_t)s.H * MS * MS);
+    L.M = c.take<float>((size_t)s.H * ms * ms);
+    L.MT = c.take<float>((size_t)s.H * ms * ms);
     if (tc_path) {
         L.nseg = tc_fwd_segments(s);
         L.Mb = c.take<__half>((size_t)s.H * MS * MS);
         L.segS = c.take<float>((size_t)s.B * s.H * L.nseg * MS * 256);
         L.segG = c.take<float>((size_t)s.B * s.H * L.nseg);
     } else {
-        L.states = c.take<float>((size_t)s.B * s.H * s.nchunk() * MS * 2 * s.D);
+        L.states = c.take<float>((size_t)s.B * s.H * s.nchunk() * ms * 2 * s.D);
     }
     L.bytes = c.off;
     return L;
@@ -118,13 +118,14 @@ struct BwdLayout {
 };
 BwdLayout bwd_layout(const Shape& s0, bool tc_path, void* ws) {
     Shape s = s0;
-    s.C = BWD_C;
+    s.C = bwd_chunk(s.sl);
+    const size_t ms = s.sl.ms;
     Carver c{static_cast<char*>(ws)};
     BwdLayout L{};
     const size_t BH = (size_t)s.B * s.H;
     const size_t nseg = (s.T + PREP_SEG - 1) / PREP_SEG;
-    L.M = c.take<float>((size_t)s.H * MS * MS);
-    L.MT = c.take<float>((size_t)s.H * MS * MS);
+    L.M = c.take<float>((size_t)s.H * ms * ms);
+    L.MT = c.take<float>((size_t)s.H * ms * ms);
     L.tok = c.take<float>((tc_path ? 7 : 5) * BH * s.T);
     L.seg = c.take<double>(2 * BH * nseg);
     L.dA_part = c.take<double>(BH * nseg);
@@ -149,15 +150,15 @@ BwdLayout bwd_layout(const Shape& s0, bool tc_path, void* ws) {
         L.dm_split = (int)(nch < 32 ? nch : 32);
         L.dMp = c.take<float>((size_t)s.H * L.dm_split * MS * MS);
     } else {
-        L.states = c.take<float>(BH * s.nchunk() * MS * 2 * s.D);
-        L.adj = c.take<float>(BH * s.nchunk() * MS * 2 * s.D);
-        L.o2 = c.take<float>(BH * s.T * MS);
-        L.do1 = c.take<float>(BH * s.T * MS);
-        L.fZ = c.take<float>(BH * s.T * MS);
-        L.fP = c.take<float>(BH * s.T * MS);
-        L.fDY = c.take<float>(BH * s.T * MS);
-        L.fDL = c.take<float>(BH * s.T * MS);
-        L.fdM = c.take<float>((size_t)s.H * MS * MS);
+        L.states = c.take<float>(BH * s.nchunk() * ms * 2 * s.D);
+        L.adj = c.take<float>(BH * s.nchunk() * ms * 2 * s.D);
+        L.o2 = c.take<float>(BH * s.T * ms);
+        L.do1 = c.take<float>(BH * s.T * ms);
+        L.fZ = c.take<float>(BH * s.T * ms);
+        L.fP = c.take<float>(BH * s.T * ms);
+        L.fDY = c.take<float>(BH * s.T * ms);
+        L.fDL = c.take<float>(BH * s.T * ms);
+        L.fdM = c.take<float>((size_t)s.H * ms * ms);
     }
     L.bytes = c.off;
     return L;
@@ -175,7 +176,7 @@ const char* cyfa_error_string(int code) {
     switch (code) {
         case CYFA_OK: return "ok";
         case CYFA_ERR_ARG: return "invalid argument (null pointer or non-positive size)";
-        case CYFA_ERR_SHAPE: return "unsupported shape (m odd in 1..127, dk == dv in {64,128,256}, chunk in {64,128}, T % chunk == 0, B*H <= 65535)";
+        case CYFA_ERR_SHAPE: return "unsupported shape (m odd in 1..255, dk == dv in {64,128,256}, chunk in {64,128}, T % chunk == 0, B*H <= 65535)";
         case CYFA_ERR_ALIGN: return "tensor pointer not 16-byte aligned";
         case CYFA_ERR_WORKSPACE: return "workspace missing or too small";
         case CYFA_ERR_CUDA: return "CUDA runtime error";
@@ -379,7 +380,7 @@ int cyfa_chunk_bwd(const cyfa_dims_t* dims, const void* q, const void* k, const 
     if (rc) return rc;
     BwdArgs a;
     a.s = s;
-    a.s.C = BWD_C;
+    a.s.C = bwd_chunk(s.sl);
     a.q = q;
     a.k = k;
     a.v = v;

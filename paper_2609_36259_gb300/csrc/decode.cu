@@ -6,9 +6,9 @@
 // block per SM walks a contiguous, head-major range of (b, h) rows; the key stream of one row,
 // the middle readout of the previous row and the value stream of the row before run at once, so
 // the HBM streams are never idle during the readout arithmetic; the state rows arrive through a
-// two-stage cp.async ring per streaming warp.  d = 64 keeps the simpler step_kernel (G batch rows
-// of one head per 256-thread block).  The middle readout applies Phi through a 127-entry cosine /
-// sine table (entry (j r) mod m of Eq. app-real-fourier) and R.
+// two-stage cp.async ring per streaming warp.  Other d and m run the simpler step_kernel (G batch rows
+// of one head per 256-thread block).  The middle readout applies Phi through an m-entry cosine /
+// sine table (entry (j r) mod m of Eq. app-real-fourier) and R; m > 127 keeps 256 storage rows.
 #include "common.cuh"
 #include "kernels.h"
 
@@ -44,21 +44,28 @@ __device__ __forceinline__ void store_row(float* p, const float (&x)[VPL]) {
     }
 }
 
-template <int D, typename TI>
+// Generic step for MSZ storage rows (128 for m <= 127, 256 above); G batch rows of one head per
+// 256-thread block.
+template <int D, int MSZ, typename TI>
 __global__ void __launch_bounds__(256) step_kernel(StepArgs a) {
     constexpr int VPL = D / 32;   // floats per lane per state row
+    constexpr int HP = MSZ / 2;   // entry pairs of a slot vector (the DC / padding pair is j = 0)
     const int h = blockIdx.y, b0 = blockIdx.x * G;
     const int ng = min(G, a.B - b0);
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const Slots sl = a.sl;
     const int m = sl.m;
-    __shared__ float s_ct[MA], s_st[MA];
-    __shared__ float s_q[G][D], s_k[G][D], s_v[G][D];
-    __shared__ float s_a[G][MS], s_o1[G][MS], s_z[G][MS], s_u[G][MS], s_l[G][MS], s_y[G][MS];
-    __shared__ float s_cs[G][64], s_sn[G][64];
+    __shared__ float s_ct[MSZ - 1], s_st[MSZ - 1];
+    // q and k, then (after the key pass has taken them into registers) the two halves of o
+    __shared__ float s_qk[2][G][D];
+    __shared__ float s_v[G][D];
+    __shared__ float s_a[G][MSZ], s_o1[G][MSZ], s_z[G][MSZ], s_u[G][MSZ], s_l[G][MSZ], s_y[G][MSZ];
+    __shared__ float s_cs[G][HP], s_sn[G][HP];
     __shared__ float s_alpha[G], s_inv[G];
     __shared__ double s_lam[G];
-    __shared__ float s_opart[2][G][D];
+    float (*s_q)[D] = s_qk[0];
+    float (*s_k)[D] = s_qk[1];
+    float (*s_opart)[G][D] = s_qk;
 
     const TI* Q = (const TI*)a.q;
     const TI* K = (const TI*)a.k;
@@ -78,9 +85,9 @@ __global__ void __launch_bounds__(256) step_kernel(StepArgs a) {
             s_v[g][i] = ldf(V, bh * D + i);
         }
     }
-    // clock, gates and rotation angles: thread (g, j) with j = 0 for the DC entry
-    {
-        const int g = tid >> 6, j = tid & 63;
+    // clock, gates and rotation angles: (g, j) with j = 0 for the DC entry
+    for (int e = tid; e < G * HP; e += 256) {
+        const int g = e / HP, j = e % HP;
         if (g < ng) {
             const size_t bh = (size_t)(b0 + g) * a.H + h;
             const double lam_new = a.lambda[bh] + (double)sigmoidf_(a.clock_logit[bh]);
@@ -90,7 +97,7 @@ __global__ void __launch_bounds__(256) step_kernel(StepArgs a) {
                 s_alpha[g] = expf(-a.A[h] * softplusf_(a.decay_logit[bh]));
                 s_lam[g] = lam_new;
                 s_a[g][0] = beta * sl.inv_sqrt_m;
-                s_a[g][127] = 0.f;
+                s_a[g][MSZ - 1] = 0.f;
                 s_cs[g][0] = 1.f;
                 s_sn[g][0] = 0.f;
             } else if (j <= sl.npair) {
@@ -115,7 +122,7 @@ __global__ void __launch_bounds__(256) step_kernel(StepArgs a) {
     const int wg = warp >> 1, half = warp & 1;
     if (wg < ng) {
         const int g = wg;
-        float* Kb = a.Kbar + ((size_t)(b0 + g) * a.H + h) * MS * D;
+        float* Kb = a.Kbar + ((size_t)(b0 + g) * a.H + h) * MSZ * D;
         const float alpha = s_alpha[g];
         float qv[VPL], kv[VPL];
 #pragma unroll
@@ -123,7 +130,7 @@ __global__ void __launch_bounds__(256) step_kernel(StepArgs a) {
             qv[u] = s_q[g][lane * VPL + u];
             kv[u] = s_k[g][lane * VPL + u];
         }
-        for (int i0 = 0; i0 < MS / 2; i0 += BATCH) {
+        for (int i0 = 0; i0 < MSZ / 2; i0 += BATCH) {
             float x[BATCH][VPL];
 #pragma unroll
             for (int bb = 0; bb < BATCH; ++bb) {
@@ -150,12 +157,12 @@ __global__ void __launch_bounds__(256) step_kernel(StepArgs a) {
 
     // middle readout (Sec. 3.3 Eq. cyfa-two-pass, middle line) for the G rows:
     // z = U(lam) o'; u = Phi z; l = R u; p = softmax(l); y' = R^T p; y = Phi^T y'; o'' = U(-lam) y
-    {
-        const int g = tid >> 6, j = tid & 63;
+    for (int e = tid; e < G * HP; e += 256) {
+        const int g = e / HP, j = e % HP;
         if (g < ng) {
             if (j == 0) {
                 s_z[g][0] = s_o1[g][0];
-                s_z[g][127] = 0.f;
+                s_z[g][MSZ - 1] = 0.f;
             } else {   // padding pairs have c = 1, sn = 0 and zero entries
                 const float c = s_cs[g][j], sn = s_sn[g][j];
                 const float xc = s_o1[g][2 * j - 1], xs = s_o1[g][2 * j];
@@ -165,8 +172,8 @@ __global__ void __launch_bounds__(256) step_kernel(StepArgs a) {
         }
     }
     __syncthreads();
-    for (int e = tid; e < G * MS; e += 256) {   // u_r = z_0/sqrt(m) + sqrt(2/m) sum_j (...)
-        const int g = e >> 7, r = e & 127;
+    for (int e = tid; e < G * MSZ; e += 256) {   // u_r = z_0/sqrt(m) + sqrt(2/m) sum_j (...)
+        const int g = e / MSZ, r = e % MSZ;
         if (g < ng && r < m) {
             float acc = 0.f;
             int idx = 0;
@@ -182,16 +189,17 @@ __global__ void __launch_bounds__(256) step_kernel(StepArgs a) {
     __syncthreads();
     const float* Rh = a.R + (size_t)h * m * m;
     for (int i = warp; i < m; i += 8) {   // l_i = sum_r R[i][r] u_r, one R row per warp
-        float rv[4];
+        constexpr int NE = MSZ / 32;
+        float rv[NE];
 #pragma unroll
-        for (int k = 0; k < 4; ++k) {
+        for (int k = 0; k < NE; ++k) {
             const int r = lane + 32 * k;
             rv[k] = r < m ? Rh[i * m + r] : 0.f;
         }
         for (int g = 0; g < ng; ++g) {
             float acc = 0.f;
 #pragma unroll
-            for (int k = 0; k < 4; ++k) {
+            for (int k = 0; k < NE; ++k) {
                 const int r = lane + 32 * k;
                 if (r < m) acc = fmaf(rv[k], s_u[g][r], acc);
             }
@@ -215,29 +223,27 @@ __global__ void __launch_bounds__(256) step_kernel(StepArgs a) {
         if (lane == 0) s_inv[g] = 1.f / sum;
     }
     __syncthreads();
-    {   // y'_r = sum_i R[i][r] p_i, thread (r, half): rows g = half, half + 2
-        const int r = tid & 127, half = tid >> 7;
-        if (r < m) {
-            float acc0 = 0.f, acc1 = 0.f;
-            const int g0 = half, g1 = half + 2;
-            for (int i = 0; i < m; ++i) {
-                const float rv = Rh[i * m + r];
-                acc0 = fmaf(rv, s_l[g0][i], acc0);
-                acc1 = fmaf(rv, s_l[g1][i], acc1);
-            }
-            if (g0 < ng) s_u[g0][r] = acc0 * s_inv[g0];
-            if (g1 < ng) s_u[g1][r] = acc1 * s_inv[g1];
+    // y'_r = sum_i R[i][r] p_i, thread (r mod 128, half): rows g = half, half + 2
+    for (int r = tid & 127; r < m; r += 128) {
+        const int g0 = tid >> 7, g1 = g0 + 2;
+        float acc0 = 0.f, acc1 = 0.f;
+        for (int i = 0; i < m; ++i) {
+            const float rv = Rh[i * m + r];
+            acc0 = fmaf(rv, s_l[g0][i], acc0);
+            acc1 = fmaf(rv, s_l[g1][i], acc1);
         }
+        if (g0 < ng) s_u[g0][r] = acc0 * s_inv[g0];
+        if (g1 < ng) s_u[g1][r] = acc1 * s_inv[g1];
     }
     __syncthreads();
-    {   // y = Phi^T y', then o'' = U(-lam) y on the pair (2j-1, 2j)
-        const int g = tid >> 6, j = tid & 63;
+    for (int e = tid; e < G * HP; e += 256) {   // y = Phi^T y', then o'' = U(-lam) y on (2j-1, 2j)
+        const int g = e / HP, j = e % HP;
         if (g < ng) {
             if (j == 0) {
                 float ac = 0.f;
                 for (int r = 0; r < m; ++r) ac += s_u[g][r];
                 s_y[g][0] = ac * sl.inv_sqrt_m;
-                s_y[g][127] = 0.f;
+                s_y[g][MSZ - 1] = 0.f;
             } else if (j > sl.npair) {   // padding slots
                 s_y[g][2 * j - 1] = 0.f;
                 s_y[g][2 * j] = 0.f;
@@ -262,7 +268,7 @@ __global__ void __launch_bounds__(256) step_kernel(StepArgs a) {
     // Vbar <- alpha Vbar + a v^T ; o = Vbar^T o''
     if (wg < ng) {
         const int g = wg;
-        float* Vb = a.Vbar + ((size_t)(b0 + g) * a.H + h) * MS * D;
+        float* Vb = a.Vbar + ((size_t)(b0 + g) * a.H + h) * MSZ * D;
         const float alpha = s_alpha[g];
         float vv[VPL], oacc[VPL];
 #pragma unroll
@@ -270,7 +276,7 @@ __global__ void __launch_bounds__(256) step_kernel(StepArgs a) {
             vv[u] = s_v[g][lane * VPL + u];
             oacc[u] = 0.f;
         }
-        for (int i0 = 0; i0 < MS / 2; i0 += BATCH) {
+        for (int i0 = 0; i0 < MSZ / 2; i0 += BATCH) {
             float x[BATCH][VPL];
 #pragma unroll
             for (int bb = 0; bb < BATCH; ++bb) {
@@ -664,6 +670,22 @@ __global__ void __launch_bounds__(P_THREADS, 1) step_pipe_kernel(StepArgs a) {
     wait_prefetch_all();
 }
 
+template <int MSZ>
+cudaError_t launch_generic(const StepArgs& a, dim3 grid, cudaStream_t st) {
+    LaunchScope ls_("decode_step", st);
+#define CYFA_STEP(DD)                                                                   \
+    if (a.D == DD) {                                                                    \
+        if (a.bf16) step_kernel<DD, MSZ, __nv_bfloat16><<<grid, 256, 0, st>>>(a);       \
+        else step_kernel<DD, MSZ, float><<<grid, 256, 0, st>>>(a);                      \
+        return cudaGetLastError();                                                      \
+    }
+    CYFA_STEP(64)
+    CYFA_STEP(128)
+    CYFA_STEP(256)
+#undef CYFA_STEP
+    return cudaErrorInvalidValue;
+}
+
 }  // namespace
 
 cudaError_t launch_step(const StepArgs& a, cudaStream_t st) {
@@ -687,17 +709,10 @@ cudaError_t launch_step(const StepArgs& a, cudaStream_t st) {
             LaunchScope ls_("decode_step", st);
             k<<<blocks, P_THREADS, smem, st>>>(a);
         }
-    } else if (a.D == 64) {
-        if (a.bf16) { LaunchScope ls_("decode_step", st); step_kernel<64, __nv_bfloat16><<<grid, 256, 0, st>>>(a); }
-        else { LaunchScope ls_("decode_step", st); step_kernel<64, float><<<grid, 256, 0, st>>>(a); }
-    } else if (a.D == 128) {   // m != 127: the generic kernel
-        if (a.bf16) { LaunchScope ls_("decode_step", st); step_kernel<128, __nv_bfloat16><<<grid, 256, 0, st>>>(a); }
-        else { LaunchScope ls_("decode_step", st); step_kernel<128, float><<<grid, 256, 0, st>>>(a); }
-    } else if (a.D == 256) {
-        if (a.bf16) { LaunchScope ls_("decode_step", st); step_kernel<256, __nv_bfloat16><<<grid, 256, 0, st>>>(a); }
-        else { LaunchScope ls_("decode_step", st); step_kernel<256, float><<<grid, 256, 0, st>>>(a); }
-    } else {
-        return cudaErrorInvalidValue;
+    } else {   // the generic kernel
+        const cudaError_t e = a.sl.ms == 128 ? launch_generic<128>(a, grid, st)
+                                             : launch_generic<256>(a, grid, st);
+        if (e != cudaSuccess) return e;
     }
     return cudaGetLastError();
 }

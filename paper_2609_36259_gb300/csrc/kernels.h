@@ -30,19 +30,22 @@ class LaunchScope {
     cudaEvent_t start_ = nullptr;
 };
 
-// Slot geometry: m active relative-time slots (odd, 1 <= m <= 127) in 128 storage rows; the
-// real Fourier basis of App. A.1 Eq. app-real-fourier has the DC row and (m-1)/2 cosine-sine
-// pairs, b = [1/sqrt(m), sqrt(2/m), 0, sqrt(2/m), 0, ...] (Eq. app-b-explicit), and rows m..127
-// stay zero.  The constants are formed once on the host.
+// Slot geometry: m active relative-time slots (odd, 1 <= m <= 255) in ms storage rows (128 for
+// m <= 127, 256 above); the real Fourier basis of App. A.1 Eq. app-real-fourier has the DC row
+// and (m-1)/2 cosine-sine pairs, b = [1/sqrt(m), sqrt(2/m), 0, sqrt(2/m), 0, ...]
+// (Eq. app-b-explicit), and rows m..ms-1 stay zero.  The constants are formed once on the host.
 struct Slots {
-    int m, npair;
+    int m, npair, ms;
     float fm, inv_m, two_over_m, inv_sqrt_m, sqrt2_over_m;
     float omega1;           // 2 pi / m, the rotation rate of pair 1
 };
+constexpr int MS_MAX = 256;   // largest number of storage rows
+inline int storage_rows(int m) { return m <= 127 ? 128 : 256; }
 inline Slots make_slots(int m) {
     Slots s;
     s.m = m;
     s.npair = (m - 1) / 2;
+    s.ms = storage_rows(m);
     s.fm = (float)m;
     s.inv_m = 1.f / (float)m;
     s.two_over_m = 2.f / (float)m;
@@ -55,7 +58,7 @@ inline Slots make_slots(int m) {
 // The same geometry as compile-time constants for m = 127 (the paper's setting): kernels
 // templated on the slot type fold every constant; runtime Slots serve the other m.
 struct Slots127 {
-    static constexpr int m = 127, npair = 63;
+    static constexpr int m = 127, npair = 63, ms = 128;
     static constexpr float fm = 127.f, inv_m = 1.f / 127.f, two_over_m = 2.f / 127.f;
     static constexpr float inv_sqrt_m = 0.088735650941611f, sqrt2_over_m = 0.125491161809579f;
     static constexpr float omega1 = 6.283185307179586f / 127.f;
@@ -93,7 +96,7 @@ cudaError_t launch_prepare_fixed_rate(const PrepareArgs& a, double rho, cudaStre
 cudaError_t prep_read_error(cudaStream_t st, int* err);
 
 // ---- readout matrix M = R Phi and its transpose (chunk_simt.cu) ----
-// R [H, m, m]; M, MT [H, 128, 128] with the rows and columns m..127 zero.
+// R [H, m, m]; M, MT [H, ms, ms] with the rows and columns m..ms-1 zero.
 cudaError_t launch_readout_matrix(int H, const float* R, float* M, float* MT, const Slots& sl,
                                   cudaStream_t st);
 
@@ -105,7 +108,7 @@ struct FwdArgs {
     const float *Kbar0, *Vbar0;
     void* o;
     float *Kout, *Vout;
-    float* states;      // workspace [B*H][nchunk][128][2D]: chunk-start [Kbar | Vbar]
+    float* states;      // workspace [B*H][nchunk][ms][2D]: chunk-start [Kbar | Vbar]
 };
 cudaError_t launch_fwd_simt(const FwdArgs& a, cudaStream_t st);
 cudaError_t launch_state_simt(const FwdArgs& a, cudaStream_t st);  // state pass only
@@ -117,23 +120,26 @@ struct BwdArgs {
     const float *clock_logit, *decay_logit, *A;
     void *dq, *dk, *dv;
     float *d_clock, *d_decay, *d_beta, *dA;
-    float* states;      // [B*H][nchunk][128][2D] chunk-start states
-    float* adj;         // [B*H][nchunk][128][2D] adjoints of the chunk-end states
-    float* o2;          // [B*H][T][128] o'' per token
-    float* do1;         // [B*H][T][128] dL/do' per token
+    float* states;      // [B*H][nchunk][ms][2D] chunk-start states
+    float* adj;         // [B*H][nchunk][ms][2D] adjoints of the chunk-end states
+    float* o2;          // [B*H][T][ms] o'' per token
+    float* do1;         // [B*H][T][ms] dL/do' per token
     float* tok;         // [4][B*T*H]: dG part 1, d lambda part 1, dG part 2 / d lambda part 2 / d beta
     double* seg;        // [2][B*H][nseg] reverse-scan partials
     double* dA_part;    // [B*H*nseg]
-    // dR (nullable): per-token z, p, dy, dl of the middle readout (fp32 [B*H][T][128], paper
-    // order), the per-head dM and the output [H][127][127]
+    // dR (nullable): per-token z, p, dy, dl of the middle readout (fp32 [B*H][T][ms], paper
+    // order), the per-head dM [H][ms][ms] and the output [H][m][m]
     float *mZ, *mP, *mDY, *mDL;
     float *dM, *dR;
 };
 // dR[h] = dM[h] Phi^T over the m active slots from dm_split partial dM blocks [H][split][128][128]
-// whose Fourier (column) index is in the tensor-core order (tc_order) or in the paper's order.
+// whose Fourier (column) index is in the tensor-core order (tc_order) or in the paper's order
+// (m <= 127).
 cudaError_t launch_dr_finalize(const float* dMp, int dm_split, int H, bool tc_order, float* dR,
                                const Slots& sl, cudaStream_t st);
-constexpr int BWD_C = 64;       // chunk length used by the SIMT backward
+constexpr int BWD_C = 64;       // chunk length used by the SIMT backward with 128 storage rows
+constexpr int BWD_C256 = 32;    // ... and with 256 (the tiles of a 64-token chunk would not fit)
+inline int bwd_chunk(const Slots& sl) { return sl.ms == 128 ? BWD_C : BWD_C256; }
 cudaError_t launch_bwd_simt(const BwdArgs& a, cudaStream_t st);
 // reverse cumulative sums of the per-token scalars in a.tok and the logit gradients
 cudaError_t launch_bwd_gates(const BwdArgs& a, cudaStream_t st);

@@ -9,20 +9,23 @@ namespace cyfa {
 constexpr int LD = 129;   // padded row stride of [C][128] shared tiles
 
 // ---------------------------------------------------------------------------------------
-// Token-wise middle readout for rows r < C of sX (in place): o'' = U(-lam) M^T softmax(M U(lam) o')
-// with M = R Phi; the padding logits (slots m..127) are excluded from the softmax and o''[m..127]
-// stay 0.  One warp per row; swarp holds 2 x 128 floats of scratch per warp.
+// Token-wise middle readout for rows r < C of sX (row stride MSZ + 1, in place):
+// o'' = U(-lam) M^T softmax(M U(lam) o') with M = R Phi ([MSZ][MSZ]); the padding logits
+// (slots m..MSZ-1) are excluded from the softmax and o''[m..MSZ-1] are 0.  One warp per row; swarp
+// holds 2 x MSZ floats of scratch per warp.
+template <int MSZ>
 static __device__ __noinline__ void middle_rows(float* sX, const float* slam, int C, const float* M, const float* MT,
                             float* swarp, const Slots& sl) {
+    constexpr int LDM = MSZ + 1, NP = MSZ / 64, NE = MSZ / 32, NPAIRS = MSZ / 2 - 1;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    float* z = swarp + warp * 256;
-    float* p = z + 128;
+    float* z = swarp + warp * 2 * MSZ;
+    float* p = z + MSZ;
     for (int r = warp; r < C; r += 8) {
-        float* x = sX + r * LD;
+        float* x = sX + r * LDM;
         const float lam = slam[r];
-        float cs[2], sn[2];
+        float cs[NP], sn[NP];
 #pragma unroll
-        for (int u = 0; u < 2; ++u) {
+        for (int u = 0; u < NP; ++u) {
             const int j = lane + 1 + 32 * u;
             cs[u] = 1.f;
             sn[u] = 0.f;
@@ -31,60 +34,69 @@ static __device__ __noinline__ void middle_rows(float* sX, const float* slam, in
                 const float xc = x[2 * j - 1], xs = x[2 * j];
                 z[2 * j - 1] = cs[u] * xc - sn[u] * xs;
                 z[2 * j] = sn[u] * xc + cs[u] * xs;
-            } else if (j <= NPAIR) {   // padding slots (zero)
+            } else if (j <= NPAIRS) {   // padding slots (zero)
                 z[2 * j - 1] = 0.f;
                 z[2 * j] = 0.f;
             }
         }
         if (lane == 0) {
             z[0] = x[0];
-            z[127] = 0.f;
+            z[MSZ - 1] = 0.f;
         }
         __syncwarp();
-        float l[4] = {0.f, 0.f, 0.f, 0.f};
-        for (int k = 0; k < MS; ++k) {
+        float l[NE];
+#pragma unroll
+        for (int u = 0; u < NE; ++u) l[u] = 0.f;
+        for (int k = 0; k < MSZ; ++k) {
             const float zk = z[k];
 #pragma unroll
-            for (int u = 0; u < 4; ++u) l[u] = fmaf(MT[k * MS + lane + 32 * u], zk, l[u]);
+            for (int u = 0; u < NE; ++u) l[u] = fmaf(MT[k * MSZ + lane + 32 * u], zk, l[u]);
         }
+        float mx = -INFINITY;
 #pragma unroll
-        for (int u = 0; u < 4; ++u)
+        for (int u = 0; u < NE; ++u) {
             if (lane + 32 * u >= sl.m) l[u] = -INFINITY;
-        float mx = fmaxf(fmaxf(l[0], l[1]), fmaxf(l[2], l[3]));
+            mx = fmaxf(mx, l[u]);
+        }
         mx = warp_max(mx);
-        float e[4], sum = 0.f;
+        float e[NE], sum = 0.f;
 #pragma unroll
-        for (int u = 0; u < 4; ++u) {
+        for (int u = 0; u < NE; ++u) {
             e[u] = expf(l[u] - mx);
             sum += e[u];
         }
         sum = warp_sum(sum);
         const float inv = 1.f / sum;
 #pragma unroll
-        for (int u = 0; u < 4; ++u) p[lane + 32 * u] = e[u] * inv;
+        for (int u = 0; u < NE; ++u) p[lane + 32 * u] = e[u] * inv;
         __syncwarp();
-        float y[4] = {0.f, 0.f, 0.f, 0.f};
+        float y[NE];
+#pragma unroll
+        for (int u = 0; u < NE; ++u) y[u] = 0.f;
         for (int i = 0; i < sl.m; ++i) {
             const float pi = p[i];
 #pragma unroll
-            for (int u = 0; u < 4; ++u) y[u] = fmaf(M[i * MS + lane + 32 * u], pi, y[u]);
+            for (int u = 0; u < NE; ++u) y[u] = fmaf(M[i * MSZ + lane + 32 * u], pi, y[u]);
         }
         __syncwarp();
 #pragma unroll
-        for (int u = 0; u < 4; ++u) z[lane + 32 * u] = y[u];
+        for (int u = 0; u < NE; ++u) z[lane + 32 * u] = y[u];
         __syncwarp();
 #pragma unroll
-        for (int u = 0; u < 2; ++u) {
+        for (int u = 0; u < NP; ++u) {
             const int j = lane + 1 + 32 * u;
             if (j <= sl.npair) {
                 const float yc = z[2 * j - 1], ys = z[2 * j];
                 x[2 * j - 1] = cs[u] * yc + sn[u] * ys;
                 x[2 * j] = -sn[u] * yc + cs[u] * ys;
+            } else if (j <= NPAIRS) {
+                x[2 * j - 1] = 0.f;
+                x[2 * j] = 0.f;
             }
         }
         if (lane == 0) {
             x[0] = z[0];
-            x[127] = 0.f;
+            x[MSZ - 1] = 0.f;
         }
         __syncwarp();
     }

@@ -43,6 +43,11 @@ class Dims(ctypes.Structure):
 CYFA_FLAG_CUDA_CORES = 1
 
 
+def storage_rows(m):
+    """Rows of a state for m active slots: 128 for m <= 127, 256 above (rows m.. stay zero)."""
+    return 128 if m <= 127 else 256
+
+
 def dims(B, T, H, d, *, chunk=64, scale=None, dtype=torch.bfloat16, m=127, cuda_cores=False):
     return Dims(B, T, H, d, d, m, chunk, float(d ** -0.5 if scale is None else scale),
                 CYFA_DTYPE_BF16 if dtype == torch.bfloat16 else CYFA_DTYPE_FP32,
@@ -302,7 +307,7 @@ def forward(d, q, k, v, lam, g, beta, R, Kbar0=None, Vbar0=None, want_state=Fals
     B, T, H, D = v.shape
     Ko = Vo = None
     if want_state:
-        Ko = torch.empty(B, H, 128, D, dtype=torch.float32, device=v.device)
+        Ko = torch.empty(B, H, storage_rows(d.m), D, dtype=torch.float32, device=v.device)
         Vo = torch.empty_like(Ko)
     if ws is None:
         ws = workspace(d, CYFA_WS_FWD, v.device)

@@ -178,8 +178,9 @@ def gpu_forward(d, inp, want_state=False, Kbar0=None, Vbar0=None, lambda0=None):
     o = gd.empty_like(v)
     Ko = Vo = None
     if want_state:
-        Ko = gd.empty((B, H, 128, D), torch.float32, v.device)
-        Vo = gd.empty((B, H, 128, D), torch.float32, v.device)
+        ms = cyfa.storage_rows(d.m)
+        Ko = gd.empty((B, H, ms, D), torch.float32, v.device)
+        Vo = gd.empty((B, H, ms, D), torch.float32, v.device)
     ws = cyfa.workspace(d, cyfa.CYFA_WS_FWD, v.device)
     cyfa.cyfa_chunk_fwd(d, inp['q'], inp['k'], v, lam, g, beta, inp['R'], Kbar0, Vbar0, o, Ko, Vo,
                         ws)

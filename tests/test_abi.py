@@ -51,11 +51,18 @@ def test_workspace_sizes(lib):
     assert 2 * 16 * 32 * 128 * 256 * 4 <= fwd_tc < fwd
     assert cyfa.cyfa_workspace_size(d, cyfa.CYFA_WS_BWD) > 0
     assert cyfa.cyfa_workspace_size(d, cyfa.CYFA_WS_PREPARE) >= 2 * 16 * 32 * 8
+    # m = 255: 256 storage rows on the CUDA-core kernels, 64-token chunks forward and 32-token
+    # chunks backward (readout matrices 2 x H x 256 x 256; one [256 x 2D] state per chunk)
+    d = cyfa.dims(1, 2048, 4, 256, m=255)
+    fwd255 = cyfa.cyfa_workspace_size(d, cyfa.CYFA_WS_FWD)
+    assert fwd255 >= 2 * 4 * 256 * 256 * 4 + 4 * 32 * 256 * 512 * 4
+    bwd255 = cyfa.cyfa_workspace_size(d, cyfa.CYFA_WS_BWD)
+    assert bwd255 >= 2 * 4 * 64 * 256 * 512 * 4 + 2 * 4 * 2048 * 256 * 4
 
 
 @pytest.mark.parametrize('field,value,code', [
-    ('m', 64, cyfa.CYFA_ERR_SHAPE), ('m', 129, cyfa.CYFA_ERR_SHAPE), ('m', 0, cyfa.CYFA_ERR_SHAPE),
-    ('m', 255, cyfa.CYFA_ERR_UNSUPPORTED), ('dk', 96, cyfa.CYFA_ERR_SHAPE),
+    ('m', 64, cyfa.CYFA_ERR_SHAPE), ('m', 256, cyfa.CYFA_ERR_SHAPE), ('m', 0, cyfa.CYFA_ERR_SHAPE),
+    ('m', 257, cyfa.CYFA_ERR_SHAPE), ('dk', 96, cyfa.CYFA_ERR_SHAPE),
     ('chunk', 32, cyfa.CYFA_ERR_SHAPE), ('T', 100, cyfa.CYFA_ERR_SHAPE), ('B', 0, cyfa.CYFA_ERR_ARG),
     ('dtype', 7, cyfa.CYFA_ERR_ARG), ('B', 65536, cyfa.CYFA_ERR_SHAPE)])
 def test_bad_dims_rejected_on_host(lib, field, value, code):
@@ -88,6 +95,7 @@ def test_saved_size(lib):
     assert cyfa.cyfa_saved_size(cyfa.dims(B, T, H, 128)) == full
     assert cyfa.cyfa_saved_size(cyfa.dims(B, T, H, 128, m=63)) == full   # odd m in 63..127
     assert cyfa.cyfa_saved_size(cyfa.dims(B, T, H, 128, m=31)) == 0
+    assert cyfa.cyfa_saved_size(cyfa.dims(B, T, H, 128, m=255)) == 0   # 256 storage rows
     assert cyfa.cyfa_saved_size(cyfa.dims(B, T, H, 256)) == 0
     assert cyfa.cyfa_saved_size(cyfa.dims(B, T, H, 128, cuda_cores=True)) == 0
     assert cyfa.cyfa_saved_size(cyfa.dims(B, T, H, 64)) == 0

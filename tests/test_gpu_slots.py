@@ -1,7 +1,7 @@
-"""Slot-count variants (the paper's ablation over m, Table ablations): every odd m <= 127 through
-the C ABI against the fp64 oracle, on the tensor-core kernels (bf16, d = 128) and on the CUDA-core
-kernels; rows m..127 of the 128 storage rows stay zero.  m = 255 (256 storage rows) is refused
-with CYFA_ERR_UNSUPPORTED."""
+"""Slot-count variants (the paper's ablation over m, Table ablations): odd m through the C ABI
+against the fp64 oracle, on the tensor-core kernels (bf16, d = 128, 63 <= m <= 127) and on the
+CUDA-core kernels.  m <= 127 keeps 128 storage rows, larger m (the ablation's m = 255) 256; the
+rows m.. of the storage stay zero."""
 import numpy as np
 import pytest
 import torch
@@ -22,11 +22,16 @@ pytestmark = pytest.mark.gpu
                                                   (63, torch.bfloat16, 128, True),
                                                   (1, torch.float32, 64, True),
                                                   (5, torch.float32, 64, True),
-                                                  (63, torch.float32, 64, True)])
+                                                  (63, torch.float32, 64, True),
+                                                  (255, torch.float32, 64, True),
+                                                  (255, torch.bfloat16, 128, False),
+                                                  (255, torch.bfloat16, 256, False),
+                                                  (131, torch.float32, 128, True)])
 def test_slots_forward_backward(m, dtype, D, cuda_cores):
     """m = 5 in bf16 runs on the CUDA-core kernels even unforced (the tensor-core kernels take
-    m >= 63).  m = 1 runs in fp32 only: its single slot sums v over the whole memory (outputs up to ~30
-    here), where the bf16 rounding of the output alone (2^-9 |o|) exceeds the 2e-2 bar."""
+    63 <= m <= 127), and so do m = 131 and m = 255 (256 storage rows).  m = 1 runs in fp32 only:
+    its single slot sums v over the whole memory (outputs up to ~30 here), where the bf16 rounding
+    of the output alone (2^-9 |o|) exceeds the 2e-2 bar."""
     B, T, H = 1, 384, 2
     inp = to_device(synth.make_inputs(B, T, H, D, seed=41, dtype=dtype, with_dO=True, m=m))
     d = cyfa.dims(B, T, H, D, chunk=64, dtype=dtype, m=m, cuda_cores=cuda_cores)
@@ -67,20 +72,34 @@ def test_slots_63_full_size_sampled():
         assert_close_bf16(pairs_np(out[gk].float(), pairs), ref[rk], 'm=63 %s' % gk)
 
 
-@pytest.mark.parametrize('m', [5, 63])
-def test_slots_decode(m):
-    B, H, D, T0, steps = 2, 3, 128, 128, 16
+def test_slots_255_paper_shape_sampled():
+    """m = 255 at the shape of the paper's ablation model (400M: H = 4, d = 256, T = 2048; B = 8
+    of its 32 here): outputs and gradients of sampled (b, h) sequences (dA and dR, sums over
+    every sequence, are checked at the small size above)."""
+    B, T, H, D, m = 8, 2048, 4, 256, 255
+    inp = synth.make_inputs(B, T, H, D, seed=5, device='cuda', with_dO=True, m=m)
+    d = cyfa.dims(B, T, H, D, chunk=64, m=m)
+    o = gpu_forward(d, inp)[0]
+    out = gpu_backward(d, inp, want_dA=False)
+    pairs = sample_pairs(B, H, 3)
+    oi = oracle_inputs(inp, pairs)
+    assert_close_bf16(pairs_np(o.float(), pairs), oracle_forward(oi)[0], 'm=255 o')
+    ref = oracle_backward(oi, pairs_np(inp['dO'], pairs))
+    for gk, rk in GRADS:
+        assert_close_bf16(pairs_np(out[gk].float(), pairs), ref[rk], 'm=255 %s' % gk)
+
+
+@pytest.mark.parametrize('m,D', [(5, 128), (63, 128), (255, 128), (255, 256)])
+def test_slots_decode(m, D):
+    B, H, T0, steps = 2, 3, 128, 16
     inp = synth.make_inputs(B, T0 + steps, H, D, seed=42, device='cuda', m=m)
     o, K, V, lam = _decode(inp, T0, steps, cyfa.dims(B, T0, H, D, chunk=64, m=m),
                            cyfa.dims(B, 1, H, D, chunk=64, m=m))
     pairs = [(b, h) for b in range(B) for h in range(H)]
-    o_ref = oracle_forward(oracle_inputs(inp, pairs))[0]
+    o_ref, Kb, _, _ = oracle_forward(oracle_inputs(inp, pairs))
     got = np.stack([o[b, :, h].double().cpu().numpy() for b, h in pairs])
     assert_close_bf16(got, o_ref[:, T0:], 'm=%d decode o' % m)
-
-
-def test_slots_255_unsupported():
-    d = cyfa.dims(1, 128, 1, 128, m=255)
-    with pytest.raises(cyfa.CyfaError) as e:
-        cyfa.workspace(d, cyfa.CYFA_WS_FWD)
-    assert e.value.code == cyfa.CYFA_ERR_UNSUPPORTED
+    Kg = np.stack([K[b, h].double().cpu().numpy() for b, h in pairs])
+    assert_close_bf16(Kg[:, :m], Kb, 'm=%d Kbar after decode' % m)
+    assert K.shape[2] == cyfa.storage_rows(m)
+    assert torch.all(K[:, :, m:] == 0) and torch.all(V[:, :, m:] == 0)   # padding rows stay zero

@@ -22,7 +22,7 @@ def _case(N, T, d, m, seed, A=0.5, jitter=0.3):
     return q, k, v, delta, alpha, beta, R
 
 
-@pytest.mark.parametrize('m,T,d', [(5, 17, 3), (7, 12, 4), (127, 9, 5)])
+@pytest.mark.parametrize('m,T,d', [(5, 17, 3), (7, 12, 4), (127, 9, 5), (255, 7, 3)])
 def test_four_forms_agree(m, T, d):
     q, k, v, delta, alpha, beta, R = _case(2, T, d, m, seed=m)
     s = 0.9
