@@ -576,6 +576,15 @@ def run_extra_shape(args, dev, rank, peaks, B, T, H, D, m, what):
     n = max(1, min(args.steps, 20))
     ms = timed(step, n)
     ms_fwd = timed(fwd, n)
+    # per-kernel split of two more steps (CUDA events around each launch)
+    cyfa.cyfa_stats_reset()
+    cyfa.cyfa_stats_timing(True)
+    for _ in range(2):
+        step()
+    torch.cuda.synchronize()
+    split = {k: round(t / 2, 4) for k, (_, t) in sorted(cyfa.cyfa_stats_get().items(),
+                                                         key=lambda kv: -kv[1][1])}
+    cyfa.cyfa_stats_timing(False)
     cyfa.cyfa_check()
     th = B * T * H
     fl = operator_flops_per_token_head(C, d=D, ms=m + 1) * th
@@ -591,7 +600,7 @@ def run_extra_shape(args, dev, rank, peaks, B, T, H, D, m, what):
             'fwd_ms': ms_fwd, 'fwd_tokens_per_s': B * T / (ms_fwd / 1e3),
             'tflops_rule': tf, 'peak_tflops': peak,
             'peak_source': 'measured bf16 burst' if tc else 'fp32 FMA: 152 x 128 x 2 x clock',
-            'frac_peak': tf / peak}
+            'frac_peak': tf / peak, 'kernel_ms_per_step': split}
 
 
 def run_mixer(args, dev, rank, peaks):

@@ -130,7 +130,6 @@ __global__ void __launch_bounds__(256) fwd_out_kernel(FwdArgs a) {
     float* seg = sg + C;
     float* slam = seg + C;
     float* sbeta = slam + C;
-    float* swarp = sbeta + C;    // [8][2 MSZ]
     const int tx = threadIdx.x & 15, ty = threadIdx.x >> 4;
     const float* Sst = a.states + ((size_t)bh * nchunk + c) * MSZ * (2 * D);
     const TI* Q = (const TI*)a.q;
@@ -190,8 +189,8 @@ __global__ void __launch_bounds__(256) fwd_out_kernel(FwdArgs a) {
         for (int j = 0; j < NJ; ++j) sX[(ty + 16 * i) * LDM + tx + 16 * j] = o1[i][j];
     __syncthreads();
 
-    middle_rows<MSZ>(sX, slam, C, a.M + (size_t)h * MSZ * MSZ, a.MT + (size_t)h * MSZ * MSZ, swarp,
-                     s.sl);
+    middle_rows<MSZ, 4>(sX, slam, C, a.M + (size_t)h * MSZ * MSZ, a.MT + (size_t)h * MSZ * MSZ,
+                        s.sl);
     __syncthreads();
 
     // P = (O'' A^T) o Gamma
@@ -261,8 +260,7 @@ cudaError_t fwd_dispatch(const FwdArgs& a, cudaStream_t st) {
     const Shape& s = a.s;
     cudaError_t e = launch_state<C, MSZ, TI>(a, "fwd_state", st);
     if (e != cudaSuccess) return e;
-    const size_t sm_out =
-        (size_t)(2 * C * (MSZ + 1) + C * (C + 1) + 4 * C + 8 * 2 * MSZ) * sizeof(float);
+    const size_t sm_out = (size_t)(2 * C * (MSZ + 1) + C * (C + 1) + 4 * C) * sizeof(float);
     auto kout = fwd_out_kernel<C, D, MSZ, TI>;
     cudaFuncSetAttribute(kout, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm_out);
     { LaunchScope ls_("fwd_out", st); kout<<<dim3(s.nchunk(), s.B * s.H), 256, sm_out, st>>>(a); }

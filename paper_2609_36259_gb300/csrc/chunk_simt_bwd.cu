@@ -57,136 +57,194 @@ __device__ __forceinline__ float warp_omega_dot(const float* x, const float* y, 
     return warp_sum(acc);
 }
 
-// Gradient of the middle readout, one warp per row:
-// given o' (sO1), o'' (sO2) and dL/do'' (sD), writes dL/do' into sD and the row scalars
-// sdG[r] = <o'', do''> and sdL[r] = <dz, Omega z> - <do'', Omega o''>.  With gz non-null the
-// row's z, p, dy, dl (for dR) go to gz / gp / gdy / gdl + MSZ r.  Rows have stride MSZ + 1;
-// swarp holds 5 x MSZ floats per warp.
-template <int MSZ>
+// Gradient of the middle readout: given o' (sO1), o'' (sO2) and dL/do'' (sD), writes dL/do' into
+// sD and the row scalars sdG[r] = <o'', do''> and sdL[r] = <dz, Omega z> - <do'', Omega o''>.
+// With gz non-null the row's z, p, dy, dl (for dR) go to gz / gp / gdy / gdl + MSZ r.  Rows have
+// stride MSZ + 1.  Each warp takes RB rows at a time, so that every entry of M and M^T it loads
+// serves RB rows; the vectors stay in registers (rotation pairs j = lane + 1 + 32 u, slot
+// entries lane + 32 v) and the products over slots broadcast the summed-over vector from its
+// owner lane by shuffles, in slot order.  C is a multiple of 8 RB.
+template <int MSZ, int RB>
 __device__ __noinline__ void middle_rows_bwd(const float* sO1, const float* sO2, float* sD,
                                              const float* slam, int C, const float* M,
-                                             const float* MT, float* swarp, float* sdG,
-                                             float* sdL, float* gz, float* gp, float* gdy,
-                                             float* gdl, const Slots& sl) {
+                                             const float* MT, float* sdG, float* sdL, float* gz,
+                                             float* gp, float* gdy, float* gdl, const Slots& sl) {
     using G = Geo<MSZ>;
-    constexpr int NP = G::NP, NE = G::NE;
+    constexpr int NP = G::NP, NE = G::NE, LDM = G::LDM;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    float* z = swarp + warp * 5 * MSZ;
-    float* p = z + MSZ;
-    float* dy = p + MSZ;
-    float* dl = dy + MSZ;
-    float* dz = dl + MSZ;
-    for (int r = warp; r < C; r += 8) {
-        const float* x1 = sO1 + r * G::LDM;
-        const float* x2 = sO2 + r * G::LDM;
-        float* xd = sD + r * G::LDM;
-        const float lam = slam[r];
-        float cs[NP], sn[NP];
+    const int npair = sl.npair, m = sl.m;
+    for (int r0 = warp * RB; r0 < C; r0 += 8 * RB) {
+        float cs[RB][NP], sn[RB][NP], zc[RB][NP], zs[RB][NP], yc[RB][NP], ys[RB][NP];
+        float z0[RB], y0[RB], g1[RB], om2[RB];
+#pragma unroll
+        for (int rb = 0; rb < RB; ++rb) {
+            const float* x1 = sO1 + (r0 + rb) * LDM;
+            const float* x2 = sO2 + (r0 + rb) * LDM;
+            const float* xd = sD + (r0 + rb) * LDM;
+            const float lam = slam[r0 + rb];
+            z0[rb] = x1[0];
+            y0[rb] = xd[0];
+#pragma unroll
+            for (int u = 0; u < NP; ++u) {
+                const int j = lane + 1 + 32 * u;
+                cs[rb][u] = 1.f;
+                sn[rb][u] = 0.f;
+                zc[rb][u] = zs[rb][u] = yc[rb][u] = ys[rb][u] = 0.f;
+                if (j <= npair) {   // z = U(lam) o', dy = U(lam) do''
+                    sincospif(phase_pi_m(lam, j, sl), &sn[rb][u], &cs[rb][u]);
+                    const float xc = x1[2 * j - 1], xs = x1[2 * j];
+                    zc[rb][u] = cs[rb][u] * xc - sn[rb][u] * xs;
+                    zs[rb][u] = sn[rb][u] * xc + cs[rb][u] * xs;
+                    const float gc = xd[2 * j - 1], gs = xd[2 * j];
+                    yc[rb][u] = cs[rb][u] * gc - sn[rb][u] * gs;
+                    ys[rb][u] = sn[rb][u] * gc + cs[rb][u] * gs;
+                }
+            }
+            float a1 = 0.f;
+#pragma unroll
+            for (int v = 0; v < NE; ++v) a1 += x2[lane + 32 * v] * xd[lane + 32 * v];
+            g1[rb] = warp_sum(a1);                                  // <o'', do''>
+            om2[rb] = warp_omega_dot<MSZ>(xd, x2, lane, sl);        // <do'', Omega o''>
+        }
+        // logits l = M z and dp = M dy (M^T rows k, entries col = lane + 32 v)
+        float l[RB][NE], dp[RB][NE];
+#pragma unroll
+        for (int v = 0; v < NE; ++v) {
+            const float mt = MT[lane + 32 * v];
+#pragma unroll
+            for (int rb = 0; rb < RB; ++rb) {
+                l[rb][v] = mt * z0[rb];
+                dp[rb][v] = mt * y0[rb];
+            }
+        }
 #pragma unroll
         for (int u = 0; u < NP; ++u) {
-            const int j = lane + 1 + 32 * u;
-            cs[u] = 1.f;
-            sn[u] = 0.f;
-            if (j <= sl.npair) {
-                sincospif(phase_pi_m(lam, j, sl), &sn[u], &cs[u]);
-                const float xc = x1[2 * j - 1], xs = x1[2 * j];
-                z[2 * j - 1] = cs[u] * xc - sn[u] * xs;
-                z[2 * j] = sn[u] * xc + cs[u] * xs;
-                const float gc = xd[2 * j - 1], gs = xd[2 * j];
-                dy[2 * j - 1] = cs[u] * gc - sn[u] * gs;     // dy = U(lam) do''
-                dy[2 * j] = sn[u] * gc + cs[u] * gs;
-            } else if (j <= G::NPAIRS) {   // padding slots (zero)
-                z[2 * j - 1] = z[2 * j] = 0.f;
-                dy[2 * j - 1] = dy[2 * j] = 0.f;
+            const int jmax = min(32, npair - 32 * u);   // pairs 32 u + 1 .. 32 u + jmax
+            for (int src = 0; src < jmax; ++src) {
+                const int kc = 2 * (32 * u + src) + 1;
+                float vzc[RB], vzs[RB], vyc[RB], vys[RB];
+#pragma unroll
+                for (int rb = 0; rb < RB; ++rb) {
+                    vzc[rb] = __shfl_sync(0xffffffffu, zc[rb][u], src);
+                    vzs[rb] = __shfl_sync(0xffffffffu, zs[rb][u], src);
+                    vyc[rb] = __shfl_sync(0xffffffffu, yc[rb][u], src);
+                    vys[rb] = __shfl_sync(0xffffffffu, ys[rb][u], src);
+                }
+                const float* mc = MT + kc * MSZ + lane;
+#pragma unroll
+                for (int v = 0; v < NE; ++v) {
+                    const float a = mc[32 * v], b = mc[MSZ + 32 * v];
+#pragma unroll
+                    for (int rb = 0; rb < RB; ++rb) {
+                        l[rb][v] = fmaf(b, vzs[rb], fmaf(a, vzc[rb], l[rb][v]));
+                        dp[rb][v] = fmaf(b, vys[rb], fmaf(a, vyc[rb], dp[rb][v]));
+                    }
+                }
             }
         }
-        if (lane == 0) {
-            z[0] = x1[0];
-            z[MSZ - 1] = 0.f;
-            dy[0] = xd[0];
-            dy[MSZ - 1] = 0.f;
-        }
-        __syncwarp();
-        float g1 = 0.f;
+        // p = softmax(l) over the m active slots (into l), dl = p o (dp - <p, dp>) (into dp)
 #pragma unroll
-        for (int u = 0; u < NE; ++u) g1 += x2[lane + 32 * u] * xd[lane + 32 * u];
-        g1 = warp_sum(g1);
-        const float om2 = warp_omega_dot<MSZ>(xd, x2, lane, sl);  // <do'', Omega o''>
-        // logits and softmax
-        float l[NE], dp[NE];
+        for (int rb = 0; rb < RB; ++rb) {
+            float mx = -INFINITY;
 #pragma unroll
-        for (int u = 0; u < NE; ++u) l[u] = dp[u] = 0.f;
-        for (int k = 0; k < MSZ; ++k) {
-            const float zk = z[k], dyk = dy[k];
-#pragma unroll
-            for (int u = 0; u < NE; ++u) {
-                const float mt = MT[k * MSZ + lane + 32 * u];
-                l[u] = fmaf(mt, zk, l[u]);
-                dp[u] = fmaf(mt, dyk, dp[u]);           // dp = M dy
+            for (int v = 0; v < NE; ++v) {
+                if (lane + 32 * v >= m) l[rb][v] = -INFINITY;
+                mx = fmaxf(mx, l[rb][v]);
             }
-        }
-        float mx = -INFINITY;
+            mx = warp_max(mx);
+            float sum = 0.f;
 #pragma unroll
-        for (int u = 0; u < NE; ++u) {
-            if (lane + 32 * u >= sl.m) l[u] = -INFINITY;
-            mx = fmaxf(mx, l[u]);
-        }
-        mx = warp_max(mx);
-        float e[NE], sum = 0.f;
+            for (int v = 0; v < NE; ++v) {
+                l[rb][v] = expf(l[rb][v] - mx);
+                sum += l[rb][v];
+            }
+            const float inv = 1.f / warp_sum(sum);
+            float pdp = 0.f;
 #pragma unroll
-        for (int u = 0; u < NE; ++u) {
-            e[u] = expf(l[u] - mx);
-            sum += e[u];
-        }
-        sum = warp_sum(sum);
-        const float inv = 1.f / sum;
-        float pdp = 0.f;
+            for (int v = 0; v < NE; ++v) {
+                l[rb][v] *= inv;
+                pdp += l[rb][v] * dp[rb][v];
+            }
+            pdp = warp_sum(pdp);
 #pragma unroll
-        for (int u = 0; u < NE; ++u) {
-            e[u] *= inv;
-            pdp += e[u] * dp[u];
+            for (int v = 0; v < NE; ++v) dp[rb][v] = l[rb][v] * (dp[rb][v] - pdp);
         }
-        pdp = warp_sum(pdp);
-#pragma unroll
-        for (int u = 0; u < NE; ++u) dl[lane + 32 * u] = e[u] * (dp[u] - pdp);
         if (gz) {
 #pragma unroll
-            for (int u = 0; u < NE; ++u) {
-                const int k = lane + 32 * u;
-                gz[r * MSZ + k] = z[k];
-                gp[r * MSZ + k] = e[u];
-                gdy[r * MSZ + k] = dy[k];
-                gdl[r * MSZ + k] = e[u] * (dp[u] - pdp);
+            for (int rb = 0; rb < RB; ++rb) {
+                const size_t o = (size_t)(r0 + rb) * MSZ;
+#pragma unroll
+                for (int v = 0; v < NE; ++v) {
+                    gp[o + lane + 32 * v] = l[rb][v];
+                    gdl[o + lane + 32 * v] = dp[rb][v];
+                }
+#pragma unroll
+                for (int u = 0; u < NP; ++u) {
+                    const int j = lane + 1 + 32 * u;
+                    if (j <= G::NPAIRS) {   // zero on the padding pairs
+                        gz[o + 2 * j - 1] = zc[rb][u];
+                        gz[o + 2 * j] = zs[rb][u];
+                        gdy[o + 2 * j - 1] = yc[rb][u];
+                        gdy[o + 2 * j] = ys[rb][u];
+                    }
+                }
+                if (lane == 0) {
+                    gz[o] = z0[rb];
+                    gz[o + MSZ - 1] = 0.f;
+                    gdy[o] = y0[rb];
+                    gdy[o + MSZ - 1] = 0.f;
+                }
+            }
+        }
+        // dz = M^T dl (entries col = lane + 32 v), into the rows of sD (do'' is consumed)
+        float g[RB][NE];
+#pragma unroll
+        for (int rb = 0; rb < RB; ++rb)
+#pragma unroll
+            for (int v = 0; v < NE; ++v) g[rb][v] = 0.f;
+#pragma unroll
+        for (int v2 = 0; v2 < NE; ++v2) {
+            const int imax = min(32, m - 32 * v2);
+            for (int src = 0; src < imax; ++src) {
+                float dv[RB];
+#pragma unroll
+                for (int rb = 0; rb < RB; ++rb) dv[rb] = __shfl_sync(0xffffffffu, dp[rb][v2], src);
+                const float* mr = M + (32 * v2 + src) * MSZ + lane;
+#pragma unroll
+                for (int v = 0; v < NE; ++v) {
+                    const float a = mr[32 * v];
+#pragma unroll
+                    for (int rb = 0; rb < RB; ++rb) g[rb][v] = fmaf(a, dv[rb], g[rb][v]);
+                }
             }
         }
         __syncwarp();
-        float g[NE];                                         // dz = M^T dl
 #pragma unroll
-        for (int u = 0; u < NE; ++u) g[u] = 0.f;
-        for (int i = 0; i < sl.m; ++i) {
-            const float di = dl[i];
+        for (int rb = 0; rb < RB; ++rb) {
+            float* xd = sD + (r0 + rb) * LDM;
 #pragma unroll
-            for (int u = 0; u < NE; ++u) g[u] = fmaf(M[i * MSZ + lane + 32 * u], di, g[u]);
+            for (int v = 0; v < NE; ++v) xd[lane + 32 * v] = g[rb][v];   // padding entries are 0
         }
-#pragma unroll
-        for (int u = 0; u < NE; ++u) dz[lane + 32 * u] = g[u];
         __syncwarp();
-        const float om1 = warp_omega_dot<MSZ>(dz, z, lane, sl);   // <dz, Omega z>
-        // do' = U(-lam) dz
 #pragma unroll
-        for (int u = 0; u < NP; ++u) {
-            const int j = lane + 1 + 32 * u;
-            if (j <= G::NPAIRS) {
-                const float gc = dz[2 * j - 1], gs = dz[2 * j];
-                xd[2 * j - 1] = cs[u] * gc + sn[u] * gs;
-                xd[2 * j] = -sn[u] * gc + cs[u] * gs;
+        for (int rb = 0; rb < RB; ++rb) {
+            float* xd = sD + (r0 + rb) * LDM;
+            float a = 0.f;   // <dz, Omega z>, then do' = U(-lam) dz on the active pairs
+#pragma unroll
+            for (int u = 0; u < NP; ++u) {
+                const int j = lane + 1 + 32 * u;
+                if (j <= npair) {
+                    const float gc = xd[2 * j - 1], gs = xd[2 * j];
+                    a += freq(j, sl) * (gs * zc[rb][u] - gc * zs[rb][u]);
+                    xd[2 * j - 1] = cs[rb][u] * gc + sn[rb][u] * gs;
+                    xd[2 * j] = -sn[rb][u] * gc + cs[rb][u] * gs;
+                }
             }
-        }
-        if (lane == 0) {
-            xd[0] = dz[0];
-            xd[MSZ - 1] = 0.f;
-            sdG[r] = g1;
-            sdL[r] = om1 - om2;
+            const float om1 = warp_sum(a);
+            if (lane == 0) {
+                sdG[r0 + rb] = g1[rb];
+                sdL[r0 + rb] = om1 - om2[rb];
+            }
         }
         __syncwarp();
     }
@@ -317,7 +375,6 @@ __global__ void __launch_bounds__(256) bwd_intra1_kernel(BwdArgs a) {
     float* sbeta = slam + CB;
     float* sdG = sbeta + CB;
     float* sdL = sdG + CB;
-    float* swarp = sdL + CB;     // [8][5 MSZ]
     const int tx = threadIdx.x & 15, ty = threadIdx.x >> 4;
     const float* Sst = a.states + ((size_t)bh * nchunk + c) * MSZ * (2 * D);
     const float* Mh = a.M + (size_t)h * MSZ * MSZ;
@@ -353,7 +410,7 @@ __global__ void __launch_bounds__(256) bwd_intra1_kernel(BwdArgs a) {
             }
     }
     __syncthreads();
-    middle_rows<MSZ>(sO2, slam, CB, Mh, MTh, swarp, s.sl);
+    middle_rows<MSZ, 4>(sO2, slam, CB, Mh, MTh, s.sl);
 
     // dO'' = gamma o (dO Vbar^T) + (dO V^T o Gamma) A
     masked_scores_tok<MSZ>(sP, sS, sg, dO, V, s, b, h, t0, 1.f);
@@ -376,7 +433,7 @@ __global__ void __launch_bounds__(256) bwd_intra1_kernel(BwdArgs a) {
     {
         const size_t rowbase = ((size_t)bh * s.T + t0) * MSZ;
         const bool dr = a.mZ != nullptr;
-        middle_rows_bwd<MSZ>(sO1, sO2, sD, slam, CB, Mh, MTh, swarp, sdG, sdL,
+        middle_rows_bwd<MSZ, MSZ == 128 ? 4 : 2>(sO1, sO2, sD, slam, CB, Mh, MTh, sdG, sdL,
                         dr ? a.mZ + rowbase : nullptr, dr ? a.mP + rowbase : nullptr,
                         dr ? a.mDY + rowbase : nullptr, dr ? a.mDL + rowbase : nullptr, s.sl);
     }
@@ -774,33 +831,83 @@ __global__ void dA_final_kernel(BwdArgs a, int nseg) {
     a.dA[h] = (float)t;
 }
 
-// dM[h][i][j] = sum over the batch and the tokens of dl[i] z[j] + p[i] dy[j] (paper order), one
-// block per (h, i), one thread per j (ms threads).
-__global__ void __launch_bounds__(MS_MAX) dm_reduce_simt(BwdArgs a) {
+// Partial dM over one range of tokens: dMp[h][sp][i][j] = sum over the sp-th of nsplit equal
+// ranges of the head's B*T tokens of dl[i] z[j] + p[i] dy[j] (paper order; the per-token vectors
+// are [B*H][T][ms] fp32).  Block (i tile, j tile, h * nsplit + sp) forms a 64 x 64 tile of dM
+// with 16 x 16 threads holding 4 x 4 outputs each; 32 tokens at a time are staged in shared
+// memory (zero past the range's end).
+constexpr int DM_TILE = 64, DM_TOK = 32;
+__global__ void __launch_bounds__(256) dm_partial_simt(BwdArgs a, int nsplit) {
     const Shape s = a.s;
     const int ms = s.sl.ms;
-    const int h = blockIdx.x, i = blockIdx.y, j = threadIdx.x;
-    float acc = 0.f;
-    for (int b = 0; b < s.B; ++b) {
-        const size_t base = ((size_t)b * s.H + h) * s.T * ms;
-        for (int t = 0; t < s.T; ++t) {
-            const size_t o = base + (size_t)t * ms;
-            acc = fmaf(a.mDL[o + i], a.mZ[o + j], acc);
-            acc = fmaf(a.mP[o + i], a.mDY[o + j], acc);
+    const int i0 = blockIdx.x * DM_TILE, j0 = blockIdx.y * DM_TILE;
+    const int h = blockIdx.z / nsplit, sp = blockIdx.z % nsplit;
+    const long long N = (long long)s.B * s.T;
+    const long long n0 = N * sp / nsplit, n1 = N * (sp + 1) / nsplit;
+    const int tid = threadIdx.x, tx = tid & 15, ty = tid >> 4;
+    __shared__ float sL[DM_TOK][DM_TILE], sP[DM_TOK][DM_TILE], sZ[DM_TOK][DM_TILE],
+        sY[DM_TOK][DM_TILE];
+    float acc[4][4];
+    zero_acc(acc);
+    for (long long nb = n0; nb < n1; nb += DM_TOK) {
+        __syncthreads();
+        for (int e = tid; e < DM_TOK * DM_TILE; e += 256) {
+            const int r = e / DM_TILE, c = e % DM_TILE;
+            const long long n = nb + r;
+            float l = 0.f, p = 0.f, z = 0.f, y = 0.f;
+            if (n < n1) {
+                const long long b = n / s.T, t = n - b * s.T;
+                const size_t o = (((size_t)b * s.H + h) * s.T + t) * ms;
+                l = a.mDL[o + i0 + c];
+                p = a.mP[o + i0 + c];
+                z = a.mZ[o + j0 + c];
+                y = a.mDY[o + j0 + c];
+            }
+            sL[r][c] = l;
+            sP[r][c] = p;
+            sZ[r][c] = z;
+            sY[r][c] = y;
+        }
+        __syncthreads();
+#pragma unroll 4
+        for (int k = 0; k < DM_TOK; ++k) {
+            float l[4], p[4], z[4], y[4];
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+                l[u] = sL[k][ty + 16 * u];
+                p[u] = sP[k][ty + 16 * u];
+                z[u] = sZ[k][tx + 16 * u];
+                y[u] = sY[k][tx + 16 * u];
+            }
+#pragma unroll
+            for (int i = 0; i < 4; ++i)
+#pragma unroll
+                for (int j = 0; j < 4; ++j) acc[i][j] = fmaf(l[i], z[j], fmaf(p[i], y[j], acc[i][j]));
         }
     }
-    a.dM[((size_t)h * ms + i) * ms + j] = acc;
+#pragma unroll
+    for (int i = 0; i < 4; ++i)
+#pragma unroll
+        for (int j = 0; j < 4; ++j)
+            a.dM[(((size_t)h * nsplit + sp) * ms + i0 + ty + 16 * i) * ms + j0 + tx + 16 * j] =
+                acc[i][j];
 }
 
 // dR[h][i][k] = sum_j dM[h][i][j] Phi[k][j] for the m active slots i, k (App. A.1
 // Eq. app-real-fourier: Phi[k][0] = 1/sqrt(m), Phi[k][2j-1] = sqrt(2/m) cos(2 pi j k / m),
-// Phi[k][2j] = sqrt(2/m) sin(2 pi j k / m)); dM [H][ms][ms] in the paper's order.  Block (h, i)
-// of ms threads.
-__global__ void __launch_bounds__(MS_MAX) dr_finalize_simt(const float* dM, float* dR, Slots sl) {
+// Phi[k][2j] = sqrt(2/m) sin(2 pi j k / m)); dM is the sum over nsplit partial blocks
+// [H][nsplit][ms][ms] in the paper's order (summed in split order).  Block (h, i) of ms threads.
+__global__ void __launch_bounds__(MS_MAX) dr_finalize_simt(const float* dMp, int nsplit, float* dR,
+                                                           Slots sl) {
     const int h = blockIdx.x, i = blockIdx.y, t = threadIdx.x;
     const int m = sl.m, ms = sl.ms;
     __shared__ float s_dm[MS_MAX], s_ct[MS_MAX], s_st[MS_MAX];
-    s_dm[t] = dM[((size_t)h * ms + i) * ms + t];
+    {
+        float acc = 0.f;
+        const float* src = dMp + ((size_t)h * nsplit * ms + i) * ms + t;
+        for (int sp = 0; sp < nsplit; ++sp) acc += src[(size_t)sp * ms * ms];
+        s_dm[t] = acc;
+    }
     if (t < m) {
         float sv, cv;
         sincospif((float)t * sl.two_over_m, &sv, &cv);
@@ -839,8 +946,7 @@ cudaError_t bwd_dispatch(const BwdArgs& a, cudaStream_t st) {
     if (e != cudaSuccess) return e;
     const dim3 gchunk(s.nchunk(), s.B * s.H);
     constexpr int SSZ = staging_floats<D, MSZ>();
-    const size_t sm1 =
-        (size_t)(4 * CB * LDM + SSZ + CB * G::LPB + 6 * CB + 8 * 5 * MSZ) * sizeof(float);
+    const size_t sm1 = (size_t)(4 * CB * LDM + SSZ + CB * G::LPB + 6 * CB) * sizeof(float);
     auto k1 = bwd_intra1_kernel<D, MSZ, TI>;
     cudaFuncSetAttribute(k1, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm1);
     { LaunchScope ls_("bwd_intra1", st); k1<<<gchunk, 256, sm1, st>>>(a); }
@@ -853,8 +959,10 @@ cudaError_t bwd_dispatch(const BwdArgs& a, cudaStream_t st) {
     cudaFuncSetAttribute(k2, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm2);
     { LaunchScope ls_("bwd_intra2", st); k2<<<gchunk, 256, sm2, st>>>(a); }
     if (a.dR) {
-        { LaunchScope ls_("bwd_dm_reduce", st); dm_reduce_simt<<<dim3(s.H, MSZ), MSZ, 0, st>>>(a); }
-        { LaunchScope ls_("bwd_dr_finalize", st); dr_finalize_simt<<<dim3(s.H, s.sl.m), MSZ, 0, st>>>(a.dM, a.dR, s.sl); }
+        const int ns = dm_splits(s);
+        const dim3 gdm(MSZ / DM_TILE, MSZ / DM_TILE, s.H * ns);
+        { LaunchScope ls_("bwd_dm_reduce", st); dm_partial_simt<<<gdm, 256, 0, st>>>(a, ns); }
+        { LaunchScope ls_("bwd_dr_finalize", st); dr_finalize_simt<<<dim3(s.H, s.sl.m), MSZ, 0, st>>>(a.dM, ns, a.dR, s.sl); }
         e = cudaGetLastError();
         if (e != cudaSuccess) return e;
     }

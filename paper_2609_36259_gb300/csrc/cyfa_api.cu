@@ -158,7 +158,7 @@ BwdLayout bwd_layout(const Shape& s0, bool tc_path, void* ws) {
         L.fP = c.take<float>(BH * s.T * ms);
         L.fDY = c.take<float>(BH * s.T * ms);
         L.fDL = c.take<float>(BH * s.T * ms);
-        L.fdM = c.take<float>((size_t)s.H * ms * ms);
+        L.fdM = c.take<float>((size_t)s.H * dm_splits(s) * ms * ms);
     }
     L.bytes = c.off;
     return L;

@@ -128,7 +128,7 @@ struct BwdArgs {
     double* seg;        // [2][B*H][nseg] reverse-scan partials
     double* dA_part;    // [B*H*nseg]
     // dR (nullable): per-token z, p, dy, dl of the middle readout (fp32 [B*H][T][ms], paper
-    // order), the per-head dM [H][ms][ms] and the output [H][m][m]
+    // order), the partial dM blocks [H][dm_splits][ms][ms] and the output [H][m][m]
     float *mZ, *mP, *mDY, *mDL;
     float *dM, *dR;
 };
@@ -140,6 +140,16 @@ cudaError_t launch_dr_finalize(const float* dMp, int dm_split, int H, bool tc_or
 constexpr int BWD_C = 64;       // chunk length used by the SIMT backward with 128 storage rows
 constexpr int BWD_C256 = 32;    // ... and with 256 (the tiles of a 64-token chunk would not fit)
 inline int bwd_chunk(const Slots& sl) { return sl.ms == 128 ? BWD_C : BWD_C256; }
+// Token ranges the CUDA-core dR reduction splits each head's B*T tokens into: about four blocks
+// per SM over the (ms / 64)^2 tiles and H heads, at least 256 tokens per range, at most 64.
+inline int dm_splits(const Shape& s) {
+    const long long tiles = (long long)(s.sl.ms / 64) * (s.sl.ms / 64) * s.H;
+    long long n = (4 * 152 + tiles - 1) / tiles;
+    const long long by_tokens = ((long long)s.B * s.T + 255) / 256;
+    if (n > by_tokens) n = by_tokens;
+    if (n > 64) n = 64;
+    return n < 1 ? 1 : (int)n;
+}
 cudaError_t launch_bwd_simt(const BwdArgs& a, cudaStream_t st);
 // reverse cumulative sums of the per-token scalars in a.tok and the logit gradients
 cudaError_t launch_bwd_gates(const BwdArgs& a, cudaStream_t st);

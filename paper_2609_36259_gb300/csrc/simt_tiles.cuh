@@ -10,93 +10,131 @@ constexpr int LD = 129;   // padded row stride of [C][128] shared tiles
 
 // ---------------------------------------------------------------------------------------
 // Token-wise middle readout for rows r < C of sX (row stride MSZ + 1, in place):
-// o'' = U(-lam) M^T softmax(M U(lam) o') with M = R Phi ([MSZ][MSZ]); the padding logits
-// (slots m..MSZ-1) are excluded from the softmax and o''[m..MSZ-1] are 0.  One warp per row; swarp
-// holds 2 x MSZ floats of scratch per warp.
-template <int MSZ>
-static __device__ __noinline__ void middle_rows(float* sX, const float* slam, int C, const float* M, const float* MT,
-                            float* swarp, const Slots& sl) {
-    constexpr int LDM = MSZ + 1, NP = MSZ / 64, NE = MSZ / 32, NPAIRS = MSZ / 2 - 1;
+// o'' = U(-lam) M^T softmax(M U(lam) o') with M = R Phi ([MSZ][MSZ], global); the padding
+// logits (slots m..MSZ-1) are excluded from the softmax and o''[m..MSZ-1] are 0.
+// Each warp takes RB rows at a time so that every entry of M and M^T it loads serves RB rows.
+// A lane keeps the rotation pairs j = lane + 1 + 32 u of its rows in registers and the logit /
+// softmax entries lane + 32 v; the products over slots broadcast the summed-over vector from
+// its owner lane by shuffles, in slot order (the same order of accumulation as a plain loop).
+// C is a multiple of 8 RB.
+template <int MSZ, int RB>
+static __device__ __noinline__ void middle_rows(float* sX, const float* slam, int C, const float* M,
+                                                const float* MT, const Slots& sl) {
+    constexpr int LDM = MSZ + 1, NP = MSZ / 64, NE = MSZ / 32;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    float* z = swarp + warp * 2 * MSZ;
-    float* p = z + MSZ;
-    for (int r = warp; r < C; r += 8) {
-        float* x = sX + r * LDM;
-        const float lam = slam[r];
-        float cs[NP], sn[NP];
+    const int npair = sl.npair, m = sl.m;
+    for (int r0 = warp * RB; r0 < C; r0 += 8 * RB) {
+        float cs[RB][NP], sn[RB][NP], zc[RB][NP], zs[RB][NP], z0[RB];
 #pragma unroll
-        for (int u = 0; u < NP; ++u) {
-            const int j = lane + 1 + 32 * u;
-            cs[u] = 1.f;
-            sn[u] = 0.f;
-            if (j <= sl.npair) {
-                sincospif(phase_pi_m(lam, j, sl), &sn[u], &cs[u]);
-                const float xc = x[2 * j - 1], xs = x[2 * j];
-                z[2 * j - 1] = cs[u] * xc - sn[u] * xs;
-                z[2 * j] = sn[u] * xc + cs[u] * xs;
-            } else if (j <= NPAIRS) {   // padding slots (zero)
-                z[2 * j - 1] = 0.f;
-                z[2 * j] = 0.f;
+        for (int rb = 0; rb < RB; ++rb) {
+            const float* x = sX + (r0 + rb) * LDM;
+            const float lam = slam[r0 + rb];
+            z0[rb] = x[0];
+#pragma unroll
+            for (int u = 0; u < NP; ++u) {
+                const int j = lane + 1 + 32 * u;
+                cs[rb][u] = 1.f;
+                sn[rb][u] = 0.f;
+                zc[rb][u] = zs[rb][u] = 0.f;
+                if (j <= npair) {   // z = U(lam) o'
+                    sincospif(phase_pi_m(lam, j, sl), &sn[rb][u], &cs[rb][u]);
+                    const float xc = x[2 * j - 1], xs = x[2 * j];
+                    zc[rb][u] = cs[rb][u] * xc - sn[rb][u] * xs;
+                    zs[rb][u] = sn[rb][u] * xc + cs[rb][u] * xs;
+                }
             }
         }
-        if (lane == 0) {
-            z[0] = x[0];
-            z[MSZ - 1] = 0.f;
+        // logits l[col] = sum_k MT[k][col] z[k], col = lane + 32 v
+        float l[RB][NE];
+#pragma unroll
+        for (int v = 0; v < NE; ++v) {
+            const float mt = MT[lane + 32 * v];
+#pragma unroll
+            for (int rb = 0; rb < RB; ++rb) l[rb][v] = mt * z0[rb];
         }
-        __syncwarp();
-        float l[NE];
-#pragma unroll
-        for (int u = 0; u < NE; ++u) l[u] = 0.f;
-        for (int k = 0; k < MSZ; ++k) {
-            const float zk = z[k];
-#pragma unroll
-            for (int u = 0; u < NE; ++u) l[u] = fmaf(MT[k * MSZ + lane + 32 * u], zk, l[u]);
-        }
-        float mx = -INFINITY;
-#pragma unroll
-        for (int u = 0; u < NE; ++u) {
-            if (lane + 32 * u >= sl.m) l[u] = -INFINITY;
-            mx = fmaxf(mx, l[u]);
-        }
-        mx = warp_max(mx);
-        float e[NE], sum = 0.f;
-#pragma unroll
-        for (int u = 0; u < NE; ++u) {
-            e[u] = expf(l[u] - mx);
-            sum += e[u];
-        }
-        sum = warp_sum(sum);
-        const float inv = 1.f / sum;
-#pragma unroll
-        for (int u = 0; u < NE; ++u) p[lane + 32 * u] = e[u] * inv;
-        __syncwarp();
-        float y[NE];
-#pragma unroll
-        for (int u = 0; u < NE; ++u) y[u] = 0.f;
-        for (int i = 0; i < sl.m; ++i) {
-            const float pi = p[i];
-#pragma unroll
-            for (int u = 0; u < NE; ++u) y[u] = fmaf(M[i * MSZ + lane + 32 * u], pi, y[u]);
-        }
-        __syncwarp();
-#pragma unroll
-        for (int u = 0; u < NE; ++u) z[lane + 32 * u] = y[u];
-        __syncwarp();
 #pragma unroll
         for (int u = 0; u < NP; ++u) {
-            const int j = lane + 1 + 32 * u;
-            if (j <= sl.npair) {
-                const float yc = z[2 * j - 1], ys = z[2 * j];
-                x[2 * j - 1] = cs[u] * yc + sn[u] * ys;
-                x[2 * j] = -sn[u] * yc + cs[u] * ys;
-            } else if (j <= NPAIRS) {
-                x[2 * j - 1] = 0.f;
-                x[2 * j] = 0.f;
+            const int jmax = min(32, npair - 32 * u);   // pairs 32 u + 1 .. 32 u + jmax
+            for (int src = 0; src < jmax; ++src) {
+                const int kc = 2 * (32 * u + src) + 1;
+                float vc[RB], vs[RB];
+#pragma unroll
+                for (int rb = 0; rb < RB; ++rb) {
+                    vc[rb] = __shfl_sync(0xffffffffu, zc[rb][u], src);
+                    vs[rb] = __shfl_sync(0xffffffffu, zs[rb][u], src);
+                }
+                const float* mc = MT + kc * MSZ + lane;
+#pragma unroll
+                for (int v = 0; v < NE; ++v) {
+                    const float a = mc[32 * v], b = mc[MSZ + 32 * v];
+#pragma unroll
+                    for (int rb = 0; rb < RB; ++rb)
+                        l[rb][v] = fmaf(b, vs[rb], fmaf(a, vc[rb], l[rb][v]));
+                }
             }
         }
-        if (lane == 0) {
-            x[0] = z[0];
-            x[MSZ - 1] = 0.f;
+        // softmax over the m active slots
+#pragma unroll
+        for (int rb = 0; rb < RB; ++rb) {
+            float mx = -INFINITY;
+#pragma unroll
+            for (int v = 0; v < NE; ++v) {
+                if (lane + 32 * v >= m) l[rb][v] = -INFINITY;
+                mx = fmaxf(mx, l[rb][v]);
+            }
+            mx = warp_max(mx);
+            float sum = 0.f;
+#pragma unroll
+            for (int v = 0; v < NE; ++v) {
+                l[rb][v] = expf(l[rb][v] - mx);
+                sum += l[rb][v];
+            }
+            const float inv = 1.f / warp_sum(sum);
+#pragma unroll
+            for (int v = 0; v < NE; ++v) l[rb][v] *= inv;
+        }
+        // y[col] = sum_{i < m} M[i][col] p[i], into the row (o' is consumed)
+        float y[RB][NE];
+#pragma unroll
+        for (int rb = 0; rb < RB; ++rb)
+#pragma unroll
+            for (int v = 0; v < NE; ++v) y[rb][v] = 0.f;
+#pragma unroll
+        for (int v2 = 0; v2 < NE; ++v2) {
+            const int imax = min(32, m - 32 * v2);
+            for (int src = 0; src < imax; ++src) {
+                float pv[RB];
+#pragma unroll
+                for (int rb = 0; rb < RB; ++rb) pv[rb] = __shfl_sync(0xffffffffu, l[rb][v2], src);
+                const float* mr = M + (32 * v2 + src) * MSZ + lane;
+#pragma unroll
+                for (int v = 0; v < NE; ++v) {
+                    const float a = mr[32 * v];
+#pragma unroll
+                    for (int rb = 0; rb < RB; ++rb) y[rb][v] = fmaf(a, pv[rb], y[rb][v]);
+                }
+            }
+        }
+        __syncwarp();
+#pragma unroll
+        for (int rb = 0; rb < RB; ++rb) {
+            float* x = sX + (r0 + rb) * LDM;
+#pragma unroll
+            for (int v = 0; v < NE; ++v) x[lane + 32 * v] = y[rb][v];   // padding entries are 0
+        }
+        __syncwarp();
+#pragma unroll
+        for (int rb = 0; rb < RB; ++rb) {   // o'' = U(-lam) y on the active pairs
+            float* x = sX + (r0 + rb) * LDM;
+#pragma unroll
+            for (int u = 0; u < NP; ++u) {
+                const int j = lane + 1 + 32 * u;
+                if (j <= npair) {
+                    const float yc = x[2 * j - 1], ys = x[2 * j];
+                    x[2 * j - 1] = cs[rb][u] * yc + sn[rb][u] * ys;
+                    x[2 * j] = -sn[rb][u] * yc + cs[rb][u] * ys;
+                }
+            }
         }
         __syncwarp();
     }
