@@ -6,8 +6,6 @@
 
 namespace cyfa {
 
-constexpr int LD = 129;   // padded row stride of [C][128] shared tiles
-
 // ---------------------------------------------------------------------------------------
 // Token-wise middle readout for rows r < C of sX (row stride MSZ + 1, in place):
 // o'' = U(-lam) M^T softmax(M U(lam) o') with M = R Phi ([MSZ][MSZ], global); the padding
