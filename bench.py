@@ -293,15 +293,15 @@ def run_ours(args):
     dq, dk, dv = torch.empty_like(inp['q']), torch.empty_like(inp['k']), torch.empty_like(inp['v'])
     dc, dd, db = torch.empty_like(lam), torch.empty_like(lam), torch.empty_like(lam)
     dA = torch.empty(H, **f32)
-    # the readout's gradient (the tensor-core kernels give it; a training step needs it)
-    dR = (torch.empty(H, 127, 127, **f32)
-          if cyfa.cyfa_saved_size(d) > 0 and not args.no_dR else None)
+    # the readout's gradient (a training step needs it)
+    dR = None if args.no_dR else torch.empty(H, 127, 127, **f32)
     ws_p = cyfa.workspace(d, cyfa.CYFA_WS_PREPARE, dev)
     ws_f = cyfa.workspace(d, cyfa.CYFA_WS_FWD, dev)
     ws_b = cyfa.workspace(d, cyfa.CYFA_WS_BWD, dev)
     # the forward saves its chunk-start states for the backward (a training step keeps them)
     saved = None if args.no_saved else cyfa.saved_buffer(d, dev)
-    tc_path = cyfa.cyfa_saved_size(d) > 0
+    # the library's rule for the tensor-core kernels (bf16 inputs, m = 127 here)
+    tc_path = not args.cuda_cores and D == 128 and T % 128 == 0
     stream = torch.cuda.current_stream()
 
     def step(x):
@@ -548,18 +548,20 @@ def run_extra_shape(args, dev, rank, peaks, B, T, H, D, m, what):
     dA, dR = torch.empty(H, **f32), torch.empty(H, m, m, **f32)
     ws = [cyfa.workspace(d, w, dev) for w in (cyfa.CYFA_WS_PREPARE, cyfa.CYFA_WS_FWD,
                                                cyfa.CYFA_WS_BWD)]
+    # the forward keeps its chunk-start states for the backward where the kernels can
+    saved = None if args.no_saved else cyfa.saved_buffer(d, dev)
 
     def fwd():
         cyfa.cyfa_prepare(d, inp['clock_logit'], inp['decay_logit'], inp['beta_logit'], inp['A'],
                           None, lam, g, beta, None, ws[0])
         cyfa.cyfa_chunk_fwd(d, inp['q'], inp['k'], inp['v'], lam, g, beta, inp['R'], None, None,
-                            o, None, None, ws[1])
+                            o, None, None, ws[1], saved=saved)
 
     def step():
         fwd()
         cyfa.cyfa_chunk_bwd(d, inp['q'], inp['k'], inp['v'], lam, g, beta, inp['R'],
                             inp['clock_logit'], inp['decay_logit'], inp['A'], inp['dO'], dq, dk,
-                            dv, dc, dd, db, dR, dA, ws[2])
+                            dv, dc, dd, db, dR, dA, ws[2], saved=saved)
 
     def timed(fn, n):
         for _ in range(3):
@@ -588,7 +590,8 @@ def run_extra_shape(args, dev, rank, peaks, B, T, H, D, m, what):
     cyfa.cyfa_check()
     th = B * T * H
     fl = operator_flops_per_token_head(C, d=D, ms=m + 1) * th
-    tc = cyfa.cyfa_saved_size(d) > 0
+    # the library's rule for the tensor-core kernels (bf16 inputs here)
+    tc = D == 128 and 63 <= m <= 127 and T % 128 == 0
     peak = peaks['bf16'] if tc else fp32_alu_peak_tflops(peaks['sm_max_mhz'])
     tf = 3 * fl / (ms / 1e3) / 1e12
     return {'workload': 'B=%d T=%d H=%d d=%d m=%d chunk %d (%s), prepare + fwd + bwd with every '
@@ -600,7 +603,8 @@ def run_extra_shape(args, dev, rank, peaks, B, T, H, D, m, what):
             'fwd_ms': ms_fwd, 'fwd_tokens_per_s': B * T / (ms_fwd / 1e3),
             'tflops_rule': tf, 'peak_tflops': peak,
             'peak_source': 'measured bf16 burst' if tc else 'fp32 FMA: 152 x 128 x 2 x clock',
-            'frac_peak': tf / peak, 'kernel_ms_per_step': split}
+            'frac_peak': tf / peak, 'saved_states': saved is not None,
+            'kernel_ms_per_step': split}
 
 
 def run_mixer(args, dev, rank, peaks):

@@ -942,7 +942,7 @@ cudaError_t bwd_dispatch(const BwdArgs& a, cudaStream_t st) {
     f.g = a.g;
     f.beta = a.beta;
     f.states = a.states;
-    cudaError_t e = launch_state_simt(f, st);
+    cudaError_t e = a.states_given ? cudaSuccess : launch_state_simt(f, st);
     if (e != cudaSuccess) return e;
     const dim3 gchunk(s.nchunk(), s.B * s.H);
     constexpr int SSZ = staging_floats<D, MSZ>();

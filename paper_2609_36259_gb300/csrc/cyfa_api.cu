@@ -205,12 +205,26 @@ int cyfa_workspace_size(const cyfa_dims_t* dims, int which, size_t* bytes) {
 // fp16 chunk-start states [B*H][T/128][2][128][128] of the tensor-core path
 size_t saved_bytes(const Shape& s) { return (size_t)s.B * s.H * (s.T / 128) * 2 * 128 * 128 * 2; }
 
+// The CUDA-core backward can read the forward's fp32 chunk-start states where both walk the same
+// chunks (128 storage rows, and a forward of 64-token chunks: caller chunk 64, or d = 256).
+bool simt_saved_ok(const Shape& s) {
+    return s.sl.ms == 128 && simt_fwd_shape(s).C == bwd_chunk(s.sl);
+}
+// fp32 chunk-start blocks [B*H][T/64][128][2d] of the CUDA-core path
+size_t saved_bytes_simt(const Shape& s) {
+    return (size_t)s.B * s.H * (s.T / BWD_C) * 128 * 2 * s.D * sizeof(float);
+}
+size_t saved_size_of(const cyfa_dims_t* d, const Shape& s) {
+    if (use_tc(d, s)) return saved_bytes(s);
+    return simt_saved_ok(s) ? saved_bytes_simt(s) : 0;
+}
+
 int cyfa_saved_size(const cyfa_dims_t* dims, size_t* bytes) {
     if (!bytes) return CYFA_ERR_ARG;
     const int rc = check_dims(dims, true);
     if (rc) return rc;
     const Shape s = shape_of(dims);
-    *bytes = use_tc(dims, s) ? saved_bytes(s) : 0;
+    *bytes = saved_size_of(dims, s);
     return CYFA_OK;
 }
 
@@ -347,7 +361,8 @@ int cyfa_chunk_fwd(const cyfa_dims_t* dims, const void* q, const void* k, const 
     a.o = o;
     a.Kout = Kbar_out;
     a.Vout = Vbar_out;
-    a.states = L.states;
+    // the chunk-start states go to the caller's buffer when it keeps them for the backward
+    a.states = (saved && simt_saved_ok(s)) ? static_cast<float*>(saved) : L.states;
     return cuda_status(launch_fwd_simt(a, st));
 }
 
@@ -378,7 +393,7 @@ int cyfa_chunk_bwd(const cyfa_dims_t* dims, const void* q, const void* k, const 
     rc = cuda_status(tc_path ? launch_readout_f16(s.H, R, L.Mb, s.sl, st)
                              : launch_readout_matrix(s.H, R, L.M, L.MT, s.sl, st));
     if (rc) return rc;
-    BwdArgs a;
+    BwdArgs a{};
     a.s = s;
     a.s.C = bwd_chunk(s.sl);
     a.q = q;
@@ -400,7 +415,8 @@ int cyfa_chunk_bwd(const cyfa_dims_t* dims, const void* q, const void* k, const 
     a.d_decay = d_decay_logit;
     a.d_beta = d_beta_logit;
     a.dA = dA;
-    a.states = L.states;
+    a.states_given = !tc_path && saved && simt_saved_ok(s);
+    a.states = a.states_given ? static_cast<float*>(const_cast<void*>(saved)) : L.states;
     a.adj = L.adj;
     a.o2 = L.o2;
     a.do1 = L.do1;

@@ -121,6 +121,7 @@ struct BwdArgs {
     void *dq, *dk, *dv;
     float *d_clock, *d_decay, *d_beta, *dA;
     float* states;      // [B*H][nchunk][ms][2D] chunk-start states
+    bool states_given;  // states holds the forward's saved states: the state pass is skipped
     float* adj;         // [B*H][nchunk][ms][2D] adjoints of the chunk-end states
     float* o2;          // [B*H][T][ms] o'' per token
     float* do1;         // [B*H][T][ms] dL/do' per token

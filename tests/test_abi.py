@@ -88,18 +88,22 @@ def test_null_and_misaligned_pointers_rejected_on_host(lib):
 
 
 def test_saved_size(lib):
-    """The saved chunk-start states: fp16 [B*H][T/128][2][128][128] on the tensor-core path,
-    nothing on the CUDA-core kernels (which also take d = 256)."""
+    """The saved chunk-start states: fp16 [B*H][T/128][2][128][128] on the tensor-core path;
+    fp32 [B*H][T/64][128][2d] on the CUDA-core kernels where their forward walks 64-token chunks
+    with 128 storage rows (the backward's chunks); nothing otherwise."""
     B, T, H = 2, 1024, 3
     full = B * H * (T // 128) * 2 * 128 * 128 * 2
+    simt = lambda d: B * H * (T // 64) * 128 * 2 * d * 4
     assert cyfa.cyfa_saved_size(cyfa.dims(B, T, H, 128)) == full
     assert cyfa.cyfa_saved_size(cyfa.dims(B, T, H, 128, m=63)) == full   # odd m in 63..127
-    assert cyfa.cyfa_saved_size(cyfa.dims(B, T, H, 128, m=31)) == 0
+    assert cyfa.cyfa_saved_size(cyfa.dims(B, T, H, 128, m=31)) == simt(128)
     assert cyfa.cyfa_saved_size(cyfa.dims(B, T, H, 128, m=255)) == 0   # 256 storage rows
-    assert cyfa.cyfa_saved_size(cyfa.dims(B, T, H, 256)) == 0
-    assert cyfa.cyfa_saved_size(cyfa.dims(B, T, H, 128, cuda_cores=True)) == 0
-    assert cyfa.cyfa_saved_size(cyfa.dims(B, T, H, 64)) == 0
-    assert cyfa.cyfa_saved_size(cyfa.dims(B, T, H, 128, dtype=torch.float32)) == 0
+    assert cyfa.cyfa_saved_size(cyfa.dims(B, T, H, 256)) == simt(256)
+    assert cyfa.cyfa_saved_size(cyfa.dims(B, T, H, 256, chunk=128)) == simt(256)   # walks 64
+    assert cyfa.cyfa_saved_size(cyfa.dims(B, T, H, 128, cuda_cores=True)) == simt(128)
+    assert cyfa.cyfa_saved_size(cyfa.dims(B, T, H, 128, chunk=128, cuda_cores=True)) == 0
+    assert cyfa.cyfa_saved_size(cyfa.dims(B, T, H, 64)) == simt(64)
+    assert cyfa.cyfa_saved_size(cyfa.dims(B, T, H, 128, dtype=torch.float32)) == simt(128)
 
 
 def test_timeout_selftest_rejects_bad_limits_on_host(lib):

@@ -131,6 +131,23 @@ def test_backward_saved_states(B, T, H):
     _compare(out, ref, pairs, assert_close_bf16, 'saved')
 
 
+@pytest.mark.parametrize('dtype,D,cuda_cores', [(torch.float32, 64, True),
+                                                (torch.bfloat16, 256, False),
+                                                (torch.bfloat16, 128, True)])
+def test_backward_saved_states_cuda_cores(dtype, D, cuda_cores):
+    """The CUDA-core backward reading the forward's fp32 chunk-start states (64-token chunks)
+    gives bit-identical gradients to the one that recomputes them (the same state pass computes
+    them either way)."""
+    B, T, H = 2, 512, 2
+    inp = to_device(synth.make_inputs(B, T, H, D, seed=13, dtype=dtype, with_dO=True))
+    d = cyfa.dims(B, T, H, D, chunk=64, dtype=dtype, cuda_cores=cuda_cores)
+    assert cyfa.cyfa_saved_size(d) == B * H * (T // 64) * 128 * 2 * D * 4
+    got = gpu_backward(d, inp, use_saved=True, want_dR=True)
+    want = gpu_backward(d, inp, want_dR=True)
+    for k, t in want.items():
+        assert torch.equal(got[k], t), k
+
+
 def test_backward_saved_full_size_sampled():
     """The 1.4B-shaped layer (B2 H16 T32768) with saved states, as the bench step runs it."""
     B, T, H = 2, 32768, 16

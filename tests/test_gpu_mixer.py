@@ -133,10 +133,12 @@ def test_mixer_full_size():
         assert rl <= 5e-3, (nm, rl)
 
 
-def test_autograd_operator_matches_c_abi_and_oracle():
-    """CyfaFunction's gradients (through autograd) against the oracle."""
+@pytest.mark.parametrize('m', [127, 63, 255])
+def test_autograd_operator_matches_c_abi_and_oracle(m):
+    """CyfaFunction's gradients (through autograd) against the oracle; m = 127 and 63 run the
+    tensor-core kernels (with saved states), m = 255 the CUDA-core kernels in 256 storage rows."""
     B, T, H, D = 1, 256, 2, 128
-    inp = to_device(synth.make_inputs(B, T, H, D, seed=54, with_dO=True))
+    inp = to_device(synth.make_inputs(B, T, H, D, seed=54, with_dO=True, m=m))
     leaves = {k: inp[k].clone().float().requires_grad_(True) if k in (
         'clock_logit', 'decay_logit', 'beta_logit', 'A', 'R') else inp[k].clone().requires_grad_(True)
         for k in ('q', 'k', 'v', 'clock_logit', 'decay_logit', 'beta_logit', 'A', 'R')}
@@ -150,6 +152,7 @@ def test_autograd_operator_matches_c_abi_and_oracle():
     for key, rk in (('q', 'dq'), ('k', 'dk'), ('v', 'dv'), ('clock_logit', 'd_clock'),
                     ('decay_logit', 'd_decay'), ('beta_logit', 'd_beta')):
         assert_close_bf16(pairs_np(leaves[key].grad.float(), pairs), ref[rk], 'autograd ' + key)
+    assert leaves['R'].grad.shape == (H, m, m)
     assert_close_rel(_np(leaves['R'].grad), ref['dR'], 'autograd dR')
 
 
