@@ -89,7 +89,7 @@ __global__ void __launch_bounds__(256) fwd_state_kernel(FwdArgs a) {
             for (int j = 0; j < 2; ++j) dst[(rz + ty + 16 * i) * W + col0 + tx + 16 * j] = S[i][j];
         const int t0 = c * C;
         load_gates(s, a.lam, a.g, a.beta, b, h, t0, C, slam, sg, sbeta);
-        stage_tok(sX, X, s, b, h, t0, C, xc0, 1.f);
+        stage_tok<C>(sX, X, s, b, h, t0, xc0, 1.f);
         __syncthreads();
         const float gC = sg[C - 1];
         build_write_rows(sA, LDM, slam, sbeta, C, s.sl, [&](int r) { return expf(gC - sg[r]); });
@@ -146,8 +146,8 @@ __global__ void __launch_bounds__(256) fwd_out_kernel(FwdArgs a) {
     zero_acc(acc);
     for (int d0 = 0; d0 < D; d0 += 32) {
         __syncthreads();
-        stage_tok(sX, Q, s, b, h, t0, C, d0, 1.f);
-        stage_tok(sX + C * 33, K, s, b, h, t0, C, d0, 1.f);
+        stage_tok<C>(sX, Q, s, b, h, t0, d0, 1.f);
+        stage_tok<C>(sX + C * 33, K, s, b, h, t0, d0, 1.f);
         __syncthreads();
         simt_mm<TM, TM>(acc, 32, [&](int r, int kk) { return sX[r * 33 + kk]; },
                         [&](int kk, int t) { return sX[C * 33 + t * 33 + kk]; });
@@ -167,11 +167,10 @@ __global__ void __launch_bounds__(256) fwd_out_kernel(FwdArgs a) {
     zero_acc(o1);
     for (int d0 = 0; d0 < D; d0 += 32) {
         __syncthreads();
-        stage_tok(sX, Q, s, b, h, t0, C, d0, 1.f);
-        for (int e = threadIdx.x; e < MSZ * 32; e += blockDim.x) {
-            const int i = e >> 5, dd = e & 31;
-            sX[C * 33 + i * 33 + dd] = Sst[i * (2 * D) + d0 + dd];
-        }
+        stage_tok<C>(sX, Q, s, b, h, t0, d0, 1.f);
+        stage_elems<MSZ * 32 / SIMT_THREADS>(
+            MSZ * 32, [&](int e) { return Sst[(e >> 5) * (2 * D) + d0 + (e & 31)]; },
+            [&](int e, float x) { sX[C * 33 + (e >> 5) * 33 + (e & 31)] = x; });
         __syncthreads();
         simt_mm<TM, NJ>(o1, 32, [&](int r, int kk) { return sX[r * 33 + kk]; },
                         [&](int kk, int i) { return sX[C * 33 + i * 33 + kk]; });
@@ -213,10 +212,9 @@ __global__ void __launch_bounds__(256) fwd_out_kernel(FwdArgs a) {
     static_assert(32 * (D + 1) <= C * LDM, "V staging exceeds its tile");
     for (int i0 = 0; i0 < MSZ; i0 += 32) {
         __syncthreads();
-        for (int e = threadIdx.x; e < 32 * D; e += blockDim.x) {
-            const int ii = e / D, dd = e % D;
-            sV[ii * (D + 1) + dd] = Sst[(i0 + ii) * (2 * D) + D + dd];
-        }
+        stage_elems<32 * D / SIMT_THREADS>(
+            32 * D, [&](int e) { return Sst[(i0 + e / D) * (2 * D) + D + e % D]; },
+            [&](int e, float x) { sV[(e / D) * (D + 1) + e % D] = x; });
         __syncthreads();
         simt_mm<TM, TN>(o, 32, [&](int r, int ii) { return sX[r * LDM + i0 + ii]; },
                         [&](int ii, int dd) { return sV[ii * (D + 1) + dd]; });
@@ -227,10 +225,10 @@ __global__ void __launch_bounds__(256) fwd_out_kernel(FwdArgs a) {
         for (int j = 0; j < TN; ++j) o[i][j] *= seg[ty + 16 * i];
     for (int s0 = 0; s0 < C; s0 += 32) {
         __syncthreads();
-        for (int e = threadIdx.x; e < 32 * D; e += blockDim.x) {
-            const int ss = e / D, dd = e % D;
-            sV[ss * (D + 1) + dd] = ldf(V, (((size_t)b * s.T + t0 + s0 + ss) * s.H + h) * D + dd);
-        }
+        stage_elems<32 * D / SIMT_THREADS>(
+            32 * D,
+            [&](int e) { return ldf(V, (((size_t)b * s.T + t0 + s0 + e / D) * s.H + h) * D + e % D); },
+            [&](int e, float x) { sV[(e / D) * (D + 1) + e % D] = x; });
         __syncthreads();
         simt_mm<TM, TN>(o, 32, [&](int r, int ss) { return sP[r * LP + s0 + ss]; },
                         [&](int ss, int dd) { return sV[ss * (D + 1) + dd]; });

@@ -281,8 +281,8 @@ __device__ __forceinline__ void masked_scores_tok(float* sP, float* sS, const fl
     zero_acc(acc);
     for (int d0 = 0; d0 < s.D; d0 += 32) {
         __syncthreads();
-        stage_tok(sS, X, s, b, h, t0, CB, d0, 1.f);
-        stage_tok(sS + CB * 33, Y, s, b, h, t0, CB, d0, 1.f);
+        stage_tok<CB>(sS, X, s, b, h, t0, d0, 1.f);
+        stage_tok<CB>(sS + CB * 33, Y, s, b, h, t0, d0, 1.f);
         __syncthreads();
         simt_mm<TMB, TMB>(acc, 32, [&](int r, int kk) { return sS[r * 33 + kk]; },
                           [&](int kk, int t) { return sS[CB * 33 + t * 33 + kk]; });
@@ -305,11 +305,10 @@ __device__ __forceinline__ void tok_times_stateT(float (&acc)[Geo<MSZ>::TMB][Geo
     constexpr int CB = G::CB;
     for (int d0 = 0; d0 < s.D; d0 += 32) {
         __syncthreads();
-        stage_tok(sS, X, s, b, h, t0, CB, d0, 1.f);
-        for (int e = threadIdx.x; e < MSZ * 32; e += blockDim.x) {
-            const int i = e >> 5, dd = e & 31;
-            sS[CB * 33 + i * 33 + dd] = Sst[i * (2 * s.D) + coff + d0 + dd];
-        }
+        stage_tok<CB>(sS, X, s, b, h, t0, d0, 1.f);
+        stage_elems<MSZ * 32 / SIMT_THREADS>(
+            MSZ * 32, [&](int e) { return Sst[(e >> 5) * (2 * s.D) + coff + d0 + (e & 31)]; },
+            [&](int e, float x) { sS[CB * 33 + (e >> 5) * 33 + (e & 31)] = x; });
         __syncthreads();
         simt_mm<G::TMB, G::NJ>(acc, 32, [&](int r, int kk) { return sS[r * 33 + kk]; },
                                [&](int kk, int i) { return sS[CB * 33 + i * 33 + kk]; });
@@ -319,15 +318,14 @@ __device__ __forceinline__ void tok_times_stateT(float (&acc)[Geo<MSZ>::TMB][Geo
 // acc[r][dd] += sum_i Y(r, i) * Sst[i][coff + dd]  (Y rows in shared memory with stride MSZ + 1)
 template <int MSZ, int TN>
 __device__ __forceinline__ void rows_times_state(float (&acc)[Geo<MSZ>::TMB][TN], float* sS,
-                                                 const float* Y, const float* Sst, int coff,
-                                                 int D) {
+                                                 const float* Y, const float* Sst, int coff) {
     using G = Geo<MSZ>;
+    constexpr int D = 16 * TN;   // the head dimension
     for (int i0 = 0; i0 < MSZ; i0 += 32) {
         __syncthreads();
-        for (int e = threadIdx.x; e < 32 * D; e += blockDim.x) {
-            const int ii = e / D, dd = e % D;
-            sS[ii * (D + 1) + dd] = Sst[(i0 + ii) * (2 * D) + coff + dd];
-        }
+        stage_elems<32 * D / SIMT_THREADS>(
+            32 * D, [&](int e) { return Sst[(i0 + e / D) * (2 * D) + coff + e % D]; },
+            [&](int e, float x) { sS[(e / D) * (D + 1) + e % D] = x; });
         __syncthreads();
         simt_mm<G::TMB, TN>(acc, 32, [&](int r, int ii) { return Y[r * G::LDM + i0 + ii]; },
                             [&](int ii, int dd) { return sS[ii * (D + 1) + dd]; });
@@ -340,13 +338,15 @@ __device__ __forceinline__ void scores_times_tok(float (&acc)[Geo<MSZ>::TMB][TN]
                                                  const FP& fp, const TI* X, const Shape& s,
                                                  int b, int h, int t0, float mul) {
     using G = Geo<MSZ>;
-    const int D = s.D;
+    constexpr int D = 16 * TN;   // the head dimension (s.D)
     for (int s0 = 0; s0 < G::CB; s0 += 32) {
         __syncthreads();
-        for (int e = threadIdx.x; e < 32 * D; e += blockDim.x) {
-            const int ss = e / D, dd = e % D;
-            sS[ss * (D + 1) + dd] = mul * ldf(X, (((size_t)b * s.T + t0 + s0 + ss) * s.H + h) * D + dd);
-        }
+        stage_elems<32 * D / SIMT_THREADS>(
+            32 * D,
+            [&](int e) {
+                return mul * ldf(X, (((size_t)b * s.T + t0 + s0 + e / D) * s.H + h) * D + e % D);
+            },
+            [&](int e, float x) { sS[(e / D) * (D + 1) + e % D] = x; });
         __syncthreads();
         simt_mm<G::TMB, TN>(acc, 32, [&](int r, int ss) { return fp(r, s0 + ss); },
                             [&](int ss, int dd) { return sS[ss * (D + 1) + dd]; });
@@ -445,7 +445,7 @@ __global__ void __launch_bounds__(256) bwd_intra1_kernel(BwdArgs a) {
     {
         float dqa[TMB][TN];
         zero_acc(dqa);
-        rows_times_state<MSZ, TN>(dqa, sS, sD, Sst, 0, D);
+        rows_times_state<MSZ, TN>(dqa, sS, sD, Sst, 0);
 #pragma unroll
         for (int i = 0; i < TMB; ++i)
 #pragma unroll
@@ -456,12 +456,15 @@ __global__ void __launch_bounds__(256) bwd_intra1_kernel(BwdArgs a) {
 #pragma unroll
         for (int i = 0; i < TMB; ++i) {
             const int r = ty + 16 * i;
+            const size_t row = (((size_t)b * s.T + t0 + r) * s.H + h) * D + tx;
+            float qv[TN];   // the row's q, loaded before any store of dq
+#pragma unroll
+            for (int j = 0; j < TN; ++j) qv[j] = ldf(Q, row + 16 * j);
             float part = 0.f;
 #pragma unroll
             for (int j = 0; j < TN; ++j) {
-                const size_t idx = (((size_t)b * s.T + t0 + r) * s.H + h) * D + tx + 16 * j;
-                part += ldf(Q, idx) * dqa[i][j];             // <q, dq~ / s> * s = <q~, dq~>
-                stf(dQ, idx, s.scale * dqa[i][j]);
+                part += qv[j] * dqa[i][j];             // <q, dq~ / s> * s = <q~, dq~>
+                stf(dQ, row + 16 * j, s.scale * dqa[i][j]);
             }
             part = half_warp_sum(part) * s.scale;
             if (tx == 0) sdG[r] += part;
@@ -520,13 +523,12 @@ __global__ void __launch_bounds__(256) adj_state_kernel(BwdArgs a) {
         const float gb = g_base(s, a.g, b, h, t0, CB);
         for (int r = threadIdx.x; r < CB; r += blockDim.x)
             sg[r] = a.g[((size_t)b * s.T + t0 + r) * s.H + h] - gb;
-        stage_tok(sX, X, s, b, h, t0, CB, xc0, xmul);
+        stage_tok<CB>(sX, X, s, b, h, t0, xc0, xmul);
         __syncthreads();
         const float* Yc = Y + ((size_t)bh * s.T + t0) * MSZ;
-        for (int e = threadIdx.x; e < CB * MSZ; e += blockDim.x) {
-            const int r = e / MSZ, i = e % MSZ;
-            sY[r * LDM + i] = Yc[e] * expf(sg[r]);
-        }
+        stage_elems<CB * MSZ / SIMT_THREADS>(
+            CB * MSZ, [&](int e) { return Yc[e] * expf(sg[e / MSZ]); },
+            [&](int e, float x) { sY[(e / MSZ) * LDM + e % MSZ] = x; });
         __syncthreads();
         const float decay = expf(sg[CB - 1]);
 #pragma unroll
@@ -570,11 +572,12 @@ __global__ void __launch_bounds__(256) bwd_intra2_kernel(BwdArgs a) {
     {
         const float* y1 = a.do1 + ((size_t)bh * s.T + t0) * MSZ;
         const float* y2 = a.o2 + ((size_t)bh * s.T + t0) * MSZ;
-        for (int e = threadIdx.x; e < CB * MSZ; e += blockDim.x) {
-            const int r = e / MSZ, i = e % MSZ;
-            sY1[r * LDM + i] = y1[e];
-            sY2[r * LDM + i] = y2[e];
-        }
+        stage_elems<CB * MSZ / SIMT_THREADS>(
+            CB * MSZ, [&](int e) { return y1[e]; },
+            [&](int e, float x) { sY1[(e / MSZ) * LDM + e % MSZ] = x; });
+        stage_elems<CB * MSZ / SIMT_THREADS>(
+            CB * MSZ, [&](int e) { return y2[e]; },
+            [&](int e, float x) { sY2[(e / MSZ) * LDM + e % MSZ] = x; });
     }
     __syncthreads();
     for (int r = threadIdx.x; r < CB; r += blockDim.x) {
@@ -590,7 +593,7 @@ __global__ void __launch_bounds__(256) bwd_intra2_kernel(BwdArgs a) {
     {
         float acc[TMB][TN];
         zero_acc(acc);
-        rows_times_state<MSZ, TN>(acc, sS, sA, Dst, 0, D);
+        rows_times_state<MSZ, TN>(acc, sS, sA, Dst, 0);
 #pragma unroll
         for (int i = 0; i < TMB; ++i)
 #pragma unroll
@@ -601,12 +604,15 @@ __global__ void __launch_bounds__(256) bwd_intra2_kernel(BwdArgs a) {
 #pragma unroll
         for (int i = 0; i < TMB; ++i) {
             const int t = ty + 16 * i;
+            const size_t row = (tokbase + (size_t)t * s.H) * D + tx;
+            float kv[TN];   // the row's k, loaded before any store of dk
+#pragma unroll
+            for (int j = 0; j < TN; ++j) kv[j] = ldf(K, row + 16 * j);
             float part = 0.f;
 #pragma unroll
             for (int j = 0; j < TN; ++j) {
-                const size_t idx = ((tokbase + (size_t)t * s.H)) * D + tx + 16 * j;
-                part += ldf(K, idx) * acc[i][j];
-                stf(dK, idx, acc[i][j]);
+                part += kv[j] * acc[i][j];
+                stf(dK, row + 16 * j, acc[i][j]);
             }
             part = half_warp_sum(part);
             if (tx == 0) sdG[t] -= part;
@@ -619,7 +625,7 @@ __global__ void __launch_bounds__(256) bwd_intra2_kernel(BwdArgs a) {
     {
         float acc[TMB][TN];
         zero_acc(acc);
-        rows_times_state<MSZ, TN>(acc, sS, sA, Dst, D, D);
+        rows_times_state<MSZ, TN>(acc, sS, sA, Dst, D);
 #pragma unroll
         for (int i = 0; i < TMB; ++i)
 #pragma unroll

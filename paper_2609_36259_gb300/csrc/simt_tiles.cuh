@@ -157,14 +157,39 @@ __device__ __forceinline__ void load_gates(const Shape& s, const float* lam, con
     }
 }
 
-// Stage rows [r0, r0+nr) x columns [c0, c0+32) of a [B,T,H,D] tensor into dst[r][33].
-template <typename TI>
-__device__ __forceinline__ void stage_tok(float* dst, const TI* X, const Shape& s, int b, int h,
-                                          int t0, int nr, int c0, float mul) {
-    for (int e = threadIdx.x; e < nr * 32; e += blockDim.x) {
-        const int r = e >> 5, cc = e & 31;
-        dst[r * 33 + cc] = mul * ldf(X, (((size_t)b * s.T + t0 + r) * s.H + h) * s.D + c0 + cc);
+// The chunk kernels run 256 threads per block.
+constexpr int SIMT_THREADS = 256;
+
+// Staging of `count` elements by the block: thread t moves e = t + 256 k (k < PER, e < count)
+// with ld(e) -> st(e, value).  Each thread issues all its loads before its first store, so its
+// global loads are in flight together (a load-store loop would wait out a full memory latency
+// per element: the compiler cannot move a load past a store that may alias it).
+template <int PER, class Ld, class St>
+__device__ __forceinline__ void stage_elems(int count, const Ld& ld, const St& st) {
+    float v[PER];
+#pragma unroll
+    for (int k = 0; k < PER; ++k) {
+        const int e = threadIdx.x + SIMT_THREADS * k;
+        v[k] = e < count ? ld(e) : 0.f;
     }
+#pragma unroll
+    for (int k = 0; k < PER; ++k) {
+        const int e = threadIdx.x + SIMT_THREADS * k;
+        if (e < count) st(e, v[k]);
+    }
+}
+
+// Stage rows [t0, t0+NR) x columns [c0, c0+32) of a [B,T,H,D] tensor into dst[r][33].
+template <int NR, typename TI>
+__device__ __forceinline__ void stage_tok(float* dst, const TI* X, const Shape& s, int b, int h,
+                                          int t0, int c0, float mul) {
+    static_assert(NR * 32 % SIMT_THREADS == 0, "rows x 32 columns in whole passes of the block");
+    stage_elems<NR * 32 / SIMT_THREADS>(
+        NR * 32,
+        [&](int e) {
+            return mul * ldf(X, (((size_t)b * s.T + t0 + (e >> 5)) * s.H + h) * s.D + c0 + (e & 31));
+        },
+        [&](int e, float x) { dst[(e >> 5) * 33 + (e & 31)] = x; });
 }
 
 }  // namespace cyfa
