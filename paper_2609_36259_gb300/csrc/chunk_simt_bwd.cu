@@ -71,6 +71,7 @@ __device__ __noinline__ void middle_rows_bwd(const float* sO1, const float* sO2,
                                              float* gp, float* gdy, float* gdl, const Slots& sl) {
     using G = Geo<MSZ>;
     constexpr int NP = G::NP, NE = G::NE, LDM = G::LDM;
+    constexpr int UNR = MSZ == 128 ? 4 : 1;   // slot steps whose M / M^T loads are in flight together
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int npair = sl.npair, m = sl.m;
     for (int r0 = warp * RB; r0 < C; r0 += 8 * RB) {
@@ -120,6 +121,7 @@ __device__ __noinline__ void middle_rows_bwd(const float* sO1, const float* sO2,
 #pragma unroll
         for (int u = 0; u < NP; ++u) {
             const int jmax = min(32, npair - 32 * u);   // pairs 32 u + 1 .. 32 u + jmax
+#pragma unroll UNR
             for (int src = 0; src < jmax; ++src) {
                 const int kc = 2 * (32 * u + src) + 1;
                 float vzc[RB], vzs[RB], vyc[RB], vys[RB];
@@ -205,6 +207,7 @@ __device__ __noinline__ void middle_rows_bwd(const float* sO1, const float* sO2,
 #pragma unroll
         for (int v2 = 0; v2 < NE; ++v2) {
             const int imax = min(32, m - 32 * v2);
+#pragma unroll UNR
             for (int src = 0; src < imax; ++src) {
                 float dv[RB];
 #pragma unroll

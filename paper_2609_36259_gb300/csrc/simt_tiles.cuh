@@ -19,6 +19,7 @@ template <int MSZ, int RB>
 static __device__ __noinline__ void middle_rows(float* sX, const float* slam, int C, const float* M,
                                                 const float* MT, const Slots& sl) {
     constexpr int LDM = MSZ + 1, NP = MSZ / 64, NE = MSZ / 32;
+    constexpr int UNR = MSZ == 128 ? 4 : 1;   // slot steps whose M / M^T loads are in flight together
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int npair = sl.npair, m = sl.m;
     for (int r0 = warp * RB; r0 < C; r0 += 8 * RB) {
@@ -53,6 +54,7 @@ static __device__ __noinline__ void middle_rows(float* sX, const float* slam, in
 #pragma unroll
         for (int u = 0; u < NP; ++u) {
             const int jmax = min(32, npair - 32 * u);   // pairs 32 u + 1 .. 32 u + jmax
+#pragma unroll UNR
             for (int src = 0; src < jmax; ++src) {
                 const int kc = 2 * (32 * u + src) + 1;
                 float vc[RB], vs[RB];
@@ -100,6 +102,7 @@ static __device__ __noinline__ void middle_rows(float* sX, const float* slam, in
 #pragma unroll
         for (int v2 = 0; v2 < NE; ++v2) {
             const int imax = min(32, m - 32 * v2);
+#pragma unroll UNR
             for (int src = 0; src < imax; ++src) {
                 float pv[RB];
 #pragma unroll
