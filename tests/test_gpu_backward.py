@@ -114,7 +114,7 @@ def test_backward_full_size_sampled(B, T, H, C, cuda_cores):
     inp = synth.make_inputs(B, T, H, 128, seed=0, device='cuda', with_dO=True)
     d = cyfa.dims(B, T, H, 128, chunk=C, cuda_cores=cuda_cores)
     out = gpu_backward(d, inp, want_dA=False)
-    pairs = sample_pairs(B, H, 2)
+    pairs = sample_pairs(B, H, 4)
     ref = oracle_backward(oracle_inputs(inp, pairs), pairs_np(inp['dO'], pairs))
     _compare(out, ref, pairs, assert_close_bf16, 'B%d T%d' % (B, T))
 
@@ -154,7 +154,7 @@ def test_backward_saved_full_size_sampled():
     inp = synth.make_inputs(B, T, H, 128, seed=1, device='cuda', with_dO=True)
     d = cyfa.dims(B, T, H, 128, chunk=64)
     out = gpu_backward(d, inp, want_dA=False, use_saved=True)
-    pairs = sample_pairs(B, H, 2)
+    pairs = sample_pairs(B, H, 4)
     ref = oracle_backward(oracle_inputs(inp, pairs), pairs_np(inp['dO'], pairs))
     _compare(out, ref, pairs, assert_close_bf16, 'saved full')
 
@@ -196,6 +196,6 @@ def test_backward_paper_kernel_shape_sampled():
     inp = synth.make_inputs(B, T, H, 256, seed=0, device='cuda', with_dO=True)
     d = cyfa.dims(B, T, H, 256, chunk=64)
     out = gpu_backward(d, inp, want_dA=False)
-    pairs = sample_pairs(B, H, 2)
+    pairs = sample_pairs(B, H, 3)
     ref = oracle_backward(oracle_inputs(inp, pairs), pairs_np(inp['dO'], pairs))
     _compare(out, ref, pairs, assert_close_bf16, 'paper shape')
