@@ -51,34 +51,34 @@ __global__ void __launch_bounds__(MS_MAX) readout_matrix_kernel(const float* R, 
 }
 
 // ---------------------------------------------------------------------------------------
-// Forward state pass: one block per (b, h, 32-column tile of [Kbar | Vbar], 128 of the MSZ
+// Forward state pass: one block per (b, h, 64-column tile of [Kbar | Vbar], 128 of the MSZ
 // storage rows); walks the chunks in order, writing the chunk-start state, then
 // Kbar <- gamma^C Kbar + A->^T K (and V), App. B Eq. app-cyfa-key-chunk / app-cyfa-value-chunk
 // (first lines).  The storage rows are independent in this recurrence.
 template <int C, int MSZ, typename TI>
 __global__ void __launch_bounds__(256) fwd_state_kernel(FwdArgs a) {
-    constexpr int LDM = MSZ + 1;
+    constexpr int LDM = MSZ + 1, NCOL = 64, NJ = NCOL / 16;
     const Shape s = a.s;
     const int D = s.D, W = 2 * s.D;
     const int bh = blockIdx.y, b = bh / s.H, h = bh % s.H;
-    const int col0 = blockIdx.x * 32;
+    const int col0 = blockIdx.x * NCOL;
     const int rz = 128 * blockIdx.z;   // first storage row of this block
     const bool isK = col0 < D;
     const TI* X = (const TI*)(isK ? a.k : a.v);
     const int xc0 = isK ? col0 : col0 - D;
     extern __shared__ float smem[];
     float* sA = smem;              // [C][LDM]
-    float* sX = sA + C * LDM;      // [C][33]
-    float* sg = sX + C * 33;
+    float* sX = sA + C * LDM;      // [C][NCOL + 1]
+    float* sg = sX + C * (NCOL + 1);
     float* slam = sg + C;
     float* sbeta = slam + C;
     const int tx = threadIdx.x & 15, ty = threadIdx.x >> 4;
-    float S[8][2];
+    float S[8][NJ];
     const float* S0 = isK ? a.Kbar0 : a.Vbar0;
 #pragma unroll
     for (int i = 0; i < 8; ++i)
 #pragma unroll
-        for (int j = 0; j < 2; ++j)
+        for (int j = 0; j < NJ; ++j)
             S[i][j] = S0 ? S0[((size_t)bh * MSZ + rz + ty + 16 * i) * D + xc0 + tx + 16 * j] : 0.f;
     const int nchunk = s.nchunk();
     for (int c = 0; c < nchunk; ++c) {
@@ -86,10 +86,10 @@ __global__ void __launch_bounds__(256) fwd_state_kernel(FwdArgs a) {
 #pragma unroll
         for (int i = 0; i < 8; ++i)
 #pragma unroll
-            for (int j = 0; j < 2; ++j) dst[(rz + ty + 16 * i) * W + col0 + tx + 16 * j] = S[i][j];
+            for (int j = 0; j < NJ; ++j) dst[(rz + ty + 16 * i) * W + col0 + tx + 16 * j] = S[i][j];
         const int t0 = c * C;
         load_gates(s, a.lam, a.g, a.beta, b, h, t0, C, slam, sg, sbeta);
-        stage_tok<C>(sX, X, s, b, h, t0, xc0, 1.f);
+        stage_tok<C, NCOL>(sX, X, s, b, h, t0, xc0, 1.f);
         __syncthreads();
         const float gC = sg[C - 1];
         build_write_rows(sA, LDM, slam, sbeta, C, s.sl, [&](int r) { return expf(gC - sg[r]); });
@@ -98,9 +98,9 @@ __global__ void __launch_bounds__(256) fwd_state_kernel(FwdArgs a) {
 #pragma unroll
         for (int i = 0; i < 8; ++i)
 #pragma unroll
-            for (int j = 0; j < 2; ++j) S[i][j] *= decay;
-        simt_mm<8, 2>(S, C, [&](int row, int t) { return sA[t * LDM + rz + row]; },
-                      [&](int t, int col) { return sX[t * 33 + col]; });
+            for (int j = 0; j < NJ; ++j) S[i][j] *= decay;
+        simt_mm<8, NJ>(S, C, [&](int row, int t) { return sA[t * LDM + rz + row]; },
+                       [&](int t, int col) { return sX[t * (NCOL + 1) + col]; });
         __syncthreads();
     }
     float* F = isK ? a.Kout : a.Vout;
@@ -108,7 +108,7 @@ __global__ void __launch_bounds__(256) fwd_state_kernel(FwdArgs a) {
 #pragma unroll
         for (int i = 0; i < 8; ++i)
 #pragma unroll
-            for (int j = 0; j < 2; ++j)
+            for (int j = 0; j < NJ; ++j)
                 F[((size_t)bh * MSZ + rz + ty + 16 * i) * D + xc0 + tx + 16 * j] = S[i][j];
     }
 }
@@ -246,10 +246,10 @@ __global__ void __launch_bounds__(256) fwd_out_kernel(FwdArgs a) {
 template <int C, int MSZ, typename TI>
 cudaError_t launch_state(const FwdArgs& a, const char* name, cudaStream_t st) {
     const Shape& s = a.s;
-    const size_t sm = (size_t)(C * (MSZ + 1) + C * 33 + 3 * C) * sizeof(float);
+    const size_t sm = (size_t)(C * (MSZ + 1) + C * 65 + 3 * C) * sizeof(float);
     auto k = fwd_state_kernel<C, MSZ, TI>;
     cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
-    { LaunchScope ls_(name, st); k<<<dim3(2 * s.D / 32, s.B * s.H, MSZ / 128), 256, sm, st>>>(a); }
+    { LaunchScope ls_(name, st); k<<<dim3(2 * s.D / 64, s.B * s.H, MSZ / 128), 256, sm, st>>>(a); }
     return cudaGetLastError();
 }
 

@@ -490,17 +490,17 @@ __global__ void __launch_bounds__(256) bwd_intra1_kernel(BwdArgs a) {
     }
 }
 
-// Reverse scan of the state adjoints, one block per (b, h, 32-column tile of [D^K | D^V], 128
+// Reverse scan of the state adjoints, one block per (b, h, 64-column tile of [D^K | D^V], 128
 // of the MSZ storage rows).  Stores, for every chunk c, the adjoint of the state at the end of
 // chunk c.
 template <int MSZ, typename TI>
 __global__ void __launch_bounds__(256) adj_state_kernel(BwdArgs a) {
     using G = Geo<MSZ>;
-    constexpr int CB = G::CB, LDM = G::LDM;
+    constexpr int CB = G::CB, LDM = G::LDM, NCOL = 64, NJ = NCOL / 16;
     const Shape s = a.s;
     const int D = s.D, W = 2 * s.D;
     const int bh = blockIdx.y, b = bh / s.H, h = bh % s.H;
-    const int col0 = blockIdx.x * 32;
+    const int col0 = blockIdx.x * NCOL;
     const int rz = 128 * blockIdx.z;   // first storage row of this block
     const bool isK = col0 < D;
     const int xc0 = isK ? col0 : col0 - D;
@@ -509,10 +509,10 @@ __global__ void __launch_bounds__(256) adj_state_kernel(BwdArgs a) {
     const float xmul = isK ? s.scale : 1.f;
     extern __shared__ float smem[];
     float* sY = smem;            // [CB][LDM]
-    float* sX = sY + CB * LDM;   // [CB][33]
-    float* sg = sX + CB * 33;
+    float* sX = sY + CB * LDM;   // [CB][NCOL + 1]
+    float* sg = sX + CB * (NCOL + 1);
     const int tx = threadIdx.x & 15, ty = threadIdx.x >> 4;
-    float S[8][2];
+    float S[8][NJ];
     zero_acc(S);
     const int nchunk = s.nchunk();
     for (int c = nchunk - 1; c >= 0; --c) {
@@ -520,13 +520,13 @@ __global__ void __launch_bounds__(256) adj_state_kernel(BwdArgs a) {
 #pragma unroll
         for (int i = 0; i < 8; ++i)
 #pragma unroll
-            for (int j = 0; j < 2; ++j) dst[(rz + ty + 16 * i) * W + col0 + tx + 16 * j] = S[i][j];
+            for (int j = 0; j < NJ; ++j) dst[(rz + ty + 16 * i) * W + col0 + tx + 16 * j] = S[i][j];
         const int t0 = c * CB;
         __syncthreads();
         const float gb = g_base(s, a.g, b, h, t0, CB);
         for (int r = threadIdx.x; r < CB; r += blockDim.x)
             sg[r] = a.g[((size_t)b * s.T + t0 + r) * s.H + h] - gb;
-        stage_tok<CB>(sX, X, s, b, h, t0, xc0, xmul);
+        stage_tok<CB, NCOL>(sX, X, s, b, h, t0, xc0, xmul);
         __syncthreads();
         const float* Yc = Y + ((size_t)bh * s.T + t0) * MSZ;
         stage_elems<CB * MSZ / SIMT_THREADS>(
@@ -537,9 +537,9 @@ __global__ void __launch_bounds__(256) adj_state_kernel(BwdArgs a) {
 #pragma unroll
         for (int i = 0; i < 8; ++i)
 #pragma unroll
-            for (int j = 0; j < 2; ++j) S[i][j] *= decay;
-        simt_mm<8, 2>(S, CB, [&](int row, int t) { return sY[t * LDM + rz + row]; },
-                      [&](int t, int col) { return sX[t * 33 + col]; });
+            for (int j = 0; j < NJ; ++j) S[i][j] *= decay;
+        simt_mm<8, NJ>(S, CB, [&](int row, int t) { return sY[t * LDM + rz + row]; },
+                       [&](int t, int col) { return sX[t * (NCOL + 1) + col]; });
     }
 }
 
@@ -959,10 +959,10 @@ cudaError_t bwd_dispatch(const BwdArgs& a, cudaStream_t st) {
     auto k1 = bwd_intra1_kernel<D, MSZ, TI>;
     cudaFuncSetAttribute(k1, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm1);
     { LaunchScope ls_("bwd_intra1", st); k1<<<gchunk, 256, sm1, st>>>(a); }
-    const size_t sma = (size_t)(CB * LDM + CB * 33 + CB) * sizeof(float);
+    const size_t sma = (size_t)(CB * LDM + CB * 65 + CB) * sizeof(float);
     auto ka = adj_state_kernel<MSZ, TI>;
     cudaFuncSetAttribute(ka, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sma);
-    { LaunchScope ls_("bwd_adjoint", st); ka<<<dim3(2 * D / 32, s.B * s.H, MSZ / 128), 256, sma, st>>>(a); }
+    { LaunchScope ls_("bwd_adjoint", st); ka<<<dim3(2 * D / 64, s.B * s.H, MSZ / 128), 256, sma, st>>>(a); }
     const size_t sm2 = (size_t)(4 * CB * LDM + SSZ + CB * G::LPB + 5 * CB) * sizeof(float);
     auto k2 = bwd_intra2_kernel<D, MSZ, TI>;
     cudaFuncSetAttribute(k2, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm2);

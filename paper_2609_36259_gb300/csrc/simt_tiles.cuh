@@ -182,17 +182,17 @@ __device__ __forceinline__ void stage_elems(int count, const Ld& ld, const St& s
     }
 }
 
-// Stage rows [t0, t0+NR) x columns [c0, c0+32) of a [B,T,H,D] tensor into dst[r][33].
-template <int NR, typename TI>
+// Stage rows [t0, t0+NR) x columns [c0, c0+NC) of a [B,T,H,D] tensor into dst[r][NC + 1].
+template <int NR, int NC = 32, typename TI>
 __device__ __forceinline__ void stage_tok(float* dst, const TI* X, const Shape& s, int b, int h,
                                           int t0, int c0, float mul) {
-    static_assert(NR * 32 % SIMT_THREADS == 0, "rows x 32 columns in whole passes of the block");
-    stage_elems<NR * 32 / SIMT_THREADS>(
-        NR * 32,
+    static_assert(NR * NC % SIMT_THREADS == 0, "rows x columns in whole passes of the block");
+    stage_elems<NR * NC / SIMT_THREADS>(
+        NR * NC,
         [&](int e) {
-            return mul * ldf(X, (((size_t)b * s.T + t0 + (e >> 5)) * s.H + h) * s.D + c0 + (e & 31));
+            return mul * ldf(X, (((size_t)b * s.T + t0 + e / NC) * s.H + h) * s.D + c0 + e % NC);
         },
-        [&](int e, float x) { dst[(e >> 5) * 33 + (e & 31)] = x; });
+        [&](int e, float x) { dst[(e / NC) * (NC + 1) + e % NC] = x; });
 }
 
 }  // namespace cyfa
