@@ -59,7 +59,8 @@ enum {
     CYFA_ERR_WORKSPACE = -4,  /* workspace null or smaller than cyfa_workspace_size() */
     CYFA_ERR_CUDA = -5,       /* a CUDA runtime call or launch failed */
     CYFA_ERR_TIMEOUT = -6,    /* a bounded device-side wait expired (see cyfa_check) */
-    CYFA_ERR_UNSUPPORTED = -7,/* a valid request this build does not implement */
+    CYFA_ERR_UNSUPPORTED = -7,/* a valid request this build does not implement (no current
+                                 call returns it; kept so codes stay stable) */
     CYFA_ERR_RANGE = -8       /* a non-finite value reached a result (see cyfa_check) */
 };
 

@@ -142,7 +142,8 @@ constexpr int BWD_C = 64;       // chunk length used by the SIMT backward with 1
 constexpr int BWD_C256 = 32;    // ... and with 256 (the tiles of a 64-token chunk would not fit)
 inline int bwd_chunk(const Slots& sl) { return sl.ms == 128 ? BWD_C : BWD_C256; }
 // Token ranges the CUDA-core dR reduction splits each head's B*T tokens into: about four blocks
-// per SM over the (ms / 64)^2 tiles and H heads, at least 256 tokens per range, at most 64.
+// per SM of the GB300's 152 over the (ms / 64)^2 tiles and H heads, at least 256 tokens per
+// range, at most 64.  A function of the shape alone, so the workspace size is fixed by the dims.
 inline int dm_splits(const Shape& s) {
     const long long tiles = (long long)(s.sl.ms / 64) * (s.sl.ms / 64) * s.H;
     long long n = (4 * 152 + tiles - 1) / tiles;
