@@ -441,8 +441,7 @@ __global__ void __launch_bounds__(512, 1) bwd_chunk1_tc(const __grid_constant__ 
         {   // do'' = gamma (dO Vbar^T) + P4 A, kept in X2
             float x[32], y[32];
             tmem_ld16x2_pair(tl + X2, x, tl + X3, y);
-    #pragma unroll
-            for (int i = 0; i < 32; ++i) x[i] = fmaf(gam, x[i], y[i]);
+            fma2_scalar(x, gam, y);
             tmem_st16x2(tl + X2, x);
             if (ok) ok = mbar_wait(&bars[1], ph);
             if (tid == 0 && ok) pend &= ~0x2u;
@@ -479,8 +478,7 @@ __global__ void __launch_bounds__(512, 1) bwd_chunk1_tc(const __grid_constant__ 
             float x[32], y[32];
             tmem_ld16x2_pair(tl + X3, x, tl + X4, y);
             const float f = scale * gam;
-    #pragma unroll
-            for (int i = 0; i < 32; ++i) x[i] = fmaf(f, x[i], y[i]);
+            fma2_scalar(x, f, y);
             rotate_q<1>(x, hf, u, lam, sl);
             store_q<__half>(T_S, row, c0, x);
             tmem_st16x2(tl + X3, x);
@@ -663,8 +661,7 @@ __global__ void __launch_bounds__(512, 1) bwd_chunk1_tc(const __grid_constant__ 
             float x[32], y[32];
             tmem_ld16x2_pair(tl + X3, x, tl + X4, y);
             const float f = scale * gam;
-    #pragma unroll
-            for (int i = 0; i < 32; ++i) x[i] = fmaf(f, x[i], y[i]);
+            fma2_scalar(x, f, y);
             load_q(T_L1, row, c0, y);
             s4 = dot32(y, x);
             // dq leaves through the staging tile (P3 is consumed) by a TMA store

@@ -43,7 +43,7 @@ __device__ __forceinline__ float cum128(const Shape& s, const float* g, int b, i
 // values carried in the Shape.
 template <class SL> __device__ __forceinline__ SL slots_of(const Shape& s);
 // m = 127: every rotation pair is active and slot 127 alone is padding (no masks to evaluate)
-template <class SL> constexpr bool full_slots() { return std::is_same<SL, Slots127>::value; }
+template <class SL> __host__ __device__ constexpr bool full_slots() { return std::is_same<SL, Slots127>::value; }
 template <> __device__ __forceinline__ Slots127 slots_of<Slots127>(const Shape&) { return {}; }
 template <> __device__ __forceinline__ Slots slots_of<Slots>(const Shape& s) { return s.sl; }
 
@@ -374,6 +374,17 @@ __device__ __forceinline__ bool slot_off(int c0, int i, const SL& sl) {
     return c0 + (i & 15) + 32 * (i >> 4) >= sl.m;
 }
 
+// x[i] = f x[i] + y[i] on 32 values, two per packed fp32 instruction (each lane rounds as fmaf).
+__device__ __forceinline__ void fma2_scalar(float (&x)[32], float f, const float (&y)[32]) {
+    const float2 f2 = make_float2(f, f);
+#pragma unroll
+    for (int i = 0; i < 32; i += 2) {
+        const float2 r = __ffma2_rn(f2, make_float2(x[i], x[i + 1]), make_float2(y[i], y[i + 1]));
+        x[i] = r.x;
+        x[i + 1] = r.y;
+    }
+}
+
 // Causal decay mask on the thread's 32 columns (tokens t = c0 + 32 blk + i of this chunk) of
 // row `row` (lane quarter q): x <- mul x 2^(g2 - g2_t) for t <= row, 0 otherwise, with g2 the
 // row's log2-domain cumulative decay and s_g2[t] the column's.  Each 16-token block is classed
@@ -396,14 +407,19 @@ __device__ __forceinline__ void mask_decay_q(float (&x)[32], float mul, int row,
             for (int i = 0; i < 16; ++i) xb[i] = 0.f;
         } else if (te < 32 * q) {
             const float ar = mul * ex2(g2 - s_g2[te]);
+            const float2 ar2 = make_float2(ar, ar);
             const float4* b4 = reinterpret_cast<const float4*>(s_b + tb);
 #pragma unroll
-            for (int k = 0; k < 4; ++k) {
+            for (int k = 0; k < 4; ++k) {   // x *= ar * b, two lanes per packed instruction
                 const float4 f = b4[k];
-                xb[4 * k + 0] *= ar * f.x;
-                xb[4 * k + 1] *= ar * f.y;
-                xb[4 * k + 2] *= ar * f.z;
-                xb[4 * k + 3] *= ar * f.w;
+                const float2 lo = __fmul2_rn(make_float2(xb[4 * k], xb[4 * k + 1]),
+                                             __fmul2_rn(ar2, make_float2(f.x, f.y)));
+                const float2 hi = __fmul2_rn(make_float2(xb[4 * k + 2], xb[4 * k + 3]),
+                                             __fmul2_rn(ar2, make_float2(f.z, f.w)));
+                xb[4 * k + 0] = lo.x;
+                xb[4 * k + 1] = lo.y;
+                xb[4 * k + 2] = hi.x;
+                xb[4 * k + 3] = hi.y;
             }
         } else {
             const float4* g4 = reinterpret_cast<const float4*>(s_g2 + tb);
