@@ -286,7 +286,9 @@ int cyfa_mixer_post_bwd(const cyfa_dims_t* dims, const void* o, const void* z, c
  * cyfa_check -- wait for `stream`, then report (and clear) the device error words that the
  * kernels set: CYFA_ERR_TIMEOUT when a bounded device-side wait gave up, else CYFA_ERR_ARG when
  * cyfa_prepare_varlen found invalid sequence offsets, else CYFA_ERR_RANGE when a non-finite
- * value reached an output of the tensor-core kernels, else CYFA_OK; CYFA_ERR_CUDA if the stream
+ * value reached an output of the tensor-core kernels, else CYFA_ERR_CUDA when a CUDA-core chunk
+ * kernel found its launch outside its shared-memory layout or block size (it then returned
+ * without touching memory: an internal error), else CYFA_OK; CYFA_ERR_CUDA also if the stream
  * itself reports an error.
  */
 int cyfa_check(void* stream);

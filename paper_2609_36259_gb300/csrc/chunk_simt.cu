@@ -72,6 +72,7 @@ __global__ void __launch_bounds__(256) fwd_state_kernel(FwdArgs a) {
     float* sg = sX + C * (NCOL + 1);
     float* slam = sg + C;
     float* sbeta = slam + C;
+    if (!launch_ok(smem, sbeta + C)) return;
     const int tx = threadIdx.x & 15, ty = threadIdx.x >> 4;
     float S[8][NJ];
     const float* S0 = isK ? a.Kbar0 : a.Vbar0;
@@ -130,6 +131,7 @@ __global__ void __launch_bounds__(256) fwd_out_kernel(FwdArgs a) {
     float* seg = sg + C;
     float* slam = seg + C;
     float* sbeta = slam + C;
+    if (!launch_ok(smem, sbeta + C)) return;
     const int tx = threadIdx.x & 15, ty = threadIdx.x >> 4;
     const float* Sst = a.states + ((size_t)bh * nchunk + c) * MSZ * (2 * D);
     const TI* Q = (const TI*)a.q;
@@ -266,6 +268,8 @@ cudaError_t fwd_dispatch(const FwdArgs& a, cudaStream_t st) {
 }
 
 }  // namespace
+
+cudaError_t simt_fwd_read_error(cudaStream_t st, int* err) { return read_simt_error(st, err); }
 
 cudaError_t launch_readout_matrix(int H, const float* R, float* M, float* MT, const Slots& sl,
                                   cudaStream_t st) {

@@ -378,6 +378,7 @@ __global__ void __launch_bounds__(256) bwd_intra1_kernel(BwdArgs a) {
     float* sbeta = slam + CB;
     float* sdG = sbeta + CB;
     float* sdL = sdG + CB;
+    if (!launch_ok(smem, sdL + CB)) return;
     const int tx = threadIdx.x & 15, ty = threadIdx.x >> 4;
     const float* Sst = a.states + ((size_t)bh * nchunk + c) * MSZ * (2 * D);
     const float* Mh = a.M + (size_t)h * MSZ * MSZ;
@@ -511,6 +512,7 @@ __global__ void __launch_bounds__(256) adj_state_kernel(BwdArgs a) {
     float* sY = smem;            // [CB][LDM]
     float* sX = sY + CB * LDM;   // [CB][NCOL + 1]
     float* sg = sX + CB * (NCOL + 1);
+    if (!launch_ok(smem, sg + CB)) return;
     const int tx = threadIdx.x & 15, ty = threadIdx.x >> 4;
     float S[8][NJ];
     zero_acc(S);
@@ -563,6 +565,7 @@ __global__ void __launch_bounds__(256) bwd_intra2_kernel(BwdArgs a) {
     float* slam = sfw + CB;
     float* sbeta = slam + CB;
     float* sdG = sbeta + CB;
+    if (!launch_ok(smem, sdG + CB)) return;
     const int tx = threadIdx.x & 15, ty = threadIdx.x >> 4;
     const float* Dst = a.adj + ((size_t)bh * nchunk + c) * MSZ * (2 * D);
     const TI* Q = (const TI*)a.q;
@@ -988,6 +991,8 @@ cudaError_t bwd_dispatch_d(const BwdArgs& a, cudaStream_t st) {
 }
 
 }  // namespace
+
+cudaError_t simt_bwd_read_error(cudaStream_t st, int* err) { return read_simt_error(st, err); }
 
 cudaError_t launch_bwd_gates(const BwdArgs& a, cudaStream_t st) {
     const Shape& s = a.s;

@@ -588,16 +588,19 @@ int cyfa_mixer_post_bwd(const cyfa_dims_t* dims, const void* o, const void* z, c
 int cyfa_check(void* stream) {
     cudaStream_t st = static_cast<cudaStream_t>(stream);
     if (cudaStreamSynchronize(st) != cudaSuccess) return CYFA_ERR_CUDA;
-    int err = 0, err2 = 0, err3 = 0;
+    int err = 0, err2 = 0, err3 = 0, err4 = 0, err5 = 0;
     if (tc_read_error(st, &err) != cudaSuccess) return CYFA_ERR_CUDA;
     if (tc_bwd_read_error(st, &err2) != cudaSuccess) return CYFA_ERR_CUDA;
     if (prep_read_error(st, &err3) != cudaSuccess) return CYFA_ERR_CUDA;
+    if (simt_fwd_read_error(st, &err4) != cudaSuccess) return CYFA_ERR_CUDA;
+    if (simt_bwd_read_error(st, &err5) != cudaSuccess) return CYFA_ERR_CUDA;
     // a timeout is reported first (its results are incomplete), then invalid sequence offsets
     // (every result after them is meaningless), then a range error (results inexact)
     if (err == CYFA_ERR_TIMEOUT || err2 == CYFA_ERR_TIMEOUT) return CYFA_ERR_TIMEOUT;
     if (err3 == CYFA_ERR_ARG) return CYFA_ERR_ARG;
     if (err == CYFA_ERR_RANGE || err2 == CYFA_ERR_RANGE) return CYFA_ERR_RANGE;
-    return (err || err2 || err3) ? CYFA_ERR_CUDA : CYFA_OK;
+    // otherwise any error word: a CUDA-core chunk kernel launched outside its layout (err4, err5)
+    return (err || err2 || err3 || err4 || err5) ? CYFA_ERR_CUDA : CYFA_OK;
 }
 
 }  // extern "C"

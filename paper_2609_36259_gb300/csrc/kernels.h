@@ -153,6 +153,10 @@ inline int dm_splits(const Shape& s) {
     return n < 1 ? 1 : (int)n;
 }
 cudaError_t launch_bwd_simt(const BwdArgs& a, cudaStream_t st);
+// Read (and clear) the launch-check error words of the CUDA-core chunk kernels (forward and
+// backward translation units); synchronise the stream.
+cudaError_t simt_fwd_read_error(cudaStream_t st, int* err);
+cudaError_t simt_bwd_read_error(cudaStream_t st, int* err);
 // reverse cumulative sums of the per-token scalars in a.tok and the logit gradients
 cudaError_t launch_bwd_gates(const BwdArgs& a, cudaStream_t st);
 

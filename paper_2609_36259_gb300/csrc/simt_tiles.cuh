@@ -1,10 +1,40 @@
 // Shared-memory tile helpers of the SIMT chunk kernels (forward and backward).
 #pragma once
 
+#include "../../include/cyfa.h"
 #include "common.cuh"
 #include "kernels.h"
 
 namespace cyfa {
+
+// The chunk kernels run 256 threads per block.
+constexpr int SIMT_THREADS = 256;
+
+// Launch check of the chunk kernels, at entry: the block has SIMT_THREADS threads (the staging
+// and the 16 x 16 thread tiles assume it) and the dynamic shared memory covers the kernel's
+// carve-up [smem, end).  A launch that does not fit records CYFA_ERR_CUDA in the translation
+// unit's error word (returned by cyfa_check) and every thread leaves before touching memory.
+static __device__ int g_simt_err;
+__device__ __forceinline__ bool launch_ok(const float* smem, const float* end) {
+    unsigned dyn;
+    asm volatile("mov.u32 %0, %%dynamic_smem_size;" : "=r"(dyn));
+    const bool ok = blockDim.x == SIMT_THREADS && blockDim.y == 1 && blockDim.z == 1 &&
+                    (size_t)(end - smem) * sizeof(float) <= (size_t)dyn;
+    if (!ok && threadIdx.x == 0) atomicExch(&g_simt_err, CYFA_ERR_CUDA);
+    return ok;
+}
+// Reads (and clears) this translation unit's error word; synchronises the stream.
+static inline cudaError_t read_simt_error(cudaStream_t st, int* err) {
+    cudaError_t e = cudaMemcpyFromSymbolAsync(err, g_simt_err, sizeof(int), 0,
+                                              cudaMemcpyDeviceToHost, st);
+    if (e != cudaSuccess) return e;
+    e = cudaStreamSynchronize(st);
+    if (e == cudaSuccess && *err) {
+        const int zero = 0;
+        e = cudaMemcpyToSymbol(g_simt_err, &zero, sizeof(int));
+    }
+    return e;
+}
 
 // ---------------------------------------------------------------------------------------
 // Token-wise middle readout for rows r < C of sX (row stride MSZ + 1, in place):
@@ -159,9 +189,6 @@ __device__ __forceinline__ void load_gates(const Shape& s, const float* lam, con
         sbeta[r] = beta[gi];
     }
 }
-
-// The chunk kernels run 256 threads per block.
-constexpr int SIMT_THREADS = 256;
 
 // Staging of `count` elements by the block: thread t moves e = t + 256 k (k < PER, e < count)
 // with ld(e) -> st(e, value).  Each thread issues all its loads before its first store, so its
