@@ -182,7 +182,8 @@ int cyfa_prepare_noalloc(const cyfa_dims_t* dims, const float* clock_logit,
  * cyfa_saved_size -- bytes of the forward intermediates that cyfa_chunk_fwd can save for
  * cyfa_chunk_bwd: the states [Kbar | Vbar] at the start of every chunk (App. B's
  * chunk-boundary states).  On the tensor-core kernels: every 128-token chunk, fp16,
- * [B*H][T/128][2][128][128] with the Fourier rows in the kernels' internal order.  On the
+ * [B*H][T/128][2][128][128] with the Fourier rows in the kernels' internal order, followed by
+ * the fp16 readout matrix M = R Phi [H][128][128] (the backward then does not recompute it).  On the
  * CUDA-core kernels with 128 storage rows and a forward walking 64-token chunks (chunk 64, or
  * d = 256): every 64-token chunk, fp32, [B*H][T/64][128][2d] in the paper's row order.  0
  * otherwise (nothing is saved).  No paper counterpart beyond those states: this is the usual

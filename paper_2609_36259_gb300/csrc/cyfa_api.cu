@@ -202,8 +202,17 @@ int cyfa_workspace_size(const cyfa_dims_t* dims, int which, size_t* bytes) {
     }
 }
 
-// fp16 chunk-start states [B*H][T/128][2][128][128] of the tensor-core path
-size_t saved_bytes(const Shape& s) { return (size_t)s.B * s.H * (s.T / 128) * 2 * 128 * 128 * 2; }
+// Tensor-core path: fp16 chunk-start states [B*H][T/128][2][128][128], then the fp16 readout
+// matrix M = R Phi [H][128][128] the forward computed (the backward reads it instead of
+// recomputing it).  The states' size is a multiple of 64 KiB, so M stays aligned.
+size_t saved_state_bytes(const Shape& s) {
+    return (size_t)s.B * s.H * (s.T / 128) * 2 * 128 * 128 * 2;
+}
+size_t saved_bytes(const Shape& s) { return saved_state_bytes(s) + (size_t)s.H * MS * MS * 2; }
+__half* saved_mb(const Shape& s, const void* saved) {
+    return reinterpret_cast<__half*>(static_cast<char*>(const_cast<void*>(saved)) +
+                                     saved_state_bytes(s));
+}
 
 // The CUDA-core backward can read the forward's fp32 chunk-start states where both walk the same
 // chunks (128 storage rows, and a forward of 64-token chunks: caller chunk 64, or d = 256).
@@ -325,7 +334,9 @@ int cyfa_chunk_fwd(const cyfa_dims_t* dims, const void* q, const void* k, const 
     if (!aligned16(workspace)) return CYFA_ERR_ALIGN;
     const FwdLayout L = fwd_layout(s, tc_path, workspace);
     cudaStream_t st = static_cast<cudaStream_t>(stream);
-    rc = cuda_status(tc_path ? launch_readout_f16(s.H, R, L.Mb, s.sl, st)
+    // with saved states on, M goes next to them for the backward
+    __half* Mb = (tc_path && saved) ? saved_mb(s, saved) : L.Mb;
+    rc = cuda_status(tc_path ? launch_readout_f16(s.H, R, Mb, s.sl, st)
                              : launch_readout_matrix(s.H, R, L.M, L.MT, s.sl, st));
     if (rc) return rc;
     if (tc_path) {
@@ -341,7 +352,7 @@ int cyfa_chunk_fwd(const cyfa_dims_t* dims, const void* q, const void* k, const 
         t.o = o;
         t.segS = L.segS;
         t.segG = L.segG;
-        t.Mb = L.Mb;
+        t.Mb = Mb;
         t.snap = static_cast<__half*>(saved);
         t.nseg = L.nseg;
         return cuda_status(launch_fwd_tc(t, q, k, v, st));
@@ -390,9 +401,13 @@ int cyfa_chunk_bwd(const cyfa_dims_t* dims, const void* q, const void* k, const 
     if (!aligned16(workspace)) return CYFA_ERR_ALIGN;
     const BwdLayout L = bwd_layout(s, tc_path, workspace);
     cudaStream_t st = static_cast<cudaStream_t>(stream);
-    rc = cuda_status(tc_path ? launch_readout_f16(s.H, R, L.Mb, s.sl, st)
-                             : launch_readout_matrix(s.H, R, L.M, L.MT, s.sl, st));
-    if (rc) return rc;
+    // the tensor-core path reads M from the saved buffer when the forward kept it there
+    __half* Mb = (tc_path && saved) ? saved_mb(s, saved) : L.Mb;
+    if (!(tc_path && saved)) {
+        rc = cuda_status(tc_path ? launch_readout_f16(s.H, R, Mb, s.sl, st)
+                                 : launch_readout_matrix(s.H, R, L.M, L.MT, s.sl, st));
+        if (rc) return rc;
+    }
     BwdArgs a{};
     a.s = s;
     a.s.C = bwd_chunk(s.sl);
@@ -437,7 +452,7 @@ int cyfa_chunk_bwd(const cyfa_dims_t* dims, const void* q, const void* k, const 
         f.beta = beta;
         f.segS = L.segS;
         f.segG = L.segG;
-        f.Mb = L.Mb;
+        f.Mb = Mb;
         f.snap = nullptr;
         f.nseg = L.nseg;
         TcBwdArgs t{};
@@ -454,7 +469,7 @@ int cyfa_chunk_bwd(const cyfa_dims_t* dims, const void* q, const void* k, const 
         t.snapA = L.snapA;
         t.O2 = L.O2b;
         t.DO1 = L.DO1b;
-        t.Mb = L.Mb;
+        t.Mb = Mb;
         t.q = q;
         t.k = k;
         t.dq = dq;

@@ -24,6 +24,11 @@ bool make_tmap_bf16(CUtensorMap* map, const void* base, int rank, const unsigned
             g_encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
     });
     if (!g_encode) return false;
+    // The encode is a driver call and needs the device's context current in this thread.  A
+    // thread whose first CUDA call this is (an autograd worker thread, say) has none yet:
+    // binding the runtime's current device makes its primary context current.
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || cudaSetDevice(dev) != cudaSuccess) return false;
     cuuint64_t gdim[5], gstr[4];
     cuuint32_t bdim[5], estr[5];
     for (int i = 0; i < rank; ++i) {

@@ -88,11 +88,11 @@ def test_null_and_misaligned_pointers_rejected_on_host(lib):
 
 
 def test_saved_size(lib):
-    """The saved chunk-start states: fp16 [B*H][T/128][2][128][128] on the tensor-core path;
-    fp32 [B*H][T/64][128][2d] on the CUDA-core kernels where their forward walks 64-token chunks
-    with 128 storage rows (the backward's chunks); nothing otherwise."""
+    """The saved chunk-start states: fp16 [B*H][T/128][2][128][128] and M [H][128][128] on the
+    tensor-core path; fp32 [B*H][T/64][128][2d] on the CUDA-core kernels where their forward
+    walks 64-token chunks with 128 storage rows (the backward's chunks); nothing otherwise."""
     B, T, H = 2, 1024, 3
-    full = B * H * (T // 128) * 2 * 128 * 128 * 2
+    full = B * H * (T // 128) * 2 * 128 * 128 * 2 + H * 128 * 128 * 2   # states, then M
     simt = lambda d: B * H * (T // 64) * 128 * 2 * d * 4
     assert cyfa.cyfa_saved_size(cyfa.dims(B, T, H, 128)) == full
     assert cyfa.cyfa_saved_size(cyfa.dims(B, T, H, 128, m=63)) == full   # odd m in 63..127

@@ -207,3 +207,50 @@ def test_backward_paper_kernel_shape_sampled():
     pairs = sample_pairs(B, H, 3)
     ref = oracle_backward(oracle_inputs(inp, pairs), pairs_np(inp['dO'], pairs))
     _compare(out, ref, pairs, assert_close_bf16, 'paper shape')
+
+
+def test_backward_from_fresh_thread():
+    """The backward called from a thread whose first CUDA work it is (as in an autograd worker
+    thread), reading the forward's saved states: it starts with tensor-map encodes, driver calls
+    that need the device's context current in that thread.  The gradients equal those of the
+    same call made from the main thread."""
+    import threading
+    B, T, H, D = 1, 256, 2, 128
+    inp = to_device(synth.make_inputs(B, T, H, D, seed=57, with_dO=True))
+    d = cyfa.dims(B, T, H, D, chunk=64)
+    lam, g, beta, _ = gpu_prepare(d, inp)
+    saved = cyfa.saved_buffer(d)
+    cyfa.forward(d, inp['q'], inp['k'], inp['v'], lam, g, beta, inp['R'], saved=saved)
+    st = torch.cuda.Stream()
+    ws = [cyfa.workspace(d, cyfa.CYFA_WS_BWD) for _ in range(2)]
+
+    def outputs():
+        return dict(dq=torch.empty_like(inp['q']), dk=torch.empty_like(inp['k']),
+                    dv=torch.empty_like(inp['v']), dc=torch.empty_like(lam),
+                    dd=torch.empty_like(lam), db=torch.empty_like(lam),
+                    dR=torch.empty_like(inp['R']), dA=torch.empty_like(inp['A']))
+    outs = [outputs(), outputs()]
+    torch.cuda.synchronize()
+
+    def bwd(i):
+        o = outs[i]
+        cyfa.cyfa_chunk_bwd(d, inp['q'], inp['k'], inp['v'], lam, g, beta, inp['R'],
+                            inp['clock_logit'], inp['decay_logit'], inp['A'], inp['dO'], o['dq'],
+                            o['dk'], o['dv'], o['dc'], o['dd'], o['db'], o['dR'], o['dA'], ws[i],
+                            stream=st, saved=saved)
+    errors = []
+
+    def worker():
+        try:
+            bwd(0)
+        except Exception as e:   # reported below, in the test's own thread
+            errors.append(e)
+    t = threading.Thread(target=worker)
+    t.start()
+    t.join()
+    assert not errors, errors
+    bwd(1)
+    st.synchronize()
+    cyfa.cyfa_check(st)
+    for k in outs[0]:
+        assert torch.equal(outs[0][k], outs[1][k]), k
