@@ -17,6 +17,9 @@
  *   o''_t    = U(-lambda_t) Phi^T R^T softmax(R Phi U(lambda_t) o'_t)
  *   o_t      = Vbar_t^T o''_t
  *
+ * Threads: any host thread may call; the calls use the runtime's current device of the calling
+ * thread (cudaSetDevice) and the caller's stream.
+ *
  * Storage conventions (all row-major, caller-owned; the library never allocates):
  *   q, k, dq, dk      [B, T, H, dk]   bf16 or fp32 (dims.dtype)
  *   v, o, dO, dv      [B, T, H, dv]   bf16 or fp32
