@@ -117,7 +117,7 @@ __global__ void __launch_bounds__(256) fwd_state_kernel(FwdArgs a) {
 // Forward outputs of one chunk (App. B, second lines of Eqs. app-cyfa-key-chunk and
 // app-cyfa-value-chunk, with the middle readout between them).
 template <int C, int D, int MSZ, typename TI>
-__global__ void __launch_bounds__(256) fwd_out_kernel(FwdArgs a) {
+__global__ void __launch_bounds__(256, (C == 64 && MSZ == 128) ? 2 : 1) fwd_out_kernel(FwdArgs a) {
     const Shape s = a.s;
     constexpr int LP = C + 1, TM = C / 16, LDM = MSZ + 1, NJ = MSZ / 16;
     const int c = blockIdx.x, bh = blockIdx.y, b = bh / s.H, h = bh % s.H;
@@ -131,7 +131,10 @@ __global__ void __launch_bounds__(256) fwd_out_kernel(FwdArgs a) {
     float* seg = sg + C;
     float* slam = seg + C;
     float* sbeta = slam + C;
-    if (!launch_ok(smem, sbeta + C)) return;
+    // staging of M^T / M for the middle readout: the score tile (free during the readout) when
+    // it is large enough, else its own region
+    float* sB = C * LP >= 32 * LDM ? sP : sbeta + C;
+    if (!launch_ok(smem, sbeta + C + (C * LP >= 32 * LDM ? 0 : 32 * LDM))) return;
     const int tx = threadIdx.x & 15, ty = threadIdx.x >> 4;
     const float* Sst = a.states + ((size_t)bh * nchunk + c) * MSZ * (2 * D);
     const TI* Q = (const TI*)a.q;
@@ -190,8 +193,8 @@ __global__ void __launch_bounds__(256) fwd_out_kernel(FwdArgs a) {
         for (int j = 0; j < NJ; ++j) sX[(ty + 16 * i) * LDM + tx + 16 * j] = o1[i][j];
     __syncthreads();
 
-    middle_rows<MSZ, 4>(sX, slam, C, a.M + (size_t)h * MSZ * MSZ, a.MT + (size_t)h * MSZ * MSZ,
-                        s.sl);
+    readout_rows_fwd<C, MSZ>(sX, sB, slam, a.M + (size_t)h * MSZ * MSZ,
+                             a.MT + (size_t)h * MSZ * MSZ, s.sl);
     __syncthreads();
 
     // P = (O'' A^T) o Gamma
@@ -260,7 +263,8 @@ cudaError_t fwd_dispatch(const FwdArgs& a, cudaStream_t st) {
     const Shape& s = a.s;
     cudaError_t e = launch_state<C, MSZ, TI>(a, "fwd_state", st);
     if (e != cudaSuccess) return e;
-    const size_t sm_out = (size_t)(2 * C * (MSZ + 1) + C * (C + 1) + 4 * C) * sizeof(float);
+    constexpr int SB_EXTRA = C * (C + 1) >= 32 * (MSZ + 1) ? 0 : 32 * (MSZ + 1);
+    const size_t sm_out = (size_t)(2 * C * (MSZ + 1) + C * (C + 1) + 4 * C + SB_EXTRA) * sizeof(float);
     auto kout = fwd_out_kernel<C, D, MSZ, TI>;
     cudaFuncSetAttribute(kout, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm_out);
     { LaunchScope ls_("fwd_out", st); kout<<<dim3(s.nchunk(), s.B * s.H), 256, sm_out, st>>>(a); }

@@ -28,7 +28,7 @@ template <int MSZ>
 struct Geo {
     static constexpr int CB = MSZ == 128 ? BWD_C : BWD_C256;
     static constexpr int LPB = CB + 1, TMB = CB / 16, LDM = MSZ + 1, NJ = MSZ / 16;
-    static constexpr int NP = MSZ / 64, NE = MSZ / 32, NPAIRS = MSZ / 2 - 1;
+    static constexpr int NP = MSZ / 64, NE = MSZ / 32;
 };
 // Floats of the staging tile: the larger of a [CB][MSZ + 1] tile, the Q / Kbar column staging
 // ((CB + MSZ) x 33) and the state-row staging (32 x (D + 1)).
@@ -57,199 +57,160 @@ __device__ __forceinline__ float warp_omega_dot(const float* x, const float* y, 
     return warp_sum(acc);
 }
 
-// Gradient of the middle readout: given o' (sO1), o'' (sO2) and dL/do'' (sD), writes dL/do' into
-// sD and the row scalars sdG[r] = <o'', do''> and sdL[r] = <dz, Omega z> - <do'', Omega o''>.
-// With gz non-null the row's z, p, dy, dl (for dR) go to gz / gp / gdy / gdl + MSZ r.  Rows have
-// stride MSZ + 1.  Each warp takes RB rows at a time, so that every entry of M and M^T it loads
-// serves RB rows; the vectors stay in registers (rotation pairs j = lane + 1 + 32 u, slot
-// entries lane + 32 v) and the products over slots broadcast the summed-over vector from its
-// owner lane by shuffles, in slot order.  C is a multiple of 8 RB.
-template <int MSZ, int RB>
-__device__ __noinline__ void middle_rows_bwd(const float* sO1, const float* sO2, float* sD,
-                                             const float* slam, int C, const float* M,
-                                             const float* MT, float* sdG, float* sdL, float* gz,
-                                             float* gp, float* gdy, float* gdl, const Slots& sl) {
+// The middle readout and its gradient for the CB rows of a chunk, as products of the row blocks
+// with M^T and M (global [MSZ][MSZ], zero beyond the m active rows and columns):
+//   z = U(lam) o',  dy = U(lam) do''             rows of sZ and sG, in place
+//   l = M z,  dp = M dy                          one pass over M^T
+//   p = softmax(l) over the m active slots,  dl = p o (dp - <p, dp>)
+//   y = M^T p,  dz = M^T dl                      one pass over M (p staged in sY, dl in sW)
+//   o'' = U(-lam) y into sY,  do' = U(-lam) dz into sG
+// with the row scalars sdG[r] = <o'', do''> = <y, dy> and
+// sdL[r] = <dz, Omega z> - <do'', Omega o''> = <dz, Omega z> - <dy, Omega y> (U is orthogonal
+// and commutes with Omega).  Entries beyond the m active ones are zero in every row.  With gz
+// non-null the rows of z, p, dy, dl (for dR) go to gz / gp / gdy / gdl + MSZ r.  sW is a
+// [CB][MSZ + 1] scratch tile and sB the [32][MSZ + 1] staging of M^T and M.  One block
+// barrier at entry (the caller's rows are complete); the results are complete after the
+// caller's next barrier.
+template <int MSZ>
+__device__ __noinline__ void readout_rows_bwd(float* sZ, float* sY, float* sG, float* sW, float* sB,
+                                              const float* slam, const float* M, const float* MT,
+                                              float* sdG, float* sdL, float* gz, float* gp,
+                                              float* gdy, float* gdl, const Slots& sl) {
     using G = Geo<MSZ>;
-    constexpr int NP = G::NP, NE = G::NE, LDM = G::LDM;
-    constexpr int UNR = MSZ == 128 ? 4 : 1;   // slot steps whose M / M^T loads are in flight together
+    constexpr int CB = G::CB, LDM = G::LDM, NP = G::NP, NE = G::NE, TMB = G::TMB, NJ = G::NJ;
+    constexpr int NW = SIMT_THREADS / 32;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int tx = threadIdx.x & 15, ty = threadIdx.x >> 4;
     const int npair = sl.npair, m = sl.m;
-    for (int r0 = warp * RB; r0 < C; r0 += 8 * RB) {
-        float cs[RB][NP], sn[RB][NP], zc[RB][NP], zs[RB][NP], yc[RB][NP], ys[RB][NP];
-        float z0[RB], y0[RB], g1[RB], om2[RB];
-#pragma unroll
-        for (int rb = 0; rb < RB; ++rb) {
-            const float* x1 = sO1 + (r0 + rb) * LDM;
-            const float* x2 = sO2 + (r0 + rb) * LDM;
-            const float* xd = sD + (r0 + rb) * LDM;
-            const float lam = slam[r0 + rb];
-            z0[rb] = x1[0];
-            y0[rb] = xd[0];
-#pragma unroll
-            for (int u = 0; u < NP; ++u) {
-                const int j = lane + 1 + 32 * u;
-                cs[rb][u] = 1.f;
-                sn[rb][u] = 0.f;
-                zc[rb][u] = zs[rb][u] = yc[rb][u] = ys[rb][u] = 0.f;
-                if (j <= npair) {   // z = U(lam) o', dy = U(lam) do''
-                    sincospif(phase_pi_m(lam, j, sl), &sn[rb][u], &cs[rb][u]);
-                    const float xc = x1[2 * j - 1], xs = x1[2 * j];
-                    zc[rb][u] = cs[rb][u] * xc - sn[rb][u] * xs;
-                    zs[rb][u] = sn[rb][u] * xc + cs[rb][u] * xs;
-                    const float gc = xd[2 * j - 1], gs = xd[2 * j];
-                    yc[rb][u] = cs[rb][u] * gc - sn[rb][u] * gs;
-                    ys[rb][u] = sn[rb][u] * gc + cs[rb][u] * gs;
-                }
-            }
-            float a1 = 0.f;
-#pragma unroll
-            for (int v = 0; v < NE; ++v) a1 += x2[lane + 32 * v] * xd[lane + 32 * v];
-            g1[rb] = warp_sum(a1);                                  // <o'', do''>
-            om2[rb] = warp_omega_dot<MSZ>(xd, x2, lane, sl);        // <do'', Omega o''>
-        }
-        // logits l = M z and dp = M dy (M^T rows k, entries col = lane + 32 v)
-        float l[RB][NE], dp[RB][NE];
-#pragma unroll
-        for (int v = 0; v < NE; ++v) {
-            const float mt = MT[lane + 32 * v];
-#pragma unroll
-            for (int rb = 0; rb < RB; ++rb) {
-                l[rb][v] = mt * z0[rb];
-                dp[rb][v] = mt * y0[rb];
-            }
-        }
+    const int K = (m + 31) & ~31;   // the products run over the active entries in steps of 32
+    __syncthreads();
+    for (int r = warp; r < CB; r += NW) {   // z, dy; inactive entries zeroed (read up to K)
+        float* z = sZ + r * LDM;
+        float* y = sG + r * LDM;
+        const float lam = slam[r];
 #pragma unroll
         for (int u = 0; u < NP; ++u) {
-            const int jmax = min(32, npair - 32 * u);   // pairs 32 u + 1 .. 32 u + jmax
-#pragma unroll UNR
-            for (int src = 0; src < jmax; ++src) {
-                const int kc = 2 * (32 * u + src) + 1;
-                float vzc[RB], vzs[RB], vyc[RB], vys[RB];
-#pragma unroll
-                for (int rb = 0; rb < RB; ++rb) {
-                    vzc[rb] = __shfl_sync(0xffffffffu, zc[rb][u], src);
-                    vzs[rb] = __shfl_sync(0xffffffffu, zs[rb][u], src);
-                    vyc[rb] = __shfl_sync(0xffffffffu, yc[rb][u], src);
-                    vys[rb] = __shfl_sync(0xffffffffu, ys[rb][u], src);
-                }
-                const float* mc = MT + kc * MSZ + lane;
-#pragma unroll
-                for (int v = 0; v < NE; ++v) {
-                    const float a = mc[32 * v], b = mc[MSZ + 32 * v];
-#pragma unroll
-                    for (int rb = 0; rb < RB; ++rb) {
-                        l[rb][v] = fmaf(b, vzs[rb], fmaf(a, vzc[rb], l[rb][v]));
-                        dp[rb][v] = fmaf(b, vys[rb], fmaf(a, vyc[rb], dp[rb][v]));
-                    }
-                }
+            const int j = lane + 1 + 32 * u;
+            if (j <= npair) {
+                float sn, cs;
+                sincospif(phase_pi_m(lam, j, sl), &sn, &cs);
+                const float xc = z[2 * j - 1], xs = z[2 * j];
+                z[2 * j - 1] = cs * xc - sn * xs;
+                z[2 * j] = sn * xc + cs * xs;
+                const float gc = y[2 * j - 1], gs = y[2 * j];
+                y[2 * j - 1] = cs * gc - sn * gs;
+                y[2 * j] = sn * gc + cs * gs;
+            } else if (j < MSZ / 2) {
+                z[2 * j - 1] = z[2 * j] = 0.f;
+                y[2 * j - 1] = y[2 * j] = 0.f;
             }
         }
-        // p = softmax(l) over the m active slots (into l), dl = p o (dp - <p, dp>) (into dp)
+        if (lane == 0) z[MSZ - 1] = y[MSZ - 1] = 0.f;
+    }
+    // logits and their adjoint (the row ty + 16 i lives on the 16 threads of a half warp)
+    float ldp[2][TMB][NJ];
+    zero_acc(ldp[0]);
+    zero_acc(ldp[1]);
+    rows_times_gmat<2, TMB, MSZ>(ldp, sB, sZ, sG, MT, K);
+    float(&l)[TMB][NJ] = ldp[0];
+    float(&dp)[TMB][NJ] = ldp[1];
 #pragma unroll
-        for (int rb = 0; rb < RB; ++rb) {
-            float mx = -INFINITY;
+    for (int i = 0; i < TMB; ++i) {
+        float mx = -INFINITY;
 #pragma unroll
-            for (int v = 0; v < NE; ++v) {
-                if (lane + 32 * v >= m) l[rb][v] = -INFINITY;
-                mx = fmaxf(mx, l[rb][v]);
-            }
-            mx = warp_max(mx);
-            float sum = 0.f;
+        for (int j = 0; j < NJ; ++j)
+            if (tx + 16 * j < m) mx = fmaxf(mx, l[i][j]);
+        mx = half_warp_max(mx);
+        float sum = 0.f;
 #pragma unroll
-            for (int v = 0; v < NE; ++v) {
-                l[rb][v] = expf(l[rb][v] - mx);
-                sum += l[rb][v];
-            }
-            const float inv = 1.f / warp_sum(sum);
-            float pdp = 0.f;
-#pragma unroll
-            for (int v = 0; v < NE; ++v) {
-                l[rb][v] *= inv;
-                pdp += l[rb][v] * dp[rb][v];
-            }
-            pdp = warp_sum(pdp);
-#pragma unroll
-            for (int v = 0; v < NE; ++v) dp[rb][v] = l[rb][v] * (dp[rb][v] - pdp);
+        for (int j = 0; j < NJ; ++j) {
+            l[i][j] = tx + 16 * j < m ? expf(l[i][j] - mx) : 0.f;
+            sum += l[i][j];
         }
-        if (gz) {
+        const float inv = 1.f / half_warp_sum(sum);
+        float pdp = 0.f;
 #pragma unroll
-            for (int rb = 0; rb < RB; ++rb) {
-                const size_t o = (size_t)(r0 + rb) * MSZ;
+        for (int j = 0; j < NJ; ++j) {
+            l[i][j] *= inv;
+            pdp = fmaf(l[i][j], dp[i][j], pdp);
+        }
+        pdp = half_warp_sum(pdp);
 #pragma unroll
-                for (int v = 0; v < NE; ++v) {
-                    gp[o + lane + 32 * v] = l[rb][v];
-                    gdl[o + lane + 32 * v] = dp[rb][v];
-                }
+        for (int j = 0; j < NJ; ++j) dp[i][j] = l[i][j] * (dp[i][j] - pdp);
+    }
 #pragma unroll
-                for (int u = 0; u < NP; ++u) {
-                    const int j = lane + 1 + 32 * u;
-                    if (j <= G::NPAIRS) {   // zero on the padding pairs
-                        gz[o + 2 * j - 1] = zc[rb][u];
-                        gz[o + 2 * j] = zs[rb][u];
-                        gdy[o + 2 * j - 1] = yc[rb][u];
-                        gdy[o + 2 * j] = ys[rb][u];
-                    }
-                }
-                if (lane == 0) {
-                    gz[o] = z0[rb];
-                    gz[o + MSZ - 1] = 0.f;
-                    gdy[o] = y0[rb];
-                    gdy[o + MSZ - 1] = 0.f;
-                }
+    for (int i = 0; i < TMB; ++i)
+#pragma unroll
+        for (int j = 0; j < NJ; ++j) {
+            const int r = ty + 16 * i, c = tx + 16 * j;
+            sY[r * LDM + c] = l[i][j];
+            sW[r * LDM + c] = dp[i][j];
+            if (gz) {
+                gp[(size_t)r * MSZ + c] = l[i][j];
+                gdl[(size_t)r * MSZ + c] = dp[i][j];
             }
         }
-        // dz = M^T dl (entries col = lane + 32 v), into the rows of sD (do'' is consumed)
-        float g[RB][NE];
+    float ydz[2][TMB][NJ];
+    zero_acc(ydz[0]);
+    zero_acc(ydz[1]);
+    rows_times_gmat<2, TMB, MSZ>(ydz, sB, sY, sW, M, K);
+    const float(&y)[TMB][NJ] = ydz[0];
+    const float(&dz)[TMB][NJ] = ydz[1];
+    __syncthreads();   // p and dl have been read
 #pragma unroll
-        for (int rb = 0; rb < RB; ++rb)
+    for (int i = 0; i < TMB; ++i)
 #pragma unroll
-            for (int v = 0; v < NE; ++v) g[rb][v] = 0.f;
+        for (int j = 0; j < NJ; ++j) {
+            const int r = ty + 16 * i, c = tx + 16 * j;
+            sY[r * LDM + c] = y[i][j];
+            sW[r * LDM + c] = dz[i][j];
+        }
+    __syncthreads();
+    for (int r = warp; r < CB; r += NW) {
+        const float* z = sZ + r * LDM;
+        const float* w = sW + r * LDM;   // dz
+        float* yv = sY + r * LDM;        // y, then o''
+        float* g = sG + r * LDM;         // dy, then do'
+        float g1 = 0.f;
 #pragma unroll
-        for (int v2 = 0; v2 < NE; ++v2) {
-            const int imax = min(32, m - 32 * v2);
-#pragma unroll UNR
-            for (int src = 0; src < imax; ++src) {
-                float dv[RB];
-#pragma unroll
-                for (int rb = 0; rb < RB; ++rb) dv[rb] = __shfl_sync(0xffffffffu, dp[rb][v2], src);
-                const float* mr = M + (32 * v2 + src) * MSZ + lane;
-#pragma unroll
-                for (int v = 0; v < NE; ++v) {
-                    const float a = mr[32 * v];
-#pragma unroll
-                    for (int rb = 0; rb < RB; ++rb) g[rb][v] = fmaf(a, dv[rb], g[rb][v]);
-                }
+        for (int v = 0; v < NE; ++v) {
+            const int e = lane + 32 * v;
+            g1 = fmaf(yv[e], g[e], g1);
+            if (gz) {
+                gz[(size_t)r * MSZ + e] = z[e];
+                gdy[(size_t)r * MSZ + e] = g[e];
             }
         }
-        __syncwarp();
+        g1 = warp_sum(g1);
+        __syncwarp();   // the row's entries have been read before their pairs are rewritten
+        const float lam = slam[r];
+        float om = 0.f;
 #pragma unroll
-        for (int rb = 0; rb < RB; ++rb) {
-            float* xd = sD + (r0 + rb) * LDM;
-#pragma unroll
-            for (int v = 0; v < NE; ++v) xd[lane + 32 * v] = g[rb][v];   // padding entries are 0
-        }
-        __syncwarp();
-#pragma unroll
-        for (int rb = 0; rb < RB; ++rb) {
-            float* xd = sD + (r0 + rb) * LDM;
-            float a = 0.f;   // <dz, Omega z>, then do' = U(-lam) dz on the active pairs
-#pragma unroll
-            for (int u = 0; u < NP; ++u) {
-                const int j = lane + 1 + 32 * u;
-                if (j <= npair) {
-                    const float gc = xd[2 * j - 1], gs = xd[2 * j];
-                    a += freq(j, sl) * (gs * zc[rb][u] - gc * zs[rb][u]);
-                    xd[2 * j - 1] = cs[rb][u] * gc + sn[rb][u] * gs;
-                    xd[2 * j] = -sn[rb][u] * gc + cs[rb][u] * gs;
-                }
-            }
-            const float om1 = warp_sum(a);
-            if (lane == 0) {
-                sdG[r0 + rb] = g1[rb];
-                sdL[r0 + rb] = om1 - om2[rb];
+        for (int u = 0; u < NP; ++u) {
+            const int j = lane + 1 + 32 * u;
+            if (j <= npair) {
+                float sn, cs;
+                sincospif(phase_pi_m(lam, j, sl), &sn, &cs);
+                const float yc = yv[2 * j - 1], ys = yv[2 * j];
+                const float gc = g[2 * j - 1], gs = g[2 * j];
+                const float dc = w[2 * j - 1], ds = w[2 * j];
+                const float zc = z[2 * j - 1], zs = z[2 * j];
+                om += freq(j, sl) * ((ds * zc - dc * zs) - (gs * yc - gc * ys));
+                yv[2 * j - 1] = cs * yc + sn * ys;
+                yv[2 * j] = -sn * yc + cs * ys;
+                g[2 * j - 1] = cs * dc + sn * ds;
+                g[2 * j] = -sn * dc + cs * ds;
+            } else if (j < MSZ / 2) {
+                g[2 * j - 1] = g[2 * j] = 0.f;
             }
         }
-        __syncwarp();
+        om = warp_sum(om);
+        if (lane == 0) {
+            g[0] = w[0];
+            g[MSZ - 1] = 0.f;
+            sdG[r] = g1;
+            sdL[r] = om;
+        }
     }
 }
 
@@ -378,7 +339,8 @@ __global__ void __launch_bounds__(256) bwd_intra1_kernel(BwdArgs a) {
     float* sbeta = slam + CB;
     float* sdG = sbeta + CB;
     float* sdL = sdG + CB;
-    if (!launch_ok(smem, sdL + CB)) return;
+    float* sB = sdL + CB;                           // [32][MSZ + 1] staging of M^T / M
+    if (!launch_ok(smem, sB + 32 * LDM)) return;
     const int tx = threadIdx.x & 15, ty = threadIdx.x >> 4;
     const float* Sst = a.states + ((size_t)bh * nchunk + c) * MSZ * (2 * D);
     const float* Mh = a.M + (size_t)h * MSZ * MSZ;
@@ -408,13 +370,9 @@ __global__ void __launch_bounds__(256) bwd_intra1_kernel(BwdArgs a) {
 #pragma unroll
         for (int i = 0; i < TMB; ++i)
 #pragma unroll
-            for (int j = 0; j < NJ; ++j) {
-                sO1[(ty + 16 * i) * LDM + tx + 16 * j] = o1[i][j];
-                sO2[(ty + 16 * i) * LDM + tx + 16 * j] = o1[i][j];
-            }
+            for (int j = 0; j < NJ; ++j) sO1[(ty + 16 * i) * LDM + tx + 16 * j] = o1[i][j];
     }
     __syncthreads();
-    middle_rows<MSZ, 4>(sO2, slam, CB, Mh, MTh, s.sl);
 
     // dO'' = gamma o (dO Vbar^T) + (dO V^T o Gamma) A
     masked_scores_tok<MSZ>(sP, sS, sg, dO, V, s, b, h, t0, 1.f);
@@ -433,13 +391,12 @@ __global__ void __launch_bounds__(256) bwd_intra1_kernel(BwdArgs a) {
 #pragma unroll
             for (int j = 0; j < NJ; ++j) sD[(ty + 16 * i) * LDM + tx + 16 * j] = g2[i][j];
     }
-    __syncthreads();
-    {
+    {   // the middle readout (o'' into sO2) and its gradient (do' into sD); sO1 ends as z
         const size_t rowbase = ((size_t)bh * s.T + t0) * MSZ;
         const bool dr = a.mZ != nullptr;
-        middle_rows_bwd<MSZ, MSZ == 128 ? 4 : 2>(sO1, sO2, sD, slam, CB, Mh, MTh, sdG, sdL,
-                        dr ? a.mZ + rowbase : nullptr, dr ? a.mP + rowbase : nullptr,
-                        dr ? a.mDY + rowbase : nullptr, dr ? a.mDL + rowbase : nullptr, s.sl);
+        readout_rows_bwd<MSZ>(sO1, sO2, sD, sS, sB, slam, Mh, MTh, sdG, sdL,
+                              dr ? a.mZ + rowbase : nullptr, dr ? a.mP + rowbase : nullptr,
+                              dr ? a.mDY + rowbase : nullptr, dr ? a.mDL + rowbase : nullptr, s.sl);
     }
     __syncthreads();
 
@@ -958,7 +915,7 @@ cudaError_t bwd_dispatch(const BwdArgs& a, cudaStream_t st) {
     if (e != cudaSuccess) return e;
     const dim3 gchunk(s.nchunk(), s.B * s.H);
     constexpr int SSZ = staging_floats<D, MSZ>();
-    const size_t sm1 = (size_t)(4 * CB * LDM + SSZ + CB * G::LPB + 6 * CB) * sizeof(float);
+    const size_t sm1 = (size_t)(4 * CB * LDM + SSZ + CB * G::LPB + 6 * CB + 32 * LDM) * sizeof(float);
     auto k1 = bwd_intra1_kernel<D, MSZ, TI>;
     cudaFuncSetAttribute(k1, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm1);
     { LaunchScope ls_("bwd_intra1", st); k1<<<gchunk, 256, sm1, st>>>(a); }

@@ -37,140 +37,6 @@ static inline cudaError_t read_simt_error(cudaStream_t st, int* err) {
 }
 
 // ---------------------------------------------------------------------------------------
-// Token-wise middle readout for rows r < C of sX (row stride MSZ + 1, in place):
-// o'' = U(-lam) M^T softmax(M U(lam) o') with M = R Phi ([MSZ][MSZ], global); the padding
-// logits (slots m..MSZ-1) are excluded from the softmax and o''[m..MSZ-1] are 0.
-// Each warp takes RB rows at a time so that every entry of M and M^T it loads serves RB rows.
-// A lane keeps the rotation pairs j = lane + 1 + 32 u of its rows in registers and the logit /
-// softmax entries lane + 32 v; the products over slots broadcast the summed-over vector from
-// its owner lane by shuffles, in slot order (the same order of accumulation as a plain loop).
-// C is a multiple of 8 RB.
-template <int MSZ, int RB>
-static __device__ __noinline__ void middle_rows(float* sX, const float* slam, int C, const float* M,
-                                                const float* MT, const Slots& sl) {
-    constexpr int LDM = MSZ + 1, NP = MSZ / 64, NE = MSZ / 32;
-    constexpr int UNR = MSZ == 128 ? 4 : 1;   // slot steps whose M / M^T loads are in flight together
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int npair = sl.npair, m = sl.m;
-    for (int r0 = warp * RB; r0 < C; r0 += 8 * RB) {
-        float cs[RB][NP], sn[RB][NP], zc[RB][NP], zs[RB][NP], z0[RB];
-#pragma unroll
-        for (int rb = 0; rb < RB; ++rb) {
-            const float* x = sX + (r0 + rb) * LDM;
-            const float lam = slam[r0 + rb];
-            z0[rb] = x[0];
-#pragma unroll
-            for (int u = 0; u < NP; ++u) {
-                const int j = lane + 1 + 32 * u;
-                cs[rb][u] = 1.f;
-                sn[rb][u] = 0.f;
-                zc[rb][u] = zs[rb][u] = 0.f;
-                if (j <= npair) {   // z = U(lam) o'
-                    sincospif(phase_pi_m(lam, j, sl), &sn[rb][u], &cs[rb][u]);
-                    const float xc = x[2 * j - 1], xs = x[2 * j];
-                    zc[rb][u] = cs[rb][u] * xc - sn[rb][u] * xs;
-                    zs[rb][u] = sn[rb][u] * xc + cs[rb][u] * xs;
-                }
-            }
-        }
-        // logits l[col] = sum_k MT[k][col] z[k], col = lane + 32 v
-        float l[RB][NE];
-#pragma unroll
-        for (int v = 0; v < NE; ++v) {
-            const float mt = MT[lane + 32 * v];
-#pragma unroll
-            for (int rb = 0; rb < RB; ++rb) l[rb][v] = mt * z0[rb];
-        }
-#pragma unroll
-        for (int u = 0; u < NP; ++u) {
-            const int jmax = min(32, npair - 32 * u);   // pairs 32 u + 1 .. 32 u + jmax
-#pragma unroll UNR
-            for (int src = 0; src < jmax; ++src) {
-                const int kc = 2 * (32 * u + src) + 1;
-                float vc[RB], vs[RB];
-#pragma unroll
-                for (int rb = 0; rb < RB; ++rb) {
-                    vc[rb] = __shfl_sync(0xffffffffu, zc[rb][u], src);
-                    vs[rb] = __shfl_sync(0xffffffffu, zs[rb][u], src);
-                }
-                const float* mc = MT + kc * MSZ + lane;
-#pragma unroll
-                for (int v = 0; v < NE; ++v) {
-                    const float a = mc[32 * v], b = mc[MSZ + 32 * v];
-#pragma unroll
-                    for (int rb = 0; rb < RB; ++rb)
-                        l[rb][v] = fmaf(b, vs[rb], fmaf(a, vc[rb], l[rb][v]));
-                }
-            }
-        }
-        // softmax over the m active slots
-#pragma unroll
-        for (int rb = 0; rb < RB; ++rb) {
-            float mx = -INFINITY;
-#pragma unroll
-            for (int v = 0; v < NE; ++v) {
-                if (lane + 32 * v >= m) l[rb][v] = -INFINITY;
-                mx = fmaxf(mx, l[rb][v]);
-            }
-            mx = warp_max(mx);
-            float sum = 0.f;
-#pragma unroll
-            for (int v = 0; v < NE; ++v) {
-                l[rb][v] = expf(l[rb][v] - mx);
-                sum += l[rb][v];
-            }
-            const float inv = 1.f / warp_sum(sum);
-#pragma unroll
-            for (int v = 0; v < NE; ++v) l[rb][v] *= inv;
-        }
-        // y[col] = sum_{i < m} M[i][col] p[i], into the row (o' is consumed)
-        float y[RB][NE];
-#pragma unroll
-        for (int rb = 0; rb < RB; ++rb)
-#pragma unroll
-            for (int v = 0; v < NE; ++v) y[rb][v] = 0.f;
-#pragma unroll
-        for (int v2 = 0; v2 < NE; ++v2) {
-            const int imax = min(32, m - 32 * v2);
-#pragma unroll UNR
-            for (int src = 0; src < imax; ++src) {
-                float pv[RB];
-#pragma unroll
-                for (int rb = 0; rb < RB; ++rb) pv[rb] = __shfl_sync(0xffffffffu, l[rb][v2], src);
-                const float* mr = M + (32 * v2 + src) * MSZ + lane;
-#pragma unroll
-                for (int v = 0; v < NE; ++v) {
-                    const float a = mr[32 * v];
-#pragma unroll
-                    for (int rb = 0; rb < RB; ++rb) y[rb][v] = fmaf(a, pv[rb], y[rb][v]);
-                }
-            }
-        }
-        __syncwarp();
-#pragma unroll
-        for (int rb = 0; rb < RB; ++rb) {
-            float* x = sX + (r0 + rb) * LDM;
-#pragma unroll
-            for (int v = 0; v < NE; ++v) x[lane + 32 * v] = y[rb][v];   // padding entries are 0
-        }
-        __syncwarp();
-#pragma unroll
-        for (int rb = 0; rb < RB; ++rb) {   // o'' = U(-lam) y on the active pairs
-            float* x = sX + (r0 + rb) * LDM;
-#pragma unroll
-            for (int u = 0; u < NP; ++u) {
-                const int j = lane + 1 + 32 * u;
-                if (j <= npair) {
-                    const float yc = x[2 * j - 1], ys = x[2 * j];
-                    x[2 * j - 1] = cs[rb][u] * yc + sn[rb][u] * ys;
-                    x[2 * j] = -sn[rb][u] * yc + cs[rb][u] * ys;
-                }
-            }
-        }
-        __syncwarp();
-    }
-}
-
 // g_cum is local to the caller's chunks of s.Cg tokens; a kernel walking shorter chunks of C
 // tokens (C divides Cg) rebases it to its own chunk start by subtracting the value just before.
 __device__ __forceinline__ float g_base(const Shape& s, const float* g, int b, int h, int t0,
@@ -220,6 +86,126 @@ __device__ __forceinline__ void stage_tok(float* dst, const TI* X, const Shape& 
             return mul * ldf(X, (((size_t)b * s.T + t0 + e / NC) * s.H + h) * s.D + c0 + e % NC);
         },
         [&](int e, float x) { dst[(e / NC) * (NC + 1) + e % NC] = x; });
+}
+
+// Row blocks times a global matrix: acc[p][i][j] += sum_{k < K} X_p(ty + 16 i, k) B(k, tx + 16 j)
+// for p < NPROD (X_0, X_1 rows in shared memory with stride MSZ + 1; X_1 unused when NPROD = 1)
+// and B a [MSZ][MSZ] global matrix whose rows are staged 32 at a time through sB
+// ([32][MSZ + 1]): one staging of B serves every product.  K is a multiple of 32, at most MSZ.
+// Begins with a block barrier; the caller places one before sB or the X rows are rewritten.
+template <int NPROD, int TM, int MSZ>
+__device__ __forceinline__ void rows_times_gmat(float (&acc)[NPROD][TM][MSZ / 16], float* sB,
+                                                const float* X0, const float* X1, const float* B,
+                                                int K) {
+    constexpr int LDM = MSZ + 1, NJ = MSZ / 16;
+    const int tx = threadIdx.x & 15, ty = threadIdx.x >> 4;
+    for (int k0 = 0; k0 < K; k0 += 32) {
+        __syncthreads();
+        stage_elems<32 * MSZ / SIMT_THREADS>(
+            32 * MSZ, [&](int e) { return B[(size_t)k0 * MSZ + e]; },
+            [&](int e, float x) { sB[(e / MSZ) * LDM + e % MSZ] = x; });
+        __syncthreads();
+#pragma unroll 2
+        for (int kk = 0; kk < 32; ++kk) {
+            float a[NPROD][TM], b[NJ];
+#pragma unroll
+            for (int i = 0; i < TM; ++i) {
+                a[0][i] = X0[(ty + 16 * i) * LDM + k0 + kk];
+                if (NPROD > 1) a[NPROD - 1][i] = X1[(ty + 16 * i) * LDM + k0 + kk];
+            }
+#pragma unroll
+            for (int j = 0; j < NJ; ++j) b[j] = sB[kk * LDM + tx + 16 * j];
+#pragma unroll
+            for (int p = 0; p < NPROD; ++p)
+#pragma unroll
+                for (int i = 0; i < TM; ++i)
+#pragma unroll
+                    for (int j = 0; j < NJ; ++j) acc[p][i][j] = fmaf(a[p][i], b[j], acc[p][i][j]);
+        }
+    }
+}
+
+// The middle readout for the C rows of a chunk (o' in the rows of sX, stride MSZ + 1, replaced by
+// o''), as products of the row block with M^T and M (global [MSZ][MSZ], zero beyond the m active
+// rows and columns): z = U(lam) o' (in place; inactive entries zeroed), l = M z (one pass over
+// M^T), p = softmax(l) over the m active slots (into sX), y = M^T p (one pass over M, into sX),
+// o'' = U(-lam) y.  The row ty + 16 i of a product lives on the 16 threads of a half warp.  sB is
+// the [32][MSZ + 1] staging of M^T and M.  Needs a block barrier before (o' complete) and after.
+template <int C, int MSZ>
+static __device__ __noinline__ void readout_rows_fwd(float* sX, float* sB, const float* slam,
+                                                     const float* M, const float* MT,
+                                                     const Slots& sl) {
+    constexpr int LDM = MSZ + 1, NP = MSZ / 64, TM = C / 16, NJ = MSZ / 16, NW = SIMT_THREADS / 32;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int tx = threadIdx.x & 15, ty = threadIdx.x >> 4;
+    const int npair = sl.npair, m = sl.m;
+    const int K = (m + 31) & ~31;   // the products run over the active entries in steps of 32
+    for (int r = warp; r < C; r += NW) {
+        float* z = sX + r * LDM;
+        const float lam = slam[r];
+#pragma unroll
+        for (int u = 0; u < NP; ++u) {
+            const int j = lane + 1 + 32 * u;
+            if (j <= npair) {
+                float sn, cs;
+                sincospif(phase_pi_m(lam, j, sl), &sn, &cs);
+                const float xc = z[2 * j - 1], xs = z[2 * j];
+                z[2 * j - 1] = cs * xc - sn * xs;
+                z[2 * j] = sn * xc + cs * xs;
+            } else if (j < MSZ / 2) {
+                z[2 * j - 1] = z[2 * j] = 0.f;
+            }
+        }
+        if (lane == 0) z[MSZ - 1] = 0.f;
+    }
+    float acc[1][TM][NJ];
+    zero_acc(acc[0]);
+    rows_times_gmat<1, TM, MSZ>(acc, sB, sX, sX, MT, K);
+#pragma unroll
+    for (int i = 0; i < TM; ++i) {
+        float mx = -INFINITY;
+#pragma unroll
+        for (int j = 0; j < NJ; ++j)
+            if (tx + 16 * j < m) mx = fmaxf(mx, acc[0][i][j]);
+        mx = half_warp_max(mx);
+        float sum = 0.f;
+#pragma unroll
+        for (int j = 0; j < NJ; ++j) {
+            acc[0][i][j] = tx + 16 * j < m ? expf(acc[0][i][j] - mx) : 0.f;
+            sum += acc[0][i][j];
+        }
+        const float inv = 1.f / half_warp_sum(sum);
+#pragma unroll
+        for (int j = 0; j < NJ; ++j) acc[0][i][j] *= inv;
+    }
+    __syncthreads();   // z has been read
+#pragma unroll
+    for (int i = 0; i < TM; ++i)
+#pragma unroll
+        for (int j = 0; j < NJ; ++j) sX[(ty + 16 * i) * LDM + tx + 16 * j] = acc[0][i][j];
+    zero_acc(acc[0]);
+    rows_times_gmat<1, TM, MSZ>(acc, sB, sX, sX, M, K);
+    __syncthreads();   // p has been read
+#pragma unroll
+    for (int i = 0; i < TM; ++i)
+#pragma unroll
+        for (int j = 0; j < NJ; ++j) sX[(ty + 16 * i) * LDM + tx + 16 * j] = acc[0][i][j];
+    __syncthreads();
+    for (int r = warp; r < C; r += NW) {   // o'' = U(-lam) y on the active pairs
+        float* x = sX + r * LDM;
+        const float lam = slam[r];
+#pragma unroll
+        for (int u = 0; u < NP; ++u) {
+            const int j = lane + 1 + 32 * u;
+            if (j <= npair) {
+                float sn, cs;
+                sincospif(phase_pi_m(lam, j, sl), &sn, &cs);
+                const float yc = x[2 * j - 1], ys = x[2 * j];
+                x[2 * j - 1] = cs * yc + sn * ys;
+                x[2 * j] = -sn * yc + cs * ys;
+            }
+        }
+    }
 }
 
 }  // namespace cyfa
