@@ -119,13 +119,18 @@ def fp32_alu_peak_tflops(sm_mhz, sms=152):
 
 # ---------------------------------------------------------------------------------- clocks
 class ClockSampler:
-    FIELDS = ('index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,'
+    """nvidia-smi clock and throttle-reason samples every 50 ms; only the samples taken between
+    begin() and end() (the timed region, by the host clock, with half a sampling interval of
+    margin) are summarised, else the nearest one on either side of it."""
+    FIELDS = ('timestamp,index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,'
               'clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,'
               'clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap')
+    PERIOD_MS = 50
 
     def __init__(self, device_index):
         self.idx = device_index
         self.proc = None
+        self.t_begin = self.t_end = None
         import tempfile
         self.path = os.path.join(tempfile.gettempdir(),
                                  'cyfa_bench_clocks_%d_%d.csv' % (os.getpid(), device_index))
@@ -136,10 +141,33 @@ class ClockSampler:
             self.fh = open(self.path, 'w')
             self.proc = subprocess.Popen(
                 ['nvidia-smi', '-i', str(self.idx), '--query-gpu=' + self.FIELDS,
-                 '--format=csv,noheader,nounits', '-lms', '200'], stdout=self.fh,
+                 '--format=csv,noheader,nounits', '-lms', str(self.PERIOD_MS)], stdout=self.fh,
                 stderr=subprocess.DEVNULL)
         except Exception:
             self.proc = None
+            return
+        deadline = time.time() + 5.0   # the sampler is running before the timed region starts
+        while time.time() < deadline and self.proc.poll() is None:
+            try:
+                if os.path.getsize(self.path) > 0:
+                    break
+            except OSError:
+                pass
+            time.sleep(0.01)
+
+    def begin(self):
+        self.t_begin = time.time()
+
+    def end(self):
+        self.t_end = time.time()
+
+    @staticmethod
+    def _when(stamp):
+        import datetime
+        try:
+            return datetime.datetime.strptime(stamp, '%Y/%m/%d %H:%M:%S.%f').timestamp()
+        except ValueError:
+            return None
 
     def stop(self):
         if self.proc is None:
@@ -150,29 +178,41 @@ class ClockSampler:
         except Exception:
             self.proc.kill()
         self.fh.close()
-        sm, smax, reasons = [], None, set()
         names = ['hw_slowdown', 'hw_thermal_slowdown', 'sw_thermal_slowdown', 'sw_power_cap']
+        rows = []
         for line in open(self.path):
             parts = [x.strip() for x in line.split(',')]
-            if len(parts) < 9:
+            if len(parts) < 10:
                 continue
             try:
-                sm.append(float(parts[1]))
-                smax = float(parts[2])
+                sm, smax = float(parts[2]), float(parts[3])
             except ValueError:
                 continue
-            for nm, val in zip(names, parts[5:9]):
-                if val.lower() == 'active':
-                    reasons.add(nm)
+            active = {nm for nm, val in zip(names, parts[6:10]) if val.lower() == 'active'}
+            rows.append((self._when(parts[0]), sm, smax, active))
         try:
             os.remove(self.path)
         except OSError:
             pass
-        if not sm:
+        if not rows:
             return None
-        sm.sort()
-        return {'sm_mhz': sm[len(sm) // 2], 'sm_max_mhz': smax, 'reasons': sorted(reasons),
-                'samples': len(sm)}
+        use, where = rows, 'all samples'
+        if self.t_begin is not None and self.t_end is not None and all(r[0] for r in rows):
+            m = 0.5e-3 * self.PERIOD_MS
+            inside = [r for r in rows if self.t_begin - m <= r[0] <= self.t_end + m]
+            if inside:
+                use, where = inside, 'timed region'
+            else:
+                before = [r for r in rows if r[0] < self.t_begin]
+                after = [r for r in rows if r[0] > self.t_end]
+                use = before[-1:] + after[:1]
+                where = 'nearest samples around the timed region'
+        sm = sorted(r[1] for r in use)
+        reasons = set()
+        for r in use:
+            reasons |= r[3]
+        return {'sm_mhz': sm[len(sm) // 2], 'sm_max_mhz': use[-1][2], 'reasons': sorted(reasons),
+                'samples': len(use), 'sampled': where, 'period_ms': self.PERIOD_MS}
 
 
 # --------------------------------------------------------------------------- cpu baseline
@@ -326,11 +366,13 @@ def run_ours(args):
     clocks.start()
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     torch.cuda.synchronize()
+    clocks.begin()
     e0.record(stream)
     for _ in range(args.steps):
         step(inp)
     e1.record(stream)
     torch.cuda.synchronize()
+    clocks.end()
     clk = clocks.stop()
     cyfa.cyfa_check()
     ms = e0.elapsed_time(e1) / args.steps
