@@ -86,7 +86,7 @@ __device__ __forceinline__ void build_write_rows(float* sA, int ld, const float*
 template <int TM, int TN, class FA, class FB>
 __device__ __forceinline__ void simt_mm(float (&acc)[TM][TN], int K, const FA& fa, const FB& fb) {
     const int tx = threadIdx.x & 15, ty = threadIdx.x >> 4;
-#pragma unroll 2
+#pragma unroll 4
     for (int kk = 0; kk < K; ++kk) {
         float a[TM], b[TN];
 #pragma unroll
