@@ -118,6 +118,21 @@ def test_omega_is_generator(m):
     np.testing.assert_allclose(dU, basis.omega(m) @ basis.U(tau, m), atol=1e-7)
 
 
+@pytest.mark.parametrize('m', [5, 127, 255])
+def test_U_commutes_with_its_generator(m):
+    # U(tau) = exp(tau Omega): U commutes with Omega, so the bilinear forms <x, y> and
+    # <x, Omega y> are the same before and after one rotation of both vectors (the CUDA-core
+    # readout gradient takes them before its final rotation by U(-lam))
+    rng = np.random.default_rng(4)
+    tau = rng.uniform(-300, 300)
+    Ut, W = basis.U(tau, m), basis.omega(m)
+    np.testing.assert_allclose(Ut @ W, W @ Ut, atol=1e-12)
+    np.testing.assert_allclose(W.T, -W, atol=0)
+    x, y = rng.standard_normal(m), rng.standard_normal(m)
+    assert abs((Ut @ x) @ (Ut @ y) - x @ y) < 1e-10
+    assert abs((Ut @ x) @ (W @ (Ut @ y)) - x @ (W @ y)) < 1e-9
+
+
 def test_state_size_accounting():
     H, ms, dk, dv, entries = _load('state_size.txt').astype(int)
     assert H * ms * (dk + dv) == entries
